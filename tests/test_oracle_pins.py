@@ -1,0 +1,259 @@
+"""Pins for the fp64 oracle: it is checked against things other than itself.
+
+Each test fixes a fact that the paper or the mathematics gives: a scalar-loop restatement on
+tiny inputs, closed forms, library routines, invariants of the definition, the identity-style
+initialisation of App. C (an exact pass-through construction), and numbers the paper prints
+(tests/golden/*.json, each with its source).
+"""
+import json
+import os
+
+import numpy as np
+import pytest
+import scipy.special
+import scipy.stats
+import torch
+
+from oracle import brute
+from oracle import still_oracle as O
+from paper_2606_07878_gb300 import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _golden(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return json.load(f)
+
+
+def _tiny(**over):
+    wl = dict(L=1, N=12, H=2, d=4, D=8, n=2, F=16, ts=(3,), theta=1e4, heavy=1)
+    wl.update(over)
+    return wl
+
+
+def _weights_f64(wl, t, n_blocks=1, cross_every_block=True, seed=0):
+    W = synth.gen_weights(wl, 0, t, "cpu", seed=seed, n_blocks=n_blocks)
+    W = O.as_f64(W)
+    # Scale weights up so that tiny widths give non-trivial attention patterns.
+    return {k: v * 10.0 for k, v in W.items()}
+
+
+# ------------------------------------------------------------------ brute force vs vectorised
+
+@pytest.mark.parametrize("variant", [
+    dict(),
+    dict(final_norm=True),
+    dict(compactor_rope=False),
+    dict(F=0),
+    dict(n_blocks=2),
+    dict(n_blocks=2, cross_every_block=False),
+    dict(logit_scale=1.0 / np.sqrt(8.0)),
+    dict(self_attn=False),
+])
+def test_brute_force_matches_vectorised(variant):
+    wl = _tiny()
+    F = variant.get("F", wl["F"])
+    wl["F"] = F
+    nb = variant.get("n_blocks", 1)
+    cfg = O.cfg_from_workload(wl, **variant)
+    t = 3
+    W = _weights_f64(wl, t, n_blocks=nb)
+    K, V = synth.gen_kv(wl, 0, N=wl["N"], positions=torch.arange(wl["N"]) * 3.5 + 7.25)
+    K, V = synth.bf16_to_f64(K), synth.bf16_to_f64(V)
+    kpos = np.arange(wl["N"]) * 3.5 + 7.25
+    Ck, Cv, opos, off = O.compact_layer(K, V, W, cfg, t, kpos)
+    Wl = {k: v.tolist() for k, v in W.items()}
+    for h in range(cfg.H):
+        bk, bv = brute.compact_head_brute(K[:, h].tolist(), V[:, h].tolist(),
+                                          W["Z"][h, :t].tolist(), Wl, cfg, kpos.tolist())
+        np.testing.assert_allclose(Ck[:, h], np.array(bk), rtol=0, atol=1e-10)
+        np.testing.assert_allclose(Cv[:, h], np.array(bv), rtol=0, atol=1e-10)
+    assert off == wl["N"] - t
+    assert np.all(np.isfinite(Ck)) and np.abs(Ck).max() > 1e-3
+
+
+# ------------------------------------------------------------------ RoPE
+
+def test_rope_roundtrip_and_zero_position():
+    rng = np.random.default_rng(0)
+    x = rng.standard_normal((64, 128))
+    pos = np.concatenate([np.arange(32) * 6250.0, rng.uniform(0, 2e5, 32)])  # up to 2e5, fractional
+    for base in (10.0, 1e4, 1e6):
+        y = O.unrope(O.rope(x, pos, base), pos, base)
+        assert np.max(np.abs(y - x)) <= 1e-14 * np.max(np.abs(x)) * 10
+        np.testing.assert_array_equal(O.rope(x, np.zeros(64), base), x)
+
+
+def test_rope_is_complex_multiplication():
+    """Half-split RoPE: (x_m + i x_{m+w/2}) * exp(i p omega_m), omega_m = base^(-2m/w)."""
+    rng = np.random.default_rng(1)
+    w, base = 16, 10.0
+    x = rng.standard_normal((5, w))
+    pos = rng.uniform(0, 1000, 5)
+    z = (x[:, : w // 2] + 1j * x[:, w // 2:])
+    omega = np.array([base ** (-(2.0 * m) / w) for m in range(w // 2)])
+    zr = z * np.exp(1j * pos[:, None] * omega[None, :])
+    ref = np.concatenate([zr.real, zr.imag], axis=1)
+    np.testing.assert_allclose(O.rope(x, pos, base), ref, atol=1e-11)
+    # rotation preserves norms
+    np.testing.assert_allclose(np.linalg.norm(O.rope(x, pos, base), axis=1),
+                               np.linalg.norm(x, axis=1), rtol=1e-13)
+
+
+# ------------------------------------------------------------------ norms, softmax, GELU
+
+def test_softmax_rows_sum_to_one_and_match_library():
+    rng = np.random.default_rng(2)
+    s = rng.standard_normal((7, 300)) * 200.0          # d_l-scaled logits
+    p = O.softmax_rows(s)
+    np.testing.assert_allclose(p.sum(axis=1), 1.0, atol=1e-14)
+    np.testing.assert_allclose(p, scipy.special.softmax(s, axis=1), rtol=1e-12, atol=1e-300)
+
+
+def test_l2norm_unit_and_zero():
+    rng = np.random.default_rng(3)
+    x = rng.standard_normal((9, 33))
+    np.testing.assert_allclose(np.linalg.norm(O.l2norm(x, 1e-12), axis=1), 1.0, atol=1e-14)
+    np.testing.assert_array_equal(O.l2norm(np.zeros((2, 5)), 1e-12), 0.0)
+
+
+def test_rmsnorm_closed_form():
+    rng = np.random.default_rng(4)
+    x = rng.standard_normal((9, 64)) * 1e-3
+    eps = 1e-6
+    ms = np.mean(x * x, axis=1)
+    y = O.rmsnorm(x, eps)
+    np.testing.assert_allclose(np.mean(y * y, axis=1), ms / (ms + eps), rtol=1e-13)
+    np.testing.assert_array_equal(O.rmsnorm(np.zeros((1, 8)), eps), 0.0)
+
+
+def test_gelu_is_x_times_normal_cdf():
+    x = np.linspace(-8, 8, 1001)
+    np.testing.assert_allclose(O.gelu(x), x * scipy.stats.norm.cdf(x), atol=1e-15)
+
+
+# ------------------------------------------------------------------ cross-attention invariants
+
+def _ca_setup(N=40, seed=5):
+    wl = _tiny(N=N)
+    cfg = O.cfg_from_workload(wl)
+    W = _weights_f64(wl, 4, seed=seed)
+    rng = np.random.default_rng(seed)
+    X = rng.standard_normal((N, 2 * wl["d"]))
+    Zn = O.rmsnorm(W["Z"][0, :4], cfg.rms_eps)
+    return wl, cfg, W, X, Zn
+
+
+def test_zero_scores_give_mean_of_projected_values():
+    """W_Q = 0, b_Q = 0 -> q = 0, every logit 0 -> head_i = mean_n(X) W_V,i."""
+    wl, cfg, W, X, Zn = _ca_setup()
+    W = dict(W)
+    W["Wq"] = np.zeros_like(W["Wq"])
+    W["bq"] = np.zeros_like(W["bq"])
+    kpos = np.arange(X.shape[0], dtype=float)
+    qpos = O.linspace_positions(0, X.shape[0] - 1, Zn.shape[0])
+    out = O.cross_attention(Zn, X, W, 0, cfg, qpos, kpos)
+    D = cfg.D
+    mean = np.mean(X, axis=0)
+    heads = np.concatenate([mean @ W["Wv"][:, i * D:(i + 1) * D] for i in range(cfg.n_c)])
+    ref = np.tile(heads @ W["Wo"], (Zn.shape[0], 1))
+    np.testing.assert_allclose(out, ref, atol=1e-12)
+
+
+def test_permutation_invariance():
+    """Jointly permuting (K row, V row, position) leaves C_k, C_v unchanged."""
+    wl = _tiny(N=30)
+    cfg = O.cfg_from_workload(wl)
+    W = _weights_f64(wl, 4)
+    kpos = np.arange(30) * 2.0 + 5.0
+    K, V = synth.gen_kv(wl, 0, N=30, positions=torch.tensor(kpos))
+    K, V = synth.bf16_to_f64(K), synth.bf16_to_f64(V)
+    perm = np.random.default_rng(6).permutation(30)
+    a = O.compact_layer(K, V, W, cfg, 4, kpos)
+    b = O.compact_layer(K[perm], V[perm], W, cfg, 4, kpos[perm])
+    np.testing.assert_allclose(a[0], b[0], atol=1e-12)
+    np.testing.assert_allclose(a[1], b[1], atol=1e-12)
+
+
+def test_compactor_rope_translation_invariance():
+    """Only p_n - p_j enters the compactor RoPE: shifting every position leaves CA unchanged."""
+    wl, cfg, W, X, Zn = _ca_setup()
+    N = X.shape[0]
+    kpos = np.arange(N, dtype=float) * 1.5
+    qpos = O.linspace_positions(kpos.min(), kpos.max(), Zn.shape[0])
+    a = O.cross_attention(Zn, X, W, 0, cfg, qpos, kpos)
+    b = O.cross_attention(Zn, X, W, 0, cfg, qpos + 1234.5, kpos + 1234.5)
+    np.testing.assert_allclose(a, b, atol=1e-9)
+
+
+# ------------------------------------------------------------------ identity-style init (App. C)
+
+def identity_init_weights(H, d, N):
+    """App. C construction with d_l = 2d, one cross head: Z = 0, W_K = 0, W_Q = 0, aligned q/k
+    biases u spread evenly over all compactor frequency pairs, W_V = W_O = I, refinement
+    outputs (S_O, W_2) zero, W_key = [I 0], W_val = [0 I]."""
+    D = 2 * d
+    rng = np.random.default_rng(11)
+    u = np.full(D, 1.0 / np.sqrt(D))
+    W = {
+        "Z": np.zeros((H, N, D)),
+        "Wq": np.zeros((D, D)), "bq": u.copy(), "Wk": np.zeros((2 * d, D)), "bk": u.copy(),
+        "Wv": np.eye(2 * d, D), "Wo": np.eye(D),
+        "Sq": rng.standard_normal((D, D)) * 0.02, "sbq": rng.standard_normal(D) * 0.02,
+        "Sk": rng.standard_normal((D, D)) * 0.02, "sbk": rng.standard_normal(D) * 0.02,
+        "Sv": rng.standard_normal((D, D)) * 0.02, "So": np.zeros((D, D)),
+        "W1": rng.standard_normal((D, 4 * D)) * 0.02, "W2": np.zeros((4 * D, D)),
+        "Wkey": np.concatenate([np.eye(d), np.zeros((d, d))], axis=0),
+        "Wval": np.concatenate([np.zeros((d, d)), np.eye(d)], axis=0),
+    }
+    return W
+
+
+def test_identity_init_passes_keys_and_values_through():
+    H, d, N = 2, 128, 96
+    W = identity_init_weights(H, d, N)
+    cfg = O.Cfg(H=H, d=d, D=2 * d, n_c=1, n_s=1, F=4 * 2 * d, theta=1e4)
+    wl = dict(N=N, H=H, d=d, theta=1e4, heavy=4)
+    K, V = synth.gen_kv(wl, 0, N=N)
+    K, V = synth.bf16_to_f64(K), synth.bf16_to_f64(V)
+    Ck, Cv, opos, off = O.compact_layer(K, V, W, cfg, N)
+    np.testing.assert_array_equal(opos, np.arange(N))
+    assert off == 0
+    np.testing.assert_allclose(Ck, K, atol=1e-9)
+    np.testing.assert_allclose(Cv, V, atol=1e-9)
+
+
+# ------------------------------------------------------------------ printed numbers
+
+def test_budgets_match_paper_table():
+    g = _golden("budgets.json")
+    for ctx, ratio, K in g["rows"]:
+        assert O.budget(g["ctx_tokens"][ctx], ratio) == K, (ctx, ratio, K)
+    assert O.budget(5, 2) == 3 and O.budget(3, 2) == 2      # halves round up
+
+
+def test_param_counts_match_paper():
+    g = _golden("param_counts.json")
+    b = g["base"]
+    for c in g["cases"]:
+        shapes = synth.weight_shapes(b["H"], b["d"], c["D"], c["n"], c["r"] * c["D"], c["t"],
+                                     n_blocks=c["B"], cross_every_block=c["cross_every_block"])
+        # Matrices only (the count ignores the small biases) plus the D-wide w_beta head.
+        per_layer = sum(int(np.prod(s)) for s in shapes.values() if len(s) > 1) + c["D"]
+        total = b["L"] * per_layer
+        assert abs(total - c["printed_total"]) <= g["tolerance_abs"], (c["name"], total)
+        assert per_layer == O.param_count(b["H"], b["d"], c["D"], c["t"], c["B"], c["n"], c["n"],
+                                          c["r"], c["cross_every_block"], c["r"] > 0)
+
+
+def test_kv_bytes_match_paper():
+    g = _golden("kv_bytes.json")
+    m = g["model"]
+    assert O.kv_bytes(m["L"], m["H"], m["d"], m["b"], 1) == g["per_token_kib"] * 1024
+    for S, gib in g["gib_at_tokens"]:
+        assert O.kv_bytes(m["L"], m["H"], m["d"], m["b"], S) / 2**30 == pytest.approx(gib, abs=5e-4)
+    for S, mib in g["mib_at_K"]:
+        assert round(O.kv_bytes(m["L"], m["H"], m["d"], m["b"], S) / 2**20) == mib
+    for S, gib in g["retained_gib_vllm"]:
+        assert O.kv_bytes(m["L"], m["H"], m["d"], m["b"], S) / 2**30 == pytest.approx(gib, abs=5e-4)
