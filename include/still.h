@@ -1,0 +1,239 @@
+/* still.h — C ABI of the Still per-layer KV-cache compactor (GB300 / sm_103a).
+ *
+ * The library computes the paper's per-layer compactor (Sec. 2.1, App. A)
+ *
+ *     g_phi^(l) : (K^(l,h), V^(l,h))_{h=1..H}  ->  (C_k^(l,h), C_v^(l,h))_{h=1..H},
+ *     C_k, C_v in R^{t x d},
+ *
+ * on one GPU: keys are un-rotated by the base model's RoPE (RoPE-fix, Sec. 2.2), t latent
+ * queries per KV-head cross-attend X = [K; V] with QK-norm, the compactor's own RoPE and logits
+ * scaled by d_l (App. A, "Cross-attention"), are refined by latent self-attention and a GELU
+ * FFN, and are projected by W_key / W_val; C_k is re-rotated at evenly spaced output positions
+ * over the compacted range (App. B, single-pass recipe, step 5). beta is not produced (the
+ * reported configuration sets beta = 0, Sec. 2.1).
+ *
+ * Conventions
+ *  - Pointers are DEVICE pointers unless their name starts with h_ (host). All calls are
+ *    stream-ordered on the given `stream` (a cudaStream_t; NULL = legacy default stream) and
+ *    asynchronous unless stated. Host output arguments (h_*) are written before return.
+ *  - Tensors are row-major, 16-bit values are bf16 (round-to-nearest-even when produced).
+ *  - Calls never throw and never abort; every failure is a still_status. A device-side
+ *    failure (a bounded wait that expired) is recorded and reported by
+ *    still_get_device_status.
+ *  - A context is bound to one device and is not thread-safe; use one per host thread.
+ */
+#ifndef STILL_H_
+#define STILL_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  STILL_OK = 0,
+  STILL_ERR_INVALID_ARG = 1, /* null pointer, bad enum or flag value */
+  STILL_ERR_UNSUPPORTED = 2, /* a configuration this build does not implement */
+  STILL_ERR_SHAPE = 3,       /* inconsistent sizes (t > N, t > t_max, N = 0, ...) */
+  STILL_ERR_ALIGNMENT = 4,   /* a pointer or stride breaks the required alignment */
+  STILL_ERR_NOT_LOADED = 5,  /* layer weights were never loaded */
+  STILL_ERR_OOM = 6,         /* device allocation failed or workspace limit exceeded */
+  STILL_ERR_CUDA = 7,        /* a CUDA runtime call failed (sticky errors included) */
+  STILL_ERR_TIMEOUT = 8      /* a device-side bounded wait expired (see device status) */
+} still_status;
+
+typedef struct still_ctx still_ctx; /* opaque: weight copies, precompute, workspace */
+
+/* One layer's compactor hyperparameters (App. A, "Canonical configuration summary").
+ * Implemented: n_blocks = 1, cross_every_block = 1, n_cross_heads = n_self_heads,
+ * d_latent % 256 == 0, head_dim in {64, 128, 256}, ffn_dim % 64 == 0 (or 0 = no FFN),
+ * compactor_rope = 1, rope_fix = 1. Other values return STILL_ERR_UNSUPPORTED. */
+typedef struct {
+  int32_t n_kv_heads;        /* H: KV-heads of the base model */
+  int32_t head_dim;          /* d: base model head dim */
+  int32_t d_latent;          /* D = d_l: compactor width; every attention head is D wide */
+  int32_t n_cross_heads;     /* n_c */
+  int32_t n_self_heads;      /* n_s */
+  int32_t ffn_dim;           /* r * d_l, 0 = no FFN sublayer */
+  int32_t n_blocks;          /* B */
+  int32_t cross_every_block; /* 1 = canonical (CA in every block), 0 = resampler */
+  int32_t t_max;             /* rows of each latent bank; a call uses rows [0, t) */
+  int32_t final_norm;        /* RMSNorm before the output heads (0 = off, the default) */
+  int32_t compactor_rope;    /* apply the compactor's RoPE in cross-attention */
+  int32_t rope_fix;          /* un-rotate cached keys / re-rotate C_k */
+  double rope_theta;         /* base model RoPE base */
+  double rope_theta_compactor; /* compactor RoPE base (canonical 10) */
+  double logit_scale;        /* 0 => d_latent (canonical) */
+  float rms_eps;             /* RMSNorm epsilon (1e-6) */
+  float l2_eps;              /* QK-norm epsilon (1e-12) */
+} still_layer_config;
+
+/* One layer's weights, device bf16, x @ W convention (row = input feature).
+ * n = n_cross_heads = n_self_heads; head i of a multi-head projection is the column block
+ * [i*D, (i+1)*D) of its [in, n*D] matrix, and row block i of an [n*D, D] output projection.
+ *   Z    [H, t_max, D]   latent banks (App. A, "Latent queries")
+ *   Wq   [D, n*D]   bq [n*D]    cross-attention query projection and bias
+ *   Wk   [2d, n*D]  bk [n*D]    cross-attention key projection and bias (X = [K; V] rows)
+ *   Wv   [2d, n*D]              cross-attention value projection (no bias)
+ *   Wo   [n*D, D]               cross-attention output projection
+ *   Sq   [D, n*D]   sbq [n*D]   self-attention query projection and bias
+ *   Sk   [D, n*D]   sbk [n*D]   self-attention key projection and bias
+ *   Sv   [D, n*D]               self-attention value projection
+ *   So   [n*D, D]               self-attention output projection
+ *   W1   [D, F]     W2 [F, D]   FFN (no biases); may be NULL when ffn_dim = 0
+ *   Wkey [D, d]     Wval [D, d] output heads
+ * The library copies (and re-lays out) everything it needs; the caller may free the inputs
+ * after the call's stream work completes. */
+typedef struct {
+  const void *Z, *Wq, *bq, *Wk, *bk, *Wv, *Wo;
+  const void *Sq, *sbq, *Sk, *sbk, *Sv, *So;
+  const void *W1, *W2, *Wkey, *Wval;
+} still_layer_weights;
+
+/* Cache positions: token i of the segment sits at start + i * step (exact fp64). Segments
+ * are concatenated in order and must cover the N tokens exactly. At most 8 per call. */
+typedef struct {
+  double start;
+  double step;
+  int64_t count;
+} still_pos_segment;
+
+/* Creates a context on `device` (makes it current). */
+still_status still_create(int device, still_ctx** out);
+/* Frees everything the context owns. Synchronizes the device first. */
+still_status still_destroy(still_ctx* ctx);
+/* Static string for a status code. */
+const char* still_status_string(still_status s);
+
+/* Copies layer `layer`'s weights into the context and runs the input-independent precompute
+ * (App. A: the block-1 latent query q^ = L2norm(RMSNorm(Z) W_Q + b_Q) per KV-head and
+ * cross head; the value/output product W_V,i W_O,i). Replaces an earlier load of the layer. */
+still_status still_load_layer_weights(still_ctx* ctx, int32_t layer,
+                                      const still_layer_config* cfg,
+                                      const still_layer_weights* w, void* stream);
+
+/* Compacts one layer (Sec. 2.1; App. B single-pass recipe steps 3-5).
+ *   K, V       [N, H, d] bf16 device, element strides strides_kv = {s_token, s_head, s_dim}
+ *              (s_dim must be 1; rows 16-byte aligned is not required)
+ *   h_segments key positions (NULL and n_segments = 0 => 0..N-1); the latent query
+ *              positions and the C_k output positions are t points spaced evenly from the
+ *              smallest to the largest key position, both ends included (App. A,
+ *              Cross-attention; App. B, step 5).
+ *   t          compact length, 1 <= t <= min(N, t_max)
+ *   Ck, Cv     [t, H, d] bf16 device outputs, caller-owned, contiguous
+ *   h_out_pos_start, h_out_pos_step  (optional) output positions start + j * step
+ *   h_pos_offset (optional) logical minus physical length, N - t (App. B, "Logical vs.
+ *              physical cache length")
+ * Returns STILL_ERR_TIMEOUT/STILL_ERR_CUDA only for failures detected at launch; use
+ * still_get_device_status after synchronizing to see device-side failures. */
+still_status still_compact_layer(still_ctx* ctx, int32_t layer, const void* K, const void* V,
+                                 const int64_t strides_kv[3],
+                                 const still_pos_segment* h_segments, int32_t n_segments,
+                                 int64_t N, int32_t t, void* Ck, void* Cv,
+                                 double* h_out_pos_start, double* h_out_pos_step,
+                                 int64_t* h_pos_offset, void* stream);
+
+/* Compacts layers 0..n_layers-1 (all loaded) over the same positions: the per-layer
+ * compactors share nothing at forward time (App. M, "No inter-layer compactor channel"), so
+ * this is one stream-ordered launch sequence over the layer stack. K[l], V[l], Ck[l], Cv[l] are device
+ * pointers (arrays of n_layers entries, host memory). */
+still_status still_compact_stack(still_ctx* ctx, int32_t n_layers, const void* const* K,
+                                 const void* const* V, const int64_t strides_kv[3],
+                                 const still_pos_segment* h_segments, int32_t n_segments,
+                                 int64_t N, int32_t t, void* const* Ck, void* const* Cv,
+                                 double* h_out_pos_start, double* h_out_pos_step,
+                                 int64_t* h_pos_offset, void* stream);
+
+/* Ragged batch of B sequences packed along the token axis.
+ *   Kpacked, Vpacked [sum N_b, H, d] bf16 (contiguous), h_cu_seqlens[B+1] token offsets
+ *   h_segments / h_seg_per_seq: sequence b uses h_seg_per_seq[b] consecutive segments
+ *     (NULL => positions 0..N_b-1 for every sequence)
+ *   h_t[B] compact lengths; h_cu_t[B+1] offsets of each sequence's rows in Ck/Cv
+ *   Ck, Cv [sum t_b, H, d] bf16; h_pos_offset[B] (optional) N_b - t_b.
+ * Sequence b uses rows [0, t_b) of every latent bank. */
+still_status still_compact_layer_ragged(still_ctx* ctx, int32_t layer, const void* Kpacked,
+                                        const void* Vpacked, const int64_t* h_cu_seqlens,
+                                        int32_t B, const still_pos_segment* h_segments,
+                                        const int32_t* h_seg_per_seq, const int32_t* h_t,
+                                        const int64_t* h_cu_t, void* Ck, void* Cv,
+                                        int64_t* h_pos_offset, void* stream);
+
+/* Ragged batch over layers 0..n_layers-1: per-layer packed K/V and Ck/Cv pointer arrays
+ * (host arrays of device pointers); the other arguments as still_compact_layer_ragged. */
+still_status still_compact_stack_ragged(still_ctx* ctx, int32_t n_layers,
+                                        const void* const* Kpacked, const void* const* Vpacked,
+                                        const int64_t* h_cu_seqlens, int32_t B,
+                                        const still_pos_segment* h_segments,
+                                        const int32_t* h_seg_per_seq, const int32_t* h_t,
+                                        const int64_t* h_cu_t, void* const* Ck,
+                                        void* const* Cv, int64_t* h_pos_offset, void* stream);
+
+/* Device workspace bytes a call with up to max_tokens tokens and compact length max_t needs
+ * for layer 0's configuration (the context allocates it on demand and keeps it). */
+still_status still_workspace_size(const still_ctx* ctx, int64_t max_tokens, int32_t max_t,
+                                  size_t* bytes);
+
+/* Upper bound on the workspace the context may allocate (default 48 GiB). Calls whose
+ * workspace would exceed it process the KV-heads in smaller groups, or fail with
+ * STILL_ERR_OOM when even one group does not fit. */
+still_status still_set_workspace_limit(still_ctx* ctx, size_t bytes);
+
+/* Synchronizes `stream`, then reports (and clears) the device error record:
+ * STILL_ERR_TIMEOUT if a kernel's bounded wait expired, STILL_ERR_CUDA if the stream
+ * reported an error. h_detail (optional, 4 ints): code, site, block, count. */
+still_status still_get_device_status(still_ctx* ctx, void* stream, int32_t* h_detail);
+
+/* Kernel classes of the launch sequence, for launch counts and timings. */
+typedef enum {
+  STILL_K_STRIP = 0,    /* RoPE-fix + [K; V] concat (hi/lo)                 */
+  STILL_K_TABLES,       /* compactor-RoPE angle table                       */
+  STILL_K_KEYPROJ,      /* k = RoPE_c(X W_K + b_K) (2-pass tcgen05 GEMM)    */
+  STILL_K_QROPE,        /* q = RoPE_c(q^) at the latent query positions     */
+  STILL_K_SCORES,       /* S = d_l q.k / |k| (3-pass tcgen05 GEMM)          */
+  STILL_K_SOFTMAX,      /* cross-attention row softmax                      */
+  STILL_K_PX,           /* O = P X (2-pass tcgen05 GEMM, split-K)           */
+  STILL_K_PXSPLIT,      /* O -> hi/lo                                       */
+  STILL_K_VO,           /* Z' = Z + O (W_V W_O) (3-pass tcgen05 GEMM)       */
+  STILL_K_NORM,         /* RMSNorm                                          */
+  STILL_K_SA_PROJ,      /* self-attention q/k projections                   */
+  STILL_K_SA_V,         /* self-attention v projection                      */
+  STILL_K_SA_SCORES,    /* self-attention scores                            */
+  STILL_K_SA_SOFTMAX,   /* self-attention row softmax                       */
+  STILL_K_SA_PV,        /* self-attention P v                               */
+  STILL_K_SO,           /* self-attention output projection + residual      */
+  STILL_K_FFN1,         /* GELU(x W_1)                                      */
+  STILL_K_FFN2,         /* (.) W_2 + residual                               */
+  STILL_K_HEADS,        /* C_k, C_v output heads + re-rotation              */
+  STILL_K_LOAD,         /* weight-load precompute GEMMs                     */
+  STILL_K_COUNT
+} still_kernel_class;
+
+/* Starts (enable = 1) or stops kernel timing and clears the counters. While enabled, every
+ * launch of the library's kernels is bracketed by a CUDA event pair on its stream. Launch
+ * counts are kept whether or not timing is enabled (reset by this call). */
+still_status still_profile_enable(still_ctx* ctx, int32_t enable);
+/* Launches and total event time (ms) of one kernel class since the last enable call.
+ * Synchronizes the device when timings are pending. */
+still_status still_profile_read(still_ctx* ctx, int32_t cls, int64_t* h_launches, double* h_ms);
+/* Static name of a kernel class ("scores", "softmax", ...). */
+const char* still_kernel_class_name(int32_t cls);
+
+/* Compact budget t = round(N / ratio) with halves rounded up (App. J exact-results table,
+ * K column: 8192 / 50 -> 164, 65536 / 50 -> 1311). Host-only. */
+int64_t still_budget(int64_t n_tokens, int64_t ratio);
+
+/* Retained KV bytes M_KV(S) = 2 L H d b S (App. B, "Deployment accounting"). Host-only. */
+int64_t still_kv_bytes(int64_t n_layers, int64_t n_kv_heads, int64_t head_dim,
+                       int64_t elem_bytes, int64_t n_slots);
+
+/* Number of per-layer compactor parameters (App. D) for a configuration: bank H*t*D,
+ * per CA block 2 n D^2 + 4 d n D, per SA block 4 n D^2, per FFN block 2 F D, heads
+ * 2 D d + D (the D-wide beta head included, as in the paper's count). Host-only. */
+int64_t still_param_count(const still_layer_config* cfg, int32_t t);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* STILL_H_ */

@@ -1,0 +1,322 @@
+// GEMM epilogues: TMEM -> registers -> fused element-wise work -> global memory.
+// Each epilogue thread owns one accumulator row (TMEM lane) of a 128 x BN tile and walks its
+// columns 32 at a time.
+#pragma once
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include "tc_gemm.cuh"
+
+namespace still {
+
+// Element offset of (batch b, row r, column c) as an affine function of their div/mod parts.
+struct AffineMap {
+  int32_t bdiv = 1, rdiv = 1 << 30, cdiv = 1 << 30;
+  int64_t b1 = 0, b0 = 0, r1 = 0, r0 = 0, c1 = 0, c0 = 0, k = 0;
+  __device__ __forceinline__ int64_t at(int b, int r, int c) const {
+    return (int64_t)(b / bdiv) * b1 + (int64_t)(b % bdiv) * b0 + (int64_t)(r / rdiv) * r1 +
+           (int64_t)(r % rdiv) * r0 + (int64_t)(c / cdiv) * c1 + (int64_t)(c % cdiv) * c0 + k;
+  }
+};
+
+enum OutKind : int32_t { OUT_F32 = 0, OUT_BF16 = 1, OUT_HILO = 2, OUT_F32_ATOMIC = 3 };
+
+__device__ __forceinline__ void split_hilo(float x, __nv_bfloat16& hi, __nv_bfloat16& lo) {
+  hi = __float2bfloat16_rn(x);
+  lo = __float2bfloat16_rn(x - __bfloat162float(hi));
+}
+
+__device__ __forceinline__ float gelu_erf(float x) {
+  return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f));
+}
+
+// General epilogue: v = acc * alpha [* colscale(c)] [* rowscale(r)] [+ bias(c)]
+//   -> [sumsq accumulation] -> [GELU] -> [+ residual] -> store (f32 / bf16 / hi-lo / atomic f32)
+// colscale / rowscale = 1 / max(sqrt(sumsq[idx]), eps) from a sum-of-squares buffer.
+// Host contract: csm, resm and (when vec_ok) om are contiguous in c (c0 == 1) with cdiv a
+// multiple of 32, so every 32-column chunk maps to 32 consecutive elements; ss_seg % 32 == 0.
+struct EpiAffine {
+  int32_t kind = OUT_F32;
+  void* out = nullptr;
+  int64_t lo_off = 0;  // OUT_HILO: lo element offset from hi
+  AffineMap om;
+  float alpha = 1.f;
+  const float* bias = nullptr;  // indexed by column
+  const float* col_ss = nullptr;
+  AffineMap csm;  // (b, 0, c) -> index
+  const float* row_ss = nullptr;
+  AffineMap rsm;  // (b, r, 0) -> index
+  float eps = 1e-12f;
+  int32_t gelu = 0;
+  int32_t res_kind = 0;  // 0 none, 1 f32, 2 bf16
+  const void* res = nullptr;
+  AffineMap resm;
+  float* sumsq = nullptr;  // accumulate sum_c v^2 over segments of ss_seg columns
+  AffineMap ssm;           // (b, r, c / ss_seg) -> index
+  int32_t ss_seg = 1 << 30;
+  int32_t vec_ok = 0;  // host: om.c0 == 1, cdiv % 32 == 0, 16-B aligned rows
+  int32_t tile_cols_ = 256;  // the tile width BN, set by the launcher
+
+  __device__ void operator()(const GemmParams& p, const TileCoord& tc, int row, uint32_t taddr,
+                             int half) const {
+    const int r = tc.tm * kBM + row;
+    const bool rvalid = r < p.M;
+    const float eps2 = eps * eps;
+    float rscale = alpha;
+    if (row_ss != nullptr && rvalid) rscale *= rsqrtf(fmaxf(row_ss[rsm.at(tc.b, r, 0)], eps2));
+    float ss = 0.f;
+    int ss_cur = -1;
+    for (int cc = 32 * half; cc < tile_cols_; cc += 64) {
+      float v[32];
+      tmem_ld32(taddr + (uint32_t)cc, v);
+      const int c0 = tc.tn * tile_cols_ + cc;
+      if (!rvalid || c0 >= p.N) continue;
+      const int nv = min(32, p.N - c0);
+#pragma unroll
+      for (int e = 0; e < 32; ++e) v[e] *= rscale;
+      if (col_ss != nullptr) {
+        const float* cs = col_ss + csm.at(tc.b, 0, c0);
+#pragma unroll
+        for (int e = 0; e < 32; ++e)
+          if (e < nv) v[e] *= rsqrtf(fmaxf(cs[e], eps2));
+      }
+      if (bias != nullptr) {
+#pragma unroll
+        for (int e = 0; e < 32; ++e)
+          if (e < nv) v[e] += bias[c0 + e];
+      }
+      if (sumsq != nullptr) {
+        const int seg = c0 / ss_seg;
+        if (seg != ss_cur) {
+          if (ss_cur >= 0) atomicAdd(&sumsq[ssm.at(tc.b, r, ss_cur)], ss);
+          ss = 0.f;
+          ss_cur = seg;
+        }
+#pragma unroll
+        for (int e = 0; e < 32; ++e)
+          if (e < nv) ss += v[e] * v[e];
+      }
+      if (gelu) {
+#pragma unroll
+        for (int e = 0; e < 32; ++e) v[e] = gelu_erf(v[e]);
+      }
+      if (res_kind != 0 && (kind != OUT_F32_ATOMIC || tc.split == 0)) {
+        const int64_t o = resm.at(tc.b, r, c0);
+        if (res_kind == 1) {
+          const float* rp = static_cast<const float*>(res) + o;
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (e < nv) v[e] += rp[e];
+        } else {
+          const __nv_bfloat16* rp = static_cast<const __nv_bfloat16*>(res) + o;
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (e < nv) v[e] += __bfloat162float(rp[e]);
+        }
+      }
+      store32(p, tc.b, r, c0, v);
+    }
+    if (sumsq != nullptr && rvalid && ss_cur >= 0) atomicAdd(&sumsq[ssm.at(tc.b, r, ss_cur)], ss);
+  }
+
+  __device__ __forceinline__ void store32(const GemmParams& p, int b, int r, int c0,
+                                          const float (&v)[32]) const {
+    const bool full = vec_ok && (c0 + 32 <= p.N);
+    if (full) {
+      const int64_t o = om.at(b, r, c0);
+      if (kind == OUT_F32) {
+        float4* dst = reinterpret_cast<float4*>(static_cast<float*>(out) + o);
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+      } else if (kind == OUT_F32_ATOMIC) {
+        float4* dst = reinterpret_cast<float4*>(static_cast<float*>(out) + o);
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          atomicAdd(dst + q, make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]));
+      } else {
+        __align__(16) __nv_bfloat16 hi[32];
+        __align__(16) __nv_bfloat16 lo[32];
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          if (kind == OUT_HILO)
+            split_hilo(v[e], hi[e], lo[e]);
+          else
+            hi[e] = __float2bfloat16_rn(v[e]);
+        }
+        uint4* dh = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(out) + o);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) dh[q] = reinterpret_cast<const uint4*>(hi)[q];
+        if (kind == OUT_HILO) {
+          uint4* dl = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(out) + o + lo_off);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) dl[q] = reinterpret_cast<const uint4*>(lo)[q];
+        }
+      }
+      return;
+    }
+#pragma unroll 4
+    for (int e = 0; e < 32; ++e) {
+      const int c = c0 + e;
+      if (c >= p.N) break;
+      const int64_t o = om.at(b, r, c);
+      if (kind == OUT_F32) {
+        static_cast<float*>(out)[o] = v[e];
+      } else if (kind == OUT_F32_ATOMIC) {
+        atomicAdd(static_cast<float*>(out) + o, v[e]);
+      } else if (kind == OUT_BF16) {
+        static_cast<__nv_bfloat16*>(out)[o] = __float2bfloat16_rn(v[e]);
+      } else {
+        __nv_bfloat16 h, l;
+        split_hilo(v[e], h, l);
+        static_cast<__nv_bfloat16*>(out)[o] = h;
+        static_cast<__nv_bfloat16*>(out)[o + lo_off] = l;
+      }
+    }
+  }
+};
+
+// Cache positions given as segments: position of token idx = start[k] + (idx - begin[k]) * step[k].
+struct PosSegs {
+  int32_t n = 0;
+  int64_t begin[9] = {0};
+  double start[8] = {0};
+  double step[8] = {0};
+};
+
+__device__ __forceinline__ double seg_position(const PosSegs& s, int64_t idx) {
+  int k = 0;
+#pragma unroll 1
+  while (k + 1 < s.n && idx >= s.begin[k + 1]) ++k;
+  return s.start[k] + (double)(idx - s.begin[k]) * s.step[k];
+}
+
+// Key projection epilogue (cross-attention keys):
+//   k~ = acc + b_K;  sumsq(token, head) += |k~|^2;  k = RoPE_c(k~, p_n)  -> hi/lo bf16.
+// Columns are in "pair-chunk" order: within each 256-column tile, columns [0,128) hold the
+// first elements of 128 RoPE pairs and [128,256) their partners, so a tile owns whole pairs.
+// The angle p_n * omega_m is split as G_g * omega_m (table, built in fp64) + delta * omega_m
+// (fp32, delta = p_n - G_g in [0, kPosGrain)), combined by the angle-addition formulas.
+constexpr int kPosGrain = 32;
+
+struct EpiRopeC {
+  __nv_bfloat16* out = nullptr;  // [H][n][N][2D]: hi at [0, D), lo at [D, 2D)
+  float* sumsq = nullptr;        // [H][n][N]
+  const float* bias = nullptr;   // [n*D], pair-chunk order
+  const float2* coarse = nullptr;  // [G][D/2]: (cos, sin)(G_g * omega_m)
+  const float* omega = nullptr;    // [D/2] fp32
+  PosSegs segs;
+  double pmin = 0;
+  int32_t D = 0, nheads = 0, ncoarse = 0;
+  int64_t Ntok = 0;
+  int32_t tile_cols_ = 256;  // must be 256: a tile holds 128 whole RoPE pairs
+
+  __device__ void operator()(const GemmParams& p, const TileCoord& tc, int row, uint32_t taddr,
+                             int half) const {
+    const int r = tc.tm * kBM + row;
+    const bool rvalid = r < p.M;
+    const int c_tile = tc.tn * 256;
+    const int head = c_tile / D;
+    const int f_tile = c_tile % D;       // column of this tile inside the head (pair-chunk order)
+    const int m_base = (f_tile / 256) * 128;  // first pair index of this tile
+    double pos = rvalid ? seg_position(segs, r) : pmin;
+    int g = (int)floor((pos - pmin) / (double)kPosGrain);
+    g = max(0, min(g, ncoarse - 1));
+    const float delta = (float)(pos - (pmin + (double)g * kPosGrain));
+    const int64_t row_out = ((int64_t)(tc.b * nheads + head) * Ntok + r) * (2 * (int64_t)D);
+    float ss = 0.f;
+    for (int u = 32 * half; u < 128; u += 64) {
+      float a[32], bb[32];
+      tmem_ld32(taddr + (uint32_t)u, a);
+      tmem_ld32(taddr + (uint32_t)(128 + u), bb);
+      if (!rvalid) continue;
+      __align__(16) __nv_bfloat16 ah[32], al[32], bh[32], bl[32];
+      const float2* crow = coarse + (int64_t)g * (D / 2) + m_base + u;
+#pragma unroll 8
+      for (int e = 0; e < 32; ++e) {
+        const int m = m_base + u + e;
+        const float x = a[e] + bias[c_tile + u + e];
+        const float y = bb[e] + bias[c_tile + 128 + u + e];
+        ss += x * x + y * y;
+        float sf, cf;
+        __sincosf(delta * omega[m], &sf, &cf);
+        const float2 cs = crow[e];
+        const float cw = cs.x * cf - cs.y * sf;  // cos(G w + delta w)
+        const float sw = cs.y * cf + cs.x * sf;  // sin(G w + delta w)
+        split_hilo(x * cw - y * sw, ah[e], al[e]);
+        split_hilo(x * sw + y * cw, bh[e], bl[e]);
+      }
+      __nv_bfloat16* o = out + row_out + f_tile + u;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        reinterpret_cast<uint4*>(o)[q] = reinterpret_cast<const uint4*>(ah)[q];
+        reinterpret_cast<uint4*>(o + 128)[q] = reinterpret_cast<const uint4*>(bh)[q];
+        reinterpret_cast<uint4*>(o + D)[q] = reinterpret_cast<const uint4*>(al)[q];
+        reinterpret_cast<uint4*>(o + D + 128)[q] = reinterpret_cast<const uint4*>(bl)[q];
+      }
+    }
+    if (rvalid) atomicAdd(&sumsq[(int64_t)(tc.b * nheads + head) * Ntok + r], ss);
+  }
+};
+
+// Output heads: columns [0, d) = Z_out W_key, re-rotated by the base RoPE at the output
+// position of latent j; columns [d, 2d) = Z_out W_val. Rows r = h * t + j. bf16 stores into
+// the caller's C_k / C_v with element strides (st, sh, sd). omega = theta^(-2m/d) in fp64;
+// the angle is reduced modulo 2 pi in fp64 before the fp32 sin/cos.
+struct EpiHeads {
+  __nv_bfloat16* ck = nullptr;
+  __nv_bfloat16* cv = nullptr;
+  int64_t st = 0, sh = 0, sd = 1;
+  int32_t t = 0, d = 0;
+  double pstart = 0, pstep = 0;
+  const double* omega = nullptr;  // [d/2]
+  int32_t rope = 1;
+  int32_t tile_cols_ = 256;
+
+  __device__ void operator()(const GemmParams& p, const TileCoord& tc, int row, uint32_t taddr,
+                             int half) const {
+    const int r = tc.tm * kBM + row;
+    const bool rvalid = r < p.M;
+    const int h = r / t, j = r % t;
+    const int c_tile = tc.tn * tile_cols_;
+    const double pos = pstart + (double)j * pstep;
+    const int64_t obase = (int64_t)j * st + (int64_t)h * sh;
+    const int hd = d / 2;
+    for (int cc = 32 * half; cc < tile_cols_; cc += 64) {
+      const int c0 = c_tile + cc;
+      if (c0 >= p.N) break;
+      if (c0 < d) {
+        // key columns: process pairs (m, m + d/2) when visiting the first half
+        if (c0 >= hd) continue;
+        float a[32], b[32];
+        tmem_ld32(taddr + (uint32_t)cc, a);
+        tmem_ld32(taddr + (uint32_t)(cc + hd), b);
+        if (!rvalid) continue;
+#pragma unroll 4
+        for (int e = 0; e < 32; ++e) {
+          const int m = c0 + e;
+          float cw = 1.f, sw = 0.f;
+          if (rope) {
+            double ang = pos * omega[m];
+            ang -= 6.283185307179586 * rint(ang * 0.15915494309189535);
+            sincosf((float)ang, &sw, &cw);
+          }
+          const float x = a[e], y = b[e];
+          ck[obase + (int64_t)m * sd] = __float2bfloat16_rn(x * cw - y * sw);
+          ck[obase + (int64_t)(m + hd) * sd] = __float2bfloat16_rn(x * sw + y * cw);
+        }
+      } else {
+        float v[32];
+        tmem_ld32(taddr + (uint32_t)cc, v);
+        if (!rvalid) continue;
+#pragma unroll 4
+        for (int e = 0; e < 32; ++e) {
+          const int f = c0 + e - d;
+          if (f < d) cv[obase + (int64_t)f * sd] = __float2bfloat16_rn(v[e]);
+        }
+      }
+    }
+  }
+};
+
+}  // namespace still

@@ -1,0 +1,94 @@
+// Host side of the tcgen05 GEMM: TMA descriptors, tile/split bookkeeping, launch.
+#pragma once
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include <cstdio>
+#include <mutex>
+
+#include "epilogues.cuh"
+
+namespace still {
+
+// A 2-D row-major 16-bit operand as TMA sees it: `rows` rows of `cols` elements, row pitch
+// `pitch` elements (pitch * 2 must be a multiple of 16 and ptr 16-byte aligned).
+struct Operand2D {
+  const void* ptr = nullptr;
+  int64_t rows = 0, cols = 0, pitch = 0;
+};
+
+inline PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  });
+  return fn;
+}
+
+// Box = box_rows x 64 elements, 128-byte swizzle, zero fill out of bounds.
+inline bool make_tmap(CUtensorMap* m, const Operand2D& op, int box_rows) {
+  auto enc = tensor_map_encoder();
+  if (enc == nullptr) return false;
+  if ((reinterpret_cast<uintptr_t>(op.ptr) & 15) != 0 || (op.pitch * 2) % 16 != 0) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)op.cols, (cuuint64_t)op.rows};
+  cuuint64_t strides[1] = {(cuuint64_t)(op.pitch * 2)};
+  cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(op.ptr), dims,
+                   strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+// Fills the derived fields of p. Returns false on an invalid description.
+template <int BN>
+inline bool finalize_gemm(GemmParams& p, int ab_fmt) {
+  if (p.M <= 0 || p.N <= 0 || p.batch <= 0 || p.npass < 1 || p.npass > 3 || p.bdiv < 1)
+    return false;
+  int iters = 0;
+  for (int i = 0; i < p.npass; ++i) {
+    if (p.pass[i].klen <= 0 || p.pass[i].klen % kBK != 0) return false;
+    if (p.pass[i].a_koff % 8 != 0 || p.pass[i].b_koff % 8 != 0) return false;
+    iters += p.pass[i].klen / kBK;
+  }
+  if ((p.a_k0 | p.a_k1 | p.b_k0 | p.b_k1) % 8 != 0) return false;
+  p.iters_total = iters;
+  if (p.ksplit < 1) p.ksplit = 1;
+  if (p.ksplit > iters) p.ksplit = iters;
+  p.tiles_m = (p.M + kBM - 1) / kBM;
+  p.tiles_n = (p.N + BN - 1) / BN;
+  const int64_t nt = (int64_t)p.tiles_m * p.tiles_n * p.ksplit * p.batch;
+  if (nt > 0x7fffffff) return false;
+  p.ntiles = (int)nt;
+  p.idesc = idesc_f16(kBM, BN, ab_fmt);
+  return true;
+}
+
+template <int BN, class Epi>
+inline cudaError_t launch_gemm(const Operand2D& A, const Operand2D& B, GemmParams p, Epi epi,
+                               int ab_fmt, int num_sms, cudaStream_t stream) {
+  using S = GemmSmem<BN>;
+  if (!finalize_gemm<BN>(p, ab_fmt)) return cudaErrorInvalidValue;
+  CUtensorMap ta, tb;
+  if (!make_tmap(&ta, A, kBM) || !make_tmap(&tb, B, BN)) return cudaErrorInvalidValue;
+  epi.tile_cols_ = BN;
+  auto kern = tc_gemm_kernel<BN, Epi>;
+  static thread_local bool attr_set = false;  // per instantiation
+  if (!attr_set) {
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::kBytes);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  const int grid = p.ntiles < num_sms ? p.ntiles : num_sms;
+  kern<<<grid, kGemmThreads, S::kBytes, stream>>>(ta, tb, p, epi);
+  return cudaGetLastError();
+}
+
+}  // namespace still

@@ -1,0 +1,465 @@
+// Memory-bound kernels of the compactor path: RoPE-fix strip, RoPE tables, query rotation,
+// softmax, hi/lo conversion, RMSNorm, weight re-layout.
+#include <algorithm>
+#include <type_traits>
+
+#include "kernels.cuh"
+
+namespace still {
+
+namespace {
+
+constexpr double kTwoPi = 6.283185307179586;
+constexpr double kInvTwoPi = 0.15915494309189535;
+constexpr float kLog2e = 1.4426950408889634f;
+
+// angle reduced to [-pi, pi] in fp64, then sin/cos in fp32 (|error| ~1e-7)
+__device__ __forceinline__ void sincos_reduced(double ang, float* s, float* c) {
+  ang -= kTwoPi * rint(ang * kInvTwoPi);
+  sincosf((float)ang, s, c);
+}
+
+constexpr int kStripTok = 32;
+
+// One CTA = 32 tokens x one KV-head. Keys: inverse base-model RoPE on pairs (m, m + d/2)
+// (Sec. 2.2, RoPE-fix); values pass through. Writes X (bf16 hi | key lo) and XT (fp16 hi, lo).
+__global__ void __launch_bounds__(256) strip_kernel(const __nv_bfloat16* __restrict__ K,
+                                                    const __nv_bfloat16* __restrict__ V,
+                                                    int64_t sN, int64_t sH, int64_t N, int H,
+                                                    int d, PosSegs segs, double theta,
+                                                    int rope_fix, __nv_bfloat16* __restrict__ X,
+                                                    __half* __restrict__ XT, int64_t Np) {
+  extern __shared__ __align__(16) uint8_t sm[];
+  const int half = d / 2;
+  double* omega = reinterpret_cast<double*>(sm);
+  constexpr int kLd = kStripTok + 2;
+  __half* thi = reinterpret_cast<__half*>(omega + half);
+  __half* tlo = thi + 2 * d * kLd;
+  const int h = blockIdx.y;
+  const int64_t n0 = (int64_t)blockIdx.x * kStripTok;
+  for (int m = threadIdx.x; m < half; m += blockDim.x) omega[m] = pow(theta, -2.0 * m / d);
+  __syncthreads();
+  const int d3 = 3 * d;
+  for (int it = threadIdx.x; it < kStripTok * half; it += blockDim.x) {
+    const int tok = it / half, m = it % half;
+    const int64_t n = n0 + tok;
+    float a = 0.f, b = 0.f;
+    if (n < N) {
+      const __nv_bfloat16* kr = K + n * sN + (int64_t)h * sH;
+      a = __bfloat162float(kr[m]);
+      b = __bfloat162float(kr[m + half]);
+      if (rope_fix) {
+        float sw, cw;
+        sincos_reduced(seg_position(segs, n) * omega[m], &sw, &cw);
+        const float x = a * cw + b * sw;
+        const float y = -a * sw + b * cw;
+        a = x;
+        b = y;
+      }
+      __nv_bfloat16* xr = X + ((int64_t)h * N + n) * d3;
+      __nv_bfloat16 hi, lo;
+      split_hilo(a, hi, lo);
+      xr[m] = hi;
+      xr[2 * d + m] = lo;
+      split_hilo(b, hi, lo);
+      xr[m + half] = hi;
+      xr[2 * d + m + half] = lo;
+    }
+    const __half ah = __float2half_rn(a), bh = __float2half_rn(b);
+    thi[m * kLd + tok] = ah;
+    thi[(m + half) * kLd + tok] = bh;
+    tlo[m * kLd + tok] = __float2half_rn(a - __half2float(ah));
+    tlo[(m + half) * kLd + tok] = __float2half_rn(b - __half2float(bh));
+  }
+  for (int it = threadIdx.x; it < kStripTok * d; it += blockDim.x) {
+    const int tok = it / d, f = it % d;
+    const int64_t n = n0 + tok;
+    float v = 0.f;
+    if (n < N) {
+      const __nv_bfloat16 vb = V[n * sN + (int64_t)h * sH + f];
+      v = __bfloat162float(vb);
+      X[((int64_t)h * N + n) * d3 + d + f] = vb;
+    }
+    const __half vh = __float2half_rn(v);
+    thi[(d + f) * kLd + tok] = vh;
+    tlo[(d + f) * kLd + tok] = __float2half_rn(v - __half2float(vh));
+  }
+  __syncthreads();
+  const int64_t ld = 2 * Np;
+  for (int it = threadIdx.x; it < 2 * d * kStripTok; it += blockDim.x) {
+    const int f = it / kStripTok, tok = it % kStripTok;
+    const int64_t n = n0 + tok;
+    if (n < Np) {
+      __half* row = XT + ((int64_t)h * 2 * d + f) * ld;
+      row[n] = thi[f * kLd + tok];
+      row[Np + n] = tlo[f * kLd + tok];
+    }
+  }
+}
+
+__global__ void rope_tables_kernel(float2* coarse, float* omega, int G, int D, double pmin,
+                                   double theta_c) {
+  const int half = D / 2;
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (int64_t)G * half) return;
+  const int g = (int)(idx / half), m = (int)(idx % half);
+  const double w = pow(theta_c, -2.0 * m / D);
+  float s, c;
+  sincos_reduced((pmin + (double)g * kPosGrain) * w, &s, &c);
+  coarse[idx] = make_float2(c, s);
+  if (g == 0) omega[m] = (float)w;
+}
+
+__global__ void q_rope_kernel(const float* __restrict__ qhat, int t_max, int b0, int nb, int t,
+                              int D, double qstart, double qstep, const double* omega_c,
+                              int use_rope, __nv_bfloat16* __restrict__ qhl) {
+  const int half = D / 2;
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (int64_t)t * half) return;
+  const int j = (int)(idx / half), m = (int)(idx % half);
+  float s = 0.f, c = 1.f;
+  if (use_rope) sincos_reduced((qstart + (double)j * qstep) * omega_c[m], &s, &c);
+  const int f1 = (m / 128) * 256 + (m % 128), f2 = f1 + 128;
+  for (int bb = 0; bb < nb; ++bb) {
+    const float* q = qhat + ((int64_t)(b0 + bb) * t_max + j) * D;
+    const float x = q[f1], y = q[f2];
+    __nv_bfloat16* o = qhl + ((int64_t)bb * t + j) * 2 * D;
+    __nv_bfloat16 hi, lo;
+    split_hilo(x * c - y * s, hi, lo);
+    o[f1] = hi;
+    o[D + f1] = lo;
+    split_hilo(x * s + y * c, hi, lo);
+    o[f2] = hi;
+    o[D + f2] = lo;
+  }
+}
+
+__device__ __forceinline__ void ml_combine(float& m, float& l, float m2, float l2) {
+  if (m2 == -INFINITY) return;
+  if (m == -INFINITY) {
+    m = m2;
+    l = l2;
+    return;
+  }
+  const float M = fmaxf(m, m2);
+  l = l * exp2f((m - M) * kLog2e) + l2 * exp2f((m2 - M) * kLog2e);
+  m = M;
+}
+
+template <typename OutT>
+__global__ void __launch_bounds__(256) softmax_kernel(const float* __restrict__ S, int64_t ncols,
+                                                      int64_t ldS, OutT* __restrict__ P,
+                                                      int64_t ldP) {
+  __shared__ float red_m[8], red_l[8];
+  const int64_t row = blockIdx.x;
+  const float* s = S + row * ldS;
+  float m = -INFINITY, l = 0.f;
+  for (int64_t c = threadIdx.x; c < ncols; c += blockDim.x) {
+    const float x = s[c];
+    if (x > m) {
+      l = (m == -INFINITY ? 0.f : l * exp2f((m - x) * kLog2e)) + 1.f;
+      m = x;
+    } else {
+      l += exp2f((x - m) * kLog2e);
+    }
+  }
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+    const float l2 = __shfl_xor_sync(0xffffffffu, l, o);
+    ml_combine(m, l, m2, l2);
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) {
+    red_m[warp] = m;
+    red_l[warp] = l;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    m = lane < 8 ? red_m[lane] : -INFINITY;
+    l = lane < 8 ? red_l[lane] : 0.f;
+    for (int o = 4; o > 0; o >>= 1) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+      const float l2 = __shfl_xor_sync(0xffffffffu, l, o);
+      ml_combine(m, l, m2, l2);
+    }
+    if (lane == 0) {
+      red_m[0] = m;
+      red_l[0] = l;
+    }
+  }
+  __syncthreads();
+  const float M = red_m[0], inv = 1.f / red_l[0];
+  OutT* p = P + row * ldP;
+  for (int64_t c = threadIdx.x; c < ldP; c += blockDim.x) {
+    const float v = c < ncols ? exp2f((s[c] - M) * kLog2e) * inv : 0.f;
+    if constexpr (sizeof(OutT) == 2 && std::is_same<OutT, __half>::value)
+      p[c] = __float2half_rn(v);
+    else
+      p[c] = __float2bfloat16_rn(v);
+  }
+}
+
+// Row softmax with the row held in registers: 256 threads, PER columns each (float4 groups).
+template <typename OutT, int PER>
+__global__ void __launch_bounds__(256) softmax_reg_kernel(const float* __restrict__ S,
+                                                          int64_t ncols, int64_t ldS,
+                                                          OutT* __restrict__ P, int64_t ldP) {
+  __shared__ float red[8];
+  const int64_t row = blockIdx.x;
+  const float* s = S + row * ldS;
+  constexpr int G = PER / 4;
+  float v[PER];
+  float m = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < G; ++i) {
+    const int64_t c = (int64_t)(i * 256 + threadIdx.x) * 4;
+    float4 x = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+    if (c + 3 < ncols) {
+      x = *reinterpret_cast<const float4*>(s + c);
+    } else if (c < ncols) {
+      x.x = s[c];
+      if (c + 1 < ncols) x.y = s[c + 1];
+      if (c + 2 < ncols) x.z = s[c + 2];
+    }
+    v[4 * i] = x.x;
+    v[4 * i + 1] = x.y;
+    v[4 * i + 2] = x.z;
+    v[4 * i + 3] = x.w;
+    m = fmaxf(m, fmaxf(fmaxf(x.x, x.y), fmaxf(x.z, x.w)));
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  if (lane == 0) red[warp] = m;
+  __syncthreads();
+  m = red[0];
+#pragma unroll
+  for (int w = 1; w < 8; ++w) m = fmaxf(m, red[w]);
+  __syncthreads();
+  float l = 0.f;
+#pragma unroll
+  for (int k = 0; k < PER; ++k) {
+    v[k] = exp2f((v[k] - m) * kLog2e);  // exp(-inf) = 0 for padding
+    l += v[k];
+  }
+  for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+  if (lane == 0) red[warp] = l;
+  __syncthreads();
+  l = 0.f;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) l += red[w];
+  const float inv = 1.f / l;
+  OutT* prow = P + row * ldP;
+#pragma unroll
+  for (int i = 0; i < G; ++i) {
+    const int64_t c = (int64_t)(i * 256 + threadIdx.x) * 4;
+    if (c < ldP) {
+      OutT o4[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const float y = v[4 * i + k] * inv;
+        if constexpr (std::is_same<OutT, __half>::value)
+          o4[k] = __float2half_rn(y);
+        else
+          o4[k] = __float2bfloat16_rn(y);
+      }
+      *reinterpret_cast<uint2*>(prow + c) = *reinterpret_cast<const uint2*>(o4);
+    }
+  }
+}
+
+__global__ void omega_kernel(double* out, int half, int width, double base) {
+  const int m = blockIdx.x * blockDim.x + threadIdx.x;
+  if (m < half) out[m] = pow(base, -2.0 * m / width);
+}
+
+__global__ void px_to_hilo_kernel(const float* __restrict__ O, int b0, int nb, int n, int t,
+                                  int d2, __nv_bfloat16* __restrict__ PX) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t total = (int64_t)nb * t * d2;
+  if (idx >= total) return;
+  const int f = (int)(idx % d2);
+  const int64_t rj = idx / d2;
+  const int j = (int)(rj % t), bb = (int)(rj / t);
+  const int b = b0 + bb, h = b / n, i = b % n;
+  const int64_t ld = 2 * (int64_t)n * d2;
+  __nv_bfloat16 hi, lo;
+  split_hilo(O[idx], hi, lo);
+  __nv_bfloat16* row = PX + ((int64_t)h * t + j) * ld;
+  row[i * d2 + f] = hi;
+  row[(int64_t)n * d2 + i * d2 + f] = lo;
+}
+
+__global__ void __launch_bounds__(256) rmsnorm_kernel(const void* __restrict__ in, int in_bf16,
+                                                      int64_t rows, int D, int64_t ldi, float eps,
+                                                      __nv_bfloat16* __restrict__ out,
+                                                      int64_t ldo, int hilo) {
+  const int64_t row = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  auto ld = [&](int c) -> float {
+    return in_bf16 ? __bfloat162float(static_cast<const __nv_bfloat16*>(in)[row * ldi + c])
+                   : static_cast<const float*>(in)[row * ldi + c];
+  };
+  float ss = 0.f;
+  for (int c = lane; c < D; c += 32) {
+    const float x = ld(c);
+    ss += x * x;
+  }
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  const float scale = 1.f / sqrtf(ss / (float)D + eps);
+  __nv_bfloat16* o = out + row * ldo;
+  for (int c = lane; c < D; c += 32) {
+    const float y = ld(c) * scale;
+    if (hilo) {
+      __nv_bfloat16 hi, lo;
+      split_hilo(y, hi, lo);
+      o[c] = hi;
+      o[D + c] = lo;
+    } else {
+      o[c] = __float2bfloat16_rn(y);
+    }
+  }
+}
+
+__global__ void l2_scale_kernel(float* x, const float* ss, int64_t rows, int D, float eps) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= rows * D) return;
+  x[idx] *= 1.f / fmaxf(sqrtf(ss[idx / D]), eps);
+}
+
+__global__ void transpose_kernel(const __nv_bfloat16* __restrict__ in, int64_t R, int64_t C,
+                                 __nv_bfloat16* __restrict__ out, int perm_D) {
+  __shared__ __nv_bfloat16 tile[32][33];
+  const int64_t c0 = (int64_t)blockIdx.x * 32, r0 = (int64_t)blockIdx.y * 32;
+  for (int k = threadIdx.y; k < 32; k += blockDim.y) {
+    const int64_t r = r0 + k, c = c0 + threadIdx.x;
+    if (r < R && c < C) {
+      const int64_t src = perm_D > 0 ? pair_chunk_src((int)c, perm_D) : c;
+      tile[k][threadIdx.x] = in[r * C + src];
+    }
+  }
+  __syncthreads();
+  for (int k = threadIdx.y; k < 32; k += blockDim.y) {
+    const int64_t c = c0 + k, r = r0 + threadIdx.x;
+    if (r < R && c < C) out[c * R + r] = tile[threadIdx.x][k];
+  }
+}
+
+__global__ void bias_kernel(const __nv_bfloat16* in, const __nv_bfloat16* in2, int64_t C,
+                            float* out, int perm_D) {
+  const int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= C) return;
+  const int64_t src = perm_D > 0 ? pair_chunk_src((int)c, perm_D) : c;
+  out[c] = __bfloat162float(in[src]);
+  if (in2 != nullptr) out[C + c] = __bfloat162float(in2[src]);
+}
+
+inline unsigned blocks_for(int64_t n, int per) { return (unsigned)((n + per - 1) / per); }
+
+}  // namespace
+
+cudaError_t launch_strip(const __nv_bfloat16* K, const __nv_bfloat16* V, int64_t sN, int64_t sH,
+                         int64_t N, int H, int d, const PosSegs& segs, double theta, int rope_fix,
+                         __nv_bfloat16* X, __half* XT, int64_t Np, cudaStream_t s) {
+  const size_t smem = (size_t)(d / 2) * sizeof(double) + 2 * (size_t)(2 * d) * (kStripTok + 2) * 2;
+  static bool attr = false;
+  if (!attr) {
+    cudaFuncSetAttribute(strip_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024);
+    attr = true;
+  }
+  dim3 grid((unsigned)(Np / kStripTok), (unsigned)H);
+  strip_kernel<<<grid, 256, smem, s>>>(K, V, sN, sH, N, H, d, segs, theta, rope_fix, X, XT, Np);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rope_tables(float2* coarse, float* omega, int G, int D, double pmin,
+                               double theta_c, cudaStream_t s) {
+  const int64_t n = (int64_t)G * (D / 2);
+  rope_tables_kernel<<<blocks_for(n, 256), 256, 0, s>>>(coarse, omega, G, D, pmin, theta_c);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_q_rope(const float* qhat, int t_max, int b0, int nb, int t, int D,
+                          double qstart, double qstep, const double* omega_c, int use_rope,
+                          __nv_bfloat16* qhl, cudaStream_t s) {
+  const int64_t n = (int64_t)t * (D / 2);
+  q_rope_kernel<<<blocks_for(n, 256), 256, 0, s>>>(qhat, t_max, b0, nb, t, D, qstart, qstep,
+                                                    omega_c, use_rope, qhl);
+  return cudaGetLastError();
+}
+
+template <typename OutT>
+static bool softmax_reg(const float* S, int64_t rows, int64_t ncols, int64_t ldS, void* P,
+                        int64_t ldP, cudaStream_t s) {
+  const int64_t need = std::max(ldP, ncols);
+  OutT* Pt = static_cast<OutT*>(P);
+  if ((ldS % 4) != 0 || (ldP % 4) != 0) return false;
+  if (need <= 1024)
+    softmax_reg_kernel<OutT, 4><<<(unsigned)rows, 256, 0, s>>>(S, ncols, ldS, Pt, ldP);
+  else if (need <= 2048)
+    softmax_reg_kernel<OutT, 8><<<(unsigned)rows, 256, 0, s>>>(S, ncols, ldS, Pt, ldP);
+  else if (need <= 4096)
+    softmax_reg_kernel<OutT, 16><<<(unsigned)rows, 256, 0, s>>>(S, ncols, ldS, Pt, ldP);
+  else if (need <= 8192)
+    softmax_reg_kernel<OutT, 32><<<(unsigned)rows, 256, 0, s>>>(S, ncols, ldS, Pt, ldP);
+  else if (need <= 16384)
+    softmax_reg_kernel<OutT, 64><<<(unsigned)rows, 256, 0, s>>>(S, ncols, ldS, Pt, ldP);
+  else
+    return false;
+  return true;
+}
+
+cudaError_t launch_omega(double* out, int half, int width, double base, cudaStream_t s) {
+  omega_kernel<<<blocks_for(half, 256), 256, 0, s>>>(out, half, width, base);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_softmax(const float* S, int64_t rows, int64_t ncols, int64_t ldS, void* P,
+                           int64_t ldP, int out_fp16, cudaStream_t s) {
+  if (rows == 0) return cudaSuccess;
+  if (out_fp16 ? softmax_reg<__half>(S, rows, ncols, ldS, P, ldP, s)
+               : softmax_reg<__nv_bfloat16>(S, rows, ncols, ldS, P, ldP, s))
+    return cudaGetLastError();
+  if (out_fp16)
+    softmax_kernel<__half><<<(unsigned)rows, 256, 0, s>>>(S, ncols, ldS,
+                                                          static_cast<__half*>(P), ldP);
+  else
+    softmax_kernel<__nv_bfloat16><<<(unsigned)rows, 256, 0, s>>>(
+        S, ncols, ldS, static_cast<__nv_bfloat16*>(P), ldP);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_px_to_hilo(const float* O, int b0, int nb, int n, int t, int d2,
+                              __nv_bfloat16* PX, cudaStream_t s) {
+  const int64_t total = (int64_t)nb * t * d2;
+  px_to_hilo_kernel<<<blocks_for(total, 256), 256, 0, s>>>(O, b0, nb, n, t, d2, PX);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rmsnorm(const void* in, int in_bf16, int64_t rows, int D, int64_t ldi,
+                           float eps, __nv_bfloat16* out, int64_t ldo, int hilo, cudaStream_t s) {
+  rmsnorm_kernel<<<blocks_for(rows, 8), 256, 0, s>>>(in, in_bf16, rows, D, ldi, eps, out, ldo,
+                                                     hilo);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_l2_scale(float* x, const float* ss, int64_t rows, int D, float eps,
+                            cudaStream_t s) {
+  l2_scale_kernel<<<blocks_for(rows * D, 256), 256, 0, s>>>(x, ss, rows, D, eps);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_transpose(const __nv_bfloat16* in, int64_t R, int64_t C, __nv_bfloat16* out,
+                             int perm_D, cudaStream_t s) {
+  dim3 grid(blocks_for(C, 32), blocks_for(R, 32));
+  transpose_kernel<<<grid, dim3(32, 8), 0, s>>>(in, R, C, out, perm_D);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_bias(const __nv_bfloat16* in, const __nv_bfloat16* in2, int64_t C,
+                        float* out, int perm_D, cudaStream_t s) {
+  bias_kernel<<<blocks_for(C, 256), 256, 0, s>>>(in, in2, C, out, perm_D);
+  return cudaGetLastError();
+}
+
+}  // namespace still

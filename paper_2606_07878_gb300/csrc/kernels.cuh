@@ -1,0 +1,71 @@
+// Memory-bound kernels of the compactor path (launchers implemented in kernels.cu).
+#pragma once
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+
+#include "epilogues.cuh"
+
+namespace still {
+
+// RoPE-fix and input concatenation (Sec. 2.2, App. A "Input concatenation"):
+//   X[h, n]  = [unRoPE(K[n, h]) | V[n, h]]  as bf16 hi (2d) + bf16 lo of the key half (d)
+//   XT[h]    = X[h]^T as fp16 hi / lo, token-contiguous, tokens padded with zeros to Np.
+// X:  [H*N][3d] bf16.  XT: [H*2d][2*Np] fp16 (hi at [0, Np), lo at [Np, 2Np)).
+cudaError_t launch_strip(const __nv_bfloat16* K, const __nv_bfloat16* V, int64_t sN, int64_t sH,
+                         int64_t N, int H, int d, const PosSegs& segs, double theta, int rope_fix,
+                         __nv_bfloat16* X, __half* XT, int64_t Np, cudaStream_t s);
+
+// Compactor-RoPE tables: coarse[g][m] = (cos, sin)((pmin + g * kPosGrain) * w_m), omega[m] = w_m
+// (fp32), w_m = theta_c^(-2m/D), angles reduced in fp64.
+cudaError_t launch_rope_tables(float2* coarse, float* omega, int G, int D, double pmin,
+                               double theta_c, cudaStream_t s);
+
+// Per-call cross-attention queries: q = RoPE_c(q^, p_j) for latents j < t, batches
+// b in [b0, b0 + nb) (b = h * n + i), as hi/lo bf16 [nb * t][2D]. q^ is [H*n][t_max][D] fp32
+// in pair-chunk column order; p_j = qstart + j * qstep.
+cudaError_t launch_q_rope(const float* qhat, int t_max, int b0, int nb, int t, int D,
+                          double qstart, double qstep, const double* omega_c, int use_rope,
+                          __nv_bfloat16* qhl, cudaStream_t s);
+
+// out[m] = base^(-2m / width) in fp64, m < half.
+cudaError_t launch_omega(double* out, int half, int width, double base, cudaStream_t s);
+
+// Row softmax: S fp32 [rows][ldS] (first ncols valid) -> P [rows][ldP], zero beyond ncols.
+// out_fp16: P is fp16, else bf16.
+cudaError_t launch_softmax(const float* S, int64_t rows, int64_t ncols, int64_t ldS, void* P,
+                           int64_t ldP, int out_fp16, cudaStream_t s);
+
+// Cross-attention head outputs O [nb][t][2d] fp32 (batch b = b0 + local) -> hi/lo bf16 rows
+// of PXcat [H*t][2 * n * 2d]: row h*t + j, columns i*2d + f (hi) and n*2d + i*2d + f (lo).
+cudaError_t launch_px_to_hilo(const float* O, int b0, int nb, int n, int t, int d2,
+                              __nv_bfloat16* PX, cudaStream_t s);
+
+// Non-parametric RMSNorm over rows of width D: out = x / sqrt(mean(x^2) + eps) as bf16 hi
+// (and lo at +D when hilo), row pitch ldo. Input fp32 or bf16 (in_bf16), row pitch ldi.
+cudaError_t launch_rmsnorm(const void* in, int in_bf16, int64_t rows, int D, int64_t ldi,
+                           float eps, __nv_bfloat16* out, int64_t ldo, int hilo, cudaStream_t s);
+
+// x[row] *= 1 / max(sqrt(ss[row]), eps) for rows of width D (fp32, in place).
+cudaError_t launch_l2_scale(float* x, const float* ss, int64_t rows, int D, float eps,
+                            cudaStream_t s);
+
+// out[c][r] = in[r][src(c)] (bf16), in is [R][C] row-major; src(c) maps pair-chunk order
+// back to natural order inside blocks of D columns when perm_D > 0.
+cudaError_t launch_transpose(const __nv_bfloat16* in, int64_t R, int64_t C, __nv_bfloat16* out,
+                             int perm_D, cudaStream_t s);
+
+// out[c] = float(in[src(c)]) (bf16 -> fp32 with the same optional permutation); in2 (optional)
+// is appended after in ([in | in2]), each of length C.
+cudaError_t launch_bias(const __nv_bfloat16* in, const __nv_bfloat16* in2, int64_t C,
+                        float* out, int perm_D, cudaStream_t s);
+
+// Natural column index of pair-chunk column c inside a block of D columns.
+__host__ __device__ inline int pair_chunk_src(int c, int D) {
+  const int blk = c / D, f = c % D;
+  const int chunk = f / 256, u = f % 256;
+  const int m = chunk * 128 + (u & 127);
+  return blk * D + (u < 128 ? m : D / 2 + m);
+}
+
+}  // namespace still

@@ -1,0 +1,1105 @@
+// Host runtime behind the C ABI (include/still.h): validation, weight re-layout and
+// precompute, workspace planning, and the per-layer launch sequence.
+//
+// Per-layer sequence for one sequence of N tokens and t latents (Sec. 2.1, App. A):
+//   strip      K, V -> X = [unRoPE(K) | V]  (hi/lo bf16 and hi/lo fp16 transposed)
+//   tables     compactor-RoPE coarse angle table for the key positions
+//   per group of (KV-head h, cross head i):
+//     keyproj  k~ = X W_K,i + b_K,i -> RoPE_c -> hi/lo, |k~|^2          (2-pass GEMM)
+//     qrope    q = RoPE_c(q^_i, p_j) -> hi/lo                         (q^ precomputed at load)
+//     scores   S = d_l * q.k / |k~|                                   (3-pass GEMM)
+//     softmax  P = softmax_rows(S) (fp16)
+//     PX       O_i = P X                                             (2-pass GEMM, split-K)
+//   VO         Z' = Z + [O_1..O_n] (W_V,i W_O,i)_i                     (3-pass GEMM)
+//   SA         Z'' = Z' + Concat_i softmax(d_l q^ k^T) v . S_O          (per KV-head bank)
+//   FFN        Z''' = Z'' + GELU(RMSNorm(Z'') W_1) W_2
+//   heads      C_k = RoPE(Z''' W_key, p_out), C_v = Z''' W_val      (2-pass, Z''' hi/lo)
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <vector>
+
+#include "../../include/still.h"
+#include "gemm_host.cuh"
+#include "kernels.cuh"
+
+using namespace still;
+
+namespace {
+
+using bf16 = __nv_bfloat16;
+
+struct LayerW {
+  bool loaded = false;
+  still_layer_config cfg{};
+  bf16* Z = nullptr;     // [H][t_max][D]
+  bf16* WkT = nullptr;   // [nD][2d]  pair-chunk order
+  float* bk = nullptr;   // [nD]      pair-chunk order
+  float* qhat = nullptr; // [H][n][t_max][D] fp32, L2-normalised, pair-chunk order
+  bf16* WvoT = nullptr;  // [D][2 * n * 2d]: (W_V,i W_O,i)^T hi | lo
+  bf16* SqkT = nullptr;  // [2nD][D]
+  float* sbqk = nullptr; // [2nD]
+  bf16* SvT = nullptr;   // [nD][D]
+  bf16* SoT = nullptr;   // [D][nD]
+  bf16* W1T = nullptr;   // [F][D]
+  bf16* W2T = nullptr;   // [D][F]
+  bf16* WhT = nullptr;   // [2d][D]
+  double* omega_b = nullptr;  // [d/2] base-model RoPE frequencies (fp64)
+  double* omega_c = nullptr;  // [D/2] compactor RoPE frequencies (fp64)
+  std::vector<void*> owned;
+};
+
+}  // namespace
+
+// Per-kernel-class launch counts and (when enabled) CUDA-event timings.
+struct Profiler {
+  bool on = false;
+  int64_t launches[STILL_K_COUNT] = {0};
+  double ms[STILL_K_COUNT] = {0};
+  struct Rec {
+    int cls;
+    cudaEvent_t a, b;
+  };
+  std::vector<Rec> recs;
+  std::vector<cudaEvent_t> pool;
+  cudaEvent_t pending = nullptr;
+
+  cudaEvent_t get() {
+    if (!pool.empty()) {
+      cudaEvent_t e = pool.back();
+      pool.pop_back();
+      return e;
+    }
+    cudaEvent_t e = nullptr;
+    cudaEventCreate(&e);
+    return e;
+  }
+  void begin(int cls, cudaStream_t s) {
+    ++launches[cls];
+    if (!on) return;
+    pending = get();
+    cudaEventRecord(pending, s);
+  }
+  void end(int cls, cudaStream_t s) {
+    if (!on || pending == nullptr) return;
+    cudaEvent_t b = get();
+    cudaEventRecord(b, s);
+    recs.push_back(Rec{cls, pending, b});
+    pending = nullptr;
+  }
+  bool resolve() {
+    if (recs.empty()) return true;
+    if (cudaDeviceSynchronize() != cudaSuccess) return false;
+    for (auto& r : recs) {
+      float t = 0.f;
+      cudaEventElapsedTime(&t, r.a, r.b);
+      ms[r.cls] += t;
+      pool.push_back(r.a);
+      pool.push_back(r.b);
+    }
+    recs.clear();
+    return true;
+  }
+  void reset() {
+    resolve();
+    for (int i = 0; i < STILL_K_COUNT; ++i) {
+      launches[i] = 0;
+      ms[i] = 0;
+    }
+  }
+  ~Profiler() {
+    for (auto& r : recs) {
+      cudaEventDestroy(r.a);
+      cudaEventDestroy(r.b);
+    }
+    for (auto e : pool) cudaEventDestroy(e);
+  }
+};
+
+struct still_ctx {
+  int device = 0;
+  int nsm = 0;
+  int* err = nullptr;  // device error record [4]
+  std::vector<LayerW> layers;
+  void* ws = nullptr;
+  size_t ws_bytes = 0;
+  size_t ws_limit = size_t(48) << 30;
+  Profiler prof;
+};
+
+namespace {
+
+#define CK(x)                                            \
+  do {                                                   \
+    cudaError_t e_ = (x);                                \
+    if (e_ != cudaSuccess) return STILL_ERR_CUDA;        \
+  } while (0)
+
+inline int64_t rup(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
+
+void free_layer(LayerW& L) {
+  for (void* p : L.owned) cudaFree(p);
+  L = LayerW();
+}
+
+template <typename T>
+still_status dalloc(LayerW& L, T** p, size_t count) {
+  void* q = nullptr;
+  if (cudaMalloc(&q, std::max<size_t>(count, 1) * sizeof(T)) != cudaSuccess) return STILL_ERR_OOM;
+  L.owned.push_back(q);
+  *p = static_cast<T*>(q);
+  return STILL_OK;
+}
+
+still_status check_cfg(const still_layer_config* c) {
+  if (c == nullptr) return STILL_ERR_INVALID_ARG;
+  if (c->n_kv_heads < 1 || c->head_dim < 1 || c->d_latent < 1 || c->n_cross_heads < 1 ||
+      c->n_self_heads < 1 || c->t_max < 1 || c->ffn_dim < 0 || c->n_blocks < 1)
+    return STILL_ERR_SHAPE;
+  if (!(std::isfinite(c->rope_theta) && c->rope_theta > 0) ||
+      !(std::isfinite(c->rope_theta_compactor) && c->rope_theta_compactor > 0) ||
+      !std::isfinite(c->logit_scale) || !(c->rms_eps >= 0) || !(c->l2_eps > 0))
+    return STILL_ERR_INVALID_ARG;
+  if (c->n_blocks != 1 || c->cross_every_block != 1 || c->n_cross_heads != c->n_self_heads ||
+      c->d_latent % 256 != 0 || !(c->head_dim == 64 || c->head_dim == 128 || c->head_dim == 256) ||
+      c->ffn_dim % 64 != 0 || c->compactor_rope != 1 || c->rope_fix != 1 ||
+      (c->final_norm != 0 && c->final_norm != 1))
+    return STILL_ERR_UNSUPPORTED;
+  return STILL_OK;
+}
+
+// ------------------------------------------------------------------------------ GEMM helper
+
+GemmParams gp(int M, int N, int batch = 1, int bdiv = 1) {
+  GemmParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.M = M;
+  p.N = N;
+  p.batch = batch;
+  p.bdiv = bdiv;
+  p.ksplit = 1;
+  return p;
+}
+
+void add_pass(GemmParams& p, int a_koff, int b_koff, int a_roff, int b_roff, int klen) {
+  p.pass[p.npass++] = GemmPass{a_koff, b_koff, a_roff, b_roff, klen};
+}
+
+Operand2D op(const void* ptr, int64_t rows, int64_t cols, int64_t pitch = -1) {
+  return Operand2D{ptr, rows, cols, pitch < 0 ? cols : pitch};
+}
+
+template <class Epi>
+still_status run_gemm(still_ctx* ctx, int cls, int bn, const Operand2D& A, const Operand2D& B,
+                      GemmParams p, const Epi& e, int ab_fmt, cudaStream_t s) {
+  p.err = ctx->err;
+  ctx->prof.begin(cls, s);
+  cudaError_t r = bn == 128 ? launch_gemm<128>(A, B, p, e, ab_fmt, ctx->nsm, s)
+                            : launch_gemm<256>(A, B, p, e, ab_fmt, ctx->nsm, s);
+  ctx->prof.end(cls, s);
+  if (r == cudaErrorInvalidValue) return STILL_ERR_INVALID_ARG;
+  return r == cudaSuccess ? STILL_OK : STILL_ERR_CUDA;
+}
+
+// Launch of one of the memory-bound kernels, timed under its class.
+#define KLAUNCH(cls, call)                  \
+  do {                                      \
+    ctx->prof.begin((cls), s);              \
+    cudaError_t e_ = (call);                \
+    ctx->prof.end((cls), s);                \
+    if (e_ != cudaSuccess) return STILL_ERR_CUDA; \
+  } while (0)
+
+// Split-K factor that brings a GEMM with few output tiles up to about two waves.
+int auto_split(int64_t tiles, int iters, int nsm) {
+  if (tiles >= nsm) return 1;
+  int s = (int)((2 * nsm + tiles - 1) / tiles);
+  return std::max(1, std::min(s, iters / 4));
+}
+
+#define TRY(x)                          \
+  do {                                  \
+    still_status st_ = (x);             \
+    if (st_ != STILL_OK) return st_;    \
+  } while (0)
+
+// ------------------------------------------------------------------------------ workspace plan
+
+struct Plan {
+  int H, d, D, n, F, t;
+  int64_t N, Np, ldS, tp, ldt;
+  int G;
+  int ca_units;   // (h, i) pairs per cross-attention group
+  int sa_heads;   // KV-heads per self-attention group
+  // byte offsets
+  size_t oX, oXT, oCoarse, oOmega, oPX, oZ1, oA1, oCat, oZ2, oA2, oG, oZ3;
+  size_t oCA, oSA;
+  size_t ca_unit_bytes, sa_unit_bytes;
+  size_t kb_b, kss_b, q_b, S_b, P_b, O_b;        // per CA unit
+  size_t qk_b, sss_b, vT_b, Ssa_b, Psa_b;        // per SA head
+  size_t total;
+};
+
+size_t a256(size_t x) { return (x + 255) & ~size_t(255); }
+
+bool make_plan(const still_layer_config& c, int64_t N, int t, double pmin, double pmax,
+               size_t limit, Plan& P) {
+  P.H = c.n_kv_heads;
+  P.d = c.head_dim;
+  P.D = c.d_latent;
+  P.n = c.n_cross_heads;
+  P.F = c.ffn_dim;
+  P.t = t;
+  P.N = N;
+  P.Np = rup(N, 64);
+  P.ldS = rup(N, 4);
+  P.tp = rup(t, 64);
+  P.ldt = rup(t, 4);
+  P.G = (int)std::floor((pmax - pmin) / kPosGrain) + 2;
+  const int64_t H = P.H, d = P.d, D = P.D, n = P.n, F = P.F, T = t;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    size_t o = off;
+    off += a256(bytes);
+    return o;
+  };
+  P.oX = take(H * N * 3 * d * 2);
+  P.oXT = take(H * 2 * d * 2 * P.Np * 2);
+  P.oCoarse = take((size_t)P.G * (D / 2) * 8);
+  P.oOmega = take((D / 2) * 4);
+  P.oPX = take(H * T * 2 * n * 2 * d * 2);
+  P.oZ1 = take(H * T * D * 4);
+  P.oA1 = take(H * T * 2 * D * 2);
+  P.oCat = take(H * T * n * D * 2);
+  P.oZ2 = take(H * T * D * 4);
+  P.oA2 = take(H * T * D * 2);
+  P.oG = take(H * T * std::max<int64_t>(F, 1) * 2);
+  P.oZ3 = take(H * T * D * 4);
+  const size_t fixed = off;
+  P.kb_b = a256(N * 2 * D * 2);
+  P.kss_b = a256(N * 4);
+  P.q_b = a256(T * 2 * D * 2);
+  P.S_b = a256(T * P.ldS * 4);
+  P.P_b = a256(T * P.Np * 2);
+  P.O_b = a256(T * 2 * d * 4);
+  P.ca_unit_bytes = P.kb_b + P.kss_b + P.q_b + P.S_b + P.P_b + P.O_b;
+  P.qk_b = a256(2 * n * T * 2 * D * 2);
+  P.sss_b = a256(2 * n * T * 4);
+  P.vT_b = a256(n * D * P.tp * 2);
+  P.Ssa_b = a256(n * T * P.ldt * 4);
+  P.Psa_b = a256(n * T * P.tp * 2);
+  P.sa_unit_bytes = P.qk_b + P.sss_b + P.vT_b + P.Ssa_b + P.Psa_b;
+  if (fixed >= limit) return false;
+  const size_t avail = limit - fixed;
+  // Cross-attention groups: whole KV-heads when possible, else a part of one head.
+  const int64_t units_total = H * n;
+  int64_t u = std::min<int64_t>(units_total, (int64_t)(avail / P.ca_unit_bytes));
+  if (u < 1) return false;
+  if (u >= n)
+    u = (u / n) * n;
+  P.ca_units = (int)u;
+  int64_t sh = std::min<int64_t>(H, (int64_t)(avail / P.sa_unit_bytes));
+  if (sh < 1) return false;
+  P.sa_heads = (int)sh;
+  P.oCA = off;
+  P.oSA = off;  // the two phases reuse the same region
+  P.total = off + std::max(P.ca_unit_bytes * P.ca_units, P.sa_unit_bytes * P.sa_heads);
+  return true;
+}
+
+still_status ensure_ws(still_ctx* ctx, size_t bytes) {
+  if (bytes <= ctx->ws_bytes) return STILL_OK;
+  if (ctx->ws != nullptr) {
+    CK(cudaDeviceSynchronize());
+    cudaFree(ctx->ws);
+    ctx->ws = nullptr;
+    ctx->ws_bytes = 0;
+  }
+  if (cudaMalloc(&ctx->ws, bytes) != cudaSuccess) {
+    cudaGetLastError();
+    return STILL_ERR_OOM;
+  }
+  ctx->ws_bytes = bytes;
+  return STILL_OK;
+}
+
+// ------------------------------------------------------------------------------ positions
+
+struct Positions {
+  PosSegs segs;
+  double pmin = 0, pmax = 0;
+};
+
+still_status make_positions(const still_pos_segment* h_segments, int32_t n_segments, int64_t N,
+                            Positions& out) {
+  out = Positions();
+  if (n_segments == 0 || h_segments == nullptr) {
+    if (n_segments != 0) return STILL_ERR_INVALID_ARG;
+    out.segs.n = 1;
+    out.segs.begin[0] = 0;
+    out.segs.begin[1] = N;
+    out.segs.start[0] = 0;
+    out.segs.step[0] = 1;
+    out.pmin = 0;
+    out.pmax = (double)(N - 1);
+    return STILL_OK;
+  }
+  if (n_segments < 0 || n_segments > 8) return STILL_ERR_UNSUPPORTED;
+  int64_t acc = 0;
+  double lo = INFINITY, hi = -INFINITY;
+  int k = 0;
+  for (int i = 0; i < n_segments; ++i) {
+    const still_pos_segment& s = h_segments[i];
+    if (s.count < 0 || !std::isfinite(s.start) || !std::isfinite(s.step))
+      return STILL_ERR_INVALID_ARG;
+    if (s.count == 0) continue;
+    const double last = s.start + (double)(s.count - 1) * s.step;
+    if (!std::isfinite(last)) return STILL_ERR_INVALID_ARG;
+    lo = std::min(lo, std::min(s.start, last));
+    hi = std::max(hi, std::max(s.start, last));
+    out.segs.begin[k] = acc;
+    out.segs.start[k] = s.start;
+    out.segs.step[k] = s.step;
+    ++k;
+    acc += s.count;
+  }
+  if (acc != N || k == 0) return STILL_ERR_SHAPE;
+  out.segs.n = k;
+  out.segs.begin[k] = acc;
+  out.pmin = lo;
+  out.pmax = hi;
+  return STILL_OK;
+}
+
+// ------------------------------------------------------------------------------ one sequence
+
+struct OutSpec {
+  bf16* ck;
+  bf16* cv;
+  int64_t st, sh;  // element strides of [t, H, d] outputs (d contiguous)
+};
+
+still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const bf16* V,
+                         int64_t sN, int64_t sH, const Positions& pos, int64_t N, int t,
+                         const OutSpec& out, cudaStream_t s) {
+  const still_layer_config& c = L.cfg;
+  Plan P;
+  if (!make_plan(c, N, t, pos.pmin, pos.pmax, ctx->ws_limit, P)) return STILL_ERR_OOM;
+  TRY(ensure_ws(ctx, P.total));
+  uint8_t* ws = static_cast<uint8_t*>(ctx->ws);
+  const int H = P.H, d = P.d, D = P.D, n = P.n, F = P.F;
+  const int64_t Np = P.Np;
+  const float scale = c.logit_scale > 0 ? (float)c.logit_scale : (float)D;
+  const double qstart = pos.pmin;
+  const double qstep = t > 1 ? (pos.pmax - pos.pmin) / (double)(t - 1) : 0.0;
+
+  bf16* X = reinterpret_cast<bf16*>(ws + P.oX);
+  __half* XT = reinterpret_cast<__half*>(ws + P.oXT);
+  float2* coarse = reinterpret_cast<float2*>(ws + P.oCoarse);
+  float* omega = reinterpret_cast<float*>(ws + P.oOmega);
+  bf16* PX = reinterpret_cast<bf16*>(ws + P.oPX);
+  float* Z1 = reinterpret_cast<float*>(ws + P.oZ1);
+  bf16* A1 = reinterpret_cast<bf16*>(ws + P.oA1);
+  bf16* cat = reinterpret_cast<bf16*>(ws + P.oCat);
+  float* Z2 = reinterpret_cast<float*>(ws + P.oZ2);
+  bf16* A2 = reinterpret_cast<bf16*>(ws + P.oA2);
+  bf16* Gb = reinterpret_cast<bf16*>(ws + P.oG);
+  void* Z3 = ws + P.oZ3;
+
+  KLAUNCH(STILL_K_STRIP, launch_strip(K, V, sN, sH, N, H, d, pos.segs, c.rope_theta, c.rope_fix, X, XT, Np, s));
+  KLAUNCH(STILL_K_TABLES, launch_rope_tables(coarse, omega, P.G, D, pos.pmin, c.rope_theta_compactor, s));
+
+  // ---------------------------------------------------------------- cross-attention groups
+  const int units_total = H * n;
+  for (int b0 = 0; b0 < units_total;) {
+    // A group is whole KV-heads [h0, h0 + nh) x all cross heads, or part of one KV-head.
+    const int h0 = b0 / n, i0 = b0 % n;
+    int nh, ni;
+    if (i0 == 0 && P.ca_units >= n) {
+      nh = std::min(P.ca_units / n, H - h0);
+      ni = n;
+    } else {
+      nh = 1;
+      ni = std::min(P.ca_units, n - i0);
+    }
+    const int nbl = nh * ni;
+    uint8_t* g = ws + P.oCA;
+    bf16* kb = reinterpret_cast<bf16*>(g);
+    g += P.kb_b * nbl;
+    float* kss = reinterpret_cast<float*>(g);
+    g += P.kss_b * nbl;
+    bf16* qhl = reinterpret_cast<bf16*>(g);
+    g += P.q_b * nbl;
+    float* S = reinterpret_cast<float*>(g);
+    g += P.S_b * nbl;
+    __half* Pm = reinterpret_cast<__half*>(g);
+    g += P.P_b * nbl;
+    float* O = reinterpret_cast<float*>(g);
+    // keyproj: rows = tokens of heads [h0, h0+nh), columns = cross heads [i0, i0+ni)
+    CK(cudaMemsetAsync(kss, 0, sizeof(float) * (size_t)nbl * N, s));
+    {
+      GemmParams p = gp((int)N, ni * D, nh, 1);
+      p.a_r1 = N;
+      add_pass(p, 0, 0, (int)(h0 * N), i0 * D, 2 * d);
+      add_pass(p, 2 * d, 0, (int)(h0 * N), i0 * D, d);
+      EpiRopeC e;
+      e.out = kb;
+      e.sumsq = kss;
+      e.bias = L.bk + (size_t)i0 * D;
+      e.coarse = coarse;
+      e.omega = omega;
+      e.segs = pos.segs;
+      e.pmin = pos.pmin;
+      e.D = D;
+      e.nheads = ni;
+      e.ncoarse = P.G;
+      e.Ntok = N;
+      TRY(run_gemm(ctx, STILL_K_KEYPROJ, 256, op(X, (int64_t)H * N, 3 * d), op(L.WkT, (int64_t)n * D, 2 * d), p, e,
+                   1, s));
+    }
+    KLAUNCH(STILL_K_QROPE, launch_q_rope(L.qhat, c.t_max, b0, nbl, t, D, qstart, qstep, L.omega_c,
+                     c.compactor_rope, qhl, s));
+    {  // S = scale * q.k / |k~|
+      GemmParams p = gp(t, (int)N, nbl, 1);
+      p.a_r1 = t;
+      p.b_r1 = N;
+      add_pass(p, 0, 0, 0, 0, D);
+      add_pass(p, 0, D, 0, 0, D);
+      add_pass(p, D, 0, 0, 0, D);
+      EpiAffine e;
+      e.kind = OUT_F32;
+      e.out = S;
+      e.om.b1 = (int64_t)t * P.ldS;
+      e.om.r0 = P.ldS;
+      e.om.c0 = 1;
+      e.alpha = scale;
+      e.col_ss = kss;
+      e.csm.b1 = N;
+      e.csm.c0 = 1;
+      e.eps = c.l2_eps;
+      e.vec_ok = 1;
+      TRY(run_gemm(ctx, STILL_K_SCORES, 256, op(qhl, (int64_t)nbl * t, 2 * D), op(kb, (int64_t)nbl * N, 2 * D), p,
+                   e, 1, s));
+    }
+    KLAUNCH(STILL_K_SOFTMAX, launch_softmax(S, (int64_t)nbl * t, N, P.ldS, Pm, Np, 1, s));
+    CK(cudaMemsetAsync(O, 0, sizeof(float) * (size_t)nbl * t * 2 * d, s));
+    {  // O = P X  (fp16 operands, X hi + X lo)
+      GemmParams p = gp(t, 2 * d, nbl, ni);
+      p.a_r1 = (int64_t)ni * t;
+      p.a_r0 = t;
+      p.b_r1 = 2 * d;
+      add_pass(p, 0, 0, 0, h0 * 2 * d, (int)Np);
+      add_pass(p, 0, (int)Np, 0, h0 * 2 * d, (int)Np);
+      const int bn = 2 * d <= 128 ? 128 : 256;
+      const int64_t tiles = (int64_t)((t + 127) / 128) * ((2 * d + bn - 1) / bn) * nbl;
+      p.ksplit = auto_split(tiles, (int)(2 * Np / 64), ctx->nsm);
+      EpiAffine e;
+      e.kind = OUT_F32_ATOMIC;
+      e.out = O;
+      e.om.bdiv = ni;
+      e.om.b1 = (int64_t)ni * t * 2 * d;
+      e.om.b0 = (int64_t)t * 2 * d;
+      e.om.r0 = 2 * d;
+      e.om.c0 = 1;
+      e.vec_ok = 1;
+      TRY(run_gemm(ctx, STILL_K_PX, bn, op(Pm, (int64_t)nbl * t, Np), op(XT, (int64_t)H * 2 * d, 2 * Np), p,
+                   e, 0, s));
+    }
+    KLAUNCH(STILL_K_PXSPLIT, launch_px_to_hilo(O, b0, nbl, n, t, 2 * d, PX, s));
+    b0 += nbl;
+  }
+
+  // ---------------------------------------------------------------- Z' = Z + PX W_VO
+  const int64_t rows = (int64_t)H * t;
+  const int n2d = n * 2 * d;
+  {
+    GemmParams p = gp((int)rows, D);
+    add_pass(p, 0, 0, 0, 0, n2d);
+    add_pass(p, 0, n2d, 0, 0, n2d);
+    add_pass(p, n2d, 0, 0, 0, n2d);
+    const int64_t tiles = ((rows + 127) / 128) * ((D + 255) / 256);
+    p.ksplit = auto_split(tiles, 3 * n2d / 64, ctx->nsm);
+    EpiAffine e;
+    e.kind = p.ksplit > 1 ? OUT_F32_ATOMIC : OUT_F32;
+    e.out = Z1;
+    e.om.r0 = D;
+    e.om.c0 = 1;
+    e.res_kind = 2;
+    e.res = L.Z;
+    e.resm.rdiv = t;
+    e.resm.r1 = (int64_t)c.t_max * D;
+    e.resm.r0 = D;
+    e.resm.c0 = 1;
+    e.vec_ok = 1;
+    if (p.ksplit > 1) CK(cudaMemsetAsync(Z1, 0, sizeof(float) * rows * D, s));
+    TRY(run_gemm(ctx, STILL_K_VO, 256, op(PX, rows, 2 * n2d), op(L.WvoT, D, 2 * n2d), p, e, 1, s));
+  }
+  KLAUNCH(STILL_K_NORM, launch_rmsnorm(Z1, 0, rows, D, D, c.rms_eps, A1, 2 * D, 1, s));
+
+  // ---------------------------------------------------------------- latent self-attention
+  for (int h0 = 0; h0 < H; h0 += P.sa_heads) {
+    const int nh = std::min(P.sa_heads, H - h0);
+    uint8_t* g = ws + P.oSA;
+    bf16* qk = reinterpret_cast<bf16*>(g);
+    g += P.qk_b * nh;
+    float* sss = reinterpret_cast<float*>(g);
+    g += P.sss_b * nh;
+    bf16* vT = reinterpret_cast<bf16*>(g);
+    g += P.vT_b * nh;
+    float* Ssa = reinterpret_cast<float*>(g);
+    g += P.Ssa_b * nh;
+    bf16* Psa = reinterpret_cast<bf16*>(g);
+    CK(cudaMemsetAsync(sss, 0, sizeof(float) * (size_t)nh * 2 * n * t, s));
+    // The P.v product reads v^T columns [t, tp) of each head against zero probabilities:
+    // they must hold finite values, and the region is shared with the cross-attention phase.
+    if (P.tp != t) CK(cudaMemsetAsync(vT, 0, P.vT_b * nh, s));
+    {  // [q~ | k~] = RMSNorm(Z') [S_Q | S_K] + [b | b]  (2-pass), |.|^2 per head
+      GemmParams p = gp(nh * t, 2 * n * D);
+      add_pass(p, 0, 0, h0 * t, 0, D);
+      add_pass(p, D, 0, h0 * t, 0, D);
+      EpiAffine e;
+      e.kind = OUT_HILO;
+      e.out = qk;
+      e.lo_off = D;
+      e.om.rdiv = t;
+      e.om.r1 = (int64_t)2 * n * t * 2 * D;
+      e.om.r0 = 2 * D;
+      e.om.cdiv = D;
+      e.om.c1 = (int64_t)t * 2 * D;
+      e.om.c0 = 1;
+      e.bias = L.sbqk;
+      e.sumsq = sss;
+      e.ssm.rdiv = t;
+      e.ssm.r1 = (int64_t)2 * n * t;
+      e.ssm.r0 = 1;
+      e.ssm.c0 = t;
+      e.ss_seg = D;
+      e.vec_ok = 1;
+      TRY(run_gemm(ctx, STILL_K_SA_PROJ, 256, op(A1, rows, 2 * D), op(L.SqkT, (int64_t)2 * n * D, D), p, e, 1, s));
+    }
+    {  // v^T = S_V^T RMSNorm(Z')^T  -> [nD][nh * tp]
+      GemmParams p = gp(n * D, nh * t);
+      add_pass(p, 0, 0, 0, h0 * t, D);
+      EpiAffine e;
+      e.kind = OUT_BF16;
+      e.out = vT;
+      e.om.r0 = (int64_t)nh * P.tp;
+      e.om.cdiv = t;
+      e.om.c1 = P.tp;
+      e.om.c0 = 1;
+      e.vec_ok = (t % 32 == 0);
+      TRY(run_gemm(ctx, STILL_K_SA_V, 256, op(L.SvT, (int64_t)n * D, D), op(A1, rows, 2 * D), p, e, 1, s));
+    }
+    {  // S = scale * q~.k~ / (|q~| |k~|)  per (head, self head)
+      GemmParams p = gp(t, t, nh * n, n);
+      p.a_r1 = (int64_t)2 * n * t;
+      p.a_r0 = t;
+      p.b_r1 = (int64_t)2 * n * t;
+      p.b_r0 = t;
+      add_pass(p, 0, 0, 0, n * t, D);
+      add_pass(p, 0, D, 0, n * t, D);
+      add_pass(p, D, 0, 0, n * t, D);
+      EpiAffine e;
+      e.kind = OUT_F32;
+      e.out = Ssa;
+      e.om.b1 = (int64_t)t * P.ldt;
+      e.om.r0 = P.ldt;
+      e.om.c0 = 1;
+      e.alpha = scale;
+      e.row_ss = sss;
+      e.rsm.bdiv = n;
+      e.rsm.b1 = (int64_t)2 * n * t;
+      e.rsm.b0 = t;
+      e.rsm.r0 = 1;
+      e.col_ss = sss;
+      e.csm.bdiv = n;
+      e.csm.b1 = (int64_t)2 * n * t;
+      e.csm.b0 = t;
+      e.csm.c0 = 1;
+      e.csm.k = (int64_t)n * t;
+      e.eps = c.l2_eps;
+      e.vec_ok = 1;
+      TRY(run_gemm(ctx, STILL_K_SA_SCORES, 256, op(qk, (int64_t)nh * 2 * n * t, 2 * D),
+                   op(qk, (int64_t)nh * 2 * n * t, 2 * D), p, e, 1, s));
+    }
+    KLAUNCH(STILL_K_SA_SOFTMAX, launch_softmax(Ssa, (int64_t)nh * n * t, t, P.ldt, Psa, P.tp, 0, s));
+    {  // heads = P v -> concat rows (h0 + hh) * t + j, columns i * D + f
+      GemmParams p = gp(t, D, nh * n, n);
+      p.a_r1 = (int64_t)n * t;
+      p.a_r0 = t;
+      p.b_r0 = D;
+      p.b_k1 = P.tp;
+      add_pass(p, 0, 0, 0, 0, (int)P.tp);
+      EpiAffine e;
+      e.kind = OUT_BF16;
+      e.out = cat;
+      e.om.bdiv = n;
+      e.om.b1 = (int64_t)t * n * D;
+      e.om.b0 = D;
+      e.om.r0 = (int64_t)n * D;
+      e.om.c0 = 1;
+      e.om.k = (int64_t)h0 * t * n * D;
+      e.vec_ok = 1;
+      TRY(run_gemm(ctx, STILL_K_SA_PV, 256, op(Psa, (int64_t)nh * n * t, P.tp),
+                   op(vT, (int64_t)n * D, (int64_t)nh * P.tp), p, e, 1, s));
+    }
+  }
+  const bool z3_bf16 = (c.final_norm == 0);
+  {  // Z'' = Z' + concat S_O
+    GemmParams p = gp((int)rows, D);
+    add_pass(p, 0, 0, 0, 0, n * D);
+    EpiAffine e;
+    const bool direct = (F == 0) && z3_bf16;
+    e.kind = direct ? OUT_HILO : OUT_F32;
+    e.out = direct ? Z3 : static_cast<void*>(Z2);
+    e.lo_off = D;
+    e.om.r0 = direct ? 2 * D : D;
+    e.om.c0 = 1;
+    e.res_kind = 1;
+    e.res = Z1;
+    e.resm.r0 = D;
+    e.resm.c0 = 1;
+    e.vec_ok = 1;
+    TRY(run_gemm(ctx, STILL_K_SO, 256, op(cat, rows, (int64_t)n * D), op(L.SoT, D, (int64_t)n * D), p, e, 1,
+                 s));
+  }
+  if (F > 0) {
+    KLAUNCH(STILL_K_NORM, launch_rmsnorm(Z2, 0, rows, D, D, c.rms_eps, A2, D, 0, s));
+    {
+      GemmParams p = gp((int)rows, F);
+      add_pass(p, 0, 0, 0, 0, D);
+      EpiAffine e;
+      e.kind = OUT_BF16;
+      e.out = Gb;
+      e.om.r0 = F;
+      e.om.c0 = 1;
+      e.gelu = 1;
+      e.vec_ok = 1;
+      TRY(run_gemm(ctx, STILL_K_FFN1, 256, op(A2, rows, D), op(L.W1T, F, D), p, e, 1, s));
+    }
+    {
+      GemmParams p = gp((int)rows, D);
+      add_pass(p, 0, 0, 0, 0, F);
+      EpiAffine e;
+      e.kind = z3_bf16 ? OUT_HILO : OUT_F32;
+      e.out = z3_bf16 ? Z3 : static_cast<void*>(Z2);
+      e.lo_off = D;
+      e.om.r0 = z3_bf16 ? 2 * D : D;
+      e.om.c0 = 1;
+      e.res_kind = 1;
+      e.res = Z2;
+      e.resm.r0 = D;
+      e.resm.c0 = 1;
+      e.vec_ok = 1;
+      // In place (Z2 -> Z2) is safe: each element is read and written by the same thread.
+      TRY(run_gemm(ctx, STILL_K_FFN2, 256, op(Gb, rows, F), op(L.W2T, D, F), p, e, 1, s));
+    }
+  }
+  if (!z3_bf16) {
+    KLAUNCH(STILL_K_NORM, launch_rmsnorm(Z2, 0, rows, D, D, c.rms_eps, reinterpret_cast<bf16*>(Z3), 2 * D, 1, s));
+  }
+  {  // output heads (2-pass on the hi/lo latent state) + re-rotation
+    GemmParams p = gp((int)rows, 2 * d);
+    add_pass(p, 0, 0, 0, 0, D);
+    add_pass(p, D, 0, 0, 0, D);
+    EpiHeads e;
+    e.ck = out.ck;
+    e.cv = out.cv;
+    e.st = out.st;
+    e.sh = out.sh;
+    e.sd = 1;
+    e.t = t;
+    e.d = d;
+    e.pstart = qstart;
+    e.pstep = qstep;
+    e.omega = L.omega_b;
+    e.rope = c.rope_fix;
+    const int bn = 2 * d <= 128 ? 128 : 256;
+    TRY(run_gemm(ctx, STILL_K_HEADS, bn, op(Z3, rows, 2 * D), op(L.WhT, 2 * d, D), p, e, 1, s));
+  }
+  return STILL_OK;
+}
+
+still_status check_ctx_layer(still_ctx* ctx, int32_t layer, const LayerW** L) {
+  if (ctx == nullptr) return STILL_ERR_INVALID_ARG;
+  if (layer < 0 || layer >= (int32_t)ctx->layers.size() || !ctx->layers[layer].loaded)
+    return STILL_ERR_NOT_LOADED;
+  *L = &ctx->layers[layer];
+  return STILL_OK;
+}
+
+}  // namespace
+
+// ============================================================================== C ABI
+
+extern "C" {
+
+const char* still_status_string(still_status s) {
+  switch (s) {
+    case STILL_OK: return "ok";
+    case STILL_ERR_INVALID_ARG: return "invalid argument";
+    case STILL_ERR_UNSUPPORTED: return "unsupported configuration";
+    case STILL_ERR_SHAPE: return "inconsistent shape";
+    case STILL_ERR_ALIGNMENT: return "misaligned pointer or stride";
+    case STILL_ERR_NOT_LOADED: return "layer weights not loaded";
+    case STILL_ERR_OOM: return "out of device memory or workspace limit";
+    case STILL_ERR_CUDA: return "CUDA error";
+    case STILL_ERR_TIMEOUT: return "device-side wait timed out";
+  }
+  return "unknown status";
+}
+
+still_status still_create(int device, still_ctx** out) {
+  if (out == nullptr) return STILL_ERR_INVALID_ARG;
+  *out = nullptr;
+  int ndev = 0;
+  if (cudaGetDeviceCount(&ndev) != cudaSuccess || device < 0 || device >= ndev) {
+    cudaGetLastError();
+    return STILL_ERR_INVALID_ARG;
+  }
+  CK(cudaSetDevice(device));
+  int major = 0, minor = 0;
+  CK(cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, device));
+  CK(cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, device));
+  if (major != 10 || minor != 3) return STILL_ERR_UNSUPPORTED;  // built for sm_103a only
+  still_ctx* c = new still_ctx();
+  c->device = device;
+  if (cudaDeviceGetAttribute(&c->nsm, cudaDevAttrMultiProcessorCount, device) != cudaSuccess ||
+      cudaMalloc(&c->err, 4 * sizeof(int)) != cudaSuccess ||
+      cudaMemset(c->err, 0, 4 * sizeof(int)) != cudaSuccess) {
+    delete c;
+    return STILL_ERR_CUDA;
+  }
+  *out = c;
+  return STILL_OK;
+}
+
+still_status still_destroy(still_ctx* ctx) {
+  if (ctx == nullptr) return STILL_ERR_INVALID_ARG;
+  cudaSetDevice(ctx->device);
+  cudaDeviceSynchronize();
+  for (auto& L : ctx->layers) free_layer(L);
+  if (ctx->ws) cudaFree(ctx->ws);
+  if (ctx->err) cudaFree(ctx->err);
+  delete ctx;
+  return STILL_OK;
+}
+
+still_status still_set_workspace_limit(still_ctx* ctx, size_t bytes) {
+  if (ctx == nullptr || bytes == 0) return STILL_ERR_INVALID_ARG;
+  ctx->ws_limit = bytes;
+  return STILL_OK;
+}
+
+still_status still_load_layer_weights(still_ctx* ctx, int32_t layer,
+                                      const still_layer_config* cfg,
+                                      const still_layer_weights* w, void* stream) {
+  if (ctx == nullptr || w == nullptr || layer < 0) return STILL_ERR_INVALID_ARG;
+  TRY(check_cfg(cfg));
+  const still_layer_config& c = *cfg;
+  const int H = c.n_kv_heads, d = c.head_dim, D = c.d_latent, n = c.n_cross_heads,
+            F = c.ffn_dim, T = c.t_max;
+  const void* req[] = {w->Z, w->Wq, w->bq, w->Wk, w->bk, w->Wv, w->Wo, w->Sq,
+                       w->sbq, w->Sk, w->sbk, w->Sv, w->So, w->Wkey, w->Wval};
+  for (const void* p : req)
+    if (p == nullptr) return STILL_ERR_INVALID_ARG;
+  if (F > 0 && (w->W1 == nullptr || w->W2 == nullptr)) return STILL_ERR_INVALID_ARG;
+  CK(cudaSetDevice(ctx->device));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if ((int32_t)ctx->layers.size() <= layer) ctx->layers.resize(layer + 1);
+  LayerW& L = ctx->layers[layer];
+  if (L.loaded) {
+    CK(cudaStreamSynchronize(s));
+    free_layer(L);
+  }
+  L.cfg = c;
+  if (L.cfg.logit_scale == 0) L.cfg.logit_scale = D;
+  const int64_t nD = (int64_t)n * D;
+  const bf16* Wq = static_cast<const bf16*>(w->Wq);
+  TRY(dalloc(L, &L.Z, (size_t)H * T * D));
+  TRY(dalloc(L, &L.WkT, (size_t)nD * 2 * d));
+  TRY(dalloc(L, &L.bk, (size_t)nD));
+  TRY(dalloc(L, &L.qhat, (size_t)H * n * T * D));
+  TRY(dalloc(L, &L.WvoT, (size_t)D * 2 * n * 2 * d));
+  TRY(dalloc(L, &L.SqkT, (size_t)2 * nD * D));
+  TRY(dalloc(L, &L.sbqk, (size_t)2 * nD));
+  TRY(dalloc(L, &L.SvT, (size_t)nD * D));
+  TRY(dalloc(L, &L.SoT, (size_t)D * nD));
+  if (F > 0) {
+    TRY(dalloc(L, &L.W1T, (size_t)F * D));
+    TRY(dalloc(L, &L.W2T, (size_t)D * F));
+  }
+  TRY(dalloc(L, &L.WhT, (size_t)2 * d * D));
+  TRY(dalloc(L, &L.omega_b, (size_t)d / 2));
+  TRY(dalloc(L, &L.omega_c, (size_t)D / 2));
+  CK(launch_omega(L.omega_b, d / 2, d, c.rope_theta, s));
+  CK(launch_omega(L.omega_c, D / 2, D, c.rope_theta_compactor, s));
+  CK(cudaMemcpyAsync(L.Z, w->Z, sizeof(bf16) * (size_t)H * T * D, cudaMemcpyDeviceToDevice, s));
+  CK(launch_transpose(static_cast<const bf16*>(w->Wk), 2 * d, nD, L.WkT, D, s));
+  CK(launch_bias(static_cast<const bf16*>(w->bk), nullptr, nD, L.bk, D, s));
+  CK(launch_transpose(static_cast<const bf16*>(w->Sq), D, nD, L.SqkT, 0, s));
+  CK(launch_transpose(static_cast<const bf16*>(w->Sk), D, nD, L.SqkT + nD * D, 0, s));
+  CK(launch_bias(static_cast<const bf16*>(w->sbq), static_cast<const bf16*>(w->sbk), nD, L.sbqk,
+                 0, s));
+  CK(launch_transpose(static_cast<const bf16*>(w->Sv), D, nD, L.SvT, 0, s));
+  CK(launch_transpose(static_cast<const bf16*>(w->So), nD, D, L.SoT, 0, s));
+  if (F > 0) {
+    CK(launch_transpose(static_cast<const bf16*>(w->W1), D, F, L.W1T, 0, s));
+    CK(launch_transpose(static_cast<const bf16*>(w->W2), F, D, L.W2T, 0, s));
+  }
+  CK(launch_transpose(static_cast<const bf16*>(w->Wkey), D, d, L.WhT, 0, s));
+  CK(launch_transpose(static_cast<const bf16*>(w->Wval), D, d, L.WhT + (size_t)d * D, 0, s));
+
+  // Temporaries for the precompute.
+  LayerW tmp;
+  bf16 *WqT = nullptr, *Zn = nullptr, *WoT = nullptr;
+  float *bq = nullptr, *qss = nullptr;
+  auto cleanup = [&]() {
+    cudaStreamSynchronize(s);
+    free_layer(tmp);
+  };
+  still_status st = STILL_OK;
+  if ((st = dalloc(tmp, &WqT, (size_t)nD * D)) != STILL_OK ||
+      (st = dalloc(tmp, &Zn, (size_t)H * T * 2 * D)) != STILL_OK ||
+      (st = dalloc(tmp, &WoT, (size_t)D * nD)) != STILL_OK ||
+      (st = dalloc(tmp, &bq, (size_t)nD)) != STILL_OK ||
+      (st = dalloc(tmp, &qss, (size_t)H * n * T)) != STILL_OK) {
+    cleanup();
+    free_layer(L);
+    return st;
+  }
+  auto body = [&]() -> still_status {
+    CK(launch_transpose(Wq, D, nD, WqT, D, s));
+    CK(launch_bias(static_cast<const bf16*>(w->bq), nullptr, nD, bq, D, s));
+    CK(launch_rmsnorm(w->Z, 1, (int64_t)H * T, D, D, c.rms_eps, Zn, 2 * D, 1, s));
+    CK(cudaMemsetAsync(qss, 0, sizeof(float) * (size_t)H * n * T, s));
+    {  // q~ = RMSNorm(Z) W_Q + b_Q  (2-pass), |q~|^2 per (row, head)
+      GemmParams p = gp(H * T, (int)nD);
+      add_pass(p, 0, 0, 0, 0, D);
+      add_pass(p, D, 0, 0, 0, D);
+      EpiAffine e;
+      e.kind = OUT_F32;
+      e.out = L.qhat;
+      e.om.rdiv = T;
+      e.om.r1 = (int64_t)n * T * D;
+      e.om.r0 = D;
+      e.om.cdiv = D;
+      e.om.c1 = (int64_t)T * D;
+      e.om.c0 = 1;
+      e.bias = bq;
+      e.sumsq = qss;
+      e.ssm.rdiv = T;
+      e.ssm.r1 = (int64_t)n * T;
+      e.ssm.r0 = 1;
+      e.ssm.c0 = T;
+      e.ss_seg = D;
+      e.vec_ok = 1;
+      TRY(run_gemm(ctx, STILL_K_LOAD, 256, op(Zn, (int64_t)H * T, 2 * D), op(WqT, nD, D), p, e, 1, s));
+    }
+    CK(launch_l2_scale(L.qhat, qss, (int64_t)H * n * T, D, c.l2_eps, s));
+    // W_VO,i = W_V,i W_O,i  -> stored transposed as hi | lo: WvoT[c][i*2d + f]
+    CK(launch_transpose(static_cast<const bf16*>(w->Wo), nD, D, WoT, 0, s));
+    {
+      GemmParams p = gp(2 * d, D, n, 1);
+      p.a_k1 = D;
+      p.b_k1 = D;
+      add_pass(p, 0, 0, 0, 0, D);
+      EpiAffine e;
+      e.kind = OUT_HILO;
+      e.out = L.WvoT;
+      e.lo_off = (int64_t)n * 2 * d;
+      e.om.b1 = 2 * d;
+      e.om.r0 = 1;
+      e.om.c0 = (int64_t)2 * n * 2 * d;
+      e.vec_ok = 0;
+      TRY(run_gemm(ctx, STILL_K_LOAD, 256, op(w->Wv, 2 * d, nD), op(WoT, D, nD), p, e, 1, s));
+    }
+    return STILL_OK;
+  };
+  st = body();
+  cleanup();
+  if (st != STILL_OK) {
+    free_layer(L);
+    return st;
+  }
+  L.loaded = true;
+  return STILL_OK;
+}
+
+still_status still_compact_layer(still_ctx* ctx, int32_t layer, const void* K, const void* V,
+                                 const int64_t strides_kv[3],
+                                 const still_pos_segment* h_segments, int32_t n_segments,
+                                 int64_t N, int32_t t, void* Ck, void* Cv,
+                                 double* h_out_pos_start, double* h_out_pos_step,
+                                 int64_t* h_pos_offset, void* stream) {
+  const LayerW* L = nullptr;
+  TRY(check_ctx_layer(ctx, layer, &L));
+  if (K == nullptr || V == nullptr || Ck == nullptr || Cv == nullptr || strides_kv == nullptr)
+    return STILL_ERR_INVALID_ARG;
+  if (N < 1 || t < 1 || t > N || t > L->cfg.t_max || N > (int64_t(1) << 30))
+    return STILL_ERR_SHAPE;
+  if (strides_kv[2] != 1 || strides_kv[0] < 1 || strides_kv[1] < 0) return STILL_ERR_SHAPE;
+  if ((reinterpret_cast<uintptr_t>(K) | reinterpret_cast<uintptr_t>(V) |
+       reinterpret_cast<uintptr_t>(Ck) | reinterpret_cast<uintptr_t>(Cv)) & 1)
+    return STILL_ERR_ALIGNMENT;
+  Positions pos;
+  TRY(make_positions(h_segments, n_segments, N, pos));
+  CK(cudaSetDevice(ctx->device));
+  const int H = L->cfg.n_kv_heads, d = L->cfg.head_dim;
+  OutSpec o{static_cast<bf16*>(Ck), static_cast<bf16*>(Cv), (int64_t)H * d, d};
+  TRY(compact_one(ctx, *L, static_cast<const bf16*>(K), static_cast<const bf16*>(V),
+                  strides_kv[0], strides_kv[1], pos, N, t, o,
+                  static_cast<cudaStream_t>(stream)));
+  if (h_out_pos_start) *h_out_pos_start = pos.pmin;
+  if (h_out_pos_step) *h_out_pos_step = t > 1 ? (pos.pmax - pos.pmin) / (double)(t - 1) : 0.0;
+  if (h_pos_offset) *h_pos_offset = N - t;
+  return STILL_OK;
+}
+
+still_status still_compact_stack(still_ctx* ctx, int32_t n_layers, const void* const* K,
+                                 const void* const* V, const int64_t strides_kv[3],
+                                 const still_pos_segment* h_segments, int32_t n_segments,
+                                 int64_t N, int32_t t, void* const* Ck, void* const* Cv,
+                                 double* h_out_pos_start, double* h_out_pos_step,
+                                 int64_t* h_pos_offset, void* stream) {
+  if (ctx == nullptr || K == nullptr || V == nullptr || Ck == nullptr || Cv == nullptr ||
+      n_layers < 1)
+    return STILL_ERR_INVALID_ARG;
+  for (int l = 0; l < n_layers; ++l) {
+    const LayerW* L = nullptr;
+    TRY(check_ctx_layer(ctx, l, &L));
+  }
+  for (int l = 0; l < n_layers; ++l)
+    TRY(still_compact_layer(ctx, l, K[l], V[l], strides_kv, h_segments, n_segments, N, t, Ck[l],
+                            Cv[l], h_out_pos_start, h_out_pos_step, h_pos_offset, stream));
+  return STILL_OK;
+}
+
+still_status still_compact_layer_ragged(still_ctx* ctx, int32_t layer, const void* Kpacked,
+                                        const void* Vpacked, const int64_t* h_cu_seqlens,
+                                        int32_t B, const still_pos_segment* h_segments,
+                                        const int32_t* h_seg_per_seq, const int32_t* h_t,
+                                        const int64_t* h_cu_t, void* Ck, void* Cv,
+                                        int64_t* h_pos_offset, void* stream) {
+  const LayerW* L = nullptr;
+  TRY(check_ctx_layer(ctx, layer, &L));
+  if (Kpacked == nullptr || Vpacked == nullptr || h_cu_seqlens == nullptr || h_t == nullptr ||
+      h_cu_t == nullptr || Ck == nullptr || Cv == nullptr || B < 1)
+    return STILL_ERR_INVALID_ARG;
+  if ((h_segments == nullptr) != (h_seg_per_seq == nullptr)) return STILL_ERR_INVALID_ARG;
+  if (h_cu_seqlens[0] != 0 || h_cu_t[0] != 0) return STILL_ERR_SHAPE;
+  for (int b = 0; b < B; ++b) {
+    if (h_cu_seqlens[b + 1] < h_cu_seqlens[b] || h_cu_t[b + 1] - h_cu_t[b] != h_t[b])
+      return STILL_ERR_SHAPE;
+    const int64_t Nb = h_cu_seqlens[b + 1] - h_cu_seqlens[b];
+    if (Nb < 1 || h_t[b] < 1 || h_t[b] > Nb || h_t[b] > L->cfg.t_max) return STILL_ERR_SHAPE;
+  }
+  const int H = L->cfg.n_kv_heads, d = L->cfg.head_dim;
+  const int64_t row = (int64_t)H * d;
+  const int64_t strides[3] = {row, d, 1};
+  int seg0 = 0;
+  for (int b = 0; b < B; ++b) {
+    const int64_t Nb = h_cu_seqlens[b + 1] - h_cu_seqlens[b];
+    const still_pos_segment* sg = h_segments ? h_segments + seg0 : nullptr;
+    const int nsg = h_seg_per_seq ? h_seg_per_seq[b] : 0;
+    seg0 += nsg;
+    TRY(still_compact_layer(
+        ctx, layer, static_cast<const bf16*>(Kpacked) + h_cu_seqlens[b] * row,
+        static_cast<const bf16*>(Vpacked) + h_cu_seqlens[b] * row, strides, sg, nsg, Nb, h_t[b],
+        static_cast<bf16*>(Ck) + h_cu_t[b] * row, static_cast<bf16*>(Cv) + h_cu_t[b] * row,
+        nullptr, nullptr, h_pos_offset ? h_pos_offset + b : nullptr, stream));
+  }
+  return STILL_OK;
+}
+
+still_status still_compact_stack_ragged(still_ctx* ctx, int32_t n_layers,
+                                        const void* const* Kpacked, const void* const* Vpacked,
+                                        const int64_t* h_cu_seqlens, int32_t B,
+                                        const still_pos_segment* h_segments,
+                                        const int32_t* h_seg_per_seq, const int32_t* h_t,
+                                        const int64_t* h_cu_t, void* const* Ck,
+                                        void* const* Cv, int64_t* h_pos_offset, void* stream) {
+  if (ctx == nullptr || Kpacked == nullptr || Vpacked == nullptr || Ck == nullptr ||
+      Cv == nullptr || n_layers < 1)
+    return STILL_ERR_INVALID_ARG;
+  for (int l = 0; l < n_layers; ++l)
+    TRY(still_compact_layer_ragged(ctx, l, Kpacked[l], Vpacked[l], h_cu_seqlens, B, h_segments,
+                                   h_seg_per_seq, h_t, h_cu_t, Ck[l], Cv[l], h_pos_offset,
+                                   stream));
+  return STILL_OK;
+}
+
+still_status still_workspace_size(const still_ctx* ctx, int64_t max_tokens, int32_t max_t,
+                                  size_t* bytes) {
+  if (ctx == nullptr || bytes == nullptr || ctx->layers.empty() || !ctx->layers[0].loaded)
+    return ctx == nullptr || bytes == nullptr ? STILL_ERR_INVALID_ARG : STILL_ERR_NOT_LOADED;
+  if (max_tokens < 1 || max_t < 1 || max_t > max_tokens) return STILL_ERR_SHAPE;
+  Plan P;
+  if (!make_plan(ctx->layers[0].cfg, max_tokens, max_t, 0.0, (double)(max_tokens - 1),
+                 ctx->ws_limit, P))
+    return STILL_ERR_OOM;
+  *bytes = P.total;
+  return STILL_OK;
+}
+
+still_status still_get_device_status(still_ctx* ctx, void* stream, int32_t* h_detail) {
+  if (ctx == nullptr) return STILL_ERR_INVALID_ARG;
+  CK(cudaSetDevice(ctx->device));
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  int rec[4] = {0, 0, 0, 0};
+  if (cudaMemcpy(rec, ctx->err, sizeof(rec), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return STILL_ERR_CUDA;
+  if (h_detail)
+    for (int i = 0; i < 4; ++i) h_detail[i] = rec[i];
+  if (rec[0] != 0) cudaMemset(ctx->err, 0, sizeof(rec));
+  if (e != cudaSuccess) return STILL_ERR_CUDA;
+  if (rec[0] == DEV_WAIT_TIMEOUT) return STILL_ERR_TIMEOUT;
+  if (rec[0] != 0) return STILL_ERR_CUDA;
+  return STILL_OK;
+}
+
+still_status still_profile_enable(still_ctx* ctx, int32_t enable) {
+  if (ctx == nullptr) return STILL_ERR_INVALID_ARG;
+  CK(cudaSetDevice(ctx->device));
+  ctx->prof.reset();
+  ctx->prof.on = enable != 0;
+  return STILL_OK;
+}
+
+still_status still_profile_read(still_ctx* ctx, int32_t cls, int64_t* h_launches, double* h_ms) {
+  if (ctx == nullptr || cls < 0 || cls >= STILL_K_COUNT) return STILL_ERR_INVALID_ARG;
+  CK(cudaSetDevice(ctx->device));
+  if (!ctx->prof.resolve()) return STILL_ERR_CUDA;
+  if (h_launches) *h_launches = ctx->prof.launches[cls];
+  if (h_ms) *h_ms = ctx->prof.ms[cls];
+  return STILL_OK;
+}
+
+const char* still_kernel_class_name(int32_t cls) {
+  static const char* names[STILL_K_COUNT] = {
+      "strip", "rope_tables", "keyproj", "q_rope", "scores", "softmax", "px", "px_split",
+      "vo", "rmsnorm", "sa_proj", "sa_v", "sa_scores", "sa_softmax", "sa_pv", "sa_out",
+      "ffn1", "ffn2", "heads", "load"};
+  return cls >= 0 && cls < STILL_K_COUNT ? names[cls] : "unknown";
+}
+
+int64_t still_budget(int64_t n_tokens, int64_t ratio) {
+  if (n_tokens < 0 || ratio < 1) return -1;
+  return (2 * n_tokens + ratio) / (2 * ratio);
+}
+
+int64_t still_kv_bytes(int64_t n_layers, int64_t n_kv_heads, int64_t head_dim,
+                       int64_t elem_bytes, int64_t n_slots) {
+  return 2 * n_layers * n_kv_heads * head_dim * elem_bytes * n_slots;
+}
+
+int64_t still_param_count(const still_layer_config* cfg, int32_t t) {
+  if (cfg == nullptr) return -1;
+  const int64_t H = cfg->n_kv_heads, d = cfg->head_dim, D = cfg->d_latent;
+  const int64_t nc = cfg->n_cross_heads, ns = cfg->n_self_heads, F = cfg->ffn_dim;
+  const int64_t B = cfg->n_blocks, Bc = cfg->cross_every_block ? B : 1;
+  return H * t * D + Bc * (2 * nc * D * D + 4 * d * nc * D) + B * (4 * ns * D * D) +
+         B * (2 * F * D) + (2 * D * d + D);
+}
+
+}  // extern "C"

@@ -1,0 +1,264 @@
+// Persistent tcgen05 GEMM with split-precision passes, for sm_103a.
+//
+//   C[b](m, n) = sum over passes p of  A_p[b](m, :) . B_p[b](n, :)       (fp32 accumulate)
+//
+// A and B are 16-bit (bf16 or fp16), K-major, read by TMA in 128-byte-swizzled boxes of
+// 64 elements along K. A pass names a K offset and a row offset into each operand, so a
+// "hi/lo" operand stored as [hi | lo] along K gives the 2- and 3-pass products that keep
+// ~fp32 accuracy on bf16 tensor cores (a_hi b_hi + a_hi b_lo + a_lo b_hi).
+//
+// CTA = 10 warps: warp 0 issues TMA, warp 1 owns TMEM and issues tcgen05.mma (one thread),
+// warps 2..9 run the epilogue from TMEM (two per lane quarter, alternating column chunks). The accumulator is double-buffered in TMEM
+// (2 x BN fp32 columns), so a tile's epilogue overlaps the next tile's main loop.
+// Tiles are 128 x BN; the grid is persistent (tile += gridDim.x), m-tiles fastest so that
+// CTAs running together share B tiles through L2.
+#pragma once
+#include "ptx.cuh"
+
+namespace still {
+
+constexpr int kBM = 128;
+constexpr int kBK = 64;
+constexpr int kEpiWarps = 8;  // two warps per TMEM lane quarter, alternating 32-column chunks
+constexpr int kGemmThreads = 64 + 32 * kEpiWarps;
+
+struct GemmPass {
+  int32_t a_koff, b_koff;  // K offset (elements) of this pass in A / B
+  int32_t a_roff, b_roff;  // row offset of this pass in A / B
+  int32_t klen;            // K extent, a multiple of 64
+};
+
+struct GemmParams {
+  int32_t M, N;         // output extent per batch
+  int32_t batch, bdiv;  // batch b splits as (b / bdiv, b % bdiv)
+  // Row / K origin of batch b in each operand: (b / bdiv) * x1 + (b % bdiv) * x0.
+  int64_t a_r1, a_r0, a_k1, a_k0;
+  int64_t b_r1, b_r0, b_k1, b_k0;
+  int32_t npass;
+  GemmPass pass[3];
+  int32_t ksplit;  // split-K factor (each split = a contiguous range of K iterations)
+  // Derived by the host launcher.
+  int32_t tiles_m, tiles_n, iters_total, ntiles;
+  uint32_t idesc;
+  int* err;  // device error record (may be null)
+};
+
+struct TileCoord {
+  int b, tm, tn, split;
+};
+
+__device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int tile) {
+  TileCoord c;
+  c.tm = tile % p.tiles_m;
+  int r = tile / p.tiles_m;
+  c.split = r % p.ksplit;
+  r /= p.ksplit;
+  c.tn = r % p.tiles_n;
+  c.b = r / p.tiles_n;
+  return c;
+}
+
+__device__ __forceinline__ void split_range(const GemmParams& p, int split, int& it0, int& it1) {
+  it0 = (int)(((int64_t)p.iters_total * split) / p.ksplit);
+  it1 = (int)(((int64_t)p.iters_total * (split + 1)) / p.ksplit);
+}
+
+template <int BN>
+struct GemmSmem {
+  static constexpr int kStages = BN >= 256 ? 4 : 6;
+  static constexpr int kABytes = kBM * kBK * 2;
+  static constexpr int kBBytes = BN * kBK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kBarOffset = kStages * kStageBytes;
+  static constexpr int kBytes = kBarOffset + 256 + 1024;  // + barriers + alignment slack
+};
+
+// Epi must provide:  __device__ void operator()(const GemmParams&, const TileCoord&,
+//                    int row_in_tile, uint32_t tmem_addr_of_this_warp_lane_quarter,
+//                    int half) const;
+// where `half` (0 or 1) selects the 32-column chunks this warp owns: chunk c is handled by the
+// warp with half == (c & 1); the functor loads TMEM and stores its own results.
+template <int BN, class Epi>
+__global__ void __launch_bounds__(kGemmThreads, 1)
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
+                   const __grid_constant__ CUtensorMap tmB, const GemmParams p, const Epi epi) {
+  using S = GemmSmem<BN>;
+  constexpr int kStages = S::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::kBarOffset);
+  uint64_t* empty = full + kStages;
+  uint64_t* tfull = empty + kStages;  // [2]
+  uint64_t* tempty = tfull + 2;       // [2]
+  uint64_t* drain = tempty + 2;       // [1]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], kEpiWarps);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, 2 * BN);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ TMA producer
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t armed = 0;  // bit s: stage s armed at least once
+      uint32_t armed_par = 0;
+      for (int tile = blockIdx.x; tile < p.ntiles && !*abort_flag; tile += gridDim.x) {
+        const TileCoord tc = decode_tile(p, tile);
+        const int bo = tc.b / p.bdiv, bi = tc.b % p.bdiv;
+        const int64_t ar = bo * p.a_r1 + bi * p.a_r0 + (int64_t)tc.tm * kBM;
+        const int64_t ak = bo * p.a_k1 + bi * p.a_k0;
+        const int64_t br = bo * p.b_r1 + bi * p.b_r0 + (int64_t)tc.tn * BN;
+        const int64_t bk = bo * p.b_k1 + bi * p.b_k0;
+        int it0, it1;
+        split_range(p, tc.split, it0, it1);
+        int pass = 0, base = 0;
+        for (int it = it0; it < it1; ++it) {
+          while (pass < p.npass - 1 && it >= base + p.pass[pass].klen / kBK) {
+            base += p.pass[pass].klen / kBK;
+            ++pass;
+          }
+          const GemmPass& ps = p.pass[pass];
+          const int kk = (it - base) * kBK;
+          if (!mbar_wait(&empty[stage], phase ^ 1)) {
+            dev_set_error(p.err, DEV_WAIT_TIMEOUT, 100);
+            *abort_flag = 1;
+            break;
+          }
+          mbar_arrive_expect_tx(&full[stage], S::kStageBytes);
+          uint8_t* sa = smem + stage * S::kStageBytes;
+          tma_load_2d(sa, &tmA, &full[stage], (int32_t)(ak + ps.a_koff + kk),
+                      (int32_t)(ar + ps.a_roff));
+          tma_load_2d(sa + S::kABytes, &tmB, &full[stage], (int32_t)(bk + ps.b_koff + kk),
+                      (int32_t)(br + ps.b_roff));
+          armed |= 1u << stage;
+          armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
+          if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      if (*abort_flag) {
+        // Let every copy this thread issued land before the CTA can exit.
+        for (int s = 0; s < kStages; ++s)
+          if (armed & (1u << s)) (void)mbar_wait(&full[s], (armed_par >> s) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ MMA issuer
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool issued = false;
+      for (int tile = blockIdx.x; tile < p.ntiles && !*abort_flag; tile += gridDim.x) {
+        const TileCoord tc = decode_tile(p, tile);
+        int it0, it1;
+        split_range(p, tc.split, it0, it1);
+        if (!mbar_wait(&tempty[acc], acc_phase ^ 1)) {
+          dev_set_error(p.err, DEV_WAIT_TIMEOUT, 101);
+          *abort_flag = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+        for (int it = it0; it < it1; ++it) {
+          if (!mbar_wait(&full[stage], phase)) {
+            dev_set_error(p.err, DEV_WAIT_TIMEOUT, 102);
+            *abort_flag = 1;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + stage * S::kStageBytes);
+          const uint64_t ad = sdesc_k_sw128(sa);
+          const uint64_t bd = sdesc_k_sw128(sa + S::kABytes);
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k)
+            tc_mma_f16(d_tmem, ad + 2 * k, bd + 2 * k, p.idesc, (it > it0 || k > 0) ? 1u : 0u);
+          issued = true;
+          tc_commit(&empty[stage]);
+          if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (*abort_flag) break;
+        tc_commit(&tfull[acc]);
+        if (++acc == 2) {
+          acc = 0;
+          acc_phase ^= 1;
+        }
+      }
+      if (*abort_flag && issued) {
+        tc_commit(drain);
+        (void)mbar_wait(drain, 0);
+      }
+    }
+  } else {
+    // -------------------------------------------------------------- epilogue (warps 2..9)
+    const int quarter = warp & 3;  // TMEM lanes this warp may access: [32q, 32q + 32)
+    const int half = (warp - 2) >> 2;
+    const int row = quarter * 32 + lane;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = blockIdx.x; tile < p.ntiles; tile += gridDim.x) {
+      const TileCoord tc = decode_tile(p, tile);
+      bool ok = mbar_wait(&tfull[acc], acc_phase);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok || *abort_flag) {
+        if (lane == 0 && !ok) {
+          dev_set_error(p.err, DEV_WAIT_TIMEOUT, 103);
+          *abort_flag = 1;
+        }
+        break;
+      }
+      tc_fence_after();
+      const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * BN);
+      epi(p, tc, row, taddr, half);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[acc]);
+      if (++acc == 2) {
+        acc = 0;
+        acc_phase ^= 1;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, 2 * BN);
+  }
+}
+
+}  // namespace still

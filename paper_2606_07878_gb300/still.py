@@ -1,0 +1,294 @@
+"""Thin Python binding of the C ABI in include/still.h (ctypes; argument marshalling only).
+
+Every compute step runs inside libstill.so. Tensors are torch CUDA tensors (device memory and
+streams are PyTorch's plumbing); the functions keep the C names. There is no fallback: if the
+library is missing or cannot load, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libstill.so")
+
+STATUS = {
+    0: "STILL_OK", 1: "STILL_ERR_INVALID_ARG", 2: "STILL_ERR_UNSUPPORTED", 3: "STILL_ERR_SHAPE",
+    4: "STILL_ERR_ALIGNMENT", 5: "STILL_ERR_NOT_LOADED", 6: "STILL_ERR_OOM", 7: "STILL_ERR_CUDA",
+    8: "STILL_ERR_TIMEOUT",
+}
+
+# Every entry point include/still.h declares.
+EXPORTS = [
+    "still_create", "still_destroy", "still_status_string", "still_load_layer_weights",
+    "still_compact_layer", "still_compact_stack", "still_compact_layer_ragged",
+    "still_compact_stack_ragged", "still_workspace_size", "still_set_workspace_limit",
+    "still_get_device_status", "still_budget", "still_kv_bytes", "still_param_count",
+    "still_profile_enable", "still_profile_read", "still_kernel_class_name",
+]
+
+KERNEL_CLASSES = ["strip", "rope_tables", "keyproj", "q_rope", "scores", "softmax", "px",
+                  "px_split", "vo", "rmsnorm", "sa_proj", "sa_v", "sa_scores", "sa_softmax",
+                  "sa_pv", "sa_out", "ffn1", "ffn2", "heads", "load"]
+
+
+class StillError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        self.name = STATUS.get(code, f"status {code}")
+        super().__init__(f"{where}: {self.name}")
+
+
+class LayerConfig(ctypes.Structure):
+    _fields_ = [
+        ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+        ("d_latent", ctypes.c_int32), ("n_cross_heads", ctypes.c_int32),
+        ("n_self_heads", ctypes.c_int32), ("ffn_dim", ctypes.c_int32),
+        ("n_blocks", ctypes.c_int32), ("cross_every_block", ctypes.c_int32),
+        ("t_max", ctypes.c_int32), ("final_norm", ctypes.c_int32),
+        ("compactor_rope", ctypes.c_int32), ("rope_fix", ctypes.c_int32),
+        ("rope_theta", ctypes.c_double), ("rope_theta_compactor", ctypes.c_double),
+        ("logit_scale", ctypes.c_double), ("rms_eps", ctypes.c_float), ("l2_eps", ctypes.c_float),
+    ]
+
+
+WEIGHT_NAMES = ["Z", "Wq", "bq", "Wk", "bk", "Wv", "Wo", "Sq", "sbq", "Sk", "sbk", "Sv", "So",
+                "W1", "W2", "Wkey", "Wval"]
+
+
+class LayerWeights(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in WEIGHT_NAMES]
+
+
+class PosSegment(ctypes.Structure):
+    _fields_ = [("start", ctypes.c_double), ("step", ctypes.c_double), ("count", ctypes.c_int64)]
+
+
+_lib = None
+
+
+def lib():
+    """Loads libstill.so (raises if it is not built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is not built: run __graft_entry__.build()")
+        L = ctypes.CDLL(LIB_PATH)
+        P, I32, I64, D = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_double
+        PI64, PD, PI32 = ctypes.POINTER(I64), ctypes.POINTER(D), ctypes.POINTER(I32)
+        PSEG = ctypes.POINTER(PosSegment)
+        sig = {
+            "still_create": ([ctypes.c_int, ctypes.POINTER(P)], ctypes.c_int),
+            "still_destroy": ([P], ctypes.c_int),
+            "still_status_string": ([ctypes.c_int], ctypes.c_char_p),
+            "still_load_layer_weights": ([P, I32, ctypes.POINTER(LayerConfig),
+                                          ctypes.POINTER(LayerWeights), P], ctypes.c_int),
+            "still_compact_layer": ([P, I32, P, P, PI64, PSEG, I32, I64, I32, P, P, PD, PD, PI64,
+                                     P], ctypes.c_int),
+            "still_compact_stack": ([P, I32, ctypes.POINTER(P), ctypes.POINTER(P), PI64, PSEG, I32,
+                                     I64, I32, ctypes.POINTER(P), ctypes.POINTER(P), PD, PD, PI64,
+                                     P], ctypes.c_int),
+            "still_compact_layer_ragged": ([P, I32, P, P, PI64, I32, PSEG, PI32, PI32, PI64, P, P,
+                                            PI64, P], ctypes.c_int),
+            "still_compact_stack_ragged": ([P, I32, ctypes.POINTER(P), ctypes.POINTER(P), PI64, I32,
+                                            PSEG, PI32, PI32, PI64, ctypes.POINTER(P),
+                                            ctypes.POINTER(P), PI64, P], ctypes.c_int),
+            "still_workspace_size": ([P, I64, I32, ctypes.POINTER(ctypes.c_size_t)], ctypes.c_int),
+            "still_set_workspace_limit": ([P, ctypes.c_size_t], ctypes.c_int),
+            "still_get_device_status": ([P, P, PI32], ctypes.c_int),
+            "still_budget": ([I64, I64], I64),
+            "still_kv_bytes": ([I64, I64, I64, I64, I64], I64),
+            "still_param_count": ([ctypes.POINTER(LayerConfig), I32], I64),
+            "still_profile_enable": ([P, I32], ctypes.c_int),
+            "still_profile_read": ([P, I32, PI64, PD], ctypes.c_int),
+            "still_kernel_class_name": ([I32], ctypes.c_char_p),
+        }
+        for name, (args, res) in sig.items():
+            f = getattr(L, name)
+            f.argtypes = args
+            f.restype = res
+        _lib = L
+    return _lib
+
+
+def _check(code: int, where: str):
+    if code != 0:
+        raise StillError(code, where)
+
+
+def _ptr(x):
+    if x is None:
+        return None
+    return ctypes.c_void_p(x.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return ctypes.c_void_p(stream)
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _segments(segments):
+    if not segments:
+        return None, 0
+    arr = (PosSegment * len(segments))(*[PosSegment(float(a), float(b), int(c))
+                                          for a, b, c in segments])
+    return arr, len(segments)
+
+
+def make_config(H, d, D, n, F, t_max, theta, theta_c=10.0, final_norm=0, logit_scale=0.0,
+                rms_eps=1e-6, l2_eps=1e-12, n_blocks=1, cross_every_block=1, compactor_rope=1,
+                rope_fix=1) -> LayerConfig:
+    return LayerConfig(H, d, D, n, n, F, n_blocks, cross_every_block, t_max, final_norm,
+                       compactor_rope, rope_fix, theta, theta_c, logit_scale, rms_eps, l2_eps)
+
+
+def config_from_workload(wl: dict, t_max: int, **over) -> LayerConfig:
+    kw = dict(H=wl["H"], d=wl["d"], D=wl["D"], n=wl["n"], F=wl["F"], t_max=t_max,
+              theta=wl["theta"])
+    kw.update(over)
+    return make_config(**kw)
+
+
+# ------------------------------------------------------------------------------ entry points
+
+def still_status_string(code: int) -> str:
+    return lib().still_status_string(code).decode()
+
+
+def still_create(device: int = 0):
+    h = ctypes.c_void_p()
+    _check(lib().still_create(device, ctypes.byref(h)), "still_create")
+    return h
+
+
+def still_destroy(ctx):
+    _check(lib().still_destroy(ctx), "still_destroy")
+
+
+def still_set_workspace_limit(ctx, nbytes: int):
+    _check(lib().still_set_workspace_limit(ctx, nbytes), "still_set_workspace_limit")
+
+
+def still_load_layer_weights(ctx, layer: int, cfg: LayerConfig, weights: dict, stream=None):
+    """weights: name -> contiguous bf16 CUDA tensor, layouts as in include/still.h."""
+    w = LayerWeights(**{n: (weights[n].data_ptr() if weights.get(n) is not None else None)
+                        for n in WEIGHT_NAMES})
+    _check(lib().still_load_layer_weights(ctx, layer, ctypes.byref(cfg), ctypes.byref(w),
+                                          _stream(stream)), "still_load_layer_weights")
+
+
+def still_compact_layer(ctx, layer: int, K, V, t: int, Ck, Cv, segments=None, stream=None):
+    """K, V [N, H, d] bf16 CUDA (d contiguous); Ck, Cv [t, H, d] bf16 CUDA outputs.
+    Returns (out_pos_start, out_pos_step, pos_offset)."""
+    strides = (ctypes.c_int64 * 3)(*K.stride())
+    assert tuple(V.stride()) == tuple(K.stride()), "K and V must share strides"
+    seg, nseg = _segments(segments)
+    ps, pst, off = ctypes.c_double(), ctypes.c_double(), ctypes.c_int64()
+    _check(lib().still_compact_layer(ctx, layer, _ptr(K), _ptr(V), strides, seg, nseg,
+                                     K.shape[0], t, _ptr(Ck), _ptr(Cv), ctypes.byref(ps),
+                                     ctypes.byref(pst), ctypes.byref(off), _stream(stream)),
+           "still_compact_layer")
+    return ps.value, pst.value, off.value
+
+
+def still_compact_stack(ctx, Ks, Vs, t: int, Cks, Cvs, segments=None, stream=None):
+    L = len(Ks)
+    P = ctypes.c_void_p
+    arr = lambda xs: (P * L)(*[x.data_ptr() for x in xs])
+    strides = (ctypes.c_int64 * 3)(*Ks[0].stride())
+    seg, nseg = _segments(segments)
+    ps, pst, off = ctypes.c_double(), ctypes.c_double(), ctypes.c_int64()
+    _check(lib().still_compact_stack(ctx, L, arr(Ks), arr(Vs), strides, seg, nseg,
+                                     Ks[0].shape[0], t, arr(Cks), arr(Cvs), ctypes.byref(ps),
+                                     ctypes.byref(pst), ctypes.byref(off), _stream(stream)),
+           "still_compact_stack")
+    return ps.value, pst.value, off.value
+
+
+def _ragged_args(cu_seqlens, ts, segments_per_seq):
+    B = len(ts)
+    cu = (ctypes.c_int64 * (B + 1))(*cu_seqlens)
+    tt = (ctypes.c_int32 * B)(*ts)
+    cut = [0]
+    for x in ts:
+        cut.append(cut[-1] + x)
+    cu_t = (ctypes.c_int64 * (B + 1))(*cut)
+    if segments_per_seq is None:
+        return B, cu, tt, cu_t, None, None
+    flat = [s for segs in segments_per_seq for s in segs]
+    seg, _ = _segments(flat)
+    per = (ctypes.c_int32 * B)(*[len(s) for s in segments_per_seq])
+    return B, cu, tt, cu_t, seg, per
+
+
+def still_compact_layer_ragged(ctx, layer, Kp, Vp, cu_seqlens, ts, Ck, Cv,
+                               segments_per_seq=None, stream=None):
+    """Kp, Vp [sum N_b, H, d]; Ck, Cv [sum t_b, H, d]. Returns the per-sequence offsets."""
+    B, cu, tt, cu_t, seg, per = _ragged_args(cu_seqlens, ts, segments_per_seq)
+    off = (ctypes.c_int64 * B)()
+    _check(lib().still_compact_layer_ragged(ctx, layer, _ptr(Kp), _ptr(Vp), cu, B, seg, per, tt,
+                                            cu_t, _ptr(Ck), _ptr(Cv), off, _stream(stream)),
+           "still_compact_layer_ragged")
+    return list(off)
+
+
+def still_compact_stack_ragged(ctx, Kps, Vps, cu_seqlens, ts, Cks, Cvs, segments_per_seq=None,
+                               stream=None):
+    L = len(Kps)
+    P = ctypes.c_void_p
+    arr = lambda xs: (P * L)(*[x.data_ptr() for x in xs])
+    B, cu, tt, cu_t, seg, per = _ragged_args(cu_seqlens, ts, segments_per_seq)
+    off = (ctypes.c_int64 * B)()
+    _check(lib().still_compact_stack_ragged(ctx, L, arr(Kps), arr(Vps), cu, B, seg, per, tt, cu_t,
+                                            arr(Cks), arr(Cvs), off, _stream(stream)),
+           "still_compact_stack_ragged")
+    return list(off)
+
+
+def still_workspace_size(ctx, max_tokens: int, max_t: int) -> int:
+    b = ctypes.c_size_t()
+    _check(lib().still_workspace_size(ctx, max_tokens, max_t, ctypes.byref(b)),
+           "still_workspace_size")
+    return b.value
+
+
+def still_get_device_status(ctx, stream=None):
+    """Synchronizes the stream; returns (status_code, [code, site, block, count])."""
+    det = (ctypes.c_int32 * 4)()
+    code = lib().still_get_device_status(ctx, _stream(stream), det)
+    return code, list(det)
+
+
+def still_budget(n_tokens: int, ratio: int) -> int:
+    return lib().still_budget(n_tokens, ratio)
+
+
+def still_kv_bytes(L, H, d, b, S) -> int:
+    return lib().still_kv_bytes(L, H, d, b, S)
+
+
+def still_param_count(cfg: LayerConfig, t: int) -> int:
+    return lib().still_param_count(ctypes.byref(cfg), t)
+
+
+def still_profile_enable(ctx, enable: bool = True):
+    _check(lib().still_profile_enable(ctx, 1 if enable else 0), "still_profile_enable")
+
+
+def still_profile_read(ctx):
+    """{class name: (launches, total ms)} since the last still_profile_enable."""
+    out = {}
+    for i, name in enumerate(KERNEL_CLASSES):
+        n, ms = ctypes.c_int64(), ctypes.c_double()
+        _check(lib().still_profile_read(ctx, i, ctypes.byref(n), ctypes.byref(ms)),
+               "still_profile_read")
+        out[name] = (n.value, ms.value)
+    return out
+
+
+def still_kernel_class_name(cls: int) -> str:
+    return lib().still_kernel_class_name(cls).decode()

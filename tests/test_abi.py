@@ -1,0 +1,64 @@
+"""CPU checks of the boundary: libstill.so loads, exports every entry point include/still.h
+declares, and its host-only accounting functions match the paper's printed numbers."""
+import json
+import os
+import re
+
+import pytest
+
+from paper_2606_07878_gb300 import still
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "still.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(still_[a-z_]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not os.path.exists(still.LIB_PATH):
+        from paper_2606_07878_gb300 import build
+        build.build()
+    return still.lib()
+
+
+def test_exports_every_declared_symbol(lib):
+    declared = _declared()
+    assert declared, "no declarations parsed"
+    assert sorted(still.EXPORTS) == declared
+    for name in declared:
+        assert hasattr(lib, name), name
+
+
+def test_status_strings(lib):
+    for code in still.STATUS:
+        assert still.still_status_string(code)
+
+
+def test_budget_matches_paper_table(lib):
+    g = json.load(open(os.path.join(GOLDEN, "budgets.json")))
+    for ctx, ratio, K in g["rows"]:
+        assert still.still_budget(g["ctx_tokens"][ctx], ratio) == K
+
+
+def test_kv_bytes_matches_paper(lib):
+    g = json.load(open(os.path.join(GOLDEN, "kv_bytes.json")))
+    m = g["model"]
+    assert still.still_kv_bytes(m["L"], m["H"], m["d"], m["b"], 1) == 144 * 1024
+    for S, gib in g["gib_at_tokens"]:
+        assert still.still_kv_bytes(m["L"], m["H"], m["d"], m["b"], S) / 2**30 == pytest.approx(
+            gib, abs=5e-4)
+
+
+def test_param_count_matches_paper(lib):
+    g = json.load(open(os.path.join(GOLDEN, "param_counts.json")))
+    b = g["base"]
+    for c in g["cases"]:
+        cfg = still.make_config(b["H"], b["d"], c["D"], c["n"], c["r"] * c["D"], c["t"], 1e6,
+                                n_blocks=c["B"], cross_every_block=int(c["cross_every_block"]))
+        total = b["L"] * still.still_param_count(cfg, c["t"])
+        assert abs(total - c["printed_total"]) <= g["tolerance_abs"], c["name"]
