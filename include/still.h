@@ -122,7 +122,7 @@ still_status still_load_layer_weights(still_ctx* ctx, int32_t layer,
  *              smallest to the largest key position, both ends included (App. A,
  *              Cross-attention; App. B, step 5).
  *   t          compact length, 1 <= t <= min(N, t_max)
- *   Ck, Cv     [t, H, d] bf16 device outputs, caller-owned, contiguous
+ *   Ck, Cv     [t, H, d] bf16 device outputs, caller-owned, contiguous, 16-byte aligned
  *   h_out_pos_start, h_out_pos_step  (optional) output positions start + j * step
  *   h_pos_offset (optional) logical minus physical length, N - t (App. B, "Logical vs.
  *              physical cache length")

@@ -30,6 +30,43 @@ __device__ __forceinline__ float gelu_erf(float x) {
   return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f));
 }
 
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(a, b);  // a -> low half, b -> high half
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// hi/lo split of two values, packed: hi = bf16(x), lo = bf16(x - hi)
+__device__ __forceinline__ void split_pack(float a, float b, uint32_t& hi, uint32_t& lo) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  const float2 hf = __bfloat1622float2(h);
+  const __nv_bfloat162 l = __floats2bfloat162_rn(a - hf.x, b - hf.y);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
+}
+
+// 32 floats -> 32 bf16 (4 x uint4) at dst (16-byte aligned)
+__device__ __forceinline__ void store_bf16x32(__nv_bfloat16* dst, const float (&v)[32]) {
+  uint4* d = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+  for (int q = 0; q < 4; ++q)
+    d[q] = make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                      pack_bf16x2(v[8 * q + 4], v[8 * q + 5]),
+                      pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+}
+
+// 32 floats -> hi (4 x uint4) at dh and lo (4 x uint4) at dl
+__device__ __forceinline__ void store_hilo_x32(__nv_bfloat16* dh, __nv_bfloat16* dl,
+                                               const float (&v)[32]) {
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    uint32_t h[4], l[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) split_pack(v[8 * q + 2 * k], v[8 * q + 2 * k + 1], h[k], l[k]);
+    reinterpret_cast<uint4*>(dh)[q] = make_uint4(h[0], h[1], h[2], h[3]);
+    reinterpret_cast<uint4*>(dl)[q] = make_uint4(l[0], l[1], l[2], l[3]);
+  }
+}
+
 // General epilogue: v = acc * alpha [* colscale(c)] [* rowscale(r)] [+ bias(c)]
 //   -> [sumsq accumulation] -> [GELU] -> [+ residual] -> store (f32 / bf16 / hi-lo / atomic f32)
 // colscale / rowscale = 1 / max(sqrt(sumsq[idx]), eps) from a sum-of-squares buffer.
@@ -134,28 +171,15 @@ struct EpiAffine {
 #pragma unroll
         for (int q = 0; q < 8; ++q)
           atomicAdd(dst + q, make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]));
+      } else if (kind == OUT_HILO) {
+        __nv_bfloat16* b = static_cast<__nv_bfloat16*>(out) + o;
+        store_hilo_x32(b, b + lo_off, v);
       } else {
-        __align__(16) __nv_bfloat16 hi[32];
-        __align__(16) __nv_bfloat16 lo[32];
-#pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          if (kind == OUT_HILO)
-            split_hilo(v[e], hi[e], lo[e]);
-          else
-            hi[e] = __float2bfloat16_rn(v[e]);
-        }
-        uint4* dh = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(out) + o);
-#pragma unroll
-        for (int q = 0; q < 4; ++q) dh[q] = reinterpret_cast<const uint4*>(hi)[q];
-        if (kind == OUT_HILO) {
-          uint4* dl = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(out) + o + lo_off);
-#pragma unroll
-          for (int q = 0; q < 4; ++q) dl[q] = reinterpret_cast<const uint4*>(lo)[q];
-        }
+        store_bf16x32(static_cast<__nv_bfloat16*>(out) + o, v);
       }
       return;
     }
-#pragma unroll 4
+#pragma unroll
     for (int e = 0; e < 32; ++e) {
       const int c = c0 + e;
       if (c >= p.N) break;
@@ -230,30 +254,25 @@ struct EpiRopeC {
       tmem_ld32(taddr + (uint32_t)u, a);
       tmem_ld32(taddr + (uint32_t)(128 + u), bb);
       if (!rvalid) continue;
-      __align__(16) __nv_bfloat16 ah[32], al[32], bh[32], bl[32];
       const float2* crow = coarse + (int64_t)g * (D / 2) + m_base + u;
-#pragma unroll 8
+      const float* om = omega + m_base + u;
+      const float* bia = bias + c_tile + u;
+#pragma unroll
       for (int e = 0; e < 32; ++e) {
-        const int m = m_base + u + e;
-        const float x = a[e] + bias[c_tile + u + e];
-        const float y = bb[e] + bias[c_tile + 128 + u + e];
+        const float x = a[e] + bia[e];
+        const float y = bb[e] + bia[128 + e];
         ss += x * x + y * y;
         float sf, cf;
-        __sincosf(delta * omega[m], &sf, &cf);
+        __sincosf(delta * om[e], &sf, &cf);
         const float2 cs = crow[e];
         const float cw = cs.x * cf - cs.y * sf;  // cos(G w + delta w)
         const float sw = cs.y * cf + cs.x * sf;  // sin(G w + delta w)
-        split_hilo(x * cw - y * sw, ah[e], al[e]);
-        split_hilo(x * sw + y * cw, bh[e], bl[e]);
+        a[e] = x * cw - y * sw;
+        bb[e] = x * sw + y * cw;
       }
       __nv_bfloat16* o = out + row_out + f_tile + u;
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        reinterpret_cast<uint4*>(o)[q] = reinterpret_cast<const uint4*>(ah)[q];
-        reinterpret_cast<uint4*>(o + 128)[q] = reinterpret_cast<const uint4*>(bh)[q];
-        reinterpret_cast<uint4*>(o + D)[q] = reinterpret_cast<const uint4*>(al)[q];
-        reinterpret_cast<uint4*>(o + D + 128)[q] = reinterpret_cast<const uint4*>(bl)[q];
-      }
+      store_hilo_x32(o, o + D, a);
+      store_hilo_x32(o + 128, o + D + 128, bb);
     }
     if (rvalid) atomicAdd(&sumsq[(int64_t)(tc.b * nheads + head) * Ntok + r], ss);
   }
@@ -261,12 +280,12 @@ struct EpiRopeC {
 
 // Output heads: columns [0, d) = Z_out W_key, re-rotated by the base RoPE at the output
 // position of latent j; columns [d, 2d) = Z_out W_val. Rows r = h * t + j. bf16 stores into
-// the caller's C_k / C_v with element strides (st, sh, sd). omega = theta^(-2m/d) in fp64;
+// the caller's C_k / C_v with element strides (st, sh). omega = theta^(-2m/d) in fp64;
 // the angle is reduced modulo 2 pi in fp64 before the fp32 sin/cos.
 struct EpiHeads {
   __nv_bfloat16* ck = nullptr;
   __nv_bfloat16* cv = nullptr;
-  int64_t st = 0, sh = 0, sd = 1;
+  int64_t st = 0, sh = 0;  // element strides of [t, H, d]; d is contiguous, rows 16-B aligned
   int32_t t = 0, d = 0;
   double pstart = 0, pstep = 0;
   const double* omega = nullptr;  // [d/2]
@@ -292,28 +311,25 @@ struct EpiHeads {
         tmem_ld32(taddr + (uint32_t)cc, a);
         tmem_ld32(taddr + (uint32_t)(cc + hd), b);
         if (!rvalid) continue;
-#pragma unroll 4
+#pragma unroll
         for (int e = 0; e < 32; ++e) {
-          const int m = c0 + e;
           float cw = 1.f, sw = 0.f;
           if (rope) {
-            double ang = pos * omega[m];
+            double ang = pos * omega[c0 + e];
             ang -= 6.283185307179586 * rint(ang * 0.15915494309189535);
             sincosf((float)ang, &sw, &cw);
           }
           const float x = a[e], y = b[e];
-          ck[obase + (int64_t)m * sd] = __float2bfloat16_rn(x * cw - y * sw);
-          ck[obase + (int64_t)(m + hd) * sd] = __float2bfloat16_rn(x * sw + y * cw);
+          a[e] = x * cw - y * sw;
+          b[e] = x * sw + y * cw;
         }
+        store_bf16x32(ck + obase + c0, a);
+        store_bf16x32(ck + obase + c0 + hd, b);
       } else {
         float v[32];
         tmem_ld32(taddr + (uint32_t)cc, v);
         if (!rvalid) continue;
-#pragma unroll 4
-        for (int e = 0; e < 32; ++e) {
-          const int f = c0 + e - d;
-          if (f < d) cv[obase + (int64_t)f * sd] = __float2bfloat16_rn(v[e]);
-        }
+        store_bf16x32(cv + obase + (c0 - d), v);
       }
     }
   }

@@ -707,7 +707,6 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
     e.cv = out.cv;
     e.st = out.st;
     e.sh = out.sh;
-    e.sd = 1;
     e.t = t;
     e.d = d;
     e.pstart = qstart;
@@ -939,8 +938,8 @@ still_status still_compact_layer(still_ctx* ctx, int32_t layer, const void* K, c
   if (N < 1 || t < 1 || t > N || t > L->cfg.t_max || N > (int64_t(1) << 30))
     return STILL_ERR_SHAPE;
   if (strides_kv[2] != 1 || strides_kv[0] < 1 || strides_kv[1] < 0) return STILL_ERR_SHAPE;
-  if ((reinterpret_cast<uintptr_t>(K) | reinterpret_cast<uintptr_t>(V) |
-       reinterpret_cast<uintptr_t>(Ck) | reinterpret_cast<uintptr_t>(Cv)) & 1)
+  if (((reinterpret_cast<uintptr_t>(K) | reinterpret_cast<uintptr_t>(V)) & 1) ||
+      ((reinterpret_cast<uintptr_t>(Ck) | reinterpret_cast<uintptr_t>(Cv)) & 15))
     return STILL_ERR_ALIGNMENT;
   Positions pos;
   TRY(make_positions(h_segments, n_segments, N, pos));
