@@ -206,6 +206,7 @@ typedef enum {
   STILL_K_FFN1,         /* GELU(x W_1)                                      */
   STILL_K_FFN2,         /* (.) W_2 + residual                               */
   STILL_K_HEADS,        /* C_k, C_v output heads + re-rotation              */
+  STILL_K_NORMS,        /* QK-norm factors from sum-of-squares partials     */
   STILL_K_LOAD,         /* weight-load precompute GEMMs                     */
   STILL_K_COUNT
 } still_kernel_class;

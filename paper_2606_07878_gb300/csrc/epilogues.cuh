@@ -19,7 +19,7 @@ struct AffineMap {
   }
 };
 
-enum OutKind : int32_t { OUT_F32 = 0, OUT_BF16 = 1, OUT_HILO = 2, OUT_F32_ATOMIC = 3 };
+enum OutKind : int32_t { OUT_F32 = 0, OUT_BF16 = 1, OUT_HILO = 2 };
 
 __device__ __forceinline__ void split_hilo(float x, __nv_bfloat16& hi, __nv_bfloat16& lo) {
   hi = __float2bfloat16_rn(x);
@@ -68,10 +68,15 @@ __device__ __forceinline__ void store_hilo_x32(__nv_bfloat16* dh, __nv_bfloat16*
 }
 
 // General epilogue: v = acc * alpha [* colscale(c)] [* rowscale(r)] [+ bias(c)]
-//   -> [sumsq accumulation] -> [GELU] -> [+ residual] -> store (f32 / bf16 / hi-lo / atomic f32)
-// colscale / rowscale = 1 / max(sqrt(sumsq[idx]), eps) from a sum-of-squares buffer.
+//   -> [sum-of-squares partial] -> [GELU] -> [+ residual (split 0)] -> store (f32/bf16/hi-lo)
+// colscale / rowscale are read from vectors of ready factors (see launch_inv_norms).
+// Sums of squares are written as partials, never accumulated atomically, so that results do
+// not depend on scheduling: per (vector, tile, half-warp) one slot, ss_parts slots per vector.
+// Split-K partial results go to out + split * split_stride and are reduced in a fixed order by
+// the consumer.
 // Host contract: csm, resm and (when vec_ok) om are contiguous in c (c0 == 1) with cdiv a
-// multiple of 32, so every 32-column chunk maps to 32 consecutive elements; ss_seg % 32 == 0.
+// multiple of 32, so every 32-column chunk maps to 32 consecutive elements; ss_seg is a
+// multiple of the tile width.
 struct EpiAffine {
   int32_t kind = OUT_F32;
   void* out = nullptr;
@@ -79,18 +84,19 @@ struct EpiAffine {
   AffineMap om;
   float alpha = 1.f;
   const float* bias = nullptr;  // indexed by column
-  const float* col_ss = nullptr;
+  const float* col_scale = nullptr;
   AffineMap csm;  // (b, 0, c) -> index
-  const float* row_ss = nullptr;
+  const float* row_scale = nullptr;
   AffineMap rsm;  // (b, r, 0) -> index
-  float eps = 1e-12f;
   int32_t gelu = 0;
   int32_t res_kind = 0;  // 0 none, 1 f32, 2 bf16
   const void* res = nullptr;
   AffineMap resm;
-  float* sumsq = nullptr;  // accumulate sum_c v^2 over segments of ss_seg columns
-  AffineMap ssm;           // (b, r, c / ss_seg) -> index
+  float* sumsq = nullptr;  // partial sums of v^2 over segments of ss_seg columns
+  AffineMap ssm;           // (b, r, c / ss_seg) -> vector index
   int32_t ss_seg = 1 << 30;
+  int32_t ss_parts = 2;    // slots per vector = 2 * ss_seg / tile width
+  int64_t split_stride = 0;
   int32_t vec_ok = 0;  // host: om.c0 == 1, cdiv % 32 == 0, 16-B aligned rows
   int32_t tile_cols_ = 256;  // the tile width BN, set by the launcher
 
@@ -98,11 +104,9 @@ struct EpiAffine {
                              int half) const {
     const int r = tc.tm * kBM + row;
     const bool rvalid = r < p.M;
-    const float eps2 = eps * eps;
     float rscale = alpha;
-    if (row_ss != nullptr && rvalid) rscale *= rsqrtf(fmaxf(row_ss[rsm.at(tc.b, r, 0)], eps2));
+    if (row_scale != nullptr && rvalid) rscale *= row_scale[rsm.at(tc.b, r, 0)];
     float ss = 0.f;
-    int ss_cur = -1;
     for (int cc = 32 * half; cc < tile_cols_; cc += 64) {
       float v[32];
       tmem_ld32(taddr + (uint32_t)cc, v);
@@ -111,11 +115,11 @@ struct EpiAffine {
       const int nv = min(32, p.N - c0);
 #pragma unroll
       for (int e = 0; e < 32; ++e) v[e] *= rscale;
-      if (col_ss != nullptr) {
-        const float* cs = col_ss + csm.at(tc.b, 0, c0);
+      if (col_scale != nullptr) {
+        const float* cs = col_scale + csm.at(tc.b, 0, c0);
 #pragma unroll
         for (int e = 0; e < 32; ++e)
-          if (e < nv) v[e] *= rsqrtf(fmaxf(cs[e], eps2));
+          if (e < nv) v[e] *= cs[e];
       }
       if (bias != nullptr) {
 #pragma unroll
@@ -123,12 +127,6 @@ struct EpiAffine {
           if (e < nv) v[e] += bias[c0 + e];
       }
       if (sumsq != nullptr) {
-        const int seg = c0 / ss_seg;
-        if (seg != ss_cur) {
-          if (ss_cur >= 0) atomicAdd(&sumsq[ssm.at(tc.b, r, ss_cur)], ss);
-          ss = 0.f;
-          ss_cur = seg;
-        }
 #pragma unroll
         for (int e = 0; e < 32; ++e)
           if (e < nv) ss += v[e] * v[e];
@@ -137,7 +135,7 @@ struct EpiAffine {
 #pragma unroll
         for (int e = 0; e < 32; ++e) v[e] = gelu_erf(v[e]);
       }
-      if (res_kind != 0 && (kind != OUT_F32_ATOMIC || tc.split == 0)) {
+      if (res_kind != 0 && tc.split == 0) {
         const int64_t o = resm.at(tc.b, r, c0);
         if (res_kind == 1) {
           const float* rp = static_cast<const float*>(res) + o;
@@ -151,26 +149,26 @@ struct EpiAffine {
             if (e < nv) v[e] += __bfloat162float(rp[e]);
         }
       }
-      store32(p, tc.b, r, c0, v);
+      store32(p, tc.b, r, c0, v, tc.split);
     }
-    if (sumsq != nullptr && rvalid && ss_cur >= 0) atomicAdd(&sumsq[ssm.at(tc.b, r, ss_cur)], ss);
+    if (sumsq != nullptr && rvalid) {
+      const int c_tile = tc.tn * tile_cols_;
+      const int slot = ((c_tile % ss_seg) / tile_cols_) * 2 + half;
+      sumsq[ssm.at(tc.b, r, c_tile / ss_seg) * ss_parts + slot] = ss;
+    }
   }
 
   __device__ __forceinline__ void store32(const GemmParams& p, int b, int r, int c0,
-                                          const float (&v)[32]) const {
+                                          const float (&v)[32], int split) const {
     const bool full = vec_ok && (c0 + 32 <= p.N);
+    const int64_t so = (int64_t)split * split_stride;
     if (full) {
-      const int64_t o = om.at(b, r, c0);
+      const int64_t o = om.at(b, r, c0) + so;
       if (kind == OUT_F32) {
         float4* dst = reinterpret_cast<float4*>(static_cast<float*>(out) + o);
 #pragma unroll
         for (int q = 0; q < 8; ++q)
           dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-      } else if (kind == OUT_F32_ATOMIC) {
-        float4* dst = reinterpret_cast<float4*>(static_cast<float*>(out) + o);
-#pragma unroll
-        for (int q = 0; q < 8; ++q)
-          atomicAdd(dst + q, make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]));
       } else if (kind == OUT_HILO) {
         __nv_bfloat16* b = static_cast<__nv_bfloat16*>(out) + o;
         store_hilo_x32(b, b + lo_off, v);
@@ -183,11 +181,9 @@ struct EpiAffine {
     for (int e = 0; e < 32; ++e) {
       const int c = c0 + e;
       if (c >= p.N) break;
-      const int64_t o = om.at(b, r, c);
+      const int64_t o = om.at(b, r, c) + so;
       if (kind == OUT_F32) {
         static_cast<float*>(out)[o] = v[e];
-      } else if (kind == OUT_F32_ATOMIC) {
-        atomicAdd(static_cast<float*>(out) + o, v[e]);
       } else if (kind == OUT_BF16) {
         static_cast<__nv_bfloat16*>(out)[o] = __float2bfloat16_rn(v[e]);
       } else {
@@ -225,7 +221,7 @@ constexpr int kPosGrain = 32;
 
 struct EpiRopeC {
   __nv_bfloat16* out = nullptr;  // [H][n][N][2D]: hi at [0, D), lo at [D, 2D)
-  float* sumsq = nullptr;        // [H][n][N]
+  float* sumsq = nullptr;        // [H][n][N][2 * D / 256] partial sums of |k~|^2
   const float* bias = nullptr;   // [n*D], pair-chunk order
   const float2* coarse = nullptr;  // [G][D/2]: (cos, sin)(G_g * omega_m)
   const float* omega = nullptr;    // [D/2] fp32
@@ -274,7 +270,10 @@ struct EpiRopeC {
       store_hilo_x32(o, o + D, a);
       store_hilo_x32(o + 128, o + D + 128, bb);
     }
-    if (rvalid) atomicAdd(&sumsq[(int64_t)(tc.b * nheads + head) * Ntok + r], ss);
+    if (rvalid) {
+      const int parts = 2 * (D / 256);
+      sumsq[((int64_t)(tc.b * nheads + head) * Ntok + r) * parts + (f_tile / 256) * 2 + half] = ss;
+    }
   }
 };
 

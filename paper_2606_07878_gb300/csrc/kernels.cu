@@ -272,18 +272,21 @@ __global__ void omega_kernel(double* out, int half, int width, double base) {
   if (m < half) out[m] = pow(base, -2.0 * m / width);
 }
 
-__global__ void px_to_hilo_kernel(const float* __restrict__ O, int b0, int nb, int n, int t,
-                                  int d2, __nv_bfloat16* __restrict__ PX) {
+__global__ void px_to_hilo_kernel(const float* __restrict__ O, int nsplit, int64_t split_stride,
+                                  int b0, int nb, int n, int t, int d2,
+                                  __nv_bfloat16* __restrict__ PX) {
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t total = (int64_t)nb * t * d2;
   if (idx >= total) return;
+  float o = O[idx];
+  for (int k = 1; k < nsplit; ++k) o += O[k * split_stride + idx];  // fixed order
   const int f = (int)(idx % d2);
   const int64_t rj = idx / d2;
   const int j = (int)(rj % t), bb = (int)(rj / t);
   const int b = b0 + bb, h = b / n, i = b % n;
   const int64_t ld = 2 * (int64_t)n * d2;
   __nv_bfloat16 hi, lo;
-  split_hilo(O[idx], hi, lo);
+  split_hilo(o, hi, lo);
   __nv_bfloat16* row = PX + ((int64_t)h * t + j) * ld;
   row[i * d2 + f] = hi;
   row[(int64_t)n * d2 + i * d2 + f] = lo;
@@ -321,10 +324,20 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const void* __restrict__ i
   }
 }
 
-__global__ void l2_scale_kernel(float* x, const float* ss, int64_t rows, int D, float eps) {
+__global__ void scale_rows_kernel(float* x, const float* inv, int64_t rows, int D) {
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= rows * D) return;
-  x[idx] *= 1.f / fmaxf(sqrtf(ss[idx / D]), eps);
+  x[idx] *= inv[idx / D];
+}
+
+__global__ void inv_norms_kernel(const float* __restrict__ parts, int64_t nvec, int nparts,
+                                 float eps, float alpha, float* __restrict__ out) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= nvec) return;
+  const float* p = parts + i * nparts;
+  float s = 0.f;
+  for (int k = 0; k < nparts; ++k) s += p[k];  // fixed order
+  out[i] = alpha / fmaxf(sqrtf(s), eps);
 }
 
 __global__ void transpose_kernel(const __nv_bfloat16* __restrict__ in, int64_t R, int64_t C,
@@ -429,10 +442,11 @@ cudaError_t launch_softmax(const float* S, int64_t rows, int64_t ncols, int64_t 
   return cudaGetLastError();
 }
 
-cudaError_t launch_px_to_hilo(const float* O, int b0, int nb, int n, int t, int d2,
-                              __nv_bfloat16* PX, cudaStream_t s) {
+cudaError_t launch_px_to_hilo(const float* O, int nsplit, int64_t split_stride, int b0, int nb,
+                              int n, int t, int d2, __nv_bfloat16* PX, cudaStream_t s) {
   const int64_t total = (int64_t)nb * t * d2;
-  px_to_hilo_kernel<<<blocks_for(total, 256), 256, 0, s>>>(O, b0, nb, n, t, d2, PX);
+  px_to_hilo_kernel<<<blocks_for(total, 256), 256, 0, s>>>(O, nsplit, split_stride, b0, nb, n,
+                                                           t, d2, PX);
   return cudaGetLastError();
 }
 
@@ -443,9 +457,14 @@ cudaError_t launch_rmsnorm(const void* in, int in_bf16, int64_t rows, int D, int
   return cudaGetLastError();
 }
 
-cudaError_t launch_l2_scale(float* x, const float* ss, int64_t rows, int D, float eps,
-                            cudaStream_t s) {
-  l2_scale_kernel<<<blocks_for(rows * D, 256), 256, 0, s>>>(x, ss, rows, D, eps);
+cudaError_t launch_scale_rows(float* x, const float* inv, int64_t rows, int D, cudaStream_t s) {
+  scale_rows_kernel<<<blocks_for(rows * D, 256), 256, 0, s>>>(x, inv, rows, D);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_inv_norms(const float* parts, int64_t nvec, int nparts, float eps,
+                             float alpha, float* out, cudaStream_t s) {
+  inv_norms_kernel<<<blocks_for(nvec, 256), 256, 0, s>>>(parts, nvec, nparts, eps, alpha, out);
   return cudaGetLastError();
 }
 

@@ -36,19 +36,24 @@ cudaError_t launch_omega(double* out, int half, int width, double base, cudaStre
 cudaError_t launch_softmax(const float* S, int64_t rows, int64_t ncols, int64_t ldS, void* P,
                            int64_t ldP, int out_fp16, cudaStream_t s);
 
-// Cross-attention head outputs O [nb][t][2d] fp32 (batch b = b0 + local) -> hi/lo bf16 rows
-// of PXcat [H*t][2 * n * 2d]: row h*t + j, columns i*2d + f (hi) and n*2d + i*2d + f (lo).
-cudaError_t launch_px_to_hilo(const float* O, int b0, int nb, int n, int t, int d2,
-                              __nv_bfloat16* PX, cudaStream_t s);
+// Cross-attention head outputs O [nsplit][nb][t][2d] fp32 split-K partials (batch b = b0 +
+// local), summed in split order -> hi/lo bf16 rows of PXcat [H*t][2 * n * 2d]: row h*t + j,
+// columns i*2d + f (hi) and n*2d + i*2d + f (lo).
+cudaError_t launch_px_to_hilo(const float* O, int nsplit, int64_t split_stride, int b0, int nb,
+                              int n, int t, int d2, __nv_bfloat16* PX, cudaStream_t s);
+
+// out[i] = alpha / max(sqrt(sum_k parts[i * nparts + k]), eps), summed in slot order: the
+// L2 / QK-norm factor of vector i from the epilogues' sum-of-squares partials.
+cudaError_t launch_inv_norms(const float* parts, int64_t nvec, int nparts, float eps,
+                             float alpha, float* out, cudaStream_t s);
 
 // Non-parametric RMSNorm over rows of width D: out = x / sqrt(mean(x^2) + eps) as bf16 hi
 // (and lo at +D when hilo), row pitch ldo. Input fp32 or bf16 (in_bf16), row pitch ldi.
 cudaError_t launch_rmsnorm(const void* in, int in_bf16, int64_t rows, int D, int64_t ldi,
                            float eps, __nv_bfloat16* out, int64_t ldo, int hilo, cudaStream_t s);
 
-// x[row] *= 1 / max(sqrt(ss[row]), eps) for rows of width D (fp32, in place).
-cudaError_t launch_l2_scale(float* x, const float* ss, int64_t rows, int D, float eps,
-                            cudaStream_t s);
+// x[row] *= inv[row] for rows of width D (fp32, in place).
+cudaError_t launch_scale_rows(float* x, const float* inv, int64_t rows, int D, cudaStream_t s);
 
 // out[c][r] = in[r][src(c)] (bf16), in is [R][C] row-major; src(c) maps pair-chunk order
 // back to natural order inside blocks of D columns when perm_D > 0.

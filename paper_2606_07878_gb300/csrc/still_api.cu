@@ -137,6 +137,8 @@ namespace {
 
 inline int64_t rup(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
 
+constexpr int kMaxSplit = 8;  // split-K factor cap (partials are reduced in a fixed order)
+
 void free_layer(LayerW& L) {
   for (void* p : L.owned) cudaFree(p);
   L = LayerW();
@@ -277,14 +279,14 @@ bool make_plan(const still_layer_config& c, int64_t N, int t, double pmin, doubl
   P.oZ3 = take(H * T * D * 4);
   const size_t fixed = off;
   P.kb_b = a256(N * 2 * D * 2);
-  P.kss_b = a256(N * 4);
+  P.kss_b = a256(N * 4 * (2 * (D / 256) + 1));  // |k~|^2 partials + inverse norms
   P.q_b = a256(T * 2 * D * 2);
   P.S_b = a256(T * P.ldS * 4);
   P.P_b = a256(T * P.Np * 2);
-  P.O_b = a256(T * 2 * d * 4);
+  P.O_b = a256(T * 2 * d * 4) * kMaxSplit;       // split-K partials of P X
   P.ca_unit_bytes = P.kb_b + P.kss_b + P.q_b + P.S_b + P.P_b + P.O_b;
   P.qk_b = a256(2 * n * T * 2 * D * 2);
-  P.sss_b = a256(2 * n * T * 4);
+  P.sss_b = a256(2 * n * T * 4 * (2 * (D / 256) + 1));
   P.vT_b = a256(n * D * P.tp * 2);
   P.Ssa_b = a256(n * T * P.ldt * 4);
   P.Psa_b = a256(n * T * P.tp * 2);
@@ -426,7 +428,9 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
     uint8_t* g = ws + P.oCA;
     bf16* kb = reinterpret_cast<bf16*>(g);
     g += P.kb_b * nbl;
-    float* kss = reinterpret_cast<float*>(g);
+    const int kparts = 2 * (D / 256);
+    float* kss = reinterpret_cast<float*>(g);        // [nbl][N][kparts]
+    float* kinv = kss + (size_t)nbl * N * kparts;    // [nbl][N]
     g += P.kss_b * nbl;
     bf16* qhl = reinterpret_cast<bf16*>(g);
     g += P.q_b * nbl;
@@ -436,7 +440,6 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
     g += P.P_b * nbl;
     float* O = reinterpret_cast<float*>(g);
     // keyproj: rows = tokens of heads [h0, h0+nh), columns = cross heads [i0, i0+ni)
-    CK(cudaMemsetAsync(kss, 0, sizeof(float) * (size_t)nbl * N, s));
     {
       GemmParams p = gp((int)N, ni * D, nh, 1);
       p.a_r1 = N;
@@ -457,6 +460,8 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
       TRY(run_gemm(ctx, STILL_K_KEYPROJ, 256, op(X, (int64_t)H * N, 3 * d), op(L.WkT, (int64_t)n * D, 2 * d), p, e,
                    1, s));
     }
+    // scale / |k~_n| per key (the d_l logit scale folded in)
+    KLAUNCH(STILL_K_NORMS, launch_inv_norms(kss, (int64_t)nbl * N, kparts, c.l2_eps, scale, kinv, s));
     KLAUNCH(STILL_K_QROPE, launch_q_rope(L.qhat, c.t_max, b0, nbl, t, D, qstart, qstep, L.omega_c,
                      c.compactor_rope, qhl, s));
     {  // S = scale * q.k / |k~|
@@ -472,18 +477,17 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
       e.om.b1 = (int64_t)t * P.ldS;
       e.om.r0 = P.ldS;
       e.om.c0 = 1;
-      e.alpha = scale;
-      e.col_ss = kss;
+      e.col_scale = kinv;
       e.csm.b1 = N;
       e.csm.c0 = 1;
-      e.eps = c.l2_eps;
       e.vec_ok = 1;
       TRY(run_gemm(ctx, STILL_K_SCORES, 256, op(qhl, (int64_t)nbl * t, 2 * D), op(kb, (int64_t)nbl * N, 2 * D), p,
                    e, 1, s));
     }
     KLAUNCH(STILL_K_SOFTMAX, launch_softmax(S, (int64_t)nbl * t, N, P.ldS, Pm, Np, 1, s));
-    CK(cudaMemsetAsync(O, 0, sizeof(float) * (size_t)nbl * t * 2 * d, s));
-    {  // O = P X  (fp16 operands, X hi + X lo)
+    int px_split = 1;
+    const int64_t px_stride = (int64_t)nbl * t * 2 * d;
+    {  // O = P X  (fp16 operands, X hi + X lo), split-K partials reduced in order below
       GemmParams p = gp(t, 2 * d, nbl, ni);
       p.a_r1 = (int64_t)ni * t;
       p.a_r0 = t;
@@ -492,10 +496,13 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
       add_pass(p, 0, (int)Np, 0, h0 * 2 * d, (int)Np);
       const int bn = 2 * d <= 128 ? 128 : 256;
       const int64_t tiles = (int64_t)((t + 127) / 128) * ((2 * d + bn - 1) / bn) * nbl;
-      p.ksplit = auto_split(tiles, (int)(2 * Np / 64), ctx->nsm);
+      p.ksplit = std::min(auto_split(tiles, (int)(2 * Np / 64), ctx->nsm), kMaxSplit);
+      p.ksplit = std::min(p.ksplit, (int)(2 * Np / 64));
+      px_split = p.ksplit;
       EpiAffine e;
-      e.kind = OUT_F32_ATOMIC;
+      e.kind = OUT_F32;
       e.out = O;
+      e.split_stride = px_stride;
       e.om.bdiv = ni;
       e.om.b1 = (int64_t)ni * t * 2 * d;
       e.om.b0 = (int64_t)t * 2 * d;
@@ -505,7 +512,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
       TRY(run_gemm(ctx, STILL_K_PX, bn, op(Pm, (int64_t)nbl * t, Np), op(XT, (int64_t)H * 2 * d, 2 * Np), p,
                    e, 0, s));
     }
-    KLAUNCH(STILL_K_PXSPLIT, launch_px_to_hilo(O, b0, nbl, n, t, 2 * d, PX, s));
+    KLAUNCH(STILL_K_PXSPLIT, launch_px_to_hilo(O, px_split, px_stride, b0, nbl, n, t, 2 * d, PX, s));
     b0 += nbl;
   }
 
@@ -517,10 +524,8 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
     add_pass(p, 0, 0, 0, 0, n2d);
     add_pass(p, 0, n2d, 0, 0, n2d);
     add_pass(p, n2d, 0, 0, 0, n2d);
-    const int64_t tiles = ((rows + 127) / 128) * ((D + 255) / 256);
-    p.ksplit = auto_split(tiles, 3 * n2d / 64, ctx->nsm);
     EpiAffine e;
-    e.kind = p.ksplit > 1 ? OUT_F32_ATOMIC : OUT_F32;
+    e.kind = OUT_F32;
     e.out = Z1;
     e.om.r0 = D;
     e.om.c0 = 1;
@@ -531,7 +536,6 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
     e.resm.r0 = D;
     e.resm.c0 = 1;
     e.vec_ok = 1;
-    if (p.ksplit > 1) CK(cudaMemsetAsync(Z1, 0, sizeof(float) * rows * D, s));
     TRY(run_gemm(ctx, STILL_K_VO, 256, op(PX, rows, 2 * n2d), op(L.WvoT, D, 2 * n2d), p, e, 1, s));
   }
   KLAUNCH(STILL_K_NORM, launch_rmsnorm(Z1, 0, rows, D, D, c.rms_eps, A1, 2 * D, 1, s));
@@ -542,14 +546,15 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
     uint8_t* g = ws + P.oSA;
     bf16* qk = reinterpret_cast<bf16*>(g);
     g += P.qk_b * nh;
-    float* sss = reinterpret_cast<float*>(g);
+    const int sparts = 2 * (D / 256);
+    float* sss = reinterpret_cast<float*>(g);                 // [nh][2n][t][sparts]
+    float* sinv = sss + (size_t)nh * 2 * n * t * sparts;       // [nh][2n][t]
     g += P.sss_b * nh;
     bf16* vT = reinterpret_cast<bf16*>(g);
     g += P.vT_b * nh;
     float* Ssa = reinterpret_cast<float*>(g);
     g += P.Ssa_b * nh;
     bf16* Psa = reinterpret_cast<bf16*>(g);
-    CK(cudaMemsetAsync(sss, 0, sizeof(float) * (size_t)nh * 2 * n * t, s));
     // The P.v product reads v^T columns [t, tp) of each head against zero probabilities:
     // they must hold finite values, and the region is shared with the cross-attention phase.
     if (P.tp != t) CK(cudaMemsetAsync(vT, 0, P.vT_b * nh, s));
@@ -574,9 +579,12 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
       e.ssm.r0 = 1;
       e.ssm.c0 = t;
       e.ss_seg = D;
+      e.ss_parts = sparts;
       e.vec_ok = 1;
       TRY(run_gemm(ctx, STILL_K_SA_PROJ, 256, op(A1, rows, 2 * D), op(L.SqkT, (int64_t)2 * n * D, D), p, e, 1, s));
     }
+    KLAUNCH(STILL_K_NORMS,
+            launch_inv_norms(sss, (int64_t)nh * 2 * n * t, sparts, c.l2_eps, 1.f, sinv, s));
     {  // v^T = S_V^T RMSNorm(Z')^T  -> [nD][nh * tp]
       GemmParams p = gp(n * D, nh * t);
       add_pass(p, 0, 0, 0, h0 * t, D);
@@ -606,18 +614,17 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
       e.om.r0 = P.ldt;
       e.om.c0 = 1;
       e.alpha = scale;
-      e.row_ss = sss;
+      e.row_scale = sinv;
       e.rsm.bdiv = n;
       e.rsm.b1 = (int64_t)2 * n * t;
       e.rsm.b0 = t;
       e.rsm.r0 = 1;
-      e.col_ss = sss;
+      e.col_scale = sinv;
       e.csm.bdiv = n;
       e.csm.b1 = (int64_t)2 * n * t;
       e.csm.b0 = t;
       e.csm.c0 = 1;
       e.csm.k = (int64_t)n * t;
-      e.eps = c.l2_eps;
       e.vec_ok = 1;
       TRY(run_gemm(ctx, STILL_K_SA_SCORES, 256, op(qk, (int64_t)nh * 2 * n * t, 2 * D),
                    op(qk, (int64_t)nh * 2 * n * t, 2 * D), p, e, 1, s));
@@ -862,7 +869,7 @@ still_status still_load_layer_weights(still_ctx* ctx, int32_t layer,
       (st = dalloc(tmp, &Zn, (size_t)H * T * 2 * D)) != STILL_OK ||
       (st = dalloc(tmp, &WoT, (size_t)D * nD)) != STILL_OK ||
       (st = dalloc(tmp, &bq, (size_t)nD)) != STILL_OK ||
-      (st = dalloc(tmp, &qss, (size_t)H * n * T)) != STILL_OK) {
+      (st = dalloc(tmp, &qss, (size_t)H * n * T * (2 * (D / 256) + 1))) != STILL_OK) {
     cleanup();
     free_layer(L);
     return st;
@@ -871,7 +878,6 @@ still_status still_load_layer_weights(still_ctx* ctx, int32_t layer,
     CK(launch_transpose(Wq, D, nD, WqT, D, s));
     CK(launch_bias(static_cast<const bf16*>(w->bq), nullptr, nD, bq, D, s));
     CK(launch_rmsnorm(w->Z, 1, (int64_t)H * T, D, D, c.rms_eps, Zn, 2 * D, 1, s));
-    CK(cudaMemsetAsync(qss, 0, sizeof(float) * (size_t)H * n * T, s));
     {  // q~ = RMSNorm(Z) W_Q + b_Q  (2-pass), |q~|^2 per (row, head)
       GemmParams p = gp(H * T, (int)nD);
       add_pass(p, 0, 0, 0, 0, D);
@@ -892,10 +898,16 @@ still_status still_load_layer_weights(still_ctx* ctx, int32_t layer,
       e.ssm.r0 = 1;
       e.ssm.c0 = T;
       e.ss_seg = D;
+      e.ss_parts = 2 * (D / 256);
       e.vec_ok = 1;
       TRY(run_gemm(ctx, STILL_K_LOAD, 256, op(Zn, (int64_t)H * T, 2 * D), op(WqT, nD, D), p, e, 1, s));
     }
-    CK(launch_l2_scale(L.qhat, qss, (int64_t)H * n * T, D, c.l2_eps, s));
+    {
+      const int64_t nq = (int64_t)H * n * T;
+      float* qinv = qss + nq * (2 * (D / 256));
+      CK(launch_inv_norms(qss, nq, 2 * (D / 256), c.l2_eps, 1.f, qinv, s));
+      CK(launch_scale_rows(L.qhat, qinv, nq, D, s));
+    }
     // W_VO,i = W_V,i W_O,i  -> stored transposed as hi | lo: WvoT[c][i*2d + f]
     CK(launch_transpose(static_cast<const bf16*>(w->Wo), nD, D, WoT, 0, s));
     {
@@ -1078,7 +1090,7 @@ const char* still_kernel_class_name(int32_t cls) {
   static const char* names[STILL_K_COUNT] = {
       "strip", "rope_tables", "keyproj", "q_rope", "scores", "softmax", "px", "px_split",
       "vo", "rmsnorm", "sa_proj", "sa_v", "sa_scores", "sa_softmax", "sa_pv", "sa_out",
-      "ffn1", "ffn2", "heads", "load"};
+      "ffn1", "ffn2", "heads", "norms", "load"};
   return cls >= 0 && cls < STILL_K_COUNT ? names[cls] : "unknown";
 }
 

@@ -29,7 +29,7 @@ EXPORTS = [
 
 KERNEL_CLASSES = ["strip", "rope_tables", "keyproj", "q_rope", "scores", "softmax", "px",
                   "px_split", "vo", "rmsnorm", "sa_proj", "sa_v", "sa_scores", "sa_softmax",
-                  "sa_pv", "sa_out", "ffn1", "ffn2", "heads", "load"]
+                  "sa_pv", "sa_out", "ffn1", "ffn2", "heads", "norms", "load"]
 
 
 class StillError(RuntimeError):

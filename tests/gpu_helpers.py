@@ -1,4 +1,7 @@
 """Shared helpers for the GPU parity tests: run the library, compare with the oracle."""
+import json
+import os
+
 import numpy as np
 import torch
 
@@ -22,6 +25,12 @@ def metrics(ref: np.ndarray, got: np.ndarray):
 
 def assert_parity(ref, got, what=""):
     err, cos = metrics(ref, got)
+    log = os.environ.get("STILL_PARITY_LOG")
+    if log:
+        with open(log, "a") as f:
+            f.write(json.dumps({"test": os.environ.get("PYTEST_CURRENT_TEST", "").split(" ")[0],
+                                "what": what, "max_err_over_rms": err, "min_row_cos": cos})
+                    + "\n")
     assert np.all(np.isfinite(got)), f"{what}: non-finite output"
     assert err <= ERR_REL and cos >= COS_MIN, f"{what}: max|err|/RMS={err:.4e} min cos={cos:.6f}"
     return err, cos
