@@ -135,6 +135,37 @@ still_status still_compact_layer(still_ctx* ctx, int32_t layer, const void* K, c
                                  double* h_out_pos_start, double* h_out_pos_step,
                                  int64_t* h_pos_offset, void* stream);
 
+/* Size of the fixed device scratch behind still_compact_layer_noalloc, in MiB. */
+#define STILL_NOALLOC_SCRATCH_MIB 64
+
+/* Same computation, arguments and results as still_compact_layer, for callers that cannot
+ * allocate device memory at call time: a serving engine that has handed all free HBM to its
+ * own pool (a cudaMalloc would fail or steal from it), a latency-critical loop that must not
+ * hit cudaMalloc/cudaFree's implicit device synchronisation, or code running where the CUDA
+ * allocator may not be entered. The paper has no counterpart: this is a deployment variant.
+ *
+ * It allocates nothing: the intermediate buffers live in one file-scope device array of
+ * STILL_NOALLOC_SCRATCH_MIB MiB compiled into the library, which every GPU that loads the
+ * library holds until the process exits. Weights must already be loaded (that call does
+ * allocate). Sizes whose workspace cannot fit in the array even when the KV-heads are
+ * processed in small groups are rejected with STILL_ERR_OOM before anything is launched
+ * (the tiny 1k-token workload fits; an 8k-token, d_l = 1024 layer does not).
+ *
+ * The first call on each device looks up the array's device address (cudaGetSymbolAddress,
+ * with that device current) and caches it; make that first call before any stream capture.
+ * Every call, from every context on the device, shares the one array and leaves its last
+ * contents there; the path clears what it needs zeroed on each call. Calls whose execution
+ * overlaps on the GPU (different streams, or concurrent host threads) race on the array:
+ * serialise them. Kernel event timing (still_profile_enable) is suspended inside this call;
+ * launch counts are still recorded. */
+still_status still_compact_layer_noalloc(still_ctx* ctx, int32_t layer, const void* K,
+                                         const void* V, const int64_t strides_kv[3],
+                                         const still_pos_segment* h_segments,
+                                         int32_t n_segments, int64_t N, int32_t t, void* Ck,
+                                         void* Cv, double* h_out_pos_start,
+                                         double* h_out_pos_step, int64_t* h_pos_offset,
+                                         void* stream);
+
 /* Compacts layers 0..n_layers-1 (all loaded) over the same positions: the per-layer
  * compactors share nothing at forward time (App. M, "No inter-layer compactor channel"), so
  * this is one stream-ordered launch sequence over the layer stack. K[l], V[l], Ck[l], Cv[l] are device

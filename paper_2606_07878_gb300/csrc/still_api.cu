@@ -17,6 +17,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <mutex>
 #include <vector>
 
 #include "../../include/still.h"
@@ -381,14 +382,18 @@ struct OutSpec {
   int64_t st, sh;  // element strides of [t, H, d] outputs (d contiguous)
 };
 
+// ws_fixed / ws_fixed_bytes: when set, the call runs in that caller-provided scratch and never
+// touches the context's (growable) workspace.
 still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const bf16* V,
                          int64_t sN, int64_t sH, const Positions& pos, int64_t N, int t,
-                         const OutSpec& out, cudaStream_t s) {
+                         const OutSpec& out, cudaStream_t s, uint8_t* ws_fixed = nullptr,
+                         size_t ws_fixed_bytes = 0) {
   const still_layer_config& c = L.cfg;
   Plan P;
-  if (!make_plan(c, N, t, pos.pmin, pos.pmax, ctx->ws_limit, P)) return STILL_ERR_OOM;
-  TRY(ensure_ws(ctx, P.total));
-  uint8_t* ws = static_cast<uint8_t*>(ctx->ws);
+  const size_t limit = ws_fixed != nullptr ? ws_fixed_bytes : ctx->ws_limit;
+  if (!make_plan(c, N, t, pos.pmin, pos.pmax, limit, P)) return STILL_ERR_OOM;
+  if (ws_fixed == nullptr) TRY(ensure_ws(ctx, P.total));
+  uint8_t* ws = ws_fixed != nullptr ? ws_fixed : static_cast<uint8_t*>(ctx->ws);
   const int H = P.H, d = P.d, D = P.D, n = P.n, F = P.F;
   const int64_t Np = P.Np;
   const float scale = c.logit_scale > 0 ? (float)c.logit_scale : (float)D;
@@ -736,6 +741,38 @@ still_status check_ctx_layer(still_ctx* ctx, int32_t layer, const LayerW** L) {
 
 }  // namespace
 
+// ============================================================================== fixed scratch
+
+// Scratch of still_compact_layer_noalloc: a file-scope device array, so that the entry point
+// never allocates. Every device that loads this library holds it until the process exits.
+constexpr size_t kNoAllocScratchBytes = size_t(STILL_NOALLOC_SCRATCH_MIB) << 20;
+static __device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocScratchBytes];
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+uint8_t* g_noalloc_ptr[kMaxDevices] = {nullptr};
+
+// Device address of the scratch array on `device` (which must be current). The host-side name
+// g_noalloc_scratch is only a stand-in symbol: kernels must be given this address instead.
+still_status noalloc_scratch(int device, uint8_t** out) {
+  if (device < 0 || device >= kMaxDevices) return STILL_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lk(g_noalloc_mu);
+  if (g_noalloc_ptr[device] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) {
+      cudaGetLastError();
+      return STILL_ERR_CUDA;
+    }
+    g_noalloc_ptr[device] = static_cast<uint8_t*>(p);
+  }
+  *out = g_noalloc_ptr[device];
+  return STILL_OK;
+}
+
+}  // namespace
+
 // ============================================================================== C ABI
 
 extern "C" {
@@ -961,6 +998,48 @@ still_status still_compact_layer(still_ctx* ctx, int32_t layer, const void* K, c
   TRY(compact_one(ctx, *L, static_cast<const bf16*>(K), static_cast<const bf16*>(V),
                   strides_kv[0], strides_kv[1], pos, N, t, o,
                   static_cast<cudaStream_t>(stream)));
+  if (h_out_pos_start) *h_out_pos_start = pos.pmin;
+  if (h_out_pos_step) *h_out_pos_step = t > 1 ? (pos.pmax - pos.pmin) / (double)(t - 1) : 0.0;
+  if (h_pos_offset) *h_pos_offset = N - t;
+  return STILL_OK;
+}
+
+still_status still_compact_layer_noalloc(still_ctx* ctx, int32_t layer, const void* K,
+                                         const void* V, const int64_t strides_kv[3],
+                                         const still_pos_segment* h_segments,
+                                         int32_t n_segments, int64_t N, int32_t t, void* Ck,
+                                         void* Cv, double* h_out_pos_start,
+                                         double* h_out_pos_step, int64_t* h_pos_offset,
+                                         void* stream) {
+  const LayerW* L = nullptr;
+  TRY(check_ctx_layer(ctx, layer, &L));
+  if (K == nullptr || V == nullptr || Ck == nullptr || Cv == nullptr || strides_kv == nullptr)
+    return STILL_ERR_INVALID_ARG;
+  if (N < 1 || t < 1 || t > N || t > L->cfg.t_max || N > (int64_t(1) << 30))
+    return STILL_ERR_SHAPE;
+  if (strides_kv[2] != 1 || strides_kv[0] < 1 || strides_kv[1] < 0) return STILL_ERR_SHAPE;
+  if (((reinterpret_cast<uintptr_t>(K) | reinterpret_cast<uintptr_t>(V)) & 1) ||
+      ((reinterpret_cast<uintptr_t>(Ck) | reinterpret_cast<uintptr_t>(Cv)) & 15))
+    return STILL_ERR_ALIGNMENT;
+  Positions pos;
+  TRY(make_positions(h_segments, n_segments, N, pos));
+  CK(cudaSetDevice(ctx->device));
+  Plan P;
+  if (!make_plan(L->cfg, N, t, pos.pmin, pos.pmax, kNoAllocScratchBytes, P))
+    return STILL_ERR_OOM;  // even the smallest grouping needs more than the fixed scratch
+  uint8_t* scratch = nullptr;
+  TRY(noalloc_scratch(ctx->device, &scratch));
+  const int H = L->cfg.n_kv_heads, d = L->cfg.head_dim;
+  OutSpec o{static_cast<bf16*>(Ck), static_cast<bf16*>(Cv), (int64_t)H * d, d};
+  // Launch counting stays on; event timing (which creates CUDA events) is suspended.
+  const bool timing = ctx->prof.on;
+  ctx->prof.on = false;
+  const still_status st =
+      compact_one(ctx, *L, static_cast<const bf16*>(K), static_cast<const bf16*>(V),
+                  strides_kv[0], strides_kv[1], pos, N, t, o,
+                  static_cast<cudaStream_t>(stream), scratch, kNoAllocScratchBytes);
+  ctx->prof.on = timing;
+  TRY(st);
   if (h_out_pos_start) *h_out_pos_start = pos.pmin;
   if (h_out_pos_step) *h_out_pos_step = t > 1 ? (pos.pmax - pos.pmin) / (double)(t - 1) : 0.0;
   if (h_pos_offset) *h_pos_offset = N - t;

@@ -25,7 +25,10 @@ EXPORTS = [
     "still_compact_stack_ragged", "still_workspace_size", "still_set_workspace_limit",
     "still_get_device_status", "still_budget", "still_kv_bytes", "still_param_count",
     "still_profile_enable", "still_profile_read", "still_kernel_class_name",
+    "still_compact_layer_noalloc",
 ]
+
+NOALLOC_SCRATCH_MIB = 64  # STILL_NOALLOC_SCRATCH_MIB in include/still.h
 
 KERNEL_CLASSES = ["strip", "rope_tables", "keyproj", "q_rope", "scores", "softmax", "px",
                   "px_split", "vo", "rmsnorm", "sa_proj", "sa_v", "sa_scores", "sa_softmax",
@@ -85,6 +88,8 @@ def lib():
                                           ctypes.POINTER(LayerWeights), P], ctypes.c_int),
             "still_compact_layer": ([P, I32, P, P, PI64, PSEG, I32, I64, I32, P, P, PD, PD, PI64,
                                      P], ctypes.c_int),
+            "still_compact_layer_noalloc": ([P, I32, P, P, PI64, PSEG, I32, I64, I32, P, P, PD,
+                                             PD, PI64, P], ctypes.c_int),
             "still_compact_stack": ([P, I32, ctypes.POINTER(P), ctypes.POINTER(P), PI64, PSEG, I32,
                                      I64, I32, ctypes.POINTER(P), ctypes.POINTER(P), PD, PD, PI64,
                                      P], ctypes.c_int),
@@ -192,6 +197,22 @@ def still_compact_layer(ctx, layer: int, K, V, t: int, Ck, Cv, segments=None, st
                                      K.shape[0], t, _ptr(Ck), _ptr(Cv), ctypes.byref(ps),
                                      ctypes.byref(pst), ctypes.byref(off), _stream(stream)),
            "still_compact_layer")
+    return ps.value, pst.value, off.value
+
+
+def still_compact_layer_noalloc(ctx, layer: int, K, V, t: int, Ck, Cv, segments=None,
+                                stream=None):
+    """still_compact_layer without any device allocation (fixed library scratch); same
+    arguments and returns."""
+    strides = (ctypes.c_int64 * 3)(*K.stride())
+    assert tuple(V.stride()) == tuple(K.stride()), "K and V must share strides"
+    seg, nseg = _segments(segments)
+    ps, pst, off = ctypes.c_double(), ctypes.c_double(), ctypes.c_int64()
+    _check(lib().still_compact_layer_noalloc(ctx, layer, _ptr(K), _ptr(V), strides, seg, nseg,
+                                             K.shape[0], t, _ptr(Ck), _ptr(Cv),
+                                             ctypes.byref(ps), ctypes.byref(pst),
+                                             ctypes.byref(off), _stream(stream)),
+           "still_compact_layer_noalloc")
     return ps.value, pst.value, off.value
 
 
