@@ -201,6 +201,38 @@ still_status still_compact_stack_ragged(still_ctx* ctx, int32_t n_layers,
                                         const int64_t* h_cu_t, void* const* Ck,
                                         void* const* Cv, int64_t* h_pos_offset, void* stream);
 
+/* Iterative re-compaction (Sec. 2.3, iterative chunked compaction; here the fixed-ratio
+ * form that appends new tokens to each sequence's compact cache): for each of B sequences,
+ * the keys and values [previous compact cache | new tokens] are compacted again to
+ * t_b = round((L_prev,b + new_b) / ratio) slots (at least 1). Previous compact slots sit at
+ * their output positions, t_prev points evenly spaced over [0, L_prev - 1]; the new tokens
+ * at L_prev .. L_prev + new - 1; the new slots are evenly spaced over [0, L_prev + new - 1].
+ * The two parts are read in place (no concatenation copy).
+ *   Kprev, Vprev [sum t_prev, H, d] bf16: sequence b at rows [h_cu_prev[b], h_cu_prev[b+1])
+ *   h_prev_len[B] logical lengths already absorbed (>= t_prev)
+ *   Knew, Vnew   [sum new, H, d] bf16, h_cu_new[B+1] (new_b may be 0)
+ *   Ck, Cv       output [sum t_b, H, d] bf16, 16-byte aligned, disjoint from the inputs;
+ *                the caller sizes them with still_budget
+ *   h_cu_out[B+1] (out) row offsets of each sequence's new compact cache
+ *   h_len_out[B]  (out, optional) new logical lengths. */
+still_status still_recompact_layer_ragged(still_ctx* ctx, int32_t layer, int32_t B,
+                                          const void* Kprev, const void* Vprev,
+                                          const int64_t* h_cu_prev, const int64_t* h_prev_len,
+                                          const void* Knew, const void* Vnew,
+                                          const int64_t* h_cu_new, int64_t ratio, void* Ck,
+                                          void* Cv, int64_t* h_cu_out, int64_t* h_len_out,
+                                          void* stream);
+
+/* still_recompact_layer_ragged over layers 0..n_layers-1 (host arrays of per-layer device
+ * pointers; the offsets and lengths are shared by all layers). */
+still_status still_recompact_stack_ragged(still_ctx* ctx, int32_t n_layers, int32_t B,
+                                          const void* const* Kprev, const void* const* Vprev,
+                                          const int64_t* h_cu_prev, const int64_t* h_prev_len,
+                                          const void* const* Knew, const void* const* Vnew,
+                                          const int64_t* h_cu_new, int64_t ratio,
+                                          void* const* Ck, void* const* Cv, int64_t* h_cu_out,
+                                          int64_t* h_len_out, void* stream);
+
 /* Device workspace bytes a call with up to max_tokens tokens and compact length max_t needs
  * for layer 0's configuration (the context allocates it on demand and keeps it). */
 still_status still_workspace_size(const still_ctx* ctx, int64_t max_tokens, int32_t max_t,

@@ -44,27 +44,34 @@ __device__ __forceinline__ void split_pack(float a, float b, uint32_t& hi, uint3
   lo = *reinterpret_cast<const uint32_t*>(&l);
 }
 
-// 32 floats -> 32 bf16 (4 x uint4) at dst (16-byte aligned)
-__device__ __forceinline__ void store_bf16x32(__nv_bfloat16* dst, const float (&v)[32]) {
-  uint4* d = reinterpret_cast<uint4*>(dst);
+// 32 floats -> 32 bf16 packed in 4 x uint4
+__device__ __forceinline__ void pack_bf16x32(const float (&v)[32], uint4 (&o)[4]) {
 #pragma unroll
   for (int q = 0; q < 4; ++q)
-    d[q] = make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+    o[q] = make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
                       pack_bf16x2(v[8 * q + 4], v[8 * q + 5]),
                       pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
 }
 
-// 32 floats -> hi (4 x uint4) at dh and lo (4 x uint4) at dl
-__device__ __forceinline__ void store_hilo_x32(__nv_bfloat16* dh, __nv_bfloat16* dl,
-                                               const float (&v)[32]) {
+// 32 floats -> hi and lo bf16, each packed in 4 x uint4
+__device__ __forceinline__ void pack_hilo_x32(const float (&v)[32], uint4 (&h4)[4],
+                                              uint4 (&l4)[4]) {
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     uint32_t h[4], l[4];
 #pragma unroll
     for (int k = 0; k < 4; ++k) split_pack(v[8 * q + 2 * k], v[8 * q + 2 * k + 1], h[k], l[k]);
-    reinterpret_cast<uint4*>(dh)[q] = make_uint4(h[0], h[1], h[2], h[3]);
-    reinterpret_cast<uint4*>(dl)[q] = make_uint4(l[0], l[1], l[2], l[3]);
+    h4[q] = make_uint4(h[0], h[1], h[2], h[3]);
+    l4[q] = make_uint4(l[0], l[1], l[2], l[3]);
   }
+}
+
+// 16 floats -> 4 x uint4 (fp32 bits)
+__device__ __forceinline__ void pack_f32x16(const float* v, uint4 (&o)[4]) {
+#pragma unroll
+  for (int q = 0; q < 4; ++q)
+    o[q] = make_uint4(__float_as_uint(v[4 * q]), __float_as_uint(v[4 * q + 1]),
+                      __float_as_uint(v[4 * q + 2]), __float_as_uint(v[4 * q + 3]));
 }
 
 // General epilogue: v = acc * alpha [* colscale(c)] [* rowscale(r)] [+ bias(c)]
@@ -101,7 +108,7 @@ struct EpiAffine {
   int32_t tile_cols_ = 256;  // the tile width BN, set by the launcher
 
   __device__ void operator()(const GemmParams& p, const TileCoord& tc, int row, uint32_t taddr,
-                             int half) const {
+                             int half, uint4* stage) const {
     const int r = tc.tm * kBM + row;
     const bool rvalid = r < p.M;
     float rscale = alpha;
@@ -111,10 +118,14 @@ struct EpiAffine {
       float v[32];
       tmem_ld32(taddr + (uint32_t)cc, v);
       const int c0 = tc.tn * tile_cols_ + cc;
-      if (!rvalid || c0 >= p.N) continue;
+      if (c0 >= p.N) continue;  // uniform across the warp
       const int nv = min(32, p.N - c0);
 #pragma unroll
       for (int e = 0; e < 32; ++e) v[e] *= rscale;
+      if (!rvalid) {
+        store32(p, tc.b, r, c0, v, tc.split, false, stage);  // keeps the warp collective
+        continue;
+      }
       if (col_scale != nullptr) {
         const float* cs = col_scale + csm.at(tc.b, 0, c0);
 #pragma unroll
@@ -149,7 +160,7 @@ struct EpiAffine {
             if (e < nv) v[e] += __bfloat162float(rp[e]);
         }
       }
-      store32(p, tc.b, r, c0, v, tc.split);
+      store32(p, tc.b, r, c0, v, tc.split, rvalid, stage);
     }
     if (sumsq != nullptr && rvalid) {
       const int c_tile = tc.tn * tile_cols_;
@@ -158,25 +169,33 @@ struct EpiAffine {
     }
   }
 
+  // Warp-collective on the vector path (every lane calls it; invalid rows store nothing).
   __device__ __forceinline__ void store32(const GemmParams& p, int b, int r, int c0,
-                                          const float (&v)[32], int split) const {
-    const bool full = vec_ok && (c0 + 32 <= p.N);
+                                          const float (&v)[32], int split, bool rvalid,
+                                          uint4* stage) const {
+    const bool full = vec_ok && (c0 + 32 <= p.N);  // uniform across the warp
     const int64_t so = (int64_t)split * split_stride;
     if (full) {
-      const int64_t o = om.at(b, r, c0) + so;
+      const int64_t o = rvalid ? om.at(b, r, c0) + so : 0;
+      uint4 a4[4], b4[4];
       if (kind == OUT_F32) {
-        float4* dst = reinterpret_cast<float4*>(static_cast<float*>(out) + o);
-#pragma unroll
-        for (int q = 0; q < 8; ++q)
-          dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        float* dst = static_cast<float*>(out) + o;
+        pack_f32x16(v, a4);
+        pack_f32x16(v + 16, b4);
+        warp_store64(stage, a4, dst, rvalid);
+        warp_store64(stage, b4, dst + 16, rvalid);
       } else if (kind == OUT_HILO) {
-        __nv_bfloat16* b = static_cast<__nv_bfloat16*>(out) + o;
-        store_hilo_x32(b, b + lo_off, v);
+        __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(out) + o;
+        pack_hilo_x32(v, a4, b4);
+        warp_store64(stage, a4, dst, rvalid);
+        warp_store64(stage, b4, dst + lo_off, rvalid);
       } else {
-        store_bf16x32(static_cast<__nv_bfloat16*>(out) + o, v);
+        pack_bf16x32(v, a4);
+        warp_store64(stage, a4, static_cast<__nv_bfloat16*>(out) + o, rvalid);
       }
       return;
     }
+    if (!rvalid) return;
 #pragma unroll
     for (int e = 0; e < 32; ++e) {
       const int c = c0 + e;
@@ -232,7 +251,7 @@ struct EpiRopeC {
   int32_t tile_cols_ = 256;  // must be 256: a tile holds 128 whole RoPE pairs
 
   __device__ void operator()(const GemmParams& p, const TileCoord& tc, int row, uint32_t taddr,
-                             int half) const {
+                             int half, uint4* stage) const {
     const int r = tc.tm * kBM + row;
     const bool rvalid = r < p.M;
     const int c_tile = tc.tn * 256;
@@ -243,32 +262,49 @@ struct EpiRopeC {
     int g = (int)floor((pos - pmin) / (double)kPosGrain);
     g = max(0, min(g, ncoarse - 1));
     const float delta = (float)(pos - (pmin + (double)g * kPosGrain));
-    const int64_t row_out = ((int64_t)(tc.b * nheads + head) * Ntok + r) * (2 * (int64_t)D);
+    const int64_t row_out = ((int64_t)(tc.b * nheads + head) * Ntok + (rvalid ? r : 0)) *
+                            (2 * (int64_t)D);
     float ss = 0.f;
-    for (int u = 32 * half; u < 128; u += 64) {
+    // half 0 owns pairs [0, 64) of the tile, half 1 pairs [64, 128): 128-byte row segments
+    for (int u = 64 * half; u < 64 * half + 64; u += 32) {
       float a[32], bb[32];
       tmem_ld32(taddr + (uint32_t)u, a);
       tmem_ld32(taddr + (uint32_t)(128 + u), bb);
-      if (!rvalid) continue;
-      const float2* crow = coarse + (int64_t)g * (D / 2) + m_base + u;
-      const float* om = omega + m_base + u;
-      const float* bia = bias + c_tile + u;
+      const float4* crow = reinterpret_cast<const float4*>(coarse + (int64_t)g * (D / 2) + m_base + u);
+      const float4* om4 = reinterpret_cast<const float4*>(omega + m_base + u);
+      const float4* ba4 = reinterpret_cast<const float4*>(bias + c_tile + u);
+      const float4* bb4 = reinterpret_cast<const float4*>(bias + c_tile + 128 + u);
 #pragma unroll
-      for (int e = 0; e < 32; ++e) {
-        const float x = a[e] + bia[e];
-        const float y = bb[e] + bia[128 + e];
-        ss += x * x + y * y;
-        float sf, cf;
-        __sincosf(delta * om[e], &sf, &cf);
-        const float2 cs = crow[e];
-        const float cw = cs.x * cf - cs.y * sf;  // cos(G w + delta w)
-        const float sw = cs.y * cf + cs.x * sf;  // sin(G w + delta w)
-        a[e] = x * cw - y * sw;
-        bb[e] = x * sw + y * cw;
+      for (int e4 = 0; e4 < 8; ++e4) {
+        const float4 w = om4[e4], xa = ba4[e4], xb = bb4[e4];
+        const float4 c01 = crow[2 * e4], c23 = crow[2 * e4 + 1];
+        const float ws[4] = {w.x, w.y, w.z, w.w};
+        const float bas[4] = {xa.x, xa.y, xa.z, xa.w};
+        const float bbs[4] = {xb.x, xb.y, xb.z, xb.w};
+        const float cc[4] = {c01.x, c01.z, c23.x, c23.z};  // cos(G w) of the 4 pairs
+        const float sc[4] = {c01.y, c01.w, c23.y, c23.w};  // sin(G w)
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int e = 4 * e4 + k;
+          const float x = a[e] + bas[k];
+          const float y = bb[e] + bbs[k];
+          ss += x * x + y * y;
+          float sf, cf;
+          __sincosf(delta * ws[k], &sf, &cf);
+          const float cw = cc[k] * cf - sc[k] * sf;  // cos(G w + delta w)
+          const float sw = sc[k] * cf + cc[k] * sf;  // sin(G w + delta w)
+          a[e] = x * cw - y * sw;
+          bb[e] = x * sw + y * cw;
+        }
       }
       __nv_bfloat16* o = out + row_out + f_tile + u;
-      store_hilo_x32(o, o + D, a);
-      store_hilo_x32(o + 128, o + D + 128, bb);
+      uint4 h4[4], l4[4];
+      pack_hilo_x32(a, h4, l4);
+      warp_store64(stage, h4, o, rvalid);
+      warp_store64(stage, l4, o + D, rvalid);
+      pack_hilo_x32(bb, h4, l4);
+      warp_store64(stage, h4, o + 128, rvalid);
+      warp_store64(stage, l4, o + D + 128, rvalid);
     }
     if (rvalid) {
       const int parts = 2 * (D / 256);
@@ -292,10 +328,10 @@ struct EpiHeads {
   int32_t tile_cols_ = 256;
 
   __device__ void operator()(const GemmParams& p, const TileCoord& tc, int row, uint32_t taddr,
-                             int half) const {
+                             int half, uint4* stage) const {
     const int r = tc.tm * kBM + row;
     const bool rvalid = r < p.M;
-    const int h = r / t, j = r % t;
+    const int h = rvalid ? r / t : 0, j = rvalid ? r % t : 0;
     const int c_tile = tc.tn * tile_cols_;
     const double pos = pstart + (double)j * pstep;
     const int64_t obase = (int64_t)j * st + (int64_t)h * sh;
@@ -309,7 +345,6 @@ struct EpiHeads {
         float a[32], b[32];
         tmem_ld32(taddr + (uint32_t)cc, a);
         tmem_ld32(taddr + (uint32_t)(cc + hd), b);
-        if (!rvalid) continue;
 #pragma unroll
         for (int e = 0; e < 32; ++e) {
           float cw = 1.f, sw = 0.f;
@@ -322,13 +357,17 @@ struct EpiHeads {
           a[e] = x * cw - y * sw;
           b[e] = x * sw + y * cw;
         }
-        store_bf16x32(ck + obase + c0, a);
-        store_bf16x32(ck + obase + c0 + hd, b);
+        uint4 o4[4];
+        pack_bf16x32(a, o4);
+        warp_store64(stage, o4, ck + obase + c0, rvalid);
+        pack_bf16x32(b, o4);
+        warp_store64(stage, o4, ck + obase + c0 + hd, rvalid);
       } else {
         float v[32];
         tmem_ld32(taddr + (uint32_t)cc, v);
-        if (!rvalid) continue;
-        store_bf16x32(cv + obase + (c0 - d), v);
+        uint4 o4[4];
+        pack_bf16x32(v, o4);
+        warp_store64(stage, o4, cv + obase + (c0 - d), rvalid);
       }
     }
   }

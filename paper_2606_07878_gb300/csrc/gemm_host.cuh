@@ -70,7 +70,7 @@ inline bool finalize_gemm(GemmParams& p, int ab_fmt) {
   return true;
 }
 
-template <int BN, class Epi>
+template <int BN, int kRole, class Epi>
 inline cudaError_t launch_gemm(const Operand2D& A, const Operand2D& B, GemmParams p, Epi epi,
                                int ab_fmt, int num_sms, cudaStream_t stream) {
   using S = GemmSmem<BN>;
@@ -78,7 +78,7 @@ inline cudaError_t launch_gemm(const Operand2D& A, const Operand2D& B, GemmParam
   CUtensorMap ta, tb;
   if (!make_tmap(&ta, A, kBM) || !make_tmap(&tb, B, BN)) return cudaErrorInvalidValue;
   epi.tile_cols_ = BN;
-  auto kern = tc_gemm_kernel<BN, Epi>;
+  auto kern = tc_gemm_kernel<BN, Epi, kRole>;
   static thread_local bool attr_set = false;  // per instantiation
   if (!attr_set) {
     cudaError_t e =

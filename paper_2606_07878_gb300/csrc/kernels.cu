@@ -23,11 +23,15 @@ constexpr int kStripTok = 32;
 
 // One CTA = 32 tokens x one KV-head. Keys: inverse base-model RoPE on pairs (m, m + d/2)
 // (Sec. 2.2, RoPE-fix); values pass through. Writes X (bf16 hi | key lo) and XT (fp16 hi, lo).
-__global__ void __launch_bounds__(256) strip_kernel(const __nv_bfloat16* __restrict__ K,
-                                                    const __nv_bfloat16* __restrict__ V,
-                                                    int64_t sN, int64_t sH, int64_t N, int H,
-                                                    int d, PosSegs segs, double theta,
-                                                    int rope_fix, __nv_bfloat16* __restrict__ X,
+__device__ __forceinline__ int64_t kv_offset(const KVSource& src, int64_t n, int h, bool& second) {
+  second = n >= src.n_split;
+  return second ? (n - src.n_split) * src.sN2 + (int64_t)h * src.sH2
+                : n * src.sN + (int64_t)h * src.sH;
+}
+
+__global__ void __launch_bounds__(256) strip_kernel(KVSource src, int64_t N, int H, int d,
+                                                    PosSegs segs, double theta, int rope_fix,
+                                                    __nv_bfloat16* __restrict__ X,
                                                     __half* __restrict__ XT, int64_t Np) {
   extern __shared__ __align__(16) uint8_t sm[];
   const int half = d / 2;
@@ -45,7 +49,9 @@ __global__ void __launch_bounds__(256) strip_kernel(const __nv_bfloat16* __restr
     const int64_t n = n0 + tok;
     float a = 0.f, b = 0.f;
     if (n < N) {
-      const __nv_bfloat16* kr = K + n * sN + (int64_t)h * sH;
+      bool second;
+      const int64_t off = kv_offset(src, n, h, second);
+      const __nv_bfloat16* kr = (second ? src.K2 : src.K) + off;
       a = __bfloat162float(kr[m]);
       b = __bfloat162float(kr[m + half]);
       if (rope_fix) {
@@ -76,7 +82,9 @@ __global__ void __launch_bounds__(256) strip_kernel(const __nv_bfloat16* __restr
     const int64_t n = n0 + tok;
     float v = 0.f;
     if (n < N) {
-      const __nv_bfloat16 vb = V[n * sN + (int64_t)h * sH + f];
+      bool second;
+      const int64_t off = kv_offset(src, n, h, second);
+      const __nv_bfloat16 vb = (second ? src.V2 : src.V)[off + f];
       v = __bfloat162float(vb);
       X[((int64_t)h * N + n) * d3 + d + f] = vb;
     }
@@ -371,9 +379,9 @@ inline unsigned blocks_for(int64_t n, int per) { return (unsigned)((n + per - 1)
 
 }  // namespace
 
-cudaError_t launch_strip(const __nv_bfloat16* K, const __nv_bfloat16* V, int64_t sN, int64_t sH,
-                         int64_t N, int H, int d, const PosSegs& segs, double theta, int rope_fix,
-                         __nv_bfloat16* X, __half* XT, int64_t Np, cudaStream_t s) {
+cudaError_t launch_strip(const KVSource& src, int64_t N, int H, int d, const PosSegs& segs,
+                         double theta, int rope_fix, __nv_bfloat16* X, __half* XT, int64_t Np,
+                         cudaStream_t s) {
   const size_t smem = (size_t)(d / 2) * sizeof(double) + 2 * (size_t)(2 * d) * (kStripTok + 2) * 2;
   static bool attr = false;
   if (!attr) {
@@ -381,7 +389,7 @@ cudaError_t launch_strip(const __nv_bfloat16* K, const __nv_bfloat16* V, int64_t
     attr = true;
   }
   dim3 grid((unsigned)(Np / kStripTok), (unsigned)H);
-  strip_kernel<<<grid, 256, smem, s>>>(K, V, sN, sH, N, H, d, segs, theta, rope_fix, X, XT, Np);
+  strip_kernel<<<grid, 256, smem, s>>>(src, N, H, d, segs, theta, rope_fix, X, XT, Np);
   return cudaGetLastError();
 }
 

@@ -8,13 +8,24 @@
 
 namespace still {
 
+// The cached tokens of one call: tokens [0, n_split) come from (K, V), tokens [n_split, N)
+// from (K2, V2) (the iterative path reads [previous compact cache | new tokens] this way,
+// without a concatenation copy). Element strides per token and per KV-head; d contiguous.
+struct KVSource {
+  const __nv_bfloat16 *K = nullptr, *V = nullptr;
+  int64_t sN = 0, sH = 0;
+  const __nv_bfloat16 *K2 = nullptr, *V2 = nullptr;
+  int64_t sN2 = 0, sH2 = 0;
+  int64_t n_split = 0;
+};
+
 // RoPE-fix and input concatenation (Sec. 2.2, App. A "Input concatenation"):
 //   X[h, n]  = [unRoPE(K[n, h]) | V[n, h]]  as bf16 hi (2d) + bf16 lo of the key half (d)
 //   XT[h]    = X[h]^T as fp16 hi / lo, token-contiguous, tokens padded with zeros to Np.
 // X:  [H*N][3d] bf16.  XT: [H*2d][2*Np] fp16 (hi at [0, Np), lo at [Np, 2Np)).
-cudaError_t launch_strip(const __nv_bfloat16* K, const __nv_bfloat16* V, int64_t sN, int64_t sH,
-                         int64_t N, int H, int d, const PosSegs& segs, double theta, int rope_fix,
-                         __nv_bfloat16* X, __half* XT, int64_t Np, cudaStream_t s);
+cudaError_t launch_strip(const KVSource& src, int64_t N, int H, int d, const PosSegs& segs,
+                         double theta, int rope_fix, __nv_bfloat16* X, __half* XT, int64_t Np,
+                         cudaStream_t s);
 
 // Compactor-RoPE tables: coarse[g][m] = (cos, sin)((pmin + g * kPosGrain) * w_m), omega[m] = w_m
 // (fp32), w_m = theta_c^(-2m/D), angles reduced in fp64.

@@ -192,16 +192,29 @@ Operand2D op(const void* ptr, int64_t rows, int64_t cols, int64_t pitch = -1) {
   return Operand2D{ptr, rows, cols, pitch < 0 ? cols : pitch};
 }
 
-template <class Epi>
-still_status run_gemm(still_ctx* ctx, int cls, int bn, const Operand2D& A, const Operand2D& B,
-                      GemmParams p, const Epi& e, int ab_fmt, cudaStream_t s) {
+// One GEMM of the launch sequence; CLS is its kernel class (profiling and kernel name).
+template <int CLS, int BN, class Epi>
+still_status run_gemm_bn(still_ctx* ctx, const Operand2D& A, const Operand2D& B, GemmParams p,
+                         const Epi& e, int ab_fmt, cudaStream_t s) {
   p.err = ctx->err;
-  ctx->prof.begin(cls, s);
-  cudaError_t r = bn == 128 ? launch_gemm<128>(A, B, p, e, ab_fmt, ctx->nsm, s)
-                            : launch_gemm<256>(A, B, p, e, ab_fmt, ctx->nsm, s);
-  ctx->prof.end(cls, s);
+  ctx->prof.begin(CLS, s);
+  cudaError_t r = launch_gemm<BN, CLS>(A, B, p, e, ab_fmt, ctx->nsm, s);
+  ctx->prof.end(CLS, s);
   if (r == cudaErrorInvalidValue) return STILL_ERR_INVALID_ARG;
   return r == cudaSuccess ? STILL_OK : STILL_ERR_CUDA;
+}
+
+template <int CLS, class Epi>
+still_status run_gemm(still_ctx* ctx, int bn, const Operand2D& A, const Operand2D& B,
+                      GemmParams p, const Epi& e, int ab_fmt, cudaStream_t s) {
+  return bn == 128 ? run_gemm_bn<CLS, 128>(ctx, A, B, p, e, ab_fmt, s)
+                   : run_gemm_bn<CLS, 256>(ctx, A, B, p, e, ab_fmt, s);
+}
+
+template <int CLS, class Epi>
+still_status run_gemm256(still_ctx* ctx, const Operand2D& A, const Operand2D& B, GemmParams p,
+                         const Epi& e, int ab_fmt, cudaStream_t s) {
+  return run_gemm_bn<CLS, 256>(ctx, A, B, p, e, ab_fmt, s);
 }
 
 // Launch of one of the memory-bound kernels, timed under its class.
@@ -384,9 +397,9 @@ struct OutSpec {
 
 // ws_fixed / ws_fixed_bytes: when set, the call runs in that caller-provided scratch and never
 // touches the context's (growable) workspace.
-still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const bf16* V,
-                         int64_t sN, int64_t sH, const Positions& pos, int64_t N, int t,
-                         const OutSpec& out, cudaStream_t s, uint8_t* ws_fixed = nullptr,
+still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
+                         const Positions& pos, int64_t N, int t, const OutSpec& out,
+                         cudaStream_t s, uint8_t* ws_fixed = nullptr,
                          size_t ws_fixed_bytes = 0) {
   const still_layer_config& c = L.cfg;
   Plan P;
@@ -413,7 +426,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
   bf16* Gb = reinterpret_cast<bf16*>(ws + P.oG);
   void* Z3 = ws + P.oZ3;
 
-  KLAUNCH(STILL_K_STRIP, launch_strip(K, V, sN, sH, N, H, d, pos.segs, c.rope_theta, c.rope_fix, X, XT, Np, s));
+  KLAUNCH(STILL_K_STRIP, launch_strip(src, N, H, d, pos.segs, c.rope_theta, c.rope_fix, X, XT, Np, s));
   KLAUNCH(STILL_K_TABLES, launch_rope_tables(coarse, omega, P.G, D, pos.pmin, c.rope_theta_compactor, s));
 
   // ---------------------------------------------------------------- cross-attention groups
@@ -462,7 +475,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
       e.nheads = ni;
       e.ncoarse = P.G;
       e.Ntok = N;
-      TRY(run_gemm(ctx, STILL_K_KEYPROJ, 256, op(X, (int64_t)H * N, 3 * d), op(L.WkT, (int64_t)n * D, 2 * d), p, e,
+      TRY(run_gemm256<STILL_K_KEYPROJ>(ctx, op(X, (int64_t)H * N, 3 * d), op(L.WkT, (int64_t)n * D, 2 * d), p, e,
                    1, s));
     }
     // scale / |k~_n| per key (the d_l logit scale folded in)
@@ -486,7 +499,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
       e.csm.b1 = N;
       e.csm.c0 = 1;
       e.vec_ok = 1;
-      TRY(run_gemm(ctx, STILL_K_SCORES, 256, op(qhl, (int64_t)nbl * t, 2 * D), op(kb, (int64_t)nbl * N, 2 * D), p,
+      TRY(run_gemm256<STILL_K_SCORES>(ctx, op(qhl, (int64_t)nbl * t, 2 * D), op(kb, (int64_t)nbl * N, 2 * D), p,
                    e, 1, s));
     }
     KLAUNCH(STILL_K_SOFTMAX, launch_softmax(S, (int64_t)nbl * t, N, P.ldS, Pm, Np, 1, s));
@@ -514,7 +527,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
       e.om.r0 = 2 * d;
       e.om.c0 = 1;
       e.vec_ok = 1;
-      TRY(run_gemm(ctx, STILL_K_PX, bn, op(Pm, (int64_t)nbl * t, Np), op(XT, (int64_t)H * 2 * d, 2 * Np), p,
+      TRY(run_gemm<STILL_K_PX>(ctx, bn, op(Pm, (int64_t)nbl * t, Np), op(XT, (int64_t)H * 2 * d, 2 * Np), p,
                    e, 0, s));
     }
     KLAUNCH(STILL_K_PXSPLIT, launch_px_to_hilo(O, px_split, px_stride, b0, nbl, n, t, 2 * d, PX, s));
@@ -541,7 +554,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
     e.resm.r0 = D;
     e.resm.c0 = 1;
     e.vec_ok = 1;
-    TRY(run_gemm(ctx, STILL_K_VO, 256, op(PX, rows, 2 * n2d), op(L.WvoT, D, 2 * n2d), p, e, 1, s));
+    TRY(run_gemm256<STILL_K_VO>(ctx, op(PX, rows, 2 * n2d), op(L.WvoT, D, 2 * n2d), p, e, 1, s));
   }
   KLAUNCH(STILL_K_NORM, launch_rmsnorm(Z1, 0, rows, D, D, c.rms_eps, A1, 2 * D, 1, s));
 
@@ -586,7 +599,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
       e.ss_seg = D;
       e.ss_parts = sparts;
       e.vec_ok = 1;
-      TRY(run_gemm(ctx, STILL_K_SA_PROJ, 256, op(A1, rows, 2 * D), op(L.SqkT, (int64_t)2 * n * D, D), p, e, 1, s));
+      TRY(run_gemm256<STILL_K_SA_PROJ>(ctx, op(A1, rows, 2 * D), op(L.SqkT, (int64_t)2 * n * D, D), p, e, 1, s));
     }
     KLAUNCH(STILL_K_NORMS,
             launch_inv_norms(sss, (int64_t)nh * 2 * n * t, sparts, c.l2_eps, 1.f, sinv, s));
@@ -601,7 +614,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
       e.om.c1 = P.tp;
       e.om.c0 = 1;
       e.vec_ok = (t % 32 == 0);
-      TRY(run_gemm(ctx, STILL_K_SA_V, 256, op(L.SvT, (int64_t)n * D, D), op(A1, rows, 2 * D), p, e, 1, s));
+      TRY(run_gemm256<STILL_K_SA_V>(ctx, op(L.SvT, (int64_t)n * D, D), op(A1, rows, 2 * D), p, e, 1, s));
     }
     {  // S = scale * q~.k~ / (|q~| |k~|)  per (head, self head)
       GemmParams p = gp(t, t, nh * n, n);
@@ -631,7 +644,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
       e.csm.c0 = 1;
       e.csm.k = (int64_t)n * t;
       e.vec_ok = 1;
-      TRY(run_gemm(ctx, STILL_K_SA_SCORES, 256, op(qk, (int64_t)nh * 2 * n * t, 2 * D),
+      TRY(run_gemm256<STILL_K_SA_SCORES>(ctx, op(qk, (int64_t)nh * 2 * n * t, 2 * D),
                    op(qk, (int64_t)nh * 2 * n * t, 2 * D), p, e, 1, s));
     }
     KLAUNCH(STILL_K_SA_SOFTMAX, launch_softmax(Ssa, (int64_t)nh * n * t, t, P.ldt, Psa, P.tp, 0, s));
@@ -652,7 +665,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
       e.om.c0 = 1;
       e.om.k = (int64_t)h0 * t * n * D;
       e.vec_ok = 1;
-      TRY(run_gemm(ctx, STILL_K_SA_PV, 256, op(Psa, (int64_t)nh * n * t, P.tp),
+      TRY(run_gemm256<STILL_K_SA_PV>(ctx, op(Psa, (int64_t)nh * n * t, P.tp),
                    op(vT, (int64_t)n * D, (int64_t)nh * P.tp), p, e, 1, s));
     }
   }
@@ -672,7 +685,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
     e.resm.r0 = D;
     e.resm.c0 = 1;
     e.vec_ok = 1;
-    TRY(run_gemm(ctx, STILL_K_SO, 256, op(cat, rows, (int64_t)n * D), op(L.SoT, D, (int64_t)n * D), p, e, 1,
+    TRY(run_gemm256<STILL_K_SO>(ctx, op(cat, rows, (int64_t)n * D), op(L.SoT, D, (int64_t)n * D), p, e, 1,
                  s));
   }
   if (F > 0) {
@@ -687,7 +700,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
       e.om.c0 = 1;
       e.gelu = 1;
       e.vec_ok = 1;
-      TRY(run_gemm(ctx, STILL_K_FFN1, 256, op(A2, rows, D), op(L.W1T, F, D), p, e, 1, s));
+      TRY(run_gemm256<STILL_K_FFN1>(ctx, op(A2, rows, D), op(L.W1T, F, D), p, e, 1, s));
     }
     {
       GemmParams p = gp((int)rows, D);
@@ -704,7 +717,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
       e.resm.c0 = 1;
       e.vec_ok = 1;
       // In place (Z2 -> Z2) is safe: each element is read and written by the same thread.
-      TRY(run_gemm(ctx, STILL_K_FFN2, 256, op(Gb, rows, F), op(L.W2T, D, F), p, e, 1, s));
+      TRY(run_gemm256<STILL_K_FFN2>(ctx, op(Gb, rows, F), op(L.W2T, D, F), p, e, 1, s));
     }
   }
   if (!z3_bf16) {
@@ -726,9 +739,19 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const bf16* K, const b
     e.omega = L.omega_b;
     e.rope = c.rope_fix;
     const int bn = 2 * d <= 128 ? 128 : 256;
-    TRY(run_gemm(ctx, STILL_K_HEADS, bn, op(Z3, rows, 2 * D), op(L.WhT, 2 * d, D), p, e, 1, s));
+    TRY(run_gemm<STILL_K_HEADS>(ctx, bn, op(Z3, rows, 2 * D), op(L.WhT, 2 * d, D), p, e, 1, s));
   }
   return STILL_OK;
+}
+
+KVSource single_source(const void* K, const void* V, const int64_t strides_kv[3], int64_t N) {
+  KVSource src;
+  src.K = static_cast<const bf16*>(K);
+  src.V = static_cast<const bf16*>(V);
+  src.sN = strides_kv[0];
+  src.sH = strides_kv[1];
+  src.n_split = N;
+  return src;
 }
 
 still_status check_ctx_layer(still_ctx* ctx, int32_t layer, const LayerW** L) {
@@ -937,7 +960,7 @@ still_status still_load_layer_weights(still_ctx* ctx, int32_t layer,
       e.ss_seg = D;
       e.ss_parts = 2 * (D / 256);
       e.vec_ok = 1;
-      TRY(run_gemm(ctx, STILL_K_LOAD, 256, op(Zn, (int64_t)H * T, 2 * D), op(WqT, nD, D), p, e, 1, s));
+      TRY(run_gemm256<STILL_K_LOAD>(ctx, op(Zn, (int64_t)H * T, 2 * D), op(WqT, nD, D), p, e, 1, s));
     }
     {
       const int64_t nq = (int64_t)H * n * T;
@@ -960,7 +983,7 @@ still_status still_load_layer_weights(still_ctx* ctx, int32_t layer,
       e.om.r0 = 1;
       e.om.c0 = (int64_t)2 * n * 2 * d;
       e.vec_ok = 0;
-      TRY(run_gemm(ctx, STILL_K_LOAD, 256, op(w->Wv, 2 * d, nD), op(WoT, D, nD), p, e, 1, s));
+      TRY(run_gemm256<STILL_K_LOAD>(ctx, op(w->Wv, 2 * d, nD), op(WoT, D, nD), p, e, 1, s));
     }
     return STILL_OK;
   };
@@ -995,8 +1018,7 @@ still_status still_compact_layer(still_ctx* ctx, int32_t layer, const void* K, c
   CK(cudaSetDevice(ctx->device));
   const int H = L->cfg.n_kv_heads, d = L->cfg.head_dim;
   OutSpec o{static_cast<bf16*>(Ck), static_cast<bf16*>(Cv), (int64_t)H * d, d};
-  TRY(compact_one(ctx, *L, static_cast<const bf16*>(K), static_cast<const bf16*>(V),
-                  strides_kv[0], strides_kv[1], pos, N, t, o,
+  TRY(compact_one(ctx, *L, single_source(K, V, strides_kv, N), pos, N, t, o,
                   static_cast<cudaStream_t>(stream)));
   if (h_out_pos_start) *h_out_pos_start = pos.pmin;
   if (h_out_pos_step) *h_out_pos_step = t > 1 ? (pos.pmax - pos.pmin) / (double)(t - 1) : 0.0;
@@ -1035,8 +1057,7 @@ still_status still_compact_layer_noalloc(still_ctx* ctx, int32_t layer, const vo
   const bool timing = ctx->prof.on;
   ctx->prof.on = false;
   const still_status st =
-      compact_one(ctx, *L, static_cast<const bf16*>(K), static_cast<const bf16*>(V),
-                  strides_kv[0], strides_kv[1], pos, N, t, o,
+      compact_one(ctx, *L, single_source(K, V, strides_kv, N), pos, N, t, o,
                   static_cast<cudaStream_t>(stream), scratch, kNoAllocScratchBytes);
   ctx->prof.on = timing;
   TRY(st);
@@ -1116,6 +1137,87 @@ still_status still_compact_stack_ragged(still_ctx* ctx, int32_t n_layers,
     TRY(still_compact_layer_ragged(ctx, l, Kpacked[l], Vpacked[l], h_cu_seqlens, B, h_segments,
                                    h_seg_per_seq, h_t, h_cu_t, Ck[l], Cv[l], h_pos_offset,
                                    stream));
+  return STILL_OK;
+}
+
+still_status still_recompact_layer_ragged(still_ctx* ctx, int32_t layer, int32_t B,
+                                          const void* Kprev, const void* Vprev,
+                                          const int64_t* h_cu_prev, const int64_t* h_prev_len,
+                                          const void* Knew, const void* Vnew,
+                                          const int64_t* h_cu_new, int64_t ratio, void* Ck,
+                                          void* Cv, int64_t* h_cu_out, int64_t* h_len_out,
+                                          void* stream) {
+  const LayerW* L = nullptr;
+  TRY(check_ctx_layer(ctx, layer, &L));
+  if (B < 1 || Kprev == nullptr || Vprev == nullptr || h_cu_prev == nullptr ||
+      h_prev_len == nullptr || h_cu_new == nullptr || Ck == nullptr || Cv == nullptr ||
+      h_cu_out == nullptr || ratio < 1)
+    return STILL_ERR_INVALID_ARG;
+  if (h_cu_prev[0] != 0 || h_cu_new[0] != 0) return STILL_ERR_SHAPE;
+  const int H = L->cfg.n_kv_heads, d = L->cfg.head_dim;
+  const int64_t row = (int64_t)H * d;
+  // Budgets first (integers only): t_b = round((L_prev + new) / ratio).
+  h_cu_out[0] = 0;
+  for (int b = 0; b < B; ++b) {
+    const int64_t tprev = h_cu_prev[b + 1] - h_cu_prev[b];
+    const int64_t nnew = h_cu_new[b + 1] - h_cu_new[b];
+    if (tprev < 1 || nnew < 0 || h_prev_len[b] < tprev) return STILL_ERR_SHAPE;
+    if (nnew > 0 && (Knew == nullptr || Vnew == nullptr)) return STILL_ERR_INVALID_ARG;
+    const int64_t Lr = h_prev_len[b] + nnew;
+    const int64_t tb = std::max<int64_t>(1, still_budget(Lr, ratio));
+    if (tb > tprev + nnew || tb > L->cfg.t_max) return STILL_ERR_SHAPE;
+    h_cu_out[b + 1] = h_cu_out[b] + tb;
+  }
+  if (((reinterpret_cast<uintptr_t>(Ck) | reinterpret_cast<uintptr_t>(Cv)) & 15) ||
+      ((reinterpret_cast<uintptr_t>(Kprev) | reinterpret_cast<uintptr_t>(Vprev)) & 1))
+    return STILL_ERR_ALIGNMENT;
+  CK(cudaSetDevice(ctx->device));
+  for (int b = 0; b < B; ++b) {
+    const int64_t tprev = h_cu_prev[b + 1] - h_cu_prev[b];
+    const int64_t nnew = h_cu_new[b + 1] - h_cu_new[b];
+    const int64_t Lp = h_prev_len[b];
+    const int64_t N = tprev + nnew;
+    const int t = (int)(h_cu_out[b + 1] - h_cu_out[b]);
+    // Segment A: the previous compact slots at their output positions (evenly spaced over
+    // [0, L_prev - 1]); segment B: the new tokens at L_prev .. L_prev + new - 1.
+    still_pos_segment seg[2] = {
+        {0.0, tprev > 1 ? (double)(Lp - 1) / (double)(tprev - 1) : 0.0, tprev},
+        {(double)Lp, 1.0, nnew}};
+    Positions pos;
+    TRY(make_positions(seg, nnew > 0 ? 2 : 1, N, pos));
+    KVSource src;
+    src.K = static_cast<const bf16*>(Kprev) + h_cu_prev[b] * row;
+    src.V = static_cast<const bf16*>(Vprev) + h_cu_prev[b] * row;
+    src.sN = row;
+    src.sH = d;
+    src.K2 = nnew > 0 ? static_cast<const bf16*>(Knew) + h_cu_new[b] * row : nullptr;
+    src.V2 = nnew > 0 ? static_cast<const bf16*>(Vnew) + h_cu_new[b] * row : nullptr;
+    src.sN2 = row;
+    src.sH2 = d;
+    src.n_split = tprev;
+    OutSpec o{static_cast<bf16*>(Ck) + h_cu_out[b] * row, static_cast<bf16*>(Cv) + h_cu_out[b] * row,
+              row, d};
+    TRY(compact_one(ctx, *L, src, pos, N, t, o, static_cast<cudaStream_t>(stream)));
+    if (h_len_out) h_len_out[b] = Lp + nnew;
+  }
+  return STILL_OK;
+}
+
+still_status still_recompact_stack_ragged(still_ctx* ctx, int32_t n_layers, int32_t B,
+                                          const void* const* Kprev, const void* const* Vprev,
+                                          const int64_t* h_cu_prev, const int64_t* h_prev_len,
+                                          const void* const* Knew, const void* const* Vnew,
+                                          const int64_t* h_cu_new, int64_t ratio,
+                                          void* const* Ck, void* const* Cv, int64_t* h_cu_out,
+                                          int64_t* h_len_out, void* stream) {
+  if (ctx == nullptr || n_layers < 1 || Kprev == nullptr || Vprev == nullptr ||
+      Ck == nullptr || Cv == nullptr)
+    return STILL_ERR_INVALID_ARG;
+  for (int l = 0; l < n_layers; ++l)
+    TRY(still_recompact_layer_ragged(ctx, l, B, Kprev[l], Vprev[l], h_cu_prev, h_prev_len,
+                                     Knew ? Knew[l] : nullptr, Vnew ? Vnew[l] : nullptr,
+                                     h_cu_new, ratio, Ck[l], Cv[l], h_cu_out, h_len_out,
+                                     stream));
   return STILL_OK;
 }
 

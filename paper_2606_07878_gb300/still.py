@@ -25,7 +25,7 @@ EXPORTS = [
     "still_compact_stack_ragged", "still_workspace_size", "still_set_workspace_limit",
     "still_get_device_status", "still_budget", "still_kv_bytes", "still_param_count",
     "still_profile_enable", "still_profile_read", "still_kernel_class_name",
-    "still_compact_layer_noalloc",
+    "still_compact_layer_noalloc", "still_recompact_layer_ragged", "still_recompact_stack_ragged",
 ]
 
 NOALLOC_SCRATCH_MIB = 64  # STILL_NOALLOC_SCRATCH_MIB in include/still.h
@@ -98,6 +98,12 @@ def lib():
             "still_compact_stack_ragged": ([P, I32, ctypes.POINTER(P), ctypes.POINTER(P), PI64, I32,
                                             PSEG, PI32, PI32, PI64, ctypes.POINTER(P),
                                             ctypes.POINTER(P), PI64, P], ctypes.c_int),
+            "still_recompact_layer_ragged": ([P, I32, I32, P, P, PI64, PI64, P, P, PI64, I64, P,
+                                              P, PI64, PI64, P], ctypes.c_int),
+            "still_recompact_stack_ragged": ([P, I32, I32, ctypes.POINTER(P), ctypes.POINTER(P),
+                                              PI64, PI64, ctypes.POINTER(P), ctypes.POINTER(P),
+                                              PI64, I64, ctypes.POINTER(P), ctypes.POINTER(P),
+                                              PI64, PI64, P], ctypes.c_int),
             "still_workspace_size": ([P, I64, I32, ctypes.POINTER(ctypes.c_size_t)], ctypes.c_int),
             "still_set_workspace_limit": ([P, ctypes.c_size_t], ctypes.c_int),
             "still_get_device_status": ([P, P, PI32], ctypes.c_int),
@@ -268,6 +274,35 @@ def still_compact_stack_ragged(ctx, Kps, Vps, cu_seqlens, ts, Cks, Cvs, segments
                                             arr(Cks), arr(Cvs), off, _stream(stream)),
            "still_compact_stack_ragged")
     return list(off)
+
+
+def still_recompact_layer_ragged(ctx, layer, Kprev, Vprev, cu_prev, prev_len, Knew, Vnew,
+                                 cu_new, ratio, Ck, Cv, stream=None):
+    """[previous compact | new tokens] -> new compact caches. Returns (cu_out, len_out)."""
+    B = len(prev_len)
+    I64 = ctypes.c_int64
+    cu_out = (I64 * (B + 1))()
+    len_out = (I64 * B)()
+    _check(lib().still_recompact_layer_ragged(
+        ctx, layer, B, _ptr(Kprev), _ptr(Vprev), (I64 * (B + 1))(*cu_prev), (I64 * B)(*prev_len),
+        _ptr(Knew), _ptr(Vnew), (I64 * (B + 1))(*cu_new), ratio, _ptr(Ck), _ptr(Cv), cu_out,
+        len_out, _stream(stream)), "still_recompact_layer_ragged")
+    return list(cu_out), list(len_out)
+
+
+def still_recompact_stack_ragged(ctx, Kprevs, Vprevs, cu_prev, prev_len, Knews, Vnews, cu_new,
+                                 ratio, Cks, Cvs, stream=None):
+    L = len(Kprevs)
+    B = len(prev_len)
+    P, I64 = ctypes.c_void_p, ctypes.c_int64
+    arr = lambda xs: (P * L)(*[x.data_ptr() for x in xs])
+    cu_out = (I64 * (B + 1))()
+    len_out = (I64 * B)()
+    _check(lib().still_recompact_stack_ragged(
+        ctx, L, B, arr(Kprevs), arr(Vprevs), (I64 * (B + 1))(*cu_prev), (I64 * B)(*prev_len),
+        arr(Knews), arr(Vnews), (I64 * (B + 1))(*cu_new), ratio, arr(Cks), arr(Cvs), cu_out,
+        len_out, _stream(stream)), "still_recompact_stack_ragged")
+    return list(cu_out), list(len_out)
 
 
 def still_workspace_size(ctx, max_tokens: int, max_t: int) -> int:
