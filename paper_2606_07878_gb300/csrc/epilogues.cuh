@@ -85,6 +85,8 @@ __device__ __forceinline__ void pack_f32x16(const float* v, uint4 (&o)[4]) {
 // multiple of 32, so every 32-column chunk maps to 32 consecutive elements; ss_seg is a
 // multiple of the tile width.
 struct EpiAffine {
+  static constexpr int kWarps = 8;  // two per lane quarter: alternating 32-column chunks
+  static constexpr int kStages = 0;  // default pipeline depth
   int32_t kind = OUT_F32;
   void* out = nullptr;
   int64_t lo_off = 0;  // OUT_HILO: lo element offset from hi
@@ -239,8 +241,13 @@ __device__ __forceinline__ double seg_position(const PosSegs& s, int64_t idx) {
 constexpr int kPosGrain = 32;
 
 struct EpiRopeC {
+  // Element-wise heavy and MMA-light (K = 3d): four warps per lane quarter, each owning 32 of
+  // the tile's 128 pairs, processed 16 at a time; a short pipeline suffices.
+  static constexpr int kWarps = 16;
+  static constexpr int kParts = kWarps / 4;
+  static constexpr int kStages = 3;
   __nv_bfloat16* out = nullptr;  // [H][n][N][2D]: hi at [0, D), lo at [D, 2D)
-  float* sumsq = nullptr;        // [H][n][N][2 * D / 256] partial sums of |k~|^2
+  float* sumsq = nullptr;        // [H][n][N][kParts * D / 256] partial sums of |k~|^2
   const float* bias = nullptr;   // [n*D], pair-chunk order
   const float2* coarse = nullptr;  // [G][D/2]: (cos, sin)(G_g * omega_m)
   const float* omega = nullptr;    // [D/2] fp32
@@ -265,17 +272,17 @@ struct EpiRopeC {
     const int64_t row_out = ((int64_t)(tc.b * nheads + head) * Ntok + (rvalid ? r : 0)) *
                             (2 * (int64_t)D);
     float ss = 0.f;
-    // half 0 owns pairs [0, 64) of the tile, half 1 pairs [64, 128): 128-byte row segments
-    for (int u = 64 * half; u < 64 * half + 64; u += 32) {
-      float a[32], bb[32];
-      tmem_ld32(taddr + (uint32_t)u, a);
-      tmem_ld32(taddr + (uint32_t)(128 + u), bb);
+    // part p owns pairs [32p, 32p + 32) of the tile, taken 16 at a time
+    for (int u = 32 * half; u < 32 * half + 32; u += 16) {
+      float a[16], bb[16];
+      tmem_ld16(taddr + (uint32_t)u, a);
+      tmem_ld16(taddr + (uint32_t)(128 + u), bb);
       const float4* crow = reinterpret_cast<const float4*>(coarse + (int64_t)g * (D / 2) + m_base + u);
       const float4* om4 = reinterpret_cast<const float4*>(omega + m_base + u);
       const float4* ba4 = reinterpret_cast<const float4*>(bias + c_tile + u);
       const float4* bb4 = reinterpret_cast<const float4*>(bias + c_tile + 128 + u);
 #pragma unroll
-      for (int e4 = 0; e4 < 8; ++e4) {
+      for (int e4 = 0; e4 < 4; ++e4) {
         const float4 w = om4[e4], xa = ba4[e4], xb = bb4[e4];
         const float4 c01 = crow[2 * e4], c23 = crow[2 * e4 + 1];
         const float ws[4] = {w.x, w.y, w.z, w.w};
@@ -298,17 +305,33 @@ struct EpiRopeC {
         }
       }
       __nv_bfloat16* o = out + row_out + f_tile + u;
-      uint4 h4[4], l4[4];
-      pack_hilo_x32(a, h4, l4);
-      warp_store64(stage, h4, o, rvalid);
-      warp_store64(stage, l4, o + D, rvalid);
-      pack_hilo_x32(bb, h4, l4);
-      warp_store64(stage, h4, o + 128, rvalid);
-      warp_store64(stage, l4, o + D + 128, rvalid);
+      uint4 h2[2], l2[2];
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        uint32_t h[4], l[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) split_pack(a[8 * q + 2 * k], a[8 * q + 2 * k + 1], h[k], l[k]);
+        h2[q] = make_uint4(h[0], h[1], h[2], h[3]);
+        l2[q] = make_uint4(l[0], l[1], l[2], l[3]);
+      }
+      warp_store32(stage, h2, o, rvalid);
+      warp_store32(stage, l2, o + D, rvalid);
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        uint32_t h[4], l[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          split_pack(bb[8 * q + 2 * k], bb[8 * q + 2 * k + 1], h[k], l[k]);
+        h2[q] = make_uint4(h[0], h[1], h[2], h[3]);
+        l2[q] = make_uint4(l[0], l[1], l[2], l[3]);
+      }
+      warp_store32(stage, h2, o + 128, rvalid);
+      warp_store32(stage, l2, o + D + 128, rvalid);
     }
     if (rvalid) {
-      const int parts = 2 * (D / 256);
-      sumsq[((int64_t)(tc.b * nheads + head) * Ntok + r) * parts + (f_tile / 256) * 2 + half] = ss;
+      const int parts = kParts * (D / 256);
+      sumsq[((int64_t)(tc.b * nheads + head) * Ntok + r) * parts + (f_tile / 256) * kParts + half] =
+          ss;
     }
   }
 };
@@ -318,6 +341,8 @@ struct EpiRopeC {
 // the caller's C_k / C_v with element strides (st, sh). omega = theta^(-2m/d) in fp64;
 // the angle is reduced modulo 2 pi in fp64 before the fp32 sin/cos.
 struct EpiHeads {
+  static constexpr int kWarps = 8;
+  static constexpr int kStages = 0;
   __nv_bfloat16* ck = nullptr;
   __nv_bfloat16* cv = nullptr;
   int64_t st = 0, sh = 0;  // element strides of [t, H, d]; d is contiguous, rows 16-B aligned

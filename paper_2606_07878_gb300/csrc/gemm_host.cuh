@@ -73,7 +73,7 @@ inline bool finalize_gemm(GemmParams& p, int ab_fmt) {
 template <int BN, int kRole, class Epi>
 inline cudaError_t launch_gemm(const Operand2D& A, const Operand2D& B, GemmParams p, Epi epi,
                                int ab_fmt, int num_sms, cudaStream_t stream) {
-  using S = GemmSmem<BN>;
+  using S = GemmSmem<BN, Epi>;
   if (!finalize_gemm<BN>(p, ab_fmt)) return cudaErrorInvalidValue;
   CUtensorMap ta, tb;
   if (!make_tmap(&ta, A, kBM) || !make_tmap(&tb, B, BN)) return cudaErrorInvalidValue;
@@ -87,7 +87,7 @@ inline cudaError_t launch_gemm(const Operand2D& A, const Operand2D& B, GemmParam
     attr_set = true;
   }
   const int grid = p.ntiles < num_sms ? p.ntiles : num_sms;
-  kern<<<grid, kGemmThreads, S::kBytes, stream>>>(ta, tb, p, epi);
+  kern<<<grid, gemm_threads<Epi>(), S::kBytes, stream>>>(ta, tb, p, epi);
   return cudaGetLastError();
 }
 

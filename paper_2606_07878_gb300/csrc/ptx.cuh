@@ -162,6 +162,21 @@ __host__ __device__ constexpr uint32_t idesc_f16(int M, int N, int ab_fmt) {
          | ((uint32_t)(M >> 4) << 24);      // M >> 4              [24, 29)
 }
 
+// 32 lanes x 16 consecutive fp32 columns: thread i of the warp receives lane (base + i).
+STILL_DEV void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
 // 32 lanes x 32 consecutive fp32 columns: thread i of the warp receives lane (base + i).
 STILL_DEV void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   uint32_t r[32];

@@ -293,7 +293,7 @@ bool make_plan(const still_layer_config& c, int64_t N, int t, double pmin, doubl
   P.oZ3 = take(H * T * D * 4);
   const size_t fixed = off;
   P.kb_b = a256(N * 2 * D * 2);
-  P.kss_b = a256(N * 4 * (2 * (D / 256) + 1));  // |k~|^2 partials + inverse norms
+  P.kss_b = a256(N * 4 * (EpiRopeC::kParts * (D / 256) + 1));  // |k~|^2 partials + inverses
   P.q_b = a256(T * 2 * D * 2);
   P.S_b = a256(T * P.ldS * 4);
   P.P_b = a256(T * P.Np * 2);
@@ -446,7 +446,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     uint8_t* g = ws + P.oCA;
     bf16* kb = reinterpret_cast<bf16*>(g);
     g += P.kb_b * nbl;
-    const int kparts = 2 * (D / 256);
+    const int kparts = EpiRopeC::kParts * (D / 256);
     float* kss = reinterpret_cast<float*>(g);        // [nbl][N][kparts]
     float* kinv = kss + (size_t)nbl * N * kparts;    // [nbl][N]
     g += P.kss_b * nbl;

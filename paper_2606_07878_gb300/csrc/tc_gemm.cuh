@@ -7,8 +7,8 @@
 // "hi/lo" operand stored as [hi | lo] along K gives the 2- and 3-pass products that keep
 // ~fp32 accuracy on bf16 tensor cores (a_hi b_hi + a_hi b_lo + a_lo b_hi).
 //
-// CTA = 10 warps: warp 0 issues TMA, warp 1 owns TMEM and issues tcgen05.mma (one thread),
-// warps 2..9 run the epilogue from TMEM (two per lane quarter, alternating column chunks). The accumulator is double-buffered in TMEM
+// CTA = 2 + Epi::kWarps warps: warp 0 issues TMA, warp 1 owns TMEM and issues tcgen05.mma
+// (one thread), the rest run the epilogue from TMEM (Epi::kWarps / 4 per lane quarter). The accumulator is double-buffered in TMEM
 // (2 x BN fp32 columns), so a tile's epilogue overlaps the next tile's main loop.
 // Tiles are 128 x BN; the grid is persistent (tile += gridDim.x), m-tiles fastest so that
 // CTAs running together share B tiles through L2.
@@ -19,8 +19,12 @@ namespace still {
 
 constexpr int kBM = 128;
 constexpr int kBK = 64;
-constexpr int kEpiWarps = 8;  // two warps per TMEM lane quarter, alternating 32-column chunks
-constexpr int kGemmThreads = 64 + 32 * kEpiWarps;
+// Epilogue warps come from the epilogue type (Epi::kWarps, a multiple of 4): kWarps / 4 warps
+// share each TMEM lane quarter and split its columns ("parts").
+template <class Epi>
+constexpr int gemm_threads() {
+  return 64 + 32 * Epi::kWarps;
+}
 
 struct GemmPass {
   int32_t a_koff, b_koff;  // K offset (elements) of this pass in A / B
@@ -67,20 +71,39 @@ __device__ __forceinline__ void split_range(const GemmParams& p, int split, int&
 constexpr int kStageRowU4 = 5;
 constexpr int kWarpStageBytes = 32 * kStageRowU4 * 16;
 
-template <int BN>
+template <int BN, class Epi>
 struct GemmSmem {
-  static constexpr int kStages = BN >= 256 ? 4 : 6;
+  static constexpr int kStages = Epi::kStages > 0 ? Epi::kStages : (BN >= 256 ? 4 : 6);
   static constexpr int kABytes = kBM * kBK * 2;
   static constexpr int kBBytes = BN * kBK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kEpiOffset = kStages * kStageBytes;
-  static constexpr int kBarOffset = kEpiOffset + kEpiWarps * kWarpStageBytes;
+  static constexpr int kBarOffset = kEpiOffset + Epi::kWarps * kWarpStageBytes;
   static constexpr int kBytes = kBarOffset + 256 + 1024;  // + barriers + alignment slack
+  static_assert(kBytes <= 232448, "shared memory budget");
 };
 
 // Coalesced row store for one warp: lane i holds 64 bytes (v[0..3]) for its own row, to be
 // written at dst (16-byte aligned) if valid. The warp exchanges them through its staging area
 // so that each store instruction writes 8 rows x 64 contiguous bytes (whole 32-byte sectors).
+// As warp_store64 with 32 bytes per lane: each store instruction writes 16 rows x 32 bytes.
+__device__ __forceinline__ void warp_store32(uint4* stage, const uint4 (&v)[2], void* dst,
+                                             bool valid) {
+  const int lane = threadIdx.x & 31;
+  stage[lane * 3] = v[0];
+  stage[lane * 3 + 1] = v[1];
+  __syncwarp();
+  const unsigned long long mine = reinterpret_cast<unsigned long long>(dst);
+#pragma unroll
+  for (int it = 0; it < 2; ++it) {
+    const int r = it * 16 + (lane >> 1), q = lane & 1;
+    const unsigned long long d = __shfl_sync(0xffffffffu, mine, r);
+    const int ok = __shfl_sync(0xffffffffu, valid ? 1 : 0, r);
+    if (ok) reinterpret_cast<uint4*>(d)[q] = stage[r * 3 + q];
+  }
+  __syncwarp();
+}
+
 __device__ __forceinline__ void warp_store64(uint4* stage, const uint4 (&v)[4], void* dst,
                                              bool valid) {
   const int lane = threadIdx.x & 31;
@@ -106,10 +129,11 @@ __device__ __forceinline__ void warp_store64(uint4* stage, const uint4 (&v)[4], 
 // kRole only names the instantiation (one per GEMM of the launch sequence) so that profilers
 // can tell the GEMMs apart; it does not change the code.
 template <int BN, class Epi, int kRole>
-__global__ void __launch_bounds__(kGemmThreads, 1)
+__global__ void __launch_bounds__(gemm_threads<Epi>(), 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
                    const __grid_constant__ CUtensorMap tmB, const GemmParams p, const Epi epi) {
-  using S = GemmSmem<BN>;
+  using S = GemmSmem<BN, Epi>;
+  constexpr int kEpiWarps = Epi::kWarps;
   constexpr int kStages = S::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -250,9 +274,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       }
     }
   } else {
-    // -------------------------------------------------------------- epilogue (warps 2..9)
+    // -------------------------------------------------------------- epilogue (warps 2..)
     const int quarter = warp & 3;  // TMEM lanes this warp may access: [32q, 32q + 32)
-    const int half = (warp - 2) >> 2;
+    const int half = (warp - 2) >> 2;  // the "part" of the quarter's columns this warp owns
     const int row = quarter * 32 + lane;
     uint4* stage = reinterpret_cast<uint4*>(smem + S::kEpiOffset + (warp - 2) * kWarpStageBytes);
     int acc = 0;
