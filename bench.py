@@ -26,6 +26,12 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 WORKLOAD = "qwen7b_8k"
+DEFAULT_T = {"qwen7b_8k": 1024, "qwen8b_32k": 2048, "gemma_128k": 655, "tiny_1k": 128}
+
+
+def describe(name, wl, t):
+    return (f"{name}: {wl['L']} layers, N={wl['N']}, H_kv={wl['H']}, d={wl['d']}, "
+            f"D={wl['D']}, {wl['n']} heads, FFN {wl['F']}, t={t} ({round(wl['N'] / t)}x)")
 
 # DRAM traffic of one scores-GEMM launch from an ncu capture (profiles/), valid only for the
 # kernel sources it was taken on.
@@ -147,26 +153,56 @@ def algorithmic_flops(wl, t, N):
 
 
 def run_cpu_baseline(wl, t, budget_s=30.0):
-    """The oracle as it stands on one (layer, KV-head) slice, extrapolated to the stack."""
-    import numpy as np
-    import torch
+    """The oracle as it stands on a bounded slice of the workload, extrapolated to the stack.
 
+    One (layer, KV-head) when that fits the budget (the full per-head compaction); for the
+    largest shapes, the cross-attention of one cross head of one KV-head, extrapolated by the
+    ratio of algorithmic flops.
+    """
     from oracle import still_oracle as O
     from paper_2606_07878_gb300 import synth
 
+    fl = algorithmic_flops(wl, t, wl["N"])
+    one_head = fl["total"] / wl["H"]
     W = synth.gen_weights(wl, 0, t, "cpu")
-    K, V = synth.gen_kv(wl, 0, device="cpu")
     cfg = O.cfg_from_workload(wl)
-    Kf, Vf, Wf = synth.bf16_to_f64(K), synth.bf16_to_f64(V), O.as_f64(W)
-    t0 = time.perf_counter()
-    O.compact_layer(Kf, Vf, Wf, cfg, t, heads=[0])
-    sec = time.perf_counter() - t0
-    slices = wl["L"] * wl["H"]
-    value = wl["N"] / (sec * slices)
+    Wf = O.as_f64(W)
+    if one_head < 2.5e12:
+        K, V = synth.gen_kv(wl, 0, device="cpu")
+        Kf, Vf = synth.bf16_to_f64(K), synth.bf16_to_f64(V)
+        t0 = time.perf_counter()
+        O.compact_layer(Kf, Vf, Wf, cfg, t, heads=[0])
+        sec = time.perf_counter() - t0
+        scale = wl["L"] * wl["H"]
+        what = f"layer 0, KV-head 0 of {wl['L']}x{wl['H']}"
+    else:
+        import numpy as np
+        K, V = synth.gen_kv(wl, 0, device="cpu")
+        Kf, Vf = synth.bf16_to_f64(K)[:, 0], synth.bf16_to_f64(V)[:, 0]
+        kpos = np.arange(wl["N"], dtype=np.float64)
+        Wi = dict(Wf)
+        D = wl["D"]
+        for k in ("Wq", "Wk", "Wv"):
+            Wi[k] = Wf[k][:, :D]
+        for k in ("bq", "bk"):
+            Wi[k] = Wf[k][:D]
+        Wi["Wo"] = Wf["Wo"][:D]
+        c1 = O.cfg_from_workload(wl, n_c=1)
+        t0 = time.perf_counter()
+        X = np.concatenate([O.unrope(Kf, kpos, cfg.theta), Vf], axis=-1)
+        Zn = O.rmsnorm(Wf["Z"][0, :t], cfg.rms_eps)
+        O.cross_attention(Zn, X, Wi, 0, c1, O.linspace_positions(0, wl["N"] - 1, t), kpos)
+        sec = time.perf_counter() - t0
+        N, d = wl["N"], wl["d"]
+        sample_fl = (2 * N * 2 * d * D + 2 * t * N * D + 2 * t * N * 2 * d + 2 * t * 2 * d * D
+                     + 2 * t * D * D)
+        scale = fl["total"] * wl["L"] / sample_fl
+        what = (f"cross-attention of 1 of {wl['n']} heads of KV-head 0, layer 0, "
+                f"extrapolated by algorithmic flops")
+    value = wl["N"] / (sec * scale)
     return {"value": value, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"layer 0, KV-head 0 of {wl['L']}x{wl['H']} (t={t}, N={wl['N']}), "
-                      f"{sec:.1f} s, extrapolated x{slices} to the stack",
-            "seconds": sec}
+            "sample": f"{what} (t={t}, N={wl['N']}), {sec:.1f} s, x{scale:.0f} to the stack",
+            "seconds": sec, "scale": scale}
 
 
 def run_reference(args):
@@ -174,14 +210,15 @@ def run_reference(args):
     if rank != 0:
         return
     from paper_2606_07878_gb300 import synth
-    wl = synth.WORKLOADS[WORKLOAD]
-    t = args.t
+    name = args.workload
+    wl = synth.WORKLOADS[name]
+    t = args.t or DEFAULT_T[name]
     secs = []
     for i in range(args.warmup + args.steps):
         r = run_cpu_baseline(wl, t)
         if i >= args.warmup:
             secs.append(r["seconds"])
-    slices = wl["L"] * wl["H"]
+    slices = r["scale"]
     mean = sum(secs) / len(secs)
     value = wl["N"] / (mean * slices)
     line = {
@@ -189,17 +226,105 @@ def run_reference(args):
         "value": value, "unit": "tokens/s", "n_gpus": args.gpus, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": mean * 1e3 * slices, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": f"{WORKLOAD}: 28 layers, N=8192, H_kv=4, d=128, D=1024, "
-                               f"8 heads, FFN 4096, t={t}", "layers": wl["L"], "N": wl["N"],
-                   "t": t},
+        "config": {"workload": describe(name, wl, t), "layers": wl["L"], "N": wl["N"], "t": t},
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": os.cpu_count(),
-                         "kind": "oracle",
-                         "sample": f"each step: layer 0, KV-head 0 of {wl['L']}x{wl['H']}, "
-                                   f"extrapolated x{slices}"},
+                         "kind": "oracle", "sample": "each step: " + r["sample"]},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line))
+
+
+def run_iterative(args):
+    """The iterative ragged serving workload: 8 sequences (lengths uniform in [8k, 32k], seed
+    7), 36 Qwen-8B-shaped layers, compacted to 32x; then rounds of +8192 new tokens per
+    sequence, each round re-compacting [compact | new] to the 32x budget. One step = one round
+    over the whole stack; the metric is new logical tokens absorbed per second."""
+    import torch
+
+    from paper_2606_07878_gb300 import still, synth
+
+    wl = synth.WORKLOADS["iterative_ragged"]
+    L, H, d, ratio, chunk = wl["L"], wl["H"], wl["d"], wl["ratio"], wl["chunk"]
+    rounds = min(args.steps, wl["rounds"])
+    lens = synth.iterative_lengths(wl)
+    B = len(lens)
+    dev = "cuda:0"
+    torch.cuda.set_device(0)
+    stream = torch.cuda.current_stream()
+    t_cap = still.still_budget(max(lens) + wl["rounds"] * chunk, ratio)
+    ctx = still.still_create(0)
+    cfg = still.config_from_workload(dict(wl, N=0), t_cap)
+    for l in range(L):
+        W = synth.gen_weights(wl, l, t_cap, dev)
+        still.still_load_layer_weights(ctx, l, cfg, W)
+        del W
+    # round 0: the initial caches, compacted once (untimed set-up)
+    ts = [still.still_budget(x, ratio) for x in lens]
+    cu = [0]
+    for x in lens:
+        cu.append(cu[-1] + x)
+    Cks, Cvs = [], []
+    for l in range(L):
+        parts = [synth.gen_kv(wl, l, N=x, device=dev, stream=b) for b, x in enumerate(lens)]
+        Kp = torch.cat([p[0] for p in parts])
+        Vp = torch.cat([p[1] for p in parts])
+        Ck = torch.empty((sum(ts), H, d), dtype=torch.bfloat16, device=dev)
+        Cv = torch.empty_like(Ck)
+        still.still_compact_layer_ragged(ctx, l, Kp, Vp, cu, ts, Ck, Cv, stream=stream)
+        Cks.append(Ck)
+        Cvs.append(Cv)
+        del Kp, Vp, parts
+    cu_prev = [0]
+    for x in ts:
+        cu_prev.append(cu_prev[-1] + x)
+    prev_len = list(lens)
+    total_ms = 0.0
+    launches = 0
+    for r in range(rounds):
+        Kn, Vn = [], []
+        for l in range(L):
+            parts = [synth.gen_kv(wl, l, N=chunk, device=dev, stream=1000 * (r + 1) + b,
+                                  positions=torch.arange(prev_len[b], prev_len[b] + chunk,
+                                                         dtype=torch.float64))
+                     for b in range(B)]
+            Kn.append(torch.cat([p[0] for p in parts]))
+            Vn.append(torch.cat([p[1] for p in parts]))
+        t_next = [still.still_budget(x + chunk, ratio) for x in prev_len]
+        Ck2 = [torch.empty((sum(t_next), H, d), dtype=torch.bfloat16, device=dev)
+               for _ in range(L)]
+        Cv2 = [torch.empty_like(c) for c in Ck2]
+        cu_new = [b * chunk for b in range(B + 1)]
+        torch.cuda.synchronize()
+        still.still_profile_enable(ctx, True)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        cu_out, len_out = still.still_recompact_stack_ragged(
+            ctx, Cks, Cvs, cu_prev, prev_len, Kn, Vn, cu_new, ratio, Ck2, Cv2, stream=stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        total_ms += e0.elapsed_time(e1)
+        prof = still.still_profile_read(ctx)
+        launches += sum(v[0] for k, v in prof.items() if k != "load")
+        Cks, Cvs, cu_prev, prev_len = Ck2, Cv2, cu_out, len_out
+        del Kn, Vn
+    code, det = still.still_get_device_status(ctx, stream)
+    if code != 0:
+        raise RuntimeError(f"device status {still.STATUS.get(code)} {det}")
+    still.still_destroy(ctx)
+    value = B * chunk * rounds / (total_ms / 1e3)
+    print(json.dumps({
+        "metric": "new logical tokens absorbed per second (iterative re-compaction, all layers)",
+        "value": value, "unit": "tokens/s", "n_gpus": 1, "steps": rounds, "warmup": 0,
+        "ms_per_step": total_ms / rounds, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"iterative_ragged: {B} sequences, lengths {lens}, {L} layers, "
+                               f"H_kv={H}, d={d}, D={wl['D']}, {wl['n']} heads, "
+                               f"{ratio}x, +{chunk} tokens per round",
+                   "final_lengths": prev_len},
+        "gpu_launches": launches,
+    }))
 
 
 def main():
@@ -208,11 +333,17 @@ def main():
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--t", type=int, default=1024)
+    ap.add_argument("--t", type=int, default=0, help="compact length (default per workload)")
+    ap.add_argument("--workload", default=WORKLOAD,
+                    choices=["qwen7b_8k", "qwen8b_32k", "gemma_128k", "tiny_1k",
+                             "iterative_ragged"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)
+        return
+    if args.workload == "iterative_ragged":
+        run_iterative(args)
         return
 
     import torch
@@ -226,8 +357,10 @@ def main():
         dist.init_process_group(backend="nccl", device_id=torch.device(f"cuda:{local}"))
     torch.cuda.set_device(local)
     dev = f"cuda:{local}"
-    wl = synth.WORKLOADS[WORKLOAD]
-    L, N, H, d, t = wl["L"], wl["N"], wl["H"], wl["d"], args.t
+    name = args.workload
+    wl = synth.WORKLOADS[name]
+    L, N, H, d = wl["L"], wl["N"], wl["H"], wl["d"]
+    t = args.t or DEFAULT_T[name]
     stream = torch.cuda.current_stream()
 
     ctx = still.still_create(local)
@@ -338,10 +471,8 @@ def main():
         "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
         "warmup": max(args.warmup, 3), "ms_per_step": ms_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": f"{WORKLOAD}: 28 layers, N=8192, H_kv=4, d=128, D=1024, "
-                               f"8 heads, FFN 4096, t={t} ({N // t}x)",
-                   "layers": L, "N": N, "t": t,
-                   "l2": "inputs larger than L2 (28 layers of K/V = "
+        "config": {"workload": describe(name, wl, t), "layers": L, "N": N, "t": t,
+                   "l2": f"inputs larger than L2 ({L} layers of K/V = "
                          f"{sum(k.numel() for k in Ks) * 4 / 1e6:.0f} MB per step)"},
         "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
@@ -356,6 +487,7 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cb = run_cpu_baseline(wl, t)
         cb.pop("seconds", None)
+        cb.pop("scale", None)
         line["cpu_baseline"] = cb
     if rank == 0:
         print(json.dumps(line))

@@ -107,10 +107,14 @@ struct EpiAffine {
   int32_t ss_parts = 2;    // slots per vector = 2 * ss_seg / tile width
   int64_t split_stride = 0;
   int32_t vec_ok = 0;  // host: om.c0 == 1, cdiv % 32 == 0, 16-B aligned rows
+  // OUT_F32 through TMA stores: the output is the 3-D view (col, row, batch) given to the
+  // launcher (boxes of 32 x 32 fp32, 128-byte swizzled staging); rows / columns past the view
+  // are clipped by the copy engine.
+  int32_t tma_f32 = 0;
   int32_t tile_cols_ = 256;  // the tile width BN, set by the launcher
 
   __device__ void operator()(const GemmParams& p, const TileCoord& tc, int row, uint32_t taddr,
-                             int half, uint4* stage) const {
+                             int half, uint4* stage, const CUtensorMap* tmc) const {
     const int r = tc.tm * kBM + row;
     const bool rvalid = r < p.M;
     float rscale = alpha;
@@ -124,8 +128,11 @@ struct EpiAffine {
       const int nv = min(32, p.N - c0);
 #pragma unroll
       for (int e = 0; e < 32; ++e) v[e] *= rscale;
-      if (!rvalid) {
-        store32(p, tc.b, r, c0, v, tc.split, false, stage);  // keeps the warp collective
+      if (!rvalid) {  // keep the warp-collective stores; the row itself is not written
+        if (tma_f32)
+          store32_tma(tc, row, c0, v, stage, tmc);
+        else
+          store32(p, tc.b, r, c0, v, tc.split, false, stage);
         continue;
       }
       if (col_scale != nullptr) {
@@ -162,12 +169,35 @@ struct EpiAffine {
             if (e < nv) v[e] += __bfloat162float(rp[e]);
         }
       }
-      store32(p, tc.b, r, c0, v, tc.split, rvalid, stage);
+      if (tma_f32)
+        store32_tma(tc, row, c0, v, stage, tmc);
+      else
+        store32(p, tc.b, r, c0, v, tc.split, rvalid, stage);
     }
     if (sumsq != nullptr && rvalid) {
       const int c_tile = tc.tn * tile_cols_;
       const int slot = ((c_tile % ss_seg) / tile_cols_) * 2 + half;
       sumsq[ssm.at(tc.b, r, c_tile / ss_seg) * ss_parts + slot] = ss;
+    }
+  }
+
+  // Warp-collective: this warp's 32 rows x 32 fp32 columns as one TMA box.
+  __device__ __forceinline__ void store32_tma(const TileCoord& tc, int row, int c0,
+                                              const float (&v)[32], uint4* stage,
+                                              const CUtensorMap* tmc) const {
+    const int lane = threadIdx.x & 31;
+    if (lane == 0) bulk_wait_read();  // the previous box has left the staging area
+    __syncwarp();
+    uint4* my = stage + lane * 8;  // 128 B per row; 16-B chunk q lands at q ^ (row & 7)
+#pragma unroll
+    for (int q = 0; q < 8; ++q)
+      my[q ^ (lane & 7)] = make_uint4(__float_as_uint(v[4 * q]), __float_as_uint(v[4 * q + 1]),
+                                      __float_as_uint(v[4 * q + 2]), __float_as_uint(v[4 * q + 3]));
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_3d(tmc, stage, c0, tc.tm * kBM + row, tc.b);
+      bulk_commit();
     }
   }
 
@@ -246,7 +276,7 @@ struct EpiRopeC {
   static constexpr int kWarps = 16;
   static constexpr int kParts = kWarps / 4;
   static constexpr int kStages = 3;
-  __nv_bfloat16* out = nullptr;  // [H][n][N][2D]: hi at [0, D), lo at [D, 2D)
+  __nv_bfloat16* out = nullptr;  // [H][n][N][2D]: hi at [0, D), lo at [D, 2D) (via the TMA view)
   float* sumsq = nullptr;        // [H][n][N][kParts * D / 256] partial sums of |k~|^2
   const float* bias = nullptr;   // [n*D], pair-chunk order
   const float2* coarse = nullptr;  // [G][D/2]: (cos, sin)(G_g * omega_m)
@@ -258,9 +288,11 @@ struct EpiRopeC {
   int32_t tile_cols_ = 256;  // must be 256: a tile holds 128 whole RoPE pairs
 
   __device__ void operator()(const GemmParams& p, const TileCoord& tc, int row, uint32_t taddr,
-                             int half, uint4* stage) const {
+                             int half, uint4* stage, const CUtensorMap* tmc) const {
     const int r = tc.tm * kBM + row;
     const bool rvalid = r < p.M;
+    const int lane = threadIdx.x & 31;
+    const int row0 = tc.tm * kBM + row - lane;  // first token row of this warp
     const int c_tile = tc.tn * 256;
     const int head = c_tile / D;
     const int f_tile = c_tile % D;       // column of this tile inside the head (pair-chunk order)
@@ -269,8 +301,6 @@ struct EpiRopeC {
     int g = (int)floor((pos - pmin) / (double)kPosGrain);
     g = max(0, min(g, ncoarse - 1));
     const float delta = (float)(pos - (pmin + (double)g * kPosGrain));
-    const int64_t row_out = ((int64_t)(tc.b * nheads + head) * Ntok + (rvalid ? r : 0)) *
-                            (2 * (int64_t)D);
     float ss = 0.f;
     // part p owns pairs [32p, 32p + 32) of the tile, taken 16 at a time
     for (int u = 32 * half; u < 32 * half + 32; u += 16) {
@@ -304,29 +334,35 @@ struct EpiRopeC {
           bb[e] = x * sw + y * cw;
         }
       }
-      __nv_bfloat16* o = out + row_out + f_tile + u;
-      uint4 h2[2], l2[2];
+      // Four boxes of 32 rows x 16 bf16 (hi a, lo a, hi b, lo b), 1 KB each, stored by TMA;
+      // rows past N are clipped by the copy engine.
+      if (lane == 0) bulk_wait_read();
+      __syncwarp();
+      uint4* box = stage + lane * 2;
 #pragma unroll
       for (int q = 0; q < 2; ++q) {
         uint32_t h[4], l[4];
 #pragma unroll
         for (int k = 0; k < 4; ++k) split_pack(a[8 * q + 2 * k], a[8 * q + 2 * k + 1], h[k], l[k]);
-        h2[q] = make_uint4(h[0], h[1], h[2], h[3]);
-        l2[q] = make_uint4(l[0], l[1], l[2], l[3]);
-      }
-      warp_store32(stage, h2, o, rvalid);
-      warp_store32(stage, l2, o + D, rvalid);
-#pragma unroll
-      for (int q = 0; q < 2; ++q) {
-        uint32_t h[4], l[4];
+        box[q] = make_uint4(h[0], h[1], h[2], h[3]);
+        box[64 + q] = make_uint4(l[0], l[1], l[2], l[3]);
 #pragma unroll
         for (int k = 0; k < 4; ++k)
           split_pack(bb[8 * q + 2 * k], bb[8 * q + 2 * k + 1], h[k], l[k]);
-        h2[q] = make_uint4(h[0], h[1], h[2], h[3]);
-        l2[q] = make_uint4(l[0], l[1], l[2], l[3]);
+        box[128 + q] = make_uint4(h[0], h[1], h[2], h[3]);
+        box[192 + q] = make_uint4(l[0], l[1], l[2], l[3]);
       }
-      warp_store32(stage, h2, o + 128, rvalid);
-      warp_store32(stage, l2, o + D + 128, rvalid);
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        const int z = tc.b * nheads + head;
+        const int x = f_tile + u;
+        tma_store_3d(tmc, stage, x, row0, z);
+        tma_store_3d(tmc, stage + 64, D + x, row0, z);
+        tma_store_3d(tmc, stage + 128, x + 128, row0, z);
+        tma_store_3d(tmc, stage + 192, D + x + 128, row0, z);
+        bulk_commit();
+      }
     }
     if (rvalid) {
       const int parts = kParts * (D / 256);
@@ -353,7 +389,7 @@ struct EpiHeads {
   int32_t tile_cols_ = 256;
 
   __device__ void operator()(const GemmParams& p, const TileCoord& tc, int row, uint32_t taddr,
-                             int half, uint4* stage) const {
+                             int half, uint4* stage, const CUtensorMap*) const {
     const int r = tc.tm * kBM + row;
     const bool rvalid = r < p.M;
     const int h = rvalid ? r / t : 0, j = rvalid ? r % t : 0;

@@ -4,6 +4,7 @@
 #include <cudaTypedefs.h>
 
 #include <cstdio>
+#include <cstring>
 #include <mutex>
 
 #include "epilogues.cuh"
@@ -29,6 +30,34 @@ inline PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
       fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
   });
   return fn;
+}
+
+// A 3-D destination for TMA stores: element (x, y, z) at base + z * zstride + y * ystride + x
+// (elements), extents (nx, ny, nz); boxes of bx x 32 x 1, optionally 128-byte swizzled.
+struct StoreView3D {
+  void* ptr = nullptr;
+  int elem_bytes = 2;
+  int64_t nx = 0, ny = 0, nz = 1, ystride = 0, zstride = 0;
+  int bx = 32;
+  bool swizzle128 = false;
+};
+
+inline bool make_store_tmap(CUtensorMap* m, const StoreView3D& v) {
+  auto enc = tensor_map_encoder();
+  if (enc == nullptr) return false;
+  const int64_t eb = v.elem_bytes;
+  if ((reinterpret_cast<uintptr_t>(v.ptr) & 15) != 0 || (v.ystride * eb) % 16 != 0 ||
+      (v.zstride * eb) % 16 != 0 || (v.bx * eb) % 16 != 0)
+    return false;
+  cuuint64_t dims[3] = {(cuuint64_t)v.nx, (cuuint64_t)v.ny, (cuuint64_t)v.nz};
+  cuuint64_t strides[2] = {(cuuint64_t)(v.ystride * eb), (cuuint64_t)(v.zstride * eb)};
+  cuuint32_t box[3] = {(cuuint32_t)v.bx, 32, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = enc(m, eb == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                   3, v.ptr, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                   v.swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                   CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
 }
 
 // Box = box_rows x 64 elements, 128-byte swizzle, zero fill out of bounds.
@@ -72,11 +101,14 @@ inline bool finalize_gemm(GemmParams& p, int ab_fmt) {
 
 template <int BN, int kRole, class Epi>
 inline cudaError_t launch_gemm(const Operand2D& A, const Operand2D& B, GemmParams p, Epi epi,
-                               int ab_fmt, int num_sms, cudaStream_t stream) {
+                               int ab_fmt, int num_sms, cudaStream_t stream,
+                               const StoreView3D* out_view = nullptr) {
   using S = GemmSmem<BN, Epi>;
   if (!finalize_gemm<BN>(p, ab_fmt)) return cudaErrorInvalidValue;
-  CUtensorMap ta, tb;
+  CUtensorMap ta, tb, tc;
   if (!make_tmap(&ta, A, kBM) || !make_tmap(&tb, B, BN)) return cudaErrorInvalidValue;
+  std::memset(&tc, 0, sizeof(tc));
+  if (out_view != nullptr && !make_store_tmap(&tc, *out_view)) return cudaErrorInvalidValue;
   epi.tile_cols_ = BN;
   auto kern = tc_gemm_kernel<BN, Epi, kRole>;
   static thread_local bool attr_set = false;  // per instantiation
@@ -87,7 +119,7 @@ inline cudaError_t launch_gemm(const Operand2D& A, const Operand2D& B, GemmParam
     attr_set = true;
   }
   const int grid = p.ntiles < num_sms ? p.ntiles : num_sms;
-  kern<<<grid, gemm_threads<Epi>(), S::kBytes, stream>>>(ta, tb, p, epi);
+  kern<<<grid, gemm_threads<Epi>(), S::kBytes, stream>>>(ta, tb, tc, p, epi);
   return cudaGetLastError();
 }
 

@@ -195,10 +195,11 @@ Operand2D op(const void* ptr, int64_t rows, int64_t cols, int64_t pitch = -1) {
 // One GEMM of the launch sequence; CLS is its kernel class (profiling and kernel name).
 template <int CLS, int BN, class Epi>
 still_status run_gemm_bn(still_ctx* ctx, const Operand2D& A, const Operand2D& B, GemmParams p,
-                         const Epi& e, int ab_fmt, cudaStream_t s) {
+                         const Epi& e, int ab_fmt, cudaStream_t s,
+                         const StoreView3D* view = nullptr) {
   p.err = ctx->err;
   ctx->prof.begin(CLS, s);
-  cudaError_t r = launch_gemm<BN, CLS>(A, B, p, e, ab_fmt, ctx->nsm, s);
+  cudaError_t r = launch_gemm<BN, CLS>(A, B, p, e, ab_fmt, ctx->nsm, s, view);
   ctx->prof.end(CLS, s);
   if (r == cudaErrorInvalidValue) return STILL_ERR_INVALID_ARG;
   return r == cudaSuccess ? STILL_OK : STILL_ERR_CUDA;
@@ -213,8 +214,24 @@ still_status run_gemm(still_ctx* ctx, int bn, const Operand2D& A, const Operand2
 
 template <int CLS, class Epi>
 still_status run_gemm256(still_ctx* ctx, const Operand2D& A, const Operand2D& B, GemmParams p,
-                         const Epi& e, int ab_fmt, cudaStream_t s) {
-  return run_gemm_bn<CLS, 256>(ctx, A, B, p, e, ab_fmt, s);
+                         const Epi& e, int ab_fmt, cudaStream_t s,
+                         const StoreView3D* view = nullptr) {
+  return run_gemm_bn<CLS, 256>(ctx, A, B, p, e, ab_fmt, s, view);
+}
+
+StoreView3D store_view(void* ptr, int elem_bytes, int64_t nx, int64_t ny, int64_t nz,
+                       int64_t ystride, int64_t zstride, int bx, bool swz) {
+  StoreView3D v;
+  v.ptr = ptr;
+  v.elem_bytes = elem_bytes;
+  v.nx = nx;
+  v.ny = ny;
+  v.nz = nz;
+  v.ystride = ystride;
+  v.zstride = zstride;
+  v.bx = bx;
+  v.swizzle128 = swz;
+  return v;
 }
 
 // Launch of one of the memory-bound kernels, timed under its class.
@@ -475,8 +492,9 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.nheads = ni;
       e.ncoarse = P.G;
       e.Ntok = N;
+      const StoreView3D kv = store_view(kb, 2, 2 * D, N, nbl, 2 * D, N * 2 * D, 16, false);
       TRY(run_gemm256<STILL_K_KEYPROJ>(ctx, op(X, (int64_t)H * N, 3 * d), op(L.WkT, (int64_t)n * D, 2 * d), p, e,
-                   1, s));
+                   1, s, &kv));
     }
     // scale / |k~_n| per key (the d_l logit scale folded in)
     KLAUNCH(STILL_K_NORMS, launch_inv_norms(kss, (int64_t)nbl * N, kparts, c.l2_eps, scale, kinv, s));
@@ -499,8 +517,10 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.csm.b1 = N;
       e.csm.c0 = 1;
       e.vec_ok = 1;
+      e.tma_f32 = 1;
+      const StoreView3D sv = store_view(S, 4, N, t, nbl, P.ldS, (int64_t)t * P.ldS, 32, true);
       TRY(run_gemm256<STILL_K_SCORES>(ctx, op(qhl, (int64_t)nbl * t, 2 * D), op(kb, (int64_t)nbl * N, 2 * D), p,
-                   e, 1, s));
+                   e, 1, s, &sv));
     }
     KLAUNCH(STILL_K_SOFTMAX, launch_softmax(S, (int64_t)nbl * t, N, P.ldS, Pm, Np, 1, s));
     int px_split = 1;
@@ -644,8 +664,11 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.csm.c0 = 1;
       e.csm.k = (int64_t)n * t;
       e.vec_ok = 1;
+      e.tma_f32 = 1;
+      const StoreView3D sv = store_view(Ssa, 4, t, t, (int64_t)nh * n, P.ldt, (int64_t)t * P.ldt,
+                                        32, true);
       TRY(run_gemm256<STILL_K_SA_SCORES>(ctx, op(qk, (int64_t)nh * 2 * n * t, 2 * D),
-                   op(qk, (int64_t)nh * 2 * n * t, 2 * D), p, e, 1, s));
+                   op(qk, (int64_t)nh * 2 * n * t, 2 * D), p, e, 1, s, &sv));
     }
     KLAUNCH(STILL_K_SA_SOFTMAX, launch_softmax(Ssa, (int64_t)nh * n * t, t, P.ldt, Psa, P.tp, 0, s));
     {  // heads = P v -> concat rows (h0 + hh) * t + j, columns i * D + f

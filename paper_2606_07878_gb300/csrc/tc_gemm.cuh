@@ -67,9 +67,10 @@ __device__ __forceinline__ void split_range(const GemmParams& p, int split, int&
   it1 = (int)(((int64_t)p.iters_total * (split + 1)) / p.ksplit);
 }
 
-// Per-epilogue-warp staging area for coalesced stores: 32 rows x 64 B, rows 80 B apart.
+// Per-epilogue-warp staging area (1024-byte aligned): 32 rows x 64 B for the LSU path (rows
+// 80 B apart), or one TMA-store box of up to 4 KB.
 constexpr int kStageRowU4 = 5;
-constexpr int kWarpStageBytes = 32 * kStageRowU4 * 16;
+constexpr int kWarpStageBytes = 4096;
 
 template <int BN, class Epi>
 struct GemmSmem {
@@ -77,7 +78,7 @@ struct GemmSmem {
   static constexpr int kABytes = kBM * kBK * 2;
   static constexpr int kBBytes = BN * kBK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
-  static constexpr int kEpiOffset = kStages * kStageBytes;
+  static constexpr int kEpiOffset = kStages * kStageBytes;  // a multiple of 1024
   static constexpr int kBarOffset = kEpiOffset + Epi::kWarps * kWarpStageBytes;
   static constexpr int kBytes = kBarOffset + 256 + 1024;  // + barriers + alignment slack
   static_assert(kBytes <= 232448, "shared memory budget");
@@ -123,7 +124,7 @@ __device__ __forceinline__ void warp_store64(uint4* stage, const uint4 (&v)[4], 
 
 // Epi must provide:  __device__ void operator()(const GemmParams&, const TileCoord&,
 //                    int row_in_tile, uint32_t tmem_addr_of_this_warp_lane_quarter,
-//                    int half, uint4* warp_stage) const;
+//                    int half, uint4* warp_stage, const CUtensorMap* out_map) const;
 // where `half` (0 or 1) selects the 32-column chunks this warp owns: chunk c is handled by the
 // warp with half == (c & 1); the functor loads TMEM and stores its own results.
 // kRole only names the instantiation (one per GEMM of the launch sequence) so that profilers
@@ -131,7 +132,8 @@ __device__ __forceinline__ void warp_store64(uint4* stage, const uint4 (&v)[4], 
 template <int BN, class Epi, int kRole>
 __global__ void __launch_bounds__(gemm_threads<Epi>(), 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
-                   const __grid_constant__ CUtensorMap tmB, const GemmParams p, const Epi epi) {
+                   const __grid_constant__ CUtensorMap tmB,
+                   const __grid_constant__ CUtensorMap tmC, const GemmParams p, const Epi epi) {
   using S = GemmSmem<BN, Epi>;
   constexpr int kEpiWarps = Epi::kWarps;
   constexpr int kStages = S::kStages;
@@ -294,7 +296,7 @@ __global__ void __launch_bounds__(gemm_threads<Epi>(), 1)
       }
       tc_fence_after();
       const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * BN);
-      epi(p, tc, row, taddr, half, stage);
+      epi(p, tc, row, taddr, half, stage, &tmC);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);
@@ -303,6 +305,7 @@ __global__ void __launch_bounds__(gemm_threads<Epi>(), 1)
         acc_phase ^= 1;
       }
     }
+    if (lane == 0) bulk_wait_all();  // TMA stores issued by this warp (if any) have landed
   }
 
   tc_fence_before();
