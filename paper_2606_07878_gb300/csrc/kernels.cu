@@ -21,97 +21,104 @@ __device__ __forceinline__ void sincos_reduced(double ang, float* s, float* c) {
 
 constexpr int kStripTok = 32;
 
-// One CTA = 32 tokens x one KV-head. Keys: inverse base-model RoPE on pairs (m, m + d/2)
-// (Sec. 2.2, RoPE-fix); values pass through. Writes X (bf16 hi | key lo) and XT (fp16 hi, lo).
 __device__ __forceinline__ int64_t kv_offset(const KVSource& src, int64_t n, int h, bool& second) {
   second = n >= src.n_split;
   return second ? (n - src.n_split) * src.sN2 + (int64_t)h * src.sH2
                 : n * src.sN + (int64_t)h * src.sH;
 }
 
+// One CTA = 32 tokens x all KV-heads. The base-RoPE angles of the tile's tokens are formed
+// once (fp64, reduced mod 2 pi) and reused by every KV-head. Keys: inverse rotation of pairs
+// (m, m + d/2) (Sec. 2.2, RoPE-fix); values pass through. Writes X (bf16 hi | key lo) and XT
+// (fp16 hi, lo).
 __global__ void __launch_bounds__(256) strip_kernel(KVSource src, int64_t N, int H, int d,
-                                                    PosSegs segs, double theta, int rope_fix,
-                                                    __nv_bfloat16* __restrict__ X,
+                                                    PosSegs segs, const double* __restrict__ omega,
+                                                    int rope_fix, __nv_bfloat16* __restrict__ X,
                                                     __half* __restrict__ XT, int64_t Np) {
   extern __shared__ __align__(16) uint8_t sm[];
   const int half = d / 2;
-  double* omega = reinterpret_cast<double*>(sm);
   constexpr int kLd = kStripTok + 2;
-  __half* thi = reinterpret_cast<__half*>(omega + half);
+  float2* rot = reinterpret_cast<float2*>(sm);              // [kStripTok][half]: (cos, sin)
+  __half* thi = reinterpret_cast<__half*>(rot + kStripTok * half);
   __half* tlo = thi + 2 * d * kLd;
-  const int h = blockIdx.y;
   const int64_t n0 = (int64_t)blockIdx.x * kStripTok;
-  for (int m = threadIdx.x; m < half; m += blockDim.x) omega[m] = pow(theta, -2.0 * m / d);
-  __syncthreads();
-  const int d3 = 3 * d;
   for (int it = threadIdx.x; it < kStripTok * half; it += blockDim.x) {
     const int tok = it / half, m = it % half;
     const int64_t n = n0 + tok;
-    float a = 0.f, b = 0.f;
-    if (n < N) {
-      bool second;
-      const int64_t off = kv_offset(src, n, h, second);
-      const __nv_bfloat16* kr = (second ? src.K2 : src.K) + off;
-      a = __bfloat162float(kr[m]);
-      b = __bfloat162float(kr[m + half]);
-      if (rope_fix) {
-        float sw, cw;
-        sincos_reduced(seg_position(segs, n) * omega[m], &sw, &cw);
-        const float x = a * cw + b * sw;
-        const float y = -a * sw + b * cw;
-        a = x;
-        b = y;
-      }
-      __nv_bfloat16* xr = X + ((int64_t)h * N + n) * d3;
-      __nv_bfloat16 hi, lo;
-      split_hilo(a, hi, lo);
-      xr[m] = hi;
-      xr[2 * d + m] = lo;
-      split_hilo(b, hi, lo);
-      xr[m + half] = hi;
-      xr[2 * d + m + half] = lo;
-    }
-    const __half ah = __float2half_rn(a), bh = __float2half_rn(b);
-    thi[m * kLd + tok] = ah;
-    thi[(m + half) * kLd + tok] = bh;
-    tlo[m * kLd + tok] = __float2half_rn(a - __half2float(ah));
-    tlo[(m + half) * kLd + tok] = __float2half_rn(b - __half2float(bh));
-  }
-  for (int it = threadIdx.x; it < kStripTok * d; it += blockDim.x) {
-    const int tok = it / d, f = it % d;
-    const int64_t n = n0 + tok;
-    float v = 0.f;
-    if (n < N) {
-      bool second;
-      const int64_t off = kv_offset(src, n, h, second);
-      const __nv_bfloat16 vb = (second ? src.V2 : src.V)[off + f];
-      v = __bfloat162float(vb);
-      X[((int64_t)h * N + n) * d3 + d + f] = vb;
-    }
-    const __half vh = __float2half_rn(v);
-    thi[(d + f) * kLd + tok] = vh;
-    tlo[(d + f) * kLd + tok] = __float2half_rn(v - __half2float(vh));
+    float sw = 0.f, cw = 1.f;
+    if (rope_fix && n < N) sincos_reduced(seg_position(segs, n) * omega[m], &sw, &cw);
+    rot[it] = make_float2(cw, sw);
   }
   __syncthreads();
+  const int d3 = 3 * d;
   const int64_t ld = 2 * Np;
-  for (int it = threadIdx.x; it < 2 * d * kStripTok; it += blockDim.x) {
-    const int f = it / kStripTok, tok = it % kStripTok;
-    const int64_t n = n0 + tok;
-    if (n < Np) {
-      __half* row = XT + ((int64_t)h * 2 * d + f) * ld;
-      row[n] = thi[f * kLd + tok];
-      row[Np + n] = tlo[f * kLd + tok];
+  for (int h = 0; h < H; ++h) {
+    for (int it = threadIdx.x; it < kStripTok * half; it += blockDim.x) {
+      const int tok = it / half, m = it % half;
+      const int64_t n = n0 + tok;
+      float a = 0.f, b = 0.f;
+      if (n < N) {
+        bool second;
+        const int64_t off = kv_offset(src, n, h, second);
+        const __nv_bfloat16* kr = (second ? src.K2 : src.K) + off;
+        a = __bfloat162float(kr[m]);
+        b = __bfloat162float(kr[m + half]);
+        const float2 cs = rot[it];
+        const float x = a * cs.x + b * cs.y;
+        const float y = -a * cs.y + b * cs.x;
+        a = x;
+        b = y;
+        __nv_bfloat16* xr = X + ((int64_t)h * N + n) * d3;
+        __nv_bfloat16 hi, lo;
+        split_hilo(a, hi, lo);
+        xr[m] = hi;
+        xr[2 * d + m] = lo;
+        split_hilo(b, hi, lo);
+        xr[m + half] = hi;
+        xr[2 * d + m + half] = lo;
+      }
+      const __half ah = __float2half_rn(a), bh = __float2half_rn(b);
+      thi[m * kLd + tok] = ah;
+      thi[(m + half) * kLd + tok] = bh;
+      tlo[m * kLd + tok] = __float2half_rn(a - __half2float(ah));
+      tlo[(m + half) * kLd + tok] = __float2half_rn(b - __half2float(bh));
     }
+    for (int it = threadIdx.x; it < kStripTok * d; it += blockDim.x) {
+      const int tok = it / d, f = it % d;
+      const int64_t n = n0 + tok;
+      float v = 0.f;
+      if (n < N) {
+        bool second;
+        const int64_t off = kv_offset(src, n, h, second);
+        const __nv_bfloat16 vb = (second ? src.V2 : src.V)[off + f];
+        v = __bfloat162float(vb);
+        X[((int64_t)h * N + n) * d3 + d + f] = vb;
+      }
+      const __half vh = __float2half_rn(v);
+      thi[(d + f) * kLd + tok] = vh;
+      tlo[(d + f) * kLd + tok] = __float2half_rn(v - __half2float(vh));
+    }
+    __syncthreads();
+    for (int it = threadIdx.x; it < 2 * d * kStripTok; it += blockDim.x) {
+      const int f = it / kStripTok, tok = it % kStripTok;
+      const int64_t n = n0 + tok;
+      if (n < Np) {
+        __half* row = XT + ((int64_t)h * 2 * d + f) * ld;
+        row[n] = thi[f * kLd + tok];
+        row[Np + n] = tlo[f * kLd + tok];
+      }
+    }
+    __syncthreads();
   }
 }
 
 __global__ void rope_tables_kernel(float2* coarse, float* omega, int G, int D, double pmin,
-                                   double theta_c) {
+                                   const double* __restrict__ omega_c) {
   const int half = D / 2;
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (int64_t)G * half) return;
   const int g = (int)(idx / half), m = (int)(idx % half);
-  const double w = pow(theta_c, -2.0 * m / D);
+  const double w = omega_c[m];
   float s, c;
   sincos_reduced((pmin + (double)g * kPosGrain) * w, &s, &c);
   coarse[idx] = make_float2(c, s);
@@ -275,6 +282,21 @@ __global__ void __launch_bounds__(256) softmax_reg_kernel(const float* __restric
   }
 }
 
+// Row softmax statistics from per-tile partials (m_p, l_p = sum exp(v - m_p)):
+// out[row] = (M * log2 e, 1 / L), M = max_p m_p, L = sum_p l_p exp(m_p - M), fixed order.
+__global__ void row_stats_kernel(const float2* __restrict__ parts, int64_t rows, int slots,
+                                 float2* __restrict__ out) {
+  const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= rows) return;
+  const float2* p = parts + r * slots;
+  float M = -INFINITY;
+  for (int k = 0; k < slots; ++k) M = fmaxf(M, p[k].x);
+  float L = 0.f;
+  for (int k = 0; k < slots; ++k)
+    if (p[k].x != -INFINITY) L += p[k].y * exp2f((p[k].x - M) * kLog2e);
+  out[r] = make_float2(M * kLog2e, 1.f / L);
+}
+
 __global__ void omega_kernel(double* out, int half, int width, double base) {
   const int m = blockIdx.x * blockDim.x + threadIdx.x;
   if (m < half) out[m] = pow(base, -2.0 * m / width);
@@ -380,23 +402,24 @@ inline unsigned blocks_for(int64_t n, int per) { return (unsigned)((n + per - 1)
 }  // namespace
 
 cudaError_t launch_strip(const KVSource& src, int64_t N, int H, int d, const PosSegs& segs,
-                         double theta, int rope_fix, __nv_bfloat16* X, __half* XT, int64_t Np,
-                         cudaStream_t s) {
-  const size_t smem = (size_t)(d / 2) * sizeof(double) + 2 * (size_t)(2 * d) * (kStripTok + 2) * 2;
+                         const double* omega, int rope_fix, __nv_bfloat16* X, __half* XT,
+                         int64_t Np, cudaStream_t s) {
+  const size_t smem = (size_t)kStripTok * (d / 2) * sizeof(float2) +
+                      2 * (size_t)(2 * d) * (kStripTok + 2) * 2;
   static bool attr = false;
   if (!attr) {
-    cudaFuncSetAttribute(strip_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024);
+    cudaFuncSetAttribute(strip_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 128 * 1024);
     attr = true;
   }
-  dim3 grid((unsigned)(Np / kStripTok), (unsigned)H);
-  strip_kernel<<<grid, 256, smem, s>>>(src, N, H, d, segs, theta, rope_fix, X, XT, Np);
+  strip_kernel<<<(unsigned)(Np / kStripTok), 256, smem, s>>>(src, N, H, d, segs, omega, rope_fix,
+                                                             X, XT, Np);
   return cudaGetLastError();
 }
 
 cudaError_t launch_rope_tables(float2* coarse, float* omega, int G, int D, double pmin,
-                               double theta_c, cudaStream_t s) {
+                               const double* omega_c, cudaStream_t s) {
   const int64_t n = (int64_t)G * (D / 2);
-  rope_tables_kernel<<<blocks_for(n, 256), 256, 0, s>>>(coarse, omega, G, D, pmin, theta_c);
+  rope_tables_kernel<<<blocks_for(n, 256), 256, 0, s>>>(coarse, omega, G, D, pmin, omega_c);
   return cudaGetLastError();
 }
 
@@ -428,6 +451,12 @@ static bool softmax_reg(const float* S, int64_t rows, int64_t ncols, int64_t ldS
   else
     return false;
   return true;
+}
+
+cudaError_t launch_row_stats(const float2* parts, int64_t rows, int slots, float2* out,
+                             cudaStream_t s) {
+  row_stats_kernel<<<blocks_for(rows, 256), 256, 0, s>>>(parts, rows, slots, out);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_omega(double* out, int half, int width, double base, cudaStream_t s) {

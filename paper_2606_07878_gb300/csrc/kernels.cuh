@@ -23,14 +23,15 @@ struct KVSource {
 //   X[h, n]  = [unRoPE(K[n, h]) | V[n, h]]  as bf16 hi (2d) + bf16 lo of the key half (d)
 //   XT[h]    = X[h]^T as fp16 hi / lo, token-contiguous, tokens padded with zeros to Np.
 // X:  [H*N][3d] bf16.  XT: [H*2d][2*Np] fp16 (hi at [0, Np), lo at [Np, 2Np)).
+// omega: [d/2] fp64 base-model frequencies theta^(-2m/d).
 cudaError_t launch_strip(const KVSource& src, int64_t N, int H, int d, const PosSegs& segs,
-                         double theta, int rope_fix, __nv_bfloat16* X, __half* XT, int64_t Np,
-                         cudaStream_t s);
+                         const double* omega, int rope_fix, __nv_bfloat16* X, __half* XT,
+                         int64_t Np, cudaStream_t s);
 
 // Compactor-RoPE tables: coarse[g][m] = (cos, sin)((pmin + g * kPosGrain) * w_m), omega[m] = w_m
-// (fp32), w_m = theta_c^(-2m/D), angles reduced in fp64.
+// (fp32), w_m = omega_c[m] = theta_c^(-2m/D) (fp64 table), angles reduced in fp64.
 cudaError_t launch_rope_tables(float2* coarse, float* omega, int G, int D, double pmin,
-                               double theta_c, cudaStream_t s);
+                               const double* omega_c, cudaStream_t s);
 
 // Per-call cross-attention queries: q = RoPE_c(q^, p_j) for latents j < t, batches
 // b in [b0, b0 + nb) (b = h * n + i), as hi/lo bf16 [nb * t][2D]. q^ is [H*n][t_max][D] fp32
@@ -38,6 +39,11 @@ cudaError_t launch_rope_tables(float2* coarse, float* omega, int G, int D, doubl
 cudaError_t launch_q_rope(const float* qhat, int t_max, int b0, int nb, int t, int D,
                           double qstart, double qstep, const double* omega_c, int use_rope,
                           __nv_bfloat16* qhl, cudaStream_t s);
+
+// Row softmax statistics from the scores epilogue's per-tile partials (max, sum of exp):
+// out[row] = (M * log2 e, 1 / L) with M the row max and L the sum of exp(s - M).
+cudaError_t launch_row_stats(const float2* parts, int64_t rows, int slots, float2* out,
+                             cudaStream_t s);
 
 // out[m] = base^(-2m / width) in fp64, m < half.
 cudaError_t launch_omega(double* out, int half, int width, double base, cudaStream_t s);

@@ -23,6 +23,7 @@
 #include "../../include/still.h"
 #include "gemm_host.cuh"
 #include "kernels.cuh"
+#include "px_fused.cuh"
 
 using namespace still;
 
@@ -313,7 +314,7 @@ bool make_plan(const still_layer_config& c, int64_t N, int t, double pmin, doubl
   P.kss_b = a256(N * 4 * (EpiRopeC::kParts * (D / 256) + 1));  // |k~|^2 partials + inverses
   P.q_b = a256(T * 2 * D * 2);
   P.S_b = a256(T * P.ldS * 4);
-  P.P_b = a256(T * P.Np * 2);
+  P.P_b = a256(T * 8 * (2 * ((N + 255) / 256) + 1));  // row-softmax partials + statistics
   P.O_b = a256(T * 2 * d * 4) * kMaxSplit;       // split-K partials of P X
   P.ca_unit_bytes = P.kb_b + P.kss_b + P.q_b + P.S_b + P.P_b + P.O_b;
   P.qk_b = a256(2 * n * T * 2 * D * 2);
@@ -443,8 +444,8 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
   bf16* Gb = reinterpret_cast<bf16*>(ws + P.oG);
   void* Z3 = ws + P.oZ3;
 
-  KLAUNCH(STILL_K_STRIP, launch_strip(src, N, H, d, pos.segs, c.rope_theta, c.rope_fix, X, XT, Np, s));
-  KLAUNCH(STILL_K_TABLES, launch_rope_tables(coarse, omega, P.G, D, pos.pmin, c.rope_theta_compactor, s));
+  KLAUNCH(STILL_K_STRIP, launch_strip(src, N, H, d, pos.segs, L.omega_b, c.rope_fix, X, XT, Np, s));
+  KLAUNCH(STILL_K_TABLES, launch_rope_tables(coarse, omega, P.G, D, pos.pmin, L.omega_c, s));
 
   // ---------------------------------------------------------------- cross-attention groups
   const int units_total = H * n;
@@ -471,7 +472,9 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     g += P.q_b * nbl;
     float* S = reinterpret_cast<float*>(g);
     g += P.S_b * nbl;
-    __half* Pm = reinterpret_cast<__half*>(g);
+    const int stat_slots = 2 * (int)((N + 255) / 256);
+    float2* stp = reinterpret_cast<float2*>(g);                      // [nbl * t][stat_slots]
+    float2* rstat = stp + (size_t)nbl * t * stat_slots;               // [nbl * t]
     g += P.P_b * nbl;
     float* O = reinterpret_cast<float*>(g);
     // keyproj: rows = tokens of heads [h0, h0+nh), columns = cross heads [i0, i0+ni)
@@ -518,25 +521,36 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.csm.c0 = 1;
       e.vec_ok = 1;
       e.tma_f32 = 1;
+      e.stat_out = stp;
+      e.stat_slots = stat_slots;
       const StoreView3D sv = store_view(S, 4, N, t, nbl, P.ldS, (int64_t)t * P.ldS, 32, true);
       TRY(run_gemm256<STILL_K_SCORES>(ctx, op(qhl, (int64_t)nbl * t, 2 * D), op(kb, (int64_t)nbl * N, 2 * D), p,
                    e, 1, s, &sv));
     }
-    KLAUNCH(STILL_K_SOFTMAX, launch_softmax(S, (int64_t)nbl * t, N, P.ldS, Pm, Np, 1, s));
+    KLAUNCH(STILL_K_SOFTMAX, launch_row_stats(stp, (int64_t)nbl * t, stat_slots, rstat, s));
     int px_split = 1;
     const int64_t px_stride = (int64_t)nbl * t * 2 * d;
-    {  // O = P X  (fp16 operands, X hi + X lo), split-K partials reduced in order below
+    {  // O = softmax(S) X: probabilities formed on the fly (fp16), X hi + key-half lo passes
       GemmParams p = gp(t, 2 * d, nbl, ni);
-      p.a_r1 = (int64_t)ni * t;
-      p.a_r0 = t;
-      p.b_r1 = 2 * d;
-      add_pass(p, 0, 0, 0, h0 * 2 * d, (int)Np);
-      add_pass(p, 0, (int)Np, 0, h0 * 2 * d, (int)Np);
+      add_pass(p, 0, 0, 0, 0, (int)Np);
       const int bn = 2 * d <= 128 ? 128 : 256;
       const int64_t tiles = (int64_t)((t + 127) / 128) * ((2 * d + bn - 1) / bn) * nbl;
-      p.ksplit = std::min(auto_split(tiles, (int)(2 * Np / 64), ctx->nsm), kMaxSplit);
-      p.ksplit = std::min(p.ksplit, (int)(2 * Np / 64));
+      p.ksplit = std::min(auto_split(tiles, (int)(Np / 64), ctx->nsm), kMaxSplit);
+      p.ksplit = std::min(p.ksplit, (int)(Np / 64));
       px_split = p.ksplit;
+      p.err = ctx->err;
+      PxParams px;
+      px.S = S;
+      px.stats = rstat;
+      px.ldS = P.ldS;
+      px.t = t;
+      px.N = (int)N;
+      px.xbase_row = h0 * 2 * d;
+      px.d2 = 2 * d;
+      px.lo_rows = d;
+      px.Np = Np;
+      px.nb = nbl;
+      px.bdiv = ni;
       EpiAffine e;
       e.kind = OUT_F32;
       e.out = O;
@@ -547,8 +561,14 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.om.r0 = 2 * d;
       e.om.c0 = 1;
       e.vec_ok = 1;
-      TRY(run_gemm<STILL_K_PX>(ctx, bn, op(Pm, (int64_t)nbl * t, Np), op(XT, (int64_t)H * 2 * d, 2 * Np), p,
-                   e, 0, s));
+      const Operand2D xt = op(XT, (int64_t)H * 2 * d, 2 * Np);
+      ctx->prof.begin(STILL_K_PX, s);
+      cudaError_t r = d == 64    ? launch_px_fused<128, 64>(xt, p, px, e, ctx->nsm, s)
+                      : d == 128 ? launch_px_fused<256, 128>(xt, p, px, e, ctx->nsm, s)
+                                 : launch_px_fused<256, 256>(xt, p, px, e, ctx->nsm, s);
+      ctx->prof.end(STILL_K_PX, s);
+      if (r == cudaErrorInvalidValue) return STILL_ERR_INVALID_ARG;
+      if (r != cudaSuccess) return STILL_ERR_CUDA;
     }
     KLAUNCH(STILL_K_PXSPLIT, launch_px_to_hilo(O, px_split, px_stride, b0, nbl, n, t, 2 * d, PX, s));
     b0 += nbl;

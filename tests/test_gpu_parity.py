@@ -11,7 +11,7 @@ import torch
 from oracle import still_oracle as O
 from paper_2606_07878_gb300 import still, synth
 
-from gpu_helpers import Runner, assert_parity, oracle_layer
+from gpu_helpers import ERR_REL, Runner, assert_parity, metrics, oracle_layer
 
 pytestmark = pytest.mark.gpu
 
@@ -229,5 +229,64 @@ def test_invalid_arguments_return_status():
                 r.ctx, 1, still.config_from_workload(wl, 32, n_blocks=2), r.W[0])
         assert e.value.name == "STILL_ERR_UNSUPPORTED"
         r.check_status()
+    finally:
+        r.close()
+
+
+def test_gemma_shape_reduced_context():
+    """Gemma-128k compactor shape (d = 256, d_l = 2048, 16 heads, FFN 8192) at t = 655 on a
+    reduced 4096-token cache with one KV-head, full oracle comparison."""
+    wl = dict(synth.WORKLOADS["gemma_128k"], N=4096, H=1)
+    t = 655
+    r = Runner(wl, t)
+    try:
+        K, V = synth.gen_kv(wl, 0, device=DEV)
+        Ck, Cv, _ = r.layer(0, K, V, t)
+        rk, rv, _, _ = oracle_layer(wl, r.W[0], K, V, t)
+        assert_parity(rk, synth.bf16_to_f64(Ck), "C_k")
+        assert_parity(rv, synth.bf16_to_f64(Cv), "C_v")
+    finally:
+        r.close()
+
+
+@pytest.mark.parametrize("t", [164, 512])
+def test_qwen8b_32k_layer_sampled_head(t):
+    """Full-size layer of the Qwen-8B-shaped workload (N = 32768, H = 8); the oracle
+    recomputes KV-head 5."""
+    wl = synth.WORKLOADS["qwen8b_32k"]
+    r = Runner(wl, t)
+    try:
+        K, V = synth.gen_kv(wl, 0, device=DEV)
+        Ck, Cv, _ = r.layer(0, K, V, t)
+        rk, rv, _, _ = oracle_layer(wl, r.W[0], K, V, t, heads=[5])
+        assert_parity(rk[:, 5], synth.bf16_to_f64(Ck[:, 5]), "C_k head 5")
+        assert_parity(rv[:, 5], synth.bf16_to_f64(Cv[:, 5]), "C_v head 5")
+    finally:
+        r.close()
+
+
+def test_gemma_128k_full_size_token_reversal_invariance():
+    """Full-size Gemma-shaped layer (N = 131072, H = 8, d = 256, d_l = 2048, t = 655): the
+    compactor is a function of the set of (token, position) pairs, so feeding the cache in
+    reverse order with reversed positions (one segment of step -1) gives the same compact
+    cache up to rounding. Both runs are GPU results: if each is within the parity bar of the
+    exact value (max|err| <= 0.02 RMS, row cosine >= 0.999), their difference is within twice
+    the bar (0.04 RMS) and their row cosine >= cos(2 acos 0.999) > 0.996. Rounding decisions
+    (fp16 probabilities, bf16 outputs) make the two runs differ by more than plain reordering
+    would suggest, so the twice-the-bar bound is the one checked here."""
+    wl = synth.WORKLOADS["gemma_128k"]
+    t = 655
+    N = wl["N"]
+    r = Runner(wl, t)
+    try:
+        K, V = synth.gen_kv(wl, 0, device=DEV)
+        Ck, Cv, (ps, pst, off) = r.layer(0, K, V, t)
+        Kr, Vr = K.flip(0).contiguous(), V.flip(0).contiguous()
+        Ck2, Cv2, (ps2, pst2, off2) = r.layer(0, Kr, Vr, t, segments=[(N - 1.0, -1.0, N)])
+        assert (ps, pst, off) == (ps2, pst2, off2) == (0.0, (N - 1.0) / (t - 1), N - t)
+        assert torch.isfinite(Ck.float()).all() and torch.isfinite(Cv.float()).all()
+        for name, a, b in (("C_k", Ck, Ck2), ("C_v", Cv, Cv2)):
+            err, cos = metrics(synth.bf16_to_f64(a), synth.bf16_to_f64(b))
+            assert err <= 2 * ERR_REL and cos >= 0.996, f"{name} reversed: {err:.4e} {cos:.6f}"
     finally:
         r.close()
