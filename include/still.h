@@ -284,6 +284,13 @@ still_status still_profile_read(still_ctx* ctx, int32_t cls, int64_t* h_launches
 /* Static name of a kernel class ("scores", "softmax", ...). */
 const char* still_kernel_class_name(int32_t cls);
 
+/* Failure-detection self-test (no counterpart in the paper): launches one kernel that waits,
+ * for at most limit_us microseconds (1 .. 2e6), on a barrier nothing will release, exactly as
+ * the library's kernels bound every wait. The wait expires, the kernel records a timeout in
+ * the device error record and returns; the next still_get_device_status reports
+ * STILL_ERR_TIMEOUT (and clears the record) and the context stays usable. */
+still_status still_selftest_wait_timeout(still_ctx* ctx, int64_t limit_us, void* stream);
+
 /* Compact budget t = round(N / ratio) with halves rounded up (App. J exact-results table,
  * K column: 8192 / 50 -> 164, 65536 / 50 -> 1311). Host-only. */
 int64_t still_budget(int64_t n_tokens, int64_t ratio);

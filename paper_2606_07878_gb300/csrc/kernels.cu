@@ -297,6 +297,24 @@ __global__ void row_stats_kernel(const float2* __restrict__ parts, int64_t rows,
   out[r] = make_float2(M * kLog2e, 1.f / L);
 }
 
+// Failure-detection self-test: waits on an mbarrier that nothing arrives on, with a short
+// bound. The wait expires, the kernel records DEV_WAIT_TIMEOUT in the error record and returns.
+__global__ void wait_timeout_selftest_kernel(int* err, unsigned long long limit_ns) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const uint32_t a = smem_u32(&bar);
+    const uint64_t t0 = globaltimer_ns();
+    bool done = false;
+    while (!done && globaltimer_ns() - t0 < limit_ns) done = mbar_try_wait(a, 0) != 0;
+    if (!done) dev_set_error(err, DEV_WAIT_TIMEOUT, 900);
+  }
+}
+
 __global__ void omega_kernel(double* out, int half, int width, double base) {
   const int m = blockIdx.x * blockDim.x + threadIdx.x;
   if (m < half) out[m] = pow(base, -2.0 * m / width);
@@ -456,6 +474,11 @@ static bool softmax_reg(const float* S, int64_t rows, int64_t ncols, int64_t ldS
 cudaError_t launch_row_stats(const float2* parts, int64_t rows, int slots, float2* out,
                              cudaStream_t s) {
   row_stats_kernel<<<blocks_for(rows, 256), 256, 0, s>>>(parts, rows, slots, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_wait_timeout_selftest(int* err, unsigned long long limit_ns, cudaStream_t s) {
+  wait_timeout_selftest_kernel<<<1, 32, 0, s>>>(err, limit_ns);
   return cudaGetLastError();
 }
 

@@ -45,6 +45,9 @@ cudaError_t launch_q_rope(const float* qhat, int t_max, int b0, int nb, int t, i
 cudaError_t launch_row_stats(const float2* parts, int64_t rows, int slots, float2* out,
                              cudaStream_t s);
 
+// One-block kernel whose bounded wait on an mbarrier can only expire (failure-detection test).
+cudaError_t launch_wait_timeout_selftest(int* err, unsigned long long limit_ns, cudaStream_t s);
+
 // out[m] = base^(-2m / width) in fp64, m < half.
 cudaError_t launch_omega(double* out, int half, int width, double base, cudaStream_t s);
 

@@ -1318,6 +1318,14 @@ const char* still_kernel_class_name(int32_t cls) {
   return cls >= 0 && cls < STILL_K_COUNT ? names[cls] : "unknown";
 }
 
+still_status still_selftest_wait_timeout(still_ctx* ctx, int64_t limit_us, void* stream) {
+  if (ctx == nullptr || limit_us < 1 || limit_us > 2000000) return STILL_ERR_INVALID_ARG;
+  CK(cudaSetDevice(ctx->device));
+  CK(launch_wait_timeout_selftest(ctx->err, (unsigned long long)limit_us * 1000ull,
+                                  static_cast<cudaStream_t>(stream)));
+  return STILL_OK;
+}
+
 int64_t still_budget(int64_t n_tokens, int64_t ratio) {
   if (n_tokens < 0 || ratio < 1) return -1;
   return (2 * n_tokens + ratio) / (2 * ratio);

@@ -26,6 +26,7 @@ EXPORTS = [
     "still_get_device_status", "still_budget", "still_kv_bytes", "still_param_count",
     "still_profile_enable", "still_profile_read", "still_kernel_class_name",
     "still_compact_layer_noalloc", "still_recompact_layer_ragged", "still_recompact_stack_ragged",
+    "still_selftest_wait_timeout",
 ]
 
 NOALLOC_SCRATCH_MIB = 64  # STILL_NOALLOC_SCRATCH_MIB in include/still.h
@@ -110,6 +111,7 @@ def lib():
             "still_budget": ([I64, I64], I64),
             "still_kv_bytes": ([I64, I64, I64, I64, I64], I64),
             "still_param_count": ([ctypes.POINTER(LayerConfig), I32], I64),
+            "still_selftest_wait_timeout": ([P, I64, P], ctypes.c_int),
             "still_profile_enable": ([P, I32], ctypes.c_int),
             "still_profile_read": ([P, I32, PI64, PD], ctypes.c_int),
             "still_kernel_class_name": ([I32], ctypes.c_char_p),
@@ -348,3 +350,8 @@ def still_profile_read(ctx):
 
 def still_kernel_class_name(cls: int) -> str:
     return lib().still_kernel_class_name(cls).decode()
+
+
+def still_selftest_wait_timeout(ctx, limit_us: int = 1000, stream=None):
+    _check(lib().still_selftest_wait_timeout(ctx, limit_us, _stream(stream)),
+           "still_selftest_wait_timeout")
