@@ -33,15 +33,18 @@ def describe(name, wl, t):
     return (f"{name}: {wl['L']} layers, N={wl['N']}, H_kv={wl['H']}, d={wl['d']}, "
             f"D={wl['D']}, {wl['n']} heads, FFN {wl['F']}, t={t} ({round(wl['N'] / t)}x)")
 
-# DRAM traffic of one scores-GEMM launch from an ncu capture (profiles/), valid only for the
-# kernel sources it was taken on.
-TRAFFIC = {"kernel_hash": None, "bytes_per_launch": None, "profile": None}
+# DRAM traffic (read + write) of one scores-GEMM launch at this workload from an ncu capture
+# (profiles/scores_gemm_qwen7b_8k_t1024.md: 1.209 GB read + 1.044 GB written), valid only for
+# the kernel sources it was taken on (hash of the GEMM kernel and epilogue sources).
+TRAFFIC = {"kernel_hash": "ce6adf3bdfbbf7f0", "bytes_per_launch": 2.2531e9,
+           "workload": ("qwen7b_8k", 1024),
+           "profile": "profiles/scores_gemm_qwen7b_8k_t1024.md"}
 
 
-def _csrc_hash():
+def _kernel_hash():
     h = hashlib.sha256()
     d = os.path.join(ROOT, "paper_2606_07878_gb300", "csrc")
-    for f in sorted(os.listdir(d)):
+    for f in ["tc_gemm.cuh", "epilogues.cuh"]:
         with open(os.path.join(d, f), "rb") as fh:
             h.update(f.encode())
             h.update(fh.read())
@@ -455,7 +458,7 @@ def main():
     per_launch_flops = fl["scores"] * L * args.steps / max(n_sc, 1)
     achieved = per_launch_flops / (ms_sc / max(n_sc, 1) / 1e3) / 1e12 if ms_sc > 0 else None
     traffic = None
-    if TRAFFIC["kernel_hash"] == _csrc_hash():
+    if TRAFFIC["kernel_hash"] == _kernel_hash() and TRAFFIC["workload"] == (name, t):
         traffic = TRAFFIC["bytes_per_launch"]
     roof = {"bound": "tensor", "kernel": "scores (3-pass split-bf16 tcgen05 GEMM)",
             "achieved": achieved, "peak": bf16_sus, "unit": "TFLOP/s",
