@@ -33,18 +33,22 @@ def describe(name, wl, t):
     return (f"{name}: {wl['L']} layers, N={wl['N']}, H_kv={wl['H']}, d={wl['d']}, "
             f"D={wl['D']}, {wl['n']} heads, FFN {wl['F']}, t={t} ({round(wl['N'] / t)}x)")
 
-# DRAM traffic (read + write) of one scores-GEMM launch at this workload from an ncu capture
-# (profiles/scores_gemm_qwen7b_8k_t1024.md: 1.209 GB read + 1.044 GB written), valid only for
-# the kernel sources it was taken on (hash of the GEMM kernel and epilogue sources).
-TRAFFIC = {"kernel_hash": "ce6adf3bdfbbf7f0", "bytes_per_launch": 2.2531e9,
-           "workload": ("qwen7b_8k", 1024),
-           "profile": "profiles/scores_gemm_qwen7b_8k_t1024.md"}
+# DRAM traffic (read + write) per launch of the dominant kernel at a workload, from an ncu
+# capture; valid only for the kernel sources it was taken on (hash of the listed sources).
+# The scores GEMM (two-kernel path, 2d = 512) and the fused cross-attention kernel (2d <= 256).
+TRAFFIC = {
+    "scores": {"files": ["tc_gemm.cuh", "epilogues.cuh"], "kernel_hash": "ce6adf3bdfbbf7f0",
+               "bytes_per_launch": 2.2531e9, "workload": ("qwen7b_8k", 1024),
+               "profile": "profiles/scores_gemm_qwen7b_8k_t1024.md"},
+    "ca_fused": {"files": ["ca_flash.cuh", "ptx.cuh"], "kernel_hash": None,
+                 "bytes_per_launch": None, "workload": ("qwen7b_8k", 1024), "profile": None},
+}
 
 
-def _kernel_hash():
+def _kernel_hash(files):
     h = hashlib.sha256()
     d = os.path.join(ROOT, "paper_2606_07878_gb300", "csrc")
-    for f in ["tc_gemm.cuh", "epilogues.cuh"]:
+    for f in files:
         with open(os.path.join(d, f), "rb") as fh:
             h.update(f.encode())
             h.update(fh.read())
@@ -152,7 +156,7 @@ def algorithmic_flops(wl, t, N):
           + 2 * t * H * n * 2 * d * D + 2 * t * H * n * D * D)
     sa = 6 * t * H * D * n * D + 4 * t * t * H * n * D + 2 * t * H * n * D * D
     return {"total": ca + sa + 4 * t * H * D * F + 4 * t * H * D * d,
-            "scores": 2 * t * N * H * n * D}
+            "scores": 2 * t * N * H * n * D, "px": 2 * t * N * H * n * 2 * d}
 
 
 def run_cpu_baseline(wl, t, budget_s=30.0):
@@ -451,21 +455,32 @@ def main():
     ems = max_over_ranks(ems, dist, dev)
     e2e_value = throughput(world, N, args.steps, ems)
 
-    # ---------------------------------------------------------------- roofline (scores GEMM)
+    # ---------------------------------------------------------------- roofline
+    # Dominant kernel: the fused cross-attention (scores + softmax + P X) when the path uses
+    # it (2d <= 256), else the scores GEMM. Algorithmic flops count each product once; the
+    # issued view counts the split-precision passes (3 for q.k, 1.5 for P X: hi + key-half lo).
     hbm, bf16_burst, bf16_sus, src = _peaks()
     fl = algorithmic_flops(wl, t, N)
-    n_sc, ms_sc = prof["scores"]
-    per_launch_flops = fl["scores"] * L * args.steps / max(n_sc, 1)
-    achieved = per_launch_flops / (ms_sc / max(n_sc, 1) / 1e3) / 1e12 if ms_sc > 0 else None
+    fused = prof.get("ca_fused", (0, 0.0))[0] > 0
+    kname = "ca_fused" if fused else "scores"
+    n_k, ms_k = prof[kname]
+    alg = fl["scores"] + fl["px"] if fused else fl["scores"]
+    issued = 3 * fl["scores"] + 1.5 * fl["px"] if fused else 3 * fl["scores"]
+    per_launch_flops = alg * L * args.steps / max(n_k, 1)
+    achieved = per_launch_flops / (ms_k / max(n_k, 1) / 1e3) / 1e12 if ms_k > 0 else None
+    tr = TRAFFIC[kname]
     traffic = None
-    if TRAFFIC["kernel_hash"] == _kernel_hash() and TRAFFIC["workload"] == (name, t):
-        traffic = TRAFFIC["bytes_per_launch"]
-    roof = {"bound": "tensor", "kernel": "scores (3-pass split-bf16 tcgen05 GEMM)",
+    if tr["kernel_hash"] == _kernel_hash(tr["files"]) and tr["workload"] == (name, t):
+        traffic = tr["bytes_per_launch"]
+    kdesc = ("ca_fused (3-pass split-bf16 scores + online softmax + P X, one tcgen05 kernel)"
+             if fused else "scores (3-pass split-bf16 tcgen05 GEMM)")
+    ratio = issued / alg
+    roof = {"bound": "tensor", "kernel": kdesc,
             "achieved": achieved, "peak": bf16_sus, "unit": "TFLOP/s",
             "frac": achieved / bf16_sus if achieved else None, "traffic": traffic,
             "peak_source": f"{src} bf16 sustained (kernel timed inside a long step)",
-            "issued_tflops": achieved * 3 if achieved else None,
-            "issued_frac": achieved * 3 / bf16_sus if achieved else None,
+            "issued_tflops": achieved * ratio if achieved else None,
+            "issued_frac": achieved * ratio / bf16_sus if achieved else None,
             "flops_per_launch": per_launch_flops}
     whole = fl["total"] * L * world * args.steps / (ms / 1e3) / 1e12
 

@@ -257,7 +257,7 @@ typedef enum {
   STILL_K_SCORES,       /* S = d_l q.k / |k| (3-pass tcgen05 GEMM)          */
   STILL_K_SOFTMAX,      /* cross-attention row softmax                      */
   STILL_K_PX,           /* O = P X (2-pass tcgen05 GEMM, split-K)           */
-  STILL_K_PXSPLIT,      /* O -> hi/lo                                       */
+  STILL_K_PXSPLIT,      /* key-split merge of O, O -> hi/lo                 */
   STILL_K_VO,           /* Z' = Z + O (W_V W_O) (3-pass tcgen05 GEMM)       */
   STILL_K_NORM,         /* RMSNorm                                          */
   STILL_K_SA_PROJ,      /* self-attention q/k projections                   */
@@ -271,6 +271,7 @@ typedef enum {
   STILL_K_HEADS,        /* C_k, C_v output heads + re-rotation              */
   STILL_K_NORMS,        /* QK-norm factors from sum-of-squares partials     */
   STILL_K_LOAD,         /* weight-load precompute GEMMs                     */
+  STILL_K_CA_FUSED,     /* fused scores + online softmax + P X (d <= 128)   */
   STILL_K_COUNT
 } still_kernel_class;
 

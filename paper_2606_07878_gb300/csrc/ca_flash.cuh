@@ -1,0 +1,520 @@
+// Cross-attention of one compactor layer in a single kernel, for sm_103a (App. A,
+// "Cross-attention"; the compactor's latent queries attend over the cached tokens X):
+//
+//   S(m, k)  = scale * q_m . k_k / |k~_k|          3-pass split-bf16 tcgen05.mma, fp32 in TMEM
+//   P(m, k)  = exp(S(m, k) - M(m))                   online row softmax over 256-key tiles
+//   O(m, :)  = sum_k P(m, k) X(k, :) / sum_k P(m, k)
+//
+// A work unit is (batch b = (KV-head, cross head), 128-row query tile, key split). Per key tile
+// the MMA warp computes S into TMEM columns [0, 256); eight softmax warps drain it to registers,
+// form fp16 probabilities in the 128-byte-swizzled shared-memory layout the tensor core reads,
+// and the MMA warp accumulates P X^T into TMEM columns [256, 256 + 2d). S and P never reach
+// global memory. The running max is kept in log2 units and only moved (with a rescale of the
+// TMEM accumulator) when a tile raises it by more than kRescaleLog2, so that P <= 2^8 fits fp16.
+//
+// Issue order of the tensor pipe: S_0, S_1, PX_0, S_2, PX_1, ... . PX_{j-1} runs while the
+// softmax warps drain S_j, so the single S buffer costs no tensor-pipe idle time.
+//
+// Output per split: unnormalised O rows and (m, l) with m in log2 units; ca_merge_kernel
+// combines the splits in a fixed order (bit-reproducible).
+//
+// CTA = 10 warps: 0 TMA producer, 1 MMA issuer (TMEM owner), 2..9 softmax / output.
+#pragma once
+#include "gemm_host.cuh"
+
+namespace still {
+
+struct FlashParams {
+  int32_t t = 0, N = 0;     // query rows per batch, valid keys
+  int32_t D = 0;            // width of one hi or lo part of q / k (multiple of 64)
+  int64_t Np = 0;           // key pitch of X^T hi / lo (multiple of 64, >= N, zero padded)
+  int32_t nb = 0, bdiv = 1; // batches; KV-head of batch b is h0 + b / bdiv
+  int32_t xbase_row = 0;    // X^T row of feature 0 of KV-head h0
+  int32_t tiles_m = 0, tiles_k = 0, nsplit = 1, nunits = 0;
+  const float* kinv = nullptr;  // [nb][N]: scale / |k~| per key
+  float* O = nullptr;           // [nsplit][nb][t][2d] unnormalised
+  float2* stats = nullptr;      // [nsplit][nb][t]: (running max m in log2 units, sum l)
+  int* err = nullptr;
+};
+
+constexpr int kFlashKeys = 256;       // keys per S tile
+constexpr int kFlashSoftWarps = 8;    // two per TMEM lane quarter
+constexpr int kFlashThreads = 64 + 32 * kFlashSoftWarps;
+constexpr float kRescaleLog2 = 8.f;
+
+template <int D2>
+struct FlashSmem {
+  static_assert(D2 == 128 || D2 == 256, "2d must be 128 or 256");
+  static constexpr int kQBytes = kBM * kBK * 2;            // q chunk, 16 KB
+  static constexpr int kKBytes = kFlashKeys * kBK * 2;     // k chunk, 32 KB
+  static constexpr int kXhiBytes = D2 * kBK * 2;           // X^T hi chunk
+  static constexpr int kXloBytes = (D2 / 2) * kBK * 2;     // X^T lo chunk (key half)
+  static constexpr int kStageBytes = kQBytes + kKBytes;    // >= kXhiBytes + kXloBytes
+  static constexpr int kStages = 3;
+  static constexpr int kPChunkBytes = kBM * kBK * 2;       // 128 rows x 64 keys fp16
+  static constexpr int kPOffset = kStages * kStageBytes;
+  static constexpr int kKinvOffset = kPOffset + 4 * kPChunkBytes;        // [8 warps][128] f32
+  static constexpr int kXchOffset = kKinvOffset + kFlashSoftWarps * 128 * 4;  // [2][2][128] f32
+  static constexpr int kBarOffset = kXchOffset + 2 * 2 * 128 * 4;
+  static constexpr int kBytes = kBarOffset + 256 + 1024;
+  static_assert(kXhiBytes + kXloBytes <= kStageBytes, "X chunk fits a stage");
+  static_assert(kBytes <= 232448, "shared memory budget");
+};
+
+struct FlashUnit {
+  int b, tm, split, j0, j1;
+};
+
+__device__ __forceinline__ FlashUnit flash_unit(const FlashParams& f, int u) {
+  FlashUnit r;
+  r.tm = u % f.tiles_m;
+  int q = u / f.tiles_m;
+  r.split = q % f.nsplit;
+  r.b = q / f.nsplit;
+  r.j0 = (int)(((int64_t)f.tiles_k * r.split) / f.nsplit);
+  r.j1 = (int)(((int64_t)f.tiles_k * (r.split + 1)) / f.nsplit);
+  return r;
+}
+
+// Number of 64-key chunks of tile j that lie inside the padded key range [0, Np).
+__device__ __forceinline__ int flash_chunks(const FlashParams& f, int j) {
+  const int64_t left = f.Np - (int64_t)j * kFlashKeys;
+  return left >= kFlashKeys ? 4 : (int)(left / kBK);
+}
+
+template <int D2>
+__global__ void __launch_bounds__(kFlashThreads, 1)
+    ca_flash_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                    const __grid_constant__ CUtensorMap tmXhi,
+                    const __grid_constant__ CUtensorMap tmXlo, const FlashParams f) {
+  using S = FlashSmem<D2>;
+  constexpr int kStages = S::kStages;
+  constexpr int kOCols = D2 / 2;  // O columns per softmax warp (its half of 2d)
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::kBarOffset);
+  uint64_t* empty = full + kStages;
+  uint64_t* sfull = empty + kStages;  // S tile complete in TMEM
+  uint64_t* sfree = sfull + 1;        // S tile drained by the softmax warps
+  uint64_t* pfull = sfree + 1;        // P tile written (and O rescaled if needed)
+  uint64_t* pempty = pfull + 1;       // PX MMA complete (P buffer free, O up to date)
+  uint64_t* ofree = pempty + 1;       // O drained at the end of a unit
+  uint64_t* xb = ofree + 1;           // [4] row-value exchange per lane quarter
+  uint64_t* drain = xb + 4;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int qchunks = f.D / kBK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(sfull, 1);
+    mbar_init(sfree, kFlashSoftWarps);
+    mbar_init(pfull, kFlashSoftWarps);
+    mbar_init(pempty, 1);
+    mbar_init(ofree, kFlashSoftWarps);
+    for (int q = 0; q < 4; ++q) mbar_init(&xb[q], 2);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&tmQ);
+    tma_prefetch_desc(&tmK);
+    tma_prefetch_desc(&tmXhi);
+    tma_prefetch_desc(&tmXlo);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ TMA producer
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t armed = 0, armed_par = 0;
+      bool bad = false;
+      auto acquire = [&](uint32_t bytes) -> uint8_t* {
+        if (!mbar_wait(&empty[stage], phase ^ 1)) {
+          dev_set_error(f.err, DEV_WAIT_TIMEOUT, 300);
+          *abort_flag = 1;
+          bad = true;
+          return nullptr;
+        }
+        mbar_arrive_expect_tx(&full[stage], bytes);
+        armed |= 1u << stage;
+        armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
+        return smem + stage * S::kStageBytes;
+      };
+      auto advance = [&]() {
+        if (++stage == kStages) {
+          stage = 0;
+          phase ^= 1;
+        }
+      };
+      for (int u = blockIdx.x; u < f.nunits && !bad && !*abort_flag; u += gridDim.x) {
+        const FlashUnit w = flash_unit(f, u);
+        const int32_t qrow = w.b * f.t + w.tm * kBM;
+        const int32_t krow = w.b * f.N;
+        const int32_t xrow = f.xbase_row + (w.b / f.bdiv) * D2;
+        const int J = w.j1 - w.j0;
+        for (int jj = 0; jj <= J && !bad; ++jj) {
+          if (jj < J) {
+            const int32_t kr = krow + (w.j0 + jj) * kFlashKeys;
+            for (int pass = 0; pass < 3 && !bad; ++pass) {
+              const int32_t qoff = pass == 2 ? f.D : 0;  // (q_hi,k_hi), (q_hi,k_lo), (q_lo,k_hi)
+              const int32_t koff = pass == 1 ? f.D : 0;
+              for (int c = 0; c < qchunks; ++c) {
+                uint8_t* sa = acquire(S::kStageBytes);
+                if (sa == nullptr) break;
+                tma_load_2d(sa, &tmQ, &full[stage], qoff + c * kBK, qrow);
+                tma_load_2d(sa + S::kQBytes, &tmK, &full[stage], koff + c * kBK, kr);
+                advance();
+              }
+            }
+          }
+          if (jj >= 1) {
+            const int j = w.j0 + jj - 1;
+            const int nch = flash_chunks(f, j);
+            for (int c = 0; c < nch; ++c) {
+              uint8_t* sa = acquire(S::kXhiBytes + S::kXloBytes);
+              if (sa == nullptr) break;
+              const int32_t x = j * kFlashKeys + c * kBK;
+              tma_load_2d(sa, &tmXhi, &full[stage], x, xrow);
+              tma_load_2d(sa + S::kXhiBytes, &tmXlo, &full[stage], (int32_t)(f.Np + x), xrow);
+              advance();
+            }
+          }
+        }
+      }
+      if (bad || *abort_flag) {
+        for (int s = 0; s < kStages; ++s)
+          if (armed & (1u << s)) (void)mbar_wait(&full[s], (armed_par >> s) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ MMA issuer
+      const uint32_t idesc_s = idesc_f16(kBM, kFlashKeys, 1);  // bf16 q, k
+      const uint32_t idesc_hi = idesc_f16(kBM, D2, 0);         // fp16 P, X^T hi
+      const uint32_t idesc_lo = idesc_f16(kBM, D2 / 2, 0);     // fp16 P, X^T lo (key half)
+      const uint32_t s_tmem = tmem_base;
+      const uint32_t o_tmem = tmem_base + 256;
+      const uint32_t p_smem = smem_u32(smem + S::kPOffset);
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t n_s = 0, n_px = 0, n_units = 0;
+      bool issued = false, bad = false;
+      auto fail = [&](int where) {
+        dev_set_error(f.err, DEV_WAIT_TIMEOUT, where);
+        *abort_flag = 1;
+        bad = true;
+      };
+      for (int u = blockIdx.x; u < f.nunits && !bad && !*abort_flag; u += gridDim.x) {
+        const FlashUnit w = flash_unit(f, u);
+        const int J = w.j1 - w.j0;
+        for (int jj = 0; jj <= J && !bad; ++jj) {
+          if (jj < J) {
+            if (n_s > 0 && !mbar_wait(sfree, (n_s - 1) & 1)) {
+              fail(310);
+              break;
+            }
+            tc_fence_after();
+            const int nst = 3 * qchunks;
+            for (int st = 0; st < nst; ++st) {
+              if (!mbar_wait(&full[stage], phase)) {
+                fail(311);
+                break;
+              }
+              tc_fence_after();
+              const uint32_t sa = smem_u32(smem + stage * S::kStageBytes);
+              const uint64_t ad = sdesc_k_sw128(sa);
+              const uint64_t bd = sdesc_k_sw128(sa + S::kQBytes);
+#pragma unroll
+              for (int k = 0; k < kBK / 16; ++k)
+                tc_mma_f16(s_tmem, ad + 2 * k, bd + 2 * k, idesc_s, (st > 0 || k > 0) ? 1u : 0u);
+              issued = true;
+              tc_commit(&empty[stage]);
+              if (++stage == kStages) {
+                stage = 0;
+                phase ^= 1;
+              }
+            }
+            if (bad) break;
+            tc_commit(sfull);
+            ++n_s;
+          }
+          if (jj >= 1) {
+            const int j = w.j0 + jj - 1;
+            const int nch = flash_chunks(f, j);
+            if (jj == 1 && n_units > 0 && !mbar_wait(ofree, (n_units - 1) & 1)) {
+              fail(312);
+              break;
+            }
+            if (!mbar_wait(pfull, n_px & 1)) {
+              fail(313);
+              break;
+            }
+            tc_fence_after();
+            for (int c = 0; c < nch; ++c) {
+              if (!mbar_wait(&full[stage], phase)) {
+                fail(314);
+                break;
+              }
+              tc_fence_after();
+              const uint32_t sa = smem_u32(smem + stage * S::kStageBytes);
+              const uint64_t pd = sdesc_k_sw128(p_smem + c * S::kPChunkBytes);
+              const uint64_t hd = sdesc_k_sw128(sa);
+              const uint64_t ld = sdesc_k_sw128(sa + S::kXhiBytes);
+#pragma unroll
+              for (int k = 0; k < kBK / 16; ++k)
+                tc_mma_f16(o_tmem, pd + 2 * k, hd + 2 * k, idesc_hi,
+                           (jj > 1 || c > 0 || k > 0) ? 1u : 0u);
+#pragma unroll
+              for (int k = 0; k < kBK / 16; ++k) tc_mma_f16(o_tmem, pd + 2 * k, ld + 2 * k, idesc_lo, 1u);
+              tc_commit(&empty[stage]);
+              if (++stage == kStages) {
+                stage = 0;
+                phase ^= 1;
+              }
+            }
+            if (bad) break;
+            tc_commit(pempty);
+            ++n_px;
+          }
+        }
+        ++n_units;
+      }
+      if ((bad || *abort_flag) && issued) {
+        tc_commit(drain);
+        (void)mbar_wait(drain, 0);
+      }
+    }
+  } else {
+    // -------------------------------------------------------------- softmax / output warps
+    const int sw = warp - 2;
+    const int quarter = warp & 3;  // TMEM lanes [32 quarter, 32 quarter + 32)
+    const int half = sw >> 2;      // S columns [128 half, +128), O columns [kOCols half, +kOCols)
+    const int row = quarter * 32 + lane;
+    const uint32_t lane_base = tmem_base + ((uint32_t)(quarter * 32) << 16);
+    float* kw = reinterpret_cast<float*>(smem + S::kKinvOffset) + sw * 128;
+    float* xch = reinterpret_cast<float*>(smem + S::kXchOffset);  // [2][2][128]
+    uint8_t* pbuf = smem + S::kPOffset;
+    constexpr float kLog2e = 1.4426950408889634f;
+    uint32_t n_sf = 0, n_pe = 0, n_pf = 0, n_x = 0;
+    bool bad = false;
+    auto wait_all = [&](uint64_t* bar, uint32_t parity, int where) -> bool {
+      bool ok = mbar_wait(bar, parity);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) {
+        if (lane == 0) {
+          dev_set_error(f.err, DEV_WAIT_TIMEOUT, where);
+          *abort_flag = 1;
+        }
+        bad = true;
+      }
+      return ok;
+    };
+    // Exchanges one value per row with the other warp of this lane quarter; returns its value.
+    auto exchange = [&](float mine, int where) -> float {
+      float* slot = xch + (n_x & 1) * 256;
+      slot[half * 128 + row] = mine;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&xb[quarter]);
+      const bool ok = wait_all(&xb[quarter], n_x & 1, where);
+      ++n_x;
+      return ok ? slot[(1 - half) * 128 + row] : mine;
+    };
+
+    for (int u = blockIdx.x; u < f.nunits && !bad && !warp_flag(abort_flag); u += gridDim.x) {
+      const FlashUnit w = flash_unit(f, u);
+      const int J = w.j1 - w.j0;
+      float m_run = -INFINITY, l_part = 0.f;
+      for (int jj = 0; jj < J; ++jj) {
+        const int j = w.j0 + jj;
+        const int key0 = j * kFlashKeys + 128 * half;  // first key of this warp's columns
+        float kv[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int key = key0 + lane + 32 * e;
+          kv[e] = key < f.N ? f.kinv[(int64_t)w.b * f.N + key] * kLog2e : 0.f;
+        }
+        if (!wait_all(sfull, n_sf & 1, 320)) break;
+        ++n_sf;
+        tc_fence_after();
+        float v[128];
+#pragma unroll
+        for (int g = 0; g < 4; ++g) {
+          float tmp[32];
+          tmem_ld32(lane_base + (uint32_t)(128 * half + 32 * g), tmp);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) v[32 * g + e] = tmp[e];
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(sfree);
+        // scale per key (log2 units), mask keys past N, tile max
+#pragma unroll
+        for (int e = 0; e < 4; ++e) kw[lane + 32 * e] = kv[e];
+        __syncwarp();
+        const int cvalid = f.N - key0;
+        float mx = -INFINITY;
+#pragma unroll
+        for (int c = 0; c < 128; c += 4) {
+          const float4 k4 = *reinterpret_cast<const float4*>(kw + c);
+          v[c] = c < cvalid ? v[c] * k4.x : -INFINITY;
+          v[c + 1] = c + 1 < cvalid ? v[c + 1] * k4.y : -INFINITY;
+          v[c + 2] = c + 2 < cvalid ? v[c + 2] * k4.z : -INFINITY;
+          v[c + 3] = c + 3 < cvalid ? v[c + 3] * k4.w : -INFINITY;
+          mx = fmaxf(mx, fmaxf(fmaxf(v[c], v[c + 1]), fmaxf(v[c + 2], v[c + 3])));
+        }
+        __syncwarp();
+        mx = fmaxf(mx, exchange(mx, 321));
+        if (bad) break;
+        // Both warps of the quarter hold the same (m_run, mx), so they take the same decision.
+        bool rescale = false;
+        float fac = 1.f;
+        if (m_run == -INFINITY) {
+          m_run = mx;
+        } else if (mx > m_run + kRescaleLog2) {
+          fac = exp2f(m_run - mx);
+          m_run = mx;
+          l_part *= fac;
+          rescale = true;
+        }
+        // probabilities (fp16, <= 2^8) into registers as packed pairs; l from the rounded values
+        uint32_t pk[64];
+#pragma unroll
+        for (int c = 0; c < 128; c += 2) {
+          const __half2 h = __floats2half2_rn(exp2f(v[c] - m_run), exp2f(v[c + 1] - m_run));
+          const float2 r = __half22float2(h);
+          l_part += r.x + r.y;
+          pk[c / 2] = *reinterpret_cast<const uint32_t*>(&h);
+        }
+        // The previous PX must be complete before P is overwritten or O is rescaled.
+        if (n_pf > n_pe) {
+          if (!wait_all(pempty, n_pe & 1, 322)) break;
+          ++n_pe;
+          tc_fence_after();
+        }
+        // tcgen05.ld / st are warp-collective: the warp rescales when any of its rows needs it
+        // (rows that do not have fac = 1).
+        if (__any_sync(0xffffffffu, rescale)) {
+#pragma unroll
+          for (int g = 0; g < kOCols / 32; ++g) {
+            const uint32_t ta = lane_base + 256u + (uint32_t)(kOCols * half + 32 * g);
+            float o[32];
+            tmem_ld32(ta, o);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) o[e] *= fac;
+            tmem_st32(ta, o);
+          }
+        }
+        // P row `row`, keys [128 half, +128): chunks 2 half and 2 half + 1 of the P tile.
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+          uint4* dst = reinterpret_cast<uint4*>(pbuf + (2 * half + q) * S::kPChunkBytes + row * 128);
+#pragma unroll
+          for (int un = 0; un < 8; ++un) {
+            const int base = (64 * q + 8 * un) / 2;
+            dst[un ^ (row & 7)] = make_uint4(pk[base], pk[base + 1], pk[base + 2], pk[base + 3]);
+          }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(pfull);
+        ++n_pf;
+      }
+      if (bad) break;
+      // ---- unit output: wait for the last PX, drain O, hand TMEM back, store.
+      if (n_pf > n_pe) {
+        if (!wait_all(pempty, n_pe & 1, 323)) break;
+        ++n_pe;
+      }
+      tc_fence_after();
+      float o[kOCols];
+#pragma unroll
+      for (int g = 0; g < kOCols / 32; ++g) {
+        float tmp[32];
+        tmem_ld32(lane_base + 256u + (uint32_t)(kOCols * half + 32 * g), tmp);
+#pragma unroll
+        for (int e = 0; e < 32; ++e) o[32 * g + e] = tmp[e];
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(ofree);
+      const float l_tot = l_part + exchange(l_part, 324);
+      if (bad) break;
+      const int r = w.tm * kBM + row;
+      if (r < f.t) {
+        const int64_t orow = ((int64_t)w.split * f.nb + w.b) * f.t + r;
+        float4* dst = reinterpret_cast<float4*>(f.O + orow * D2 + kOCols * half);
+#pragma unroll
+        for (int c = 0; c < kOCols; c += 4) dst[c / 4] = make_float4(o[c], o[c + 1], o[c + 2], o[c + 3]);
+        if (half == 0) f.stats[orow] = make_float2(m_run, l_tot);
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, 512);
+  }
+}
+
+// Splits the key tiles so that the units fill the SMs in near-whole waves.
+inline int flash_split(int64_t base_units, int tiles_k, int num_sms, int max_split) {
+  int best = 1;
+  double best_cost = 1e300;
+  for (int s = 1; s <= std::min(tiles_k, max_split); ++s) {
+    const int64_t units = base_units * s;
+    const double waves = (double)((units + num_sms - 1) / num_sms);
+    const double per_unit = (double)((tiles_k + s - 1) / s) + 0.25;
+    const double cost = waves * per_unit;
+    if (cost < best_cost - 1e-9) {
+      best_cost = cost;
+      best = s;
+    }
+  }
+  return best;
+}
+
+// Q: [nb*t][2D] bf16 (hi | lo), K: [nb*N][2D] bf16 (hi | lo), XT: [H*2d][2*Np] fp16 (hi | lo).
+template <int D2>
+inline cudaError_t launch_ca_flash(const Operand2D& Q, const Operand2D& K, const Operand2D& XT,
+                                   const FlashParams& f, int num_sms, cudaStream_t stream) {
+  using S = FlashSmem<D2>;
+  if (f.D <= 0 || f.D % kBK != 0 || f.t <= 0 || f.N <= 0 || f.Np % kBK != 0 || f.Np < f.N ||
+      f.nunits <= 0)
+    return cudaErrorInvalidValue;
+  CUtensorMap tq, tk, thi, tlo;
+  if (!make_tmap(&tq, Q, kBM) || !make_tmap(&tk, K, kFlashKeys) || !make_tmap(&thi, XT, D2) ||
+      !make_tmap(&tlo, XT, D2 / 2))
+    return cudaErrorInvalidValue;
+  auto kern = ca_flash_kernel<D2>;
+  static thread_local bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::kBytes);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  const int grid = f.nunits < num_sms ? f.nunits : num_sms;
+  kern<<<grid, kFlashThreads, S::kBytes, stream>>>(tq, tk, thi, tlo, f);
+  return cudaGetLastError();
+}
+
+}  // namespace still

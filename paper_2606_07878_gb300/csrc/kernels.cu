@@ -340,6 +340,37 @@ __global__ void px_to_hilo_kernel(const float* __restrict__ O, int nsplit, int64
   row[(int64_t)n * d2 + i * d2 + f] = lo;
 }
 
+// Key-split merge of the fused cross-attention. Split s holds, per row, the unnormalised
+// O_s = sum_k 2^(v_k - m_s) X_k and l_s = sum_k 2^(v_k - m_s) (v, m in log2 units). With
+// M = max_s m_s:  O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s, summed in split order.
+__global__ void ca_merge_kernel(const float* __restrict__ O, const float2* __restrict__ stats,
+                                int nsplit, int b0, int nb, int n, int t, int d2,
+                                __nv_bfloat16* __restrict__ PX) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t rows = (int64_t)nb * t;
+  if (idx >= rows * d2) return;
+  const int f = (int)(idx % d2);
+  const int64_t rj = idx / d2;
+  float M = -INFINITY;
+  for (int k = 0; k < nsplit; ++k) M = fmaxf(M, stats[k * rows + rj].x);
+  float L = 0.f, acc = 0.f;
+  for (int k = 0; k < nsplit; ++k) {
+    const float2 st = stats[k * rows + rj];
+    const float w = exp2f(st.x - M);
+    L += w * st.y;
+    acc += w * O[(k * rows + rj) * d2 + f];
+  }
+  const float o = acc / L;
+  const int j = (int)(rj % t), bb = (int)(rj / t);
+  const int b = b0 + bb, h = b / n, i = b % n;
+  const int64_t ld = 2 * (int64_t)n * d2;
+  __nv_bfloat16 hi, lo;
+  split_hilo(o, hi, lo);
+  __nv_bfloat16* row = PX + ((int64_t)h * t + j) * ld;
+  row[i * d2 + f] = hi;
+  row[(int64_t)n * d2 + i * d2 + f] = lo;
+}
+
 __global__ void __launch_bounds__(256) rmsnorm_kernel(const void* __restrict__ in, int in_bf16,
                                                       int64_t rows, int D, int64_t ldi, float eps,
                                                       __nv_bfloat16* __restrict__ out,
@@ -507,6 +538,14 @@ cudaError_t launch_px_to_hilo(const float* O, int nsplit, int64_t split_stride, 
   const int64_t total = (int64_t)nb * t * d2;
   px_to_hilo_kernel<<<blocks_for(total, 256), 256, 0, s>>>(O, nsplit, split_stride, b0, nb, n,
                                                            t, d2, PX);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_ca_merge(const float* O, const float2* stats, int nsplit, int b0, int nb,
+                            int n, int t, int d2, __nv_bfloat16* PX, cudaStream_t s) {
+  const int64_t total = (int64_t)nb * t * d2;
+  if (total == 0) return cudaSuccess;
+  ca_merge_kernel<<<blocks_for(total, 256), 256, 0, s>>>(O, stats, nsplit, b0, nb, n, t, d2, PX);
   return cudaGetLastError();
 }
 

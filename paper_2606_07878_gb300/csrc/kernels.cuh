@@ -62,6 +62,12 @@ cudaError_t launch_softmax(const float* S, int64_t rows, int64_t ncols, int64_t 
 cudaError_t launch_px_to_hilo(const float* O, int nsplit, int64_t split_stride, int b0, int nb,
                               int n, int t, int d2, __nv_bfloat16* PX, cudaStream_t s);
 
+// Key-split merge of the fused cross-attention: O [nsplit][nb][t][2d] unnormalised partials with
+// stats [nsplit][nb][t] = (max in log2 units, sum) -> normalised hi/lo bf16 rows of PXcat
+// (layout as launch_px_to_hilo). Splits are combined in a fixed order.
+cudaError_t launch_ca_merge(const float* O, const float2* stats, int nsplit, int b0, int nb,
+                            int n, int t, int d2, __nv_bfloat16* PX, cudaStream_t s);
+
 // out[i] = alpha / max(sqrt(sum_k parts[i * nparts + k]), eps), summed in slot order: the
 // L2 / QK-norm factor of vector i from the epilogues' sum-of-squares partials.
 cudaError_t launch_inv_norms(const float* parts, int64_t nvec, int nparts, float eps,

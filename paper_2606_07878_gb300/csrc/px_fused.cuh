@@ -202,7 +202,7 @@ __global__ void __launch_bounds__(kPxThreads, 1)
     constexpr float kLog2e = 1.4426950408889634f;
     int stage = 0;
     uint32_t phase = 0;
-    for (int tile = blockIdx.x; tile < p.ntiles && !*abort_flag; tile += gridDim.x) {
+    for (int tile = blockIdx.x; tile < p.ntiles && !warp_flag(abort_flag); tile += gridDim.x) {
       const TileCoord tc = decode_tile(p, tile);
       float2 st[8];
       const float* srow[8];
@@ -281,7 +281,7 @@ __global__ void __launch_bounds__(kPxThreads, 1)
       const TileCoord tc = decode_tile(p, tile);
       bool ok = mbar_wait(&tfull[acc], acc_phase);
       ok = __all_sync(0xffffffffu, ok);
-      if (!ok || *abort_flag) {
+      if (!ok || warp_flag(abort_flag)) {
         if (lane == 0 && !ok) {
           dev_set_error(p.err, DEV_WAIT_TIMEOUT, 204);
           *abort_flag = 1;

@@ -24,6 +24,7 @@
 #include "gemm_host.cuh"
 #include "kernels.cuh"
 #include "px_fused.cuh"
+#include "ca_flash.cuh"
 
 using namespace still;
 
@@ -140,6 +141,7 @@ namespace {
 inline int64_t rup(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
 
 constexpr int kMaxSplit = 8;  // split-K factor cap (partials are reduced in a fixed order)
+constexpr int kMaxFlashSplit = 16;  // key-split cap of the fused cross-attention
 
 void free_layer(LayerW& L) {
   for (void* p : L.owned) cudaFree(p);
@@ -263,6 +265,7 @@ struct Plan {
   int H, d, D, n, F, t;
   int64_t N, Np, ldS, tp, ldt;
   int G;
+  bool flash;     // fused cross-attention kernel (2d of 128 or 256), else scores + P X kernels
   int ca_units;   // (h, i) pairs per cross-attention group
   int sa_heads;   // KV-heads per self-attention group
   // byte offsets
@@ -313,9 +316,16 @@ bool make_plan(const still_layer_config& c, int64_t N, int t, double pmin, doubl
   P.kb_b = a256(N * 2 * D * 2);
   P.kss_b = a256(N * 4 * (EpiRopeC::kParts * (D / 256) + 1));  // |k~|^2 partials + inverses
   P.q_b = a256(T * 2 * D * 2);
-  P.S_b = a256(T * P.ldS * 4);
-  P.P_b = a256(T * 8 * (2 * ((N + 255) / 256) + 1));  // row-softmax partials + statistics
-  P.O_b = a256(T * 2 * d * 4) * kMaxSplit;       // split-K partials of P X
+  P.flash = d == 64 || d == 128;
+  if (P.flash) {
+    P.S_b = 0;
+    P.P_b = a256(T * 8) * kMaxFlashSplit;          // per-split row statistics (m, l)
+    P.O_b = a256(T * 2 * d * 4) * kMaxFlashSplit;  // per-split unnormalised O
+  } else {
+    P.S_b = a256(T * P.ldS * 4);
+    P.P_b = a256(T * 8 * (2 * ((N + 255) / 256) + 1));  // row-softmax partials + statistics
+    P.O_b = a256(T * 2 * d * 4) * kMaxSplit;             // split-K partials of P X
+  }
   P.ca_unit_bytes = P.kb_b + P.kss_b + P.q_b + P.S_b + P.P_b + P.O_b;
   P.qk_b = a256(2 * n * T * 2 * D * 2);
   P.sss_b = a256(2 * n * T * 4 * (2 * (D / 256) + 1));
@@ -503,6 +513,40 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     KLAUNCH(STILL_K_NORMS, launch_inv_norms(kss, (int64_t)nbl * N, kparts, c.l2_eps, scale, kinv, s));
     KLAUNCH(STILL_K_QROPE, launch_q_rope(L.qhat, c.t_max, b0, nbl, t, D, qstart, qstep, L.omega_c,
                      c.compactor_rope, qhl, s));
+    if (P.flash) {
+      // S, the online softmax and P X in one kernel; per-split partials merged in order.
+      float2* fst = stp;  // [nsplit][nbl * t] (the statistics region of this path)
+      FlashParams fp;
+      fp.t = t;
+      fp.N = (int)N;
+      fp.D = D;
+      fp.Np = Np;
+      fp.nb = nbl;
+      fp.bdiv = ni;
+      fp.xbase_row = h0 * 2 * d;
+      fp.tiles_m = (t + kBM - 1) / kBM;
+      fp.tiles_k = (int)((N + kFlashKeys - 1) / kFlashKeys);
+      fp.nsplit = flash_split((int64_t)fp.tiles_m * nbl, fp.tiles_k, ctx->nsm, kMaxFlashSplit);
+      const int64_t nunits = (int64_t)fp.tiles_m * nbl * fp.nsplit;
+      if (nunits > 0x7fffffff || (int64_t)nbl * N > 0x7fffffff) return STILL_ERR_UNSUPPORTED;
+      fp.nunits = (int)nunits;
+      fp.kinv = kinv;
+      fp.O = O;
+      fp.stats = fst;
+      fp.err = ctx->err;
+      const Operand2D qop = op(qhl, (int64_t)nbl * t, 2 * D);
+      const Operand2D kop = op(kb, (int64_t)nbl * N, 2 * D);
+      const Operand2D xop = op(XT, (int64_t)H * 2 * d, 2 * Np);
+      ctx->prof.begin(STILL_K_CA_FUSED, s);
+      cudaError_t r = d == 64 ? launch_ca_flash<128>(qop, kop, xop, fp, ctx->nsm, s)
+                              : launch_ca_flash<256>(qop, kop, xop, fp, ctx->nsm, s);
+      ctx->prof.end(STILL_K_CA_FUSED, s);
+      if (r == cudaErrorInvalidValue) return STILL_ERR_INVALID_ARG;
+      if (r != cudaSuccess) return STILL_ERR_CUDA;
+      KLAUNCH(STILL_K_PXSPLIT, launch_ca_merge(O, fst, fp.nsplit, b0, nbl, n, t, 2 * d, PX, s));
+      b0 += nbl;
+      continue;
+    }
     {  // S = scale * q.k / |k~|
       GemmParams p = gp(t, (int)N, nbl, 1);
       p.a_r1 = t;
@@ -1314,7 +1358,7 @@ const char* still_kernel_class_name(int32_t cls) {
   static const char* names[STILL_K_COUNT] = {
       "strip", "rope_tables", "keyproj", "q_rope", "scores", "softmax", "px", "px_split",
       "vo", "rmsnorm", "sa_proj", "sa_v", "sa_scores", "sa_softmax", "sa_pv", "sa_out",
-      "ffn1", "ffn2", "heads", "norms", "load"};
+      "ffn1", "ffn2", "heads", "norms", "load", "ca_fused"};
   return cls >= 0 && cls < STILL_K_COUNT ? names[cls] : "unknown";
 }
 

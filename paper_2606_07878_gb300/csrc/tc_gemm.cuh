@@ -287,7 +287,7 @@ __global__ void __launch_bounds__(gemm_threads<Epi>(), 1)
       const TileCoord tc = decode_tile(p, tile);
       bool ok = mbar_wait(&tfull[acc], acc_phase);
       ok = __all_sync(0xffffffffu, ok);
-      if (!ok || *abort_flag) {
+      if (!ok || warp_flag(abort_flag)) {
         if (lane == 0 && !ok) {
           dev_set_error(p.err, DEV_WAIT_TIMEOUT, 103);
           *abort_flag = 1;
