@@ -27,20 +27,40 @@ __device__ __forceinline__ int64_t kv_offset(const KVSource& src, int64_t n, int
                 : n * src.sN + (int64_t)h * src.sH;
 }
 
+// Eight consecutive bf16 of a K / V row as fp32 (one 16-byte load when aligned).
+__device__ __forceinline__ void load8(const __nv_bfloat16* p, bool vec, float (&v)[8]) {
+  if (vec) {
+    const uint4 u = *reinterpret_cast<const uint4*>(p);
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[k]));
+      v[2 * k] = f.x;
+      v[2 * k + 1] = f.y;
+    }
+  } else {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) v[e] = __bfloat162float(p[e]);
+  }
+}
+
 // One CTA = 32 tokens x all KV-heads. The base-RoPE angles of the tile's tokens are formed
 // once (fp64, reduced mod 2 pi) and reused by every KV-head. Keys: inverse rotation of pairs
 // (m, m + d/2) (Sec. 2.2, RoPE-fix); values pass through. Writes X (bf16 hi | key lo) and XT
-// (fp16 hi, lo).
+// (fp16 hi for all 2d features, fp16 lo for the key half; the value half's lo is exactly zero
+// and is never read). Rows are moved in 16-byte pieces; the transpose for XT goes through
+// shared memory with an odd word pitch (conflict-free column reads).
 __global__ void __launch_bounds__(256) strip_kernel(KVSource src, int64_t N, int H, int d,
                                                     PosSegs segs, const double* __restrict__ omega,
-                                                    int rope_fix, __nv_bfloat16* __restrict__ X,
+                                                    int rope_fix, int vec,
+                                                    __nv_bfloat16* __restrict__ X,
                                                     __half* __restrict__ XT, int64_t Np) {
   extern __shared__ __align__(16) uint8_t sm[];
   const int half = d / 2;
-  constexpr int kLd = kStripTok + 2;
-  float2* rot = reinterpret_cast<float2*>(sm);              // [kStripTok][half]: (cos, sin)
-  __half* thi = reinterpret_cast<__half*>(rot + kStripTok * half);
-  __half* tlo = thi + 2 * d * kLd;
+  const int ph = 2 * d + 2, pl = d + 2;  // pitches (halves) of the transpose tiles
+  float2* rot = reinterpret_cast<float2*>(sm);  // [kStripTok][half]: (cos, sin)
+  __half* thi = reinterpret_cast<__half*>(rot + kStripTok * half);  // [kStripTok][ph]
+  __half* tlo = thi + kStripTok * ph;                                 // [kStripTok][pl]
   const int64_t n0 = (int64_t)blockIdx.x * kStripTok;
   for (int it = threadIdx.x; it < kStripTok * half; it += blockDim.x) {
     const int tok = it / half, m = it % half;
@@ -52,61 +72,110 @@ __global__ void __launch_bounds__(256) strip_kernel(KVSource src, int64_t N, int
   __syncthreads();
   const int d3 = 3 * d;
   const int64_t ld = 2 * Np;
+  const int kg = half / 8, vg = d / 8;  // 8-element groups per token: key pairs, values
   for (int h = 0; h < H; ++h) {
-    for (int it = threadIdx.x; it < kStripTok * half; it += blockDim.x) {
-      const int tok = it / half, m = it % half;
+    // keys: group g holds pairs m = 8g .. 8g + 7
+    for (int it = threadIdx.x; it < kStripTok * kg; it += blockDim.x) {
+      const int tok = it / kg, m0 = 8 * (it % kg);
       const int64_t n = n0 + tok;
-      float a = 0.f, b = 0.f;
+      float a[8], b[8];
       if (n < N) {
         bool second;
         const int64_t off = kv_offset(src, n, h, second);
         const __nv_bfloat16* kr = (second ? src.K2 : src.K) + off;
-        a = __bfloat162float(kr[m]);
-        b = __bfloat162float(kr[m + half]);
-        const float2 cs = rot[it];
-        const float x = a * cs.x + b * cs.y;
-        const float y = -a * cs.y + b * cs.x;
-        a = x;
-        b = y;
+        float ka[8], kb[8];
+        load8(kr + m0, vec, ka);
+        load8(kr + half + m0, vec, kb);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float2 cs = rot[tok * half + m0 + e];
+          a[e] = ka[e] * cs.x + kb[e] * cs.y;
+          b[e] = -ka[e] * cs.y + kb[e] * cs.x;
+        }
+        uint32_t ah[4], al[4], bh[4], bl[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          split_pack(a[2 * k], a[2 * k + 1], ah[k], al[k]);
+          split_pack(b[2 * k], b[2 * k + 1], bh[k], bl[k]);
+        }
         __nv_bfloat16* xr = X + ((int64_t)h * N + n) * d3;
-        __nv_bfloat16 hi, lo;
-        split_hilo(a, hi, lo);
-        xr[m] = hi;
-        xr[2 * d + m] = lo;
-        split_hilo(b, hi, lo);
-        xr[m + half] = hi;
-        xr[2 * d + m + half] = lo;
+        if (vec) {
+          *reinterpret_cast<uint4*>(xr + m0) = make_uint4(ah[0], ah[1], ah[2], ah[3]);
+          *reinterpret_cast<uint4*>(xr + half + m0) = make_uint4(bh[0], bh[1], bh[2], bh[3]);
+          *reinterpret_cast<uint4*>(xr + 2 * d + m0) = make_uint4(al[0], al[1], al[2], al[3]);
+          *reinterpret_cast<uint4*>(xr + 2 * d + half + m0) = make_uint4(bl[0], bl[1], bl[2], bl[3]);
+        } else {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            reinterpret_cast<uint32_t*>(xr + m0)[k] = ah[k];
+            reinterpret_cast<uint32_t*>(xr + half + m0)[k] = bh[k];
+            reinterpret_cast<uint32_t*>(xr + 2 * d + m0)[k] = al[k];
+            reinterpret_cast<uint32_t*>(xr + 2 * d + half + m0)[k] = bl[k];
+          }
+        }
+      } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) a[e] = b[e] = 0.f;
       }
-      const __half ah = __float2half_rn(a), bh = __float2half_rn(b);
-      thi[m * kLd + tok] = ah;
-      thi[(m + half) * kLd + tok] = bh;
-      tlo[m * kLd + tok] = __float2half_rn(a - __half2float(ah));
-      tlo[(m + half) * kLd + tok] = __float2half_rn(b - __half2float(bh));
+      __half* hr = thi + tok * ph;
+      __half* lr = tlo + tok * pl;
+#pragma unroll
+      for (int e = 0; e < 8; e += 2) {
+        const __half2 ha = __floats2half2_rn(a[e], a[e + 1]);
+        const __half2 hb = __floats2half2_rn(b[e], b[e + 1]);
+        const float2 fa = __half22float2(ha), fb = __half22float2(hb);
+        *reinterpret_cast<__half2*>(hr + m0 + e) = ha;
+        *reinterpret_cast<__half2*>(hr + half + m0 + e) = hb;
+        *reinterpret_cast<__half2*>(lr + m0 + e) = __floats2half2_rn(a[e] - fa.x, a[e + 1] - fa.y);
+        *reinterpret_cast<__half2*>(lr + half + m0 + e) =
+            __floats2half2_rn(b[e] - fb.x, b[e + 1] - fb.y);
+      }
     }
-    for (int it = threadIdx.x; it < kStripTok * d; it += blockDim.x) {
-      const int tok = it / d, f = it % d;
+    // values: group g holds features 8g .. 8g + 7 (bf16 values are exact in fp16)
+    for (int it = threadIdx.x; it < kStripTok * vg; it += blockDim.x) {
+      const int tok = it / vg, f0 = 8 * (it % vg);
       const int64_t n = n0 + tok;
-      float v = 0.f;
+      float v[8];
       if (n < N) {
         bool second;
         const int64_t off = kv_offset(src, n, h, second);
-        const __nv_bfloat16 vb = (second ? src.V2 : src.V)[off + f];
-        v = __bfloat162float(vb);
-        X[((int64_t)h * N + n) * d3 + d + f] = vb;
+        const __nv_bfloat16* vr = (second ? src.V2 : src.V) + off + f0;
+        load8(vr, vec, v);
+        __nv_bfloat16* xr = X + ((int64_t)h * N + n) * d3 + d + f0;
+        if (vec) {
+          *reinterpret_cast<uint4*>(xr) = *reinterpret_cast<const uint4*>(vr);
+        } else {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) xr[e] = vr[e];
+        }
+      } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[e] = 0.f;
       }
-      const __half vh = __float2half_rn(v);
-      thi[(d + f) * kLd + tok] = vh;
-      tlo[(d + f) * kLd + tok] = __float2half_rn(v - __half2float(vh));
+      __half* hr = thi + tok * ph + d + f0;
+#pragma unroll
+      for (int e = 0; e < 8; e += 2)
+        *reinterpret_cast<__half2*>(hr + e) = __floats2half2_rn(v[e], v[e + 1]);
     }
     __syncthreads();
-    for (int it = threadIdx.x; it < 2 * d * kStripTok; it += blockDim.x) {
-      const int f = it / kStripTok, tok = it % kStripTok;
-      const int64_t n = n0 + tok;
-      if (n < Np) {
-        __half* row = XT + ((int64_t)h * 2 * d + f) * ld;
-        row[n] = thi[f * kLd + tok];
-        row[Np + n] = tlo[f * kLd + tok];
+    // XT: feature rows of 32 tokens, 8 tokens (16 B) per store; hi rows [0, 2d), lo rows [0, d)
+    constexpr int kTg = kStripTok / 8;
+    const int nhi = 2 * d * kTg;
+    for (int it = threadIdx.x; it < 3 * d * kTg; it += blockDim.x) {
+      const bool lo = it >= nhi;
+      const int q = lo ? it - nhi : it;
+      const int f = q / kTg, t0 = 8 * (q % kTg);
+      const __half* col = lo ? tlo + f : thi + f;
+      const int pitch = lo ? pl : ph;
+      uint32_t w[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const __half x0 = col[(t0 + 2 * k) * pitch], x1 = col[(t0 + 2 * k + 1) * pitch];
+        const __half2 pr = __halves2half2(x0, x1);
+        w[k] = *reinterpret_cast<const uint32_t*>(&pr);
       }
+      __half* dst = XT + ((int64_t)h * 2 * d + f) * ld + (lo ? Np : 0) + n0 + t0;
+      *reinterpret_cast<uint4*>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
     }
     __syncthreads();
   }
@@ -343,32 +412,43 @@ __global__ void px_to_hilo_kernel(const float* __restrict__ O, int nsplit, int64
 // Key-split merge of the fused cross-attention. Split s holds, per row, the unnormalised
 // O_s = sum_k 2^(v_k - m_s) X_k and l_s = sum_k 2^(v_k - m_s) (v, m in log2 units). With
 // M = max_s m_s:  O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s, summed in split order.
-__global__ void ca_merge_kernel(const float* __restrict__ O, const float2* __restrict__ stats,
-                                int nsplit, int b0, int nb, int n, int t, int d2,
-                                __nv_bfloat16* __restrict__ PX) {
-  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+// One warp per row; each lane owns 4-column groups (16-byte loads).
+__global__ void __launch_bounds__(256) ca_merge_kernel(const float* __restrict__ O,
+                                                       const float2* __restrict__ stats,
+                                                       int nsplit, int b0, int nb, int n, int t,
+                                                       int d2, __nv_bfloat16* __restrict__ PX) {
   const int64_t rows = (int64_t)nb * t;
-  if (idx >= rows * d2) return;
-  const int f = (int)(idx % d2);
-  const int64_t rj = idx / d2;
+  const int64_t rj = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (rj >= rows) return;
   float M = -INFINITY;
   for (int k = 0; k < nsplit; ++k) M = fmaxf(M, stats[k * rows + rj].x);
-  float L = 0.f, acc = 0.f;
+  float L = 0.f;
   for (int k = 0; k < nsplit; ++k) {
     const float2 st = stats[k * rows + rj];
-    const float w = exp2f(st.x - M);
-    L += w * st.y;
-    acc += w * O[(k * rows + rj) * d2 + f];
+    L += exp2f(st.x - M) * st.y;
   }
-  const float o = acc / L;
+  const float invL = 1.f / L;
   const int j = (int)(rj % t), bb = (int)(rj / t);
   const int b = b0 + bb, h = b / n, i = b % n;
   const int64_t ld = 2 * (int64_t)n * d2;
-  __nv_bfloat16 hi, lo;
-  split_hilo(o, hi, lo);
-  __nv_bfloat16* row = PX + ((int64_t)h * t + j) * ld;
-  row[i * d2 + f] = hi;
-  row[(int64_t)n * d2 + i * d2 + f] = lo;
+  __nv_bfloat16* row = PX + ((int64_t)h * t + j) * ld + (int64_t)i * d2;
+  for (int c = 4 * lane; c < d2; c += 128) {
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int k = 0; k < nsplit; ++k) {
+      const float w = exp2f(stats[k * rows + rj].x - M);
+      const float4 o = *reinterpret_cast<const float4*>(O + (k * rows + rj) * d2 + c);
+      acc.x += w * o.x;
+      acc.y += w * o.y;
+      acc.z += w * o.z;
+      acc.w += w * o.w;
+    }
+    uint32_t h01, l01, h23, l23;
+    split_pack(acc.x * invL, acc.y * invL, h01, l01);
+    split_pack(acc.z * invL, acc.w * invL, h23, l23);
+    *reinterpret_cast<uint2*>(row + c) = make_uint2(h01, h23);
+    *reinterpret_cast<uint2*>(row + (int64_t)n * d2 + c) = make_uint2(l01, l23);
+  }
 }
 
 __global__ void __launch_bounds__(256) rmsnorm_kernel(const void* __restrict__ in, int in_bf16,
@@ -453,15 +533,21 @@ inline unsigned blocks_for(int64_t n, int per) { return (unsigned)((n + per - 1)
 cudaError_t launch_strip(const KVSource& src, int64_t N, int H, int d, const PosSegs& segs,
                          const double* omega, int rope_fix, __nv_bfloat16* X, __half* XT,
                          int64_t Np, cudaStream_t s) {
+  if (d % 16 != 0 || Np % kStripTok != 0) return cudaErrorInvalidValue;
   const size_t smem = (size_t)kStripTok * (d / 2) * sizeof(float2) +
-                      2 * (size_t)(2 * d) * (kStripTok + 2) * 2;
+                      (size_t)kStripTok * ((2 * d + 2) + (d + 2)) * 2;
+  auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
+  const bool second = src.n_split < N;
+  const int vec = al16(src.K) && al16(src.V) && src.sN % 8 == 0 && src.sH % 8 == 0 &&
+                  (!second || (al16(src.K2) && al16(src.V2) && src.sN2 % 8 == 0 &&
+                               src.sH2 % 8 == 0));
   static bool attr = false;
   if (!attr) {
     cudaFuncSetAttribute(strip_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 128 * 1024);
     attr = true;
   }
   strip_kernel<<<(unsigned)(Np / kStripTok), 256, smem, s>>>(src, N, H, d, segs, omega, rope_fix,
-                                                             X, XT, Np);
+                                                             vec, X, XT, Np);
   return cudaGetLastError();
 }
 
@@ -545,7 +631,9 @@ cudaError_t launch_ca_merge(const float* O, const float2* stats, int nsplit, int
                             int n, int t, int d2, __nv_bfloat16* PX, cudaStream_t s) {
   const int64_t total = (int64_t)nb * t * d2;
   if (total == 0) return cudaSuccess;
-  ca_merge_kernel<<<blocks_for(total, 256), 256, 0, s>>>(O, stats, nsplit, b0, nb, n, t, d2, PX);
+  if (d2 % 4 != 0) return cudaErrorInvalidValue;
+  ca_merge_kernel<<<blocks_for((int64_t)nb * t, 8), 256, 0, s>>>(O, stats, nsplit, b0, nb, n, t,
+                                                                  d2, PX);
   return cudaGetLastError();
 }
 
