@@ -26,6 +26,7 @@ __device__ __forceinline__ void split_hilo(float x, __nv_bfloat16& hi, __nv_bflo
   lo = __float2bfloat16_rn(x - __bfloat162float(hi));
 }
 
+// GELU with the exact (erf) form, 0.5 x (1 + erf(x / sqrt 2)) (App. A, Feed-forward).
 __device__ __forceinline__ float gelu_erf(float x) {
   return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f));
 }
@@ -87,6 +88,7 @@ __device__ __forceinline__ void pack_f32x16(const float* v, uint4 (&o)[4]) {
 struct EpiAffine {
   static constexpr int kWarps = 8;  // two per lane quarter: alternating 32-column chunks
   static constexpr int kStages = 0;  // default pipeline depth
+  static constexpr int kStoreBufs = 1;
   int32_t kind = OUT_F32;
   void* out = nullptr;
   int64_t lo_off = 0;  // OUT_HILO: lo element offset from hi
@@ -117,6 +119,20 @@ struct EpiAffine {
   int32_t stat_slots = 0;
   int32_t tile_cols_ = 256;  // the tile width BN, set by the launcher
 
+  // The residual rows of this warp's columns are pulled into L2 while the main loop runs.
+  __device__ void prefetch(const GemmParams& p, const TileCoord& tc, int row, int half) const {
+    if (res_kind == 0 || tc.split != 0) return;
+    const int r = tc.tm * kBM + row;
+    if (r >= p.M) return;
+    const int esz = res_kind == 1 ? 4 : 2;
+    for (int cc = 32 * half; cc < tile_cols_; cc += 64) {
+      const int c0 = tc.tn * tile_cols_ + cc;
+      if (c0 >= p.N) break;
+      const char* base = static_cast<const char*>(res) + resm.at(tc.b, r, c0) * esz;
+      for (int off = 0; off < 32 * esz; off += 32) prefetch_l2(base + off);  // per 32-B sector
+    }
+  }
+
   __device__ void operator()(const GemmParams& p, const TileCoord& tc, int row, uint32_t taddr,
                              int half, uint4* stage, const CUtensorMap* tmc) const {
     const int r = tc.tm * kBM + row;
@@ -133,6 +149,37 @@ struct EpiAffine {
       const int nv = min(32, p.N - c0);
 #pragma unroll
       for (int e = 0; e < 32; ++e) v[e] *= rscale;
+      // Residual rows read coalesced by the whole warp (before the invalid-row exit: every
+      // lane takes part). Not on the TMA-store path, whose staging area may still be in use.
+      const bool res_vec = res_kind != 0 && tc.split == 0 && vec_ok && !tma_f32 && nv == 32;
+      float resv[32];
+      if (res_vec) {
+        const int64_t o = rvalid ? resm.at(tc.b, r, c0) : 0;
+        if (res_kind == 1) {
+          uint4 u[8];
+          warp_load_rows<8>(stage, static_cast<const float*>(res) + o, rvalid, u);
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            resv[4 * q] = __uint_as_float(u[q].x);
+            resv[4 * q + 1] = __uint_as_float(u[q].y);
+            resv[4 * q + 2] = __uint_as_float(u[q].z);
+            resv[4 * q + 3] = __uint_as_float(u[q].w);
+          }
+        } else {
+          uint4 u[4];
+          warp_load_rows<4>(stage, static_cast<const __nv_bfloat16*>(res) + o, rvalid, u);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const uint32_t w[4] = {u[q].x, u[q].y, u[q].z, u[q].w};
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[k]));
+              resv[8 * q + 2 * k] = f.x;
+              resv[8 * q + 2 * k + 1] = f.y;
+            }
+          }
+        }
+      }
       if (!rvalid) {  // keep the warp-collective stores; the row itself is not written
         if (tma_f32)
           store32_tma(tc, row, c0, v, stage, tmc);
@@ -173,7 +220,10 @@ struct EpiAffine {
 #pragma unroll
         for (int e = 0; e < 32; ++e) v[e] = gelu_erf(v[e]);
       }
-      if (res_kind != 0 && tc.split == 0) {
+      if (res_vec) {
+#pragma unroll
+        for (int e = 0; e < 32; ++e) v[e] += resv[e];
+      } else if (res_kind != 0 && tc.split == 0) {
         const int64_t o = resm.at(tc.b, r, c0);
         if (res_kind == 1) {
           const float* rp = static_cast<const float*>(res) + o;
@@ -287,7 +337,9 @@ __device__ __forceinline__ double seg_position(const PosSegs& s, int64_t idx) {
 // Columns are in "pair-chunk" order: within each 256-column tile, columns [0,128) hold the
 // first elements of 128 RoPE pairs and [128,256) their partners, so a tile owns whole pairs.
 // The angle p_n * omega_m is split as G_g * omega_m (table, built in fp64) + delta * omega_m
-// (fp32, delta = p_n - G_g in [0, kPosGrain)), combined by the angle-addition formulas.
+// (fp32, delta = p_n - G_g in [0, kPosGrain)), combined by the angle-addition formulas. The
+// per-token (g, delta) come from a table formed once per call in fp64 (gd[n] = (g, delta)), so
+// the epilogue itself does no fp64 arithmetic.
 constexpr int kPosGrain = 32;
 
 struct EpiRopeC {
@@ -296,16 +348,18 @@ struct EpiRopeC {
   static constexpr int kWarps = 16;
   static constexpr int kParts = kWarps / 4;
   static constexpr int kStages = 3;
+  static constexpr int kStoreBufs = 1;  // 4 KB TMA-store staging buffers per warp
   __nv_bfloat16* out = nullptr;  // [H][n][N][2D]: hi at [0, D), lo at [D, 2D) (via the TMA view)
   float* sumsq = nullptr;        // [H][n][N][kParts * D / 256] partial sums of |k~|^2
   const float* bias = nullptr;   // [n*D], pair-chunk order
   const float2* coarse = nullptr;  // [G][D/2]: (cos, sin)(G_g * omega_m)
   const float* omega = nullptr;    // [D/2] fp32
-  PosSegs segs;
-  double pmin = 0;
+  const float2* gd = nullptr;      // [Ntok]: (coarse index g as float, delta)
   int32_t D = 0, nheads = 0, ncoarse = 0;
   int64_t Ntok = 0;
   int32_t tile_cols_ = 256;  // must be 256: a tile holds 128 whole RoPE pairs
+
+  __device__ void prefetch(const GemmParams&, const TileCoord&, int, int) const {}
 
   __device__ void operator()(const GemmParams& p, const TileCoord& tc, int row, uint32_t taddr,
                              int half, uint4* stage, const CUtensorMap* tmc) const {
@@ -317,32 +371,41 @@ struct EpiRopeC {
     const int head = c_tile / D;
     const int f_tile = c_tile % D;       // column of this tile inside the head (pair-chunk order)
     const int m_base = (f_tile / 256) * 128;  // first pair index of this tile
-    double pos = rvalid ? seg_position(segs, r) : pmin;
-    int g = (int)floor((pos - pmin) / (double)kPosGrain);
-    g = max(0, min(g, ncoarse - 1));
-    const float delta = (float)(pos - (pmin + (double)g * kPosGrain));
+    const float2 gdr = rvalid ? gd[r] : make_float2(0.f, 0.f);
+    const int g = max(0, min((int)gdr.x, ncoarse - 1));
+    const float delta = gdr.y;
     float ss = 0.f;
-    // part p owns pairs [32p, 32p + 32) of the tile, taken 16 at a time
-    for (int u = 32 * half; u < 32 * half + 32; u += 16) {
-      float a[16], bb[16];
-      tmem_ld16(taddr + (uint32_t)u, a);
-      tmem_ld16(taddr + (uint32_t)(128 + u), bb);
+    // Part p owns pairs [32p, 32p + 32) of the tile, taken 16 at a time. With kStoreBufs = 2 the
+    // staging area holds two 4 KB buffers used alternately, so one iteration's TMA stores can
+    // still be reading while the next fills the other buffer.
+    for (int it = 0; it < 2; ++it) {
+      const int u = 32 * half + 16 * it;
+      // tables first: their latency overlaps the TMEM loads
       const float4* crow = reinterpret_cast<const float4*>(coarse + (int64_t)g * (D / 2) + m_base + u);
       const float4* om4 = reinterpret_cast<const float4*>(omega + m_base + u);
       const float4* ba4 = reinterpret_cast<const float4*>(bias + c_tile + u);
       const float4* bb4 = reinterpret_cast<const float4*>(bias + c_tile + 128 + u);
+      float4 w[4], xa[4], xb[4], cs[8];
 #pragma unroll
-      for (int e4 = 0; e4 < 4; ++e4) {
-        const float4 w = om4[e4], xa = ba4[e4], xb = bb4[e4];
-        const float4 c01 = crow[2 * e4], c23 = crow[2 * e4 + 1];
-        const float ws[4] = {w.x, w.y, w.z, w.w};
-        const float bas[4] = {xa.x, xa.y, xa.z, xa.w};
-        const float bbs[4] = {xb.x, xb.y, xb.z, xb.w};
-        const float cc[4] = {c01.x, c01.z, c23.x, c23.z};  // cos(G w) of the 4 pairs
-        const float sc[4] = {c01.y, c01.w, c23.y, c23.w};  // sin(G w)
+      for (int q = 0; q < 4; ++q) {
+        w[q] = om4[q];
+        xa[q] = ba4[q];
+        xb[q] = bb4[q];
+        cs[2 * q] = crow[2 * q];
+        cs[2 * q + 1] = crow[2 * q + 1];
+      }
+      float a[16], bb[16];
+      tmem_ld16x2(taddr + (uint32_t)u, taddr + (uint32_t)(128 + u), a, bb);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float ws[4] = {w[q].x, w[q].y, w[q].z, w[q].w};
+        const float bas[4] = {xa[q].x, xa[q].y, xa[q].z, xa[q].w};
+        const float bbs[4] = {xb[q].x, xb[q].y, xb[q].z, xb[q].w};
+        const float cc[4] = {cs[2 * q].x, cs[2 * q].z, cs[2 * q + 1].x, cs[2 * q + 1].z};
+        const float sc[4] = {cs[2 * q].y, cs[2 * q].w, cs[2 * q + 1].y, cs[2 * q + 1].w};
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-          const int e = 4 * e4 + k;
+          const int e = 4 * q + k;
           const float x = a[e] + bas[k];
           const float y = bb[e] + bbs[k];
           ss += x * x + y * y;
@@ -356,31 +419,37 @@ struct EpiRopeC {
       }
       // Four boxes of 32 rows x 16 bf16 (hi a, lo a, hi b, lo b), 1 KB each, stored by TMA;
       // rows past N are clipped by the copy engine.
-      if (lane == 0) bulk_wait_read();
+      uint4* box = stage + (kStoreBufs == 2 ? (it & 1) * 256 : 0);
+      if (lane == 0) {
+        if (kStoreBufs == 2)
+          bulk_wait_read1();
+        else
+          bulk_wait_read();
+      }
       __syncwarp();
-      uint4* box = stage + lane * 2;
+      uint4* bl = box + lane * 2;
 #pragma unroll
       for (int q = 0; q < 2; ++q) {
         uint32_t h[4], l[4];
 #pragma unroll
         for (int k = 0; k < 4; ++k) split_pack(a[8 * q + 2 * k], a[8 * q + 2 * k + 1], h[k], l[k]);
-        box[q] = make_uint4(h[0], h[1], h[2], h[3]);
-        box[64 + q] = make_uint4(l[0], l[1], l[2], l[3]);
+        bl[q] = make_uint4(h[0], h[1], h[2], h[3]);
+        bl[64 + q] = make_uint4(l[0], l[1], l[2], l[3]);
 #pragma unroll
         for (int k = 0; k < 4; ++k)
           split_pack(bb[8 * q + 2 * k], bb[8 * q + 2 * k + 1], h[k], l[k]);
-        box[128 + q] = make_uint4(h[0], h[1], h[2], h[3]);
-        box[192 + q] = make_uint4(l[0], l[1], l[2], l[3]);
+        bl[128 + q] = make_uint4(h[0], h[1], h[2], h[3]);
+        bl[192 + q] = make_uint4(l[0], l[1], l[2], l[3]);
       }
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) {
         const int z = tc.b * nheads + head;
         const int x = f_tile + u;
-        tma_store_3d(tmc, stage, x, row0, z);
-        tma_store_3d(tmc, stage + 64, D + x, row0, z);
-        tma_store_3d(tmc, stage + 128, x + 128, row0, z);
-        tma_store_3d(tmc, stage + 192, D + x + 128, row0, z);
+        tma_store_3d(tmc, box, x, row0, z);
+        tma_store_3d(tmc, box + 64, D + x, row0, z);
+        tma_store_3d(tmc, box + 128, x + 128, row0, z);
+        tma_store_3d(tmc, box + 192, D + x + 128, row0, z);
         bulk_commit();
       }
     }
@@ -394,19 +463,20 @@ struct EpiRopeC {
 
 // Output heads: columns [0, d) = Z_out W_key, re-rotated by the base RoPE at the output
 // position of latent j; columns [d, 2d) = Z_out W_val. Rows r = h * t + j. bf16 stores into
-// the caller's C_k / C_v with element strides (st, sh). omega = theta^(-2m/d) in fp64;
-// the angle is reduced modulo 2 pi in fp64 before the fp32 sin/cos.
+// the caller's C_k / C_v with element strides (st, sh). rot[j][m] = (cos, sin)(p_j * omega_m),
+// a table formed once per call with the angle reduced modulo 2 pi in fp64.
 struct EpiHeads {
   static constexpr int kWarps = 8;
   static constexpr int kStages = 0;
+  static constexpr int kStoreBufs = 1;
   __nv_bfloat16* ck = nullptr;
   __nv_bfloat16* cv = nullptr;
   int64_t st = 0, sh = 0;  // element strides of [t, H, d]; d is contiguous, rows 16-B aligned
   int32_t t = 0, d = 0;
-  double pstart = 0, pstep = 0;
-  const double* omega = nullptr;  // [d/2]
-  int32_t rope = 1;
+  const float2* rot = nullptr;  // [t][d/2]
   int32_t tile_cols_ = 256;
+
+  __device__ void prefetch(const GemmParams&, const TileCoord&, int, int) const {}
 
   __device__ void operator()(const GemmParams& p, const TileCoord& tc, int row, uint32_t taddr,
                              int half, uint4* stage, const CUtensorMap*) const {
@@ -414,7 +484,7 @@ struct EpiHeads {
     const bool rvalid = r < p.M;
     const int h = rvalid ? r / t : 0, j = rvalid ? r % t : 0;
     const int c_tile = tc.tn * tile_cols_;
-    const double pos = pstart + (double)j * pstep;
+    const float2* rrow = rot + (int64_t)j * (d / 2);
     const int64_t obase = (int64_t)j * st + (int64_t)h * sh;
     const int hd = d / 2;
     for (int cc = 32 * half; cc < tile_cols_; cc += 64) {
@@ -428,12 +498,8 @@ struct EpiHeads {
         tmem_ld32(taddr + (uint32_t)(cc + hd), b);
 #pragma unroll
         for (int e = 0; e < 32; ++e) {
-          float cw = 1.f, sw = 0.f;
-          if (rope) {
-            double ang = pos * omega[c0 + e];
-            ang -= 6.283185307179586 * rint(ang * 0.15915494309189535);
-            sincosf((float)ang, &sw, &cw);
-          }
+          const float2 cs = rrow[c0 + e];
+          const float cw = cs.x, sw = cs.y;
           const float x = a[e], y = b[e];
           a[e] = x * cw - y * sw;
           b[e] = x * sw + y * cw;

@@ -54,19 +54,33 @@ __global__ void __launch_bounds__(256) strip_kernel(KVSource src, int64_t N, int
                                                     PosSegs segs, const double* __restrict__ omega,
                                                     int rope_fix, int vec,
                                                     __nv_bfloat16* __restrict__ X,
-                                                    __half* __restrict__ XT, int64_t Np) {
+                                                    __half* __restrict__ XT, int64_t Np,
+                                                    float2* __restrict__ gd, double pmin, int G) {
   extern __shared__ __align__(16) uint8_t sm[];
+  __shared__ double tpos[kStripTok];
   const int half = d / 2;
   const int ph = 2 * d + 2, pl = d + 2;  // pitches (halves) of the transpose tiles
   float2* rot = reinterpret_cast<float2*>(sm);  // [kStripTok][half]: (cos, sin)
   __half* thi = reinterpret_cast<__half*>(rot + kStripTok * half);  // [kStripTok][ph]
   __half* tlo = thi + kStripTok * ph;                                 // [kStripTok][pl]
   const int64_t n0 = (int64_t)blockIdx.x * kStripTok;
+  if (threadIdx.x < kStripTok) {
+    // token position (fp64) once per token; also the compactor-RoPE coarse index and residual
+    const int64_t n = n0 + threadIdx.x;
+    const double pos = n < N ? seg_position(segs, n) : pmin;
+    tpos[threadIdx.x] = pos;
+    if (n < N) {
+      int g = (int)floor((pos - pmin) / (double)kPosGrain);
+      g = max(0, min(g, G - 1));
+      gd[n] = make_float2((float)g, (float)(pos - (pmin + (double)g * kPosGrain)));
+    }
+  }
+  __syncthreads();
   for (int it = threadIdx.x; it < kStripTok * half; it += blockDim.x) {
     const int tok = it / half, m = it % half;
     const int64_t n = n0 + tok;
     float sw = 0.f, cw = 1.f;
-    if (rope_fix && n < N) sincos_reduced(seg_position(segs, n) * omega[m], &sw, &cw);
+    if (rope_fix && n < N) sincos_reduced(tpos[tok] * omega[m], &sw, &cw);
     rot[it] = make_float2(cw, sw);
   }
   __syncthreads();
@@ -194,27 +208,57 @@ __global__ void rope_tables_kernel(float2* coarse, float* omega, int G, int D, d
   if (g == 0) omega[m] = (float)w;
 }
 
+// rot[j][m] = (cos, sin)(p_j * omega[m]), p_j = pstart + j * pstep, angle reduced in fp64;
+// (1, 0) when use_rope is 0.
+__global__ void heads_rot_kernel(float2* rot, int t, int hd, double pstart, double pstep,
+                                 const double* __restrict__ omega, int use_rope) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (int64_t)t * hd) return;
+  const int j = (int)(idx / hd), m = (int)(idx % hd);
+  float s = 0.f, c = 1.f;
+  if (use_rope) sincos_reduced((pstart + (double)j * pstep) * omega[m], &s, &c);
+  rot[idx] = make_float2(c, s);
+}
+
+// Thread = (latent j, 4 consecutive pairs m); the angles are formed once and reused for every
+// batch. Columns are in pair-chunk order: pair m sits at f1 = (m / 128) * 256 + m % 128 and its
+// partner at f1 + 128, so four consecutive pairs are four consecutive columns.
 __global__ void q_rope_kernel(const float* __restrict__ qhat, int t_max, int b0, int nb, int t,
                               int D, double qstart, double qstep, const double* omega_c,
                               int use_rope, __nv_bfloat16* __restrict__ qhl) {
-  const int half = D / 2;
+  const int half = D / 2, q4 = half / 4;
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= (int64_t)t * half) return;
-  const int j = (int)(idx / half), m = (int)(idx % half);
-  float s = 0.f, c = 1.f;
-  if (use_rope) sincos_reduced((qstart + (double)j * qstep) * omega_c[m], &s, &c);
-  const int f1 = (m / 128) * 256 + (m % 128), f2 = f1 + 128;
+  if (idx >= (int64_t)t * q4) return;
+  const int j = (int)(idx / q4), m0 = 4 * (int)(idx % q4);
+  float s[4], c[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    s[e] = 0.f;
+    c[e] = 1.f;
+    if (use_rope) sincos_reduced((qstart + (double)j * qstep) * omega_c[m0 + e], &s[e], &c[e]);
+  }
+  const int f1 = (m0 / 128) * 256 + (m0 % 128), f2 = f1 + 128;
   for (int bb = 0; bb < nb; ++bb) {
     const float* q = qhat + ((int64_t)(b0 + bb) * t_max + j) * D;
-    const float x = q[f1], y = q[f2];
+    const float4 x4 = *reinterpret_cast<const float4*>(q + f1);
+    const float4 y4 = *reinterpret_cast<const float4*>(q + f2);
+    const float x[4] = {x4.x, x4.y, x4.z, x4.w}, y[4] = {y4.x, y4.y, y4.z, y4.w};
+    float a[4], b[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      a[e] = x[e] * c[e] - y[e] * s[e];
+      b[e] = x[e] * s[e] + y[e] * c[e];
+    }
+    uint32_t ah[2], al[2], bh[2], bl[2];
+    split_pack(a[0], a[1], ah[0], al[0]);
+    split_pack(a[2], a[3], ah[1], al[1]);
+    split_pack(b[0], b[1], bh[0], bl[0]);
+    split_pack(b[2], b[3], bh[1], bl[1]);
     __nv_bfloat16* o = qhl + ((int64_t)bb * t + j) * 2 * D;
-    __nv_bfloat16 hi, lo;
-    split_hilo(x * c - y * s, hi, lo);
-    o[f1] = hi;
-    o[D + f1] = lo;
-    split_hilo(x * s + y * c, hi, lo);
-    o[f2] = hi;
-    o[D + f2] = lo;
+    *reinterpret_cast<uint2*>(o + f1) = make_uint2(ah[0], ah[1]);
+    *reinterpret_cast<uint2*>(o + D + f1) = make_uint2(al[0], al[1]);
+    *reinterpret_cast<uint2*>(o + f2) = make_uint2(bh[0], bh[1]);
+    *reinterpret_cast<uint2*>(o + D + f2) = make_uint2(bl[0], bl[1]);
   }
 }
 
@@ -532,7 +576,7 @@ inline unsigned blocks_for(int64_t n, int per) { return (unsigned)((n + per - 1)
 
 cudaError_t launch_strip(const KVSource& src, int64_t N, int H, int d, const PosSegs& segs,
                          const double* omega, int rope_fix, __nv_bfloat16* X, __half* XT,
-                         int64_t Np, cudaStream_t s) {
+                         int64_t Np, float2* gd, double pmin, int G, cudaStream_t s) {
   if (d % 16 != 0 || Np % kStripTok != 0) return cudaErrorInvalidValue;
   const size_t smem = (size_t)kStripTok * (d / 2) * sizeof(float2) +
                       (size_t)kStripTok * ((2 * d + 2) + (d + 2)) * 2;
@@ -547,7 +591,14 @@ cudaError_t launch_strip(const KVSource& src, int64_t N, int H, int d, const Pos
     attr = true;
   }
   strip_kernel<<<(unsigned)(Np / kStripTok), 256, smem, s>>>(src, N, H, d, segs, omega, rope_fix,
-                                                             vec, X, XT, Np);
+                                                             vec, X, XT, Np, gd, pmin, G);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_heads_rot(float2* rot, int t, int hd, double pstart, double pstep,
+                             const double* omega, int use_rope, cudaStream_t s) {
+  const int64_t n = (int64_t)t * hd;
+  heads_rot_kernel<<<blocks_for(n, 256), 256, 0, s>>>(rot, t, hd, pstart, pstep, omega, use_rope);
   return cudaGetLastError();
 }
 
@@ -561,7 +612,8 @@ cudaError_t launch_rope_tables(float2* coarse, float* omega, int G, int D, doubl
 cudaError_t launch_q_rope(const float* qhat, int t_max, int b0, int nb, int t, int D,
                           double qstart, double qstep, const double* omega_c, int use_rope,
                           __nv_bfloat16* qhl, cudaStream_t s) {
-  const int64_t n = (int64_t)t * (D / 2);
+  if (D % 256 != 0) return cudaErrorInvalidValue;
+  const int64_t n = (int64_t)t * (D / 8);
   q_rope_kernel<<<blocks_for(n, 256), 256, 0, s>>>(qhat, t_max, b0, nb, t, D, qstart, qstep,
                                                     omega_c, use_rope, qhl);
   return cudaGetLastError();

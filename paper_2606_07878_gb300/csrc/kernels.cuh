@@ -22,11 +22,18 @@ struct KVSource {
 // RoPE-fix and input concatenation (Sec. 2.2, App. A "Input concatenation"):
 //   X[h, n]  = [unRoPE(K[n, h]) | V[n, h]]  as bf16 hi (2d) + bf16 lo of the key half (d)
 //   XT[h]    = X[h]^T as fp16 hi / lo, token-contiguous, tokens padded with zeros to Np.
-// X:  [H*N][3d] bf16.  XT: [H*2d][2*Np] fp16 (hi at [0, Np), lo at [Np, 2Np)).
-// omega: [d/2] fp64 base-model frequencies theta^(-2m/d).
+// X:  [H*N][3d] bf16.  XT: [H*2d][2*Np] fp16 (hi at [0, Np), lo at [Np, 2Np); lo rows of
+// the value half are not written). omega: [d/2] fp64 base-model frequencies theta^(-2m/d).
+// Also gd[n] = (g, p_n - (pmin + g * kPosGrain)) with g = floor((p_n - pmin) / kPosGrain)
+// clamped to [0, G): the compactor-RoPE coarse index and residual of token n (n < N).
 cudaError_t launch_strip(const KVSource& src, int64_t N, int H, int d, const PosSegs& segs,
                          const double* omega, int rope_fix, __nv_bfloat16* X, __half* XT,
-                         int64_t Np, cudaStream_t s);
+                         int64_t Np, float2* gd, double pmin, int G, cudaStream_t s);
+
+// rot[j][m] = (cos, sin)((pstart + j * pstep) * omega[m]) for j < t, m < hd (angle reduced
+// modulo 2 pi in fp64); (1, 0) when use_rope is 0. The output heads' re-rotation table.
+cudaError_t launch_heads_rot(float2* rot, int t, int hd, double pstart, double pstep,
+                             const double* omega, int use_rope, cudaStream_t s);
 
 // Compactor-RoPE tables: coarse[g][m] = (cos, sin)((pmin + g * kPosGrain) * w_m), omega[m] = w_m
 // (fp32), w_m = omega_c[m] = theta_c^(-2m/D) (fp64 table), angles reduced in fp64.

@@ -269,7 +269,7 @@ struct Plan {
   int ca_units;   // (h, i) pairs per cross-attention group
   int sa_heads;   // KV-heads per self-attention group
   // byte offsets
-  size_t oX, oXT, oCoarse, oOmega, oPX, oZ1, oA1, oCat, oZ2, oA2, oG, oZ3;
+  size_t oX, oXT, oCoarse, oOmega, oGD, oHrot, oPX, oZ1, oA1, oCat, oZ2, oA2, oG, oZ3;
   size_t oCA, oSA;
   size_t ca_unit_bytes, sa_unit_bytes;
   size_t kb_b, kss_b, q_b, S_b, P_b, O_b;        // per CA unit
@@ -304,6 +304,8 @@ bool make_plan(const still_layer_config& c, int64_t N, int t, double pmin, doubl
   P.oXT = take(H * 2 * d * 2 * P.Np * 2);
   P.oCoarse = take((size_t)P.G * (D / 2) * 8);
   P.oOmega = take((D / 2) * 4);
+  P.oGD = take((size_t)P.Np * 8);
+  P.oHrot = take(T * (d / 2) * 8);
   P.oPX = take(H * T * 2 * n * 2 * d * 2);
   P.oZ1 = take(H * T * D * 4);
   P.oA1 = take(H * T * 2 * D * 2);
@@ -445,6 +447,8 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
   __half* XT = reinterpret_cast<__half*>(ws + P.oXT);
   float2* coarse = reinterpret_cast<float2*>(ws + P.oCoarse);
   float* omega = reinterpret_cast<float*>(ws + P.oOmega);
+  float2* gd = reinterpret_cast<float2*>(ws + P.oGD);
+  float2* hrot = reinterpret_cast<float2*>(ws + P.oHrot);
   bf16* PX = reinterpret_cast<bf16*>(ws + P.oPX);
   float* Z1 = reinterpret_cast<float*>(ws + P.oZ1);
   bf16* A1 = reinterpret_cast<bf16*>(ws + P.oA1);
@@ -454,8 +458,10 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
   bf16* Gb = reinterpret_cast<bf16*>(ws + P.oG);
   void* Z3 = ws + P.oZ3;
 
-  KLAUNCH(STILL_K_STRIP, launch_strip(src, N, H, d, pos.segs, L.omega_b, c.rope_fix, X, XT, Np, s));
+  KLAUNCH(STILL_K_STRIP, launch_strip(src, N, H, d, pos.segs, L.omega_b, c.rope_fix, X, XT, Np,
+                                      gd, pos.pmin, P.G, s));
   KLAUNCH(STILL_K_TABLES, launch_rope_tables(coarse, omega, P.G, D, pos.pmin, L.omega_c, s));
+  KLAUNCH(STILL_K_TABLES, launch_heads_rot(hrot, t, d / 2, qstart, qstep, L.omega_b, c.rope_fix, s));
 
   // ---------------------------------------------------------------- cross-attention groups
   const int units_total = H * n;
@@ -499,8 +505,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.bias = L.bk + (size_t)i0 * D;
       e.coarse = coarse;
       e.omega = omega;
-      e.segs = pos.segs;
-      e.pmin = pos.pmin;
+      e.gd = gd;
       e.D = D;
       e.nheads = ni;
       e.ncoarse = P.G;
@@ -821,10 +826,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     e.sh = out.sh;
     e.t = t;
     e.d = d;
-    e.pstart = qstart;
-    e.pstep = qstep;
-    e.omega = L.omega_b;
-    e.rope = c.rope_fix;
+    e.rot = hrot;
     const int bn = 2 * d <= 128 ? 128 : 256;
     TRY(run_gemm<STILL_K_HEADS>(ctx, bn, op(Z3, rows, 2 * D), op(L.WhT, 2 * d, D), p, e, 1, s));
   }

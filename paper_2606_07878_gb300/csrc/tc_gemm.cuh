@@ -79,7 +79,8 @@ struct GemmSmem {
   static constexpr int kBBytes = BN * kBK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kEpiOffset = kStages * kStageBytes;  // a multiple of 1024
-  static constexpr int kBarOffset = kEpiOffset + Epi::kWarps * kWarpStageBytes;
+  static constexpr int kWarpStage = kWarpStageBytes * Epi::kStoreBufs;  // per epilogue warp
+  static constexpr int kBarOffset = kEpiOffset + Epi::kWarps * kWarpStage;
   static constexpr int kBytes = kBarOffset + 256 + 1024;  // + barriers + alignment slack
   static_assert(kBytes <= 232448, "shared memory budget");
 };
@@ -122,7 +123,34 @@ __device__ __forceinline__ void warp_store64(uint4* stage, const uint4 (&v)[4], 
   __syncwarp();
 }
 
-// Epi must provide:  __device__ void operator()(const GemmParams&, const TileCoord&,
+// Coalesced row load for one warp, the inverse of warp_store64: lane i receives `bytes` (64 or
+// 128) contiguous bytes starting at its own src (16-byte aligned), zeros when !valid. Each load
+// instruction reads whole rows (8 lanes x 16 B per 128-B row); the warp's staging area
+// (4 KB, rows 128 B apart, 16-B chunk q of row r at q ^ (r & 7)) does the transpose.
+template <int kChunks>  // 16-byte chunks per row: 4 (64 B) or 8 (128 B)
+__device__ __forceinline__ void warp_load_rows(uint4* stage, const void* src, bool valid,
+                                               uint4 (&out)[kChunks]) {
+  static_assert(kChunks == 4 || kChunks == 8, "64 or 128 bytes per row");
+  const int lane = threadIdx.x & 31;
+  const unsigned long long mine = reinterpret_cast<unsigned long long>(src);
+  constexpr int kRowsPerIt = 32 / kChunks;
+#pragma unroll
+  for (int it = 0; it < kChunks; ++it) {
+    const int r = it * kRowsPerIt + lane / kChunks, q = lane % kChunks;
+    const unsigned long long s = __shfl_sync(0xffffffffu, mine, r);
+    const int ok = __shfl_sync(0xffffffffu, valid ? 1 : 0, r);
+    const uint4 x = ok ? reinterpret_cast<const uint4*>(s)[q] : make_uint4(0u, 0u, 0u, 0u);
+    stage[r * 8 + (q ^ (r & 7))] = x;
+  }
+  __syncwarp();
+#pragma unroll
+  for (int q = 0; q < kChunks; ++q) out[q] = stage[lane * 8 + (q ^ (lane & 7))];
+  __syncwarp();
+}
+
+// Epi must provide:  __device__ void prefetch(const GemmParams&, const TileCoord&, int row,
+//                    int half) const  (called before the tile's accumulator is ready), and
+//                    __device__ void operator()(const GemmParams&, const TileCoord&,
 //                    int row_in_tile, uint32_t tmem_addr_of_this_warp_lane_quarter,
 //                    int half, uint4* warp_stage, const CUtensorMap* out_map) const;
 // where `half` (0 or 1) selects the 32-column chunks this warp owns: chunk c is handled by the
@@ -280,11 +308,12 @@ __global__ void __launch_bounds__(gemm_threads<Epi>(), 1)
     const int quarter = warp & 3;  // TMEM lanes this warp may access: [32q, 32q + 32)
     const int half = (warp - 2) >> 2;  // the "part" of the quarter's columns this warp owns
     const int row = quarter * 32 + lane;
-    uint4* stage = reinterpret_cast<uint4*>(smem + S::kEpiOffset + (warp - 2) * kWarpStageBytes);
+    uint4* stage = reinterpret_cast<uint4*>(smem + S::kEpiOffset + (warp - 2) * S::kWarpStage);
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = blockIdx.x; tile < p.ntiles; tile += gridDim.x) {
       const TileCoord tc = decode_tile(p, tile);
+      epi.prefetch(p, tc, row, half);  // inputs that do not depend on the accumulator
       bool ok = mbar_wait(&tfull[acc], acc_phase);
       ok = __all_sync(0xffffffffu, ok);
       if (!ok || warp_flag(abort_flag)) {
