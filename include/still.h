@@ -243,6 +243,13 @@ still_status still_workspace_size(const still_ctx* ctx, int64_t max_tokens, int3
  * STILL_ERR_OOM when even one group does not fit. */
 still_status still_set_workspace_limit(still_ctx* ctx, size_t bytes);
 
+/* Size limit, per layer, of the precomputed latent queries q^ = L2n(RMSNorm(Z) W_Q + b_Q)
+ * (H * n * t_max * D fp32, App. A "Cross-attention"; input-independent, so by default formed
+ * once at weight load). Layers loaded while their q^ would exceed `bytes` keep W_Q and b_Q
+ * instead and form q^ for the call's t latents inside each compaction call, with the same
+ * kernels and the same results. Default 2 GiB; applies to later still_load_layer_weights. */
+still_status still_set_qhat_eager_limit(still_ctx* ctx, size_t bytes);
+
 /* Synchronizes `stream`, then reports (and clears) the device error record:
  * STILL_ERR_TIMEOUT if a kernel's bounded wait expired, STILL_ERR_CUDA if the stream
  * reported an error. h_detail (optional, 4 ints): code, site, block, count. */

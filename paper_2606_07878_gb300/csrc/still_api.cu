@@ -39,6 +39,9 @@ struct LayerW {
   bf16* WkT = nullptr;   // [nD][2d]  pair-chunk order
   float* bk = nullptr;   // [nD]      pair-chunk order
   float* qhat = nullptr; // [H][n][t_max][D] fp32, L2-normalised, pair-chunk order
+  bool qhat_lazy = false; // q^ formed per call from Z, WqT, bq (qhat unused)
+  bf16* WqT = nullptr;   // [nD][D] pair-chunk order (lazy q^ only)
+  float* bq = nullptr;   // [nD]    pair-chunk order (lazy q^ only)
   bf16* WvoT = nullptr;  // [D][2 * n * 2d]: (W_V,i W_O,i)^T hi | lo
   bf16* SqkT = nullptr;  // [2nD][D]
   float* sbqk = nullptr; // [2nD]
@@ -127,6 +130,7 @@ struct still_ctx {
   void* ws = nullptr;
   size_t ws_bytes = 0;
   size_t ws_limit = size_t(48) << 30;
+  size_t qhat_eager_limit = size_t(2) << 30;
   Profiler prof;
 };
 
@@ -268,19 +272,23 @@ struct Plan {
   bool flash;     // fused cross-attention kernel (2d of 128 or 256), else scores + P X kernels
   int ca_units;   // (h, i) pairs per cross-attention group
   int sa_heads;   // KV-heads per self-attention group
+  int sa_sub;     // self heads per scores / softmax / P.v pass (n unless one bank is too big)
   // byte offsets
   size_t oX, oXT, oCoarse, oOmega, oGD, oHrot, oPX, oZ1, oA1, oCat, oZ2, oA2, oG, oZ3;
   size_t oCA, oSA;
   size_t ca_unit_bytes, sa_unit_bytes;
-  size_t kb_b, kss_b, q_b, S_b, P_b, O_b;        // per CA unit
-  size_t qk_b, sss_b, vT_b, Ssa_b, Psa_b;        // per SA head
+  size_t kb_b, kss_b, q_b, S_b, P_b, O_b, qt_b;  // per CA unit
+  bool lazy_q;
+  size_t oZn;
+  size_t qk_b, sss_b, vT_b, Ssa_b, Psa_b;        // per SA bank (KV-head)
+  size_t Ssah_b, Psah_b;                          // per self head (unpadded)
   size_t total;
 };
 
 size_t a256(size_t x) { return (x + 255) & ~size_t(255); }
 
-bool make_plan(const still_layer_config& c, int64_t N, int t, double pmin, double pmax,
-               size_t limit, Plan& P) {
+bool make_plan(const still_layer_config& c, bool lazy_q, int64_t N, int t, double pmin,
+               double pmax, size_t limit, Plan& P) {
   P.H = c.n_kv_heads;
   P.d = c.head_dim;
   P.D = c.d_latent;
@@ -314,6 +322,8 @@ bool make_plan(const still_layer_config& c, int64_t N, int t, double pmin, doubl
   P.oA2 = take(H * T * D * 2);
   P.oG = take(H * T * std::max<int64_t>(F, 1) * 2);
   P.oZ3 = take(H * T * D * 4);
+  P.lazy_q = lazy_q;
+  P.oZn = lazy_q ? take(H * T * 2 * D * 2) : 0;  // RMSNorm(Z) hi | lo for the call's t latents
   const size_t fixed = off;
   P.kb_b = a256(N * 2 * D * 2);
   P.kss_b = a256(N * 4 * (EpiRopeC::kParts * (D / 256) + 1));  // |k~|^2 partials + inverses
@@ -328,12 +338,16 @@ bool make_plan(const still_layer_config& c, int64_t N, int t, double pmin, doubl
     P.P_b = a256(T * 8 * (2 * ((N + 255) / 256) + 1));  // row-softmax partials + statistics
     P.O_b = a256(T * 2 * d * 4) * kMaxSplit;             // split-K partials of P X
   }
-  P.ca_unit_bytes = P.kb_b + P.kss_b + P.q_b + P.S_b + P.P_b + P.O_b;
+  // lazy q^: fp32 q~ of the unit and its sum-of-squares partials + inverse norms
+  P.qt_b = lazy_q ? a256(T * D * 4) + a256(T * 4 * (2 * (D / 256) + 1)) : 0;
+  P.ca_unit_bytes = P.kb_b + P.kss_b + P.q_b + P.S_b + P.P_b + P.O_b + P.qt_b;
   P.qk_b = a256(2 * n * T * 2 * D * 2);
   P.sss_b = a256(2 * n * T * 4 * (2 * (D / 256) + 1));
   P.vT_b = a256(n * D * P.tp * 2);
   P.Ssa_b = a256(n * T * P.ldt * 4);
   P.Psa_b = a256(n * T * P.tp * 2);
+  P.Ssah_b = (size_t)T * P.ldt * 4;
+  P.Psah_b = (size_t)T * P.tp * 2;
   P.sa_unit_bytes = P.qk_b + P.sss_b + P.vT_b + P.Ssa_b + P.Psa_b;
   if (fixed >= limit) return false;
   const size_t avail = limit - fixed;
@@ -345,11 +359,23 @@ bool make_plan(const still_layer_config& c, int64_t N, int t, double pmin, doubl
     u = (u / n) * n;
   P.ca_units = (int)u;
   int64_t sh = std::min<int64_t>(H, (int64_t)(avail / P.sa_unit_bytes));
-  if (sh < 1) return false;
-  P.sa_heads = (int)sh;
+  size_t sa_bytes;
+  if (sh >= 1) {
+    P.sa_heads = (int)sh;
+    P.sa_sub = (int)n;
+    sa_bytes = P.sa_unit_bytes * P.sa_heads;
+  } else {
+    // One bank at a time, its self heads in sub-groups (scores and probabilities per head).
+    const size_t bank = P.qk_b + P.sss_b + P.vT_b;
+    const size_t head = P.Ssah_b + P.Psah_b;
+    if (avail < bank + head + 1024) return false;
+    P.sa_heads = 1;
+    P.sa_sub = (int)std::min<int64_t>(n, (int64_t)((avail - bank - 1024) / head));
+    sa_bytes = bank + a256(P.sa_sub * P.Ssah_b) + a256(P.sa_sub * P.Psah_b);
+  }
   P.oCA = off;
   P.oSA = off;  // the two phases reuse the same region
-  P.total = off + std::max(P.ca_unit_bytes * P.ca_units, P.sa_unit_bytes * P.sa_heads);
+  P.total = off + std::max(P.ca_unit_bytes * P.ca_units, sa_bytes);
   return true;
 }
 
@@ -434,7 +460,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
   const still_layer_config& c = L.cfg;
   Plan P;
   const size_t limit = ws_fixed != nullptr ? ws_fixed_bytes : ctx->ws_limit;
-  if (!make_plan(c, N, t, pos.pmin, pos.pmax, limit, P)) return STILL_ERR_OOM;
+  if (!make_plan(c, L.qhat_lazy, N, t, pos.pmin, pos.pmax, limit, P)) return STILL_ERR_OOM;
   if (ws_fixed == nullptr) TRY(ensure_ws(ctx, P.total));
   uint8_t* ws = ws_fixed != nullptr ? ws_fixed : static_cast<uint8_t*>(ctx->ws);
   const int H = P.H, d = P.d, D = P.D, n = P.n, F = P.F;
@@ -462,6 +488,12 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
                                       gd, pos.pmin, P.G, s));
   KLAUNCH(STILL_K_TABLES, launch_rope_tables(coarse, omega, P.G, D, pos.pmin, L.omega_c, s));
   KLAUNCH(STILL_K_TABLES, launch_heads_rot(hrot, t, d / 2, qstart, qstep, L.omega_b, c.rope_fix, s));
+  bf16* Zn = P.lazy_q ? reinterpret_cast<bf16*>(ws + P.oZn) : nullptr;
+  if (P.lazy_q) {  // RMSNorm(Z) hi | lo for latents j < t of every KV-head bank
+    for (int h = 0; h < H; ++h)
+      KLAUNCH(STILL_K_LOAD, launch_rmsnorm(L.Z + (size_t)h * c.t_max * D, 1, t, D, D, c.rms_eps,
+                                           Zn + (size_t)h * t * 2 * D, 2 * D, 1, s));
+  }
 
   // ---------------------------------------------------------------- cross-attention groups
   const int units_total = H * n;
@@ -493,10 +525,49 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     float2* rstat = stp + (size_t)nbl * t * stat_slots;               // [nbl * t]
     g += P.P_b * nbl;
     float* O = reinterpret_cast<float*>(g);
+    g += P.O_b * nbl;
+    // lazy q^: q~ [nbl][t][D] fp32 and its sum-of-squares partials / inverse norms
+    float* qt = reinterpret_cast<float*>(g);
+    float* qss = reinterpret_cast<float*>(g + a256((size_t)t * D * 4) * nbl);
+    const float* qsrc = L.qhat;  // [.][t_max][D], batch index b0 + local
+    int q_tmax = c.t_max, q_b0 = b0;
+    if (P.lazy_q) {
+      // q~ = RMSNorm(Z) W_Q + b_Q (2-pass), as at weight load, for this group's (h, i) only
+      GemmParams p = gp(t, ni * D, nh, 1);
+      p.a_r1 = t;
+      add_pass(p, 0, 0, h0 * t, i0 * D, D);
+      add_pass(p, D, 0, h0 * t, i0 * D, D);
+      EpiAffine e;
+      e.kind = OUT_F32;
+      e.out = qt;
+      e.om.b1 = (int64_t)ni * t * D;
+      e.om.r0 = D;
+      e.om.cdiv = D;
+      e.om.c1 = (int64_t)t * D;
+      e.om.c0 = 1;
+      e.bias = L.bq + (size_t)i0 * D;
+      e.sumsq = qss;
+      e.ssm.b1 = (int64_t)ni * t;
+      e.ssm.r0 = 1;
+      e.ssm.c0 = t;
+      e.ss_seg = D;
+      e.ss_parts = 2 * (D / 256);
+      e.vec_ok = 1;
+      TRY(run_gemm256<STILL_K_LOAD>(ctx, op(Zn, (int64_t)H * t, 2 * D), op(L.WqT, (int64_t)n * D, D),
+                                    p, e, 1, s));
+      const int64_t nq = (int64_t)nbl * t;
+      float* qinv = qss + nq * (2 * (D / 256));
+      KLAUNCH(STILL_K_NORMS, launch_inv_norms(qss, nq, 2 * (D / 256), c.l2_eps, 1.f, qinv, s));
+      KLAUNCH(STILL_K_NORMS, launch_scale_rows(qt, qinv, nq, D, s));
+      qsrc = qt;
+      q_tmax = t;
+      q_b0 = 0;
+    }
     // keyproj: rows = tokens of heads [h0, h0+nh), columns = cross heads [i0, i0+ni)
     {
       GemmParams p = gp((int)N, ni * D, nh, 1);
       p.a_r1 = N;
+      p.n_fast = 1;  // X rows of a KV-head can exceed L2; the W_K block fits
       add_pass(p, 0, 0, (int)(h0 * N), i0 * D, 2 * d);
       add_pass(p, 2 * d, 0, (int)(h0 * N), i0 * D, d);
       EpiRopeC e;
@@ -516,8 +587,8 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     }
     // scale / |k~_n| per key (the d_l logit scale folded in)
     KLAUNCH(STILL_K_NORMS, launch_inv_norms(kss, (int64_t)nbl * N, kparts, c.l2_eps, scale, kinv, s));
-    KLAUNCH(STILL_K_QROPE, launch_q_rope(L.qhat, c.t_max, b0, nbl, t, D, qstart, qstep, L.omega_c,
-                     c.compactor_rope, qhl, s));
+    KLAUNCH(STILL_K_QROPE, launch_q_rope(qsrc, q_tmax, q_b0, nbl, t, D, qstart, qstep, L.omega_c,
+                                         c.compactor_rope, qhl, s));
     if (P.flash) {
       // S, the online softmax and P X in one kernel; per-split partials merged in order.
       float2* fst = stp;  // [nsplit][nbl * t] (the statistics region of this path)
@@ -660,7 +731,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     bf16* vT = reinterpret_cast<bf16*>(g);
     g += P.vT_b * nh;
     float* Ssa = reinterpret_cast<float*>(g);
-    g += P.Ssa_b * nh;
+    g += a256((size_t)nh * P.sa_sub * P.Ssah_b);
     bf16* Psa = reinterpret_cast<bf16*>(g);
     // The P.v product reads v^T columns [t, tp) of each head against zero probabilities:
     // they must hold finite values, and the region is shared with the cross-attention phase.
@@ -705,60 +776,66 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.vec_ok = (t % 32 == 0);
       TRY(run_gemm256<STILL_K_SA_V>(ctx, op(L.SvT, (int64_t)n * D, D), op(A1, rows, 2 * D), p, e, 1, s));
     }
-    {  // S = scale * q~.k~ / (|q~| |k~|)  per (head, self head)
-      GemmParams p = gp(t, t, nh * n, n);
-      p.a_r1 = (int64_t)2 * n * t;
-      p.a_r0 = t;
-      p.b_r1 = (int64_t)2 * n * t;
-      p.b_r0 = t;
-      add_pass(p, 0, 0, 0, n * t, D);
-      add_pass(p, 0, D, 0, n * t, D);
-      add_pass(p, D, 0, 0, n * t, D);
-      EpiAffine e;
-      e.kind = OUT_F32;
-      e.out = Ssa;
-      e.om.b1 = (int64_t)t * P.ldt;
-      e.om.r0 = P.ldt;
-      e.om.c0 = 1;
-      e.alpha = scale;
-      e.row_scale = sinv;
-      e.rsm.bdiv = n;
-      e.rsm.b1 = (int64_t)2 * n * t;
-      e.rsm.b0 = t;
-      e.rsm.r0 = 1;
-      e.col_scale = sinv;
-      e.csm.bdiv = n;
-      e.csm.b1 = (int64_t)2 * n * t;
-      e.csm.b0 = t;
-      e.csm.c0 = 1;
-      e.csm.k = (int64_t)n * t;
-      e.vec_ok = 1;
-      e.tma_f32 = 1;
-      const StoreView3D sv = store_view(Ssa, 4, t, t, (int64_t)nh * n, P.ldt, (int64_t)t * P.ldt,
-                                        32, true);
-      TRY(run_gemm256<STILL_K_SA_SCORES>(ctx, op(qk, (int64_t)nh * 2 * n * t, 2 * D),
-                   op(qk, (int64_t)nh * 2 * n * t, 2 * D), p, e, 1, s, &sv));
-    }
-    KLAUNCH(STILL_K_SA_SOFTMAX, launch_softmax(Ssa, (int64_t)nh * n * t, t, P.ldt, Psa, P.tp, 0, s));
-    {  // heads = P v -> concat rows (h0 + hh) * t + j, columns i * D + f
-      GemmParams p = gp(t, D, nh * n, n);
-      p.a_r1 = (int64_t)n * t;
-      p.a_r0 = t;
-      p.b_r0 = D;
-      p.b_k1 = P.tp;
-      add_pass(p, 0, 0, 0, 0, (int)P.tp);
-      EpiAffine e;
-      e.kind = OUT_BF16;
-      e.out = cat;
-      e.om.bdiv = n;
-      e.om.b1 = (int64_t)t * n * D;
-      e.om.b0 = D;
-      e.om.r0 = (int64_t)n * D;
-      e.om.c0 = 1;
-      e.om.k = (int64_t)h0 * t * n * D;
-      e.vec_ok = 1;
-      TRY(run_gemm256<STILL_K_SA_PV>(ctx, op(Psa, (int64_t)nh * n * t, P.tp),
-                   op(vT, (int64_t)n * D, (int64_t)nh * P.tp), p, e, 1, s));
+    // Self heads [i0, i0 + ns) of the nh banks per pass (all n unless one bank is too big).
+    for (int i0 = 0; i0 < n; i0 += P.sa_sub) {
+      const int ns = std::min(P.sa_sub, n - i0);
+      {  // S = scale * q~.k~ / (|q~| |k~|)  per (bank hh, self head i0 + bi), batch hh * ns + bi
+        GemmParams p = gp(t, t, nh * ns, ns);
+        p.a_r1 = (int64_t)2 * n * t;
+        p.a_r0 = t;
+        p.b_r1 = (int64_t)2 * n * t;
+        p.b_r0 = t;
+        add_pass(p, 0, 0, i0 * t, (n + i0) * t, D);
+        add_pass(p, 0, D, i0 * t, (n + i0) * t, D);
+        add_pass(p, D, 0, i0 * t, (n + i0) * t, D);
+        EpiAffine e;
+        e.kind = OUT_F32;
+        e.out = Ssa;
+        e.om.b1 = (int64_t)t * P.ldt;
+        e.om.r0 = P.ldt;
+        e.om.c0 = 1;
+        e.alpha = scale;
+        e.row_scale = sinv;
+        e.rsm.bdiv = ns;
+        e.rsm.b1 = (int64_t)2 * n * t;
+        e.rsm.b0 = t;
+        e.rsm.r0 = 1;
+        e.rsm.k = (int64_t)i0 * t;
+        e.col_scale = sinv;
+        e.csm.bdiv = ns;
+        e.csm.b1 = (int64_t)2 * n * t;
+        e.csm.b0 = t;
+        e.csm.c0 = 1;
+        e.csm.k = (int64_t)(n + i0) * t;
+        e.vec_ok = 1;
+        e.tma_f32 = 1;
+        const StoreView3D sv = store_view(Ssa, 4, t, t, (int64_t)nh * ns, P.ldt,
+                                          (int64_t)t * P.ldt, 32, true);
+        TRY(run_gemm256<STILL_K_SA_SCORES>(ctx, op(qk, (int64_t)nh * 2 * n * t, 2 * D),
+                                           op(qk, (int64_t)nh * 2 * n * t, 2 * D), p, e, 1, s, &sv));
+      }
+      KLAUNCH(STILL_K_SA_SOFTMAX,
+              launch_softmax(Ssa, (int64_t)nh * ns * t, t, P.ldt, Psa, P.tp, 0, s));
+      {  // heads = P v -> concat rows (h0 + hh) * t + j, columns (i0 + bi) * D + f
+        GemmParams p = gp(t, D, nh * ns, ns);
+        p.a_r1 = (int64_t)ns * t;
+        p.a_r0 = t;
+        p.b_r0 = D;
+        p.b_k1 = P.tp;
+        add_pass(p, 0, 0, 0, i0 * D, (int)P.tp);
+        EpiAffine e;
+        e.kind = OUT_BF16;
+        e.out = cat;
+        e.om.bdiv = ns;
+        e.om.b1 = (int64_t)t * n * D;
+        e.om.b0 = D;
+        e.om.r0 = (int64_t)n * D;
+        e.om.c0 = 1;
+        e.om.k = (int64_t)h0 * t * n * D + (int64_t)i0 * D;
+        e.vec_ok = 1;
+        TRY(run_gemm256<STILL_K_SA_PV>(ctx, op(Psa, (int64_t)nh * ns * t, P.tp),
+                                       op(vT, (int64_t)n * D, (int64_t)nh * P.tp), p, e, 1, s));
+      }
     }
   }
   const bool z3_bf16 = (c.final_norm == 0);
@@ -940,6 +1017,12 @@ still_status still_destroy(still_ctx* ctx) {
   return STILL_OK;
 }
 
+still_status still_set_qhat_eager_limit(still_ctx* ctx, size_t bytes) {
+  if (ctx == nullptr) return STILL_ERR_INVALID_ARG;
+  ctx->qhat_eager_limit = bytes;
+  return STILL_OK;
+}
+
 still_status still_set_workspace_limit(still_ctx* ctx, size_t bytes) {
   if (ctx == nullptr || bytes == 0) return STILL_ERR_INVALID_ARG;
   ctx->ws_limit = bytes;
@@ -974,7 +1057,8 @@ still_status still_load_layer_weights(still_ctx* ctx, int32_t layer,
   TRY(dalloc(L, &L.Z, (size_t)H * T * D));
   TRY(dalloc(L, &L.WkT, (size_t)nD * 2 * d));
   TRY(dalloc(L, &L.bk, (size_t)nD));
-  TRY(dalloc(L, &L.qhat, (size_t)H * n * T * D));
+  L.qhat_lazy = (size_t)H * n * T * D * sizeof(float) > ctx->qhat_eager_limit;
+  if (!L.qhat_lazy) TRY(dalloc(L, &L.qhat, (size_t)H * n * T * D));
   TRY(dalloc(L, &L.WvoT, (size_t)D * 2 * n * 2 * d));
   TRY(dalloc(L, &L.SqkT, (size_t)2 * nD * D));
   TRY(dalloc(L, &L.sbqk, (size_t)2 * nD));
@@ -1014,11 +1098,14 @@ still_status still_load_layer_weights(still_ctx* ctx, int32_t layer,
     free_layer(tmp);
   };
   still_status st = STILL_OK;
-  if ((st = dalloc(tmp, &WqT, (size_t)nD * D)) != STILL_OK ||
-      (st = dalloc(tmp, &Zn, (size_t)H * T * 2 * D)) != STILL_OK ||
+  // W_Q and b_Q are kept with the layer when q^ is formed per call, else temporaries.
+  LayerW& qown = L.qhat_lazy ? L : tmp;
+  if ((st = dalloc(qown, &WqT, (size_t)nD * D)) != STILL_OK ||
+      (st = dalloc(qown, &bq, (size_t)nD)) != STILL_OK ||
       (st = dalloc(tmp, &WoT, (size_t)D * nD)) != STILL_OK ||
-      (st = dalloc(tmp, &bq, (size_t)nD)) != STILL_OK ||
-      (st = dalloc(tmp, &qss, (size_t)H * n * T * (2 * (D / 256) + 1))) != STILL_OK) {
+      (!L.qhat_lazy && (st = dalloc(tmp, &Zn, (size_t)H * T * 2 * D)) != STILL_OK) ||
+      (!L.qhat_lazy &&
+       (st = dalloc(tmp, &qss, (size_t)H * n * T * (2 * (D / 256) + 1))) != STILL_OK)) {
     cleanup();
     free_layer(L);
     return st;
@@ -1026,8 +1113,12 @@ still_status still_load_layer_weights(still_ctx* ctx, int32_t layer,
   auto body = [&]() -> still_status {
     CK(launch_transpose(Wq, D, nD, WqT, D, s));
     CK(launch_bias(static_cast<const bf16*>(w->bq), nullptr, nD, bq, D, s));
-    CK(launch_rmsnorm(w->Z, 1, (int64_t)H * T, D, D, c.rms_eps, Zn, 2 * D, 1, s));
-    {  // q~ = RMSNorm(Z) W_Q + b_Q  (2-pass), |q~|^2 per (row, head)
+    if (L.qhat_lazy) {
+      L.WqT = WqT;
+      L.bq = bq;
+    }
+    if (!L.qhat_lazy) CK(launch_rmsnorm(w->Z, 1, (int64_t)H * T, D, D, c.rms_eps, Zn, 2 * D, 1, s));
+    if (!L.qhat_lazy) {  // q~ = RMSNorm(Z) W_Q + b_Q  (2-pass), |q~|^2 per (row, head)
       GemmParams p = gp(H * T, (int)nD);
       add_pass(p, 0, 0, 0, 0, D);
       add_pass(p, D, 0, 0, 0, D);
@@ -1051,7 +1142,7 @@ still_status still_load_layer_weights(still_ctx* ctx, int32_t layer,
       e.vec_ok = 1;
       TRY(run_gemm256<STILL_K_LOAD>(ctx, op(Zn, (int64_t)H * T, 2 * D), op(WqT, nD, D), p, e, 1, s));
     }
-    {
+    if (!L.qhat_lazy) {
       const int64_t nq = (int64_t)H * n * T;
       float* qinv = qss + nq * (2 * (D / 256));
       CK(launch_inv_norms(qss, nq, 2 * (D / 256), c.l2_eps, 1.f, qinv, s));
@@ -1136,7 +1227,7 @@ still_status still_compact_layer_noalloc(still_ctx* ctx, int32_t layer, const vo
   TRY(make_positions(h_segments, n_segments, N, pos));
   CK(cudaSetDevice(ctx->device));
   Plan P;
-  if (!make_plan(L->cfg, N, t, pos.pmin, pos.pmax, kNoAllocScratchBytes, P))
+  if (!make_plan(L->cfg, L->qhat_lazy, N, t, pos.pmin, pos.pmax, kNoAllocScratchBytes, P))
     return STILL_ERR_OOM;  // even the smallest grouping needs more than the fixed scratch
   uint8_t* scratch = nullptr;
   TRY(noalloc_scratch(ctx->device, &scratch));
@@ -1316,8 +1407,8 @@ still_status still_workspace_size(const still_ctx* ctx, int64_t max_tokens, int3
     return ctx == nullptr || bytes == nullptr ? STILL_ERR_INVALID_ARG : STILL_ERR_NOT_LOADED;
   if (max_tokens < 1 || max_t < 1 || max_t > max_tokens) return STILL_ERR_SHAPE;
   Plan P;
-  if (!make_plan(ctx->layers[0].cfg, max_tokens, max_t, 0.0, (double)(max_tokens - 1),
-                 ctx->ws_limit, P))
+  if (!make_plan(ctx->layers[0].cfg, ctx->layers[0].qhat_lazy, max_tokens, max_t, 0.0,
+                 (double)(max_tokens - 1), ctx->ws_limit, P))
     return STILL_ERR_OOM;
   *bytes = P.total;
   return STILL_OK;

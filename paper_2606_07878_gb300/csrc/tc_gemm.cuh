@@ -41,6 +41,10 @@ struct GemmParams {
   int32_t npass;
   GemmPass pass[3];
   int32_t ksplit;  // split-K factor (each split = a contiguous range of K iterations)
+  // Tile order: m-tiles fastest (default; concurrent CTAs share B tiles through L2) or, with
+  // n_fast, n-tiles fastest (concurrent CTAs share A tiles: for an A operand larger than L2
+  // and a B operand that fits, A is then read from HBM once).
+  int32_t n_fast;
   // Derived by the host launcher.
   int32_t tiles_m, tiles_n, iters_total, ntiles;
   uint32_t idesc;
@@ -53,6 +57,15 @@ struct TileCoord {
 
 __device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int tile) {
   TileCoord c;
+  if (p.n_fast) {
+    c.tn = tile % p.tiles_n;
+    int r = tile / p.tiles_n;
+    c.split = r % p.ksplit;
+    r /= p.ksplit;
+    c.tm = r % p.tiles_m;
+    c.b = r / p.tiles_m;
+    return c;
+  }
   c.tm = tile % p.tiles_m;
   int r = tile / p.tiles_m;
   c.split = r % p.ksplit;

@@ -23,6 +23,7 @@ EXPORTS = [
     "still_create", "still_destroy", "still_status_string", "still_load_layer_weights",
     "still_compact_layer", "still_compact_stack", "still_compact_layer_ragged",
     "still_compact_stack_ragged", "still_workspace_size", "still_set_workspace_limit",
+    "still_set_qhat_eager_limit",
     "still_get_device_status", "still_budget", "still_kv_bytes", "still_param_count",
     "still_profile_enable", "still_profile_read", "still_kernel_class_name",
     "still_compact_layer_noalloc", "still_recompact_layer_ragged", "still_recompact_stack_ragged",
@@ -107,6 +108,7 @@ def lib():
                                               PI64, PI64, P], ctypes.c_int),
             "still_workspace_size": ([P, I64, I32, ctypes.POINTER(ctypes.c_size_t)], ctypes.c_int),
             "still_set_workspace_limit": ([P, ctypes.c_size_t], ctypes.c_int),
+            "still_set_qhat_eager_limit": ([P, ctypes.c_size_t], ctypes.c_int),
             "still_get_device_status": ([P, P, PI32], ctypes.c_int),
             "still_budget": ([I64, I64], I64),
             "still_kv_bytes": ([I64, I64, I64, I64, I64], I64),
@@ -184,6 +186,10 @@ def still_destroy(ctx):
 
 def still_set_workspace_limit(ctx, nbytes: int):
     _check(lib().still_set_workspace_limit(ctx, nbytes), "still_set_workspace_limit")
+
+
+def still_set_qhat_eager_limit(ctx, nbytes: int):
+    _check(lib().still_set_qhat_eager_limit(ctx, nbytes), "still_set_qhat_eager_limit")
 
 
 def still_load_layer_weights(ctx, layer: int, cfg: LayerConfig, weights: dict, stream=None):

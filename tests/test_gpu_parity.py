@@ -265,8 +265,10 @@ def test_qwen8b_32k_layer_sampled_head(t):
         r.close()
 
 
-def test_gemma_128k_full_size_token_reversal_invariance():
-    """Full-size Gemma-shaped layer (N = 131072, H = 8, d = 256, d_l = 2048, t = 655): the
+@pytest.mark.parametrize("t", [655, 16384])
+def test_gemma_128k_full_size_token_reversal_invariance(t):
+    """Full-size Gemma-shaped layer (N = 131072, H = 8, d = 256, d_l = 2048, t = 655 and 16384,
+    ratios 200x and 8x; at t = 16384 the latent queries are formed per call): the
     compactor is a function of the set of (token, position) pairs, so feeding the cache in
     reverse order with reversed positions (one segment of step -1) gives the same compact
     cache up to rounding. Both runs are GPU results: if each is within the parity bar of the
@@ -275,7 +277,6 @@ def test_gemma_128k_full_size_token_reversal_invariance():
     (fp16 probabilities, bf16 outputs) make the two runs differ by more than plain reordering
     would suggest, so the twice-the-bar bound is the one checked here."""
     wl = synth.WORKLOADS["gemma_128k"]
-    t = 655
     N = wl["N"]
     r = Runner(wl, t)
     try:
@@ -288,5 +289,66 @@ def test_gemma_128k_full_size_token_reversal_invariance():
         for name, a, b in (("C_k", Ck, Ck2), ("C_v", Cv, Cv2)):
             err, cos = metrics(synth.bf16_to_f64(a), synth.bf16_to_f64(b))
             assert err <= 2 * ERR_REL and cos >= 0.996, f"{name} reversed: {err:.4e} {cos:.6f}"
+    finally:
+        r.close()
+
+
+@pytest.mark.parametrize("wl_name,t_max,t", [("tiny_1k", 128, 128), ("qwen7b_8k", 1024, 256)])
+def test_lazy_qhat_matches_eager(wl_name, t_max, t):
+    """Latent queries formed per call (the path large t_max takes) give the same bits as the
+    load-time precompute, also for t < t_max, and meet the oracle bar."""
+    wl = synth.WORKLOADS[wl_name]
+    K, V = synth.gen_kv(wl, 0, device=DEV)
+    eager = Runner(wl, t_max)
+    ctx = still.still_create(0)
+    try:
+        still.still_set_qhat_eager_limit(ctx, 0)
+        still.still_load_layer_weights(ctx, 0, still.config_from_workload(wl, t_max), eager.W[0])
+        Ck_e, Cv_e, _ = eager.layer(0, K, V, t)
+        Ck_l = torch.empty_like(Ck_e)
+        Cv_l = torch.empty_like(Cv_e)
+        still.still_compact_layer(ctx, 0, K, V, t, Ck_l, Cv_l)
+        code, det = still.still_get_device_status(ctx)
+        assert code == 0, det
+        assert torch.equal(Ck_l, Ck_e) and torch.equal(Cv_l, Cv_e)
+        heads = [0] if wl["H"] > 2 else None
+        rk, rv, _, _ = oracle_layer(wl, eager.W[0], K, V, t, heads=heads)
+        hs = heads if heads is not None else range(wl["H"])
+        for h in hs:
+            assert_parity(rk[:, h], synth.bf16_to_f64(Ck_l[:, h]), f"lazy C_k head {h}")
+            assert_parity(rv[:, h], synth.bf16_to_f64(Cv_l[:, h]), f"lazy C_v head {h}")
+    finally:
+        still.still_destroy(ctx)
+        eager.close()
+
+
+def test_workspace_limits_regroup_and_keep_parity():
+    """Smaller workspace limits make the library process fewer (KV-head, head) units per
+    cross-attention group and, once one self-attention bank no longer fits, the bank's self
+    heads a few at a time. The shape (t = N = 512, 8 heads, D = 256) makes a bank's q/k
+    projection alone larger than a cross-attention unit, so the smallest limits that still work
+    run the self-attention in head sub-groups. Every grouping must meet the oracle bar."""
+    wl = _small(N=512, H=1, d=64, D=256, n=8, F=512, ts=(512,))
+    t = 512
+    r = Runner(wl, t)
+    try:
+        K, V = synth.gen_kv(wl, 0, device=DEV)
+        rk, rv, _, _ = oracle_layer(wl, r.W[0], K, V, t)
+        total = still.still_workspace_size(r.ctx, wl["N"], t)
+        ok_limits = []
+        for frac in (1.0, 0.8, 0.6, 0.5, 0.4, 0.35, 0.3, 0.25, 0.2, 0.15):
+            limit = int(total * frac)
+            still.still_set_workspace_limit(r.ctx, limit)
+            Ck, Cv = r.out(t)
+            try:
+                still.still_compact_layer(r.ctx, 0, K, V, t, Ck, Cv)
+            except still.StillError as e:
+                assert e.name == "STILL_ERR_OOM", e.name
+                continue
+            r.check_status()
+            assert_parity(rk[:, 0], synth.bf16_to_f64(Ck[:, 0]), f"C_k limit {frac}")
+            assert_parity(rv[:, 0], synth.bf16_to_f64(Cv[:, 0]), f"C_v limit {frac}")
+            ok_limits.append(frac)
+        assert len(ok_limits) >= 4 and min(ok_limits) <= 0.5, ok_limits
     finally:
         r.close()
