@@ -107,6 +107,9 @@ struct EpiAffine {
   AffineMap ssm;           // (b, r, c / ss_seg) -> vector index
   int32_t ss_seg = 1 << 30;
   int32_t ss_parts = 2;    // slots per vector = 2 * ss_seg / tile width
+  // Vectors in blocks of ss_block consecutive indices, stored part-major (see launch_inv_norms),
+  // so that a warp's 32 rows write 32 consecutive floats of one part.
+  int64_t ss_block = 1;
   int64_t split_stride = 0;
   int32_t vec_ok = 0;  // host: om.c0 == 1, cdiv % 32 == 0, 16-B aligned rows
   // OUT_F32 through TMA stores: the output is the 3-D view (col, row, batch) given to the
@@ -247,7 +250,8 @@ struct EpiAffine {
     if (sumsq != nullptr && rvalid) {
       const int c_tile = tc.tn * tile_cols_;
       const int slot = ((c_tile % ss_seg) / tile_cols_) * 2 + half;
-      sumsq[ssm.at(tc.b, r, c_tile / ss_seg) * ss_parts + slot] = ss;
+      const int64_t vec = ssm.at(tc.b, r, c_tile / ss_seg);
+      sumsq[(vec / ss_block) * ss_parts * ss_block + slot * ss_block + vec % ss_block] = ss;
     }
   }
 
@@ -350,7 +354,7 @@ struct EpiRopeC {
   static constexpr int kStages = 3;
   static constexpr int kStoreBufs = 1;  // 4 KB TMA-store staging buffers per warp
   __nv_bfloat16* out = nullptr;  // [H][n][N][2D]: hi at [0, D), lo at [D, 2D) (via the TMA view)
-  float* sumsq = nullptr;        // [H][n][N][kParts * D / 256] partial sums of |k~|^2
+  float* sumsq = nullptr;        // [H][n][kParts * D / 256][N] partial sums of |k~|^2 (part-major)
   const float* bias = nullptr;   // [n*D], pair-chunk order
   const float2* coarse = nullptr;  // [G][D/2]: (cos, sin)(G_g * omega_m)
   const float* omega = nullptr;    // [D/2] fp32
@@ -455,7 +459,7 @@ struct EpiRopeC {
     }
     if (rvalid) {
       const int parts = kParts * (D / 256);
-      sumsq[((int64_t)(tc.b * nheads + head) * Ntok + r) * parts + (f_tile / 256) * kParts + half] =
+      sumsq[((int64_t)(tc.b * nheads + head) * parts + (f_tile / 256) * kParts + half) * Ntok + r] =
           ss;
     }
   }

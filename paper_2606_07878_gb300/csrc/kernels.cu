@@ -534,12 +534,12 @@ __global__ void scale_rows_kernel(float* x, const float* inv, int64_t rows, int 
 }
 
 __global__ void inv_norms_kernel(const float* __restrict__ parts, int64_t nvec, int nparts,
-                                 float eps, float alpha, float* __restrict__ out) {
+                                 int64_t block, float eps, float alpha, float* __restrict__ out) {
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= nvec) return;
-  const float* p = parts + i * nparts;
+  const float* p = parts + (i / block) * nparts * block + i % block;
   float s = 0.f;
-  for (int k = 0; k < nparts; ++k) s += p[k];  // fixed order
+  for (int k = 0; k < nparts; ++k) s += p[k * block];  // fixed order
   out[i] = alpha / fmaxf(sqrtf(s), eps);
 }
 
@@ -701,9 +701,11 @@ cudaError_t launch_scale_rows(float* x, const float* inv, int64_t rows, int D, c
   return cudaGetLastError();
 }
 
-cudaError_t launch_inv_norms(const float* parts, int64_t nvec, int nparts, float eps,
+cudaError_t launch_inv_norms(const float* parts, int64_t nvec, int nparts, int64_t block, float eps,
                              float alpha, float* out, cudaStream_t s) {
-  inv_norms_kernel<<<blocks_for(nvec, 256), 256, 0, s>>>(parts, nvec, nparts, eps, alpha, out);
+  if (block < 1) return cudaErrorInvalidValue;
+  inv_norms_kernel<<<blocks_for(nvec, 256), 256, 0, s>>>(parts, nvec, nparts, block, eps, alpha,
+                                                         out);
   return cudaGetLastError();
 }
 

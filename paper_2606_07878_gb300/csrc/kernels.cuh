@@ -75,9 +75,11 @@ cudaError_t launch_px_to_hilo(const float* O, int nsplit, int64_t split_stride, 
 cudaError_t launch_ca_merge(const float* O, const float2* stats, int nsplit, int b0, int nb,
                             int n, int t, int d2, __nv_bfloat16* PX, cudaStream_t s);
 
-// out[i] = alpha / max(sqrt(sum_k parts[i * nparts + k]), eps), summed in slot order: the
-// L2 / QK-norm factor of vector i from the epilogues' sum-of-squares partials.
-cudaError_t launch_inv_norms(const float* parts, int64_t nvec, int nparts, float eps,
+// out[i] = alpha / max(sqrt(sum_k part(i, k)), eps), summed in slot order: the L2 / QK-norm
+// factor of vector i from the epilogues' sum-of-squares partials. Vectors come in blocks of
+// `block` consecutive indices stored part-major: part(i, k) is at
+// (i / block) * nparts * block + k * block + i % block (block = 1: [vector][part]).
+cudaError_t launch_inv_norms(const float* parts, int64_t nvec, int nparts, int64_t block, float eps,
                              float alpha, float* out, cudaStream_t s);
 
 // Non-parametric RMSNorm over rows of width D: out = x / sqrt(mean(x^2) + eps) as bf16 hi

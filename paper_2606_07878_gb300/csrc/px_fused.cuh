@@ -3,19 +3,51 @@
 //   O[s][b](m, :) = sum over tokens k of split s:  P(m, k) X(k, :),
 //   P(m, k) = exp(S[b](m, k) - M[b](m)) / L[b](m)                    (row softmax, App. A)
 //
-// The scores S (fp32, written by the scores GEMM) are read once: four "transform" warps turn
+// The scores S (fp32, written by the scores GEMM) are read once: eight "transform" warps turn
 // each 128 x 64 slice into fp16 probabilities directly in the 128-byte-swizzled shared-memory
 // layout tcgen05.mma reads, so the probabilities never exist in global memory. X^T arrives by
 // TMA as fp16 hi and lo (the lo part only for the key half of X: the value half is exact in
 // fp16). Row statistics (M, L) come from the scores epilogue's per-tile partials.
 //
-// CTA = 2 + 4 + Epi::kWarps warps: TMA producer, MMA issuer, transform warps, epilogue.
+// Each transform warp keeps the next 64-token block's scores in flight while it converts the
+// current one.
+//
+// CTA = 2 + 8 + 8 warps: TMA producer, MMA issuer, transform warps, epilogue.
 #pragma once
 #include "gemm_host.cuh"
 
 namespace still {
 
-constexpr int kPxTransformWarps = 4;
+constexpr int kPxTransformWarps = 8;
+constexpr int kPxRowSteps = kBM / (4 * kPxTransformWarps);  // 4-row steps per transform warp
+
+// Epilogue of the P X kernel: the tile's fp32 accumulator rows go to the split's partial
+// output, out + split * split_stride + om(b, r, c), with coalesced warp stores.
+struct EpiPxOut {
+  static constexpr int kWarps = 8;
+  float* out = nullptr;
+  int64_t split_stride = 0;
+  AffineMap om;
+  int32_t tile_cols_ = 256;
+
+  __device__ void operator()(const GemmParams& p, const TileCoord& tc, int row, uint32_t taddr,
+                             int half, uint4* stage, const CUtensorMap*) const {
+    const int r = tc.tm * kBM + row;
+    const bool rvalid = r < p.M;
+    for (int cc = 32 * half; cc < tile_cols_; cc += 64) {
+      const int c0 = tc.tn * tile_cols_ + cc;
+      if (c0 >= p.N) break;  // uniform across the warp
+      float v[32];
+      tmem_ld32(taddr + (uint32_t)cc, v);
+      float* dst = out + (rvalid ? om.at(tc.b, r, c0) + (int64_t)tc.split * split_stride : 0);
+      uint4 a4[4], b4[4];
+      pack_f32x16(v, a4);
+      pack_f32x16(v + 16, b4);
+      warp_store64(stage, a4, dst, rvalid);
+      warp_store64(stage, b4, dst + 16, rvalid);
+    }
+  }
+};
 
 struct PxParams {
   const float* S = nullptr;      // [nb][t][ldS] scores (natural-log units)
@@ -36,7 +68,7 @@ struct PxSmem {
   static constexpr int kBBytes = BN * kBK * 2;        // X^T hi tile
   static constexpr int kLoBytes = LOB * kBK * 2;      // X^T lo tile
   static constexpr int kStageBytes = kABytes + kBBytes + kLoBytes;
-  static constexpr int kEpiBytes = EpiAffine::kWarps * kWarpStageBytes;
+  static constexpr int kEpiBytes = EpiPxOut::kWarps * kWarpStageBytes;
   static constexpr int kStages = (232448 - kEpiBytes - 2048) / kStageBytes >= 3 ? 3 : 2;
   static constexpr int kEpiOffset = kStages * kStageBytes;
   static constexpr int kBarOffset = kEpiOffset + kEpiBytes;
@@ -46,17 +78,17 @@ struct PxSmem {
 
 // The GemmParams carry M = t, N = BN-tiled output width (2d), batch = nb, ksplit; a single
 // "pass" of klen = Np describes the token range (iters_total = Np / 64).
-constexpr int kPxThreads = 64 + 32 * kPxTransformWarps + 32 * EpiAffine::kWarps;
+constexpr int kPxThreads = 64 + 32 * kPxTransformWarps + 32 * EpiPxOut::kWarps;
 
 template <int BN, int LOB>
 __global__ void __launch_bounds__(kPxThreads, 1)
     px_fused_kernel(const __grid_constant__ CUtensorMap tmXhi,
                     const __grid_constant__ CUtensorMap tmXlo,
                     const __grid_constant__ CUtensorMap tmC, const GemmParams p,
-                    const PxParams px, const EpiAffine epi) {
+                    const PxParams px, const EpiPxOut epi) {
   using S = PxSmem<BN, LOB>;
   constexpr int kStages = S::kStages;
-  constexpr int kEpiWarps = EpiAffine::kWarps;
+  constexpr int kEpiWarps = EpiPxOut::kWarps;
   constexpr int kTW = kPxTransformWarps;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -195,7 +227,7 @@ __global__ void __launch_bounds__(kPxThreads, 1)
     }
   } else if (warp < first_epi) {
     // -------------------------------------------------------------- transform warps
-    // Warp w writes rows [32w, 32w + 32) of each P tile; a step covers 4 rows x 64 tokens,
+    // Warp w writes rows [16w, 16w + 16) of each P tile; a step covers 4 rows x 64 tokens,
     // 8 lanes per row, 8 tokens (one 16-byte fp16 chunk) per lane.
     const int w = warp - 2;
     const int sub = lane >> 3, chunk = lane & 7;
@@ -204,37 +236,41 @@ __global__ void __launch_bounds__(kPxThreads, 1)
     uint32_t phase = 0;
     for (int tile = blockIdx.x; tile < p.ntiles && !warp_flag(abort_flag); tile += gridDim.x) {
       const TileCoord tc = decode_tile(p, tile);
-      float2 st[8];
-      const float* srow[8];
+      float2 st[kPxRowSteps];
+      const float* srow[kPxRowSteps];
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        const int m = tc.tm * kBM + 32 * w + 4 * q + sub;
+      for (int q = 0; q < kPxRowSteps; ++q) {
+        const int m = tc.tm * kBM + 4 * kPxRowSteps * w + 4 * q + sub;
         const bool ok = m < px.t;
         st[q] = ok ? px.stats[(int64_t)tc.b * px.t + m] : make_float2(0.f, 0.f);
         srow[q] = ok ? px.S + ((int64_t)tc.b * px.t + m) * px.ldS : nullptr;
       }
       int it0, it1;
       split_range(p, tc.split, it0, it1);
-      for (int it = it0; it < it1; ++it) {
-        // All sixteen loads of this k-block are issued before any use (one memory latency per
-        // k-block rather than one per row).
+      // The sixteen loads of a k-block are issued together, one k-block ahead of their use:
+      // while block it is converted, block it + 1 is in flight (software pipelining).
+      auto load_block = [&](int it, float4 (&xo)[kPxRowSteps][2]) {
         const int k0 = it * kBK + chunk * 8;
-        float4 x[8][2];
         const bool full_k = k0 + 8 <= px.N;
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
+        for (int q = 0; q < kPxRowSteps; ++q) {
           if (srow[q] != nullptr && full_k) {
-            x[q][0] = __ldg(reinterpret_cast<const float4*>(srow[q] + k0));
-            x[q][1] = __ldg(reinterpret_cast<const float4*>(srow[q] + k0) + 1);
+            xo[q][0] = __ldg(reinterpret_cast<const float4*>(srow[q] + k0));
+            xo[q][1] = __ldg(reinterpret_cast<const float4*>(srow[q] + k0) + 1);
           } else {
             float t8[8];
 #pragma unroll
             for (int e = 0; e < 8; ++e)
               t8[e] = (srow[q] != nullptr && k0 + e < px.N) ? srow[q][k0 + e] : -INFINITY;
-            x[q][0] = make_float4(t8[0], t8[1], t8[2], t8[3]);
-            x[q][1] = make_float4(t8[4], t8[5], t8[6], t8[7]);
+            xo[q][0] = make_float4(t8[0], t8[1], t8[2], t8[3]);
+            xo[q][1] = make_float4(t8[4], t8[5], t8[6], t8[7]);
           }
         }
+      };
+      float4 x[kPxRowSteps][2], xn[kPxRowSteps][2];
+      if (it0 < it1) load_block(it0, x);
+      for (int it = it0; it < it1; ++it) {
+        if (it + 1 < it1) load_block(it + 1, xn);
         bool ok = mbar_wait(&empty[stage], phase ^ 1);
         ok = __all_sync(0xffffffffu, ok);
         if (!ok) {
@@ -246,8 +282,8 @@ __global__ void __launch_bounds__(kPxThreads, 1)
         }
         uint4* a = reinterpret_cast<uint4*>(smem + stage * S::kStageBytes);
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          const int r = 32 * w + 4 * q + sub;  // row inside the tile
+        for (int q = 0; q < kPxRowSteps; ++q) {
+          const int r = 4 * kPxRowSteps * w + 4 * q + sub;  // row inside the tile
           const float v0[8] = {x[q][0].x, x[q][0].y, x[q][0].z, x[q][0].w,
                                x[q][1].x, x[q][1].y, x[q][1].z, x[q][1].w};
           float v[8];
@@ -265,6 +301,11 @@ __global__ void __launch_bounds__(kPxThreads, 1)
         if (++stage == kStages) {
           stage = 0;
           phase ^= 1;
+        }
+#pragma unroll
+        for (int q = 0; q < kPxRowSteps; ++q) {
+          x[q][0] = xn[q][0];
+          x[q][1] = xn[q][1];
         }
       }
     }
@@ -317,7 +358,7 @@ namespace still {
 // Launches px_fused_kernel: A = probabilities from S (transform warps), B = X^T hi / lo.
 template <int BN, int LOB>
 inline cudaError_t launch_px_fused(const Operand2D& XT, GemmParams p, const PxParams& px,
-                                   EpiAffine epi, int num_sms, cudaStream_t stream) {
+                                   EpiPxOut epi, int num_sms, cudaStream_t stream) {
   using S = PxSmem<BN, LOB>;
   if (!finalize_gemm<BN>(p, 0)) return cudaErrorInvalidValue;
   CUtensorMap thi, tlo, tc;

@@ -552,12 +552,13 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.ssm.c0 = t;
       e.ss_seg = D;
       e.ss_parts = 2 * (D / 256);
+      e.ss_block = t;
       e.vec_ok = 1;
       TRY(run_gemm256<STILL_K_LOAD>(ctx, op(Zn, (int64_t)H * t, 2 * D), op(L.WqT, (int64_t)n * D, D),
                                     p, e, 1, s));
       const int64_t nq = (int64_t)nbl * t;
       float* qinv = qss + nq * (2 * (D / 256));
-      KLAUNCH(STILL_K_NORMS, launch_inv_norms(qss, nq, 2 * (D / 256), c.l2_eps, 1.f, qinv, s));
+      KLAUNCH(STILL_K_NORMS, launch_inv_norms(qss, nq, 2 * (D / 256), t, c.l2_eps, 1.f, qinv, s));
       KLAUNCH(STILL_K_NORMS, launch_scale_rows(qt, qinv, nq, D, s));
       qsrc = qt;
       q_tmax = t;
@@ -586,7 +587,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
                    1, s, &kv));
     }
     // scale / |k~_n| per key (the d_l logit scale folded in)
-    KLAUNCH(STILL_K_NORMS, launch_inv_norms(kss, (int64_t)nbl * N, kparts, c.l2_eps, scale, kinv, s));
+    KLAUNCH(STILL_K_NORMS, launch_inv_norms(kss, (int64_t)nbl * N, kparts, N, c.l2_eps, scale, kinv, s));
     KLAUNCH(STILL_K_QROPE, launch_q_rope(qsrc, q_tmax, q_b0, nbl, t, D, qstart, qstep, L.omega_c,
                                          c.compactor_rope, qhl, s));
     if (P.flash) {
@@ -653,7 +654,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     {  // O = softmax(S) X: probabilities formed on the fly (fp16), X hi + key-half lo passes
       GemmParams p = gp(t, 2 * d, nbl, ni);
       add_pass(p, 0, 0, 0, 0, (int)Np);
-      const int bn = 2 * d <= 128 ? 128 : 256;
+      const int bn = 256;
       const int64_t tiles = (int64_t)((t + 127) / 128) * ((2 * d + bn - 1) / bn) * nbl;
       p.ksplit = std::min(auto_split(tiles, (int)(Np / 64), ctx->nsm), kMaxSplit);
       p.ksplit = std::min(p.ksplit, (int)(Np / 64));
@@ -671,8 +672,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       px.Np = Np;
       px.nb = nbl;
       px.bdiv = ni;
-      EpiAffine e;
-      e.kind = OUT_F32;
+      EpiPxOut e;
       e.out = O;
       e.split_stride = px_stride;
       e.om.bdiv = ni;
@@ -680,12 +680,11 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.om.b0 = (int64_t)t * 2 * d;
       e.om.r0 = 2 * d;
       e.om.c0 = 1;
-      e.vec_ok = 1;
       const Operand2D xt = op(XT, (int64_t)H * 2 * d, 2 * Np);
+      // This path serves 2d = 512 (smaller heads take the fused kernel).
+      if (d != 256) return STILL_ERR_UNSUPPORTED;
       ctx->prof.begin(STILL_K_PX, s);
-      cudaError_t r = d == 64    ? launch_px_fused<128, 64>(xt, p, px, e, ctx->nsm, s)
-                      : d == 128 ? launch_px_fused<256, 128>(xt, p, px, e, ctx->nsm, s)
-                                 : launch_px_fused<256, 256>(xt, p, px, e, ctx->nsm, s);
+      cudaError_t r = launch_px_fused<256, 256>(xt, p, px, e, ctx->nsm, s);
       ctx->prof.end(STILL_K_PX, s);
       if (r == cudaErrorInvalidValue) return STILL_ERR_INVALID_ARG;
       if (r != cudaSuccess) return STILL_ERR_CUDA;
@@ -758,11 +757,12 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.ssm.c0 = t;
       e.ss_seg = D;
       e.ss_parts = sparts;
+      e.ss_block = t;
       e.vec_ok = 1;
       TRY(run_gemm256<STILL_K_SA_PROJ>(ctx, op(A1, rows, 2 * D), op(L.SqkT, (int64_t)2 * n * D, D), p, e, 1, s));
     }
     KLAUNCH(STILL_K_NORMS,
-            launch_inv_norms(sss, (int64_t)nh * 2 * n * t, sparts, c.l2_eps, 1.f, sinv, s));
+            launch_inv_norms(sss, (int64_t)nh * 2 * n * t, sparts, t, c.l2_eps, 1.f, sinv, s));
     {  // v^T = S_V^T RMSNorm(Z')^T  -> [nD][nh * tp]
       GemmParams p = gp(n * D, nh * t);
       add_pass(p, 0, 0, 0, h0 * t, D);
@@ -1139,13 +1139,14 @@ still_status still_load_layer_weights(still_ctx* ctx, int32_t layer,
       e.ssm.c0 = T;
       e.ss_seg = D;
       e.ss_parts = 2 * (D / 256);
+      e.ss_block = T;
       e.vec_ok = 1;
       TRY(run_gemm256<STILL_K_LOAD>(ctx, op(Zn, (int64_t)H * T, 2 * D), op(WqT, nD, D), p, e, 1, s));
     }
     if (!L.qhat_lazy) {
       const int64_t nq = (int64_t)H * n * T;
       float* qinv = qss + nq * (2 * (D / 256));
-      CK(launch_inv_norms(qss, nq, 2 * (D / 256), c.l2_eps, 1.f, qinv, s));
+      CK(launch_inv_norms(qss, nq, 2 * (D / 256), T, c.l2_eps, 1.f, qinv, s));
       CK(launch_scale_rows(L.qhat, qinv, nq, D, s));
     }
     // W_VO,i = W_V,i W_O,i  -> stored transposed as hi | lo: WvoT[c][i*2d + f]
