@@ -286,6 +286,10 @@ typedef enum {
  * launch of the library's kernels is bracketed by a CUDA event pair on its stream. Launch
  * counts are kept whether or not timing is enabled (reset by this call). */
 still_status still_profile_enable(still_ctx* ctx, int32_t enable);
+/* As still_profile_enable, with event timing only for the kernel classes whose bit
+ * (1 << class) is set in `mask` (0 stops timing). Timing one class costs two events per launch
+ * of that class only, so a step can be timed with its dominant kernel measured inside it. */
+still_status still_profile_enable_classes(still_ctx* ctx, uint64_t mask);
 /* Launches and total event time (ms) of one kernel class since the last enable call.
  * Synchronizes the device when timings are pending. */
 still_status still_profile_read(still_ctx* ctx, int32_t cls, int64_t* h_launches, double* h_ms);

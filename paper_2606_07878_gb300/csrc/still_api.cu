@@ -60,6 +60,7 @@ struct LayerW {
 // Per-kernel-class launch counts and (when enabled) CUDA-event timings.
 struct Profiler {
   bool on = false;
+  uint64_t mask = ~uint64_t(0);  // classes with event timing while on
   int64_t launches[STILL_K_COUNT] = {0};
   double ms[STILL_K_COUNT] = {0};
   struct Rec {
@@ -82,7 +83,7 @@ struct Profiler {
   }
   void begin(int cls, cudaStream_t s) {
     ++launches[cls];
-    if (!on) return;
+    if (!on || !((mask >> cls) & 1)) return;
     pending = get();
     cudaEventRecord(pending, s);
   }
@@ -1436,6 +1437,16 @@ still_status still_profile_enable(still_ctx* ctx, int32_t enable) {
   CK(cudaSetDevice(ctx->device));
   ctx->prof.reset();
   ctx->prof.on = enable != 0;
+  ctx->prof.mask = ~uint64_t(0);
+  return STILL_OK;
+}
+
+still_status still_profile_enable_classes(still_ctx* ctx, uint64_t mask) {
+  if (ctx == nullptr) return STILL_ERR_INVALID_ARG;
+  CK(cudaSetDevice(ctx->device));
+  ctx->prof.reset();
+  ctx->prof.on = mask != 0;
+  ctx->prof.mask = mask;
   return STILL_OK;
 }
 

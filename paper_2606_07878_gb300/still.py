@@ -23,7 +23,7 @@ EXPORTS = [
     "still_create", "still_destroy", "still_status_string", "still_load_layer_weights",
     "still_compact_layer", "still_compact_stack", "still_compact_layer_ragged",
     "still_compact_stack_ragged", "still_workspace_size", "still_set_workspace_limit",
-    "still_set_qhat_eager_limit",
+    "still_set_qhat_eager_limit", "still_profile_enable_classes",
     "still_get_device_status", "still_budget", "still_kv_bytes", "still_param_count",
     "still_profile_enable", "still_profile_read", "still_kernel_class_name",
     "still_compact_layer_noalloc", "still_recompact_layer_ragged", "still_recompact_stack_ragged",
@@ -115,6 +115,7 @@ def lib():
             "still_param_count": ([ctypes.POINTER(LayerConfig), I32], I64),
             "still_selftest_wait_timeout": ([P, I64, P], ctypes.c_int),
             "still_profile_enable": ([P, I32], ctypes.c_int),
+            "still_profile_enable_classes": ([P, ctypes.c_uint64], ctypes.c_int),
             "still_profile_read": ([P, I32, PI64, PD], ctypes.c_int),
             "still_kernel_class_name": ([I32], ctypes.c_char_p),
         }
@@ -341,6 +342,14 @@ def still_param_count(cfg: LayerConfig, t: int) -> int:
 
 def still_profile_enable(ctx, enable: bool = True):
     _check(lib().still_profile_enable(ctx, 1 if enable else 0), "still_profile_enable")
+
+
+def still_profile_enable_classes(ctx, names):
+    """Event timing only for the named kernel classes (an empty list stops timing)."""
+    mask = 0
+    for n in names:
+        mask |= 1 << KERNEL_CLASSES.index(n)
+    _check(lib().still_profile_enable_classes(ctx, mask), "still_profile_enable_classes")
 
 
 def still_profile_read(ctx):
