@@ -238,6 +238,15 @@ still_status still_recompact_stack_ragged(still_ctx* ctx, int32_t n_layers, int3
 still_status still_workspace_size(const still_ctx* ctx, int64_t max_tokens, int32_t max_t,
                                   size_t* bytes);
 
+/* Allocates now the workspace a call with up to max_tokens tokens and compact length max_t
+ * needs (layer 0's configuration), so that later calls of at most those sizes allocate
+ * nothing. still_compact_layer and still_compact_stack enqueue work only on their stream and
+ * neither allocate nor synchronize when the workspace suffices (and after one earlier call has
+ * set the kernels' shared-memory attributes): such calls can be captured into a CUDA graph
+ * and replayed. Kernel timing (still_profile_*) should cover only the classes needed while
+ * capturing: timed launches become event nodes of the graph. */
+still_status still_reserve_workspace(still_ctx* ctx, int64_t max_tokens, int32_t max_t);
+
 /* Upper bound on the workspace the context may allocate (default 48 GiB). Calls whose
  * workspace would exceed it process the KV-heads in smaller groups, or fail with
  * STILL_ERR_OOM when even one group does not fit. */

@@ -70,6 +70,7 @@ struct Profiler {
   std::vector<Rec> recs;
   std::vector<cudaEvent_t> pool;
   cudaEvent_t pending = nullptr;
+  int64_t untimed = 0;  // event pairs that could not be timed since the last reset
 
   cudaEvent_t get() {
     if (!pool.empty()) {
@@ -81,16 +82,25 @@ struct Profiler {
     cudaEventCreate(&e);
     return e;
   }
+  // Inside a stream capture an event must be recorded as an external node to be recorded again
+  // on every replay of the graph (a plain record there only orders the captured work).
+  static void record(cudaEvent_t e, cudaStream_t s) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(s, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusActive)
+      cudaEventRecordWithFlags(e, s, cudaEventRecordExternal);
+    else
+      cudaEventRecord(e, s);
+  }
   void begin(int cls, cudaStream_t s) {
     ++launches[cls];
     if (!on || !((mask >> cls) & 1)) return;
     pending = get();
-    cudaEventRecord(pending, s);
+    record(pending, s);
   }
   void end(int cls, cudaStream_t s) {
     if (!on || pending == nullptr) return;
     cudaEvent_t b = get();
-    cudaEventRecord(b, s);
+    record(b, s);
     recs.push_back(Rec{cls, pending, b});
     pending = nullptr;
   }
@@ -99,7 +109,11 @@ struct Profiler {
     if (cudaDeviceSynchronize() != cudaSuccess) return false;
     for (auto& r : recs) {
       float t = 0.f;
-      cudaEventElapsedTime(&t, r.a, r.b);
+      if (cudaEventElapsedTime(&t, r.a, r.b) != cudaSuccess) {
+        cudaGetLastError();  // not a device fault: do not leave it to the next launch check
+        untimed += 1;
+        t = 0.f;
+      }
       ms[r.cls] += t;
       pool.push_back(r.a);
       pool.push_back(r.b);
@@ -109,6 +123,7 @@ struct Profiler {
   }
   void reset() {
     resolve();
+    untimed = 0;
     for (int i = 0; i < STILL_K_COUNT; ++i) {
       launches[i] = 0;
       ms[i] = 0;
@@ -1414,6 +1429,13 @@ still_status still_workspace_size(const still_ctx* ctx, int64_t max_tokens, int3
     return STILL_ERR_OOM;
   *bytes = P.total;
   return STILL_OK;
+}
+
+still_status still_reserve_workspace(still_ctx* ctx, int64_t max_tokens, int32_t max_t) {
+  size_t bytes = 0;
+  TRY(still_workspace_size(ctx, max_tokens, max_t, &bytes));
+  CK(cudaSetDevice(ctx->device));
+  return ensure_ws(ctx, bytes);
 }
 
 still_status still_get_device_status(still_ctx* ctx, void* stream, int32_t* h_detail) {

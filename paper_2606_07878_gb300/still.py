@@ -23,7 +23,7 @@ EXPORTS = [
     "still_create", "still_destroy", "still_status_string", "still_load_layer_weights",
     "still_compact_layer", "still_compact_stack", "still_compact_layer_ragged",
     "still_compact_stack_ragged", "still_workspace_size", "still_set_workspace_limit",
-    "still_set_qhat_eager_limit", "still_profile_enable_classes",
+    "still_set_qhat_eager_limit", "still_profile_enable_classes", "still_reserve_workspace",
     "still_get_device_status", "still_budget", "still_kv_bytes", "still_param_count",
     "still_profile_enable", "still_profile_read", "still_kernel_class_name",
     "still_compact_layer_noalloc", "still_recompact_layer_ragged", "still_recompact_stack_ragged",
@@ -116,6 +116,7 @@ def lib():
             "still_selftest_wait_timeout": ([P, I64, P], ctypes.c_int),
             "still_profile_enable": ([P, I32], ctypes.c_int),
             "still_profile_enable_classes": ([P, ctypes.c_uint64], ctypes.c_int),
+            "still_reserve_workspace": ([P, I64, I32], ctypes.c_int),
             "still_profile_read": ([P, I32, PI64, PD], ctypes.c_int),
             "still_kernel_class_name": ([I32], ctypes.c_char_p),
         }
@@ -312,6 +313,10 @@ def still_recompact_stack_ragged(ctx, Kprevs, Vprevs, cu_prev, prev_len, Knews, 
         arr(Knews), arr(Vnews), (I64 * (B + 1))(*cu_new), ratio, arr(Cks), arr(Cvs), cu_out,
         len_out, _stream(stream)), "still_recompact_stack_ragged")
     return list(cu_out), list(len_out)
+
+
+def still_reserve_workspace(ctx, max_tokens: int, max_t: int):
+    _check(lib().still_reserve_workspace(ctx, max_tokens, max_t), "still_reserve_workspace")
 
 
 def still_workspace_size(ctx, max_tokens: int, max_t: int) -> int:

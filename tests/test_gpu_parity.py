@@ -352,3 +352,46 @@ def test_workspace_limits_regroup_and_keep_parity():
         assert len(ok_limits) >= 4 and min(ok_limits) <= 0.5, ok_limits
     finally:
         r.close()
+
+
+def test_stack_graph_capture_replays_identically():
+    """The stack call captured into a CUDA graph (workspace reserved first) replays to the same
+    bits as the eager call, also after the inputs are overwritten in place between replays."""
+    wl = dict(synth.WORKLOADS["tiny_1k"], L=2)
+    t = wl["ts"][0]
+    r = Runner(wl, t, layers=(0, 1))
+    try:
+        Ks, Vs = zip(*(synth.gen_kv(wl, l, device=DEV) for l in range(2)))
+        Ks, Vs = list(Ks), list(Vs)
+        out = [r.out(t) for _ in range(2)]
+        Ck, Cv = [o[0] for o in out], [o[1] for o in out]
+        still.still_compact_stack(r.ctx, Ks, Vs, t, Ck, Cv)
+        torch.cuda.synchronize()
+        ref = [(c.clone(), v.clone()) for c, v in zip(Ck, Cv)]
+        still.still_reserve_workspace(r.ctx, wl["N"], t)
+        s = torch.cuda.Stream()
+        g = torch.cuda.CUDAGraph()
+        for c in Ck + Cv:
+            c.zero_()
+        torch.cuda.synchronize()
+        with torch.cuda.graph(g, stream=s):
+            still.still_compact_stack(r.ctx, Ks, Vs, t, Ck, Cv, stream=s)
+        g.replay()
+        torch.cuda.synchronize()
+        r.check_status()
+        for (c0, v0), c, v in zip(ref, Ck, Cv):
+            assert torch.equal(c, c0) and torch.equal(v, v0)
+        # new inputs written into the captured buffers: the replay computes on them
+        K2, V2 = synth.gen_kv(wl, 0, device=DEV, seed=5)
+        Ks[0].copy_(K2)
+        Vs[0].copy_(V2)
+        g.replay()
+        torch.cuda.synchronize()
+        Ck_e, Cv_e = r.out(t)
+        still.still_compact_layer(r.ctx, 0, Ks[0], Vs[0], t, Ck_e, Cv_e)
+        torch.cuda.synchronize()
+        assert torch.equal(Ck[0], Ck_e) and torch.equal(Cv[0], Cv_e)
+        assert not torch.equal(Ck[0], ref[0][0])
+        del g
+    finally:
+        r.close()
