@@ -20,6 +20,7 @@ so that each step can be checked against the text by eye:
     ..................................................... App. A "Output projections"; App. B
   * compact budget t = round(N / c) ........ App. J exact-results table (K column)
   * position offset T - t ................................ App. B, logical vs physical length
+  * iterative chunked schedule with lookahead: passes, chunks, retained cache . Sec. 2.3
 
 Readings taken where the paper is silent (each listed with its basis in the design notes):
 half-split RoPE pairs (m, m + w/2) with omega_m = base^(-2m/w); RMSNorm x/sqrt(mean x^2 + 1e-6)
@@ -87,6 +88,48 @@ def budget(N: int, c: int) -> int:
 def position_offset(logical_len: int, t: int) -> int:
     """Continuation positions are offset by logical length minus physical length (App. B)."""
     return logical_len - t
+
+
+# ----------------------------------------------------------------------------- lookahead schedule
+
+def lookahead_pass(k: int, c: int, t: int) -> dict:
+    """Pass k of the iterative chunked schedule with lookahead (Sec. 2.3; App. B, iterative
+    chunked compaction), chunks of ct tokens, walked through as the text describes them.
+
+    Pass 0 prefills the first two chunks with no past and compacts chunk 0. Pass k > 0
+    prefills chunk k + 1 while the past holds the k chunks already compacted (t slots each)
+    followed by raw chunk k, then compacts chunk k, the one just before the new chunk.
+    After pass k the cache holds chunks 0..k compacted and chunk k + 1 raw (the lookahead).
+    """
+    ct = c * t
+    compacted_before = k                                  # chunks 0..k-1
+    if k == 0:
+        prefill = (0, 2 * ct)
+        past = 0
+    else:
+        prefill = ((k + 1) * ct, ct)                      # chunk k + 1
+        past = compacted_before * t + ct                  # compact prefix, then raw chunk k
+    compacted_after = k + 1
+    raw_after = ct                                        # chunk k + 1
+    logical_after = (k + 2) * ct                          # tokens prefilled so far
+    retained_after = compacted_after * t + raw_after
+    return {
+        "chunk_start": k * ct, "chunk_len": ct,
+        "prefill_start": prefill[0], "prefill_len": prefill[1], "prefill_past": past,
+        "compact_row": compacted_before * t,
+        "retained_after": retained_after, "logical_after": logical_after,
+        "pos_offset_after": logical_after - retained_after,
+    }
+
+
+def lookahead_totals(T: int, c: int, t: int) -> tuple[int, int]:
+    """(passes, retained cache entries) once T tokens have been compacted: every chunk of ct
+    tokens costs one pass, and the last pass leaves one raw lookahead chunk (Sec. 2.3)."""
+    ct = c * t
+    if T <= 0 or T % ct:
+        raise ValueError("T must be a positive multiple of the chunk length c*t")
+    passes = T // ct
+    return passes, lookahead_pass(passes - 1, c, t)["retained_after"]
 
 
 def rope_angles(pos: np.ndarray, width: int, base: float) -> np.ndarray:

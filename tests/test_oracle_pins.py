@@ -257,3 +257,46 @@ def test_kv_bytes_match_paper():
         assert round(O.kv_bytes(m["L"], m["H"], m["d"], m["b"], S) / 2**20) == mib
     for S, gib in g["retained_gib_vllm"]:
         assert O.kv_bytes(m["L"], m["H"], m["d"], m["b"], S) / 2**30 == pytest.approx(gib, abs=5e-4)
+
+
+# ------------------------------------------------------------------ lookahead schedule
+
+def test_lookahead_schedule_matches_paper_counts():
+    g = _golden("iterative_slots.json")
+    t = g["t"]
+    for c, tokens in g["chunk_tokens"]:
+        assert O.lookahead_pass(0, c, t)["chunk_len"] == tokens
+    for case in g["cases"]:
+        passes, retained = O.lookahead_totals(case["T"], case["c"], t)
+        if "passes" in case:
+            assert passes == case["passes"], case
+        if "retained" in case:
+            assert retained == case["retained"], case
+
+
+@pytest.mark.parametrize("c,t", [(8, 128), (3, 5), (1, 1), (32, 7)])
+def test_lookahead_schedule_invariants(c, t):
+    ct = c * t
+    n = 20
+    passes = [O.lookahead_pass(k, c, t) for k in range(n)]
+    # chunks are compacted in order, each once; every token is prefilled exactly once, in order
+    assert [p["chunk_start"] for p in passes] == [k * ct for k in range(n)]
+    prefilled = []
+    for p in passes:
+        prefilled.extend(range(p["prefill_start"], p["prefill_start"] + p["prefill_len"]))
+    assert prefilled == list(range((n + 1) * ct))
+    for k, p in enumerate(passes):
+        # by the end of the pass the chunk and one more (the lookahead) have been prefilled
+        assert p["prefill_start"] + p["prefill_len"] == p["chunk_start"] + 2 * ct
+        if k:
+            assert p["prefill_start"] == p["chunk_start"] + ct  # the chunk just before the new one
+            assert p["prefill_past"] == (k + c) * t            # (N + c) t in Sec. 2.3
+        compacted = (k + 1) * ct
+        assert p["retained_after"] == compacted // c + ct      # T / c + ct
+        assert p["compact_row"] == k * t
+        assert p["logical_after"] - p["pos_offset_after"] == p["retained_after"]
+    with pytest.raises(ValueError):
+        O.lookahead_totals(0, c, t)
+    if ct > 1:
+        with pytest.raises(ValueError):
+            O.lookahead_totals(ct + 1, c, t)
