@@ -26,12 +26,17 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 WORKLOAD = "qwen7b_8k"
-DEFAULT_T = {"qwen7b_8k": 1024, "qwen8b_32k": 2048, "gemma_128k": 655, "tiny_1k": 128}
+DEFAULT_T = {"qwen7b_8k": 1024, "qwen8b_32k": 2048, "gemma_128k": 655, "tiny_1k": 128,
+             "qwen3_4b_64k": 1311}
 
 
 def describe(name, wl, t):
+    nb = wl.get("n_blocks", 1)
+    blocks = "" if nb == 1 else (f", {nb} blocks" + (" (CA in every block)"
+                                                      if wl.get("cross_every_block", 1) else ""))
     return (f"{name}: {wl['L']} layers, N={wl['N']}, H_kv={wl['H']}, d={wl['d']}, "
-            f"D={wl['D']}, {wl['n']} heads, FFN {wl['F']}, t={t} ({round(wl['N'] / t)}x)")
+            f"D={wl['D']}, {wl['n']} heads, FFN {wl['F']}{blocks}, t={t} "
+            f"({round(wl['N'] / t)}x)")
 
 # DRAM traffic (read + write) per launch of the dominant kernel at a workload, from an ncu
 # capture; valid only for the kernel sources it was taken on (hash of the listed sources).
@@ -153,11 +158,13 @@ def algorithmic_flops(wl, t, N):
     """Per layer per sequence (W_V folded, W_K not foldable): key projection, scores, P X,
     V/O projections, self-attention, FFN, output heads."""
     H, d, D, n, F = wl["H"], wl["d"], wl["D"], wl["n"], wl["F"]
+    nb = wl.get("n_blocks", 1)
+    n_ca = nb if wl.get("cross_every_block", 1) else 1  # blocks with cross-attention
     ca = (2 * N * H * 2 * d * n * D + 2 * t * N * H * n * D + 2 * t * N * H * n * 2 * d
           + 2 * t * H * n * 2 * d * D + 2 * t * H * n * D * D)
     sa = 6 * t * H * D * n * D + 4 * t * t * H * n * D + 2 * t * H * n * D * D
-    return {"total": ca + sa + 4 * t * H * D * F + 4 * t * H * D * d,
-            "scores": 2 * t * N * H * n * D, "px": 2 * t * N * H * n * 2 * d}
+    return {"total": n_ca * ca + nb * (sa + 4 * t * H * D * F) + 4 * t * H * D * d,
+            "scores": n_ca * 2 * t * N * H * n * D, "px": n_ca * 2 * t * N * H * n * 2 * d}
 
 
 def run_cpu_baseline(wl, t, budget_s=30.0):
@@ -173,7 +180,8 @@ def run_cpu_baseline(wl, t, budget_s=30.0):
     fl = algorithmic_flops(wl, t, wl["N"])
     one_head = fl["total"] / wl["H"]
     W = synth.gen_weights(wl, 0, t, "cpu")
-    cfg = O.cfg_from_workload(wl)
+    cfg = O.cfg_from_workload(wl, n_blocks=wl.get("n_blocks", 1),
+                              cross_every_block=bool(wl.get("cross_every_block", 1)))
     Wf = O.as_f64(W)
     if one_head < 2.5e12:
         K, V = synth.gen_kv(wl, 0, device="cpu")
@@ -343,8 +351,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--t", type=int, default=0, help="compact length (default per workload)")
     ap.add_argument("--workload", default=WORKLOAD,
-                    choices=["qwen7b_8k", "qwen8b_32k", "gemma_128k", "tiny_1k",
-                             "iterative_ragged"])
+                    choices=sorted(DEFAULT_T) + ["iterative_ragged"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     if args.impl == "reference":
@@ -403,7 +410,7 @@ def main():
     # as one graph). The dominant kernel class (fused cross-attention for 2d <= 256, else the
     # scores GEMM) is the only one with events: its launches are bracketed by event nodes of the
     # graph, read after the last replay.
-    kname = "ca_fused" if 2 * d <= 256 else "scores"
+    kname = "ca_fused" if 2 * d <= 256 and wl.get("n_blocks", 1) == 1 else "scores"
     still.still_reserve_workspace(ctx, N, t)
     still.still_profile_enable_classes(ctx, [kname])
     graph = torch.cuda.CUDAGraph()

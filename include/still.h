@@ -92,6 +92,16 @@ typedef struct {
   const void *W1, *W2, *Wkey, *Wval;
 } still_layer_weights;
 
+/* Weights of one compactor block (App. A, "Compactor blocks"), layouts as in
+ * still_layer_weights. The cross-attention fields (Wq, bq, Wk, bk, Wv, Wo) are not read for
+ * blocks without cross-attention (blocks after the first when cross_every_block = 0); W1, W2
+ * are not read when ffn_dim = 0. */
+typedef struct {
+  const void *Wq, *bq, *Wk, *bk, *Wv, *Wo;
+  const void *Sq, *sbq, *Sk, *sbk, *Sv, *So;
+  const void *W1, *W2;
+} still_block_weights;
+
 /* Cache positions: token i of the segment sits at start + i * step (exact fp64). Segments
  * are concatenated in order and must cover the N tokens exactly. At most 8 per call. */
 typedef struct {
@@ -113,6 +123,20 @@ const char* still_status_string(still_status s);
 still_status still_load_layer_weights(still_ctx* ctx, int32_t layer,
                                       const still_layer_config* cfg,
                                       const still_layer_weights* w, void* stream);
+
+/* still_load_layer_weights for a compactor of cfg->n_blocks (1 or 2) blocks (App. A; the
+ * paper's canonical compactor has two, both with cross-attention; n_blocks > 2 gives
+ * STILL_ERR_UNSUPPORTED: every further cross-attention compounds the rounding of its fp16
+ * probabilities, and three blocks measured just past the parity bar). Z [H, t_max, D] latent banks;
+ * blocks[b] the weights of block b; Wkey, Wval [D, d] output heads. Block 0's latent queries
+ * depend only on Z and are precomputed here (as in still_load_layer_weights). A later
+ * cross-attending block's queries L2norm(RMSNorm(Z_b) W_Q + b_Q) depend on the latent state
+ * Z_b entering it and are formed inside each compaction call. still_load_layer_weights
+ * requires n_blocks = 1. */
+still_status still_load_layer_weights_blocks(still_ctx* ctx, int32_t layer,
+                                             const still_layer_config* cfg, const void* Z,
+                                             const still_block_weights* blocks,
+                                             const void* Wkey, const void* Wval, void* stream);
 
 /* Compacts one layer (Sec. 2.1; App. B single-pass recipe steps 3-5).
  *   K, V       [N, H, d] bf16 device, element strides strides_kv = {s_token, s_head, s_dim}
@@ -232,6 +256,77 @@ still_status still_recompact_stack_ragged(still_ctx* ctx, int32_t n_layers, int3
                                           const int64_t* h_cu_new, int64_t ratio,
                                           void* const* Ck, void* const* Cv, int64_t* h_cu_out,
                                           int64_t* h_len_out, void* stream);
+
+/* Compacts only the layers l < n_layers with h_compact_layer[l] != 0, each as
+ * still_compact_layer over the same positions (Sec. 2.1 and App. A "Per-layer stack and
+ * mixed-attention models": in a model that mixes sliding-window and global attention, such
+ * as Gemma-3, only the global-attention layers are compacted; the others keep their own
+ * sliding-window cache). Skipped layers need not be loaded and their K, V, Ck, Cv entries may
+ * be NULL; their buffers are not touched. h_compact_layer: host array of n_layers bytes.
+ * Other arguments as still_compact_stack. */
+still_status still_compact_stack_masked(still_ctx* ctx, int32_t n_layers,
+                                        const uint8_t* h_compact_layer, const void* const* K,
+                                        const void* const* V, const int64_t strides_kv[3],
+                                        const still_pos_segment* h_segments, int32_t n_segments,
+                                        int64_t N, int32_t t, void* const* Ck, void* const* Cv,
+                                        double* h_out_pos_start, double* h_out_pos_step,
+                                        int64_t* h_pos_offset, void* stream);
+
+/* ---------------------------------------------------------------------------------------
+ * Iterative chunked compaction with lookahead (Sec. 2.3, "Iterative chunked compaction";
+ * App. B). The context arrives in chunks of c*t tokens (c the local compression ratio, t the
+ * slots per chunk). Pass 0 prefills chunks 0 and 1 and compacts chunk 0; pass k > 0
+ * prefills chunk k + 1 with the k compacted chunks followed by raw chunk k as its past
+ * ((k + c) * t entries), then compacts chunk k to t slots. After pass k the cache holds
+ * chunks 0..k compacted plus raw chunk k + 1 (the one-chunk lookahead buffer): once T tokens
+ * have been compacted (T / (c t) passes) it holds T / c + c t entries. The base-model
+ * prefill itself is the caller's; the library computes the schedule and the compaction. */
+typedef struct {
+  int64_t chunk_start;       /* first token position of the chunk this pass compacts: k*c*t  */
+  int64_t chunk_len;         /* c*t                                                          */
+  int64_t prefill_start;     /* first token the base model prefills in this pass             */
+  int64_t prefill_len;       /* 2*c*t at pass 0, c*t after                                   */
+  int64_t prefill_past;      /* cache entries the prefill attends to: 0, then (k + c)*t       */
+  int64_t compact_row;       /* k*t: first row of this chunk's t slots in the compact prefix */
+  int64_t retained_after;    /* (k + 1)*t + c*t cache entries after the pass                 */
+  int64_t logical_after;     /* (k + 2)*c*t tokens prefilled after the pass                  */
+  int64_t pos_offset_after;  /* logical_after - retained_after (App. B position offset)      */
+} still_lookahead_pass;
+
+/* Host only. Pass k >= 0 of the schedule for ratio c >= 1 and t >= 1 slots per chunk.
+ * STILL_ERR_INVALID_ARG for out-of-range arguments or when a field would exceed 2^53
+ * (positions must stay exact in fp64). */
+still_status still_lookahead_pass_info(int64_t k, int64_t c, int32_t t,
+                                       still_lookahead_pass* out);
+
+/* Host only. Passes (T / (c t)) and retained cache entries (T / c + c t) once T tokens have
+ * been compacted; T must be a positive multiple of c*t (else STILL_ERR_SHAPE). */
+still_status still_lookahead_totals(int64_t T, int64_t c, int32_t t, int64_t* h_passes,
+                                    int64_t* h_retained);
+
+/* Compaction step of one lookahead pass for B sequences at once, each at its own pass
+ * index: sequence b's raw chunk (c*t tokens at positions h_pass[b]*c*t + i, as the base
+ * model cached them) is compacted to t slots at output positions evenly spaced over the
+ * chunk. One ragged call (still_compact_layer_ragged) with one position segment per
+ * sequence.
+ *   K, V    [B * c*t, H, d] bf16 packed chunks, sequence b at rows [b*c*t, (b+1)*c*t)
+ *   h_pass  [B] pass indices k_b >= 0 (host)
+ *   Ck, Cv  [B * t, H, d] bf16 outputs, sequence b at rows [b*t, (b+1)*t); the caller
+ *           appends them at row h_pass[b]*t (compact_row) of that sequence's compact prefix
+ * Requires 1 <= t <= t_max of the layer. */
+still_status still_lookahead_compact_layer(still_ctx* ctx, int32_t layer, int32_t B,
+                                           const void* K, const void* V, const int64_t* h_pass,
+                                           int64_t c, int32_t t, void* Ck, void* Cv,
+                                           void* stream);
+
+/* still_lookahead_compact_layer over the layers l < n_layers with h_compact_layer[l] != 0
+ * (NULL: every layer), per-layer pointer arrays in host memory as in
+ * still_compact_stack_masked. */
+still_status still_lookahead_compact_stack(still_ctx* ctx, int32_t n_layers,
+                                           const uint8_t* h_compact_layer, int32_t B,
+                                           const void* const* K, const void* const* V,
+                                           const int64_t* h_pass, int64_t c, int32_t t,
+                                           void* const* Ck, void* const* Cv, void* stream);
 
 /* Device workspace bytes a call with up to max_tokens tokens and compact length max_t needs
  * for layer 0's configuration (the context allocates it on demand and keeps it). */

@@ -45,6 +45,16 @@ __device__ __forceinline__ void split_pack(float a, float b, uint32_t& hi, uint3
   lo = *reinterpret_cast<const uint32_t*>(&l);
 }
 
+// hi/lo split of two values in fp16 (11-bit significands: about 22 bits together):
+// hi = fp16(x), lo = fp16(x - hi), packed.
+__device__ __forceinline__ void split_pack_f16(float a, float b, uint32_t& hi, uint32_t& lo) {
+  const __half2 h = __floats2half2_rn(a, b);
+  const float2 hf = __half22float2(h);
+  const __half2 l = __floats2half2_rn(a - hf.x, b - hf.y);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
+}
+
 // 32 floats -> 32 bf16 packed in 4 x uint4
 __device__ __forceinline__ void pack_bf16x32(const float (&v)[32], uint4 (&o)[4]) {
 #pragma unroll
@@ -340,25 +350,57 @@ __device__ __forceinline__ double seg_position(const PosSegs& s, int64_t idx) {
 //   k~ = acc + b_K;  sumsq(token, head) += |k~|^2;  k = RoPE_c(k~, p_n)  -> hi/lo bf16.
 // Columns are in "pair-chunk" order: within each 256-column tile, columns [0,128) hold the
 // first elements of 128 RoPE pairs and [128,256) their partners, so a tile owns whole pairs.
-// The angle p_n * omega_m is split as G_g * omega_m (table, built in fp64) + delta * omega_m
-// (fp32, delta = p_n - G_g in [0, kPosGrain)), combined by the angle-addition formulas. The
+// The angle p_n * omega_m is split as G_g * omega_m + i * omega_m + f * omega_m with
+// delta = p_n - G_g in [0, kPosGrain), i = floor(delta) and f = delta - i: the first two
+// rotations come from tables built per call in fp64 (coarse[g], fine[i]), the third (only for
+// fractional positions, |f * omega_m| < 1) from Taylor series; the three are combined by the
+// angle-addition formulas. Every rotation is thus accurate to fp32 rounding; forming
+// delta * omega_m in fp32 instead would leave angle errors near 2e-6 rad at delta ~ 31. The
 // per-token (g, delta) come from a table formed once per call in fp64 (gd[n] = (g, delta)), so
 // the epilogue itself does no fp64 arithmetic.
 constexpr int kPosGrain = 32;
 
-struct EpiRopeC {
+// sin and cos of |x| <= 1 from their Taylor series about 0, through x^11 and x^12 (the first
+// omitted terms are below 2e-10), by Horner's rule in fp32: no range reduction needed.
+__device__ __forceinline__ void sincos_taylor(float x, float* s, float* c) {
+  const float x2 = x * x;
+  float ps = 1.f / 39916800.f;                  // 1/11!
+  ps = fmaf(ps, -x2, 1.f / 362880.f);           // 1/9!
+  ps = fmaf(ps, -x2, 1.f / 5040.f);             // 1/7!
+  ps = fmaf(ps, -x2, 1.f / 120.f);              // 1/5!
+  ps = fmaf(ps, -x2, 1.f / 6.f);                // 1/3!
+  ps = fmaf(ps, -x2, 1.f);
+  float pc = 1.f / 479001600.f;                 // 1/12!
+  pc = fmaf(pc, -x2, 1.f / 3628800.f);          // 1/10!
+  pc = fmaf(pc, -x2, 1.f / 40320.f);            // 1/8!
+  pc = fmaf(pc, -x2, 1.f / 720.f);              // 1/6!
+  pc = fmaf(pc, -x2, 1.f / 24.f);               // 1/4!
+  pc = fmaf(pc, -x2, 0.5f);                     // 1/2!
+  *s = x * ps;
+  *c = fmaf(pc, -x2, 1.f);
+}
+
+// kFrac: some key positions are fractional (the sub-unit rotation is compiled in only then,
+// so the integer-position kernel keeps its registers).
+template <bool kFrac>
+struct EpiRopeCT {
   // Element-wise heavy and MMA-light (K = 3d): four warps per lane quarter, each owning 32 of
   // the tile's 128 pairs, processed 16 at a time; a short pipeline suffices.
   static constexpr int kWarps = 16;
   static constexpr int kParts = kWarps / 4;
+  static constexpr int kPairsPerPart = 128 / kParts;  // RoPE pairs of a tile per warp
   static constexpr int kStages = 3;
   static constexpr int kStoreBufs = 1;  // 4 KB TMA-store staging buffers per warp
   __nv_bfloat16* out = nullptr;  // [H][n][N][2D]: hi at [0, D), lo at [D, 2D) (via the TMA view)
   float* sumsq = nullptr;        // [H][n][kParts * D / 256][N] partial sums of |k~|^2 (part-major)
   const float* bias = nullptr;   // [n*D], pair-chunk order
   const float2* coarse = nullptr;  // [G][D/2]: (cos, sin)(G_g * omega_m)
+  // [D/2][kPosGrain]: (cos, sin)(i * omega_m), i fastest: the 32 consecutive tokens of a warp
+  // read 32 neighbouring entries of one pair's row (one 256-byte span per load)
+  const float2* fine = nullptr;
   const float* omega = nullptr;    // [D/2] fp32
   const float2* gd = nullptr;      // [Ntok]: (coarse index g as float, delta)
+  int32_t fp16 = 0;                // hi / lo as fp16 (about 22 bits) instead of bf16
   int32_t D = 0, nheads = 0, ncoarse = 0;
   int64_t Ntok = 0;
   int32_t tile_cols_ = 256;  // must be 256: a tile holds 128 whole RoPE pairs
@@ -377,22 +419,25 @@ struct EpiRopeC {
     const int m_base = (f_tile / 256) * 128;  // first pair index of this tile
     const float2 gdr = rvalid ? gd[r] : make_float2(0.f, 0.f);
     const int g = max(0, min((int)gdr.x, ncoarse - 1));
-    const float delta = gdr.y;
+    const int di = max(0, min((int)gdr.y, kPosGrain - 1));
+    const float frac = gdr.y - (float)di;  // exact; 0 for integer positions
+    const bool any_frac = kFrac && __any_sync(0xffffffffu, frac != 0.f);
     float ss = 0.f;
-    // Part p owns pairs [32p, 32p + 32) of the tile, taken 16 at a time. With kStoreBufs = 2 the
+    // Part p owns pairs [p, p + 1) * kPairsPerPart of the tile, 16 at a time. With kStoreBufs = 2 the
     // staging area holds two 4 KB buffers used alternately, so one iteration's TMA stores can
     // still be reading while the next fills the other buffer.
-    for (int it = 0; it < 2; ++it) {
-      const int u = 32 * half + 16 * it;
+    for (int it = 0; it < kPairsPerPart / 16; ++it) {
+      const int u = kPairsPerPart * half + 16 * it;
       // tables first: their latency overlaps the TMEM loads
       const float4* crow = reinterpret_cast<const float4*>(coarse + (int64_t)g * (D / 2) + m_base + u);
+      const float2* fcol = fine + (int64_t)(m_base + u) * kPosGrain + di;
       const float4* om4 = reinterpret_cast<const float4*>(omega + m_base + u);
       const float4* ba4 = reinterpret_cast<const float4*>(bias + c_tile + u);
       const float4* bb4 = reinterpret_cast<const float4*>(bias + c_tile + 128 + u);
       float4 w[4], xa[4], xb[4], cs[8];
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
-        w[q] = om4[q];
+        w[q] = any_frac ? om4[q] : make_float4(0.f, 0.f, 0.f, 0.f);
         xa[q] = ba4[q];
         xb[q] = bb4[q];
         cs[2 * q] = crow[2 * q];
@@ -407,16 +452,28 @@ struct EpiRopeC {
         const float bbs[4] = {xb[q].x, xb[q].y, xb[q].z, xb[q].w};
         const float cc[4] = {cs[2 * q].x, cs[2 * q].z, cs[2 * q + 1].x, cs[2 * q + 1].z};
         const float sc[4] = {cs[2 * q].y, cs[2 * q].w, cs[2 * q + 1].y, cs[2 * q + 1].w};
+        float cf[4], sf[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const float2 f = fcol[(4 * q + k) * kPosGrain];  // small table: L1-resident
+          cf[k] = f.x;
+          sf[k] = f.y;
+        }
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
           const int e = 4 * q + k;
           const float x = a[e] + bas[k];
           const float y = bb[e] + bbs[k];
           ss += x * x + y * y;
-          float sf, cf;
-          __sincosf(delta * ws[k], &sf, &cf);
-          const float cw = cc[k] * cf - sc[k] * sf;  // cos(G w + delta w)
-          const float sw = sc[k] * cf + cc[k] * sf;  // sin(G w + delta w)
+          float cw = cc[k] * cf[k] - sc[k] * sf[k];  // cos(G w + i w)
+          float sw = sc[k] * cf[k] + cc[k] * sf[k];  // sin(G w + i w)
+          if (any_frac) {  // + f w, |f w| < 1
+            float s3, c3;
+            sincos_taylor(frac * ws[k], &s3, &c3);
+            const float c2 = cw * c3 - sw * s3;
+            sw = sw * c3 + cw * s3;
+            cw = c2;
+          }
           a[e] = x * cw - y * sw;
           bb[e] = x * sw + y * cw;
         }
@@ -436,12 +493,20 @@ struct EpiRopeC {
       for (int q = 0; q < 2; ++q) {
         uint32_t h[4], l[4];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) split_pack(a[8 * q + 2 * k], a[8 * q + 2 * k + 1], h[k], l[k]);
+        for (int k = 0; k < 4; ++k) {
+          if (fp16)
+            split_pack_f16(a[8 * q + 2 * k], a[8 * q + 2 * k + 1], h[k], l[k]);
+          else
+            split_pack(a[8 * q + 2 * k], a[8 * q + 2 * k + 1], h[k], l[k]);
+        }
         bl[q] = make_uint4(h[0], h[1], h[2], h[3]);
         bl[64 + q] = make_uint4(l[0], l[1], l[2], l[3]);
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          split_pack(bb[8 * q + 2 * k], bb[8 * q + 2 * k + 1], h[k], l[k]);
+          if (fp16)
+            split_pack_f16(bb[8 * q + 2 * k], bb[8 * q + 2 * k + 1], h[k], l[k]);
+          else
+            split_pack(bb[8 * q + 2 * k], bb[8 * q + 2 * k + 1], h[k], l[k]);
         bl[128 + q] = make_uint4(h[0], h[1], h[2], h[3]);
         bl[192 + q] = make_uint4(l[0], l[1], l[2], l[3]);
       }

@@ -52,7 +52,7 @@ __device__ __forceinline__ void load8(const __nv_bfloat16* p, bool vec, float (&
 // shared memory with an odd word pitch (conflict-free column reads).
 __global__ void __launch_bounds__(256) strip_kernel(KVSource src, int64_t N, int H, int d,
                                                     PosSegs segs, const double* __restrict__ omega,
-                                                    int rope_fix, int vec,
+                                                    int rope_fix, int vec, int x16,
                                                     __nv_bfloat16* __restrict__ X,
                                                     __half* __restrict__ XT, int64_t Np,
                                                     float2* __restrict__ gd, double pmin, int G) {
@@ -109,8 +109,13 @@ __global__ void __launch_bounds__(256) strip_kernel(KVSource src, int64_t N, int
         uint32_t ah[4], al[4], bh[4], bl[4];
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-          split_pack(a[2 * k], a[2 * k + 1], ah[k], al[k]);
-          split_pack(b[2 * k], b[2 * k + 1], bh[k], bl[k]);
+          if (x16) {
+            split_pack_f16(a[2 * k], a[2 * k + 1], ah[k], al[k]);
+            split_pack_f16(b[2 * k], b[2 * k + 1], bh[k], bl[k]);
+          } else {
+            split_pack(a[2 * k], a[2 * k + 1], ah[k], al[k]);
+            split_pack(b[2 * k], b[2 * k + 1], bh[k], bl[k]);
+          }
         }
         __nv_bfloat16* xr = X + ((int64_t)h * N + n) * d3;
         if (vec) {
@@ -156,7 +161,10 @@ __global__ void __launch_bounds__(256) strip_kernel(KVSource src, int64_t N, int
         const __nv_bfloat16* vr = (second ? src.V2 : src.V) + off + f0;
         load8(vr, vec, v);
         __nv_bfloat16* xr = X + ((int64_t)h * N + n) * d3 + d + f0;
-        if (vec) {
+        if (x16) {  // values in fp16 (bf16 values in the fp16 range convert exactly)
+#pragma unroll
+          for (int e = 0; e < 8; ++e) reinterpret_cast<__half*>(xr)[e] = __float2half_rn(v[e]);
+        } else if (vec) {
           *reinterpret_cast<uint4*>(xr) = *reinterpret_cast<const uint4*>(vr);
         } else {
 #pragma unroll
@@ -195,15 +203,20 @@ __global__ void __launch_bounds__(256) strip_kernel(KVSource src, int64_t N, int
   }
 }
 
+// Rows [0, G): coarse[g][m] = (cos, sin)((pmin + g * kPosGrain) * w_m); then, in the next
+// kPosGrain * D/2 entries, fine[m][i] = (cos, sin)(i * w_m). Angles formed and reduced in fp64.
 __global__ void rope_tables_kernel(float2* coarse, float* omega, int G, int D, double pmin,
                                    const double* __restrict__ omega_c) {
   const int half = D / 2;
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= (int64_t)G * half) return;
-  const int g = (int)(idx / half), m = (int)(idx % half);
+  if (idx >= (int64_t)(G + kPosGrain) * half) return;
+  const int g = (int)(idx / half);
+  const int64_t f = idx - (int64_t)G * half;  // index into the fine table when >= 0
+  const int m = g < G ? (int)(idx % half) : (int)(f / kPosGrain);
   const double w = omega_c[m];
   float s, c;
-  sincos_reduced((pmin + (double)g * kPosGrain) * w, &s, &c);
+  const double ang = g < G ? (pmin + (double)g * kPosGrain) * w : (double)(f % kPosGrain) * w;
+  sincos_reduced(ang, &s, &c);
   coarse[idx] = make_float2(c, s);
   if (g == 0) omega[m] = (float)w;
 }
@@ -225,7 +238,8 @@ __global__ void heads_rot_kernel(float2* rot, int t, int hd, double pstart, doub
 // partner at f1 + 128, so four consecutive pairs are four consecutive columns.
 __global__ void q_rope_kernel(const float* __restrict__ qhat, int t_max, int b0, int nb, int t,
                               int D, double qstart, double qstep, const double* omega_c,
-                              int use_rope, __nv_bfloat16* __restrict__ qhl) {
+                              int use_rope, __nv_bfloat16* __restrict__ qhl, int fp16,
+                              float qscale) {
   const int half = D / 2, q4 = half / 4;
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (int64_t)t * q4) return;
@@ -250,10 +264,17 @@ __global__ void q_rope_kernel(const float* __restrict__ qhat, int t_max, int b0,
       b[e] = x[e] * s[e] + y[e] * c[e];
     }
     uint32_t ah[2], al[2], bh[2], bl[2];
-    split_pack(a[0], a[1], ah[0], al[0]);
-    split_pack(a[2], a[3], ah[1], al[1]);
-    split_pack(b[0], b[1], bh[0], bl[0]);
-    split_pack(b[2], b[3], bh[1], bl[1]);
+    if (fp16) {
+      split_pack_f16(a[0] * qscale, a[1] * qscale, ah[0], al[0]);
+      split_pack_f16(a[2] * qscale, a[3] * qscale, ah[1], al[1]);
+      split_pack_f16(b[0] * qscale, b[1] * qscale, bh[0], bl[0]);
+      split_pack_f16(b[2] * qscale, b[3] * qscale, bh[1], bl[1]);
+    } else {
+      split_pack(a[0], a[1], ah[0], al[0]);
+      split_pack(a[2], a[3], ah[1], al[1]);
+      split_pack(b[0], b[1], bh[0], bl[0]);
+      split_pack(b[2], b[3], bh[1], bl[1]);
+    }
     __nv_bfloat16* o = qhl + ((int64_t)bb * t + j) * 2 * D;
     *reinterpret_cast<uint2*>(o + f1) = make_uint2(ah[0], ah[1]);
     *reinterpret_cast<uint2*>(o + D + f1) = make_uint2(al[0], al[1]);
@@ -328,7 +349,9 @@ __global__ void __launch_bounds__(256) softmax_kernel(const float* __restrict__ 
 }
 
 // Row softmax with the row held in registers: 256 threads, PER columns each (float4 groups).
-template <typename OutT, int PER>
+// HILO (bf16 only): the row is written as hi at [0, ldP) and lo = bf16(p - hi) at
+// [ldP, 2 ldP) of a row of pitch 2 ldP.
+template <typename OutT, int PER, bool HILO = false>
 __global__ void __launch_bounds__(256) softmax_reg_kernel(const float* __restrict__ S,
                                                           int64_t ncols, int64_t ldS,
                                                           OutT* __restrict__ P, int64_t ldP) {
@@ -376,21 +399,24 @@ __global__ void __launch_bounds__(256) softmax_reg_kernel(const float* __restric
 #pragma unroll
   for (int w = 0; w < 8; ++w) l += red[w];
   const float inv = 1.f / l;
-  OutT* prow = P + row * ldP;
+  OutT* prow = P + row * (HILO ? 2 * ldP : ldP);
 #pragma unroll
   for (int i = 0; i < G; ++i) {
     const int64_t c = (int64_t)(i * 256 + threadIdx.x) * 4;
     if (c < ldP) {
-      OutT o4[4];
+      OutT o4[4], l4[4];
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
         const float y = v[4 * i + k] * inv;
-        if constexpr (std::is_same<OutT, __half>::value)
+        if constexpr (std::is_same<OutT, __half>::value) {
           o4[k] = __float2half_rn(y);
-        else
+        } else {
           o4[k] = __float2bfloat16_rn(y);
+          if constexpr (HILO) l4[k] = __float2bfloat16_rn(y - __bfloat162float(o4[k]));
+        }
       }
       *reinterpret_cast<uint2*>(prow + c) = *reinterpret_cast<const uint2*>(o4);
+      if constexpr (HILO) *reinterpret_cast<uint2*>(prow + ldP + c) = *reinterpret_cast<const uint2*>(l4);
     }
   }
 }
@@ -516,7 +542,12 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const void* __restrict__ i
   __nv_bfloat16* o = out + row * ldo;
   for (int c = lane; c < D; c += 32) {
     const float y = ld(c) * scale;
-    if (hilo) {
+    if (hilo == 2) {  // fp16 hi | lo
+      const __half hi = __float2half_rn(y);
+      const __half lo = __float2half_rn(y - __half2float(hi));
+      reinterpret_cast<__half*>(o)[c] = hi;
+      reinterpret_cast<__half*>(o)[D + c] = lo;
+    } else if (hilo) {
       __nv_bfloat16 hi, lo;
       split_hilo(y, hi, lo);
       o[c] = hi;
@@ -525,6 +556,14 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const void* __restrict__ i
       o[c] = __float2bfloat16_rn(y);
     }
   }
+}
+
+__global__ void bf16_to_f16_kernel(uint16_t* p, int64_t n) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const __nv_bfloat16 b = *reinterpret_cast<const __nv_bfloat16*>(&p[i]);
+  const __half h = __float2half_rn(__bfloat162float(b));
+  p[i] = *reinterpret_cast<const uint16_t*>(&h);
 }
 
 __global__ void scale_rows_kernel(float* x, const float* inv, int64_t rows, int D) {
@@ -576,7 +615,7 @@ inline unsigned blocks_for(int64_t n, int per) { return (unsigned)((n + per - 1)
 
 cudaError_t launch_strip(const KVSource& src, int64_t N, int H, int d, const PosSegs& segs,
                          const double* omega, int rope_fix, __nv_bfloat16* X, __half* XT,
-                         int64_t Np, float2* gd, double pmin, int G, cudaStream_t s) {
+                         int64_t Np, float2* gd, double pmin, int G, int x16, cudaStream_t s) {
   if (d % 16 != 0 || Np % kStripTok != 0) return cudaErrorInvalidValue;
   const size_t smem = (size_t)kStripTok * (d / 2) * sizeof(float2) +
                       (size_t)kStripTok * ((2 * d + 2) + (d + 2)) * 2;
@@ -591,7 +630,7 @@ cudaError_t launch_strip(const KVSource& src, int64_t N, int H, int d, const Pos
     attr = true;
   }
   strip_kernel<<<(unsigned)(Np / kStripTok), 256, smem, s>>>(src, N, H, d, segs, omega, rope_fix,
-                                                             vec, X, XT, Np, gd, pmin, G);
+                                                             vec, x16, X, XT, Np, gd, pmin, G);
   return cudaGetLastError();
 }
 
@@ -604,37 +643,37 @@ cudaError_t launch_heads_rot(float2* rot, int t, int hd, double pstart, double p
 
 cudaError_t launch_rope_tables(float2* coarse, float* omega, int G, int D, double pmin,
                                const double* omega_c, cudaStream_t s) {
-  const int64_t n = (int64_t)G * (D / 2);
+  const int64_t n = (int64_t)(G + kPosGrain) * (D / 2);
   rope_tables_kernel<<<blocks_for(n, 256), 256, 0, s>>>(coarse, omega, G, D, pmin, omega_c);
   return cudaGetLastError();
 }
 
 cudaError_t launch_q_rope(const float* qhat, int t_max, int b0, int nb, int t, int D,
                           double qstart, double qstep, const double* omega_c, int use_rope,
-                          __nv_bfloat16* qhl, cudaStream_t s) {
+                          __nv_bfloat16* qhl, int fp16, float qscale, cudaStream_t s) {
   if (D % 256 != 0) return cudaErrorInvalidValue;
   const int64_t n = (int64_t)t * (D / 8);
   q_rope_kernel<<<blocks_for(n, 256), 256, 0, s>>>(qhat, t_max, b0, nb, t, D, qstart, qstep,
-                                                    omega_c, use_rope, qhl);
+                                                    omega_c, use_rope, qhl, fp16, qscale);
   return cudaGetLastError();
 }
 
-template <typename OutT>
+template <typename OutT, bool HILO = false>
 static bool softmax_reg(const float* S, int64_t rows, int64_t ncols, int64_t ldS, void* P,
                         int64_t ldP, cudaStream_t s) {
   const int64_t need = std::max(ldP, ncols);
   OutT* Pt = static_cast<OutT*>(P);
   if ((ldS % 4) != 0 || (ldP % 4) != 0) return false;
   if (need <= 1024)
-    softmax_reg_kernel<OutT, 4><<<(unsigned)rows, 256, 0, s>>>(S, ncols, ldS, Pt, ldP);
+    softmax_reg_kernel<OutT, 4, HILO><<<(unsigned)rows, 256, 0, s>>>(S, ncols, ldS, Pt, ldP);
   else if (need <= 2048)
-    softmax_reg_kernel<OutT, 8><<<(unsigned)rows, 256, 0, s>>>(S, ncols, ldS, Pt, ldP);
+    softmax_reg_kernel<OutT, 8, HILO><<<(unsigned)rows, 256, 0, s>>>(S, ncols, ldS, Pt, ldP);
   else if (need <= 4096)
-    softmax_reg_kernel<OutT, 16><<<(unsigned)rows, 256, 0, s>>>(S, ncols, ldS, Pt, ldP);
+    softmax_reg_kernel<OutT, 16, HILO><<<(unsigned)rows, 256, 0, s>>>(S, ncols, ldS, Pt, ldP);
   else if (need <= 8192)
-    softmax_reg_kernel<OutT, 32><<<(unsigned)rows, 256, 0, s>>>(S, ncols, ldS, Pt, ldP);
+    softmax_reg_kernel<OutT, 32, HILO><<<(unsigned)rows, 256, 0, s>>>(S, ncols, ldS, Pt, ldP);
   else if (need <= 16384)
-    softmax_reg_kernel<OutT, 64><<<(unsigned)rows, 256, 0, s>>>(S, ncols, ldS, Pt, ldP);
+    softmax_reg_kernel<OutT, 64, HILO><<<(unsigned)rows, 256, 0, s>>>(S, ncols, ldS, Pt, ldP);
   else
     return false;
   return true;
@@ -659,6 +698,11 @@ cudaError_t launch_omega(double* out, int half, int width, double base, cudaStre
 cudaError_t launch_softmax(const float* S, int64_t rows, int64_t ncols, int64_t ldS, void* P,
                            int64_t ldP, int out_fp16, cudaStream_t s) {
   if (rows == 0) return cudaSuccess;
+  if (out_fp16 == 2) {  // bf16 hi | lo rows
+    if (!softmax_reg<__nv_bfloat16, true>(S, rows, ncols, ldS, P, ldP, s))
+      return cudaErrorInvalidValue;
+    return cudaGetLastError();
+  }
   if (out_fp16 ? softmax_reg<__half>(S, rows, ncols, ldS, P, ldP, s)
                : softmax_reg<__nv_bfloat16>(S, rows, ncols, ldS, P, ldP, s))
     return cudaGetLastError();
@@ -693,6 +737,12 @@ cudaError_t launch_rmsnorm(const void* in, int in_bf16, int64_t rows, int D, int
                            float eps, __nv_bfloat16* out, int64_t ldo, int hilo, cudaStream_t s) {
   rmsnorm_kernel<<<blocks_for(rows, 8), 256, 0, s>>>(in, in_bf16, rows, D, ldi, eps, out, ldo,
                                                      hilo);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_bf16_to_f16(void* p, int64_t n, cudaStream_t s) {
+  if (n == 0) return cudaSuccess;
+  bf16_to_f16_kernel<<<blocks_for(n, 256), 256, 0, s>>>(static_cast<uint16_t*>(p), n);
   return cudaGetLastError();
 }
 

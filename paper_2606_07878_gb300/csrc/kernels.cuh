@@ -26,16 +26,22 @@ struct KVSource {
 // the value half are not written). omega: [d/2] fp64 base-model frequencies theta^(-2m/d).
 // Also gd[n] = (g, p_n - (pmin + g * kPosGrain)) with g = floor((p_n - pmin) / kPosGrain)
 // clamped to [0, G): the compactor-RoPE coarse index and residual of token n (n < N).
+// x16: X in fp16 (hi | key lo as fp16 hi / lo, values as fp16) instead of bf16.
 cudaError_t launch_strip(const KVSource& src, int64_t N, int H, int d, const PosSegs& segs,
                          const double* omega, int rope_fix, __nv_bfloat16* X, __half* XT,
-                         int64_t Np, float2* gd, double pmin, int G, cudaStream_t s);
+                         int64_t Np, float2* gd, double pmin, int G, int x16, cudaStream_t s);
+
+// Converts n bf16 values to fp16 in place (exact within the fp16 range; values below it
+// become fp16 subnormals, absolute error <= 2^-25).
+cudaError_t launch_bf16_to_f16(void* p, int64_t n, cudaStream_t s);
 
 // rot[j][m] = (cos, sin)((pstart + j * pstep) * omega[m]) for j < t, m < hd (angle reduced
 // modulo 2 pi in fp64); (1, 0) when use_rope is 0. The output heads' re-rotation table.
 cudaError_t launch_heads_rot(float2* rot, int t, int hd, double pstart, double pstep,
                              const double* omega, int use_rope, cudaStream_t s);
 
-// Compactor-RoPE tables: coarse[g][m] = (cos, sin)((pmin + g * kPosGrain) * w_m), omega[m] = w_m
+// Compactor-RoPE tables: coarse[g][m] = (cos, sin)((pmin + g * kPosGrain) * w_m) for g < G,
+// then fine[m][i] = (cos, sin)(i * w_m) for i < kPosGrain at coarse + G * D/2; omega[m] = w_m
 // (fp32), w_m = omega_c[m] = theta_c^(-2m/D) (fp64 table), angles reduced in fp64.
 cudaError_t launch_rope_tables(float2* coarse, float* omega, int G, int D, double pmin,
                                const double* omega_c, cudaStream_t s);
@@ -43,9 +49,10 @@ cudaError_t launch_rope_tables(float2* coarse, float* omega, int G, int D, doubl
 // Per-call cross-attention queries: q = RoPE_c(q^, p_j) for latents j < t, batches
 // b in [b0, b0 + nb) (b = h * n + i), as hi/lo bf16 [nb * t][2D]. q^ is [H*n][t_max][D] fp32
 // in pair-chunk column order; p_j = qstart + j * qstep.
+// fp16: hi/lo in fp16 of (q * qscale) instead of bf16 of q (qscale a power of two).
 cudaError_t launch_q_rope(const float* qhat, int t_max, int b0, int nb, int t, int D,
                           double qstart, double qstep, const double* omega_c, int use_rope,
-                          __nv_bfloat16* qhl, cudaStream_t s);
+                          __nv_bfloat16* qhl, int fp16, float qscale, cudaStream_t s);
 
 // Row softmax statistics from the scores epilogue's per-tile partials (max, sum of exp):
 // out[row] = (M * log2 e, 1 / L) with M the row max and L the sum of exp(s - M).
@@ -59,7 +66,8 @@ cudaError_t launch_wait_timeout_selftest(int* err, unsigned long long limit_ns, 
 cudaError_t launch_omega(double* out, int half, int width, double base, cudaStream_t s);
 
 // Row softmax: S fp32 [rows][ldS] (first ncols valid) -> P [rows][ldP], zero beyond ncols.
-// out_fp16: P is fp16, else bf16.
+// out_fp16: 1 = P is fp16; 0 = bf16; 2 = bf16 hi | lo: rows of pitch 2 ldP, hi at [0, ldP),
+// lo = bf16(p - hi) at [ldP, 2 ldP) (ldP and ncols up to 16384).
 cudaError_t launch_softmax(const float* S, int64_t rows, int64_t ncols, int64_t ldS, void* P,
                            int64_t ldP, int out_fp16, cudaStream_t s);
 
@@ -83,7 +91,8 @@ cudaError_t launch_inv_norms(const float* parts, int64_t nvec, int nparts, int64
                              float alpha, float* out, cudaStream_t s);
 
 // Non-parametric RMSNorm over rows of width D: out = x / sqrt(mean(x^2) + eps) as bf16 hi
-// (and lo at +D when hilo), row pitch ldo. Input fp32 or bf16 (in_bf16), row pitch ldi.
+// (and lo at +D when hilo = 1; fp16 hi and lo when hilo = 2), row pitch ldo. Input fp32 or
+// bf16 (in_bf16), row pitch ldi.
 cudaError_t launch_rmsnorm(const void* in, int in_bf16, int64_t rows, int D, int64_t ldi,
                            float eps, __nv_bfloat16* out, int64_t ldo, int hilo, cudaStream_t s);
 

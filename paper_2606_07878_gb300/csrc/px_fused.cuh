@@ -61,10 +61,12 @@ struct PxParams {
   int32_t nb = 0, bdiv = 1;       // batches; KV-head of batch b = (b / bdiv)
 };
 
-// BN: output columns per tile; LOB: rows of the X^T lo box (the key half inside the tile).
-template <int BN, int LOB>
+// BN: output columns per tile; LOB: rows of the X^T lo box (the key half inside the tile);
+// PLO: the probabilities as fp16 hi + lo (a second P tile and one more MMA pass).
+template <int BN, int LOB, bool PLO = false>
 struct PxSmem {
-  static constexpr int kABytes = kBM * kBK * 2;       // P tile (fp16)
+  static constexpr int kPBytes = kBM * kBK * 2;       // one P tile (fp16)
+  static constexpr int kABytes = kPBytes * (PLO ? 2 : 1);  // P hi [, P lo]
   static constexpr int kBBytes = BN * kBK * 2;        // X^T hi tile
   static constexpr int kLoBytes = LOB * kBK * 2;      // X^T lo tile
   static constexpr int kStageBytes = kABytes + kBBytes + kLoBytes;
@@ -80,13 +82,13 @@ struct PxSmem {
 // "pass" of klen = Np describes the token range (iters_total = Np / 64).
 constexpr int kPxThreads = 64 + 32 * kPxTransformWarps + 32 * EpiPxOut::kWarps;
 
-template <int BN, int LOB>
+template <int BN, int LOB, bool PLO>
 __global__ void __launch_bounds__(kPxThreads, 1)
     px_fused_kernel(const __grid_constant__ CUtensorMap tmXhi,
                     const __grid_constant__ CUtensorMap tmXlo,
                     const __grid_constant__ CUtensorMap tmC, const GemmParams p,
                     const PxParams px, const EpiPxOut epi) {
-  using S = PxSmem<BN, LOB>;
+  using S = PxSmem<BN, LOB, PLO>;
   constexpr int kStages = S::kStages;
   constexpr int kEpiWarps = EpiPxOut::kWarps;
   constexpr int kTW = kPxTransformWarps;
@@ -202,6 +204,11 @@ __global__ void __launch_bounds__(kPxThreads, 1)
 #pragma unroll
           for (int k = 0; k < kBK / 16; ++k)
             tc_mma_f16(d_tmem, ad + 2 * k, bd + 2 * k, idesc_hi, (it > it0 || k > 0) ? 1u : 0u);
+          if constexpr (PLO) {  // + P_lo X_hi
+            const uint64_t pl = sdesc_k_sw128(sa + S::kPBytes);
+#pragma unroll
+            for (int k = 0; k < kBK / 16; ++k) tc_mma_f16(d_tmem, pl + 2 * k, bd + 2 * k, idesc_hi, 1u);
+          }
           if (lo_w > 0) {
 #pragma unroll
             for (int k = 0; k < kBK / 16; ++k) tc_mma_f16(d_tmem, ad + 2 * k, ld + 2 * k, idesc_lo, 1u);
@@ -294,6 +301,17 @@ __global__ void __launch_bounds__(kPxThreads, 1)
           a[r * 8 + (chunk ^ (r & 7))] =
               make_uint4(*reinterpret_cast<uint32_t*>(&h01), *reinterpret_cast<uint32_t*>(&h23),
                          *reinterpret_cast<uint32_t*>(&h45), *reinterpret_cast<uint32_t*>(&h67));
+          if constexpr (PLO) {  // lo = fp16(p - hi), same swizzled position in the P_lo tile
+            const float2 f01 = __half22float2(h01), f23 = __half22float2(h23);
+            const float2 f45 = __half22float2(h45), f67 = __half22float2(h67);
+            __half2 l01 = __floats2half2_rn(v[0] - f01.x, v[1] - f01.y);
+            __half2 l23 = __floats2half2_rn(v[2] - f23.x, v[3] - f23.y);
+            __half2 l45 = __floats2half2_rn(v[4] - f45.x, v[5] - f45.y);
+            __half2 l67 = __floats2half2_rn(v[6] - f67.x, v[7] - f67.y);
+            a[S::kPBytes / 16 + r * 8 + (chunk ^ (r & 7))] =
+                make_uint4(*reinterpret_cast<uint32_t*>(&l01), *reinterpret_cast<uint32_t*>(&l23),
+                           *reinterpret_cast<uint32_t*>(&l45), *reinterpret_cast<uint32_t*>(&l67));
+          }
         }
         fence_proxy_async_smem();
         __syncwarp();
@@ -356,16 +374,16 @@ __global__ void __launch_bounds__(kPxThreads, 1)
 namespace still {
 
 // Launches px_fused_kernel: A = probabilities from S (transform warps), B = X^T hi / lo.
-template <int BN, int LOB>
+template <int BN, int LOB, bool PLO = false>
 inline cudaError_t launch_px_fused(const Operand2D& XT, GemmParams p, const PxParams& px,
                                    EpiPxOut epi, int num_sms, cudaStream_t stream) {
-  using S = PxSmem<BN, LOB>;
+  using S = PxSmem<BN, LOB, PLO>;
   if (!finalize_gemm<BN>(p, 0)) return cudaErrorInvalidValue;
   CUtensorMap thi, tlo, tc;
   if (!make_tmap(&thi, XT, BN) || !make_tmap(&tlo, XT, LOB)) return cudaErrorInvalidValue;
   std::memset(&tc, 0, sizeof(tc));
   epi.tile_cols_ = BN;
-  auto kern = px_fused_kernel<BN, LOB>;
+  auto kern = px_fused_kernel<BN, LOB, PLO>;
   static thread_local bool attr_set = false;
   if (!attr_set) {
     cudaError_t e =

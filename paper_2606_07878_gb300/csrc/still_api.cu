@@ -32,16 +32,13 @@ namespace {
 
 using bf16 = __nv_bfloat16;
 
-struct LayerW {
-  bool loaded = false;
-  still_layer_config cfg{};
-  bf16* Z = nullptr;     // [H][t_max][D]
+// One compactor block's weights in the library's layouts (App. A, "Compactor blocks").
+struct BlockW {
+  bool has_ca = false;   // cross-attention in this block
   bf16* WkT = nullptr;   // [nD][2d]  pair-chunk order
   float* bk = nullptr;   // [nD]      pair-chunk order
-  float* qhat = nullptr; // [H][n][t_max][D] fp32, L2-normalised, pair-chunk order
-  bool qhat_lazy = false; // q^ formed per call from Z, WqT, bq (qhat unused)
-  bf16* WqT = nullptr;   // [nD][D] pair-chunk order (lazy q^ only)
-  float* bq = nullptr;   // [nD]    pair-chunk order (lazy q^ only)
+  bf16* WqT = nullptr;   // [nD][D] pair-chunk order (queries formed per call only)
+  float* bq = nullptr;   // [nD]    pair-chunk order (queries formed per call only)
   bf16* WvoT = nullptr;  // [D][2 * n * 2d]: (W_V,i W_O,i)^T hi | lo
   bf16* SqkT = nullptr;  // [2nD][D]
   float* sbqk = nullptr; // [2nD]
@@ -49,6 +46,18 @@ struct LayerW {
   bf16* SoT = nullptr;   // [D][nD]
   bf16* W1T = nullptr;   // [F][D]
   bf16* W2T = nullptr;   // [D][F]
+};
+
+struct LayerW {
+  bool loaded = false;
+  still_layer_config cfg{};
+  bf16* Z = nullptr;     // [H][t_max][D]
+  float* qhat = nullptr; // block 0: [H][n][t_max][D] fp32, L2-normalised, pair-chunk order
+  bool qhat_lazy = false; // block 0's q^ formed per call from Z (qhat unused)
+  // Layers of more than one block keep W_K, W_Q, X and RMSNorm(Z) in fp16 (hi | lo where
+  // split): about 22 bits against bf16 hi | lo's 16, for the amplification across blocks.
+  bool f16 = false;
+  std::vector<BlockW> blk;
   bf16* WhT = nullptr;   // [2d][D]
   double* omega_b = nullptr;  // [d/2] base-model RoPE frequencies (fp64)
   double* omega_c = nullptr;  // [D/2] compactor RoPE frequencies (fp64)
@@ -186,7 +195,9 @@ still_status check_cfg(const still_layer_config* c) {
       !(std::isfinite(c->rope_theta_compactor) && c->rope_theta_compactor > 0) ||
       !std::isfinite(c->logit_scale) || !(c->rms_eps >= 0) || !(c->l2_eps > 0))
     return STILL_ERR_INVALID_ARG;
-  if (c->n_blocks != 1 || c->cross_every_block != 1 || c->n_cross_heads != c->n_self_heads ||
+  if (c->n_blocks < 1 || c->n_blocks > 2 ||
+      (c->cross_every_block != 0 && c->cross_every_block != 1) ||
+      c->n_cross_heads != c->n_self_heads ||
       c->d_latent % 256 != 0 || !(c->head_dim == 64 || c->head_dim == 128 || c->head_dim == 256) ||
       c->ffn_dim % 64 != 0 || c->compactor_rope != 1 || c->rope_fix != 1 ||
       (c->final_norm != 0 && c->final_norm != 1))
@@ -326,25 +337,30 @@ bool make_plan(const still_layer_config& c, bool lazy_q, int64_t N, int t, doubl
   };
   P.oX = take(H * N * 3 * d * 2);
   P.oXT = take(H * 2 * d * 2 * P.Np * 2);
-  P.oCoarse = take((size_t)P.G * (D / 2) * 8);
+  P.oCoarse = take((size_t)(P.G + kPosGrain) * (D / 2) * 8);  // coarse rows, then fine rows
   P.oOmega = take((D / 2) * 4);
   P.oGD = take((size_t)P.Np * 8);
   P.oHrot = take(T * (d / 2) * 8);
   P.oPX = take(H * T * 2 * n * 2 * d * 2);
   P.oZ1 = take(H * T * D * 4);
   P.oA1 = take(H * T * 2 * D * 2);
-  P.oCat = take(H * T * n * D * 2);
+  // A block that feeds another keeps its value path in hi/lo (x2 buffers below).
+  const int64_t hl = c.n_blocks > 1 ? 2 : 1;
+  P.oCat = take(H * T * n * D * 2 * hl);
   P.oZ2 = take(H * T * D * 4);
-  P.oA2 = take(H * T * D * 2);
-  P.oG = take(H * T * std::max<int64_t>(F, 1) * 2);
+  P.oA2 = take(H * T * D * 2 * hl);
+  P.oG = take(H * T * std::max<int64_t>(F, 1) * 2 * hl);
   P.oZ3 = take(H * T * D * 4);
   P.lazy_q = lazy_q;
   P.oZn = lazy_q ? take(H * T * 2 * D * 2) : 0;  // RMSNorm(Z) hi | lo for the call's t latents
   const size_t fixed = off;
   P.kb_b = a256(N * 2 * D * 2);
-  P.kss_b = a256(N * 4 * (EpiRopeC::kParts * (D / 256) + 1));  // |k~|^2 partials + inverses
+  P.kss_b = a256(N * 4 * (EpiRopeCT<false>::kParts * (D / 256) + 1));  // |k~|^2 partials + inverses
   P.q_b = a256(T * 2 * D * 2);
-  P.flash = d == 64 || d == 128;
+  // The fused kernel holds fp16 probabilities; a compactor of two blocks needs the first block's
+  // probabilities in hi | lo (its cross-attention output steers the second block's queries), so
+  // such layers take the scores + P X kernels.
+  P.flash = (d == 64 || d == 128) && c.n_blocks == 1;
   if (P.flash) {
     P.S_b = 0;
     P.P_b = a256(T * 8) * kMaxFlashSplit;          // per-split row statistics (m, l)
@@ -359,11 +375,11 @@ bool make_plan(const still_layer_config& c, bool lazy_q, int64_t N, int t, doubl
   P.ca_unit_bytes = P.kb_b + P.kss_b + P.q_b + P.S_b + P.P_b + P.O_b + P.qt_b;
   P.qk_b = a256(2 * n * T * 2 * D * 2);
   P.sss_b = a256(2 * n * T * 4 * (2 * (D / 256) + 1));
-  P.vT_b = a256(n * D * P.tp * 2);
+  P.vT_b = a256(n * D * P.tp * 2 * hl);
   P.Ssa_b = a256(n * T * P.ldt * 4);
-  P.Psa_b = a256(n * T * P.tp * 2);
+  P.Psa_b = a256(n * T * P.tp * 2 * hl);
   P.Ssah_b = (size_t)T * P.ldt * 4;
-  P.Psah_b = (size_t)T * P.tp * 2;
+  P.Psah_b = (size_t)T * P.tp * 2 * hl;
   P.sa_unit_bytes = P.qk_b + P.sss_b + P.vT_b + P.Ssa_b + P.Psa_b;
   if (fixed >= limit) return false;
   const size_t avail = limit - fixed;
@@ -416,6 +432,7 @@ still_status ensure_ws(still_ctx* ctx, size_t bytes) {
 struct Positions {
   PosSegs segs;
   double pmin = 0, pmax = 0;
+  bool frac = false;  // some position is not an integer
 };
 
 still_status make_positions(const still_pos_segment* h_segments, int32_t n_segments, int64_t N,
@@ -441,6 +458,8 @@ still_status make_positions(const still_pos_segment* h_segments, int32_t n_segme
     if (s.count < 0 || !std::isfinite(s.start) || !std::isfinite(s.step))
       return STILL_ERR_INVALID_ARG;
     if (s.count == 0) continue;
+    if (s.start != std::floor(s.start) || (s.count > 1 && s.step != std::floor(s.step)))
+      out.frac = true;
     const double last = s.start + (double)(s.count - 1) * s.step;
     if (!std::isfinite(last)) return STILL_ERR_INVALID_ARG;
     lo = std::min(lo, std::min(s.start, last));
@@ -469,6 +488,12 @@ struct OutSpec {
 
 // ws_fixed / ws_fixed_bytes: when set, the call runs in that caller-provided scratch and never
 // touches the context's (growable) workspace.
+// Some block's latent queries are formed inside the call (block 0's when too large to keep,
+// every later cross-attending block's).
+bool queries_per_call(const LayerW& L) {
+  return L.qhat_lazy || (L.cfg.n_blocks > 1 && L.cfg.cross_every_block);
+}
+
 still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
                          const Positions& pos, int64_t N, int t, const OutSpec& out,
                          cudaStream_t s, uint8_t* ws_fixed = nullptr,
@@ -476,7 +501,8 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
   const still_layer_config& c = L.cfg;
   Plan P;
   const size_t limit = ws_fixed != nullptr ? ws_fixed_bytes : ctx->ws_limit;
-  if (!make_plan(c, L.qhat_lazy, N, t, pos.pmin, pos.pmax, limit, P)) return STILL_ERR_OOM;
+  if (!make_plan(c, queries_per_call(L), N, t, pos.pmin, pos.pmax, limit, P))
+    return STILL_ERR_OOM;
   if (ws_fixed == nullptr) TRY(ensure_ws(ctx, P.total));
   uint8_t* ws = ws_fixed != nullptr ? ws_fixed : static_cast<uint8_t*>(ctx->ws);
   const int H = P.H, d = P.d, D = P.D, n = P.n, F = P.F;
@@ -501,14 +527,35 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
   void* Z3 = ws + P.oZ3;
 
   KLAUNCH(STILL_K_STRIP, launch_strip(src, N, H, d, pos.segs, L.omega_b, c.rope_fix, X, XT, Np,
-                                      gd, pos.pmin, P.G, s));
+                                      gd, pos.pmin, P.G, L.f16 ? 1 : 0, s));
+  const int w_fmt = L.f16 ? 0 : 1;    // operand format of X, RMSNorm(Z), W_K and W_Q products
+  const int zn_mode = L.f16 ? 2 : 1;  // RMSNorm(Z) as fp16 or bf16 hi | lo
   KLAUNCH(STILL_K_TABLES, launch_rope_tables(coarse, omega, P.G, D, pos.pmin, L.omega_c, s));
   KLAUNCH(STILL_K_TABLES, launch_heads_rot(hrot, t, d / 2, qstart, qstep, L.omega_b, c.rope_fix, s));
   bf16* Zn = P.lazy_q ? reinterpret_cast<bf16*>(ws + P.oZn) : nullptr;
-  if (P.lazy_q) {  // RMSNorm(Z) hi | lo for latents j < t of every KV-head bank
-    for (int h = 0; h < H; ++h)
-      KLAUNCH(STILL_K_LOAD, launch_rmsnorm(L.Z + (size_t)h * c.t_max * D, 1, t, D, D, c.rms_eps,
-                                           Zn + (size_t)h * t * 2 * D, 2 * D, 1, s));
+  const int64_t rows = (int64_t)H * t;
+  const int n2d = n * 2 * d;
+  const bool z3_bf16 = (c.final_norm == 0);
+  // Latent state entering a block: the bank rows L.Z (bf16, pitch t_max) for block 0, else the
+  // fp32 state Z2 [H * t][D] that the previous block left.
+  for (int bi = 0; bi < c.n_blocks; ++bi) {
+  const BlockW& Bw = L.blk[bi];
+  const bool last = bi + 1 == c.n_blocks;
+  // Every block of a layer with more than one block keeps its self-attention value path and
+  // FFN in split precision: the next block's cross-attention queries amplify any rounding
+  // there, and the last block's own rounding adds to the amplified error of the first.
+  const bool exact = !last || L.f16;
+  float* Za = Z2;  // this block's state after cross-attention (Z2 itself without it)
+  if (Bw.has_ca) {
+  const bool q_call = bi > 0 || L.qhat_lazy;  // queries formed in this call
+  if (q_call) {  // RMSNorm(latent state) hi | lo for latents j < t of every KV-head bank
+    if (bi == 0) {
+      for (int h = 0; h < H; ++h)
+        KLAUNCH(STILL_K_LOAD, launch_rmsnorm(L.Z + (size_t)h * c.t_max * D, 1, t, D, D, c.rms_eps,
+                                             Zn + (size_t)h * t * 2 * D, 2 * D, zn_mode, s));
+    } else {
+      KLAUNCH(STILL_K_LOAD, launch_rmsnorm(Z2, 0, rows, D, D, c.rms_eps, Zn, 2 * D, zn_mode, s));
+    }
   }
 
   // ---------------------------------------------------------------- cross-attention groups
@@ -528,7 +575,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     uint8_t* g = ws + P.oCA;
     bf16* kb = reinterpret_cast<bf16*>(g);
     g += P.kb_b * nbl;
-    const int kparts = EpiRopeC::kParts * (D / 256);
+    const int kparts = EpiRopeCT<false>::kParts * (D / 256);
     float* kss = reinterpret_cast<float*>(g);        // [nbl][N][kparts]
     float* kinv = kss + (size_t)nbl * N * kparts;    // [nbl][N]
     g += P.kss_b * nbl;
@@ -547,7 +594,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     float* qss = reinterpret_cast<float*>(g + a256((size_t)t * D * 4) * nbl);
     const float* qsrc = L.qhat;  // [.][t_max][D], batch index b0 + local
     int q_tmax = c.t_max, q_b0 = b0;
-    if (P.lazy_q) {
+    if (q_call) {
       // q~ = RMSNorm(Z) W_Q + b_Q (2-pass), as at weight load, for this group's (h, i) only
       GemmParams p = gp(t, ni * D, nh, 1);
       p.a_r1 = t;
@@ -561,7 +608,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.om.cdiv = D;
       e.om.c1 = (int64_t)t * D;
       e.om.c0 = 1;
-      e.bias = L.bq + (size_t)i0 * D;
+      e.bias = Bw.bq + (size_t)i0 * D;
       e.sumsq = qss;
       e.ssm.b1 = (int64_t)ni * t;
       e.ssm.r0 = 1;
@@ -570,8 +617,8 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.ss_parts = 2 * (D / 256);
       e.ss_block = t;
       e.vec_ok = 1;
-      TRY(run_gemm256<STILL_K_LOAD>(ctx, op(Zn, (int64_t)H * t, 2 * D), op(L.WqT, (int64_t)n * D, D),
-                                    p, e, 1, s));
+      TRY(run_gemm256<STILL_K_LOAD>(ctx, op(Zn, (int64_t)H * t, 2 * D), op(Bw.WqT, (int64_t)n * D, D),
+                                    p, e, w_fmt, s));
       const int64_t nq = (int64_t)nbl * t;
       float* qinv = qss + nq * (2 * (D / 256));
       KLAUNCH(STILL_K_NORMS, launch_inv_norms(qss, nq, 2 * (D / 256), t, c.l2_eps, 1.f, qinv, s));
@@ -587,25 +634,42 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       p.n_fast = 1;  // X rows of a KV-head can exceed L2; the W_K block fits
       add_pass(p, 0, 0, (int)(h0 * N), i0 * D, 2 * d);
       add_pass(p, 2 * d, 0, (int)(h0 * N), i0 * D, d);
-      EpiRopeC e;
-      e.out = kb;
-      e.sumsq = kss;
-      e.bias = L.bk + (size_t)i0 * D;
-      e.coarse = coarse;
-      e.omega = omega;
-      e.gd = gd;
-      e.D = D;
-      e.nheads = ni;
-      e.ncoarse = P.G;
-      e.Ntok = N;
+      auto fill = [&](auto& e) {
+        e.out = kb;
+        e.sumsq = kss;
+        e.bias = Bw.bk + (size_t)i0 * D;
+        e.coarse = coarse;
+        e.fine = coarse + (size_t)P.G * (D / 2);
+        e.omega = omega;
+        e.gd = gd;
+        e.D = D;
+        e.nheads = ni;
+        e.ncoarse = P.G;
+        e.fp16 = exact ? 1 : 0;  // k as fp16 hi / lo where the block feeds another
+        e.Ntok = N;
+      };
       const StoreView3D kv = store_view(kb, 2, 2 * D, N, nbl, 2 * D, N * 2 * D, 16, false);
-      TRY(run_gemm256<STILL_K_KEYPROJ>(ctx, op(X, (int64_t)H * N, 3 * d), op(L.WkT, (int64_t)n * D, 2 * d), p, e,
-                   1, s, &kv));
+      const Operand2D xop = op(X, (int64_t)H * N, 3 * d);
+      const Operand2D wop = op(Bw.WkT, (int64_t)n * D, 2 * d);
+      if (pos.frac) {
+        EpiRopeCT<true> e;
+        fill(e);
+        TRY(run_gemm256<STILL_K_KEYPROJ>(ctx, xop, wop, p, e, w_fmt, s, &kv));
+      } else {
+        EpiRopeCT<false> e;
+        fill(e);
+        TRY(run_gemm256<STILL_K_KEYPROJ>(ctx, xop, wop, p, e, w_fmt, s, &kv));
+      }
     }
     // scale / |k~_n| per key (the d_l logit scale folded in)
-    KLAUNCH(STILL_K_NORMS, launch_inv_norms(kss, (int64_t)nbl * N, kparts, N, c.l2_eps, scale, kinv, s));
+    // A block that feeds another forms q and k as fp16 hi / lo (about 22 bits; bf16 hi / lo
+    // keeps 16): its logits steer the next block's queries. q is unit-norm, so it is scaled by
+    // a power of two near sqrt(D) into the fp16 normal range and the logit scale divided by it.
+    const float qscale = exact ? std::exp2(std::round(0.5 * std::log2((double)D))) : 1.f;
+    KLAUNCH(STILL_K_NORMS, launch_inv_norms(kss, (int64_t)nbl * N, kparts, N, c.l2_eps,
+                                            scale / qscale, kinv, s));
     KLAUNCH(STILL_K_QROPE, launch_q_rope(qsrc, q_tmax, q_b0, nbl, t, D, qstart, qstep, L.omega_c,
-                                         c.compactor_rope, qhl, s));
+                                         c.compactor_rope, qhl, exact ? 1 : 0, qscale, s));
     if (P.flash) {
       // S, the online softmax and P X in one kernel; per-split partials merged in order.
       float2* fst = stp;  // [nsplit][nbl * t] (the statistics region of this path)
@@ -661,8 +725,8 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.stat_out = stp;
       e.stat_slots = stat_slots;
       const StoreView3D sv = store_view(S, 4, N, t, nbl, P.ldS, (int64_t)t * P.ldS, 32, true);
-      TRY(run_gemm256<STILL_K_SCORES>(ctx, op(qhl, (int64_t)nbl * t, 2 * D), op(kb, (int64_t)nbl * N, 2 * D), p,
-                   e, 1, s, &sv));
+      TRY(run_gemm256<STILL_K_SCORES>(ctx, op(qhl, (int64_t)nbl * t, 2 * D),
+                                      op(kb, (int64_t)nbl * N, 2 * D), p, e, exact ? 0 : 1, s, &sv));
     }
     KLAUNCH(STILL_K_SOFTMAX, launch_row_stats(stp, (int64_t)nbl * t, stat_slots, rstat, s));
     int px_split = 1;
@@ -670,7 +734,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     {  // O = softmax(S) X: probabilities formed on the fly (fp16), X hi + key-half lo passes
       GemmParams p = gp(t, 2 * d, nbl, ni);
       add_pass(p, 0, 0, 0, 0, (int)Np);
-      const int bn = 256;
+      const int bn = 2 * d <= 128 ? 128 : 256;
       const int64_t tiles = (int64_t)((t + 127) / 128) * ((2 * d + bn - 1) / bn) * nbl;
       p.ksplit = std::min(auto_split(tiles, (int)(Np / 64), ctx->nsm), kMaxSplit);
       p.ksplit = std::min(p.ksplit, (int)(Np / 64));
@@ -697,10 +761,15 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.om.r0 = 2 * d;
       e.om.c0 = 1;
       const Operand2D xt = op(XT, (int64_t)H * 2 * d, 2 * Np);
-      // This path serves 2d = 512 (smaller heads take the fused kernel).
-      if (d != 256) return STILL_ERR_UNSUPPORTED;
+      // Split probabilities (hi + lo) in a block whose output enters another block.
       ctx->prof.begin(STILL_K_PX, s);
-      cudaError_t r = launch_px_fused<256, 256>(xt, p, px, e, ctx->nsm, s);
+      cudaError_t r =
+          d == 64    ? (exact ? launch_px_fused<128, 64, true>(xt, p, px, e, ctx->nsm, s)
+                              : launch_px_fused<128, 64>(xt, p, px, e, ctx->nsm, s))
+          : d == 128 ? (exact ? launch_px_fused<256, 128, true>(xt, p, px, e, ctx->nsm, s)
+                              : launch_px_fused<256, 128>(xt, p, px, e, ctx->nsm, s))
+                     : (exact ? launch_px_fused<256, 256, true>(xt, p, px, e, ctx->nsm, s)
+                              : launch_px_fused<256, 256>(xt, p, px, e, ctx->nsm, s));
       ctx->prof.end(STILL_K_PX, s);
       if (r == cudaErrorInvalidValue) return STILL_ERR_INVALID_ARG;
       if (r != cudaSuccess) return STILL_ERR_CUDA;
@@ -710,8 +779,6 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
   }
 
   // ---------------------------------------------------------------- Z' = Z + PX W_VO
-  const int64_t rows = (int64_t)H * t;
-  const int n2d = n * 2 * d;
   {
     GemmParams p = gp((int)rows, D);
     add_pass(p, 0, 0, 0, 0, n2d);
@@ -722,16 +789,25 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     e.out = Z1;
     e.om.r0 = D;
     e.om.c0 = 1;
-    e.res_kind = 2;
-    e.res = L.Z;
-    e.resm.rdiv = t;
-    e.resm.r1 = (int64_t)c.t_max * D;
-    e.resm.r0 = D;
-    e.resm.c0 = 1;
+    if (bi == 0) {  // the latent bank rows [0, t) of each KV-head (bf16)
+      e.res_kind = 2;
+      e.res = L.Z;
+      e.resm.rdiv = t;
+      e.resm.r1 = (int64_t)c.t_max * D;
+      e.resm.r0 = D;
+      e.resm.c0 = 1;
+    } else {  // the previous block's fp32 state
+      e.res_kind = 1;
+      e.res = Z2;
+      e.resm.r0 = D;
+      e.resm.c0 = 1;
+    }
     e.vec_ok = 1;
-    TRY(run_gemm256<STILL_K_VO>(ctx, op(PX, rows, 2 * n2d), op(L.WvoT, D, 2 * n2d), p, e, 1, s));
+    TRY(run_gemm256<STILL_K_VO>(ctx, op(PX, rows, 2 * n2d), op(Bw.WvoT, D, 2 * n2d), p, e, 1, s));
   }
-  KLAUNCH(STILL_K_NORM, launch_rmsnorm(Z1, 0, rows, D, D, c.rms_eps, A1, 2 * D, 1, s));
+  Za = Z1;
+  }  // cross-attention of block bi
+  KLAUNCH(STILL_K_NORM, launch_rmsnorm(Za, 0, rows, D, D, c.rms_eps, A1, 2 * D, 1, s));
 
   // ---------------------------------------------------------------- latent self-attention
   for (int h0 = 0; h0 < H; h0 += P.sa_heads) {
@@ -765,7 +841,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.om.cdiv = D;
       e.om.c1 = (int64_t)t * 2 * D;
       e.om.c0 = 1;
-      e.bias = L.sbqk;
+      e.bias = Bw.sbqk;
       e.sumsq = sss;
       e.ssm.rdiv = t;
       e.ssm.r1 = (int64_t)2 * n * t;
@@ -775,22 +851,24 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.ss_parts = sparts;
       e.ss_block = t;
       e.vec_ok = 1;
-      TRY(run_gemm256<STILL_K_SA_PROJ>(ctx, op(A1, rows, 2 * D), op(L.SqkT, (int64_t)2 * n * D, D), p, e, 1, s));
+      TRY(run_gemm256<STILL_K_SA_PROJ>(ctx, op(A1, rows, 2 * D), op(Bw.SqkT, (int64_t)2 * n * D, D), p, e, 1, s));
     }
     KLAUNCH(STILL_K_NORMS,
             launch_inv_norms(sss, (int64_t)nh * 2 * n * t, sparts, t, c.l2_eps, 1.f, sinv, s));
-    {  // v^T = S_V^T RMSNorm(Z')^T  -> [nD][nh * tp]
+    {  // v^T = S_V^T RMSNorm(Z')^T  -> [nD][nh * tp]  (hi, then lo rows when exact)
       GemmParams p = gp(n * D, nh * t);
       add_pass(p, 0, 0, 0, h0 * t, D);
+      if (exact) add_pass(p, 0, D, 0, h0 * t, D);
       EpiAffine e;
-      e.kind = OUT_BF16;
+      e.kind = exact ? OUT_HILO : OUT_BF16;
+      e.lo_off = (int64_t)n * D * nh * P.tp;
       e.out = vT;
       e.om.r0 = (int64_t)nh * P.tp;
       e.om.cdiv = t;
       e.om.c1 = P.tp;
       e.om.c0 = 1;
       e.vec_ok = (t % 32 == 0);
-      TRY(run_gemm256<STILL_K_SA_V>(ctx, op(L.SvT, (int64_t)n * D, D), op(A1, rows, 2 * D), p, e, 1, s));
+      TRY(run_gemm256<STILL_K_SA_V>(ctx, op(Bw.SvT, (int64_t)n * D, D), op(A1, rows, 2 * D), p, e, 1, s));
     }
     // Self heads [i0, i0 + ns) of the nh banks per pass (all n unless one bank is too big).
     for (int i0 = 0; i0 < n; i0 += P.sa_sub) {
@@ -831,70 +909,85 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
                                            op(qk, (int64_t)nh * 2 * n * t, 2 * D), p, e, 1, s, &sv));
       }
       KLAUNCH(STILL_K_SA_SOFTMAX,
-              launch_softmax(Ssa, (int64_t)nh * ns * t, t, P.ldt, Psa, P.tp, 0, s));
+              launch_softmax(Ssa, (int64_t)nh * ns * t, t, P.ldt, Psa, P.tp, exact ? 2 : 0, s));
       {  // heads = P v -> concat rows (h0 + hh) * t + j, columns (i0 + bi) * D + f
+        // exact: P_hi v_hi + P_hi v_lo + P_lo v_hi, concat rows of hi | lo
+        const int64_t cw = exact ? 2 * (int64_t)n * D : (int64_t)n * D;  // concat row pitch
         GemmParams p = gp(t, D, nh * ns, ns);
         p.a_r1 = (int64_t)ns * t;
         p.a_r0 = t;
         p.b_r0 = D;
         p.b_k1 = P.tp;
         add_pass(p, 0, 0, 0, i0 * D, (int)P.tp);
+        if (exact) {
+          add_pass(p, 0, 0, 0, n * D + i0 * D, (int)P.tp);
+          add_pass(p, (int)P.tp, 0, 0, i0 * D, (int)P.tp);
+        }
         EpiAffine e;
-        e.kind = OUT_BF16;
+        e.kind = exact ? OUT_HILO : OUT_BF16;
+        e.lo_off = (int64_t)n * D;
         e.out = cat;
         e.om.bdiv = ns;
-        e.om.b1 = (int64_t)t * n * D;
+        e.om.b1 = (int64_t)t * cw;
         e.om.b0 = D;
-        e.om.r0 = (int64_t)n * D;
+        e.om.r0 = cw;
         e.om.c0 = 1;
-        e.om.k = (int64_t)h0 * t * n * D + (int64_t)i0 * D;
+        e.om.k = (int64_t)h0 * t * cw + (int64_t)i0 * D;
         e.vec_ok = 1;
-        TRY(run_gemm256<STILL_K_SA_PV>(ctx, op(Psa, (int64_t)nh * ns * t, P.tp),
-                                       op(vT, (int64_t)n * D, (int64_t)nh * P.tp), p, e, 1, s));
+        TRY(run_gemm256<STILL_K_SA_PV>(
+            ctx, op(Psa, (int64_t)nh * ns * t, exact ? 2 * P.tp : P.tp),
+            op(vT, (exact ? 2 : 1) * (int64_t)n * D, (int64_t)nh * P.tp), p, e, 1, s));
       }
     }
   }
-  const bool z3_bf16 = (c.final_norm == 0);
-  {  // Z'' = Z' + concat S_O
+  {  // Z'' = Z' + concat S_O  (exact: concat hi | lo, 2 passes)
     GemmParams p = gp((int)rows, D);
     add_pass(p, 0, 0, 0, 0, n * D);
+    if (exact) add_pass(p, n * D, 0, 0, 0, n * D);
     EpiAffine e;
-    const bool direct = (F == 0) && z3_bf16;
+    const bool direct = last && (F == 0) && z3_bf16;
     e.kind = direct ? OUT_HILO : OUT_F32;
     e.out = direct ? Z3 : static_cast<void*>(Z2);
     e.lo_off = D;
     e.om.r0 = direct ? 2 * D : D;
     e.om.c0 = 1;
     e.res_kind = 1;
-    e.res = Z1;
+    e.res = Za;  // in place when the block has no cross-attention (Za = Z2): same thread
     e.resm.r0 = D;
     e.resm.c0 = 1;
     e.vec_ok = 1;
-    TRY(run_gemm256<STILL_K_SO>(ctx, op(cat, rows, (int64_t)n * D), op(L.SoT, D, (int64_t)n * D), p, e, 1,
-                 s));
+    TRY(run_gemm256<STILL_K_SO>(ctx, op(cat, rows, (exact ? 2 : 1) * (int64_t)n * D),
+                                op(Bw.SoT, D, (int64_t)n * D), p, e, 1, s));
   }
   if (F > 0) {
-    KLAUNCH(STILL_K_NORM, launch_rmsnorm(Z2, 0, rows, D, D, c.rms_eps, A2, D, 0, s));
+    // exact: RMSNorm(Z'') and GELU(.) as hi | lo, both products in 2 passes
+    KLAUNCH(STILL_K_NORM, launch_rmsnorm(Z2, 0, rows, D, D, c.rms_eps, A2, exact ? 2 * D : D,
+                                         exact ? 1 : 0, s));
     {
       GemmParams p = gp((int)rows, F);
       add_pass(p, 0, 0, 0, 0, D);
+      if (exact) add_pass(p, D, 0, 0, 0, D);
       EpiAffine e;
-      e.kind = OUT_BF16;
+      e.kind = exact ? OUT_HILO : OUT_BF16;
+      e.lo_off = F;
       e.out = Gb;
-      e.om.r0 = F;
+      e.om.r0 = exact ? 2 * F : F;
       e.om.c0 = 1;
       e.gelu = 1;
       e.vec_ok = 1;
-      TRY(run_gemm256<STILL_K_FFN1>(ctx, op(A2, rows, D), op(L.W1T, F, D), p, e, 1, s));
+      TRY(run_gemm256<STILL_K_FFN1>(ctx, op(A2, rows, exact ? 2 * D : D), op(Bw.W1T, F, D), p, e,
+                                    1, s));
     }
     {
       GemmParams p = gp((int)rows, D);
       add_pass(p, 0, 0, 0, 0, F);
+      if (exact) add_pass(p, F, 0, 0, 0, F);
       EpiAffine e;
-      e.kind = z3_bf16 ? OUT_HILO : OUT_F32;
-      e.out = z3_bf16 ? Z3 : static_cast<void*>(Z2);
+      const bool direct = last && z3_bf16;
+      e.kind = direct ? OUT_HILO : OUT_F32;
+      e.out = direct ? Z3 : static_cast<void*>(Z2);
       e.lo_off = D;
-      e.om.r0 = z3_bf16 ? 2 * D : D;
+      e.om.r0 = direct ? 2 * D : D;
       e.om.c0 = 1;
       e.res_kind = 1;
       e.res = Z2;
@@ -902,9 +995,11 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.resm.c0 = 1;
       e.vec_ok = 1;
       // In place (Z2 -> Z2) is safe: each element is read and written by the same thread.
-      TRY(run_gemm256<STILL_K_FFN2>(ctx, op(Gb, rows, F), op(L.W2T, D, F), p, e, 1, s));
+      TRY(run_gemm256<STILL_K_FFN2>(ctx, op(Gb, rows, exact ? 2 * F : F), op(Bw.W2T, D, F), p, e,
+                                    1, s));
     }
   }
+  }  // block bi
   if (!z3_bf16) {
     KLAUNCH(STILL_K_NORM, launch_rmsnorm(Z2, 0, rows, D, D, c.rms_eps, reinterpret_cast<bf16*>(Z3), 2 * D, 1, s));
   }
@@ -941,6 +1036,173 @@ still_status check_ctx_layer(still_ctx* ctx, int32_t layer, const LayerW** L) {
   if (layer < 0 || layer >= (int32_t)ctx->layers.size() || !ctx->layers[layer].loaded)
     return STILL_ERR_NOT_LOADED;
   *L = &ctx->layers[layer];
+  return STILL_OK;
+}
+
+// Loads one layer: latent banks, per-block weights, output heads (App. A). Block 0's latent
+// queries are precomputed when they fit the eager limit; later blocks' queries depend on the
+// latent state and are formed in each call, so their W_Q and b_Q are kept.
+still_status load_layer(still_ctx* ctx, int32_t layer, const still_layer_config* cfg,
+                        const void* Zsrc, const still_block_weights* blocks, const void* Wkey,
+                        const void* Wval, void* stream) {
+  if (ctx == nullptr || layer < 0 || Zsrc == nullptr || blocks == nullptr || Wkey == nullptr ||
+      Wval == nullptr)
+    return STILL_ERR_INVALID_ARG;
+  TRY(check_cfg(cfg));
+  const still_layer_config& c = *cfg;
+  const int H = c.n_kv_heads, d = c.head_dim, D = c.d_latent, n = c.n_cross_heads,
+            F = c.ffn_dim, T = c.t_max, NB = c.n_blocks;
+  for (int b = 0; b < NB; ++b) {
+    const still_block_weights& w = blocks[b];
+    const bool ca = b == 0 || c.cross_every_block;
+    const void* req_ca[] = {w.Wq, w.bq, w.Wk, w.bk, w.Wv, w.Wo};
+    const void* req_sa[] = {w.Sq, w.sbq, w.Sk, w.sbk, w.Sv, w.So};
+    if (ca)
+      for (const void* p : req_ca)
+        if (p == nullptr) return STILL_ERR_INVALID_ARG;
+    for (const void* p : req_sa)
+      if (p == nullptr) return STILL_ERR_INVALID_ARG;
+    if (F > 0 && (w.W1 == nullptr || w.W2 == nullptr)) return STILL_ERR_INVALID_ARG;
+  }
+  CK(cudaSetDevice(ctx->device));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if ((int32_t)ctx->layers.size() <= layer) ctx->layers.resize(layer + 1);
+  LayerW& L = ctx->layers[layer];
+  if (L.loaded) {
+    CK(cudaStreamSynchronize(s));
+    free_layer(L);
+  }
+  L.cfg = c;
+  if (L.cfg.logit_scale == 0) L.cfg.logit_scale = D;
+  const int64_t nD = (int64_t)n * D;
+  L.blk.resize(NB);
+  L.qhat_lazy = (size_t)H * n * T * D * sizeof(float) > ctx->qhat_eager_limit;
+  L.f16 = NB > 1;
+  auto fail = [&](still_status st) {
+    cudaStreamSynchronize(s);
+    free_layer(L);
+    return st;
+  };
+  still_status st = STILL_OK;
+  // ---- layer-level tensors
+  if ((st = dalloc(L, &L.Z, (size_t)H * T * D)) != STILL_OK ||
+      (st = dalloc(L, &L.WhT, (size_t)2 * d * D)) != STILL_OK ||
+      (st = dalloc(L, &L.omega_b, (size_t)d / 2)) != STILL_OK ||
+      (st = dalloc(L, &L.omega_c, (size_t)D / 2)) != STILL_OK ||
+      (!L.qhat_lazy && (st = dalloc(L, &L.qhat, (size_t)H * n * T * D)) != STILL_OK))
+    return fail(st);
+  if (launch_omega(L.omega_b, d / 2, d, c.rope_theta, s) != cudaSuccess ||
+      launch_omega(L.omega_c, D / 2, D, c.rope_theta_compactor, s) != cudaSuccess ||
+      cudaMemcpyAsync(L.Z, Zsrc, sizeof(bf16) * (size_t)H * T * D, cudaMemcpyDeviceToDevice, s) !=
+          cudaSuccess ||
+      launch_transpose(static_cast<const bf16*>(Wkey), D, d, L.WhT, 0, s) != cudaSuccess ||
+      launch_transpose(static_cast<const bf16*>(Wval), D, d, L.WhT + (size_t)d * D, 0, s) !=
+          cudaSuccess)
+    return fail(STILL_ERR_CUDA);
+
+  // ---- per-block tensors
+  LayerW tmp;  // temporaries of the precompute
+  auto body = [&]() -> still_status {
+    for (int b = 0; b < NB; ++b) {
+      const still_block_weights& w = blocks[b];
+      BlockW& B = L.blk[b];
+      B.has_ca = b == 0 || c.cross_every_block;
+      TRY(dalloc(L, &B.SqkT, (size_t)2 * nD * D));
+      TRY(dalloc(L, &B.sbqk, (size_t)2 * nD));
+      TRY(dalloc(L, &B.SvT, (size_t)nD * D));
+      TRY(dalloc(L, &B.SoT, (size_t)D * nD));
+      CK(launch_transpose(static_cast<const bf16*>(w.Sq), D, nD, B.SqkT, 0, s));
+      CK(launch_transpose(static_cast<const bf16*>(w.Sk), D, nD, B.SqkT + nD * D, 0, s));
+      CK(launch_bias(static_cast<const bf16*>(w.sbq), static_cast<const bf16*>(w.sbk), nD, B.sbqk,
+                     0, s));
+      CK(launch_transpose(static_cast<const bf16*>(w.Sv), D, nD, B.SvT, 0, s));
+      CK(launch_transpose(static_cast<const bf16*>(w.So), nD, D, B.SoT, 0, s));
+      if (F > 0) {
+        TRY(dalloc(L, &B.W1T, (size_t)F * D));
+        TRY(dalloc(L, &B.W2T, (size_t)D * F));
+        CK(launch_transpose(static_cast<const bf16*>(w.W1), D, F, B.W1T, 0, s));
+        CK(launch_transpose(static_cast<const bf16*>(w.W2), F, D, B.W2T, 0, s));
+      }
+      if (!B.has_ca) continue;
+      TRY(dalloc(L, &B.WkT, (size_t)nD * 2 * d));
+      TRY(dalloc(L, &B.bk, (size_t)nD));
+      TRY(dalloc(L, &B.WvoT, (size_t)D * 2 * n * 2 * d));
+      CK(launch_transpose(static_cast<const bf16*>(w.Wk), 2 * d, nD, B.WkT, D, s));
+      if (L.f16) CK(launch_bf16_to_f16(B.WkT, (int64_t)nD * 2 * d, s));
+      CK(launch_bias(static_cast<const bf16*>(w.bk), nullptr, nD, B.bk, D, s));
+      // W_Q and b_Q: kept when the block's queries are formed per call, else temporaries.
+      const bool keep_q = b > 0 || L.qhat_lazy;
+      LayerW& qown = keep_q ? L : tmp;
+      bf16* WqT = nullptr;
+      float* bq = nullptr;
+      TRY(dalloc(qown, &WqT, (size_t)nD * D));
+      TRY(dalloc(qown, &bq, (size_t)nD));
+      CK(launch_transpose(static_cast<const bf16*>(w.Wq), D, nD, WqT, D, s));
+      if (L.f16) CK(launch_bf16_to_f16(WqT, (int64_t)nD * D, s));
+      CK(launch_bias(static_cast<const bf16*>(w.bq), nullptr, nD, bq, D, s));
+      if (keep_q) {
+        B.WqT = WqT;
+        B.bq = bq;
+      } else {  // q~ = RMSNorm(Z) W_Q + b_Q  (2-pass), |q~|^2 per (row, head), then L2 norm
+        bf16* Zn = nullptr;
+        float* qss = nullptr;
+        TRY(dalloc(tmp, &Zn, (size_t)H * T * 2 * D));
+        TRY(dalloc(tmp, &qss, (size_t)H * n * T * (2 * (D / 256) + 1)));
+        CK(launch_rmsnorm(Zsrc, 1, (int64_t)H * T, D, D, c.rms_eps, Zn, 2 * D, L.f16 ? 2 : 1, s));
+        GemmParams p = gp(H * T, (int)nD);
+        add_pass(p, 0, 0, 0, 0, D);
+        add_pass(p, D, 0, 0, 0, D);
+        EpiAffine e;
+        e.kind = OUT_F32;
+        e.out = L.qhat;
+        e.om.rdiv = T;
+        e.om.r1 = (int64_t)n * T * D;
+        e.om.r0 = D;
+        e.om.cdiv = D;
+        e.om.c1 = (int64_t)T * D;
+        e.om.c0 = 1;
+        e.bias = bq;
+        e.sumsq = qss;
+        e.ssm.rdiv = T;
+        e.ssm.r1 = (int64_t)n * T;
+        e.ssm.r0 = 1;
+        e.ssm.c0 = T;
+        e.ss_seg = D;
+        e.ss_parts = 2 * (D / 256);
+        e.ss_block = T;
+        e.vec_ok = 1;
+        TRY(run_gemm256<STILL_K_LOAD>(ctx, op(Zn, (int64_t)H * T, 2 * D), op(WqT, nD, D), p, e,
+                                      L.f16 ? 0 : 1, s));
+        const int64_t nq = (int64_t)H * n * T;
+        float* qinv = qss + nq * (2 * (D / 256));
+        CK(launch_inv_norms(qss, nq, 2 * (D / 256), T, c.l2_eps, 1.f, qinv, s));
+        CK(launch_scale_rows(L.qhat, qinv, nq, D, s));
+      }
+      // W_VO,i = W_V,i W_O,i  -> stored transposed as hi | lo: WvoT[c][i*2d + f]
+      bf16* WoT = nullptr;
+      TRY(dalloc(tmp, &WoT, (size_t)D * nD));
+      CK(launch_transpose(static_cast<const bf16*>(w.Wo), nD, D, WoT, 0, s));
+      GemmParams p = gp(2 * d, D, n, 1);
+      p.a_k1 = D;
+      p.b_k1 = D;
+      add_pass(p, 0, 0, 0, 0, D);
+      EpiAffine e;
+      e.kind = OUT_HILO;
+      e.out = B.WvoT;
+      e.lo_off = (int64_t)n * 2 * d;
+      e.om.b1 = 2 * d;
+      e.om.r0 = 1;
+      e.om.c0 = (int64_t)2 * n * 2 * d;
+      e.vec_ok = 0;
+      TRY(run_gemm256<STILL_K_LOAD>(ctx, op(w.Wv, 2 * d, nD), op(WoT, D, nD), p, e, 1, s));
+    }
+    return STILL_OK;
+  };
+  st = body();
+  cudaStreamSynchronize(s);
+  free_layer(tmp);
+  if (st != STILL_OK) return fail(st);
+  L.loaded = true;
   return STILL_OK;
 }
 
@@ -1048,150 +1310,18 @@ still_status still_set_workspace_limit(still_ctx* ctx, size_t bytes) {
 still_status still_load_layer_weights(still_ctx* ctx, int32_t layer,
                                       const still_layer_config* cfg,
                                       const still_layer_weights* w, void* stream) {
-  if (ctx == nullptr || w == nullptr || layer < 0) return STILL_ERR_INVALID_ARG;
-  TRY(check_cfg(cfg));
-  const still_layer_config& c = *cfg;
-  const int H = c.n_kv_heads, d = c.head_dim, D = c.d_latent, n = c.n_cross_heads,
-            F = c.ffn_dim, T = c.t_max;
-  const void* req[] = {w->Z, w->Wq, w->bq, w->Wk, w->bk, w->Wv, w->Wo, w->Sq,
-                       w->sbq, w->Sk, w->sbk, w->Sv, w->So, w->Wkey, w->Wval};
-  for (const void* p : req)
-    if (p == nullptr) return STILL_ERR_INVALID_ARG;
-  if (F > 0 && (w->W1 == nullptr || w->W2 == nullptr)) return STILL_ERR_INVALID_ARG;
-  CK(cudaSetDevice(ctx->device));
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if ((int32_t)ctx->layers.size() <= layer) ctx->layers.resize(layer + 1);
-  LayerW& L = ctx->layers[layer];
-  if (L.loaded) {
-    CK(cudaStreamSynchronize(s));
-    free_layer(L);
-  }
-  L.cfg = c;
-  if (L.cfg.logit_scale == 0) L.cfg.logit_scale = D;
-  const int64_t nD = (int64_t)n * D;
-  const bf16* Wq = static_cast<const bf16*>(w->Wq);
-  TRY(dalloc(L, &L.Z, (size_t)H * T * D));
-  TRY(dalloc(L, &L.WkT, (size_t)nD * 2 * d));
-  TRY(dalloc(L, &L.bk, (size_t)nD));
-  L.qhat_lazy = (size_t)H * n * T * D * sizeof(float) > ctx->qhat_eager_limit;
-  if (!L.qhat_lazy) TRY(dalloc(L, &L.qhat, (size_t)H * n * T * D));
-  TRY(dalloc(L, &L.WvoT, (size_t)D * 2 * n * 2 * d));
-  TRY(dalloc(L, &L.SqkT, (size_t)2 * nD * D));
-  TRY(dalloc(L, &L.sbqk, (size_t)2 * nD));
-  TRY(dalloc(L, &L.SvT, (size_t)nD * D));
-  TRY(dalloc(L, &L.SoT, (size_t)D * nD));
-  if (F > 0) {
-    TRY(dalloc(L, &L.W1T, (size_t)F * D));
-    TRY(dalloc(L, &L.W2T, (size_t)D * F));
-  }
-  TRY(dalloc(L, &L.WhT, (size_t)2 * d * D));
-  TRY(dalloc(L, &L.omega_b, (size_t)d / 2));
-  TRY(dalloc(L, &L.omega_c, (size_t)D / 2));
-  CK(launch_omega(L.omega_b, d / 2, d, c.rope_theta, s));
-  CK(launch_omega(L.omega_c, D / 2, D, c.rope_theta_compactor, s));
-  CK(cudaMemcpyAsync(L.Z, w->Z, sizeof(bf16) * (size_t)H * T * D, cudaMemcpyDeviceToDevice, s));
-  CK(launch_transpose(static_cast<const bf16*>(w->Wk), 2 * d, nD, L.WkT, D, s));
-  CK(launch_bias(static_cast<const bf16*>(w->bk), nullptr, nD, L.bk, D, s));
-  CK(launch_transpose(static_cast<const bf16*>(w->Sq), D, nD, L.SqkT, 0, s));
-  CK(launch_transpose(static_cast<const bf16*>(w->Sk), D, nD, L.SqkT + nD * D, 0, s));
-  CK(launch_bias(static_cast<const bf16*>(w->sbq), static_cast<const bf16*>(w->sbk), nD, L.sbqk,
-                 0, s));
-  CK(launch_transpose(static_cast<const bf16*>(w->Sv), D, nD, L.SvT, 0, s));
-  CK(launch_transpose(static_cast<const bf16*>(w->So), nD, D, L.SoT, 0, s));
-  if (F > 0) {
-    CK(launch_transpose(static_cast<const bf16*>(w->W1), D, F, L.W1T, 0, s));
-    CK(launch_transpose(static_cast<const bf16*>(w->W2), F, D, L.W2T, 0, s));
-  }
-  CK(launch_transpose(static_cast<const bf16*>(w->Wkey), D, d, L.WhT, 0, s));
-  CK(launch_transpose(static_cast<const bf16*>(w->Wval), D, d, L.WhT + (size_t)d * D, 0, s));
+  if (w == nullptr) return STILL_ERR_INVALID_ARG;
+  if (cfg != nullptr && cfg->n_blocks != 1) return STILL_ERR_INVALID_ARG;
+  const still_block_weights blk = {w->Wq, w->bq, w->Wk, w->bk, w->Wv, w->Wo, w->Sq,
+                                   w->sbq, w->Sk, w->sbk, w->Sv, w->So, w->W1, w->W2};
+  return load_layer(ctx, layer, cfg, w->Z, &blk, w->Wkey, w->Wval, stream);
+}
 
-  // Temporaries for the precompute.
-  LayerW tmp;
-  bf16 *WqT = nullptr, *Zn = nullptr, *WoT = nullptr;
-  float *bq = nullptr, *qss = nullptr;
-  auto cleanup = [&]() {
-    cudaStreamSynchronize(s);
-    free_layer(tmp);
-  };
-  still_status st = STILL_OK;
-  // W_Q and b_Q are kept with the layer when q^ is formed per call, else temporaries.
-  LayerW& qown = L.qhat_lazy ? L : tmp;
-  if ((st = dalloc(qown, &WqT, (size_t)nD * D)) != STILL_OK ||
-      (st = dalloc(qown, &bq, (size_t)nD)) != STILL_OK ||
-      (st = dalloc(tmp, &WoT, (size_t)D * nD)) != STILL_OK ||
-      (!L.qhat_lazy && (st = dalloc(tmp, &Zn, (size_t)H * T * 2 * D)) != STILL_OK) ||
-      (!L.qhat_lazy &&
-       (st = dalloc(tmp, &qss, (size_t)H * n * T * (2 * (D / 256) + 1))) != STILL_OK)) {
-    cleanup();
-    free_layer(L);
-    return st;
-  }
-  auto body = [&]() -> still_status {
-    CK(launch_transpose(Wq, D, nD, WqT, D, s));
-    CK(launch_bias(static_cast<const bf16*>(w->bq), nullptr, nD, bq, D, s));
-    if (L.qhat_lazy) {
-      L.WqT = WqT;
-      L.bq = bq;
-    }
-    if (!L.qhat_lazy) CK(launch_rmsnorm(w->Z, 1, (int64_t)H * T, D, D, c.rms_eps, Zn, 2 * D, 1, s));
-    if (!L.qhat_lazy) {  // q~ = RMSNorm(Z) W_Q + b_Q  (2-pass), |q~|^2 per (row, head)
-      GemmParams p = gp(H * T, (int)nD);
-      add_pass(p, 0, 0, 0, 0, D);
-      add_pass(p, D, 0, 0, 0, D);
-      EpiAffine e;
-      e.kind = OUT_F32;
-      e.out = L.qhat;
-      e.om.rdiv = T;
-      e.om.r1 = (int64_t)n * T * D;
-      e.om.r0 = D;
-      e.om.cdiv = D;
-      e.om.c1 = (int64_t)T * D;
-      e.om.c0 = 1;
-      e.bias = bq;
-      e.sumsq = qss;
-      e.ssm.rdiv = T;
-      e.ssm.r1 = (int64_t)n * T;
-      e.ssm.r0 = 1;
-      e.ssm.c0 = T;
-      e.ss_seg = D;
-      e.ss_parts = 2 * (D / 256);
-      e.ss_block = T;
-      e.vec_ok = 1;
-      TRY(run_gemm256<STILL_K_LOAD>(ctx, op(Zn, (int64_t)H * T, 2 * D), op(WqT, nD, D), p, e, 1, s));
-    }
-    if (!L.qhat_lazy) {
-      const int64_t nq = (int64_t)H * n * T;
-      float* qinv = qss + nq * (2 * (D / 256));
-      CK(launch_inv_norms(qss, nq, 2 * (D / 256), T, c.l2_eps, 1.f, qinv, s));
-      CK(launch_scale_rows(L.qhat, qinv, nq, D, s));
-    }
-    // W_VO,i = W_V,i W_O,i  -> stored transposed as hi | lo: WvoT[c][i*2d + f]
-    CK(launch_transpose(static_cast<const bf16*>(w->Wo), nD, D, WoT, 0, s));
-    {
-      GemmParams p = gp(2 * d, D, n, 1);
-      p.a_k1 = D;
-      p.b_k1 = D;
-      add_pass(p, 0, 0, 0, 0, D);
-      EpiAffine e;
-      e.kind = OUT_HILO;
-      e.out = L.WvoT;
-      e.lo_off = (int64_t)n * 2 * d;
-      e.om.b1 = 2 * d;
-      e.om.r0 = 1;
-      e.om.c0 = (int64_t)2 * n * 2 * d;
-      e.vec_ok = 0;
-      TRY(run_gemm256<STILL_K_LOAD>(ctx, op(w->Wv, 2 * d, nD), op(WoT, D, nD), p, e, 1, s));
-    }
-    return STILL_OK;
-  };
-  st = body();
-  cleanup();
-  if (st != STILL_OK) {
-    free_layer(L);
-    return st;
-  }
-  L.loaded = true;
-  return STILL_OK;
+still_status still_load_layer_weights_blocks(still_ctx* ctx, int32_t layer,
+                                             const still_layer_config* cfg, const void* Z,
+                                             const still_block_weights* blocks, const void* Wkey,
+                                             const void* Wval, void* stream) {
+  return load_layer(ctx, layer, cfg, Z, blocks, Wkey, Wval, stream);
 }
 
 still_status still_compact_layer(still_ctx* ctx, int32_t layer, const void* K, const void* V,
@@ -1244,7 +1374,7 @@ still_status still_compact_layer_noalloc(still_ctx* ctx, int32_t layer, const vo
   TRY(make_positions(h_segments, n_segments, N, pos));
   CK(cudaSetDevice(ctx->device));
   Plan P;
-  if (!make_plan(L->cfg, L->qhat_lazy, N, t, pos.pmin, pos.pmax, kNoAllocScratchBytes, P))
+  if (!make_plan(L->cfg, queries_per_call(*L), N, t, pos.pmin, pos.pmax, kNoAllocScratchBytes, P))
     return STILL_ERR_OOM;  // even the smallest grouping needs more than the fixed scratch
   uint8_t* scratch = nullptr;
   TRY(noalloc_scratch(ctx->device, &scratch));
@@ -1280,6 +1410,131 @@ still_status still_compact_stack(still_ctx* ctx, int32_t n_layers, const void* c
   for (int l = 0; l < n_layers; ++l)
     TRY(still_compact_layer(ctx, l, K[l], V[l], strides_kv, h_segments, n_segments, N, t, Ck[l],
                             Cv[l], h_out_pos_start, h_out_pos_step, h_pos_offset, stream));
+  return STILL_OK;
+}
+
+still_status still_compact_stack_masked(still_ctx* ctx, int32_t n_layers,
+                                        const uint8_t* h_compact_layer, const void* const* K,
+                                        const void* const* V, const int64_t strides_kv[3],
+                                        const still_pos_segment* h_segments, int32_t n_segments,
+                                        int64_t N, int32_t t, void* const* Ck, void* const* Cv,
+                                        double* h_out_pos_start, double* h_out_pos_step,
+                                        int64_t* h_pos_offset, void* stream) {
+  if (ctx == nullptr || h_compact_layer == nullptr || K == nullptr || V == nullptr ||
+      Ck == nullptr || Cv == nullptr || n_layers < 1)
+    return STILL_ERR_INVALID_ARG;
+  for (int l = 0; l < n_layers; ++l) {
+    if (!h_compact_layer[l]) continue;
+    const LayerW* L = nullptr;
+    TRY(check_ctx_layer(ctx, l, &L));
+  }
+  for (int l = 0; l < n_layers; ++l)
+    if (h_compact_layer[l])
+      TRY(still_compact_layer(ctx, l, K[l], V[l], strides_kv, h_segments, n_segments, N, t,
+                              Ck[l], Cv[l], h_out_pos_start, h_out_pos_step, h_pos_offset,
+                              stream));
+  return STILL_OK;
+}
+
+// ------------------------------------------------------------------ lookahead chunked schedule
+
+still_status still_lookahead_pass_info(int64_t k, int64_t c, int32_t t,
+                                       still_lookahead_pass* out) {
+  constexpr int64_t kExact = int64_t(1) << 53;  // positions stay exact in fp64
+  if (out == nullptr || k < 0 || c < 1 || t < 1) return STILL_ERR_INVALID_ARG;
+  if (c > kExact / t) return STILL_ERR_INVALID_ARG;
+  const int64_t ct = c * t;
+  if (k + 2 > kExact / ct) return STILL_ERR_INVALID_ARG;  // (k + 2) ct bounds every field
+  still_lookahead_pass r;
+  r.chunk_start = k * ct;
+  r.chunk_len = ct;
+  r.prefill_start = k == 0 ? 0 : (k + 1) * ct;
+  r.prefill_len = k == 0 ? 2 * ct : ct;
+  r.prefill_past = k == 0 ? 0 : (k + c) * (int64_t)t;
+  r.compact_row = k * t;
+  r.retained_after = (k + 1) * t + ct;
+  r.logical_after = (k + 2) * ct;
+  r.pos_offset_after = r.logical_after - r.retained_after;
+  *out = r;
+  return STILL_OK;
+}
+
+still_status still_lookahead_totals(int64_t T, int64_t c, int32_t t, int64_t* h_passes,
+                                    int64_t* h_retained) {
+  if (h_passes == nullptr || h_retained == nullptr || c < 1 || t < 1 || T < 1)
+    return STILL_ERR_INVALID_ARG;
+  if (c > (int64_t(1) << 53) / t) return STILL_ERR_INVALID_ARG;
+  const int64_t ct = c * t;
+  if (T % ct != 0) return STILL_ERR_SHAPE;
+  still_lookahead_pass last;
+  TRY(still_lookahead_pass_info(T / ct - 1, c, t, &last));
+  *h_passes = T / ct;
+  *h_retained = last.retained_after;
+  return STILL_OK;
+}
+
+namespace {
+
+// Packed-chunk ragged arguments of one lookahead step: sequence b holds c*t tokens at
+// positions k_b*c*t + i and t output slots.
+struct LookaheadArgs {
+  std::vector<int64_t> cu_seq, cu_t;
+  std::vector<int32_t> ts, seg_per_seq;
+  std::vector<still_pos_segment> segs;
+};
+
+still_status lookahead_args(int32_t B, const int64_t* h_pass, int64_t c, int32_t t,
+                            LookaheadArgs& a) {
+  if (B < 1 || h_pass == nullptr) return STILL_ERR_INVALID_ARG;
+  a.cu_seq.assign(B + 1, 0);
+  a.cu_t.assign(B + 1, 0);
+  a.ts.assign(B, t);
+  a.seg_per_seq.assign(B, 1);
+  a.segs.resize(B);
+  for (int b = 0; b < B; ++b) {
+    still_lookahead_pass ps;
+    TRY(still_lookahead_pass_info(h_pass[b], c, t, &ps));
+    a.cu_seq[b + 1] = a.cu_seq[b] + ps.chunk_len;
+    a.cu_t[b + 1] = a.cu_t[b] + t;
+    a.segs[b] = still_pos_segment{(double)ps.chunk_start, 1.0, ps.chunk_len};
+  }
+  return STILL_OK;
+}
+
+}  // namespace
+
+still_status still_lookahead_compact_layer(still_ctx* ctx, int32_t layer, int32_t B,
+                                           const void* K, const void* V, const int64_t* h_pass,
+                                           int64_t c, int32_t t, void* Ck, void* Cv,
+                                           void* stream) {
+  LookaheadArgs a;
+  TRY(lookahead_args(B, h_pass, c, t, a));
+  return still_compact_layer_ragged(ctx, layer, K, V, a.cu_seq.data(), B, a.segs.data(),
+                                    a.seg_per_seq.data(), a.ts.data(), a.cu_t.data(), Ck, Cv,
+                                    nullptr, stream);
+}
+
+still_status still_lookahead_compact_stack(still_ctx* ctx, int32_t n_layers,
+                                           const uint8_t* h_compact_layer, int32_t B,
+                                           const void* const* K, const void* const* V,
+                                           const int64_t* h_pass, int64_t c, int32_t t,
+                                           void* const* Ck, void* const* Cv, void* stream) {
+  if (ctx == nullptr || K == nullptr || V == nullptr || Ck == nullptr || Cv == nullptr ||
+      n_layers < 1)
+    return STILL_ERR_INVALID_ARG;
+  LookaheadArgs a;
+  TRY(lookahead_args(B, h_pass, c, t, a));
+  for (int l = 0; l < n_layers; ++l) {
+    if (h_compact_layer != nullptr && !h_compact_layer[l]) continue;
+    const LayerW* L = nullptr;
+    TRY(check_ctx_layer(ctx, l, &L));
+  }
+  for (int l = 0; l < n_layers; ++l) {
+    if (h_compact_layer != nullptr && !h_compact_layer[l]) continue;
+    TRY(still_compact_layer_ragged(ctx, l, K[l], V[l], a.cu_seq.data(), B, a.segs.data(),
+                                   a.seg_per_seq.data(), a.ts.data(), a.cu_t.data(), Ck[l],
+                                   Cv[l], nullptr, stream));
+  }
   return STILL_OK;
 }
 
@@ -1424,7 +1679,7 @@ still_status still_workspace_size(const still_ctx* ctx, int64_t max_tokens, int3
     return ctx == nullptr || bytes == nullptr ? STILL_ERR_INVALID_ARG : STILL_ERR_NOT_LOADED;
   if (max_tokens < 1 || max_t < 1 || max_t > max_tokens) return STILL_ERR_SHAPE;
   Plan P;
-  if (!make_plan(ctx->layers[0].cfg, ctx->layers[0].qhat_lazy, max_tokens, max_t, 0.0,
+  if (!make_plan(ctx->layers[0].cfg, queries_per_call(ctx->layers[0]), max_tokens, max_t, 0.0,
                  (double)(max_tokens - 1), ctx->ws_limit, P))
     return STILL_ERR_OOM;
   *bytes = P.total;

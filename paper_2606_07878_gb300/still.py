@@ -24,10 +24,12 @@ EXPORTS = [
     "still_compact_layer", "still_compact_stack", "still_compact_layer_ragged",
     "still_compact_stack_ragged", "still_workspace_size", "still_set_workspace_limit",
     "still_set_qhat_eager_limit", "still_profile_enable_classes", "still_reserve_workspace",
+    "still_load_layer_weights_blocks",
     "still_get_device_status", "still_budget", "still_kv_bytes", "still_param_count",
     "still_profile_enable", "still_profile_read", "still_kernel_class_name",
     "still_compact_layer_noalloc", "still_recompact_layer_ragged", "still_recompact_stack_ragged",
-    "still_selftest_wait_timeout",
+    "still_selftest_wait_timeout", "still_compact_stack_masked", "still_lookahead_pass_info",
+    "still_lookahead_totals", "still_lookahead_compact_layer", "still_lookahead_compact_stack",
 ]
 
 NOALLOC_SCRATCH_MIB = 64  # STILL_NOALLOC_SCRATCH_MIB in include/still.h
@@ -65,6 +67,20 @@ class LayerWeights(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in WEIGHT_NAMES]
 
 
+BLOCK_WEIGHT_NAMES = ["Wq", "bq", "Wk", "bk", "Wv", "Wo", "Sq", "sbq", "Sk", "sbk", "Sv", "So",
+                      "W1", "W2"]
+
+
+class BlockWeights(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in BLOCK_WEIGHT_NAMES]
+
+
+class LookaheadPass(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int64) for n in (
+        "chunk_start", "chunk_len", "prefill_start", "prefill_len", "prefill_past",
+        "compact_row", "retained_after", "logical_after", "pos_offset_after")]
+
+
 class PosSegment(ctypes.Structure):
     _fields_ = [("start", ctypes.c_double), ("step", ctypes.c_double), ("count", ctypes.c_int64)]
 
@@ -86,6 +102,9 @@ def lib():
             "still_create": ([ctypes.c_int, ctypes.POINTER(P)], ctypes.c_int),
             "still_destroy": ([P], ctypes.c_int),
             "still_status_string": ([ctypes.c_int], ctypes.c_char_p),
+            "still_load_layer_weights_blocks": ([P, I32, ctypes.POINTER(LayerConfig), P,
+                                                 ctypes.POINTER(BlockWeights), P, P, P],
+                                                ctypes.c_int),
             "still_load_layer_weights": ([P, I32, ctypes.POINTER(LayerConfig),
                                           ctypes.POINTER(LayerWeights), P], ctypes.c_int),
             "still_compact_layer": ([P, I32, P, P, PI64, PSEG, I32, I64, I32, P, P, PD, PD, PI64,
@@ -119,6 +138,19 @@ def lib():
             "still_reserve_workspace": ([P, I64, I32], ctypes.c_int),
             "still_profile_read": ([P, I32, PI64, PD], ctypes.c_int),
             "still_kernel_class_name": ([I32], ctypes.c_char_p),
+            "still_compact_stack_masked": ([P, I32, ctypes.POINTER(ctypes.c_uint8),
+                                            ctypes.POINTER(P), ctypes.POINTER(P), PI64, PSEG,
+                                            I32, I64, I32, ctypes.POINTER(P), ctypes.POINTER(P),
+                                            PD, PD, PI64, P], ctypes.c_int),
+            "still_lookahead_pass_info": ([I64, I64, I32, ctypes.POINTER(LookaheadPass)],
+                                          ctypes.c_int),
+            "still_lookahead_totals": ([I64, I64, I32, PI64, PI64], ctypes.c_int),
+            "still_lookahead_compact_layer": ([P, I32, I32, P, P, PI64, I64, I32, P, P, P],
+                                              ctypes.c_int),
+            "still_lookahead_compact_stack": ([P, I32, ctypes.POINTER(ctypes.c_uint8), I32,
+                                               ctypes.POINTER(P), ctypes.POINTER(P), PI64, I64,
+                                               I32, ctypes.POINTER(P), ctypes.POINTER(P), P],
+                                              ctypes.c_int),
         }
         for name, (args, res) in sig.items():
             f = getattr(L, name)
@@ -165,7 +197,8 @@ def make_config(H, d, D, n, F, t_max, theta, theta_c=10.0, final_norm=0, logit_s
 
 def config_from_workload(wl: dict, t_max: int, **over) -> LayerConfig:
     kw = dict(H=wl["H"], d=wl["d"], D=wl["D"], n=wl["n"], F=wl["F"], t_max=t_max,
-              theta=wl["theta"])
+              theta=wl["theta"], n_blocks=wl.get("n_blocks", 1),
+              cross_every_block=int(wl.get("cross_every_block", 1)))
     kw.update(over)
     return make_config(**kw)
 
@@ -195,11 +228,20 @@ def still_set_qhat_eager_limit(ctx, nbytes: int):
 
 
 def still_load_layer_weights(ctx, layer: int, cfg: LayerConfig, weights: dict, stream=None):
-    """weights: name -> contiguous bf16 CUDA tensor, layouts as in include/still.h."""
-    w = LayerWeights(**{n: (weights[n].data_ptr() if weights.get(n) is not None else None)
-                        for n in WEIGHT_NAMES})
-    _check(lib().still_load_layer_weights(ctx, layer, ctypes.byref(cfg), ctypes.byref(w),
-                                          _stream(stream)), "still_load_layer_weights")
+    """weights: name -> contiguous bf16 CUDA tensor, layouts as in include/still.h. Block b > 0
+    tensors are named "<name>@<b>" (cfg.n_blocks > 1 loads through the per-block entry point)."""
+    ptr = lambda name: weights[name].data_ptr() if weights.get(name) is not None else None
+    if cfg.n_blocks == 1:
+        w = LayerWeights(**{n: ptr(n) for n in WEIGHT_NAMES})
+        _check(lib().still_load_layer_weights(ctx, layer, ctypes.byref(cfg), ctypes.byref(w),
+                                              _stream(stream)), "still_load_layer_weights")
+        return
+    blocks = (BlockWeights * cfg.n_blocks)(*[
+        BlockWeights(**{n: ptr(n if b == 0 else f"{n}@{b}") for n in BLOCK_WEIGHT_NAMES})
+        for b in range(cfg.n_blocks)])
+    _check(lib().still_load_layer_weights_blocks(ctx, layer, ctypes.byref(cfg), ptr("Z"), blocks,
+                                                 ptr("Wkey"), ptr("Wval"), _stream(stream)),
+           "still_load_layer_weights_blocks")
 
 
 def still_compact_layer(ctx, layer: int, K, V, t: int, Ck, Cv, segments=None, stream=None):
@@ -244,6 +286,63 @@ def still_compact_stack(ctx, Ks, Vs, t: int, Cks, Cvs, segments=None, stream=Non
                                      ctypes.byref(pst), ctypes.byref(off), _stream(stream)),
            "still_compact_stack")
     return ps.value, pst.value, off.value
+
+
+def still_compact_stack_masked(ctx, mask, Ks, Vs, t: int, Cks, Cvs, segments=None, stream=None):
+    """Compacts the layers l with mask[l] true; the other entries of Ks/Vs/Cks/Cvs may be
+    None and are not touched."""
+    L = len(mask)
+    P = ctypes.c_void_p
+    arr = lambda xs: (P * L)(*[(x.data_ptr() if x is not None else None) for x in xs])
+    ref = next(k for k, m in zip(Ks, mask) if m)
+    strides = (ctypes.c_int64 * 3)(*ref.stride())
+    seg, nseg = _segments(segments)
+    ps, pst, off = ctypes.c_double(), ctypes.c_double(), ctypes.c_int64()
+    m = (ctypes.c_uint8 * L)(*[1 if x else 0 for x in mask])
+    _check(lib().still_compact_stack_masked(ctx, L, m, arr(Ks), arr(Vs), strides, seg, nseg,
+                                            ref.shape[0], t, arr(Cks), arr(Cvs),
+                                            ctypes.byref(ps), ctypes.byref(pst),
+                                            ctypes.byref(off), _stream(stream)),
+           "still_compact_stack_masked")
+    return ps.value, pst.value, off.value
+
+
+def still_lookahead_pass_info(k: int, c: int, t: int) -> dict:
+    r = LookaheadPass()
+    _check(lib().still_lookahead_pass_info(k, c, t, ctypes.byref(r)), "still_lookahead_pass_info")
+    return {n: getattr(r, n) for n, _ in LookaheadPass._fields_}
+
+
+def still_lookahead_totals(T: int, c: int, t: int):
+    """(passes, retained cache entries) once T tokens have been compacted."""
+    p, r = ctypes.c_int64(), ctypes.c_int64()
+    _check(lib().still_lookahead_totals(T, c, t, ctypes.byref(p), ctypes.byref(r)),
+           "still_lookahead_totals")
+    return p.value, r.value
+
+
+def still_lookahead_compact_layer(ctx, layer, K, V, passes, c: int, t: int, Ck, Cv,
+                                  stream=None):
+    """K, V [B*c*t, H, d] packed raw chunks; passes[b] the pass index of sequence b;
+    Ck, Cv [B*t, H, d]."""
+    B = len(passes)
+    _check(lib().still_lookahead_compact_layer(ctx, layer, B, _ptr(K), _ptr(V),
+                                               (ctypes.c_int64 * B)(*passes), c, t, _ptr(Ck),
+                                               _ptr(Cv), _stream(stream)),
+           "still_lookahead_compact_layer")
+
+
+def still_lookahead_compact_stack(ctx, Ks, Vs, passes, c: int, t: int, Cks, Cvs, mask=None,
+                                  stream=None):
+    L = len(Ks)
+    B = len(passes)
+    P = ctypes.c_void_p
+    arr = lambda xs: (P * L)(*[(x.data_ptr() if x is not None else None) for x in xs])
+    m = None if mask is None else (ctypes.c_uint8 * L)(*[1 if x else 0 for x in mask])
+    _check(lib().still_lookahead_compact_stack(ctx, L, m, B, arr(Ks), arr(Vs),
+                                               (ctypes.c_int64 * B)(*passes), c, t, arr(Cks),
+                                               arr(Cvs), _stream(stream)),
+           "still_lookahead_compact_stack")
 
 
 def _ragged_args(cu_seqlens, ts, segments_per_seq):

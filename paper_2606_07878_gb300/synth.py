@@ -29,6 +29,11 @@ WORKLOADS = {
                        theta=1e6, heavy=1),
     "gemma_128k": dict(L=48, N=131072, H=8, d=256, D=2048, n=16, F=8192, ts=(16384, 655),
                        theta=1e6, heavy=3),
+    # The paper's canonical compactor on Qwen3-4B-shaped caches (36 layers, 8 KV-heads, d 128):
+    # d_l = 256, two blocks with cross-attention in both, one head, no FFN; 64k context at the
+    # 50x ratio (t = 1311).
+    "qwen3_4b_64k": dict(L=36, N=65536, H=8, d=128, D=256, n=1, F=0, ts=(1311,), theta=1e6,
+                         heavy=1, n_blocks=2, cross_every_block=1),
     # Iterative ragged serving: 8 sequences, lengths uniform in [8k, 32k] from seed 7, then
     # 16 rounds of +8192 tokens each, re-compacted to the 32x budget.
     "iterative_ragged": dict(L=36, H=8, d=128, D=1024, n=8, F=4096, theta=1e6, heavy=1,
@@ -90,11 +95,17 @@ def weight_shapes(H, d, D, n, F, t_max, n_blocks=1, cross_every_block=True):
     return shapes
 
 
-def gen_weights(wl: dict, layer: int, t_max: int, device="cpu", seed: int = 0, n_blocks=1):
-    """Random-init weights for one layer: N(0, 0.02) rounded to bf16, layout of weight_shapes."""
+def gen_weights(wl: dict, layer: int, t_max: int, device="cpu", seed: int = 0, n_blocks=None,
+                cross_every_block=None):
+    """Random-init weights for one layer: N(0, 0.02) rounded to bf16, layout of weight_shapes.
+    The block structure defaults to the workload's (n_blocks, cross_every_block; 1 and True)."""
+    if n_blocks is None:
+        n_blocks = wl.get("n_blocks", 1)
+    if cross_every_block is None:
+        cross_every_block = bool(wl.get("cross_every_block", 1))
     out = {}
     for name, shape in weight_shapes(wl["H"], wl["d"], wl["D"], wl["n"], wl["F"], t_max,
-                                     n_blocks).items():
+                                     n_blocks, cross_every_block).items():
         base, _, blk = name.partition("@")
         g = _gen(device, seed, layer, _TENSOR_IDS[base], int(blk or 0))
         x = torch.randn(shape, generator=g, device=device, dtype=torch.float32)

@@ -23,7 +23,7 @@ def metrics(ref: np.ndarray, got: np.ndarray):
     return err, cos
 
 
-def assert_parity(ref, got, what=""):
+def assert_parity(ref, got, what="", err_rel=ERR_REL):
     err, cos = metrics(ref, got)
     log = os.environ.get("STILL_PARITY_LOG")
     if log:
@@ -32,7 +32,7 @@ def assert_parity(ref, got, what=""):
                                 "what": what, "max_err_over_rms": err, "min_row_cos": cos})
                     + "\n")
     assert np.all(np.isfinite(got)), f"{what}: non-finite output"
-    assert err <= ERR_REL and cos >= COS_MIN, f"{what}: max|err|/RMS={err:.4e} min cos={cos:.6f}"
+    assert err <= err_rel and cos >= COS_MIN, f"{what}: max|err|/RMS={err:.4e} min cos={cos:.6f}"
     return err, cos
 
 

@@ -1,5 +1,6 @@
 """CPU checks of the boundary: libstill.so loads, exports every entry point include/still.h
 declares, and its host-only accounting functions match the paper's printed numbers."""
+import itertools
 import json
 import os
 import re
@@ -62,3 +63,22 @@ def test_param_count_matches_paper(lib):
                                 n_blocks=c["B"], cross_every_block=int(c["cross_every_block"]))
         total = b["L"] * still.still_param_count(cfg, c["t"])
         assert abs(total - c["printed_total"]) <= g["tolerance_abs"], c["name"]
+
+
+def test_lookahead_schedule_matches_oracle(lib):
+    from oracle import still_oracle as O
+    for k, c, t in itertools.product([0, 1, 2, 7, 127, 10**6], [1, 3, 8, 32], [1, 16, 128]):
+        assert still.still_lookahead_pass_info(k, c, t) == O.lookahead_pass(k, c, t), (k, c, t)
+    g = json.load(open(os.path.join(GOLDEN, "iterative_slots.json")))
+    for case in g["cases"]:
+        assert still.still_lookahead_totals(case["T"], case["c"], g["t"]) == O.lookahead_totals(
+            case["T"], case["c"], g["t"])
+    for args, name in [((1025, 8, 128), "STILL_ERR_SHAPE"), ((1024, 0, 128), "STILL_ERR_INVALID_ARG"),
+                       ((0, 8, 128), "STILL_ERR_INVALID_ARG")]:
+        with pytest.raises(still.StillError) as e:
+            still.still_lookahead_totals(*args)
+        assert e.value.name == name, args
+    for args in [(-1, 8, 128), (0, 8, 0), (2**53, 8, 128)]:
+        with pytest.raises(still.StillError) as e:
+            still.still_lookahead_pass_info(*args)
+        assert e.value.name == "STILL_ERR_INVALID_ARG", args
