@@ -163,8 +163,12 @@ def algorithmic_flops(wl, t, N):
     ca = (2 * N * H * 2 * d * n * D + 2 * t * N * H * n * D + 2 * t * N * H * n * 2 * d
           + 2 * t * H * n * 2 * d * D + 2 * t * H * n * D * D)
     sa = 6 * t * H * D * n * D + 4 * t * t * H * n * D + 2 * t * H * n * D * D
+    # The last block's cross-attention is one fused kernel when 2d <= 256; earlier blocks
+    # (and every block at 2d = 512) take the scores GEMM.
+    fused_last = 2 * d <= 256 and (nb == 1 or wl.get("cross_every_block", 1))
     return {"total": n_ca * ca + nb * (sa + 4 * t * H * D * F) + 4 * t * H * D * d,
-            "scores": n_ca * 2 * t * N * H * n * D, "px": n_ca * 2 * t * N * H * n * 2 * d}
+            "scores": n_ca * 2 * t * N * H * n * D, "px": n_ca * 2 * t * N * H * n * 2 * d,
+            "scores_gemm": (n_ca - (1 if fused_last else 0)) * 2 * t * N * H * n * D}
 
 
 def run_cpu_baseline(wl, t, budget_s=30.0):
@@ -503,8 +507,8 @@ def main():
     fl = algorithmic_flops(wl, t, N)
     fused = kname == "ca_fused"
     n_k, ms_k = prof_timed[kname]  # one step's launches (the captured event pairs)
-    alg = fl["scores"] + fl["px"] if fused else fl["scores"]
-    issued = 3 * fl["scores"] + 1.5 * fl["px"] if fused else 3 * fl["scores"]
+    alg = fl["scores"] + fl["px"] if fused else fl["scores_gemm"]
+    issued = 3 * fl["scores"] + 1.5 * fl["px"] if fused else 3 * fl["scores_gemm"]
     per_launch_flops = alg * L / max(n_k, 1)
     achieved = per_launch_flops / (ms_k / max(n_k, 1) / 1e3) / 1e12 if ms_k > 0 else None
     tr = TRAFFIC[kname]

@@ -296,7 +296,8 @@ struct Plan {
   int H, d, D, n, F, t;
   int64_t N, Np, ldS, tp, ldt;
   int G;
-  bool flash;     // fused cross-attention kernel (2d of 128 or 256), else scores + P X kernels
+  bool flash;     // fused cross-attention kernel (2d of 128 or 256) for the last block
+  bool split_ca;  // some block takes the scores + P X kernels
   int ca_units;   // (h, i) pairs per cross-attention group
   int sa_heads;   // KV-heads per self-attention group
   int sa_sub;     // self heads per scores / softmax / P.v pass (n unless one bank is too big)
@@ -357,18 +358,23 @@ bool make_plan(const still_layer_config& c, bool lazy_q, int64_t N, int t, doubl
   P.kb_b = a256(N * 2 * D * 2);
   P.kss_b = a256(N * 4 * (EpiRopeCT<false>::kParts * (D / 256) + 1));  // |k~|^2 partials + inverses
   P.q_b = a256(T * 2 * D * 2);
-  // The fused kernel holds fp16 probabilities; a compactor of two blocks needs the first block's
-  // probabilities in hi | lo (its cross-attention output steers the second block's queries), so
-  // such layers take the scores + P X kernels.
-  P.flash = (d == 64 || d == 128) && c.n_blocks == 1;
+  // The fused kernel holds fp16 probabilities and bf16 hi | lo q, k; a block that feeds
+  // another needs its probabilities in hi | lo and fp16 hi | lo q, k (its cross-attention
+  // output steers the next block's queries), so such blocks take the scores + P X kernels
+  // and only the last block is fused. The unit holds the larger of the two layouts.
+  P.flash = d == 64 || d == 128;
+  P.split_ca = !P.flash || c.n_blocks > 1;
+  P.S_b = 0;
+  P.P_b = 0;
+  P.O_b = 0;
   if (P.flash) {
-    P.S_b = 0;
     P.P_b = a256(T * 8) * kMaxFlashSplit;          // per-split row statistics (m, l)
     P.O_b = a256(T * 2 * d * 4) * kMaxFlashSplit;  // per-split unnormalised O
-  } else {
+  }
+  if (P.split_ca) {
     P.S_b = a256(T * P.ldS * 4);
-    P.P_b = a256(T * 8 * (2 * ((N + 255) / 256) + 1));  // row-softmax partials + statistics
-    P.O_b = a256(T * 2 * d * 4) * kMaxSplit;             // split-K partials of P X
+    P.P_b = std::max(P.P_b, a256(T * 8 * (2 * ((N + 255) / 256) + 1)));  // softmax partials
+    P.O_b = std::max(P.O_b, a256(T * 2 * d * 4) * kMaxSplit);  // split-K partials of P X
   }
   // lazy q^: fp32 q~ of the unit and its sum-of-squares partials + inverse norms
   P.qt_b = lazy_q ? a256(T * D * 4) + a256(T * 4 * (2 * (D / 256) + 1)) : 0;
@@ -541,10 +547,10 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
   for (int bi = 0; bi < c.n_blocks; ++bi) {
   const BlockW& Bw = L.blk[bi];
   const bool last = bi + 1 == c.n_blocks;
-  // Every block of a layer with more than one block keeps its self-attention value path and
-  // FFN in split precision: the next block's cross-attention queries amplify any rounding
-  // there, and the last block's own rounding adds to the amplified error of the first.
-  const bool exact = !last || L.f16;
+  // A block whose output enters another block keeps its cross-attention, self-attention
+  // value path and FFN in split precision: the next block's cross-attention queries amplify
+  // any rounding there.
+  const bool exact = !last;
   float* Za = Z2;  // this block's state after cross-attention (Z2 itself without it)
   if (Bw.has_ca) {
   const bool q_call = bi > 0 || L.qhat_lazy;  // queries formed in this call
@@ -670,7 +676,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
                                             scale / qscale, kinv, s));
     KLAUNCH(STILL_K_QROPE, launch_q_rope(qsrc, q_tmax, q_b0, nbl, t, D, qstart, qstep, L.omega_c,
                                          c.compactor_rope, qhl, exact ? 1 : 0, qscale, s));
-    if (P.flash) {
+    if (P.flash && !exact) {
       // S, the online softmax and P X in one kernel; per-split partials merged in order.
       float2* fst = stp;  // [nsplit][nbl * t] (the statistics region of this path)
       FlashParams fp;
