@@ -20,6 +20,8 @@ so that each step can be checked against the text by eye:
     ..................................................... App. A "Output projections"; App. B
   * compact budget t = round(N / c) ........ App. J exact-results table (K column)
   * position offset T - t ................................ App. B, logical vs physical length
+  * beta = Z_out w_beta, saturation, mass matching ......... App. A, Output projections / beta
+  * attention over [C_k; K_fix] with bias [beta; 0] .......... App. B, Bias semantics
   * iterative chunked schedule with lookahead: passes, chunks, retained cache . Sec. 2.3
 
 Readings taken where the paper is silent (each listed with its basis in the design notes):
@@ -253,10 +255,10 @@ def ffn(Zn: np.ndarray, W: dict, b: int) -> np.ndarray:
 # ----------------------------------------------------------------------------- compactor
 
 def compact_head(Kh: np.ndarray, Vh: np.ndarray, Zh: np.ndarray, W: dict, cfg: Cfg,
-                 kpos: np.ndarray, row_chunk: int = 4096):
+                 kpos: np.ndarray, row_chunk: int = 4096, return_state: bool = False):
     """One KV-head: cached (K_h, V_h) [N, d] and its latent bank Z_h [t, D] -> (C_k, C_v) [t, d].
 
-    Returns (C_k, C_v, out_positions).
+    Returns (C_k, C_v, out_positions), and the final latent state Z_out when return_state.
     """
     t = Zh.shape[0]
     pmin, pmax = float(np.min(kpos)), float(np.max(kpos))
@@ -277,7 +279,36 @@ def compact_head(Kh: np.ndarray, Vh: np.ndarray, Zh: np.ndarray, W: dict, cfg: C
     if cfg.rope_fix:
         Ck = rope(Ck, opos, cfg.theta)                 # back into the base model's RoPE frame
     Cv = Zout @ W["Wval"]
+    if return_state:
+        return Ck, Cv, opos, Zout
     return Ck, Cv, opos
+
+
+def beta_head(Zout: np.ndarray, w_beta: np.ndarray, beta_max: float = 0.0, mass_match: int = 0,
+              log_x: float = 0.0, T: float | None = None) -> np.ndarray:
+    """Per-slot logit bias of one KV-head, beta = Z_out w_beta (App. A, Output projections),
+    with the optional shaping of App. A ("Optional beta shaping"), applied in that order:
+      saturation     beta <- beta_max * tanh(beta / beta_max)          when beta_max > 0
+      mass matching  beta <- beta + log(T / t)                        mass_match = 1
+                     beta <- beta + log(x) + log(T / t), log_x = log x  mass_match = 2
+    T is the number of cached tokens the t slots replace."""
+    t = Zout.shape[0]
+    beta = Zout @ w_beta
+    if beta_max > 0:
+        beta = beta_max * np.tanh(beta / beta_max)
+    if mass_match:
+        beta = beta + np.log(T / t) + (log_x if mass_match == 2 else 0.0)
+    return beta
+
+
+def biased_attention(q: np.ndarray, Ck: np.ndarray, Cv: np.ndarray, beta: np.ndarray,
+                     Kfix: np.ndarray, Vfix: np.ndarray, scale: float) -> np.ndarray:
+    """Attention of query rows q [m, d] over the compact prefix followed by uncompacted entries,
+    with beta added to the compact-prefix logits and 0 to the others (App. B, "Bias semantics
+    in attention"): softmax over [scale q C_k^T + beta, scale q K_fix^T] applied to
+    [C_v; V_fix]."""
+    logits = np.concatenate([scale * (q @ Ck.T) + beta[None, :], scale * (q @ Kfix.T)], axis=1)
+    return softmax_rows(logits) @ np.concatenate([Cv, Vfix], axis=0)
 
 
 def compact_layer(K: np.ndarray, V: np.ndarray, W: dict, cfg: Cfg, t: int,
@@ -300,6 +331,27 @@ def compact_layer(K: np.ndarray, V: np.ndarray, W: dict, cfg: Cfg, t: int,
         Ck[:, h], Cv[:, h], opos = compact_head(K[:, h], V[:, h], Z[h, :t], W, cfg, kpos,
                                                 row_chunk)
     return Ck, Cv, opos, position_offset(N, t)
+
+
+def compact_layer_beta(K: np.ndarray, V: np.ndarray, W: dict, cfg: Cfg, t: int, w_beta,
+                       beta_max: float = 0.0, mass_match: int = 0, log_x: float = 0.0,
+                       kpos: np.ndarray | None = None, heads=None):
+    """compact_layer plus the beta head: returns (C_k, C_v, beta [t, H]); the mass-matching
+    T is the number of cached tokens N (the entries the t slots replace)."""
+    N = K.shape[0]
+    if kpos is None:
+        kpos = np.arange(N, dtype=np.float64)
+    kpos = np.asarray(kpos, dtype=np.float64)
+    Z = np.asarray(W["Z"], dtype=np.float64)
+    Ck = np.full((t, cfg.H, cfg.d), np.nan)
+    Cv = np.full((t, cfg.H, cfg.d), np.nan)
+    B = np.full((t, cfg.H), np.nan)
+    for h in (range(cfg.H) if heads is None else heads):
+        Ck[:, h], Cv[:, h], _, Zout = compact_head(K[:, h], V[:, h], Z[h, :t], W, cfg, kpos,
+                                                   return_state=True)
+        B[:, h] = beta_head(Zout, np.asarray(w_beta, dtype=np.float64), beta_max, mass_match,
+                            log_x, T=N)
+    return Ck, Cv, B
 
 
 def as_f64(weights: dict) -> dict:

@@ -300,3 +300,79 @@ def test_lookahead_schedule_invariants(c, t):
     if ct > 1:
         with pytest.raises(ValueError):
             O.lookahead_totals(ct + 1, c, t)
+
+
+# ------------------------------------------------------------------ beta channel
+
+def test_beta_head_identity_init_and_shaping():
+    rng = np.random.default_rng(5)
+    Zout = rng.standard_normal((12, 32))
+    # identity-style initialisation sets w_beta = 0 (App. C): no bias at all
+    assert np.all(O.beta_head(Zout, np.zeros(32)) == 0)
+    # ... and exact mass matching alone then gives the uniform offset log(T / t)
+    np.testing.assert_allclose(O.beta_head(Zout, np.zeros(32), mass_match=1, T=600),
+                               np.log(600 / 12), rtol=0, atol=1e-15)
+    w = rng.standard_normal(32)
+    raw = Zout @ w
+    np.testing.assert_allclose(O.beta_head(Zout, w), raw, rtol=1e-15)
+    sat = O.beta_head(Zout, 0.5 * w, beta_max=3.0)
+    assert np.all(np.abs(sat) < 3.0) and np.all(np.sign(sat) == np.sign(raw))
+    assert np.all(np.abs(sat) < np.abs(0.5 * raw))      # tanh(x) < x for x > 0
+    # far below beta_max the saturation is the identity to second order
+    # (relative deviation (beta / beta_max)^2 / 3 < 1e-9 here)
+    np.testing.assert_allclose(O.beta_head(Zout, 1e-4 * w, beta_max=50.0), 1e-4 * raw,
+                               rtol=1e-8)
+    # learnable mass matching at x0 = 1e-3 starts 3 ln 10 below exact mass matching
+    d = (O.beta_head(Zout, w, mass_match=2, log_x=np.log(1e-3), T=600)
+         - O.beta_head(Zout, w, mass_match=1, T=600))
+    np.testing.assert_allclose(d, -3 * np.log(10), rtol=1e-14)
+
+
+def test_biased_attention_reduces_to_softmax_attention():
+    rng = np.random.default_rng(6)
+    d = 16
+    q = rng.standard_normal((3, d))
+    Ck, Cv = rng.standard_normal((5, d)), rng.standard_normal((5, d))
+    Kf, Vf = rng.standard_normal((7, d)), rng.standard_normal((7, d))
+    s = 1 / np.sqrt(d)
+    out = O.biased_attention(q, Ck, Cv, np.zeros(5), Kf, Vf, s)
+    K, V = np.concatenate([Ck, Kf]), np.concatenate([Cv, Vf])
+    ref = scipy.special.softmax(s * q @ K.T, axis=1) @ V
+    np.testing.assert_allclose(out, ref, rtol=1e-12, atol=1e-14)
+    # no uncompacted entries, or no compact prefix
+    np.testing.assert_allclose(O.biased_attention(q, Ck, Cv, np.zeros(5), Kf[:0], Vf[:0], s),
+                               scipy.special.softmax(s * q @ Ck.T, axis=1) @ Cv, rtol=1e-12)
+    np.testing.assert_allclose(O.biased_attention(q, Ck[:0], Cv[:0], np.zeros(0), Kf, Vf, s),
+                               scipy.special.softmax(s * q @ Kf.T, axis=1) @ Vf, rtol=1e-12)
+
+
+def test_bias_log_m_equals_m_copies_of_the_slot():
+    """A compact slot carrying beta = log m attends exactly like m identical raw entries."""
+    rng = np.random.default_rng(7)
+    d = 8
+    q = rng.standard_normal((4, d))
+    Ck, Cv = rng.standard_normal((3, d)), rng.standard_normal((3, d))
+    Kf, Vf = rng.standard_normal((5, d)), rng.standard_normal((5, d))
+    m = np.array([1, 4, 9])
+    out = O.biased_attention(q, Ck, Cv, np.log(m), Kf, Vf, 0.3)
+    Kx = np.concatenate([np.repeat(Ck, m, axis=0), Kf])
+    Vx = np.concatenate([np.repeat(Cv, m, axis=0), Vf])
+    rows = []
+    for qi in q:                      # brute force, one query at a time
+        w = np.exp(0.3 * Kx @ qi - np.max(0.3 * Kx @ qi))
+        rows.append(w @ Vx / w.sum())
+    np.testing.assert_allclose(out, np.array(rows), rtol=1e-12, atol=1e-14)
+
+
+def test_mass_matching_restores_the_prefix_share_under_uniform_attention():
+    """With equal logits (q = 0), slots offset by log(T / t) take the share T / (T + S) of the
+    attention that T uncompacted prefix tokens would take next to S others."""
+    d, t, T, S = 8, 6, 300, 40
+    rng = np.random.default_rng(8)
+    Ck = rng.standard_normal((t, d))
+    Cv = np.ones((t, d))
+    Kf = rng.standard_normal((S, d))
+    Vf = np.zeros((S, d))
+    beta = O.beta_head(rng.standard_normal((t, 4)), np.zeros(4), mass_match=1, T=T)
+    share = O.biased_attention(np.zeros((1, d)), Ck, Cv, beta, Kf, Vf, 1.0)[0, 0]
+    assert share == pytest.approx(T / (T + S), rel=1e-13)
