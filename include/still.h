@@ -190,6 +190,51 @@ still_status still_compact_layer_noalloc(still_ctx* ctx, int32_t layer, const vo
                                          double* h_out_pos_step, int64_t* h_pos_offset,
                                          void* stream);
 
+/* ---------------------------------------------------------------------------------------
+ * Optional per-slot logit bias (App. A, "Output projections" and "Optional beta shaping";
+ * App. B, "Bias semantics in attention"). A third head beta = Z_out w_beta, shared across
+ * KV-heads like W_key and W_val, optionally shaped:
+ *   saturation     beta <- beta_max * tanh(beta / beta_max)         (beta_max > 0)
+ *   mass matching  beta <- beta + log(T / t)                        (mass_match = 1)
+ *                  beta <- beta + log_x + log(T / t)                (mass_match = 2, log_x = log x)
+ * in that order, with T the number of cached entries the t slots replace (N of the call). */
+typedef struct {
+  float beta_max;      /* 0: no saturation */
+  int32_t mass_match;  /* 0, 1 or 2 as above */
+  float log_x;         /* learnable offset log x (the paper initialises x at 1e-3) */
+} still_beta_config;
+
+/* Sets (or replaces) the beta head of a loaded layer: w_beta [d_latent] bf16 device pointer
+ * (copied), shaping bc (host). STILL_ERR_NOT_LOADED if the layer is not loaded. */
+still_status still_set_beta_head(still_ctx* ctx, int32_t layer, const void* w_beta,
+                                 const still_beta_config* bc, void* stream);
+
+/* still_compact_layer that also writes the per-slot bias: beta [t][H] fp32 device pointer
+ * (4-byte aligned; slot j of KV-head h at j * H + h). STILL_ERR_NOT_LOADED without a beta head. */
+still_status still_compact_layer_beta(still_ctx* ctx, int32_t layer, const void* K,
+                                      const void* V, const int64_t strides_kv[3],
+                                      const still_pos_segment* h_segments, int32_t n_segments,
+                                      int64_t N, int32_t t, void* Ck, void* Cv, float* beta,
+                                      double* h_out_pos_start, double* h_out_pos_step,
+                                      int64_t* h_pos_offset, void* stream);
+
+/* The consumer of a compact cache at decode time (App. B, "Bias semantics in attention"):
+ * for each query row, softmax over [scale q C_k^T + beta, scale q K_fix^T] applied to
+ * [C_v; V_fix], with grouped query heads (query head i reads KV-head i / (Hq / H)).
+ *   q      [nq][Hq][d] bf16
+ *   Ck, Cv [t][H][d] bf16 compact prefix (the layout still_compact_layer writes); t >= 0
+ *   beta   [t][H] fp32 per-slot bias, or NULL for none (must be finite)
+ *   Kfix, Vfix [S][H][d] bf16 uncompacted entries (RoPE already applied, as cached); S >= 0
+ *   out    [nq][Hq][d] bf16
+ *   scale  logit scale; 0 means 1 / sqrt(d)
+ * d in {64, 128, 256}, t + S >= 1, nq * Hq / H <= 64; tensor pointers 16-byte aligned.
+ * Keys are processed in chunks of 128 whose partial results are merged in a fixed order; the
+ * context's workspace holds the partials (grown on demand). Stream-ordered. */
+still_status still_attend_biased(still_ctx* ctx, const void* q, int32_t nq, int32_t Hq,
+                                 const void* Ck, const void* Cv, const float* beta, int64_t t,
+                                 const void* Kfix, const void* Vfix, int64_t S, int32_t H,
+                                 int32_t d, float scale, void* out, void* stream);
+
 /* Compacts layers 0..n_layers-1 (all loaded) over the same positions: the per-layer
  * compactors share nothing at forward time (App. M, "No inter-layer compactor channel"), so
  * this is one stream-ordered launch sequence over the layer stack. K[l], V[l], Ck[l], Cv[l] are device
@@ -383,6 +428,8 @@ typedef enum {
   STILL_K_NORMS,        /* QK-norm factors from sum-of-squares partials     */
   STILL_K_LOAD,         /* weight-load precompute GEMMs                     */
   STILL_K_CA_FUSED,     /* fused scores + online softmax + P X (d <= 128)   */
+  STILL_K_BETA,         /* beta head: Z_out w_beta, shaped                  */
+  STILL_K_DECODE,       /* biased decode attention (chunks + merge)         */
   STILL_K_COUNT
 } still_kernel_class;
 

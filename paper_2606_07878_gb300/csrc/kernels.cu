@@ -609,9 +609,185 @@ __global__ void bias_kernel(const __nv_bfloat16* in, const __nv_bfloat16* in2, i
   if (in2 != nullptr) out[C + c] = __bfloat162float(in2[src]);
 }
 
+// ----------------------------------------------------------------------- beta channel
+
+// beta[j][h] of latent row (h, j): Z_out (hi + lo) . w, then saturation and the mass-matching
+// offset (App. A, output projections and optional beta shaping). One warp per row.
+__global__ void beta_kernel(const __nv_bfloat16* __restrict__ Z, int64_t rows, int t, int H,
+                            int D, const float* __restrict__ w, float beta_max, float offset,
+                            float* __restrict__ beta) {
+  const int64_t row = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const __nv_bfloat16* z = Z + row * 2 * D;
+  float acc = 0.f;
+  for (int c = lane; c < D; c += 32)
+    acc += (__bfloat162float(z[c]) + __bfloat162float(z[D + c])) * w[c];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  if (lane == 0) {
+    if (beta_max > 0.f) acc = beta_max * tanhf(acc / beta_max);
+    const int h = (int)(row / t), j = (int)(row % t);
+    beta[(int64_t)j * H + h] = acc + offset;
+  }
+}
+
+// ----------------------------------------------------------------- biased decode attention
+//
+// Attention of query rows over the entries [C (t compact slots, logit bias beta) ; F (S
+// uncompacted entries, bias 0)] (App. B, "Bias semantics in attention"). Grid (chunk, KV-head):
+// a CTA stages one chunk of kDecChunk entries of its KV-head (keys transposed, values as rows,
+// bf16 in shared memory), serves every query row of the KV-head's query heads from it, and
+// writes per-row partials (max m, sum l, unnormalised O); decode_merge_kernel combines the
+// chunks in order.
+constexpr int kDecChunk = 128;
+constexpr int kDecThreads = 128;
+
+__global__ void __launch_bounds__(kDecThreads)
+    decode_chunk_kernel(DecodeArgs a, float* __restrict__ part_o, float2* __restrict__ part_ml) {
+  extern __shared__ uint8_t dsm[];
+  const int d = a.d;
+  const int h = blockIdx.y, chunk = blockIdx.x;
+  const int g = a.Hq / a.H;        // query heads per KV-head
+  const int G = a.nq * g;          // query rows served by this CTA
+  __nv_bfloat16* kt = reinterpret_cast<__nv_bfloat16*>(dsm);   // [d][kDecChunk]
+  __nv_bfloat16* vr = kt + (size_t)d * kDecChunk;              // [kDecChunk][d]
+  float* qs = reinterpret_cast<float*>(vr + (size_t)kDecChunk * d);  // [G][d]
+  float* pw = qs + (size_t)G * d;                                     // [kDecChunk]
+  float* red = pw + kDecChunk;                                        // [2][4]
+  const int64_t e0 = (int64_t)chunk * kDecChunk;
+  const int64_t E = a.t + a.S;
+  // stage keys (transposed) and values; entries past E are zero (masked below)
+  const int vecs = d / 8;
+  for (int it = threadIdx.x; it < kDecChunk * vecs; it += kDecThreads) {
+    const int i = it / vecs, c0 = 8 * (it % vecs);
+    const int64_t e = e0 + i;
+    uint4 kq = make_uint4(0, 0, 0, 0), vq = make_uint4(0, 0, 0, 0);
+    if (e < E) {
+      const int64_t off = (e < a.t ? e * a.cst : (e - a.t) * a.fst) + (int64_t)h * d + c0;
+      const __nv_bfloat16* kp = (e < a.t ? a.Ck : a.Kf) + off;
+      const __nv_bfloat16* vp = (e < a.t ? a.Cv : a.Vf) + off;
+      kq = *reinterpret_cast<const uint4*>(kp);
+      vq = *reinterpret_cast<const uint4*>(vp);
+    }
+    const __nv_bfloat16* ke = reinterpret_cast<const __nv_bfloat16*>(&kq);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) kt[(size_t)(c0 + k) * kDecChunk + i] = ke[k];
+    *reinterpret_cast<uint4*>(vr + (size_t)i * d + c0) = vq;
+  }
+  // query rows of this KV-head: row r = (query n, head h * g + k) with r = n * g + k
+  for (int it = threadIdx.x; it < G * d; it += kDecThreads) {
+    const int r = it / d, c = it % d;
+    const int n = r / g, qh = h * g + r % g;
+    qs[it] = __bfloat162float(a.q[((int64_t)n * a.Hq + qh) * d + c]);
+  }
+  __syncthreads();
+  const int i = threadIdx.x;  // this thread's entry in the chunk
+  const int64_t e = e0 + i;
+  const bool valid = e < E;
+  const float bias = (valid && e < a.t && a.beta != nullptr) ? a.beta[e * a.H + h] : 0.f;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t nch = gridDim.x;
+  for (int r = 0; r < G; ++r) {
+    const float* qr = qs + (size_t)r * d;
+    float acc = 0.f;
+    for (int c = 0; c < d; ++c) acc = fmaf(qr[c], __bfloat162float(kt[(size_t)c * kDecChunk + i]), acc);
+    const float logit = valid ? acc * a.scale + bias : -INFINITY;
+    // chunk max
+    float m = logit;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    if (lane == 0) red[warp] = m;
+    __syncthreads();
+    m = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
+    const float p = valid ? __expf(logit - m) : 0.f;
+    float l = p;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+    pw[i] = p;
+    if (lane == 0) red[4 + warp] = l;
+    __syncthreads();
+    const float lsum = red[4] + red[5] + red[6] + red[7];
+    // O[c] = sum_i p_i V[i][c]
+    const int n = r / g, qh = h * g + r % g;
+    const int64_t prow = ((int64_t)n * a.Hq + qh) * nch + chunk;
+    for (int c = threadIdx.x; c < d; c += kDecThreads) {
+      float o = 0.f;
+      for (int k = 0; k < kDecChunk; ++k) o = fmaf(pw[k], __bfloat162float(vr[(size_t)k * d + c]), o);
+      part_o[prow * d + c] = o;
+    }
+    if (threadIdx.x == 0) part_ml[prow] = make_float2(m, lsum);
+    __syncthreads();  // pw and red are reused by the next row
+  }
+}
+
+// Output row (query n, query head qh): sum_s e^(m_s - M) O_s / sum_s e^(m_s - M) l_s over the
+// chunk partials, in chunk order. One warp per row.
+__global__ void decode_merge_kernel(const float* __restrict__ part_o,
+                                    const float2* __restrict__ part_ml, int64_t rows, int nch,
+                                    int d, __nv_bfloat16* __restrict__ out) {
+  const int64_t row = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const float2* ml = part_ml + row * nch;
+  float M = -INFINITY;
+  for (int s = 0; s < nch; ++s) M = fmaxf(M, ml[s].x);
+  float L = 0.f;
+  for (int s = 0; s < nch; ++s)
+    if (ml[s].x != -INFINITY) L += __expf(ml[s].x - M) * ml[s].y;
+  const float inv = 1.f / L;
+  for (int c = lane; c < d; c += 32) {
+    float o = 0.f;
+    for (int s = 0; s < nch; ++s)
+      if (ml[s].x != -INFINITY) o += __expf(ml[s].x - M) * part_o[(row * nch + s) * d + c];
+    out[row * d + c] = __float2bfloat16_rn(o * inv);
+  }
+}
+
+}  // namespace
+
+namespace {
+
 inline unsigned blocks_for(int64_t n, int per) { return (unsigned)((n + per - 1) / per); }
 
 }  // namespace
+
+size_t decode_workspace_bytes(int64_t rows, int64_t entries, int d) {
+  const int64_t nch = (entries + kDecChunk - 1) / kDecChunk;
+  return (size_t)rows * nch * d * 4 + (size_t)rows * nch * 8 + 256;
+}
+
+cudaError_t launch_decode_biased(const DecodeArgs& a, void* ws, cudaStream_t s) {
+  const int64_t E = a.t + a.S;
+  const int nch = (int)((E + kDecChunk - 1) / kDecChunk);
+  const int g = a.Hq / a.H;
+  const int G = a.nq * g;
+  const int64_t rows = (int64_t)a.nq * a.Hq;
+  float* part_o = static_cast<float*>(ws);
+  float2* part_ml = reinterpret_cast<float2*>(
+      static_cast<uint8_t*>(ws) + (((size_t)rows * nch * a.d * 4 + 255) & ~size_t(255)));
+  const size_t smem = (size_t)2 * kDecChunk * a.d * 2 + (size_t)G * a.d * 4 + kDecChunk * 4 + 64;
+  static thread_local size_t smem_set = 48 * 1024;
+  if (smem > smem_set) {
+    cudaError_t e = cudaFuncSetAttribute(decode_chunk_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    smem_set = smem;
+  }
+  decode_chunk_kernel<<<dim3(nch, a.H), kDecThreads, smem, s>>>(a, part_o, part_ml);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  decode_merge_kernel<<<blocks_for(rows, 8), 256, 0, s>>>(part_o, part_ml, rows, nch, a.d, a.out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_beta(const __nv_bfloat16* Z, int t, int H, int D, const float* w,
+                        float beta_max, float offset, float* beta, cudaStream_t s) {
+  const int64_t rows = (int64_t)H * t;
+  if (rows == 0) return cudaSuccess;
+  beta_kernel<<<blocks_for(rows, 8), 256, 0, s>>>(Z, rows, t, H, D, w, beta_max, offset, beta);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_strip(const KVSource& src, int64_t N, int H, int d, const PosSegs& segs,
                          const double* omega, int rope_fix, __nv_bfloat16* X, __half* XT,

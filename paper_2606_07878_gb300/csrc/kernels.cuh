@@ -31,6 +31,29 @@ cudaError_t launch_strip(const KVSource& src, int64_t N, int H, int d, const Pos
                          const double* omega, int rope_fix, __nv_bfloat16* X, __half* XT,
                          int64_t Np, float2* gd, double pmin, int G, int x16, cudaStream_t s);
 
+// Per-slot logit bias from the final latent state Z ([H * t][2D] bf16 hi | lo, rows h * t + j):
+// beta[j][h] = sat(Z_hi + Z_lo) . w) + offset, sat(x) = beta_max tanh(x / beta_max) when
+// beta_max > 0 (App. A, output projections; optional beta shaping).
+cudaError_t launch_beta(const __nv_bfloat16* Z, int t, int H, int D, const float* w,
+                        float beta_max, float offset, float* beta, cudaStream_t s);
+
+// Decode-time attention over a compact prefix with logit bias followed by uncompacted entries
+// (App. B, "Bias semantics in attention").
+struct DecodeArgs {
+  const __nv_bfloat16* q = nullptr;   // [nq][Hq][d]
+  const __nv_bfloat16* Ck = nullptr;  // slot j of KV-head h at j * cst + h * d
+  const __nv_bfloat16* Cv = nullptr;
+  const float* beta = nullptr;        // [t][H] or null (no bias)
+  const __nv_bfloat16* Kf = nullptr;  // entry j of KV-head h at j * fst + h * d
+  const __nv_bfloat16* Vf = nullptr;
+  __nv_bfloat16* out = nullptr;       // [nq][Hq][d]
+  int64_t t = 0, S = 0, cst = 0, fst = 0;
+  int32_t nq = 0, Hq = 0, H = 0, d = 0;
+  float scale = 0.f;
+};
+size_t decode_workspace_bytes(int64_t rows, int64_t entries, int d);
+cudaError_t launch_decode_biased(const DecodeArgs& a, void* ws, cudaStream_t s);
+
 // Converts n bf16 values to fp16 in place (exact within the fp16 range; values below it
 // become fp16 subnormals, absolute error <= 2^-25).
 cudaError_t launch_bf16_to_f16(void* p, int64_t n, cudaStream_t s);

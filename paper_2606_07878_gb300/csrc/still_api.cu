@@ -61,6 +61,8 @@ struct LayerW {
   bf16* WhT = nullptr;   // [2d][D]
   double* omega_b = nullptr;  // [d/2] base-model RoPE frequencies (fp64)
   double* omega_c = nullptr;  // [D/2] compactor RoPE frequencies (fp64)
+  float* wbeta = nullptr;     // [D] beta head w_beta (fp32), when set
+  still_beta_config beta{};
   std::vector<void*> owned;
 };
 
@@ -489,7 +491,8 @@ still_status make_positions(const still_pos_segment* h_segments, int32_t n_segme
 struct OutSpec {
   bf16* ck;
   bf16* cv;
-  int64_t st, sh;  // element strides of [t, H, d] outputs (d contiguous)
+  int64_t st, sh;          // element strides of [t, H, d] outputs (d contiguous)
+  float* beta = nullptr;   // [t][H] per-slot logit bias (optional; needs a beta head)
 };
 
 // ws_fixed / ws_fixed_bytes: when set, the call runs in that caller-provided scratch and never
@@ -1024,6 +1027,14 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     const int bn = 2 * d <= 128 ? 128 : 256;
     TRY(run_gemm<STILL_K_HEADS>(ctx, bn, op(Z3, rows, 2 * D), op(L.WhT, 2 * d, D), p, e, 1, s));
   }
+  if (out.beta != nullptr) {  // beta = Z_out w_beta, shaped; T = the N entries replaced
+    const double off = L.beta.mass_match == 0
+                           ? 0.0
+                           : std::log((double)N / (double)t) +
+                                 (L.beta.mass_match == 2 ? (double)L.beta.log_x : 0.0);
+    KLAUNCH(STILL_K_BETA, launch_beta(reinterpret_cast<const bf16*>(Z3), t, H, D, L.wbeta,
+                                       L.beta.beta_max, (float)off, out.beta, s));
+  }
   return STILL_OK;
 }
 
@@ -1330,14 +1341,18 @@ still_status still_load_layer_weights_blocks(still_ctx* ctx, int32_t layer,
   return load_layer(ctx, layer, cfg, Z, blocks, Wkey, Wval, stream);
 }
 
-still_status still_compact_layer(still_ctx* ctx, int32_t layer, const void* K, const void* V,
-                                 const int64_t strides_kv[3],
-                                 const still_pos_segment* h_segments, int32_t n_segments,
-                                 int64_t N, int32_t t, void* Ck, void* Cv,
-                                 double* h_out_pos_start, double* h_out_pos_step,
-                                 int64_t* h_pos_offset, void* stream) {
+namespace {
+
+still_status compact_layer_impl(still_ctx* ctx, int32_t layer, const void* K, const void* V,
+                                const int64_t strides_kv[3],
+                                const still_pos_segment* h_segments, int32_t n_segments,
+                                int64_t N, int32_t t, void* Ck, void* Cv, float* beta,
+                                double* h_out_pos_start, double* h_out_pos_step,
+                                int64_t* h_pos_offset, void* stream) {
   const LayerW* L = nullptr;
   TRY(check_ctx_layer(ctx, layer, &L));
+  if (beta != nullptr && (L->wbeta == nullptr || (reinterpret_cast<uintptr_t>(beta) & 3)))
+    return L->wbeta == nullptr ? STILL_ERR_NOT_LOADED : STILL_ERR_ALIGNMENT;
   if (K == nullptr || V == nullptr || Ck == nullptr || Cv == nullptr || strides_kv == nullptr)
     return STILL_ERR_INVALID_ARG;
   if (N < 1 || t < 1 || t > N || t > L->cfg.t_max || N > (int64_t(1) << 30))
@@ -1351,11 +1366,97 @@ still_status still_compact_layer(still_ctx* ctx, int32_t layer, const void* K, c
   CK(cudaSetDevice(ctx->device));
   const int H = L->cfg.n_kv_heads, d = L->cfg.head_dim;
   OutSpec o{static_cast<bf16*>(Ck), static_cast<bf16*>(Cv), (int64_t)H * d, d};
+  o.beta = beta;
   TRY(compact_one(ctx, *L, single_source(K, V, strides_kv, N), pos, N, t, o,
                   static_cast<cudaStream_t>(stream)));
   if (h_out_pos_start) *h_out_pos_start = pos.pmin;
   if (h_out_pos_step) *h_out_pos_step = t > 1 ? (pos.pmax - pos.pmin) / (double)(t - 1) : 0.0;
   if (h_pos_offset) *h_pos_offset = N - t;
+  return STILL_OK;
+}
+
+}  // namespace
+
+still_status still_compact_layer(still_ctx* ctx, int32_t layer, const void* K, const void* V,
+                                 const int64_t strides_kv[3],
+                                 const still_pos_segment* h_segments, int32_t n_segments,
+                                 int64_t N, int32_t t, void* Ck, void* Cv,
+                                 double* h_out_pos_start, double* h_out_pos_step,
+                                 int64_t* h_pos_offset, void* stream) {
+  return compact_layer_impl(ctx, layer, K, V, strides_kv, h_segments, n_segments, N, t, Ck, Cv,
+                            nullptr, h_out_pos_start, h_out_pos_step, h_pos_offset, stream);
+}
+
+still_status still_compact_layer_beta(still_ctx* ctx, int32_t layer, const void* K,
+                                      const void* V, const int64_t strides_kv[3],
+                                      const still_pos_segment* h_segments, int32_t n_segments,
+                                      int64_t N, int32_t t, void* Ck, void* Cv, float* beta,
+                                      double* h_out_pos_start, double* h_out_pos_step,
+                                      int64_t* h_pos_offset, void* stream) {
+  if (beta == nullptr) return STILL_ERR_INVALID_ARG;
+  return compact_layer_impl(ctx, layer, K, V, strides_kv, h_segments, n_segments, N, t, Ck, Cv,
+                            beta, h_out_pos_start, h_out_pos_step, h_pos_offset, stream);
+}
+
+still_status still_set_beta_head(still_ctx* ctx, int32_t layer, const void* w_beta,
+                                 const still_beta_config* bc, void* stream) {
+  if (ctx == nullptr || w_beta == nullptr || bc == nullptr) return STILL_ERR_INVALID_ARG;
+  if (layer < 0 || layer >= (int32_t)ctx->layers.size() || !ctx->layers[layer].loaded)
+    return STILL_ERR_NOT_LOADED;
+  if (!(bc->beta_max >= 0.f) || !std::isfinite(bc->beta_max) || bc->mass_match < 0 ||
+      bc->mass_match > 2 || !std::isfinite(bc->log_x))
+    return STILL_ERR_INVALID_ARG;
+  LayerW& L = ctx->layers[layer];
+  CK(cudaSetDevice(ctx->device));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int D = L.cfg.d_latent;
+  if (L.wbeta == nullptr) TRY(dalloc(L, &L.wbeta, (size_t)D));
+  CK(launch_bias(static_cast<const bf16*>(w_beta), nullptr, D, L.wbeta, 0, s));
+  L.beta = *bc;
+  return STILL_OK;
+}
+
+still_status still_attend_biased(still_ctx* ctx, const void* q, int32_t nq, int32_t Hq,
+                                 const void* Ck, const void* Cv, const float* beta, int64_t t,
+                                 const void* Kfix, const void* Vfix, int64_t S, int32_t H,
+                                 int32_t d, float scale, void* out, void* stream) {
+  if (ctx == nullptr || q == nullptr || out == nullptr) return STILL_ERR_INVALID_ARG;
+  if (nq < 1 || H < 1 || Hq < H || Hq % H != 0 || t < 0 || S < 0 || t + S < 1 ||
+      (t > 0 && (Ck == nullptr || Cv == nullptr)) || (S > 0 && (Kfix == nullptr || Vfix == nullptr)))
+    return STILL_ERR_INVALID_ARG;
+  if ((d != 64 && d != 128 && d != 256) || (int64_t)nq * (Hq / H) > 64 ||
+      t + S > (int64_t(1) << 31) - 128)
+    return STILL_ERR_UNSUPPORTED;
+  if (!(scale >= 0.f) || !std::isfinite(scale)) return STILL_ERR_INVALID_ARG;
+  const uintptr_t al = reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(out) |
+                       reinterpret_cast<uintptr_t>(Ck) | reinterpret_cast<uintptr_t>(Cv) |
+                       reinterpret_cast<uintptr_t>(Kfix) | reinterpret_cast<uintptr_t>(Vfix);
+  if ((al & 15) || (reinterpret_cast<uintptr_t>(beta) & 3)) return STILL_ERR_ALIGNMENT;
+  CK(cudaSetDevice(ctx->device));
+  DecodeArgs a;
+  a.q = static_cast<const bf16*>(q);
+  a.Ck = static_cast<const bf16*>(Ck);
+  a.Cv = static_cast<const bf16*>(Cv);
+  a.beta = beta;
+  a.Kf = static_cast<const bf16*>(Kfix);
+  a.Vf = static_cast<const bf16*>(Vfix);
+  a.out = static_cast<bf16*>(out);
+  a.t = t;
+  a.S = S;
+  a.cst = (int64_t)H * d;
+  a.fst = (int64_t)H * d;
+  a.nq = nq;
+  a.Hq = Hq;
+  a.H = H;
+  a.d = d;
+  a.scale = scale > 0.f ? scale : 1.f / std::sqrt((float)d);
+  TRY(ensure_ws(ctx, decode_workspace_bytes((int64_t)nq * Hq, t + S, d)));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  ctx->prof.begin(STILL_K_DECODE, s);
+  cudaError_t r = launch_decode_biased(a, ctx->ws, s);
+  ctx->prof.end(STILL_K_DECODE, s);
+  ctx->prof.launches[STILL_K_DECODE] += 1;  // the merge kernel (begin counted the first)
+  if (r != cudaSuccess) return STILL_ERR_CUDA;
   return STILL_OK;
 }
 
@@ -1746,7 +1847,7 @@ const char* still_kernel_class_name(int32_t cls) {
   static const char* names[STILL_K_COUNT] = {
       "strip", "rope_tables", "keyproj", "q_rope", "scores", "softmax", "px", "px_split",
       "vo", "rmsnorm", "sa_proj", "sa_v", "sa_scores", "sa_softmax", "sa_pv", "sa_out",
-      "ffn1", "ffn2", "heads", "norms", "load", "ca_fused"};
+      "ffn1", "ffn2", "heads", "norms", "load", "ca_fused", "beta", "decode"};
   return cls >= 0 && cls < STILL_K_COUNT ? names[cls] : "unknown";
 }
 

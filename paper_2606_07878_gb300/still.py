@@ -30,13 +30,15 @@ EXPORTS = [
     "still_compact_layer_noalloc", "still_recompact_layer_ragged", "still_recompact_stack_ragged",
     "still_selftest_wait_timeout", "still_compact_stack_masked", "still_lookahead_pass_info",
     "still_lookahead_totals", "still_lookahead_compact_layer", "still_lookahead_compact_stack",
+    "still_set_beta_head", "still_compact_layer_beta", "still_attend_biased",
 ]
 
 NOALLOC_SCRATCH_MIB = 64  # STILL_NOALLOC_SCRATCH_MIB in include/still.h
 
 KERNEL_CLASSES = ["strip", "rope_tables", "keyproj", "q_rope", "scores", "softmax", "px",
                   "px_split", "vo", "rmsnorm", "sa_proj", "sa_v", "sa_scores", "sa_softmax",
-                  "sa_pv", "sa_out", "ffn1", "ffn2", "heads", "norms", "load", "ca_fused"]
+                  "sa_pv", "sa_out", "ffn1", "ffn2", "heads", "norms", "load", "ca_fused",
+                  "beta", "decode"]
 
 
 class StillError(RuntimeError):
@@ -73,6 +75,11 @@ BLOCK_WEIGHT_NAMES = ["Wq", "bq", "Wk", "bk", "Wv", "Wo", "Sq", "sbq", "Sk", "sb
 
 class BlockWeights(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in BLOCK_WEIGHT_NAMES]
+
+
+class BetaConfig(ctypes.Structure):
+    _fields_ = [("beta_max", ctypes.c_float), ("mass_match", ctypes.c_int32),
+                ("log_x", ctypes.c_float)]
 
 
 class LookaheadPass(ctypes.Structure):
@@ -142,6 +149,11 @@ def lib():
                                             ctypes.POINTER(P), ctypes.POINTER(P), PI64, PSEG,
                                             I32, I64, I32, ctypes.POINTER(P), ctypes.POINTER(P),
                                             PD, PD, PI64, P], ctypes.c_int),
+            "still_set_beta_head": ([P, I32, P, ctypes.POINTER(BetaConfig), P], ctypes.c_int),
+            "still_compact_layer_beta": ([P, I32, P, P, PI64, PSEG, I32, I64, I32, P, P, P, PD,
+                                          PD, PI64, P], ctypes.c_int),
+            "still_attend_biased": ([P, P, I32, I32, P, P, P, I64, P, P, I64, I32, I32,
+                                     ctypes.c_float, P, P], ctypes.c_int),
             "still_lookahead_pass_info": ([I64, I64, I32, ctypes.POINTER(LookaheadPass)],
                                           ctypes.c_int),
             "still_lookahead_totals": ([I64, I64, I32, PI64, PI64], ctypes.c_int),
@@ -305,6 +317,41 @@ def still_compact_stack_masked(ctx, mask, Ks, Vs, t: int, Cks, Cvs, segments=Non
                                             ctypes.byref(off), _stream(stream)),
            "still_compact_stack_masked")
     return ps.value, pst.value, off.value
+
+
+def still_set_beta_head(ctx, layer: int, w_beta, beta_max=0.0, mass_match=0, log_x=0.0,
+                        stream=None):
+    """w_beta [d_latent] bf16 CUDA tensor; shaping as in include/still.h."""
+    bc = BetaConfig(beta_max, mass_match, log_x)
+    _check(lib().still_set_beta_head(ctx, layer, _ptr(w_beta), ctypes.byref(bc), _stream(stream)),
+           "still_set_beta_head")
+
+
+def still_compact_layer_beta(ctx, layer: int, K, V, t: int, Ck, Cv, beta, segments=None,
+                             stream=None):
+    """still_compact_layer plus beta [t, H] fp32; returns (out_pos_start, out_pos_step,
+    pos_offset)."""
+    strides = (ctypes.c_int64 * 3)(*K.stride())
+    assert tuple(V.stride()) == tuple(K.stride()), "K and V must share strides"
+    seg, nseg = _segments(segments)
+    ps, pst, off = ctypes.c_double(), ctypes.c_double(), ctypes.c_int64()
+    _check(lib().still_compact_layer_beta(ctx, layer, _ptr(K), _ptr(V), strides, seg, nseg,
+                                          K.shape[0], t, _ptr(Ck), _ptr(Cv), _ptr(beta),
+                                          ctypes.byref(ps), ctypes.byref(pst), ctypes.byref(off),
+                                          _stream(stream)), "still_compact_layer_beta")
+    return ps.value, pst.value, off.value
+
+
+def still_attend_biased(ctx, q, Ck, Cv, beta, Kfix, Vfix, out, scale=0.0, stream=None):
+    """q [nq, Hq, d]; Ck, Cv [t, H, d]; beta [t, H] fp32 or None; Kfix, Vfix [S, H, d];
+    out [nq, Hq, d] (bf16 CUDA tensors)."""
+    nq, Hq, d = q.shape
+    t, H = Ck.shape[0], Ck.shape[1]
+    S = Kfix.shape[0]
+    _check(lib().still_attend_biased(ctx, _ptr(q), nq, Hq, _ptr(Ck) if t else None,
+                                     _ptr(Cv) if t else None, _ptr(beta), t,
+                                     _ptr(Kfix) if S else None, _ptr(Vfix) if S else None, S, H,
+                                     d, scale, _ptr(out), _stream(stream)), "still_attend_biased")
 
 
 def still_lookahead_pass_info(k: int, c: int, t: int) -> dict:
