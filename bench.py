@@ -27,15 +27,27 @@ sys.path.insert(0, ROOT)
 
 WORKLOAD = "qwen7b_8k"
 DEFAULT_T = {"qwen7b_8k": 1024, "qwen8b_32k": 2048, "gemma_128k": 655, "tiny_1k": 128,
-             "qwen3_4b_64k": 1311}
+             "qwen3_4b_64k": 1311, "qwen7b_8k_norope": 1024}
+
+
+def folded(wl):
+    """Whether the library folds W_K into the queries for this workload (no compactor RoPE, one
+    block, 2d <= 256, x~ = [x; 1] padded to 64 narrower than d_l); returns the padded width."""
+    d, D = wl["d"], wl["D"]
+    Kp = (2 * d + 1 + 63) // 64 * 64
+    ok = (not wl.get("compactor_rope", 1) and wl.get("n_blocks", 1) == 1 and d in (64, 128)
+          and Kp < D)
+    return Kp if ok else 0
 
 
 def describe(name, wl, t):
     nb = wl.get("n_blocks", 1)
     blocks = "" if nb == 1 else (f", {nb} blocks" + (" (CA in every block)"
                                                       if wl.get("cross_every_block", 1) else ""))
+    rope = "" if wl.get("compactor_rope", 1) else (
+        ", no compactor RoPE" + (" (W_K folded into the queries)" if folded(wl) else ""))
     return (f"{name}: {wl['L']} layers, N={wl['N']}, H_kv={wl['H']}, d={wl['d']}, "
-            f"D={wl['D']}, {wl['n']} heads, FFN {wl['F']}{blocks}, t={t} "
+            f"D={wl['D']}, {wl['n']} heads, FFN {wl['F']}{blocks}{rope}, t={t} "
             f"({round(wl['N'] / t)}x)")
 
 # DRAM traffic (read + write) per launch of the dominant kernel at a workload, from an ncu
@@ -44,9 +56,9 @@ def describe(name, wl, t):
 TRAFFIC = {
     "scores": {"files": ["tc_gemm.cuh", "epilogues.cuh"], "kernel_hash": None,
                "bytes_per_launch": None, "workload": None, "profile": None},
-    # 1.280 GB read + 0.132 GB written per launch (profiles/ca_fused_qwen7b_8k_t1024.md)
-    "ca_fused": {"files": ["ca_flash.cuh", "ptx.cuh"], "kernel_hash": "e8fbfe01d9bcd37f",
-                 "bytes_per_launch": 1.4117e9, "workload": ("qwen7b_8k", 1024),
+    # 1.285 GB read + 0.132 GB written per launch (profiles/ca_fused_qwen7b_8k_t1024.md)
+    "ca_fused": {"files": ["ca_flash.cuh", "ptx.cuh"], "kernel_hash": "de7c73bd49c1000d",
+                 "bytes_per_launch": 1.4171e9, "workload": ("qwen7b_8k", 1024),
                  "profile": "profiles/ca_fused_qwen7b_8k_t1024.md"},
 }
 
@@ -160,14 +172,19 @@ def algorithmic_flops(wl, t, N):
     H, d, D, n, F = wl["H"], wl["d"], wl["D"], wl["n"], wl["F"]
     nb = wl.get("n_blocks", 1)
     n_ca = nb if wl.get("cross_every_block", 1) else 1  # blocks with cross-attention
-    ca = (2 * N * H * 2 * d * n * D + 2 * t * N * H * n * D + 2 * t * N * H * n * 2 * d
+    # With the fold the keys are never projected: the logits contract over x~ (width Kp) and
+    # the key norms are x~ G x~ (Kp^2 per token and head).
+    Kp = folded(wl)
+    kw = Kp if Kp else D
+    kproj = 2 * N * H * n * Kp * Kp if Kp else 2 * N * H * 2 * d * n * D
+    ca = (kproj + 2 * t * N * H * n * kw + 2 * t * N * H * n * 2 * d
           + 2 * t * H * n * 2 * d * D + 2 * t * H * n * D * D)
     sa = 6 * t * H * D * n * D + 4 * t * t * H * n * D + 2 * t * H * n * D * D
     # The last block's cross-attention is one fused kernel when 2d <= 256; earlier blocks
     # (and every block at 2d = 512) take the scores GEMM.
     fused_last = 2 * d <= 256 and (nb == 1 or wl.get("cross_every_block", 1))
     return {"total": n_ca * ca + nb * (sa + 4 * t * H * D * F) + 4 * t * H * D * d,
-            "scores": n_ca * 2 * t * N * H * n * D, "px": n_ca * 2 * t * N * H * n * 2 * d,
+            "scores": n_ca * 2 * t * N * H * n * kw, "px": n_ca * 2 * t * N * H * n * 2 * d,
             "scores_gemm": (n_ca - (1 if fused_last else 0)) * 2 * t * N * H * n * D}
 
 
@@ -185,6 +202,7 @@ def run_cpu_baseline(wl, t, budget_s=30.0):
     one_head = fl["total"] / wl["H"]
     W = synth.gen_weights(wl, 0, t, "cpu")
     cfg = O.cfg_from_workload(wl, n_blocks=wl.get("n_blocks", 1),
+                              compactor_rope=bool(wl.get("compactor_rope", 1)),
                               cross_every_block=bool(wl.get("cross_every_block", 1)))
     Wf = O.as_f64(W)
     if one_head < 2.5e12:

@@ -47,9 +47,9 @@ typedef enum {
 typedef struct still_ctx still_ctx; /* opaque: weight copies, precompute, workspace */
 
 /* One layer's compactor hyperparameters (App. A, "Canonical configuration summary").
- * Implemented: n_blocks = 1, cross_every_block = 1, n_cross_heads = n_self_heads,
+ * Implemented: n_blocks 1 or 2, cross_every_block 0 or 1, n_cross_heads = n_self_heads,
  * d_latent % 256 == 0, head_dim in {64, 128, 256}, ffn_dim % 64 == 0 (or 0 = no FFN),
- * compactor_rope = 1, rope_fix = 1. Other values return STILL_ERR_UNSUPPORTED. */
+ * compactor_rope 0 or 1, rope_fix = 1. Other values return STILL_ERR_UNSUPPORTED. */
 typedef struct {
   int32_t n_kv_heads;        /* H: KV-heads of the base model */
   int32_t head_dim;          /* d: base model head dim */
@@ -61,7 +61,8 @@ typedef struct {
   int32_t cross_every_block; /* 1 = canonical (CA in every block), 0 = resampler */
   int32_t t_max;             /* rows of each latent bank; a call uses rows [0, t) */
   int32_t final_norm;        /* RMSNorm before the output heads (0 = off, the default) */
-  int32_t compactor_rope;    /* apply the compactor's RoPE in cross-attention */
+  int32_t compactor_rope;    /* apply the compactor's RoPE in cross-attention (0: no RoPE; see
+                                still_set_key_fold) */
   int32_t rope_fix;          /* un-rotate cached keys / re-rotate C_k */
   double rope_theta;         /* base model RoPE base */
   double rope_theta_compactor; /* compactor RoPE base (canonical 10) */
@@ -398,6 +399,14 @@ still_status still_set_workspace_limit(still_ctx* ctx, size_t bytes);
  * instead and form q^ for the call's t latents inside each compaction call, with the same
  * kernels and the same results. Default 2 GiB; applies to later still_load_layer_weights. */
 still_status still_set_qhat_eager_limit(still_ctx* ctx, size_t bytes);
+
+/* Layers without compactor RoPE (compactor_rope = 0) fold the key projection into the
+ * queries when they have one block, 2d <= 256, precomputed queries and 2d + 1 (padded to a
+ * multiple of 64) below d_latent: with x~ = [x; 1] and W~ = [W_K; b_K], the logits are
+ * d_l (x~ . W~ q^) / |x~ W~| and |x~ W~|^2 = x~ (W~ W~^T) x~^T, so the cached tokens are
+ * never projected to d_latent (App. A, "Cross-attention": the logits of QK-normed heads).
+ * enable = 0 keeps the explicit projection for layers loaded afterwards (default 1). */
+still_status still_set_key_fold(still_ctx* ctx, int32_t enable);
 
 /* Synchronizes `stream`, then reports (and clears) the device error record:
  * STILL_ERR_TIMEOUT if a kernel's bounded wait expired, STILL_ERR_CUDA if the stream

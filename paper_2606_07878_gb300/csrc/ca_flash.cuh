@@ -30,6 +30,10 @@ struct FlashParams {
   int64_t Np = 0;           // key pitch of X^T hi / lo (multiple of 64, >= N, zero padded)
   int32_t nb = 0, bdiv = 1; // batches; KV-head of batch b is h0 + b / bdiv
   int32_t xbase_row = 0;    // X^T row of feature 0 of KV-head h0
+  // Q rows of batch b start at q_row0 + b * q_pitch (q_pitch 0: t). K rows of batch b start at
+  // k_row0 + b * N, or at k_row0 + (b / kdiv) * N when kdiv > 0 (keys shared by kdiv batches).
+  int64_t q_row0 = 0, k_row0 = 0;
+  int32_t q_pitch = 0, kdiv = 0;
   int32_t tiles_m = 0, tiles_k = 0, nsplit = 1, nunits = 0;
   const float* kinv = nullptr;  // [nb][N]: scale / |k~| per key
   float* O = nullptr;           // [nsplit][nb][t][2d] unnormalised
@@ -164,8 +168,10 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
       };
       for (int u = blockIdx.x; u < f.nunits && !bad && !*abort_flag; u += gridDim.x) {
         const FlashUnit w = flash_unit(f, u);
-        const int32_t qrow = w.b * f.t + w.tm * kBM;
-        const int32_t krow = w.b * f.N;
+        const int32_t qrow =
+            (int32_t)(f.q_row0 + (int64_t)w.b * (f.q_pitch > 0 ? f.q_pitch : f.t)) + w.tm * kBM;
+        const int32_t krow =
+            (int32_t)(f.k_row0 + (int64_t)(f.kdiv > 0 ? w.b / f.kdiv : w.b) * f.N);
         const int32_t xrow = f.xbase_row + (w.b / f.bdiv) * D2;
         const int J = w.j1 - w.j0;
         for (int jj = 0; jj <= J && !bad; ++jj) {

@@ -534,6 +534,54 @@ struct EpiRopeCT {
 // position of latent j; columns [d, 2d) = Z_out W_val. Rows r = h * t + j. bf16 stores into
 // the caller's C_k / C_v with element strides (st, sh). rot[j][m] = (cos, sin)(p_j * omega_m),
 // a table formed once per call with the angle reduced modulo 2 pi in fp64.
+// Folded key path (no compactor RoPE): |k~_n|^2 = x~_n G x~_n^T with G = W~ W~^T. The GEMM
+// gives Y = x~ G (rows = tokens of one KV-head, columns = the Kp entries of one cross head);
+// the epilogue dots each 32-column chunk of Y with the same columns of x~ (hi + lo, read back
+// from global memory) and stores the partial, part-major: part[(b * Kp/32 + chunk) * Ntok + n].
+struct EpiQuad {
+  static constexpr int kWarps = 8;   // two per lane quarter: alternating 32-column chunks
+  static constexpr int kStages = 0;
+  static constexpr int kStoreBufs = 1;
+  float* part = nullptr;
+  const __nv_bfloat16* xt = nullptr;  // x~ rows [hi | lo], pitch 2 Kp, of the group's first KV-head
+  int64_t Ntok = 0;
+  int32_t Kp = 0;
+  int32_t tile_cols_ = 256;
+
+  __device__ void prefetch(const GemmParams&, const TileCoord&, int, int) const {}
+
+  __device__ void operator()(const GemmParams& p, const TileCoord& tc, int row, uint32_t taddr,
+                             int half, uint4*, const CUtensorMap*) const {
+    const int r = tc.tm * kBM + row;
+    const bool rvalid = r < p.M;
+    const int parts = Kp / 32;
+    const __nv_bfloat16* xr =
+        xt + ((int64_t)(tc.b / p.bdiv) * Ntok + (rvalid ? r : 0)) * 2 * Kp;
+    for (int cc = 32 * half; cc < tile_cols_; cc += 64) {
+      float v[32];
+      tmem_ld32(taddr + (uint32_t)cc, v);  // warp-collective: before any per-lane exit
+      const int c0 = tc.tn * tile_cols_ + cc;
+      if (c0 >= p.N || !rvalid) continue;
+      const uint4* hp = reinterpret_cast<const uint4*>(xr + c0);
+      const uint4* lp = reinterpret_cast<const uint4*>(xr + Kp + c0);
+      float acc = 0.f;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint4 hq = hp[q], lq = lp[q];
+        const uint32_t hw[4] = {hq.x, hq.y, hq.z, hq.w}, lw[4] = {lq.x, lq.y, lq.z, lq.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const float2 h2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&hw[k]));
+          const float2 l2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&lw[k]));
+          acc = fmaf(v[8 * q + 2 * k], h2.x + l2.x, acc);
+          acc = fmaf(v[8 * q + 2 * k + 1], h2.y + l2.y, acc);
+        }
+      }
+      part[((int64_t)tc.b * parts + c0 / 32) * Ntok + r] = acc;
+    }
+  }
+};
+
 struct EpiHeads {
   static constexpr int kWarps = 8;
   static constexpr int kStages = 0;

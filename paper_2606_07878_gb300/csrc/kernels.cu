@@ -50,9 +50,11 @@ __device__ __forceinline__ void load8(const __nv_bfloat16* p, bool vec, float (&
 // (fp16 hi for all 2d features, fp16 lo for the key half; the value half's lo is exactly zero
 // and is never read). Rows are moved in 16-byte pieces; the transpose for XT goes through
 // shared memory with an odd word pitch (conflict-free column reads).
+// Kp > 0 writes X in the layout of the folded key path instead: rows of 2 Kp elements,
+// [x~ hi | x~ lo] with x~ = [unRoPE(K) | V | 1 | 0 ...] (Kp >= 2d + 1, a multiple of 64).
 __global__ void __launch_bounds__(256) strip_kernel(KVSource src, int64_t N, int H, int d,
                                                     PosSegs segs, const double* __restrict__ omega,
-                                                    int rope_fix, int vec, int x16,
+                                                    int rope_fix, int vec, int x16, int Kp,
                                                     __nv_bfloat16* __restrict__ X,
                                                     __half* __restrict__ XT, int64_t Np,
                                                     float2* __restrict__ gd, double pmin, int G) {
@@ -84,7 +86,8 @@ __global__ void __launch_bounds__(256) strip_kernel(KVSource src, int64_t N, int
     rot[it] = make_float2(cw, sw);
   }
   __syncthreads();
-  const int d3 = 3 * d;
+  const int d3 = Kp > 0 ? 2 * Kp : 3 * d;  // X row pitch
+  const int lo0 = Kp > 0 ? Kp : 2 * d;     // column of the key lo part
   const int64_t ld = 2 * Np;
   const int kg = half / 8, vg = d / 8;  // 8-element groups per token: key pairs, values
   for (int h = 0; h < H; ++h) {
@@ -121,15 +124,15 @@ __global__ void __launch_bounds__(256) strip_kernel(KVSource src, int64_t N, int
         if (vec) {
           *reinterpret_cast<uint4*>(xr + m0) = make_uint4(ah[0], ah[1], ah[2], ah[3]);
           *reinterpret_cast<uint4*>(xr + half + m0) = make_uint4(bh[0], bh[1], bh[2], bh[3]);
-          *reinterpret_cast<uint4*>(xr + 2 * d + m0) = make_uint4(al[0], al[1], al[2], al[3]);
-          *reinterpret_cast<uint4*>(xr + 2 * d + half + m0) = make_uint4(bl[0], bl[1], bl[2], bl[3]);
+          *reinterpret_cast<uint4*>(xr + lo0 + m0) = make_uint4(al[0], al[1], al[2], al[3]);
+          *reinterpret_cast<uint4*>(xr + lo0 + half + m0) = make_uint4(bl[0], bl[1], bl[2], bl[3]);
         } else {
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
             reinterpret_cast<uint32_t*>(xr + m0)[k] = ah[k];
             reinterpret_cast<uint32_t*>(xr + half + m0)[k] = bh[k];
-            reinterpret_cast<uint32_t*>(xr + 2 * d + m0)[k] = al[k];
-            reinterpret_cast<uint32_t*>(xr + 2 * d + half + m0)[k] = bl[k];
+            reinterpret_cast<uint32_t*>(xr + lo0 + m0)[k] = al[k];
+            reinterpret_cast<uint32_t*>(xr + lo0 + half + m0)[k] = bl[k];
           }
         }
       } else {
@@ -178,6 +181,18 @@ __global__ void __launch_bounds__(256) strip_kernel(KVSource src, int64_t N, int
 #pragma unroll
       for (int e = 0; e < 8; e += 2)
         *reinterpret_cast<__half2*>(hr + e) = __floats2half2_rn(v[e], v[e + 1]);
+    }
+    if (Kp > 0) {  // folded layout: [.. | 1 | 0 ...] after the values, zeros after the key lo
+      const int nc = (Kp - 2 * d) / 8, nz = (Kp - d) / 8;  // 16-byte groups per token
+      for (int it = threadIdx.x; it < kStripTok * (nc + nz); it += blockDim.x) {
+        const int tok = it / (nc + nz), q = it % (nc + nz);
+        const int64_t n = n0 + tok;
+        if (n >= N) continue;
+        __nv_bfloat16* xr = X + ((int64_t)h * N + n) * d3;
+        uint4 val = make_uint4(0, 0, 0, 0);
+        if (q == 0) val.x = x16 ? 0x3C00u : 0x3F80u;  // 1.0 in the first element (fp16 / bf16)
+        *reinterpret_cast<uint4*>(xr + (q < nc ? 2 * d + 8 * q : Kp + d + 8 * (q - nc))) = val;
+      }
     }
     __syncthreads();
     // XT: feature rows of 32 tokens, 8 tokens (16 B) per store; hi rows [0, 2d), lo rows [0, d)
@@ -579,7 +594,7 @@ __global__ void inv_norms_kernel(const float* __restrict__ parts, int64_t nvec, 
   const float* p = parts + (i / block) * nparts * block + i % block;
   float s = 0.f;
   for (int k = 0; k < nparts; ++k) s += p[k * block];  // fixed order
-  out[i] = alpha / fmaxf(sqrtf(s), eps);
+  out[i] = alpha / fmaxf(sqrtf(fmaxf(s, 0.f)), eps);  // a quadratic form may round below 0
 }
 
 __global__ void transpose_kernel(const __nv_bfloat16* __restrict__ in, int64_t R, int64_t C,
@@ -607,6 +622,41 @@ __global__ void bias_kernel(const __nv_bfloat16* in, const __nv_bfloat16* in2, i
   const int64_t src = perm_D > 0 ? pair_chunk_src((int)c, perm_D) : c;
   out[c] = __bfloat162float(in[src]);
   if (in2 != nullptr) out[C + c] = __bfloat162float(in2[src]);
+}
+
+// ---------------------------------------------------------------- folded key projection
+
+// Wt[i][c][j] = W_K,i[c][j] (c < 2d), b_K,i[j] (c = 2d), 0 (2d < c < Kp): the rows of
+// W~_i = [W_K,i ; b_K,i], from the pair-chunk-ordered transposed copy WkT[i D + j][c] and
+// bias bk[i D + j] (fp32 copies of bf16 values, so the conversion back is exact).
+__global__ void fold_weights_kernel(const __nv_bfloat16* __restrict__ WkT,
+                                    const float* __restrict__ bk, int n, int D, int d2, int Kp,
+                                    __nv_bfloat16* __restrict__ Wt) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (int64_t)n * Kp * D) return;
+  const int j = (int)(idx % D);
+  const int c = (int)((idx / D) % Kp);
+  const int i = (int)(idx / ((int64_t)D * Kp));
+  const int64_t col = (int64_t)i * D + j;
+  __nv_bfloat16 v = __float2bfloat16_rn(0.f);
+  if (c < d2)
+    v = WkT[col * d2 + c];
+  else if (c == d2)
+    v = __float2bfloat16_rn(bk[col]);
+  Wt[idx] = v;
+}
+
+// out[r] = [bf16 hi(x) | bf16 lo(x)] of fp32 rows x of width C.
+__global__ void f32_hilo_kernel(const float* __restrict__ x, int64_t rows, int C,
+                                __nv_bfloat16* __restrict__ out) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= rows * C) return;
+  const int64_t r = idx / C;
+  const int c = (int)(idx % C);
+  __nv_bfloat16 hi, lo;
+  split_hilo(x[idx], hi, lo);
+  out[r * 2 * C + c] = hi;
+  out[r * 2 * C + C + c] = lo;
 }
 
 // ----------------------------------------------------------------------- beta channel
@@ -781,6 +831,20 @@ cudaError_t launch_decode_biased(const DecodeArgs& a, void* ws, cudaStream_t s) 
   return cudaGetLastError();
 }
 
+cudaError_t launch_fold_weights(const __nv_bfloat16* WkT, const float* bk, int n, int D, int d2,
+                                int Kp, __nv_bfloat16* Wt, cudaStream_t s) {
+  const int64_t total = (int64_t)n * Kp * D;
+  fold_weights_kernel<<<blocks_for(total, 256), 256, 0, s>>>(WkT, bk, n, D, d2, Kp, Wt);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_f32_hilo(const float* x, int64_t rows, int C, __nv_bfloat16* out,
+                            cudaStream_t s) {
+  if (rows == 0) return cudaSuccess;
+  f32_hilo_kernel<<<blocks_for(rows * C, 256), 256, 0, s>>>(x, rows, C, out);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_beta(const __nv_bfloat16* Z, int t, int H, int D, const float* w,
                         float beta_max, float offset, float* beta, cudaStream_t s) {
   const int64_t rows = (int64_t)H * t;
@@ -791,8 +855,10 @@ cudaError_t launch_beta(const __nv_bfloat16* Z, int t, int H, int D, const float
 
 cudaError_t launch_strip(const KVSource& src, int64_t N, int H, int d, const PosSegs& segs,
                          const double* omega, int rope_fix, __nv_bfloat16* X, __half* XT,
-                         int64_t Np, float2* gd, double pmin, int G, int x16, cudaStream_t s) {
-  if (d % 16 != 0 || Np % kStripTok != 0) return cudaErrorInvalidValue;
+                         int64_t Np, float2* gd, double pmin, int G, int x16, int Kp,
+                         cudaStream_t s) {
+  if (d % 16 != 0 || Np % kStripTok != 0 || (Kp != 0 && (Kp % 64 != 0 || Kp < 2 * d + 1)))
+    return cudaErrorInvalidValue;
   const size_t smem = (size_t)kStripTok * (d / 2) * sizeof(float2) +
                       (size_t)kStripTok * ((2 * d + 2) + (d + 2)) * 2;
   auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
@@ -806,7 +872,7 @@ cudaError_t launch_strip(const KVSource& src, int64_t N, int H, int d, const Pos
     attr = true;
   }
   strip_kernel<<<(unsigned)(Np / kStripTok), 256, smem, s>>>(src, N, H, d, segs, omega, rope_fix,
-                                                             vec, x16, X, XT, Np, gd, pmin, G);
+                                                             vec, x16, Kp, X, XT, Np, gd, pmin, G);
   return cudaGetLastError();
 }
 

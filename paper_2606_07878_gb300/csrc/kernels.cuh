@@ -27,9 +27,21 @@ struct KVSource {
 // Also gd[n] = (g, p_n - (pmin + g * kPosGrain)) with g = floor((p_n - pmin) / kPosGrain)
 // clamped to [0, G): the compactor-RoPE coarse index and residual of token n (n < N).
 // x16: X in fp16 (hi | key lo as fp16 hi / lo, values as fp16) instead of bf16.
+// Kp > 0: X rows of 2 Kp elements, [x~ hi | x~ lo] with x~ = [unRoPE(K) | V | 1 | 0 ...]
+// (the folded key path; Kp a multiple of 64, >= 2d + 1).
 cudaError_t launch_strip(const KVSource& src, int64_t N, int H, int d, const PosSegs& segs,
                          const double* omega, int rope_fix, __nv_bfloat16* X, __half* XT,
-                         int64_t Np, float2* gd, double pmin, int G, int x16, cudaStream_t s);
+                         int64_t Np, float2* gd, double pmin, int G, int x16, int Kp,
+                         cudaStream_t s);
+
+// Folded key projection (no compactor RoPE): Wt [n][Kp][D] bf16, rows of W~_i = [W_K,i; b_K,i]
+// padded with zero rows to Kp, columns in pair-chunk order (from WkT [nD][2d] and bk [nD]).
+cudaError_t launch_fold_weights(const __nv_bfloat16* WkT, const float* bk, int n, int D, int d2,
+                                int Kp, __nv_bfloat16* Wt, cudaStream_t s);
+
+// Rows of fp32 x [rows][C] -> bf16 [rows][2C]: hi | lo.
+cudaError_t launch_f32_hilo(const float* x, int64_t rows, int C, __nv_bfloat16* out,
+                            cudaStream_t s);
 
 // Per-slot logit bias from the final latent state Z ([H * t][2D] bf16 hi | lo, rows h * t + j):
 // beta[j][h] = sat(Z_hi + Z_lo) . w) + offset, sat(x) = beta_max tanh(x / beta_max) when

@@ -61,6 +61,13 @@ struct LayerW {
   bf16* WhT = nullptr;   // [2d][D]
   double* omega_b = nullptr;  // [d/2] base-model RoPE frequencies (fp64)
   double* omega_c = nullptr;  // [D/2] compactor RoPE frequencies (fp64)
+  // Without compactor RoPE the key projection folds into the queries (fold): the scores are
+  // x~ . u with x~ = [x; 1] and u = W~ q^ (W~ = [W_K; b_K]), the key norms x~ G x~ with
+  // G = W~ W~^T, so the N-token cache is never projected.
+  bool fold = false;
+  int Kp = 0;                 // width of x~ padded to a multiple of 64
+  bf16* U = nullptr;          // [H][n][t_max][2 Kp]: u = W~_i q^ as hi | lo
+  bf16* G = nullptr;          // [n][Kp][2 Kp]: W~_i W~_i^T as hi | lo
   float* wbeta = nullptr;     // [D] beta head w_beta (fp32), when set
   still_beta_config beta{};
   std::vector<void*> owned;
@@ -158,6 +165,7 @@ struct still_ctx {
   size_t ws_bytes = 0;
   size_t ws_limit = size_t(48) << 30;
   size_t qhat_eager_limit = size_t(2) << 30;
+  bool key_fold = true;  // fold W_K into the queries where the layer allows it
   Profiler prof;
 };
 
@@ -201,7 +209,8 @@ still_status check_cfg(const still_layer_config* c) {
       (c->cross_every_block != 0 && c->cross_every_block != 1) ||
       c->n_cross_heads != c->n_self_heads ||
       c->d_latent % 256 != 0 || !(c->head_dim == 64 || c->head_dim == 128 || c->head_dim == 256) ||
-      c->ffn_dim % 64 != 0 || c->compactor_rope != 1 || c->rope_fix != 1 ||
+      c->ffn_dim % 64 != 0 || (c->compactor_rope != 0 && c->compactor_rope != 1) ||
+      c->rope_fix != 1 ||
       (c->final_norm != 0 && c->final_norm != 1))
     return STILL_ERR_UNSUPPORTED;
   return STILL_OK;
@@ -317,7 +326,7 @@ struct Plan {
 
 size_t a256(size_t x) { return (x + 255) & ~size_t(255); }
 
-bool make_plan(const still_layer_config& c, bool lazy_q, int64_t N, int t, double pmin,
+bool make_plan(const still_layer_config& c, bool lazy_q, int Kp, int64_t N, int t, double pmin,
                double pmax, size_t limit, Plan& P) {
   P.H = c.n_kv_heads;
   P.d = c.head_dim;
@@ -338,7 +347,7 @@ bool make_plan(const still_layer_config& c, bool lazy_q, int64_t N, int t, doubl
     off += a256(bytes);
     return o;
   };
-  P.oX = take(H * N * 3 * d * 2);
+  P.oX = take(H * N * std::max<int64_t>(3 * d, 2 * Kp) * 2);  // Kp > 0: the folded x~ rows
   P.oXT = take(H * 2 * d * 2 * P.Np * 2);
   P.oCoarse = take((size_t)(P.G + kPosGrain) * (D / 2) * 8);  // coarse rows, then fine rows
   P.oOmega = take((D / 2) * 4);
@@ -357,9 +366,11 @@ bool make_plan(const still_layer_config& c, bool lazy_q, int64_t N, int t, doubl
   P.lazy_q = lazy_q;
   P.oZn = lazy_q ? take(H * T * 2 * D * 2) : 0;  // RMSNorm(Z) hi | lo for the call's t latents
   const size_t fixed = off;
-  P.kb_b = a256(N * 2 * D * 2);
-  P.kss_b = a256(N * 4 * (EpiRopeCT<false>::kParts * (D / 256) + 1));  // |k~|^2 partials + inverses
-  P.q_b = a256(T * 2 * D * 2);
+  // |k~|^2 partials + inverses; the folded path needs neither k nor per-call q
+  const int64_t kparts = std::max<int64_t>(EpiRopeCT<false>::kParts * (D / 256), Kp / 32);
+  P.kb_b = Kp > 0 ? 0 : a256(N * 2 * D * 2);
+  P.kss_b = a256(N * 4 * (kparts + 1));
+  P.q_b = Kp > 0 ? 0 : a256(T * 2 * D * 2);
   // The fused kernel holds fp16 probabilities and bf16 hi | lo q, k; a block that feeds
   // another needs its probabilities in hi | lo and fp16 hi | lo q, k (its cross-attention
   // output steers the next block's queries), so such blocks take the scores + P X kernels
@@ -503,6 +514,8 @@ bool queries_per_call(const LayerW& L) {
   return L.qhat_lazy || (L.cfg.n_blocks > 1 && L.cfg.cross_every_block);
 }
 
+int fold_kp(const LayerW& L) { return L.fold ? L.Kp : 0; }
+
 still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
                          const Positions& pos, int64_t N, int t, const OutSpec& out,
                          cudaStream_t s, uint8_t* ws_fixed = nullptr,
@@ -510,7 +523,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
   const still_layer_config& c = L.cfg;
   Plan P;
   const size_t limit = ws_fixed != nullptr ? ws_fixed_bytes : ctx->ws_limit;
-  if (!make_plan(c, queries_per_call(L), N, t, pos.pmin, pos.pmax, limit, P))
+  if (!make_plan(c, queries_per_call(L), fold_kp(L), N, t, pos.pmin, pos.pmax, limit, P))
     return STILL_ERR_OOM;
   if (ws_fixed == nullptr) TRY(ensure_ws(ctx, P.total));
   uint8_t* ws = ws_fixed != nullptr ? ws_fixed : static_cast<uint8_t*>(ctx->ws);
@@ -536,7 +549,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
   void* Z3 = ws + P.oZ3;
 
   KLAUNCH(STILL_K_STRIP, launch_strip(src, N, H, d, pos.segs, L.omega_b, c.rope_fix, X, XT, Np,
-                                      gd, pos.pmin, P.G, L.f16 ? 1 : 0, s));
+                                      gd, pos.pmin, P.G, L.f16 ? 1 : 0, fold_kp(L), s));
   const int w_fmt = L.f16 ? 0 : 1;    // operand format of X, RMSNorm(Z), W_K and W_Q products
   const int zn_mode = L.f16 ? 2 : 1;  // RMSNorm(Z) as fp16 or bf16 hi | lo
   KLAUNCH(STILL_K_TABLES, launch_rope_tables(coarse, omega, P.G, D, pos.pmin, L.omega_c, s));
@@ -584,7 +597,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     uint8_t* g = ws + P.oCA;
     bf16* kb = reinterpret_cast<bf16*>(g);
     g += P.kb_b * nbl;
-    const int kparts = EpiRopeCT<false>::kParts * (D / 256);
+    const int kparts = L.fold ? L.Kp / 32 : EpiRopeCT<false>::kParts * (D / 256);
     float* kss = reinterpret_cast<float*>(g);        // [nbl][N][kparts]
     float* kinv = kss + (size_t)nbl * N * kparts;    // [nbl][N]
     g += P.kss_b * nbl;
@@ -636,8 +649,23 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       q_tmax = t;
       q_b0 = 0;
     }
-    // keyproj: rows = tokens of heads [h0, h0+nh), columns = cross heads [i0, i0+ni)
-    {
+    if (L.fold) {
+      // |k~|^2 = x~ G_i x~: Y = x~ G_i (3-pass hi / lo, K = Kp), dotted with x~ in the epilogue
+      const int Kp = L.Kp;
+      GemmParams p = gp((int)N, Kp, nbl, ni);
+      p.a_r1 = N;    // x~ rows of KV-head h0 + b / ni
+      p.b_r0 = Kp;   // G rows of cross head i0 + b % ni
+      add_pass(p, 0, 0, (int)(h0 * N), i0 * Kp, Kp);
+      add_pass(p, 0, Kp, (int)(h0 * N), i0 * Kp, Kp);
+      add_pass(p, Kp, 0, (int)(h0 * N), i0 * Kp, Kp);
+      EpiQuad e;
+      e.part = kss;
+      e.xt = X + (size_t)h0 * N * 2 * Kp;
+      e.Ntok = N;
+      e.Kp = Kp;
+      TRY(run_gemm256<STILL_K_KEYPROJ>(ctx, op(X, (int64_t)H * N, 2 * Kp),
+                                       op(L.G, (int64_t)n * Kp, 2 * Kp), p, e, 1, s));
+    } else {  // keyproj: rows = tokens of heads [h0, h0+nh), columns = cross heads [i0, i0+ni)
       GemmParams p = gp((int)N, ni * D, nh, 1);
       p.a_r1 = N;
       p.n_fast = 1;  // X rows of a KV-head can exceed L2; the W_K block fits
@@ -669,7 +697,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
         fill(e);
         TRY(run_gemm256<STILL_K_KEYPROJ>(ctx, xop, wop, p, e, w_fmt, s, &kv));
       }
-    }
+    }  // key projection
     // scale / |k~_n| per key (the d_l logit scale folded in)
     // A block that feeds another forms q and k as fp16 hi / lo (about 22 bits; bf16 hi / lo
     // keeps 16): its logits steer the next block's queries. q is unit-norm, so it is scaled by
@@ -677,8 +705,10 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     const float qscale = exact ? std::exp2(std::round(0.5 * std::log2((double)D))) : 1.f;
     KLAUNCH(STILL_K_NORMS, launch_inv_norms(kss, (int64_t)nbl * N, kparts, N, c.l2_eps,
                                             scale / qscale, kinv, s));
-    KLAUNCH(STILL_K_QROPE, launch_q_rope(qsrc, q_tmax, q_b0, nbl, t, D, qstart, qstep, L.omega_c,
-                                         c.compactor_rope, qhl, exact ? 1 : 0, qscale, s));
+    if (!L.fold)
+      KLAUNCH(STILL_K_QROPE, launch_q_rope(qsrc, q_tmax, q_b0, nbl, t, D, qstart, qstep,
+                                           L.omega_c, c.compactor_rope, qhl, exact ? 1 : 0,
+                                           qscale, s));
     if (P.flash && !exact) {
       // S, the online softmax and P X in one kernel; per-split partials merged in order.
       float2* fst = stp;  // [nsplit][nbl * t] (the statistics region of this path)
@@ -700,8 +730,18 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       fp.O = O;
       fp.stats = fst;
       fp.err = ctx->err;
-      const Operand2D qop = op(qhl, (int64_t)nbl * t, 2 * D);
-      const Operand2D kop = op(kb, (int64_t)nbl * N, 2 * D);
+      Operand2D qop = op(qhl, (int64_t)nbl * t, 2 * D);
+      Operand2D kop = op(kb, (int64_t)nbl * N, 2 * D);
+      if (L.fold) {  // q := u (precomputed, t_max rows per (h, i)), k := x~ shared per KV-head
+        const int Kp = L.Kp;
+        fp.D = Kp;
+        fp.q_row0 = ((int64_t)h0 * n + i0) * c.t_max;
+        fp.q_pitch = c.t_max;
+        fp.k_row0 = (int64_t)h0 * N;
+        fp.kdiv = ni;
+        qop = op(L.U, (int64_t)H * n * c.t_max, 2 * Kp);
+        kop = op(X, (int64_t)H * N, 2 * Kp);
+      }
       const Operand2D xop = op(XT, (int64_t)H * 2 * d, 2 * Np);
       ctx->prof.begin(STILL_K_CA_FUSED, s);
       cudaError_t r = d == 64 ? launch_ca_flash<128>(qop, kop, xop, fp, ctx->nsm, s)
@@ -1095,6 +1135,11 @@ still_status load_layer(still_ctx* ctx, int32_t layer, const still_layer_config*
   L.blk.resize(NB);
   L.qhat_lazy = (size_t)H * n * T * D * sizeof(float) > ctx->qhat_eager_limit;
   L.f16 = NB > 1;
+  // The folded key path: no compactor RoPE, one block whose queries are precomputed, the fused
+  // kernel (2d <= 256), and a padded x~ narrower than d_l (else projecting k is cheaper).
+  L.Kp = (int)rup(2 * d + 1, 64);
+  L.fold = ctx->key_fold && c.compactor_rope == 0 && NB == 1 && (d == 64 || d == 128) &&
+           !L.qhat_lazy && L.Kp < D;
   auto fail = [&](still_status st) {
     cudaStreamSynchronize(s);
     free_layer(L);
@@ -1108,8 +1153,11 @@ still_status load_layer(still_ctx* ctx, int32_t layer, const still_layer_config*
       (st = dalloc(L, &L.omega_c, (size_t)D / 2)) != STILL_OK ||
       (!L.qhat_lazy && (st = dalloc(L, &L.qhat, (size_t)H * n * T * D)) != STILL_OK))
     return fail(st);
+  // Without compactor RoPE its frequencies are zero: every rotation is exactly the identity.
   if (launch_omega(L.omega_b, d / 2, d, c.rope_theta, s) != cudaSuccess ||
-      launch_omega(L.omega_c, D / 2, D, c.rope_theta_compactor, s) != cudaSuccess ||
+      (c.compactor_rope ? launch_omega(L.omega_c, D / 2, D, c.rope_theta_compactor, s)
+                        : cudaMemsetAsync(L.omega_c, 0, sizeof(double) * (D / 2), s)) !=
+          cudaSuccess ||
       cudaMemcpyAsync(L.Z, Zsrc, sizeof(bf16) * (size_t)H * T * D, cudaMemcpyDeviceToDevice, s) !=
           cudaSuccess ||
       launch_transpose(static_cast<const bf16*>(Wkey), D, d, L.WhT, 0, s) != cudaSuccess ||
@@ -1216,6 +1264,59 @@ still_status load_layer(still_ctx* ctx, int32_t layer, const still_layer_config*
     return STILL_OK;
   };
   st = body();
+  if (st == STILL_OK && L.fold) {  // u = W~_i q^ and G_i = W~_i W~_i^T, hi | lo (block 0)
+    auto fold = [&]() -> still_status {
+      const BlockW& B0 = L.blk[0];
+      const int Kp = L.Kp;
+      bf16* Wt = nullptr;
+      bf16* qhl = nullptr;
+      TRY(dalloc(tmp, &Wt, (size_t)n * Kp * D));
+      TRY(dalloc(tmp, &qhl, (size_t)H * n * T * 2 * D));
+      TRY(dalloc(L, &L.U, (size_t)H * n * T * 2 * Kp));
+      TRY(dalloc(L, &L.G, (size_t)n * Kp * 2 * Kp));
+      CK(launch_fold_weights(B0.WkT, B0.bk, (int)n, D, 2 * d, Kp, Wt, s));
+      CK(launch_f32_hilo(L.qhat, (int64_t)H * n * T, D, qhl, s));
+      {  // U rows (h, i, m): batch b = h n + i over q^ hi | lo (2 passes) x W~_i
+        GemmParams p = gp(T, Kp, H * (int)n, (int)n);
+        p.a_r1 = n * T;
+        p.a_r0 = T;
+        p.b_r1 = 0;
+        p.b_r0 = Kp;
+        add_pass(p, 0, 0, 0, 0, D);
+        add_pass(p, D, 0, 0, 0, D);
+        EpiAffine e;
+        e.kind = OUT_HILO;
+        e.out = L.U;
+        e.lo_off = Kp;
+        e.om.b1 = n * T * 2 * Kp;
+        e.om.b0 = T * 2 * Kp;
+        e.om.bdiv = n;
+        e.om.r0 = 2 * Kp;
+        e.om.c0 = 1;
+        e.vec_ok = 0;
+        TRY(run_gemm256<STILL_K_LOAD>(ctx, op(qhl, (int64_t)H * n * T, 2 * D),
+                                      op(Wt, (int64_t)n * Kp, D), p, e, 1, s));
+      }
+      {  // G_i = W~_i W~_i^T (bf16 operands, exact products)
+        GemmParams p = gp(Kp, Kp, (int)n, 1);
+        p.a_r1 = Kp;
+        p.b_r1 = Kp;
+        add_pass(p, 0, 0, 0, 0, D);
+        EpiAffine e;
+        e.kind = OUT_HILO;
+        e.out = L.G;
+        e.lo_off = Kp;
+        e.om.b1 = (int64_t)Kp * 2 * Kp;
+        e.om.r0 = 2 * Kp;
+        e.om.c0 = 1;
+        e.vec_ok = 0;
+        TRY(run_gemm256<STILL_K_LOAD>(ctx, op(Wt, (int64_t)n * Kp, D), op(Wt, (int64_t)n * Kp, D),
+                                      p, e, 1, s));
+      }
+      return STILL_OK;
+    };
+    st = fold();
+  }
   cudaStreamSynchronize(s);
   free_layer(tmp);
   if (st != STILL_OK) return fail(st);
@@ -1315,6 +1416,12 @@ still_status still_destroy(still_ctx* ctx) {
 still_status still_set_qhat_eager_limit(still_ctx* ctx, size_t bytes) {
   if (ctx == nullptr) return STILL_ERR_INVALID_ARG;
   ctx->qhat_eager_limit = bytes;
+  return STILL_OK;
+}
+
+still_status still_set_key_fold(still_ctx* ctx, int32_t enable) {
+  if (ctx == nullptr || (enable != 0 && enable != 1)) return STILL_ERR_INVALID_ARG;
+  ctx->key_fold = enable != 0;
   return STILL_OK;
 }
 
@@ -1481,7 +1588,8 @@ still_status still_compact_layer_noalloc(still_ctx* ctx, int32_t layer, const vo
   TRY(make_positions(h_segments, n_segments, N, pos));
   CK(cudaSetDevice(ctx->device));
   Plan P;
-  if (!make_plan(L->cfg, queries_per_call(*L), N, t, pos.pmin, pos.pmax, kNoAllocScratchBytes, P))
+  if (!make_plan(L->cfg, queries_per_call(*L), fold_kp(*L), N, t, pos.pmin, pos.pmax,
+                 kNoAllocScratchBytes, P))
     return STILL_ERR_OOM;  // even the smallest grouping needs more than the fixed scratch
   uint8_t* scratch = nullptr;
   TRY(noalloc_scratch(ctx->device, &scratch));
@@ -1786,7 +1894,8 @@ still_status still_workspace_size(const still_ctx* ctx, int64_t max_tokens, int3
     return ctx == nullptr || bytes == nullptr ? STILL_ERR_INVALID_ARG : STILL_ERR_NOT_LOADED;
   if (max_tokens < 1 || max_t < 1 || max_t > max_tokens) return STILL_ERR_SHAPE;
   Plan P;
-  if (!make_plan(ctx->layers[0].cfg, queries_per_call(ctx->layers[0]), max_tokens, max_t, 0.0,
+  if (!make_plan(ctx->layers[0].cfg, queries_per_call(ctx->layers[0]), fold_kp(ctx->layers[0]),
+                 max_tokens, max_t, 0.0,
                  (double)(max_tokens - 1), ctx->ws_limit, P))
     return STILL_ERR_OOM;
   *bytes = P.total;

@@ -30,7 +30,7 @@ EXPORTS = [
     "still_compact_layer_noalloc", "still_recompact_layer_ragged", "still_recompact_stack_ragged",
     "still_selftest_wait_timeout", "still_compact_stack_masked", "still_lookahead_pass_info",
     "still_lookahead_totals", "still_lookahead_compact_layer", "still_lookahead_compact_stack",
-    "still_set_beta_head", "still_compact_layer_beta", "still_attend_biased",
+    "still_set_beta_head", "still_compact_layer_beta", "still_attend_biased", "still_set_key_fold",
 ]
 
 NOALLOC_SCRATCH_MIB = 64  # STILL_NOALLOC_SCRATCH_MIB in include/still.h
@@ -135,6 +135,7 @@ def lib():
             "still_workspace_size": ([P, I64, I32, ctypes.POINTER(ctypes.c_size_t)], ctypes.c_int),
             "still_set_workspace_limit": ([P, ctypes.c_size_t], ctypes.c_int),
             "still_set_qhat_eager_limit": ([P, ctypes.c_size_t], ctypes.c_int),
+            "still_set_key_fold": ([P, I32], ctypes.c_int),
             "still_get_device_status": ([P, P, PI32], ctypes.c_int),
             "still_budget": ([I64, I64], I64),
             "still_kv_bytes": ([I64, I64, I64, I64, I64], I64),
@@ -210,7 +211,8 @@ def make_config(H, d, D, n, F, t_max, theta, theta_c=10.0, final_norm=0, logit_s
 def config_from_workload(wl: dict, t_max: int, **over) -> LayerConfig:
     kw = dict(H=wl["H"], d=wl["d"], D=wl["D"], n=wl["n"], F=wl["F"], t_max=t_max,
               theta=wl["theta"], n_blocks=wl.get("n_blocks", 1),
-              cross_every_block=int(wl.get("cross_every_block", 1)))
+              cross_every_block=int(wl.get("cross_every_block", 1)),
+              compactor_rope=int(wl.get("compactor_rope", 1)))
     kw.update(over)
     return make_config(**kw)
 
@@ -459,6 +461,10 @@ def still_recompact_stack_ragged(ctx, Kprevs, Vprevs, cu_prev, prev_len, Knews, 
         arr(Knews), arr(Vnews), (I64 * (B + 1))(*cu_new), ratio, arr(Cks), arr(Cvs), cu_out,
         len_out, _stream(stream)), "still_recompact_stack_ragged")
     return list(cu_out), list(len_out)
+
+
+def still_set_key_fold(ctx, enable: bool):
+    _check(lib().still_set_key_fold(ctx, 1 if enable else 0), "still_set_key_fold")
 
 
 def still_reserve_workspace(ctx, max_tokens: int, max_t: int):

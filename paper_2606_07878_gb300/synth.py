@@ -34,6 +34,10 @@ WORKLOADS = {
     # 50x ratio (t = 1311).
     "qwen3_4b_64k": dict(L=36, N=65536, H=8, d=128, D=256, n=1, F=0, ts=(1311,), theta=1e6,
                          heavy=1, n_blocks=2, cross_every_block=1),
+    # The compactor-RoPE-free ablation (App. M) of the qwen7b_8k shape: the key projection
+    # folds into the queries.
+    "qwen7b_8k_norope": dict(L=28, N=8192, H=4, d=128, D=1024, n=8, F=4096, ts=(1024, 256),
+                             theta=1e6, heavy=4, compactor_rope=0),
     # Iterative ragged serving: 8 sequences, lengths uniform in [8k, 32k] from seed 7, then
     # 16 rounds of +8192 tokens each, re-compacted to the 32x budget.
     "iterative_ragged": dict(L=36, H=8, d=128, D=1024, n=8, F=4096, theta=1e6, heavy=1,
