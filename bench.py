@@ -180,12 +180,14 @@ def algorithmic_flops(wl, t, N):
     ca = (kproj + 2 * t * N * H * n * kw + 2 * t * N * H * n * 2 * d
           + 2 * t * H * n * 2 * d * D + 2 * t * H * n * D * D)
     sa = 6 * t * H * D * n * D + 4 * t * t * H * n * D + 2 * t * H * n * D * D
-    # The last block's cross-attention is one fused kernel when 2d <= 256; earlier blocks
-    # (and every block at 2d = 512) take the scores GEMM.
-    fused_last = 2 * d <= 256 and (nb == 1 or wl.get("cross_every_block", 1))
+    # Every block's cross-attention is one fused kernel when 2d <= 256 (a block that feeds
+    # another in its split-precision form, P X in 2.5 passes); 2d = 512 takes the scores GEMM.
+    fused = 2 * d <= 256
     return {"total": n_ca * ca + nb * (sa + 4 * t * H * D * F) + 4 * t * H * D * d,
             "scores": n_ca * 2 * t * N * H * n * kw, "px": n_ca * 2 * t * N * H * n * 2 * d,
-            "scores_gemm": (n_ca - (1 if fused_last else 0)) * 2 * t * N * H * n * D}
+            "scores_gemm": 0 if fused else n_ca * 2 * t * N * H * n * D,
+            # passes of P X issued over all blocks with cross-attention (the last 1.5, others 2.5)
+            "px_passes": 1.5 + 2.5 * (n_ca - 1), "px_blk": 2 * t * N * H * n * 2 * d}
 
 
 def run_cpu_baseline(wl, t, budget_s=30.0):
@@ -271,6 +273,133 @@ def run_reference(args):
                 "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line))
+
+
+# The compact cache's consumer at decode time: one generated token of one sequence through the
+# biased attention of every layer of a Qwen3-4B-shaped model (32 query heads over 8 KV-heads,
+# d = 128), over the canonical compaction of a 64k context (t = 1311 slots with a bias) followed
+# by one raw lookahead chunk of 4096 tokens.
+DECODE = dict(L=36, H=8, Hq=32, d=128, t=1311, S=4096, nq=1)
+
+
+def run_decode(args):
+    """Biased decode attention (App. B, "Bias semantics in attention") over [C_k; K_fix] for
+    every layer, captured as one CUDA graph; one step = one decode token through all layers."""
+    import numpy as np
+    import torch
+
+    from oracle import still_oracle as O
+    from paper_2606_07878_gb300 import still
+
+    c = DECODE
+    L, H, Hq, d, t, S, nq = c["L"], c["H"], c["Hq"], c["d"], c["t"], c["S"], c["nq"]
+    dev = "cuda:0"
+    torch.cuda.set_device(0)
+    stream = torch.cuda.Stream()
+    torch.cuda.set_stream(stream)
+    g = torch.Generator(device=dev).manual_seed(3)
+    rnd = lambda *shape: torch.randn(shape, generator=g, device=dev).to(torch.bfloat16)
+    Cks = [rnd(t, H, d) for _ in range(L)]
+    Cvs = [rnd(t, H, d) for _ in range(L)]
+    betas = [torch.randn((t, H), generator=g, device=dev) for _ in range(L)]
+    Kfs = [rnd(S, H, d) for _ in range(L)]
+    Vfs = [rnd(S, H, d) for _ in range(L)]
+    qs = [rnd(nq, Hq, d) for _ in range(L)]
+    outs = [torch.empty((nq, Hq, d), dtype=torch.bfloat16, device=dev) for _ in range(L)]
+    ctx = still.still_create(0)
+
+    def step():
+        for l in range(L):
+            still.still_attend_biased(ctx, qs[l], Cks[l], Cvs[l], betas[l], Kfs[l], Vfs[l],
+                                      outs[l], stream=stream)
+
+    still.still_profile_enable(ctx, True)
+    for _ in range(max(args.warmup, 3)):
+        step()
+    torch.cuda.synchronize()
+    still.still_profile_enable_classes(ctx, ["decode"])
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        step()
+    graph.replay()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(0)
+    clocks.start()
+    time.sleep(0.3)
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    steps = max(args.steps, 20)  # a step is short: time at least 20
+    ev0.record(stream)
+    for _ in range(steps):
+        graph.replay()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1)
+    prof = still.still_profile_read(ctx)
+    still.still_profile_enable(ctx, False)
+    clk = clocks.stop()
+    code, det = still.still_get_device_status(ctx, stream)
+    if code != 0:
+        raise RuntimeError(f"device status {still.STATUS.get(code)} {det}")
+    del graph
+    n_dec, ms_dec = prof["decode"]  # the last replay's launches (chunk + merge per layer)
+    # Algorithmic bytes of one layer's attention: the compact slots and raw entries (K and V),
+    # the bias, the query and the output.
+    layer_bytes = (t + S) * H * d * 2 * 2 + t * H * 4 + 2 * nq * Hq * d * 2
+    calls = n_dec // 2
+    achieved = layer_bytes * calls / (ms_dec / 1e3) / 1e9 if ms_dec > 0 else None
+    hbm, _, _, src = _peaks()
+    # end to end: the step's queries from pinned host memory in, outputs back to the host
+    q_host = [x.cpu().pin_memory() for x in qs]
+    o_host = [torch.empty((nq, Hq, d), dtype=torch.bfloat16).pin_memory() for _ in range(L)]
+    ds = torch.cuda.default_stream()
+
+    def e2e_step():
+        for l in range(L):
+            qs[l].copy_(q_host[l], non_blocking=True)
+            still.still_attend_biased(ctx, qs[l], Cks[l], Cvs[l], betas[l], Kfs[l], Vfs[l],
+                                      outs[l], stream=ds)
+            o_host[l].copy_(outs[l], non_blocking=True)
+        ds.synchronize()
+
+    with torch.cuda.stream(ds):
+        e2e_step()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(steps):
+            e2e_step()
+        e2e_s = time.perf_counter() - t0
+    still.still_destroy(ctx)
+    cpu = None
+    if not args.no_cpu_baseline:
+        f = lambda x: x.double().cpu().numpy()
+        qn, ck, cv, bn, kf, vf = f(qs[0]), f(Cks[0]), f(Cvs[0]), f(betas[0]), f(Kfs[0]), f(Vfs[0])
+        t0 = time.perf_counter()
+        for qh in range(Hq):
+            h = qh // (Hq // H)
+            O.biased_attention(qn[:, qh], ck[:, h], cv[:, h], bn[:, h], kf[:, h], vf[:, h],
+                               1 / np.sqrt(d))
+        sec = (time.perf_counter() - t0) * L
+        cpu = {"value": 1.0 / sec, "unit": "decode tokens/s", "cores": os.cpu_count(),
+               "kind": "oracle", "sample": f"layer 0 of {L} (all {Hq} query heads), x{L}"}
+    print(json.dumps({
+        "metric": "decode tokens/s through the compact cache (biased attention over [C_k; K_fix], all layers)",
+        "value": steps / (ms / 1e3), "unit": "tokens/s", "n_gpus": 1, "steps": steps,
+        "warmup": max(args.warmup, 3), "ms_per_step": ms / steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"decode_qwen3_4b: {L} layers, {Hq} query heads over {H} KV-heads, "
+                               f"d={d}, {nq} query token, t={t} compact slots with bias + "
+                               f"{S} raw entries",
+                   "l2": f"inputs larger than L2 ({L * layer_bytes / 1e6:.0f} MB per step)"},
+        "e2e": {"value": steps / e2e_s, "unit": "tokens/s",
+                "h2d_bytes_per_step": L * nq * Hq * d * 2, "d2h_bytes_per_step": L * nq * Hq * d * 2},
+        "gpu_launches": n_dec,
+        "roofline": {"bound": "hbm", "kernel": "decode attention (chunks + merge)",
+                     "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                     "frac": achieved / hbm if achieved else None, "traffic": None,
+                     "peak_source": f"{src} HBM copy bandwidth",
+                     "bytes_per_launch": layer_bytes},
+        "cpu_baseline": cpu, "clocks": clk}))
 
 
 def run_iterative(args):
@@ -373,7 +502,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--t", type=int, default=0, help="compact length (default per workload)")
     ap.add_argument("--workload", default=WORKLOAD,
-                    choices=sorted(DEFAULT_T) + ["iterative_ragged"])
+                    choices=sorted(DEFAULT_T) + ["iterative_ragged", "decode_qwen3_4b"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     if args.impl == "reference":
@@ -381,6 +510,9 @@ def main():
         return
     if args.workload == "iterative_ragged":
         run_iterative(args)
+        return
+    if args.workload == "decode_qwen3_4b":
+        run_decode(args)
         return
 
     import torch
@@ -432,7 +564,7 @@ def main():
     # as one graph). The dominant kernel class (fused cross-attention for 2d <= 256, else the
     # scores GEMM) is the only one with events: its launches are bracketed by event nodes of the
     # graph, read after the last replay.
-    kname = "ca_fused" if 2 * d <= 256 and wl.get("n_blocks", 1) == 1 else "scores"
+    kname = "ca_fused" if 2 * d <= 256 else "scores"
     still.still_reserve_workspace(ctx, N, t)
     still.still_profile_enable_classes(ctx, [kname])
     graph = torch.cuda.CUDAGraph()
@@ -526,14 +658,17 @@ def main():
     fused = kname == "ca_fused"
     n_k, ms_k = prof_timed[kname]  # one step's launches (the captured event pairs)
     alg = fl["scores"] + fl["px"] if fused else fl["scores_gemm"]
-    issued = 3 * fl["scores"] + 1.5 * fl["px"] if fused else 3 * fl["scores_gemm"]
+    issued = (3 * fl["scores"] + fl["px_passes"] * fl["px_blk"] if fused
+              else 3 * fl["scores_gemm"])
     per_launch_flops = alg * L / max(n_k, 1)
     achieved = per_launch_flops / (ms_k / max(n_k, 1) / 1e3) / 1e12 if ms_k > 0 else None
     tr = TRAFFIC[kname]
     traffic = None
     if tr["kernel_hash"] == _kernel_hash(tr["files"]) and tr["workload"] == (name, t):
         traffic = tr["bytes_per_launch"]
-    kdesc = ("ca_fused (3-pass split-bf16 scores + online softmax + P X, one tcgen05 kernel)"
+    kdesc = ("ca_fused (3-pass split-bf16 scores + online softmax + P X, one tcgen05 kernel"
+             + ("; the first block's launches in split fp16 with P hi + lo)"
+                if wl.get("n_blocks", 1) > 1 and wl.get("cross_every_block", 1) else ")")
              if fused else "scores (3-pass split-bf16 tcgen05 GEMM)")
     ratio = issued / alg
     roof = {"bound": "tensor", "kernel": kdesc,

@@ -18,6 +18,9 @@
 // Output per split: unnormalised O rows and (m, l) with m in log2 units; ca_merge_kernel
 // combines the splits in a fixed order (bit-reproducible).
 //
+// EX (a block whose output feeds another block): q, k in fp16 hi | lo, probabilities as fp16
+// hi + lo with one more P X pass, 128-key tiles (S in TMEM columns [0, 128)).
+//
 // CTA = 10 warps: 0 TMA producer, 1 MMA issuer (TMEM owner), 2..9 softmax / output.
 #pragma once
 #include "gemm_host.cuh"
@@ -41,21 +44,27 @@ struct FlashParams {
   int* err = nullptr;
 };
 
-constexpr int kFlashKeys = 256;       // keys per S tile
+constexpr int kFlashKeys = 256;       // keys per S tile (EX: 128)
 constexpr int kFlashSoftWarps = 8;    // two per TMEM lane quarter
 constexpr int kFlashThreads = 64 + 32 * kFlashSoftWarps;
 constexpr float kRescaleLog2 = 8.f;
 
-template <int D2>
+// EX (split precision, for a block whose output feeds another block): q, k as fp16 hi | lo and
+// the probabilities as fp16 hi + lo (one more P X pass); key tiles of 128 so that the P_hi and
+// P_lo tiles together take the shared memory of one 256-key P tile.
+template <int D2, bool EX = false>
 struct FlashSmem {
   static_assert(D2 == 128 || D2 == 256, "2d must be 128 or 256");
+  static constexpr int kKeys = EX ? 128 : kFlashKeys;     // keys per S tile
   static constexpr int kQBytes = kBM * kBK * 2;            // q chunk, 16 KB
-  static constexpr int kKBytes = kFlashKeys * kBK * 2;     // k chunk, 32 KB
+  static constexpr int kKBytes = kKeys * kBK * 2;          // k chunk
   static constexpr int kXhiBytes = D2 * kBK * 2;           // X^T hi chunk
   static constexpr int kXloBytes = (D2 / 2) * kBK * 2;     // X^T lo chunk (key half)
-  static constexpr int kStageBytes = kQBytes + kKBytes;    // >= kXhiBytes + kXloBytes
+  static constexpr int kStageBytes = (kQBytes + kKBytes) > (kXhiBytes + kXloBytes)
+                                         ? (kQBytes + kKBytes) : (kXhiBytes + kXloBytes);
   static constexpr int kStages = 3;
   static constexpr int kPChunkBytes = kBM * kBK * 2;       // 128 rows x 64 keys fp16
+  static constexpr int kPChunks = kKeys / kBK;             // chunks of one P tile (hi)
   static constexpr int kPOffset = kStages * kStageBytes;
   static constexpr int kKinvOffset = kPOffset + 4 * kPChunkBytes;        // [8 warps][128] f32
   static constexpr int kXchOffset = kKinvOffset + kFlashSoftWarps * 128 * 4;  // [2][2][128] f32
@@ -80,20 +89,23 @@ __device__ __forceinline__ FlashUnit flash_unit(const FlashParams& f, int u) {
   return r;
 }
 
-// Number of 64-key chunks of tile j that lie inside the padded key range [0, Np).
+// Number of 64-key chunks of tile j (of KEYS keys) that lie inside the padded key range [0, Np).
+template <int KEYS>
 __device__ __forceinline__ int flash_chunks(const FlashParams& f, int j) {
-  const int64_t left = f.Np - (int64_t)j * kFlashKeys;
-  return left >= kFlashKeys ? 4 : (int)(left / kBK);
+  const int64_t left = f.Np - (int64_t)j * KEYS;
+  return left >= KEYS ? KEYS / kBK : (int)(left / kBK);
 }
 
-template <int D2>
+template <int D2, bool EX>
 __global__ void __launch_bounds__(kFlashThreads, 1)
     ca_flash_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                     const __grid_constant__ CUtensorMap tmXhi,
                     const __grid_constant__ CUtensorMap tmXlo, const FlashParams f) {
-  using S = FlashSmem<D2>;
+  using S = FlashSmem<D2, EX>;
+  constexpr int kKeys = S::kKeys;
   constexpr int kStages = S::kStages;
   constexpr int kOCols = D2 / 2;  // O columns per softmax warp (its half of 2d)
+  constexpr int kCols = kKeys / 2;  // S columns per softmax warp (its half of the key tile)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -176,12 +188,12 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
         const int J = w.j1 - w.j0;
         for (int jj = 0; jj <= J && !bad; ++jj) {
           if (jj < J) {
-            const int32_t kr = krow + (w.j0 + jj) * kFlashKeys;
+            const int32_t kr = krow + (w.j0 + jj) * kKeys;
             for (int pass = 0; pass < 3 && !bad; ++pass) {
               const int32_t qoff = pass == 2 ? f.D : 0;  // (q_hi,k_hi), (q_hi,k_lo), (q_lo,k_hi)
               const int32_t koff = pass == 1 ? f.D : 0;
               for (int c = 0; c < qchunks; ++c) {
-                uint8_t* sa = acquire(S::kStageBytes);
+                uint8_t* sa = acquire(S::kQBytes + S::kKBytes);  // the bytes these two copies bring
                 if (sa == nullptr) break;
                 tma_load_2d(sa, &tmQ, &full[stage], qoff + c * kBK, qrow);
                 tma_load_2d(sa + S::kQBytes, &tmK, &full[stage], koff + c * kBK, kr);
@@ -191,11 +203,11 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
           }
           if (jj >= 1) {
             const int j = w.j0 + jj - 1;
-            const int nch = flash_chunks(f, j);
+            const int nch = flash_chunks<kKeys>(f, j);
             for (int c = 0; c < nch; ++c) {
               uint8_t* sa = acquire(S::kXhiBytes + S::kXloBytes);
               if (sa == nullptr) break;
-              const int32_t x = j * kFlashKeys + c * kBK;
+              const int32_t x = j * kKeys + c * kBK;
               tma_load_2d(sa, &tmXhi, &full[stage], x, xrow);
               tma_load_2d(sa + S::kXhiBytes, &tmXlo, &full[stage], (int32_t)(f.Np + x), xrow);
               advance();
@@ -211,7 +223,7 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
   } else if (warp == 1) {
     if (lane == 0) {
       // ------------------------------------------------------------ MMA issuer
-      const uint32_t idesc_s = idesc_f16(kBM, kFlashKeys, 1);  // bf16 q, k
+      const uint32_t idesc_s = idesc_f16(kBM, kKeys, EX ? 0 : 1);  // fp16 (EX) or bf16 q, k
       const uint32_t idesc_hi = idesc_f16(kBM, D2, 0);         // fp16 P, X^T hi
       const uint32_t idesc_lo = idesc_f16(kBM, D2 / 2, 0);     // fp16 P, X^T lo (key half)
       const uint32_t s_tmem = tmem_base;
@@ -262,7 +274,7 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
           }
           if (jj >= 1) {
             const int j = w.j0 + jj - 1;
-            const int nch = flash_chunks(f, j);
+            const int nch = flash_chunks<kKeys>(f, j);
             if (jj == 1 && n_units > 0 && !mbar_wait(ofree, (n_units - 1) & 1)) {
               fail(312);
               break;
@@ -288,6 +300,13 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
                            (jj > 1 || c > 0 || k > 0) ? 1u : 0u);
 #pragma unroll
               for (int k = 0; k < kBK / 16; ++k) tc_mma_f16(o_tmem, pd + 2 * k, ld + 2 * k, idesc_lo, 1u);
+              if constexpr (EX) {  // + P_lo X^T hi
+                const uint64_t pld =
+                    sdesc_k_sw128(p_smem + (S::kPChunks + c) * S::kPChunkBytes);
+#pragma unroll
+                for (int k = 0; k < kBK / 16; ++k)
+                  tc_mma_f16(o_tmem, pld + 2 * k, hd + 2 * k, idesc_hi, 1u);
+              }
               tc_commit(&empty[stage]);
               if (++stage == kStages) {
                 stage = 0;
@@ -348,21 +367,21 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
       float m_run = -INFINITY, l_part = 0.f;
       for (int jj = 0; jj < J; ++jj) {
         const int j = w.j0 + jj;
-        const int key0 = j * kFlashKeys + 128 * half;  // first key of this warp's columns
-        float kv[4];
+        const int key0 = j * kKeys + kCols * half;  // first key of this warp's columns
+        float kv[kCols / 32];
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
+        for (int e = 0; e < kCols / 32; ++e) {
           const int key = key0 + lane + 32 * e;
           kv[e] = key < f.N ? f.kinv[(int64_t)w.b * f.N + key] * kLog2e : 0.f;
         }
         if (!wait_all(sfull, n_sf & 1, 320)) break;
         ++n_sf;
         tc_fence_after();
-        float v[128];
+        float v[kCols];
 #pragma unroll
-        for (int g = 0; g < 4; ++g) {
+        for (int g = 0; g < kCols / 32; ++g) {
           float tmp[32];
-          tmem_ld32(lane_base + (uint32_t)(128 * half + 32 * g), tmp);
+          tmem_ld32(lane_base + (uint32_t)(kCols * half + 32 * g), tmp);
 #pragma unroll
           for (int e = 0; e < 32; ++e) v[32 * g + e] = tmp[e];
         }
@@ -371,12 +390,12 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
         if (lane == 0) mbar_arrive(sfree);
         // scale per key (log2 units), mask keys past N, tile max
 #pragma unroll
-        for (int e = 0; e < 4; ++e) kw[lane + 32 * e] = kv[e];
+        for (int e = 0; e < kCols / 32; ++e) kw[lane + 32 * e] = kv[e];
         __syncwarp();
         const int cvalid = f.N - key0;
         float mx = -INFINITY;
 #pragma unroll
-        for (int c = 0; c < 128; c += 4) {
+        for (int c = 0; c < kCols; c += 4) {
           const float4 k4 = *reinterpret_cast<const float4*>(kw + c);
           v[c] = c < cvalid ? v[c] * k4.x : -INFINITY;
           v[c + 1] = c + 1 < cvalid ? v[c + 1] * k4.y : -INFINITY;
@@ -399,13 +418,23 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
           rescale = true;
         }
         // probabilities (fp16, <= 2^8) into registers as packed pairs; l from the rounded values
-        uint32_t pk[64];
+        // (EX: hi and lo = fp16(p - hi), l from hi + lo)
+        uint32_t pk[kCols / 2];
+        uint32_t pkl[EX ? kCols / 2 : 1];
 #pragma unroll
-        for (int c = 0; c < 128; c += 2) {
-          const __half2 h = __floats2half2_rn(exp2f(v[c] - m_run), exp2f(v[c + 1] - m_run));
+        for (int c = 0; c < kCols; c += 2) {
+          const float p0 = exp2f(v[c] - m_run), p1 = exp2f(v[c + 1] - m_run);
+          const __half2 h = __floats2half2_rn(p0, p1);
           const float2 r = __half22float2(h);
-          l_part += r.x + r.y;
           pk[c / 2] = *reinterpret_cast<const uint32_t*>(&h);
+          if constexpr (EX) {
+            const __half2 lo = __floats2half2_rn(p0 - r.x, p1 - r.y);
+            const float2 rl = __half22float2(lo);
+            l_part += (r.x + rl.x) + (r.y + rl.y);
+            pkl[c / 2] = *reinterpret_cast<const uint32_t*>(&lo);
+          } else {
+            l_part += r.x + r.y;
+          }
         }
         // The previous PX must be complete before P is overwritten or O is rescaled.
         if (n_pf > n_pe) {
@@ -426,14 +455,26 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
             tmem_st32(ta, o);
           }
         }
-        // P row `row`, keys [128 half, +128): chunks 2 half and 2 half + 1 of the P tile.
+        // P row `row`, keys [kCols half, +kCols): chunks kCols/64 * half + q of the P tile
+        // (EX: the lo values in the same chunks of the second tile, kPChunks further).
 #pragma unroll
-        for (int q = 0; q < 2; ++q) {
-          uint4* dst = reinterpret_cast<uint4*>(pbuf + (2 * half + q) * S::kPChunkBytes + row * 128);
+        for (int q = 0; q < kCols / 64; ++q) {
+          const int chunk = (kCols / 64) * half + q;
+          uint4* dst = reinterpret_cast<uint4*>(pbuf + chunk * S::kPChunkBytes + row * 128);
 #pragma unroll
           for (int un = 0; un < 8; ++un) {
             const int base = (64 * q + 8 * un) / 2;
             dst[un ^ (row & 7)] = make_uint4(pk[base], pk[base + 1], pk[base + 2], pk[base + 3]);
+          }
+          if constexpr (EX) {
+            uint4* dl = reinterpret_cast<uint4*>(pbuf + (S::kPChunks + chunk) * S::kPChunkBytes +
+                                                 row * 128);
+#pragma unroll
+            for (int un = 0; un < 8; ++un) {
+              const int base = (64 * q + 8 * un) / 2;
+              dl[un ^ (row & 7)] =
+                  make_uint4(pkl[base], pkl[base + 1], pkl[base + 2], pkl[base + 3]);
+            }
           }
         }
         fence_proxy_async_smem();
@@ -498,19 +539,20 @@ inline int flash_split(int64_t base_units, int tiles_k, int num_sms, int max_spl
   return best;
 }
 
-// Q: [nb*t][2D] bf16 (hi | lo), K: [nb*N][2D] bf16 (hi | lo), XT: [H*2d][2*Np] fp16 (hi | lo).
-template <int D2>
+// Q: [nb*t][2D] bf16 (hi | lo), K: [nb*N][2D] bf16 (hi | lo), XT: [H*2d][2*Np] fp16 (hi | lo);
+// EX: Q and K fp16 hi | lo, key tiles of S::kKeys = 128 (f.tiles_k counts those).
+template <int D2, bool EX = false>
 inline cudaError_t launch_ca_flash(const Operand2D& Q, const Operand2D& K, const Operand2D& XT,
                                    const FlashParams& f, int num_sms, cudaStream_t stream) {
-  using S = FlashSmem<D2>;
+  using S = FlashSmem<D2, EX>;
   if (f.D <= 0 || f.D % kBK != 0 || f.t <= 0 || f.N <= 0 || f.Np % kBK != 0 || f.Np < f.N ||
       f.nunits <= 0)
     return cudaErrorInvalidValue;
   CUtensorMap tq, tk, thi, tlo;
-  if (!make_tmap(&tq, Q, kBM) || !make_tmap(&tk, K, kFlashKeys) || !make_tmap(&thi, XT, D2) ||
+  if (!make_tmap(&tq, Q, kBM) || !make_tmap(&tk, K, S::kKeys) || !make_tmap(&thi, XT, D2) ||
       !make_tmap(&tlo, XT, D2 / 2))
     return cudaErrorInvalidValue;
-  auto kern = ca_flash_kernel<D2>;
+  auto kern = ca_flash_kernel<D2, EX>;
   static thread_local bool attr_set = false;
   if (!attr_set) {
     cudaError_t e =

@@ -686,112 +686,181 @@ __global__ void beta_kernel(const __nv_bfloat16* __restrict__ Z, int64_t rows, i
 //
 // Attention of query rows over the entries [C (t compact slots, logit bias beta) ; F (S
 // uncompacted entries, bias 0)] (App. B, "Bias semantics in attention"). Grid (chunk, KV-head):
-// a CTA stages one chunk of kDecChunk entries of its KV-head (keys transposed, values as rows,
-// bf16 in shared memory), serves every query row of the KV-head's query heads from it, and
-// writes per-row partials (max m, sum l, unnormalised O); decode_merge_kernel combines the
-// chunks in order.
-constexpr int kDecChunk = 128;
-constexpr int kDecThreads = 128;
+// a CTA of 8 warps covers dec_chunk entries of its KV-head (16 per warp, 8 at d = 256). A lane
+// holds DPL = d/32 dimensions of each of its warp's keys and values in registers (coalesced
+// loads, all issued up front), so the cache is read once and straight from global memory. Per
+// query row of the KV-head's query heads, each warp forms its logits (warp-sum of the lane
+// partials), their
+// max, weights and weighted values; the 8 warps' (max, sum, O) are combined through shared
+// memory into one partial per (row, chunk), and decode_merge_kernel combines the chunks in order.
+constexpr int kDecThreads = 256;
+constexpr int kDecRowGroup = 4;  // query rows per pass
+// entries per warp: 16 (8 at d = 256, whose 8 dimensions per lane double the registers)
+__host__ __device__ constexpr int dec_per_warp(int dpl) { return dpl == 8 ? 8 : 16; }
+__host__ __device__ constexpr int dec_chunk(int dpl) { return dec_per_warp(dpl) * kDecThreads / 32; }
 
+// DPL consecutive bf16 as DPL / 2 packed pairs (one 4-, 8- or 16-byte load).
+template <int DPL>
+__device__ __forceinline__ void load_pairs(const __nv_bfloat16* p, uint32_t (&x)[DPL / 2]) {
+  if constexpr (DPL == 2) {
+    x[0] = *reinterpret_cast<const uint32_t*>(p);
+  } else if constexpr (DPL == 4) {
+    const uint2 u = *reinterpret_cast<const uint2*>(p);
+    x[0] = u.x;
+    x[1] = u.y;
+  } else {
+    const uint4 u = *reinterpret_cast<const uint4*>(p);
+    x[0] = u.x;
+    x[1] = u.y;
+    x[2] = u.z;
+    x[3] = u.w;
+  }
+}
+
+__device__ __forceinline__ float2 unpack_pair(uint32_t w) {
+  return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w));
+}
+
+template <int DPL>
 __global__ void __launch_bounds__(kDecThreads)
     decode_chunk_kernel(DecodeArgs a, float* __restrict__ part_o, float2* __restrict__ part_ml) {
-  extern __shared__ uint8_t dsm[];
-  const int d = a.d;
+  extern __shared__ float dsm[];
+  constexpr int d = 32 * DPL;
+  constexpr int kW = kDecThreads / 32;
+  constexpr int kDecPerWarp = dec_per_warp(DPL);
+  constexpr int kDecChunk = dec_chunk(DPL);
   const int h = blockIdx.y, chunk = blockIdx.x;
   const int g = a.Hq / a.H;        // query heads per KV-head
   const int G = a.nq * g;          // query rows served by this CTA
-  __nv_bfloat16* kt = reinterpret_cast<__nv_bfloat16*>(dsm);   // [d][kDecChunk]
-  __nv_bfloat16* vr = kt + (size_t)d * kDecChunk;              // [kDecChunk][d]
-  float* qs = reinterpret_cast<float*>(vr + (size_t)kDecChunk * d);  // [G][d]
-  float* pw = qs + (size_t)G * d;                                     // [kDecChunk]
-  float* red = pw + kDecChunk;                                        // [2][4]
-  const int64_t e0 = (int64_t)chunk * kDecChunk;
+  float* qs = dsm;                                  // [G][d]
+  float* red = qs + (size_t)G * d;                  // [kW][kDecRowGroup][d + 2]
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t E = a.t + a.S;
-  // stage keys (transposed) and values; entries past E are zero (masked below)
-  const int vecs = d / 8;
-  for (int it = threadIdx.x; it < kDecChunk * vecs; it += kDecThreads) {
-    const int i = it / vecs, c0 = 8 * (it % vecs);
-    const int64_t e = e0 + i;
-    uint4 kq = make_uint4(0, 0, 0, 0), vq = make_uint4(0, 0, 0, 0);
-    if (e < E) {
-      const int64_t off = (e < a.t ? e * a.cst : (e - a.t) * a.fst) + (int64_t)h * d + c0;
-      const __nv_bfloat16* kp = (e < a.t ? a.Ck : a.Kf) + off;
-      const __nv_bfloat16* vp = (e < a.t ? a.Cv : a.Vf) + off;
-      kq = *reinterpret_cast<const uint4*>(kp);
-      vq = *reinterpret_cast<const uint4*>(vp);
-    }
-    const __nv_bfloat16* ke = reinterpret_cast<const __nv_bfloat16*>(&kq);
+  // this warp's keys and values (lane dims [DPL lane, +DPL))
+  uint32_t kx[kDecPerWarp][DPL / 2], vx[kDecPerWarp][DPL / 2];  // packed bf16 pairs
+  float bias[kDecPerWarp];
+  bool valid[kDecPerWarp];
 #pragma unroll
-    for (int k = 0; k < 8; ++k) kt[(size_t)(c0 + k) * kDecChunk + i] = ke[k];
-    *reinterpret_cast<uint4*>(vr + (size_t)i * d + c0) = vq;
+  for (int k = 0; k < kDecPerWarp; ++k) {
+    const int64_t e = (int64_t)chunk * kDecChunk + warp * kDecPerWarp + k;
+    valid[k] = e < E;
+    bias[k] = 0.f;
+    if (valid[k]) {
+      const bool comp = e < a.t;
+      const int64_t off = (comp ? e * a.cst : (e - a.t) * a.fst) + (int64_t)h * d + DPL * lane;
+      load_pairs<DPL>((comp ? a.Ck : a.Kf) + off, kx[k]);
+      load_pairs<DPL>((comp ? a.Cv : a.Vf) + off, vx[k]);
+      if (comp && a.beta != nullptr) bias[k] = a.beta[e * a.H + h];
+    } else {
+#pragma unroll
+      for (int i = 0; i < DPL / 2; ++i) kx[k][i] = vx[k][i] = 0u;
+    }
   }
-  // query rows of this KV-head: row r = (query n, head h * g + k) with r = n * g + k
+  // query rows of this KV-head: row r = (query n, head h * g + r % g), n = r / g
   for (int it = threadIdx.x; it < G * d; it += kDecThreads) {
     const int r = it / d, c = it % d;
     const int n = r / g, qh = h * g + r % g;
     qs[it] = __bfloat162float(a.q[((int64_t)n * a.Hq + qh) * d + c]);
   }
   __syncthreads();
-  const int i = threadIdx.x;  // this thread's entry in the chunk
-  const int64_t e = e0 + i;
-  const bool valid = e < E;
-  const float bias = (valid && e < a.t && a.beta != nullptr) ? a.beta[e * a.H + h] : 0.f;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t nch = gridDim.x;
-  for (int r = 0; r < G; ++r) {
-    const float* qr = qs + (size_t)r * d;
-    float acc = 0.f;
-    for (int c = 0; c < d; ++c) acc = fmaf(qr[c], __bfloat162float(kt[(size_t)c * kDecChunk + i]), acc);
-    const float logit = valid ? acc * a.scale + bias : -INFINITY;
-    // chunk max
-    float m = logit;
+  for (int r0 = 0; r0 < G; r0 += kDecRowGroup) {
+    const int nr = min(kDecRowGroup, G - r0);
+#pragma unroll 1
+    for (int rr = 0; rr < nr; ++rr) {
+      float qv[DPL];
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-    if (lane == 0) red[warp] = m;
-    __syncthreads();
-    m = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
-    const float p = valid ? __expf(logit - m) : 0.f;
-    float l = p;
+      for (int i = 0; i < DPL; ++i) qv[i] = qs[(size_t)(r0 + rr) * d + DPL * lane + i];
+      float lg[kDecPerWarp];
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-    pw[i] = p;
-    if (lane == 0) red[4 + warp] = l;
-    __syncthreads();
-    const float lsum = red[4] + red[5] + red[6] + red[7];
-    // O[c] = sum_i p_i V[i][c]
-    const int n = r / g, qh = h * g + r % g;
-    const int64_t prow = ((int64_t)n * a.Hq + qh) * nch + chunk;
-    for (int c = threadIdx.x; c < d; c += kDecThreads) {
-      float o = 0.f;
-      for (int k = 0; k < kDecChunk; ++k) o = fmaf(pw[k], __bfloat162float(vr[(size_t)k * d + c]), o);
-      part_o[prow * d + c] = o;
+      for (int k = 0; k < kDecPerWarp; ++k) {
+        float s = 0.f;
+#pragma unroll
+        for (int i = 0; i < DPL / 2; ++i) {
+          const float2 kf = unpack_pair(kx[k][i]);
+          s = fmaf(qv[2 * i], kf.x, fmaf(qv[2 * i + 1], kf.y, s));
+        }
+        lg[k] = s;
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+        for (int k = 0; k < kDecPerWarp; ++k) lg[k] += __shfl_xor_sync(0xffffffffu, lg[k], o);
+      }
+      float m = -INFINITY;
+#pragma unroll
+      for (int k = 0; k < kDecPerWarp; ++k) {
+        lg[k] = valid[k] ? lg[k] * a.scale + bias[k] : -INFINITY;
+        m = fmaxf(m, lg[k]);
+      }
+      float l = 0.f, ov[DPL];
+#pragma unroll
+      for (int i = 0; i < DPL; ++i) ov[i] = 0.f;
+#pragma unroll
+      for (int k = 0; k < kDecPerWarp; ++k) {
+        const float p = valid[k] ? __expf(lg[k] - m) : 0.f;
+        l += p;
+#pragma unroll
+        for (int i = 0; i < DPL / 2; ++i) {
+          const float2 vf = unpack_pair(vx[k][i]);
+          ov[2 * i] = fmaf(p, vf.x, ov[2 * i]);
+          ov[2 * i + 1] = fmaf(p, vf.y, ov[2 * i + 1]);
+        }
+      }
+      float* slot = red + ((size_t)warp * kDecRowGroup + rr) * (d + 2);
+#pragma unroll
+      for (int i = 0; i < DPL; ++i) slot[DPL * lane + i] = ov[i];
+      if (lane == 0) {
+        slot[d] = m;
+        slot[d + 1] = l;
+      }
     }
-    if (threadIdx.x == 0) part_ml[prow] = make_float2(m, lsum);
-    __syncthreads();  // pw and red are reused by the next row
+    __syncthreads();
+    // combine the warps' partials: one thread per (row, column)
+    for (int it = threadIdx.x; it < nr * d; it += kDecThreads) {
+      const int rr = it / d, c = it % d;
+      float M = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < kW; ++w) M = fmaxf(M, red[((size_t)w * kDecRowGroup + rr) * (d + 2) + d]);
+      float L = 0.f, O = 0.f;
+#pragma unroll
+      for (int w = 0; w < kW; ++w) {
+        const float* sl = red + ((size_t)w * kDecRowGroup + rr) * (d + 2);
+        const float wt = sl[d] == -INFINITY ? 0.f : __expf(sl[d] - M);
+        L += wt * sl[d + 1];
+        O += wt * sl[c];
+      }
+      const int r = r0 + rr;
+      const int n = r / g, qh = h * g + r % g;
+      const int64_t prow = ((int64_t)n * a.Hq + qh) * nch + chunk;
+      part_o[prow * d + c] = O;
+      if (c == 0) part_ml[prow] = make_float2(M, L);
+    }
+    __syncthreads();  // red is reused by the next row group
   }
 }
 
 // Output row (query n, query head qh): sum_s e^(m_s - M) O_s / sum_s e^(m_s - M) l_s over the
-// chunk partials, in chunk order. One warp per row.
+// chunk partials, in chunk order. One CTA of d threads per row, one column per thread.
 __global__ void decode_merge_kernel(const float* __restrict__ part_o,
                                     const float2* __restrict__ part_ml, int64_t rows, int nch,
                                     int d, __nv_bfloat16* __restrict__ out) {
-  const int64_t row = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
-  const int lane = threadIdx.x & 31;
-  if (row >= rows) return;
+  const int64_t row = blockIdx.x;
+  const int c = threadIdx.x;
+  if (row >= rows || c >= d) return;
   const float2* ml = part_ml + row * nch;
   float M = -INFINITY;
   for (int s = 0; s < nch; ++s) M = fmaxf(M, ml[s].x);
-  float L = 0.f;
-  for (int s = 0; s < nch; ++s)
-    if (ml[s].x != -INFINITY) L += __expf(ml[s].x - M) * ml[s].y;
-  const float inv = 1.f / L;
-  for (int c = lane; c < d; c += 32) {
-    float o = 0.f;
-    for (int s = 0; s < nch; ++s)
-      if (ml[s].x != -INFINITY) o += __expf(ml[s].x - M) * part_o[(row * nch + s) * d + c];
-    out[row * d + c] = __float2bfloat16_rn(o * inv);
+  float L = 0.f, o = 0.f;
+  const float* po = part_o + row * nch * d + c;
+#pragma unroll 8
+  for (int s = 0; s < nch; ++s) {
+    const float2 m = ml[s];
+    const float w = m.x != -INFINITY ? __expf(m.x - M) : 0.f;
+    L += w * m.y;
+    o += w * po[(int64_t)s * d];
   }
+  out[row * d + c] = __float2bfloat16_rn(o / L);
 }
 
 }  // namespace
@@ -803,31 +872,36 @@ inline unsigned blocks_for(int64_t n, int per) { return (unsigned)((n + per - 1)
 }  // namespace
 
 size_t decode_workspace_bytes(int64_t rows, int64_t entries, int d) {
-  const int64_t nch = (entries + kDecChunk - 1) / kDecChunk;
+  const int chunk = dec_chunk(d / 32);
+  const int64_t nch = (entries + chunk - 1) / chunk;
   return (size_t)rows * nch * d * 4 + (size_t)rows * nch * 8 + 256;
 }
 
 cudaError_t launch_decode_biased(const DecodeArgs& a, void* ws, cudaStream_t s) {
   const int64_t E = a.t + a.S;
-  const int nch = (int)((E + kDecChunk - 1) / kDecChunk);
+  const int chunk = dec_chunk(a.d / 32);
+  const int nch = (int)((E + chunk - 1) / chunk);
   const int g = a.Hq / a.H;
   const int G = a.nq * g;
   const int64_t rows = (int64_t)a.nq * a.Hq;
   float* part_o = static_cast<float*>(ws);
   float2* part_ml = reinterpret_cast<float2*>(
       static_cast<uint8_t*>(ws) + (((size_t)rows * nch * a.d * 4 + 255) & ~size_t(255)));
-  const size_t smem = (size_t)2 * kDecChunk * a.d * 2 + (size_t)G * a.d * 4 + kDecChunk * 4 + 64;
-  static thread_local size_t smem_set = 48 * 1024;
-  if (smem > smem_set) {
-    cudaError_t e = cudaFuncSetAttribute(decode_chunk_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  const size_t smem = ((size_t)G * a.d + (size_t)(kDecThreads / 32) * kDecRowGroup * (a.d + 2)) * 4;
+  auto kern = a.d == 64 ? decode_chunk_kernel<2>
+                        : a.d == 128 ? decode_chunk_kernel<4> : decode_chunk_kernel<8>;
+  static thread_local size_t smem_set[3] = {48 * 1024, 48 * 1024, 48 * 1024};
+  const int ki = a.d == 64 ? 0 : a.d == 128 ? 1 : 2;
+  if (smem > smem_set[ki]) {
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    smem_set = smem;
+    smem_set[ki] = smem;
   }
-  decode_chunk_kernel<<<dim3(nch, a.H), kDecThreads, smem, s>>>(a, part_o, part_ml);
+  kern<<<dim3(nch, a.H), kDecThreads, smem, s>>>(a, part_o, part_ml);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  decode_merge_kernel<<<blocks_for(rows, 8), 256, 0, s>>>(part_o, part_ml, rows, nch, a.d, a.out);
+  decode_merge_kernel<<<(unsigned)rows, a.d, 0, s>>>(part_o, part_ml, rows, nch, a.d, a.out);
   return cudaGetLastError();
 }
 

@@ -371,12 +371,10 @@ bool make_plan(const still_layer_config& c, bool lazy_q, int Kp, int64_t N, int 
   P.kb_b = Kp > 0 ? 0 : a256(N * 2 * D * 2);
   P.kss_b = a256(N * 4 * (kparts + 1));
   P.q_b = Kp > 0 ? 0 : a256(T * 2 * D * 2);
-  // The fused kernel holds fp16 probabilities and bf16 hi | lo q, k; a block that feeds
-  // another needs its probabilities in hi | lo and fp16 hi | lo q, k (its cross-attention
-  // output steers the next block's queries), so such blocks take the scores + P X kernels
-  // and only the last block is fused. The unit holds the larger of the two layouts.
+  // The fused kernel serves every block when 2d <= 256 (a block that feeds another takes its
+  // split-precision variant); 2d = 512 takes the scores + P X kernels.
   P.flash = d == 64 || d == 128;
-  P.split_ca = !P.flash || c.n_blocks > 1;
+  P.split_ca = !P.flash;
   P.S_b = 0;
   P.P_b = 0;
   P.O_b = 0;
@@ -709,7 +707,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       KLAUNCH(STILL_K_QROPE, launch_q_rope(qsrc, q_tmax, q_b0, nbl, t, D, qstart, qstep,
                                            L.omega_c, c.compactor_rope, qhl, exact ? 1 : 0,
                                            qscale, s));
-    if (P.flash && !exact) {
+    if (P.flash) {
       // S, the online softmax and P X in one kernel; per-split partials merged in order.
       float2* fst = stp;  // [nsplit][nbl * t] (the statistics region of this path)
       FlashParams fp;
@@ -721,7 +719,8 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       fp.bdiv = ni;
       fp.xbase_row = h0 * 2 * d;
       fp.tiles_m = (t + kBM - 1) / kBM;
-      fp.tiles_k = (int)((N + kFlashKeys - 1) / kFlashKeys);
+      const int fkeys = exact ? FlashSmem<256, true>::kKeys : kFlashKeys;
+      fp.tiles_k = (int)((N + fkeys - 1) / fkeys);
       fp.nsplit = flash_split((int64_t)fp.tiles_m * nbl, fp.tiles_k, ctx->nsm, kMaxFlashSplit);
       const int64_t nunits = (int64_t)fp.tiles_m * nbl * fp.nsplit;
       if (nunits > 0x7fffffff || (int64_t)nbl * N > 0x7fffffff) return STILL_ERR_UNSUPPORTED;
@@ -744,8 +743,11 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       }
       const Operand2D xop = op(XT, (int64_t)H * 2 * d, 2 * Np);
       ctx->prof.begin(STILL_K_CA_FUSED, s);
-      cudaError_t r = d == 64 ? launch_ca_flash<128>(qop, kop, xop, fp, ctx->nsm, s)
-                              : launch_ca_flash<256>(qop, kop, xop, fp, ctx->nsm, s);
+      cudaError_t r =
+          exact ? (d == 64 ? launch_ca_flash<128, true>(qop, kop, xop, fp, ctx->nsm, s)
+                           : launch_ca_flash<256, true>(qop, kop, xop, fp, ctx->nsm, s))
+                : (d == 64 ? launch_ca_flash<128>(qop, kop, xop, fp, ctx->nsm, s)
+                           : launch_ca_flash<256>(qop, kop, xop, fp, ctx->nsm, s));
       ctx->prof.end(STILL_K_CA_FUSED, s);
       if (r == cudaErrorInvalidValue) return STILL_ERR_INVALID_ARG;
       if (r != cudaSuccess) return STILL_ERR_CUDA;
