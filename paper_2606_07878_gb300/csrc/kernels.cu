@@ -722,7 +722,7 @@ __device__ __forceinline__ float2 unpack_pair(uint32_t w) {
 }
 
 template <int DPL>
-__global__ void __launch_bounds__(kDecThreads)
+__global__ void __launch_bounds__(kDecThreads, DPL == 2 ? 2 : 1)
     decode_chunk_kernel(DecodeArgs a, float* __restrict__ part_o, float2* __restrict__ part_ml) {
   extern __shared__ float dsm[];
   constexpr int d = 32 * DPL;
@@ -845,17 +845,18 @@ __global__ void __launch_bounds__(kDecThreads)
 __global__ void decode_merge_kernel(const float* __restrict__ part_o,
                                     const float2* __restrict__ part_ml, int64_t rows, int nch,
                                     int d, __nv_bfloat16* __restrict__ out) {
+  extern __shared__ float2 mls[];  // the row's (m, l) per chunk, then (weight, -)
   const int64_t row = blockIdx.x;
   const int c = threadIdx.x;
-  if (row >= rows || c >= d) return;
-  const float2* ml = part_ml + row * nch;
+  for (int s = c; s < nch; s += blockDim.x) mls[s] = part_ml[row * nch + s];  // coalesced
+  __syncthreads();
   float M = -INFINITY;
-  for (int s = 0; s < nch; ++s) M = fmaxf(M, ml[s].x);
+  for (int s = 0; s < nch; ++s) M = fmaxf(M, mls[s].x);
   float L = 0.f, o = 0.f;
   const float* po = part_o + row * nch * d + c;
 #pragma unroll 8
   for (int s = 0; s < nch; ++s) {
-    const float2 m = ml[s];
+    const float2 m = mls[s];
     const float w = m.x != -INFINITY ? __expf(m.x - M) : 0.f;
     L += w * m.y;
     o += w * po[(int64_t)s * d];
@@ -901,7 +902,9 @@ cudaError_t launch_decode_biased(const DecodeArgs& a, void* ws, cudaStream_t s) 
   kern<<<dim3(nch, a.H), kDecThreads, smem, s>>>(a, part_o, part_ml);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  decode_merge_kernel<<<(unsigned)rows, a.d, 0, s>>>(part_o, part_ml, rows, nch, a.d, a.out);
+  const size_t msm = (size_t)nch * sizeof(float2);
+  if (msm > 48 * 1024) return cudaErrorInvalidValue;  // more than 6144 chunks
+  decode_merge_kernel<<<(unsigned)rows, a.d, msm, s>>>(part_o, part_ml, rows, nch, a.d, a.out);
   return cudaGetLastError();
 }
 
