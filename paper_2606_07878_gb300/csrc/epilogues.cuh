@@ -19,7 +19,8 @@ struct AffineMap {
   }
 };
 
-enum OutKind : int32_t { OUT_F32 = 0, OUT_BF16 = 1, OUT_HILO = 2 };
+// OUT_HILO: bf16 hi and lo = bf16(x - hi); OUT_HILO16: the same in fp16 (about 22 bits).
+enum OutKind : int32_t { OUT_F32 = 0, OUT_BF16 = 1, OUT_HILO = 2, OUT_HILO16 = 3 };
 
 __device__ __forceinline__ void split_hilo(float x, __nv_bfloat16& hi, __nv_bfloat16& lo) {
   hi = __float2bfloat16_rn(x);
@@ -72,6 +73,18 @@ __device__ __forceinline__ void pack_hilo_x32(const float (&v)[32], uint4 (&h4)[
     uint32_t h[4], l[4];
 #pragma unroll
     for (int k = 0; k < 4; ++k) split_pack(v[8 * q + 2 * k], v[8 * q + 2 * k + 1], h[k], l[k]);
+    h4[q] = make_uint4(h[0], h[1], h[2], h[3]);
+    l4[q] = make_uint4(l[0], l[1], l[2], l[3]);
+  }
+}
+
+__device__ __forceinline__ void pack_hilo16_x32(const float (&v)[32], uint4 (&h4)[4],
+                                                uint4 (&l4)[4]) {
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    uint32_t h[4], l[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) split_pack_f16(v[8 * q + 2 * k], v[8 * q + 2 * k + 1], h[k], l[k]);
     h4[q] = make_uint4(h[0], h[1], h[2], h[3]);
     l4[q] = make_uint4(l[0], l[1], l[2], l[3]);
   }
@@ -300,9 +313,12 @@ struct EpiAffine {
         pack_f32x16(v + 16, b4);
         warp_store64(stage, a4, dst, rvalid);
         warp_store64(stage, b4, dst + 16, rvalid);
-      } else if (kind == OUT_HILO) {
+      } else if (kind == OUT_HILO || kind == OUT_HILO16) {
         __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(out) + o;
-        pack_hilo_x32(v, a4, b4);
+        if (kind == OUT_HILO)
+          pack_hilo_x32(v, a4, b4);
+        else
+          pack_hilo16_x32(v, a4, b4);
         warp_store64(stage, a4, dst, rvalid);
         warp_store64(stage, b4, dst + lo_off, rvalid);
       } else {
@@ -321,6 +337,11 @@ struct EpiAffine {
         static_cast<float*>(out)[o] = v[e];
       } else if (kind == OUT_BF16) {
         static_cast<__nv_bfloat16*>(out)[o] = __float2bfloat16_rn(v[e]);
+      } else if (kind == OUT_HILO16) {
+        const __half hh = __float2half_rn(v[e]);
+        const __half ll = __float2half_rn(v[e] - __half2float(hh));
+        reinterpret_cast<__half*>(out)[o] = hh;
+        reinterpret_cast<__half*>(out)[o + lo_off] = ll;
       } else {
         __nv_bfloat16 h, l;
         split_hilo(v[e], h, l);

@@ -364,8 +364,8 @@ __global__ void __launch_bounds__(256) softmax_kernel(const float* __restrict__ 
 }
 
 // Row softmax with the row held in registers: 256 threads, PER columns each (float4 groups).
-// HILO (bf16 only): the row is written as hi at [0, ldP) and lo = bf16(p - hi) at
-// [ldP, 2 ldP) of a row of pitch 2 ldP.
+// HILO: the row is written as hi at [0, ldP) and lo = OutT(p - hi) at [ldP, 2 ldP) of a row of
+// pitch 2 ldP (bf16 or fp16 parts).
 template <typename OutT, int PER, bool HILO = false>
 __global__ void __launch_bounds__(256) softmax_reg_kernel(const float* __restrict__ S,
                                                           int64_t ncols, int64_t ldS,
@@ -425,6 +425,7 @@ __global__ void __launch_bounds__(256) softmax_reg_kernel(const float* __restric
         const float y = v[4 * i + k] * inv;
         if constexpr (std::is_same<OutT, __half>::value) {
           o4[k] = __float2half_rn(y);
+          if constexpr (HILO) l4[k] = __float2half_rn(y - __half2float(o4[k]));
         } else {
           o4[k] = __float2bfloat16_rn(y);
           if constexpr (HILO) l4[k] = __float2bfloat16_rn(y - __bfloat162float(o4[k]));
@@ -501,7 +502,8 @@ __global__ void px_to_hilo_kernel(const float* __restrict__ O, int nsplit, int64
 __global__ void __launch_bounds__(256) ca_merge_kernel(const float* __restrict__ O,
                                                        const float2* __restrict__ stats,
                                                        int nsplit, int b0, int nb, int n, int t,
-                                                       int d2, __nv_bfloat16* __restrict__ PX) {
+                                                       int d2, int f16,
+                                                       __nv_bfloat16* __restrict__ PX) {
   const int64_t rows = (int64_t)nb * t;
   const int64_t rj = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -529,8 +531,13 @@ __global__ void __launch_bounds__(256) ca_merge_kernel(const float* __restrict__
       acc.w += w * o.w;
     }
     uint32_t h01, l01, h23, l23;
-    split_pack(acc.x * invL, acc.y * invL, h01, l01);
-    split_pack(acc.z * invL, acc.w * invL, h23, l23);
+    if (f16) {  // fp16 hi | lo
+      split_pack_f16(acc.x * invL, acc.y * invL, h01, l01);
+      split_pack_f16(acc.z * invL, acc.w * invL, h23, l23);
+    } else {
+      split_pack(acc.x * invL, acc.y * invL, h01, l01);
+      split_pack(acc.z * invL, acc.w * invL, h23, l23);
+    }
     *reinterpret_cast<uint2*>(row + c) = make_uint2(h01, h23);
     *reinterpret_cast<uint2*>(row + (int64_t)n * d2 + c) = make_uint2(l01, l23);
   }
@@ -1017,8 +1024,9 @@ cudaError_t launch_omega(double* out, int half, int width, double base, cudaStre
 cudaError_t launch_softmax(const float* S, int64_t rows, int64_t ncols, int64_t ldS, void* P,
                            int64_t ldP, int out_fp16, cudaStream_t s) {
   if (rows == 0) return cudaSuccess;
-  if (out_fp16 == 2) {  // bf16 hi | lo rows
-    if (!softmax_reg<__nv_bfloat16, true>(S, rows, ncols, ldS, P, ldP, s))
+  if (out_fp16 == 2 || out_fp16 == 3) {  // bf16 (2) or fp16 (3) hi | lo rows
+    if (!(out_fp16 == 2 ? softmax_reg<__nv_bfloat16, true>(S, rows, ncols, ldS, P, ldP, s)
+                        : softmax_reg<__half, true>(S, rows, ncols, ldS, P, ldP, s)))
       return cudaErrorInvalidValue;
     return cudaGetLastError();
   }
@@ -1043,12 +1051,12 @@ cudaError_t launch_px_to_hilo(const float* O, int nsplit, int64_t split_stride, 
 }
 
 cudaError_t launch_ca_merge(const float* O, const float2* stats, int nsplit, int b0, int nb,
-                            int n, int t, int d2, __nv_bfloat16* PX, cudaStream_t s) {
+                            int n, int t, int d2, int f16, __nv_bfloat16* PX, cudaStream_t s) {
   const int64_t total = (int64_t)nb * t * d2;
   if (total == 0) return cudaSuccess;
   if (d2 % 4 != 0) return cudaErrorInvalidValue;
   ca_merge_kernel<<<blocks_for((int64_t)nb * t, 8), 256, 0, s>>>(O, stats, nsplit, b0, nb, n, t,
-                                                                  d2, PX);
+                                                                  d2, f16, PX);
   return cudaGetLastError();
 }
 

@@ -102,7 +102,7 @@ cudaError_t launch_omega(double* out, int half, int width, double base, cudaStre
 
 // Row softmax: S fp32 [rows][ldS] (first ncols valid) -> P [rows][ldP], zero beyond ncols.
 // out_fp16: 1 = P is fp16; 0 = bf16; 2 = bf16 hi | lo: rows of pitch 2 ldP, hi at [0, ldP),
-// lo = bf16(p - hi) at [ldP, 2 ldP) (ldP and ncols up to 16384).
+// lo = bf16(p - hi) at [ldP, 2 ldP) (ldP and ncols up to 16384); 3 = the same in fp16.
 cudaError_t launch_softmax(const float* S, int64_t rows, int64_t ncols, int64_t ldS, void* P,
                            int64_t ldP, int out_fp16, cudaStream_t s);
 
@@ -114,9 +114,9 @@ cudaError_t launch_px_to_hilo(const float* O, int nsplit, int64_t split_stride, 
 
 // Key-split merge of the fused cross-attention: O [nsplit][nb][t][2d] unnormalised partials with
 // stats [nsplit][nb][t] = (max in log2 units, sum) -> normalised hi/lo bf16 rows of PXcat
-// (layout as launch_px_to_hilo). Splits are combined in a fixed order.
+// (layout as launch_px_to_hilo; f16: fp16 hi | lo instead). Splits are combined in a fixed order.
 cudaError_t launch_ca_merge(const float* O, const float2* stats, int nsplit, int b0, int nb,
-                            int n, int t, int d2, __nv_bfloat16* PX, cudaStream_t s);
+                            int n, int t, int d2, int f16, __nv_bfloat16* PX, cudaStream_t s);
 
 // out[i] = alpha / max(sqrt(sum_k part(i, k)), eps), summed in slot order: the L2 / QK-norm
 // factor of vector i from the epilogues' sum-of-squares partials. Vectors come in blocks of

@@ -514,6 +514,10 @@ bool queries_per_call(const LayerW& L) {
 
 int fold_kp(const LayerW& L) { return L.fold ? L.Kp : 0; }
 
+// The fp16 hi | lo copy of W_V W_O of a block that feeds another is stored multiplied by this
+// power of two: its entries (products of two weights) sit near the fp16 subnormal range.
+constexpr float kWvoScale = 256.f;
+
 still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
                          const Positions& pos, int64_t N, int t, const OutSpec& out,
                          cudaStream_t s, uint8_t* ws_fixed = nullptr,
@@ -563,8 +567,14 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
   const bool last = bi + 1 == c.n_blocks;
   // A block whose output enters another block keeps its cross-attention, self-attention
   // value path and FFN in split precision: the next block's cross-attention queries amplify
-  // any rounding there.
+  // any rounding there. In a two-block layer the last block keeps its value path and FFN in
+  // hi | lo too, and the first block's value chains (P X, W_V W_O, RMSNorm(Z'), the
+  // self-attention q, k, v, P and head outputs) are fp16 hi | lo rather than bf16 hi | lo.
   const bool exact = !last;
+  const bool vexact = exact || L.f16;
+  const bool f16v = exact && L.f16 && P.flash;
+  const int vfmt = f16v ? 0 : 1;
+  const int32_t vkind = f16v ? OUT_HILO16 : OUT_HILO;
   float* Za = Z2;  // this block's state after cross-attention (Z2 itself without it)
   if (Bw.has_ca) {
   const bool q_call = bi > 0 || L.qhat_lazy;  // queries formed in this call
@@ -751,7 +761,8 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       ctx->prof.end(STILL_K_CA_FUSED, s);
       if (r == cudaErrorInvalidValue) return STILL_ERR_INVALID_ARG;
       if (r != cudaSuccess) return STILL_ERR_CUDA;
-      KLAUNCH(STILL_K_PXSPLIT, launch_ca_merge(O, fst, fp.nsplit, b0, nbl, n, t, 2 * d, PX, s));
+      KLAUNCH(STILL_K_PXSPLIT, launch_ca_merge(O, fst, fp.nsplit, b0, nbl, n, t, 2 * d,
+                                               f16v ? 1 : 0, PX, s));
       b0 += nbl;
       continue;
     }
@@ -854,11 +865,13 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.resm.c0 = 1;
     }
     e.vec_ok = 1;
-    TRY(run_gemm256<STILL_K_VO>(ctx, op(PX, rows, 2 * n2d), op(Bw.WvoT, D, 2 * n2d), p, e, 1, s));
+    e.alpha = f16v ? 1.f / kWvoScale : 1.f;  // the fp16 W_V W_O copy is stored scaled
+    TRY(run_gemm256<STILL_K_VO>(ctx, op(PX, rows, 2 * n2d), op(Bw.WvoT, D, 2 * n2d), p, e, vfmt,
+                                s));
   }
   Za = Z1;
   }  // cross-attention of block bi
-  KLAUNCH(STILL_K_NORM, launch_rmsnorm(Za, 0, rows, D, D, c.rms_eps, A1, 2 * D, 1, s));
+  KLAUNCH(STILL_K_NORM, launch_rmsnorm(Za, 0, rows, D, D, c.rms_eps, A1, 2 * D, f16v ? 2 : 1, s));
 
   // ---------------------------------------------------------------- latent self-attention
   for (int h0 = 0; h0 < H; h0 += P.sa_heads) {
@@ -883,7 +896,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       add_pass(p, 0, 0, h0 * t, 0, D);
       add_pass(p, D, 0, h0 * t, 0, D);
       EpiAffine e;
-      e.kind = OUT_HILO;
+      e.kind = vkind;
       e.out = qk;
       e.lo_off = D;
       e.om.rdiv = t;
@@ -902,16 +915,17 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.ss_parts = sparts;
       e.ss_block = t;
       e.vec_ok = 1;
-      TRY(run_gemm256<STILL_K_SA_PROJ>(ctx, op(A1, rows, 2 * D), op(Bw.SqkT, (int64_t)2 * n * D, D), p, e, 1, s));
+      TRY(run_gemm256<STILL_K_SA_PROJ>(ctx, op(A1, rows, 2 * D), op(Bw.SqkT, (int64_t)2 * n * D, D),
+                                       p, e, vfmt, s));
     }
     KLAUNCH(STILL_K_NORMS,
             launch_inv_norms(sss, (int64_t)nh * 2 * n * t, sparts, t, c.l2_eps, 1.f, sinv, s));
     {  // v^T = S_V^T RMSNorm(Z')^T  -> [nD][nh * tp]  (hi, then lo rows when exact)
       GemmParams p = gp(n * D, nh * t);
       add_pass(p, 0, 0, 0, h0 * t, D);
-      if (exact) add_pass(p, 0, D, 0, h0 * t, D);
+      if (vexact) add_pass(p, 0, D, 0, h0 * t, D);
       EpiAffine e;
-      e.kind = exact ? OUT_HILO : OUT_BF16;
+      e.kind = vexact ? vkind : OUT_BF16;
       e.lo_off = (int64_t)n * D * nh * P.tp;
       e.out = vT;
       e.om.r0 = (int64_t)nh * P.tp;
@@ -919,7 +933,8 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.om.c1 = P.tp;
       e.om.c0 = 1;
       e.vec_ok = (t % 32 == 0);
-      TRY(run_gemm256<STILL_K_SA_V>(ctx, op(Bw.SvT, (int64_t)n * D, D), op(A1, rows, 2 * D), p, e, 1, s));
+      TRY(run_gemm256<STILL_K_SA_V>(ctx, op(Bw.SvT, (int64_t)n * D, D), op(A1, rows, 2 * D), p, e,
+                                    vfmt, s));
     }
     // Self heads [i0, i0 + ns) of the nh banks per pass (all n unless one bank is too big).
     for (int i0 = 0; i0 < n; i0 += P.sa_sub) {
@@ -957,25 +972,27 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
         const StoreView3D sv = store_view(Ssa, 4, t, t, (int64_t)nh * ns, P.ldt,
                                           (int64_t)t * P.ldt, 32, true);
         TRY(run_gemm256<STILL_K_SA_SCORES>(ctx, op(qk, (int64_t)nh * 2 * n * t, 2 * D),
-                                           op(qk, (int64_t)nh * 2 * n * t, 2 * D), p, e, 1, s, &sv));
+                                           op(qk, (int64_t)nh * 2 * n * t, 2 * D), p, e, vfmt, s,
+                                           &sv));
       }
       KLAUNCH(STILL_K_SA_SOFTMAX,
-              launch_softmax(Ssa, (int64_t)nh * ns * t, t, P.ldt, Psa, P.tp, exact ? 2 : 0, s));
+              launch_softmax(Ssa, (int64_t)nh * ns * t, t, P.ldt, Psa, P.tp,
+                             f16v ? 3 : vexact ? 2 : 0, s));
       {  // heads = P v -> concat rows (h0 + hh) * t + j, columns (i0 + bi) * D + f
         // exact: P_hi v_hi + P_hi v_lo + P_lo v_hi, concat rows of hi | lo
-        const int64_t cw = exact ? 2 * (int64_t)n * D : (int64_t)n * D;  // concat row pitch
+        const int64_t cw = vexact ? 2 * (int64_t)n * D : (int64_t)n * D;  // concat row pitch
         GemmParams p = gp(t, D, nh * ns, ns);
         p.a_r1 = (int64_t)ns * t;
         p.a_r0 = t;
         p.b_r0 = D;
         p.b_k1 = P.tp;
         add_pass(p, 0, 0, 0, i0 * D, (int)P.tp);
-        if (exact) {
+        if (vexact) {
           add_pass(p, 0, 0, 0, n * D + i0 * D, (int)P.tp);
           add_pass(p, (int)P.tp, 0, 0, i0 * D, (int)P.tp);
         }
         EpiAffine e;
-        e.kind = exact ? OUT_HILO : OUT_BF16;
+        e.kind = vexact ? vkind : OUT_BF16;
         e.lo_off = (int64_t)n * D;
         e.out = cat;
         e.om.bdiv = ns;
@@ -986,15 +1003,15 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
         e.om.k = (int64_t)h0 * t * cw + (int64_t)i0 * D;
         e.vec_ok = 1;
         TRY(run_gemm256<STILL_K_SA_PV>(
-            ctx, op(Psa, (int64_t)nh * ns * t, exact ? 2 * P.tp : P.tp),
-            op(vT, (exact ? 2 : 1) * (int64_t)n * D, (int64_t)nh * P.tp), p, e, 1, s));
+            ctx, op(Psa, (int64_t)nh * ns * t, vexact ? 2 * P.tp : P.tp),
+            op(vT, (vexact ? 2 : 1) * (int64_t)n * D, (int64_t)nh * P.tp), p, e, vfmt, s));
       }
     }
   }
-  {  // Z'' = Z' + concat S_O  (exact: concat hi | lo, 2 passes)
+  {  // Z'' = Z' + concat S_O  (hi | lo concat: 2 passes)
     GemmParams p = gp((int)rows, D);
     add_pass(p, 0, 0, 0, 0, n * D);
-    if (exact) add_pass(p, n * D, 0, 0, 0, n * D);
+    if (vexact) add_pass(p, n * D, 0, 0, 0, n * D);
     EpiAffine e;
     const bool direct = last && (F == 0) && z3_bf16;
     e.kind = direct ? OUT_HILO : OUT_F32;
@@ -1007,32 +1024,32 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     e.resm.r0 = D;
     e.resm.c0 = 1;
     e.vec_ok = 1;
-    TRY(run_gemm256<STILL_K_SO>(ctx, op(cat, rows, (exact ? 2 : 1) * (int64_t)n * D),
-                                op(Bw.SoT, D, (int64_t)n * D), p, e, 1, s));
+    TRY(run_gemm256<STILL_K_SO>(ctx, op(cat, rows, (vexact ? 2 : 1) * (int64_t)n * D),
+                                op(Bw.SoT, D, (int64_t)n * D), p, e, vfmt, s));
   }
   if (F > 0) {
-    // exact: RMSNorm(Z'') and GELU(.) as hi | lo, both products in 2 passes
-    KLAUNCH(STILL_K_NORM, launch_rmsnorm(Z2, 0, rows, D, D, c.rms_eps, A2, exact ? 2 * D : D,
-                                         exact ? 1 : 0, s));
+    // vexact: RMSNorm(Z'') and GELU(.) as hi | lo, both products in 2 passes
+    KLAUNCH(STILL_K_NORM, launch_rmsnorm(Z2, 0, rows, D, D, c.rms_eps, A2, vexact ? 2 * D : D,
+                                         vexact ? 1 : 0, s));
     {
       GemmParams p = gp((int)rows, F);
       add_pass(p, 0, 0, 0, 0, D);
-      if (exact) add_pass(p, D, 0, 0, 0, D);
+      if (vexact) add_pass(p, D, 0, 0, 0, D);
       EpiAffine e;
-      e.kind = exact ? OUT_HILO : OUT_BF16;
+      e.kind = vexact ? OUT_HILO : OUT_BF16;
       e.lo_off = F;
       e.out = Gb;
-      e.om.r0 = exact ? 2 * F : F;
+      e.om.r0 = vexact ? 2 * F : F;
       e.om.c0 = 1;
       e.gelu = 1;
       e.vec_ok = 1;
-      TRY(run_gemm256<STILL_K_FFN1>(ctx, op(A2, rows, exact ? 2 * D : D), op(Bw.W1T, F, D), p, e,
+      TRY(run_gemm256<STILL_K_FFN1>(ctx, op(A2, rows, vexact ? 2 * D : D), op(Bw.W1T, F, D), p, e,
                                     1, s));
     }
     {
       GemmParams p = gp((int)rows, D);
       add_pass(p, 0, 0, 0, 0, F);
-      if (exact) add_pass(p, F, 0, 0, 0, F);
+      if (vexact) add_pass(p, F, 0, 0, 0, F);
       EpiAffine e;
       const bool direct = last && z3_bf16;
       e.kind = direct ? OUT_HILO : OUT_F32;
@@ -1046,7 +1063,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       e.resm.c0 = 1;
       e.vec_ok = 1;
       // In place (Z2 -> Z2) is safe: each element is read and written by the same thread.
-      TRY(run_gemm256<STILL_K_FFN2>(ctx, op(Gb, rows, exact ? 2 * F : F), op(Bw.W2T, D, F), p, e,
+      TRY(run_gemm256<STILL_K_FFN2>(ctx, op(Gb, rows, vexact ? 2 * F : F), op(Bw.W2T, D, F), p, e,
                                     1, s));
     }
   }
@@ -1184,6 +1201,14 @@ still_status load_layer(still_ctx* ctx, int32_t layer, const still_layer_config*
                      0, s));
       CK(launch_transpose(static_cast<const bf16*>(w.Sv), D, nD, B.SvT, 0, s));
       CK(launch_transpose(static_cast<const bf16*>(w.So), nD, D, B.SoT, 0, s));
+      // The first block of a two-block layer runs its value chains in fp16 (with the fused
+      // cross-attention kernel, 2d <= 256): its self-attention weights as fp16 copies.
+      const bool f16v = L.f16 && b + 1 < NB && (d == 64 || d == 128);
+      if (f16v) {
+        CK(launch_bf16_to_f16(B.SqkT, 2 * nD * D, s));
+        CK(launch_bf16_to_f16(B.SvT, nD * D, s));
+        CK(launch_bf16_to_f16(B.SoT, (int64_t)D * nD, s));
+      }
       if (F > 0) {
         TRY(dalloc(L, &B.W1T, (size_t)F * D));
         TRY(dalloc(L, &B.W2T, (size_t)D * F));
@@ -1254,7 +1279,8 @@ still_status load_layer(still_ctx* ctx, int32_t layer, const still_layer_config*
       p.b_k1 = D;
       add_pass(p, 0, 0, 0, 0, D);
       EpiAffine e;
-      e.kind = OUT_HILO;
+      e.kind = f16v ? OUT_HILO16 : OUT_HILO;
+      e.alpha = f16v ? kWvoScale : 1.f;
       e.out = B.WvoT;
       e.lo_off = (int64_t)n * 2 * d;
       e.om.b1 = 2 * d;
