@@ -446,9 +446,11 @@ def test_qwen3_4b_canonical_4k_all_heads():
 # Full-size canonical layer: max|err| bound. Rounding the oracle's own outputs to bf16 already
 # costs 0.012-0.016 x RMS on this layer (its elements reach 5 x RMS), and evaluating the
 # oracle's steps in fp32 lands at 0.011-0.018 x RMS: the second block's cross-attention over
-# 65536 keys magnifies first-block rounding in a few latents. The GPU path measures
-# 0.016-0.031 on KV-heads 0, 1 and 5 (row medians at the bf16 floor, 1.7e-3); the cosine bar
-# is kept. At 4k tokens the same compactor meets the standard bar on every head (above).
+# 65536 keys magnifies first-block rounding in a few latents. The GPU path measures 0.0166,
+# 0.0157 and 0.0307 on KV-heads 0, 1 and 5 (row medians at the bf16 floor, 1.7e-3); the last
+# comes from one latent whose second-block logits are nearly tied (gap 0.048), where the row
+# error (1.0e-2) did not move under any operand-precision change tried. The cosine bar is
+# kept. At 4k tokens the same compactor meets the standard bar on every head (above).
 CANONICAL_64K_ERR = 0.04
 
 
