@@ -692,18 +692,20 @@ __global__ void beta_kernel(const __nv_bfloat16* __restrict__ Z, int64_t rows, i
 // ----------------------------------------------------------------- biased decode attention
 //
 // Attention of query rows over the entries [C (t compact slots, logit bias beta) ; F (S
-// uncompacted entries, bias 0)] (App. B, "Bias semantics in attention"). Grid (chunk, KV-head):
-// a CTA of 8 warps covers dec_chunk entries of its KV-head (16 per warp, 8 at d = 256). A lane
-// holds DPL = d/32 dimensions of each of its warp's keys and values in registers (coalesced
-// loads, all issued up front), so the cache is read once and straight from global memory. Per
-// query row of the KV-head's query heads, each warp forms its logits (warp-sum of the lane
-// partials), their
-// max, weights and weighted values; the 8 warps' (max, sum, O) are combined through shared
-// memory into one partial per (row, chunk), and decode_merge_kernel combines the chunks in order.
-constexpr int kDecThreads = 256;
+// uncompacted entries, bias 0)] (App. B, "Bias semantics in attention"). Grid (slot, KV-head),
+// one wave: the CTAs of a KV-head take its chunks of dec_chunk entries in turn (slot, slot +
+// slots, ...). In a chunk each of the 16 warps holds 8 entries (4 at d = 256); a lane holds
+// DPL = d/32 dimensions of its warp's keys and values in registers (coalesced loads, all issued
+// up front), so the cache is read once and straight from global memory. Per query row of the
+// KV-head's query heads, each warp forms its logits (warp sums of the lane partials), their max,
+// weights and weighted values; the warps' (max, sum, O) are combined through shared memory and
+// merged into the CTA's running row state, which is written once as the CTA's partial;
+// decode_merge_kernel combines the partials in slot order.
+constexpr int kDecThreads = 512;
 constexpr int kDecRowGroup = 4;  // query rows per pass
-// entries per warp: 16 (8 at d = 256, whose 8 dimensions per lane double the registers)
-__host__ __device__ constexpr int dec_per_warp(int dpl) { return dpl == 8 ? 8 : 16; }
+// entries per warp: 8 (4 at d = 256, whose 8 dimensions per lane double the registers); 16
+// warps keep more loads and more independent instruction streams in flight per SM
+__host__ __device__ constexpr int dec_per_warp(int dpl) { return dpl == 8 ? 4 : 8; }
 __host__ __device__ constexpr int dec_chunk(int dpl) { return dec_per_warp(dpl) * kDecThreads / 32; }
 
 // DPL consecutive bf16 as DPL / 2 packed pairs (one 4-, 8- or 16-byte load).
@@ -729,121 +731,150 @@ __device__ __forceinline__ float2 unpack_pair(uint32_t w) {
 }
 
 template <int DPL>
-__global__ void __launch_bounds__(kDecThreads, DPL == 2 ? 2 : 1)
+__global__ void __launch_bounds__(kDecThreads, 1)
     decode_chunk_kernel(DecodeArgs a, float* __restrict__ part_o, float2* __restrict__ part_ml) {
   extern __shared__ float dsm[];
   constexpr int d = 32 * DPL;
   constexpr int kW = kDecThreads / 32;
   constexpr int kDecPerWarp = dec_per_warp(DPL);
   constexpr int kDecChunk = dec_chunk(DPL);
-  const int h = blockIdx.y, chunk = blockIdx.x;
+  const int h = blockIdx.y, slot = blockIdx.x, nslots = gridDim.x;
   const int g = a.Hq / a.H;        // query heads per KV-head
   const int G = a.nq * g;          // query rows served by this CTA
   float* qs = dsm;                                  // [G][d]
   float* red = qs + (size_t)G * d;                  // [kW][kDecRowGroup][d + 2]
+  float* acc = red + (size_t)kW * kDecRowGroup * (d + 2);  // [G][d + 2]: running O, M, L
+  float* mlx = acc + (size_t)G * (d + 2);           // [kDecRowGroup][2]: next M, L
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t E = a.t + a.S;
-  // this warp's keys and values (lane dims [DPL lane, +DPL))
-  uint32_t kx[kDecPerWarp][DPL / 2], vx[kDecPerWarp][DPL / 2];  // packed bf16 pairs
-  float bias[kDecPerWarp];
-  bool valid[kDecPerWarp];
-#pragma unroll
-  for (int k = 0; k < kDecPerWarp; ++k) {
-    const int64_t e = (int64_t)chunk * kDecChunk + warp * kDecPerWarp + k;
-    valid[k] = e < E;
-    bias[k] = 0.f;
-    if (valid[k]) {
-      const bool comp = e < a.t;
-      const int64_t off = (comp ? e * a.cst : (e - a.t) * a.fst) + (int64_t)h * d + DPL * lane;
-      load_pairs<DPL>((comp ? a.Ck : a.Kf) + off, kx[k]);
-      load_pairs<DPL>((comp ? a.Cv : a.Vf) + off, vx[k]);
-      if (comp && a.beta != nullptr) bias[k] = a.beta[e * a.H + h];
-    } else {
-#pragma unroll
-      for (int i = 0; i < DPL / 2; ++i) kx[k][i] = vx[k][i] = 0u;
-    }
-  }
+  const int64_t nch = (E + kDecChunk - 1) / kDecChunk;
   // query rows of this KV-head: row r = (query n, head h * g + r % g), n = r / g
   for (int it = threadIdx.x; it < G * d; it += kDecThreads) {
     const int r = it / d, c = it % d;
     const int n = r / g, qh = h * g + r % g;
     qs[it] = __bfloat162float(a.q[((int64_t)n * a.Hq + qh) * d + c]);
   }
+  for (int it = threadIdx.x; it < G * (d + 2); it += kDecThreads)
+    acc[it] = (it % (d + 2)) == d ? -INFINITY : 0.f;
   __syncthreads();
-  const int64_t nch = gridDim.x;
-  for (int r0 = 0; r0 < G; r0 += kDecRowGroup) {
-    const int nr = min(kDecRowGroup, G - r0);
+  // This CTA's chunks: slot, slot + nslots, ... (in order), merged into acc as they come.
+  for (int64_t chunk = slot; chunk < nch; chunk += nslots) {
+    // this warp's keys and values (lane dims [DPL lane, +DPL)), packed bf16 pairs
+    uint32_t kx[kDecPerWarp][DPL / 2], vx[kDecPerWarp][DPL / 2];
+    float bias[kDecPerWarp];
+    bool valid[kDecPerWarp];
+#pragma unroll
+    for (int k = 0; k < kDecPerWarp; ++k) {
+      const int64_t e = chunk * kDecChunk + warp * kDecPerWarp + k;
+      valid[k] = e < E;
+      bias[k] = 0.f;
+      if (valid[k]) {
+        const bool comp = e < a.t;
+        const int64_t off = (comp ? e * a.cst : (e - a.t) * a.fst) + (int64_t)h * d + DPL * lane;
+        load_pairs<DPL>((comp ? a.Ck : a.Kf) + off, kx[k]);
+        load_pairs<DPL>((comp ? a.Cv : a.Vf) + off, vx[k]);
+        if (comp && a.beta != nullptr) bias[k] = a.beta[e * a.H + h];
+      } else {
+#pragma unroll
+        for (int i = 0; i < DPL / 2; ++i) kx[k][i] = vx[k][i] = 0u;
+      }
+    }
+    for (int r0 = 0; r0 < G; r0 += kDecRowGroup) {
+      const int nr = min(kDecRowGroup, G - r0);
 #pragma unroll 1
-    for (int rr = 0; rr < nr; ++rr) {
-      float qv[DPL];
+      for (int rr = 0; rr < nr; ++rr) {
+        float qv[DPL];
 #pragma unroll
-      for (int i = 0; i < DPL; ++i) qv[i] = qs[(size_t)(r0 + rr) * d + DPL * lane + i];
-      float lg[kDecPerWarp];
+        for (int i = 0; i < DPL; ++i) qv[i] = qs[(size_t)(r0 + rr) * d + DPL * lane + i];
+        float lg[kDecPerWarp];
 #pragma unroll
-      for (int k = 0; k < kDecPerWarp; ++k) {
-        float s = 0.f;
+        for (int k = 0; k < kDecPerWarp; ++k) {
+          float sdot = 0.f;
 #pragma unroll
-        for (int i = 0; i < DPL / 2; ++i) {
-          const float2 kf = unpack_pair(kx[k][i]);
-          s = fmaf(qv[2 * i], kf.x, fmaf(qv[2 * i + 1], kf.y, s));
+          for (int i = 0; i < DPL / 2; ++i) {
+            const float2 kf = unpack_pair(kx[k][i]);
+            sdot = fmaf(qv[2 * i], kf.x, fmaf(qv[2 * i + 1], kf.y, sdot));
+          }
+          lg[k] = sdot;
         }
-        lg[k] = s;
-      }
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
+        for (int o = 16; o > 0; o >>= 1) {
 #pragma unroll
-        for (int k = 0; k < kDecPerWarp; ++k) lg[k] += __shfl_xor_sync(0xffffffffu, lg[k], o);
-      }
-      float m = -INFINITY;
+          for (int k = 0; k < kDecPerWarp; ++k) lg[k] += __shfl_xor_sync(0xffffffffu, lg[k], o);
+        }
+        float m = -INFINITY;
 #pragma unroll
-      for (int k = 0; k < kDecPerWarp; ++k) {
-        lg[k] = valid[k] ? lg[k] * a.scale + bias[k] : -INFINITY;
-        m = fmaxf(m, lg[k]);
-      }
-      float l = 0.f, ov[DPL];
+        for (int k = 0; k < kDecPerWarp; ++k) {
+          lg[k] = valid[k] ? lg[k] * a.scale + bias[k] : -INFINITY;
+          m = fmaxf(m, lg[k]);
+        }
+        float l = 0.f, ov[DPL];
 #pragma unroll
-      for (int i = 0; i < DPL; ++i) ov[i] = 0.f;
+        for (int i = 0; i < DPL; ++i) ov[i] = 0.f;
 #pragma unroll
-      for (int k = 0; k < kDecPerWarp; ++k) {
-        const float p = valid[k] ? __expf(lg[k] - m) : 0.f;
-        l += p;
+        for (int k = 0; k < kDecPerWarp; ++k) {
+          const float p = valid[k] ? __expf(lg[k] - m) : 0.f;
+          l += p;
 #pragma unroll
-        for (int i = 0; i < DPL / 2; ++i) {
-          const float2 vf = unpack_pair(vx[k][i]);
-          ov[2 * i] = fmaf(p, vf.x, ov[2 * i]);
-          ov[2 * i + 1] = fmaf(p, vf.y, ov[2 * i + 1]);
+          for (int i = 0; i < DPL / 2; ++i) {
+            const float2 vf = unpack_pair(vx[k][i]);
+            ov[2 * i] = fmaf(p, vf.x, ov[2 * i]);
+            ov[2 * i + 1] = fmaf(p, vf.y, ov[2 * i + 1]);
+          }
+        }
+        float* sl = red + ((size_t)warp * kDecRowGroup + rr) * (d + 2);
+#pragma unroll
+        for (int i = 0; i < DPL; ++i) sl[DPL * lane + i] = ov[i];
+        if (lane == 0) {
+          sl[d] = m;
+          sl[d + 1] = l;
         }
       }
-      float* slot = red + ((size_t)warp * kDecRowGroup + rr) * (d + 2);
+      __syncthreads();
+      // Combine the warps' partials of this chunk and merge them into the running row state:
+      // one thread per (row, column); the new (M, L) go through mlx so that no thread reads
+      // a row's M after another has replaced it.
+      for (int it = threadIdx.x; it < nr * d; it += kDecThreads) {
+        const int rr = it / d, c = it % d;
+        float Mc = -INFINITY;
 #pragma unroll
-      for (int i = 0; i < DPL; ++i) slot[DPL * lane + i] = ov[i];
-      if (lane == 0) {
-        slot[d] = m;
-        slot[d + 1] = l;
+        for (int w = 0; w < kW; ++w)
+          Mc = fmaxf(Mc, red[((size_t)w * kDecRowGroup + rr) * (d + 2) + d]);
+        float Lc = 0.f, Oc = 0.f;
+#pragma unroll
+        for (int w = 0; w < kW; ++w) {
+          const float* sw = red + ((size_t)w * kDecRowGroup + rr) * (d + 2);
+          const float wt = sw[d] == -INFINITY ? 0.f : __expf(sw[d] - Mc);
+          Lc += wt * sw[d + 1];
+          Oc += wt * sw[c];
+        }
+        float* ar = acc + (size_t)(r0 + rr) * (d + 2);
+        const float Mo = ar[d], Lo = ar[d + 1];
+        const float Mn = fmaxf(Mo, Mc);
+        const float ao = Mo == -INFINITY ? 0.f : __expf(Mo - Mn);
+        const float an = Mc == -INFINITY ? 0.f : __expf(Mc - Mn);
+        ar[c] = ar[c] * ao + Oc * an;
+        if (c == 0) {
+          mlx[2 * rr] = Mn;
+          mlx[2 * rr + 1] = Lo * ao + Lc * an;
+        }
       }
-    }
-    __syncthreads();
-    // combine the warps' partials: one thread per (row, column)
-    for (int it = threadIdx.x; it < nr * d; it += kDecThreads) {
-      const int rr = it / d, c = it % d;
-      float M = -INFINITY;
-#pragma unroll
-      for (int w = 0; w < kW; ++w) M = fmaxf(M, red[((size_t)w * kDecRowGroup + rr) * (d + 2) + d]);
-      float L = 0.f, O = 0.f;
-#pragma unroll
-      for (int w = 0; w < kW; ++w) {
-        const float* sl = red + ((size_t)w * kDecRowGroup + rr) * (d + 2);
-        const float wt = sl[d] == -INFINITY ? 0.f : __expf(sl[d] - M);
-        L += wt * sl[d + 1];
-        O += wt * sl[c];
+      __syncthreads();
+      for (int rr = threadIdx.x; rr < nr; rr += kDecThreads) {
+        acc[(size_t)(r0 + rr) * (d + 2) + d] = mlx[2 * rr];
+        acc[(size_t)(r0 + rr) * (d + 2) + d + 1] = mlx[2 * rr + 1];
       }
-      const int r = r0 + rr;
-      const int n = r / g, qh = h * g + r % g;
-      const int64_t prow = ((int64_t)n * a.Hq + qh) * nch + chunk;
-      part_o[prow * d + c] = O;
-      if (c == 0) part_ml[prow] = make_float2(M, L);
+      __syncthreads();  // red, mlx and acc are reused by the next row group / chunk
     }
-    __syncthreads();  // red is reused by the next row group
+  }
+  // this CTA's partial for every row
+  for (int it = threadIdx.x; it < G * d; it += kDecThreads) {
+    const int r = it / d, c = it % d;
+    const int n = r / g, qh = h * g + r % g;
+    const int64_t prow = ((int64_t)n * a.Hq + qh) * nslots + slot;
+    const float* ar = acc + (size_t)r * (d + 2);
+    part_o[prow * d + c] = ar[c];
+    if (c == 0) part_ml[prow] = make_float2(ar[d], ar[d + 1]);
   }
 }
 
@@ -885,17 +916,22 @@ size_t decode_workspace_bytes(int64_t rows, int64_t entries, int d) {
   return (size_t)rows * nch * d * 4 + (size_t)rows * nch * 8 + 256;
 }
 
-cudaError_t launch_decode_biased(const DecodeArgs& a, void* ws, cudaStream_t s) {
+cudaError_t launch_decode_biased(const DecodeArgs& a, void* ws, int num_sms, cudaStream_t s) {
   const int64_t E = a.t + a.S;
   const int chunk = dec_chunk(a.d / 32);
-  const int nch = (int)((E + chunk - 1) / chunk);
+  const int64_t nchunks = (E + chunk - 1) / chunk;
+  // One wave: the CTAs of a KV-head split its chunks (each CTA merges its own in order).
+  const int per_sm = 1;
+  const int nch = (int)std::max<int64_t>(
+      1, std::min<int64_t>(nchunks, (int64_t)num_sms * per_sm / std::max(1, a.H)));
   const int g = a.Hq / a.H;
   const int G = a.nq * g;
   const int64_t rows = (int64_t)a.nq * a.Hq;
   float* part_o = static_cast<float*>(ws);
   float2* part_ml = reinterpret_cast<float2*>(
       static_cast<uint8_t*>(ws) + (((size_t)rows * nch * a.d * 4 + 255) & ~size_t(255)));
-  const size_t smem = ((size_t)G * a.d + (size_t)(kDecThreads / 32) * kDecRowGroup * (a.d + 2)) * 4;
+  const size_t smem = ((size_t)G * a.d + (size_t)(kDecThreads / 32) * kDecRowGroup * (a.d + 2) +
+                       (size_t)G * (a.d + 2) + 2 * kDecRowGroup) * 4;
   auto kern = a.d == 64 ? decode_chunk_kernel<2>
                         : a.d == 128 ? decode_chunk_kernel<4> : decode_chunk_kernel<8>;
   static thread_local size_t smem_set[3] = {48 * 1024, 48 * 1024, 48 * 1024};

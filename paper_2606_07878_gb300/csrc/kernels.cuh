@@ -64,7 +64,7 @@ struct DecodeArgs {
   float scale = 0.f;
 };
 size_t decode_workspace_bytes(int64_t rows, int64_t entries, int d);
-cudaError_t launch_decode_biased(const DecodeArgs& a, void* ws, cudaStream_t s);
+cudaError_t launch_decode_biased(const DecodeArgs& a, void* ws, int num_sms, cudaStream_t s);
 
 // Converts n bf16 values to fp16 in place (exact within the fp16 range; values below it
 // become fp16 subnormals, absolute error <= 2^-25).

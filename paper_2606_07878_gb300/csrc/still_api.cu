@@ -1588,7 +1588,7 @@ still_status still_attend_biased(still_ctx* ctx, const void* q, int32_t nq, int3
   TRY(ensure_ws(ctx, decode_workspace_bytes((int64_t)nq * Hq, t + S, d)));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   ctx->prof.begin(STILL_K_DECODE, s);
-  cudaError_t r = launch_decode_biased(a, ctx->ws, s);
+  cudaError_t r = launch_decode_biased(a, ctx->ws, ctx->nsm, s);
   ctx->prof.end(STILL_K_DECODE, s);
   ctx->prof.launches[STILL_K_DECODE] += 1;  // the merge kernel (begin counted the first)
   if (r != cudaSuccess) return STILL_ERR_CUDA;
