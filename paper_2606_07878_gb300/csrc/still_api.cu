@@ -920,19 +920,21 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     }
     KLAUNCH(STILL_K_NORMS,
             launch_inv_norms(sss, (int64_t)nh * 2 * n * t, sparts, t, c.l2_eps, 1.f, sinv, s));
-    {  // v^T = S_V^T RMSNorm(Z')^T  -> [nD][nh * tp]  (hi, then lo rows when exact)
-      GemmParams p = gp(n * D, nh * t);
+    {  // v^T = S_V^T RMSNorm(Z')^T  -> [nD][nh * tp]  (hi, then lo rows when exact);
+       // one batch per bank, so that each bank's t columns start on a 64-column boundary
+       // and are stored by whole-row vector writes
+      GemmParams p = gp(n * D, t, nh, 1);
+      p.b_r1 = t;
       add_pass(p, 0, 0, 0, h0 * t, D);
       if (vexact) add_pass(p, 0, D, 0, h0 * t, D);
       EpiAffine e;
       e.kind = vexact ? vkind : OUT_BF16;
       e.lo_off = (int64_t)n * D * nh * P.tp;
       e.out = vT;
+      e.om.b1 = P.tp;
       e.om.r0 = (int64_t)nh * P.tp;
-      e.om.cdiv = t;
-      e.om.c1 = P.tp;
       e.om.c0 = 1;
-      e.vec_ok = (t % 32 == 0);
+      e.vec_ok = 1;
       TRY(run_gemm256<STILL_K_SA_V>(ctx, op(Bw.SvT, (int64_t)n * D, D), op(A1, rows, 2 * D), p, e,
                                     vfmt, s));
     }
