@@ -230,7 +230,8 @@ still_status still_compact_layer_beta(still_ctx* ctx, int32_t layer, const void*
  *   scale  logit scale; 0 means 1 / sqrt(d)
  * d in {64, 128, 256}, t + S >= 1, nq * Hq / H <= 64; tensor pointers 16-byte aligned.
  * Keys are processed in chunks of 128 whose partial results are merged in a fixed order; the
- * context's workspace holds the partials (grown on demand). Stream-ordered. */
+ * context's workspace holds the partials (grown on demand), so calls that share a context (this
+ * one and the compaction calls) must be ordered on one stream or otherwise serialised. */
 still_status still_attend_biased(still_ctx* ctx, const void* q, int32_t nq, int32_t Hq,
                                  const void* Ck, const void* Cv, const float* beta, int64_t t,
                                  const void* Kfix, const void* Vfix, int64_t S, int32_t H,
