@@ -730,6 +730,69 @@ __device__ __forceinline__ float2 unpack_pair(uint32_t w) {
   return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w));
 }
 
+// Warp sums of K values (K = 8 or 4) by recursive halving: each lane ends with the sum over all
+// 32 lanes of one value, index dec_idx<K>(lane); 9 (K = 8) or 7 (K = 4) shuffles instead of
+// 5 K.
+template <int K>
+__device__ __forceinline__ int dec_idx(int lane) {
+  return K == 8 ? ((lane >> 4) & 1) * 4 + ((lane >> 3) & 1) * 2 + ((lane >> 2) & 1)
+                : ((lane >> 4) & 1) * 2 + ((lane >> 3) & 1);
+}
+
+template <int K>
+__device__ __forceinline__ int dec_src(int k) {  // a lane holding value k after dec_halve
+  return K == 8 ? ((k >> 2) & 1) * 16 + ((k >> 1) & 1) * 8 + (k & 1) * 4
+                : ((k >> 1) & 1) * 16 + (k & 1) * 8;
+}
+
+template <int K>
+__device__ __forceinline__ float dec_halve(const float (&v)[K], int lane) {
+  constexpr unsigned kFull = 0xffffffffu;
+  float a[K / 2];
+  {
+    const bool up = lane & 16;
+#pragma unroll
+    for (int j = 0; j < K / 2; ++j) {
+      const float send = up ? v[j] : v[j + K / 2];
+      const float keep = up ? v[j + K / 2] : v[j];
+      a[j] = keep + __shfl_xor_sync(kFull, send, 16);
+    }
+  }
+  float c;
+  if constexpr (K == 8) {
+    float b[2];
+    const bool up = lane & 8;
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const float send = up ? a[j] : a[j + 2];
+      const float keep = up ? a[j + 2] : a[j];
+      b[j] = keep + __shfl_xor_sync(kFull, send, 8);
+    }
+    const bool up2 = lane & 4;
+    c = (up2 ? b[1] : b[0]) + __shfl_xor_sync(kFull, up2 ? b[0] : b[1], 4);
+    c += __shfl_xor_sync(kFull, c, 2);
+    c += __shfl_xor_sync(kFull, c, 1);
+  } else {
+    const bool up = lane & 8;
+    c = (up ? a[1] : a[0]) + __shfl_xor_sync(kFull, up ? a[0] : a[1], 8);
+    c += __shfl_xor_sync(kFull, c, 4);
+    c += __shfl_xor_sync(kFull, c, 2);
+    c += __shfl_xor_sync(kFull, c, 1);
+  }
+  return c;
+}
+
+// Max (op 0) or sum (op 1) over the K distinct values held after dec_halve.
+template <int K, int OP>
+__device__ __forceinline__ float dec_across(float x) {
+#pragma unroll
+  for (int o = (K == 8 ? 4 : 8); o <= 16; o <<= 1) {
+    const float y = __shfl_xor_sync(0xffffffffu, x, o);
+    x = OP == 0 ? fmaxf(x, y) : x + y;
+  }
+  return x;
+}
+
 template <int DPL>
 __global__ void __launch_bounds__(kDecThreads, 1)
     decode_chunk_kernel(DecodeArgs a, float* __restrict__ part_o, float2* __restrict__ part_ml) {
@@ -779,6 +842,16 @@ __global__ void __launch_bounds__(kDecThreads, 1)
         for (int i = 0; i < DPL / 2; ++i) kx[k][i] = vx[k][i] = 0u;
       }
     }
+    // the entry whose logit this lane will hold after the warp sums
+    const int my = dec_idx<kDecPerWarp>(lane);
+    float my_bias = 0.f;
+    bool my_valid = false;
+#pragma unroll
+    for (int k = 0; k < kDecPerWarp; ++k)
+      if (k == my) {
+        my_bias = bias[k];
+        my_valid = valid[k];
+      }
     for (int r0 = 0; r0 < G; r0 += kDecRowGroup) {
       const int nr = min(kDecRowGroup, G - r0);
 #pragma unroll 1
@@ -797,24 +870,17 @@ __global__ void __launch_bounds__(kDecThreads, 1)
           }
           lg[k] = sdot;
         }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-#pragma unroll
-          for (int k = 0; k < kDecPerWarp; ++k) lg[k] += __shfl_xor_sync(0xffffffffu, lg[k], o);
-        }
-        float m = -INFINITY;
-#pragma unroll
-        for (int k = 0; k < kDecPerWarp; ++k) {
-          lg[k] = valid[k] ? lg[k] * a.scale + bias[k] : -INFINITY;
-          m = fmaxf(m, lg[k]);
-        }
-        float l = 0.f, ov[DPL];
+        const float lsum = dec_halve<kDecPerWarp>(lg, lane);  // logit of entry `my`
+        const float lgt = my_valid ? lsum * a.scale + my_bias : -INFINITY;
+        const float m = dec_across<kDecPerWarp, 0>(lgt);
+        const float pm = my_valid ? __expf(lgt - m) : 0.f;
+        const float l = dec_across<kDecPerWarp, 1>(pm);
+        float ov[DPL];
 #pragma unroll
         for (int i = 0; i < DPL; ++i) ov[i] = 0.f;
 #pragma unroll
         for (int k = 0; k < kDecPerWarp; ++k) {
-          const float p = valid[k] ? __expf(lg[k] - m) : 0.f;
-          l += p;
+          const float p = __shfl_sync(0xffffffffu, pm, dec_src<kDecPerWarp>(k));
 #pragma unroll
           for (int i = 0; i < DPL / 2; ++i) {
             const float2 vf = unpack_pair(vx[k][i]);
