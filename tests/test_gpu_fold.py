@@ -83,3 +83,31 @@ def test_fold_agrees_with_explicit_projection(logit_scale):
     finally:
         ra.close()
         rb.close()
+
+
+def test_fold_keeps_parity_when_groups_split_kv_heads():
+    """Smaller workspace limits split the cross-attention groups down to single (KV-head,
+    cross head) units; the folded path addresses u rows and shared x~ rows per group."""
+    wl = _small(d=128, D=1024, n=4, H=2, N=600, F=0)
+    t = 60
+    r = _run(wl, t, dict(compactor_rope=0))
+    try:
+        K, V = synth.gen_kv(wl, 0, device=DEV)
+        rk, rv, _, _ = oracle_layer(wl, r.W[0], K, V, t, cfg_over=dict(compactor_rope=False))
+        total = still.still_workspace_size(r.ctx, wl["N"], t)
+        ran = []
+        for frac in (1.0, 0.6, 0.4, 0.3, 0.2):
+            still.still_set_workspace_limit(r.ctx, int(total * frac))
+            Ck, Cv = r.out(t)
+            try:
+                still.still_compact_layer(r.ctx, 0, K, V, t, Ck, Cv)
+            except still.StillError as e:
+                assert e.name == "STILL_ERR_OOM", e.name
+                continue
+            r.check_status()
+            assert_parity(rk, synth.bf16_to_f64(Ck), f"C_k limit {frac}")
+            assert_parity(rv, synth.bf16_to_f64(Cv), f"C_v limit {frac}")
+            ran.append(frac)
+        assert len(ran) >= 3 and min(ran) <= 0.4, ran
+    finally:
+        r.close()
