@@ -56,9 +56,9 @@ def describe(name, wl, t):
 TRAFFIC = {
     "scores": {"files": ["tc_gemm.cuh", "epilogues.cuh"], "kernel_hash": None,
                "bytes_per_launch": None, "workload": None, "profile": None},
-    # 1.285 GB read + 0.132 GB written per launch (profiles/ca_fused_qwen7b_8k_t1024.md)
-    "ca_fused": {"files": ["ca_flash.cuh", "ptx.cuh"], "kernel_hash": "de7c73bd49c1000d",
-                 "bytes_per_launch": 1.4171e9, "workload": ("qwen7b_8k", 1024),
+    # 1.287 GB read + 0.132 GB written per launch (profiles/ca_fused_qwen7b_8k_t1024.md)
+    "ca_fused": {"files": ["ca_flash.cuh", "ptx.cuh"], "kernel_hash": "1024714c3c99a223",
+                 "bytes_per_launch": 1.4191e9, "workload": ("qwen7b_8k", 1024),
                  "profile": "profiles/ca_fused_qwen7b_8k_t1024.md"},
 }
 
