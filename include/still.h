@@ -8,9 +8,11 @@
  * on one GPU: keys are un-rotated by the base model's RoPE (RoPE-fix, Sec. 2.2), t latent
  * queries per KV-head cross-attend X = [K; V] with QK-norm, the compactor's own RoPE and logits
  * scaled by d_l (App. A, "Cross-attention"), are refined by latent self-attention and a GELU
- * FFN, and are projected by W_key / W_val; C_k is re-rotated at evenly spaced output positions
- * over the compacted range (App. B, single-pass recipe, step 5). beta is not produced (the
- * reported configuration sets beta = 0, Sec. 2.1).
+ * FFN (one or two such blocks), and are projected by W_key / W_val; C_k is re-rotated at evenly
+ * spaced output positions over the compacted range (App. B, single-pass recipe, step 5). The
+ * reported configuration sets beta = 0 (Sec. 2.1); the optional per-slot bias and its
+ * decode-time consumer are separate calls (still_set_beta_head, still_compact_layer_beta,
+ * still_attend_biased).
  *
  * Conventions
  *  - Pointers are DEVICE pointers unless their name starts with h_ (host). All calls are
@@ -126,9 +128,10 @@ still_status still_load_layer_weights(still_ctx* ctx, int32_t layer,
                                       const still_layer_weights* w, void* stream);
 
 /* still_load_layer_weights for a compactor of cfg->n_blocks (1 or 2) blocks (App. A; the
- * paper's canonical compactor has two, both with cross-attention; n_blocks > 2 gives
- * STILL_ERR_UNSUPPORTED: every further cross-attention compounds the rounding of its fp16
- * probabilities, and three blocks measured just past the parity bar). Z [H, t_max, D] latent banks;
+ * paper's canonical compactor has two, both with cross-attention). A block whose output feeds
+ * another runs in split precision (fp16 hi / lo operand chains), since the next block's
+ * cross-attention magnifies its rounding; n_blocks > 2 gives STILL_ERR_UNSUPPORTED (three
+ * blocks measured past the parity bar). Z [H, t_max, D] latent banks;
  * blocks[b] the weights of block b; Wkey, Wval [D, d] output heads. Block 0's latent queries
  * depend only on Z and are precomputed here (as in still_load_layer_weights). A later
  * cross-attending block's queries L2norm(RMSNorm(Z_b) W_Q + b_Q) depend on the latent state
