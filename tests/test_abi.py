@@ -82,3 +82,25 @@ def test_lookahead_schedule_matches_oracle(lib):
         with pytest.raises(still.StillError) as e:
             still.still_lookahead_pass_info(*args)
         assert e.value.name == "STILL_ERR_INVALID_ARG", args
+
+
+def test_new_entry_points_validate_on_the_host(lib):
+    """Argument checks of the later entry points run before any device work (no GPU needed)."""
+    import ctypes
+    INVALID = 1
+    assert lib.still_set_key_fold(None, 1) == INVALID
+    assert lib.still_set_beta_head(None, 0, None, None, None) == INVALID
+    assert lib.still_attend_biased(None, None, 1, 8, None, None, None, 0, None, None, 1, 8, 128,
+                                   0.0, None, None) == INVALID
+    mask = (ctypes.c_uint8 * 2)(1, 0)
+    assert lib.still_compact_stack_masked(None, 2, mask, None, None, None, None, 0, 1, 1, None,
+                                          None, None, None, None, None) == INVALID
+    passes = (ctypes.c_int64 * 1)(0)
+    assert lib.still_lookahead_compact_layer(None, 0, 1, None, None, passes, 8, 16, None, None,
+                                             None) == INVALID
+    assert lib.still_lookahead_compact_stack(None, 1, None, 1, None, None, passes, 8, 16, None,
+                                             None, None) == INVALID
+    # a negative pass index or a zero ratio is refused before the context is looked at
+    bad = (ctypes.c_int64 * 1)(-1)
+    assert lib.still_lookahead_compact_layer(None, 0, 1, None, None, bad, 8, 16, None, None,
+                                             None) == INVALID
