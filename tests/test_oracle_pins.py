@@ -224,6 +224,34 @@ def test_identity_init_passes_keys_and_values_through():
     np.testing.assert_allclose(Cv, V, atol=1e-9)
 
 
+def test_identity_init_two_blocks_passes_through():
+    """App. C for a compactor of two blocks: the later block's cross-attention output projection
+    and the refinement outputs are zero, so the pass-through survives the second block whatever
+    its other weights (random here). Same shape as the one-block construction above, whose
+    block-diagonal attention makes the pass-through exact to rounding."""
+    H, d, N = 2, 128, 96
+    D = 2 * d
+    W = identity_init_weights(H, d, N)
+    rng = np.random.default_rng(12)
+    for name, shape in (("Wq", (D, D)), ("bq", (D,)), ("Wk", (2 * d, D)), ("bk", (D,)),
+                        ("Wv", (2 * d, D)), ("Sq", (D, D)), ("sbq", (D,)), ("Sk", (D, D)),
+                        ("sbk", (D,)), ("Sv", (D, D)), ("W1", (D, 4 * D))):
+        W[name + "@1"] = rng.standard_normal(shape) * 0.05
+    for name, shape in (("Wo", (D, D)), ("So", (D, D)), ("W2", (4 * D, D))):
+        W[name + "@1"] = np.zeros(shape)
+    cfg = O.Cfg(H=H, d=d, D=D, n_c=1, n_s=1, F=4 * D, theta=1e4, n_blocks=2)
+    wl = dict(N=N, H=H, d=d, theta=1e4, heavy=4)
+    K, V = synth.gen_kv(wl, 0, N=N)
+    K, V = synth.bf16_to_f64(K), synth.bf16_to_f64(V)
+    Ck, Cv, _, _ = O.compact_layer(K, V, W, cfg, N)
+    np.testing.assert_allclose(Ck, K, atol=1e-9)
+    np.testing.assert_allclose(Cv, V, atol=1e-9)
+    # a non-zero later output projection breaks it (the pin sees the second block)
+    W["Wo@1"] = np.eye(D) * 0.1
+    Ck2, _, _, _ = O.compact_layer(K, V, W, cfg, N)
+    assert np.abs(Ck2 - K).max() > 1e-3
+
+
 # ------------------------------------------------------------------ printed numbers
 
 def test_budgets_match_paper_table():
