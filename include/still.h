@@ -50,8 +50,9 @@ typedef struct still_ctx still_ctx; /* opaque: weight copies, precompute, worksp
 
 /* One layer's compactor hyperparameters (App. A, "Canonical configuration summary").
  * Implemented: n_blocks 1 or 2, cross_every_block 0 or 1, n_cross_heads = n_self_heads,
- * d_latent % 256 == 0, head_dim in {64, 128, 256}, ffn_dim % 64 == 0 (or 0 = no FFN),
- * compactor_rope 0 or 1, rope_fix = 1. Other values return STILL_ERR_UNSUPPORTED. */
+ * d_latent % 256 == 0, head_dim in {64, 128, 256} (two blocks: 64 or 128), ffn_dim % 64 == 0
+ * (or 0 = no FFN), compactor_rope 0 or 1, rope_fix = 1. Other values return
+ * STILL_ERR_UNSUPPORTED. */
 typedef struct {
   int32_t n_kv_heads;        /* H: KV-heads of the base model */
   int32_t head_dim;          /* d: base model head dim */

@@ -213,6 +213,10 @@ still_status check_cfg(const still_layer_config* c) {
       c->rope_fix != 1 ||
       (c->final_norm != 0 && c->final_norm != 1))
     return STILL_ERR_UNSUPPORTED;
+  // Two-block layers run every block through the fused cross-attention kernel, which needs
+  // 2d <= 256; the first block of a 2d = 512 layer would take the unfused split-fp16 path,
+  // which the parity tests do not cover.
+  if (c->n_blocks > 1 && c->head_dim == 256) return STILL_ERR_UNSUPPORTED;
   return STILL_OK;
 }
 
