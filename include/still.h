@@ -185,8 +185,10 @@ still_status still_compact_layer(still_ctx* ctx, int32_t layer, const void* K, c
  * Every call, from every context on the device, shares the one array and leaves its last
  * contents there; the path clears what it needs zeroed on each call. Calls whose execution
  * overlaps on the GPU (different streams, or concurrent host threads) race on the array:
- * serialise them. Kernel event timing (still_profile_enable) is suspended inside this call;
- * launch counts are still recorded. */
+ * serialise them. Kernel event timing (still_profile_enable) is skipped for the kernels of
+ * this call, on the calling host thread only and without changing the context's profiling
+ * setting; launch counts are still recorded. A context is not thread-safe: host threads that
+ * share one must serialise their calls. */
 still_status still_compact_layer_noalloc(still_ctx* ctx, int32_t layer, const void* K,
                                          const void* V, const int64_t strides_kv[3],
                                          const still_pos_segment* h_segments,

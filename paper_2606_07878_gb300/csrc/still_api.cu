@@ -109,9 +109,16 @@ struct Profiler {
     else
       cudaEventRecord(e, s);
   }
+  // Set on the calling host thread while it runs an allocation-free call: event timing creates
+  // CUDA events, so it is skipped there (launch counting stays on). Per thread, so that no
+  // shared state of the context is written.
+  static bool& untimed_thread() {
+    static thread_local bool v = false;
+    return v;
+  }
   void begin(int cls, cudaStream_t s) {
     ++launches[cls];
-    if (!on || !((mask >> cls) & 1)) return;
+    if (!on || untimed_thread() || !((mask >> cls) & 1)) return;
     pending = get();
     record(pending, s);
   }
@@ -1484,12 +1491,14 @@ still_status still_load_layer_weights_blocks(still_ctx* ctx, int32_t layer,
 
 namespace {
 
+// noalloc: run in the library's fixed device scratch (still_compact_layer_noalloc) instead of
+// the context's growable workspace, with event timing suspended on this thread.
 still_status compact_layer_impl(still_ctx* ctx, int32_t layer, const void* K, const void* V,
                                 const int64_t strides_kv[3],
                                 const still_pos_segment* h_segments, int32_t n_segments,
                                 int64_t N, int32_t t, void* Ck, void* Cv, float* beta,
                                 double* h_out_pos_start, double* h_out_pos_step,
-                                int64_t* h_pos_offset, void* stream) {
+                                int64_t* h_pos_offset, void* stream, bool noalloc = false) {
   const LayerW* L = nullptr;
   TRY(check_ctx_layer(ctx, layer, &L));
   if (beta != nullptr && (L->wbeta == nullptr || (reinterpret_cast<uintptr_t>(beta) & 3)))
@@ -1508,8 +1517,20 @@ still_status compact_layer_impl(still_ctx* ctx, int32_t layer, const void* K, co
   const int H = L->cfg.n_kv_heads, d = L->cfg.head_dim;
   OutSpec o{static_cast<bf16*>(Ck), static_cast<bf16*>(Cv), (int64_t)H * d, d};
   o.beta = beta;
-  TRY(compact_one(ctx, *L, single_source(K, V, strides_kv, N), pos, N, t, o,
-                  static_cast<cudaStream_t>(stream)));
+  if (noalloc) {
+    uint8_t* scratch = nullptr;
+    TRY(noalloc_scratch(ctx->device, &scratch));
+    bool& untimed = Profiler::untimed_thread();
+    untimed = true;
+    const still_status st =
+        compact_one(ctx, *L, single_source(K, V, strides_kv, N), pos, N, t, o,
+                    static_cast<cudaStream_t>(stream), scratch, kNoAllocScratchBytes);
+    untimed = false;
+    TRY(st);  // STILL_ERR_OOM: even the smallest grouping needs more than the fixed scratch
+  } else {
+    TRY(compact_one(ctx, *L, single_source(K, V, strides_kv, N), pos, N, t, o,
+                    static_cast<cudaStream_t>(stream)));
+  }
   if (h_out_pos_start) *h_out_pos_start = pos.pmin;
   if (h_out_pos_step) *h_out_pos_step = t > 1 ? (pos.pmax - pos.pmin) / (double)(t - 1) : 0.0;
   if (h_pos_offset) *h_pos_offset = N - t;
@@ -1608,39 +1629,9 @@ still_status still_compact_layer_noalloc(still_ctx* ctx, int32_t layer, const vo
                                          void* Cv, double* h_out_pos_start,
                                          double* h_out_pos_step, int64_t* h_pos_offset,
                                          void* stream) {
-  const LayerW* L = nullptr;
-  TRY(check_ctx_layer(ctx, layer, &L));
-  if (K == nullptr || V == nullptr || Ck == nullptr || Cv == nullptr || strides_kv == nullptr)
-    return STILL_ERR_INVALID_ARG;
-  if (N < 1 || t < 1 || t > N || t > L->cfg.t_max || N > (int64_t(1) << 30))
-    return STILL_ERR_SHAPE;
-  if (strides_kv[2] != 1 || strides_kv[0] < 1 || strides_kv[1] < 0) return STILL_ERR_SHAPE;
-  if (((reinterpret_cast<uintptr_t>(K) | reinterpret_cast<uintptr_t>(V)) & 1) ||
-      ((reinterpret_cast<uintptr_t>(Ck) | reinterpret_cast<uintptr_t>(Cv)) & 15))
-    return STILL_ERR_ALIGNMENT;
-  Positions pos;
-  TRY(make_positions(h_segments, n_segments, N, pos));
-  CK(cudaSetDevice(ctx->device));
-  Plan P;
-  if (!make_plan(L->cfg, queries_per_call(*L), fold_kp(*L), N, t, pos.pmin, pos.pmax,
-                 kNoAllocScratchBytes, P))
-    return STILL_ERR_OOM;  // even the smallest grouping needs more than the fixed scratch
-  uint8_t* scratch = nullptr;
-  TRY(noalloc_scratch(ctx->device, &scratch));
-  const int H = L->cfg.n_kv_heads, d = L->cfg.head_dim;
-  OutSpec o{static_cast<bf16*>(Ck), static_cast<bf16*>(Cv), (int64_t)H * d, d};
-  // Launch counting stays on; event timing (which creates CUDA events) is suspended.
-  const bool timing = ctx->prof.on;
-  ctx->prof.on = false;
-  const still_status st =
-      compact_one(ctx, *L, single_source(K, V, strides_kv, N), pos, N, t, o,
-                  static_cast<cudaStream_t>(stream), scratch, kNoAllocScratchBytes);
-  ctx->prof.on = timing;
-  TRY(st);
-  if (h_out_pos_start) *h_out_pos_start = pos.pmin;
-  if (h_out_pos_step) *h_out_pos_step = t > 1 ? (pos.pmax - pos.pmin) / (double)(t - 1) : 0.0;
-  if (h_pos_offset) *h_pos_offset = N - t;
-  return STILL_OK;
+  return compact_layer_impl(ctx, layer, K, V, strides_kv, h_segments, n_segments, N, t, Ck, Cv,
+                            nullptr, h_out_pos_start, h_out_pos_step, h_pos_offset, stream,
+                            true);
 }
 
 still_status still_compact_stack(still_ctx* ctx, int32_t n_layers, const void* const* K,

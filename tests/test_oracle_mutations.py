@@ -31,6 +31,12 @@ MUTANTS = [
     ("self-attention scores transposed",
      "heads.append(softmax_rows(cfg.scale * (q @ k.T)) @ v)",
      "heads.append(softmax_rows(cfg.scale * (k @ q.T)) @ v)"),
+    ("self-attention values projected by the key weights",
+     "v = Zn @ Sv[:, cols]",
+     "v = Zn @ Sk[:, cols]"),
+    ("self-attention output projection by the value weights",
+     "return np.concatenate(heads, axis=-1) @ So",
+     "return np.concatenate(heads, axis=-1) @ Sv.T"),
     ("self-attention query bias dropped",
      "q = l2norm(Zn @ Sq[:, cols] + sbq[cols], cfg.l2_eps)",
      "q = l2norm(Zn @ Sq[:, cols], cfg.l2_eps)"),

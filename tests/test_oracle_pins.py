@@ -161,6 +161,24 @@ def test_zero_scores_give_mean_of_projected_values():
     np.testing.assert_allclose(out, ref, atol=1e-12)
 
 
+def test_self_attention_zero_scores_give_mean_of_values():
+    """S_Q = S_K = 0 and zero query/key biases -> q = k = 0 (the L2 norm keeps a zero vector
+    zero), every self-attention logit 0 -> each latent receives Concat_i(mean_j v_ij) S_O with
+    v_i = Zn S_V,i (App. A, Latent self-attention), compared with np.mean."""
+    wl, cfg, W, X, Zn = _ca_setup()
+    W = dict(W)
+    for k in ("Sq", "sbq", "Sk", "sbk"):
+        W[k] = np.zeros_like(W[k])
+    out = O.self_attention(Zn, W, 0, cfg)
+    D = cfg.D
+    heads = np.concatenate([np.mean(Zn @ W["Sv"][:, i * D:(i + 1) * D], axis=0)
+                            for i in range(cfg.n_s)])
+    ref = np.tile(heads @ W["So"], (Zn.shape[0], 1))
+    np.testing.assert_allclose(out, ref, atol=1e-12)
+    # the rows of Zn differ, so a per-row (not averaged) value would not match
+    assert np.abs(Zn @ W["Sv"][:, :D] - np.mean(Zn @ W["Sv"][:, :D], axis=0)).max() > 1e-3
+
+
 def test_permutation_invariance():
     """Jointly permuting (K row, V row, position) leaves C_k, C_v unchanged."""
     wl = _tiny(N=30)
