@@ -55,7 +55,8 @@ def describe(name, wl, t):
 
 # DRAM traffic (read + write) per launch of the dominant kernel at a workload, from an ncu
 # capture; valid only for the kernel sources it was taken on (hash of the listed sources).
-# The scores GEMM (two-kernel path, 2d = 512) and the fused cross-attention kernel (2d <= 256).
+# The fused cross-attention kernel (the scores GEMM entry is kept for the record: no workload
+# takes it any more).
 TRAFFIC = {
     "scores": {"files": ["tc_gemm.cuh", "epilogues.cuh"], "kernel_hash": None,
                "bytes_per_launch": None, "workload": None, "profile": None},
@@ -183,9 +184,9 @@ def algorithmic_flops(wl, t, N):
     ca = (kproj + 2 * t * N * H * n * kw + 2 * t * N * H * n * 2 * d
           + 2 * t * H * n * 2 * d * D + 2 * t * H * n * D * D)
     sa = 6 * t * H * D * n * D + 4 * t * t * H * n * D + 2 * t * H * n * D * D
-    # Every block's cross-attention is one fused kernel when 2d <= 256 (a block that feeds
-    # another in its split-precision form, P X in 2.5 passes); 2d = 512 takes the scores GEMM.
-    fused = 2 * d <= 256
+    # Every block's cross-attention is one fused kernel (a block that feeds another in its
+    # split-precision form, P X in 2.5 passes; 2d = 512 on clusters of two CTAs).
+    fused = True
     return {"total": n_ca * ca + nb * (sa + 4 * t * H * D * F) + 4 * t * H * D * d,
             "scores": n_ca * 2 * t * N * H * n * kw, "px": n_ca * 2 * t * N * H * n * 2 * d,
             "scores_gemm": 0 if fused else n_ca * 2 * t * N * H * n * D,
@@ -583,10 +584,9 @@ def main():
         raise RuntimeError(f"device status {still.STATUS.get(code)} {det}")
 
     # One stack step is captured into a CUDA graph and replayed (the layer-stack launch sequence
-    # as one graph). The dominant kernel class (fused cross-attention for 2d <= 256, else the
-    # scores GEMM) is the only one with events: its launches are bracketed by event nodes of the
-    # graph, read after the last replay.
-    kname = "ca_fused" if 2 * d <= 256 else "scores"
+    # as one graph). The dominant kernel class, the fused cross-attention, is the only one with
+    # events: its launches are bracketed by event nodes of the graph, read after the last replay.
+    kname = "ca_fused"
     still.still_reserve_workspace(ctx, N, t)
     still.still_profile_enable_classes(ctx, [kname])
     graph = torch.cuda.CUDAGraph()
@@ -674,8 +674,8 @@ def main():
     e2e_value = throughput(world, N, e2e_steps, ems)
 
     # ---------------------------------------------------------------- roofline
-    # Dominant kernel: the fused cross-attention (scores + softmax + P X) when the path uses
-    # it (2d <= 256), else the scores GEMM. Algorithmic flops count each product once; the
+    # Dominant kernel: the fused cross-attention (scores + softmax + P X). Algorithmic flops
+    # count each product once; the
     # issued view counts the split-precision passes (3 for q.k, 1.5 for P X: hi + key-half lo).
     hbm, bf16_burst, bf16_sus, src = _peaks()
     fl = algorithmic_flops(wl, t, N)
@@ -691,6 +691,7 @@ def main():
     if tr["kernel_hash"] == _kernel_hash(tr["files"]) and tr["workload"] == (name, t):
         traffic = tr["bytes_per_launch"]
     kdesc = ("ca_fused (3-pass split-bf16 scores + online softmax + P X, one tcgen05 kernel"
+             + ("; clusters of two CTAs that split the 512 O columns" if 2 * d == 512 else "")
              + ("; the first block's launches in split fp16 with P hi + lo)"
                 if wl.get("n_blocks", 1) > 1 and wl.get("cross_every_block", 1) else ")")
              if fused else "scores (3-pass split-bf16 tcgen05 GEMM)")
@@ -717,7 +718,7 @@ def main():
         "gpu_launches": launches,
         "roofline": roof,
         "whole_path_alg_tflops": whole,
-        "kernel_ms_per_step": {k: v[1] / args.steps for k, v in prof.items()
+        "kernel_ms_per_step": {k: v[1] / brk for k, v in prof.items()
                                if k != "load" and v[0] > 0},
         "clocks": clk,
     }

@@ -565,4 +565,12 @@ inline cudaError_t launch_ca_flash(const Operand2D& Q, const Operand2D& K, const
   return cudaGetLastError();
 }
 
+// 2d = 512 (head dim 256): the same computation on a cluster of two CTAs that split the O
+// columns and take turns computing S (ca_pair.cu). Q, K as for launch_ca_flash; XT: [H*512][2*Np]
+// fp16 (hi | lo). num_sms: SMs of the device (two per cluster).
+cudaError_t launch_ca_pair(const Operand2D& Q, const Operand2D& K, const Operand2D& XT,
+                           const FlashParams& f, int num_sms, cudaStream_t stream);
+// Clusters of that kernel that can be resident at once (its persistent grid size).
+int ca_pair_clusters(int num_sms);
+
 }  // namespace still

@@ -1,0 +1,625 @@
+// Cross-attention of one compactor layer for 2d = 512 (head dim 256), flash-style, for sm_103a
+// (App. A, "Cross-attention"):
+//
+//   S(m, k)  = scale * q_m . k_k / |k~_k|          3-pass split-bf16 tcgen05.mma, fp32 in TMEM
+//   P(m, k)  = 2^(S(m, k) log2e - M(m))             online row softmax over 256-key tiles
+//   O(m, :)  = sum_k P(m, k) X(k, :)                unnormalised, with the row sum l per split
+//
+// The accumulator of a 128-row query tile over 2d = 512 columns fills a whole TMEM (512
+// fp32 columns), leaving no room for S. A cluster of two CTAs therefore shares each work unit
+// (batch b = (KV-head, cross head), 128-row query tile, key split): CTA r keeps the O columns
+// of features [128 r, 128 r + 128) of K~ and of V (256 columns, TMEM [256, 512)) and computes
+// S for every other 256-key tile (TMEM [0, 256)). The CTA that owns a tile forms its fp16
+// probabilities, sends the tile's running row maximum to its peer as soon as it is decided,
+// and copies the probability tile into the peer's shared memory with a bulk DSMEM copy; both
+// CTAs then accumulate P X for their column half. S and P never reach global memory.
+//
+// Both CTAs apply the same running-maximum sequence (the owner's decision travels with the
+// tile), so their O halves, and the row sums each accumulates from its own tiles, stay on one
+// reference. The running max moves only when a tile raises it by more than kRescaleLog2
+// (log2 units), so P <= 2^8 fits fp16.
+//
+// Tensor-pipe issue order per CTA: before each of its own S tiles j, every P X tile up to
+// j - 2 (own or peer), so that a P buffer is never held behind a long S computation; the
+// softmax of tile j overlaps the peer's S computation of tile j + 1.
+//
+// Synchronisation between the two CTAs (all waits bounded):
+//   mmsg   the owner's per-row running max of a tile (st.shared::cluster + remote arrive)
+//   pfull  P of the tile in this CTA's buffer and O rescaled: 8 local arrivals; for a peer
+//          tile one of them expects the 64 KB that the peer's bulk copies complete
+//   rfree  the peer's P X of the previous tile is done (its P buffer may be overwritten)
+//   lmsg   the peer's row sum at the end of a unit
+//
+// Output per split: unnormalised O rows (natural feature order) and (m, l), m in log2 units;
+// ca_merge_kernel combines the splits in a fixed order.
+//
+// CTA = 10 warps: 0 TMA producer, 1 MMA issuer (TMEM owner), 2..9 softmax / output.
+#include <algorithm>
+
+#include "ca_flash.cuh"
+
+namespace still {
+
+namespace {
+
+constexpr int kPairKeys = 256;   // keys per S tile
+constexpr int kPairOCols = 256;  // O columns per CTA
+constexpr uint32_t kPairPBytes = kBM * kPairKeys * 2;  // one fp16 P tile, 64 KB
+
+struct PairSmem {
+  static constexpr int kQBytes = kBM * kBK * 2;                // q chunk, 16 KB
+  static constexpr int kKBytes = kPairKeys * kBK * 2;          // k chunk, 32 KB
+  static constexpr int kXBox = 128 * kBK * 2;                  // one 128-row X^T box, 16 KB
+  static constexpr int kStageBytes = kQBytes + kKBytes;        // = 3 X^T boxes
+  static constexpr int kStages = 3;
+  static constexpr int kPChunkBytes = kBM * kBK * 2;           // 128 rows x 64 keys fp16
+  static constexpr int kPOffset = kStages * kStageBytes;
+  static constexpr int kKinvOffset = kPOffset + (int)kPairPBytes;            // [8][128] f32
+  static constexpr int kXchOffset = kKinvOffset + kFlashSoftWarps * 128 * 4;  // [2][2][128]
+  static constexpr int kMsgOffset = kXchOffset + 2 * 2 * 128 * 4;             // [2][128] m
+  static constexpr int kLslotOffset = kMsgOffset + 2 * 128 * 4;              // [128] l
+  static constexpr int kBarOffset = kLslotOffset + 128 * 4;
+  static constexpr int kBytes = kBarOffset + 256 + 1024;
+  static_assert(3 * kXBox == kStageBytes, "an X^T chunk fills a stage");
+  static_assert(kBytes <= 232448, "shared memory budget");
+};
+
+// Owner of tile jj of a unit: CTA (jj & 1). Before its own tile jj a CTA issues every P X
+// tile up to jj - 2; the remaining ones after its last own tile.
+__device__ __forceinline__ bool pair_owner(int jj, uint32_t rank) {
+  return (uint32_t)(jj & 1) == rank;
+}
+
+__global__ void __launch_bounds__(kFlashThreads, 1)
+    ca_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                   const __grid_constant__ CUtensorMap tmX, const FlashParams f) {
+  using S = PairSmem;
+  constexpr int kStages = S::kStages;
+  constexpr int kCols = kPairKeys / 2;   // S columns per softmax warp (its half of the tile)
+  constexpr int kOCols = kPairOCols / 2;  // O columns per softmax warp
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::kBarOffset);
+  uint64_t* empty = full + kStages;
+  uint64_t* sfull = empty + kStages;  // own S tile complete in TMEM
+  uint64_t* sfree = sfull + 1;        // own S tile drained
+  uint64_t* pfull = sfree + 1;        // P of the tile in the local buffer, O rescaled
+  uint64_t* pempty = pfull + 1;       // local P X complete
+  uint64_t* ofree = pempty + 1;       // O drained at the end of a unit
+  uint64_t* xb = ofree + 1;           // [4] row-value exchange per lane quarter
+  uint64_t* mmsg = xb + 4;            // peer's running max of a tile (4 remote arrivals)
+  uint64_t* rfree = mmsg + 1;         // peer's P X of the previous tile done (8 remote)
+  uint64_t* lmsg = rfree + 1;         // peer's row sums at the end of a unit (4 remote)
+  uint64_t* drain = lmsg + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int qchunks = f.D / kBK;
+  const uint32_t rank = cluster_ctarank();
+  const uint32_t peer = rank ^ 1u;
+  const int cid = (int)cluster_id_x(), ncl = (int)cluster_count_x();
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(sfull, 1);
+    mbar_init(sfree, kFlashSoftWarps);
+    mbar_init(pfull, kFlashSoftWarps);
+    mbar_init(pempty, 1);
+    mbar_init(ofree, kFlashSoftWarps);
+    for (int q = 0; q < 4; ++q) mbar_init(&xb[q], 2);
+    mbar_init(mmsg, 4);
+    mbar_init(rfree, kFlashSoftWarps);
+    mbar_init(lmsg, 4);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&tmQ);
+    tma_prefetch_desc(&tmK);
+    tma_prefetch_desc(&tmX);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  // Both CTAs' barriers are initialised before either arrives on the other's.
+  cluster_sync();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ TMA producer
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t armed = 0, armed_par = 0;
+      bool bad = false;
+      auto acquire = [&](uint32_t bytes) -> uint8_t* {
+        if (!mbar_wait(&empty[stage], phase ^ 1)) {
+          dev_set_error(f.err, DEV_WAIT_TIMEOUT, 400);
+          *abort_flag = 1;
+          bad = true;
+          return nullptr;
+        }
+        mbar_arrive_expect_tx(&full[stage], bytes);
+        armed |= 1u << stage;
+        armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
+        return smem + stage * S::kStageBytes;
+      };
+      auto advance = [&]() {
+        if (++stage == kStages) {
+          stage = 0;
+          phase ^= 1;
+        }
+      };
+      for (int u = cid; u < f.nunits && !bad && !*abort_flag; u += ncl) {
+        const FlashUnit w = flash_unit(f, u);
+        const int32_t qrow =
+            (int32_t)(f.q_row0 + (int64_t)w.b * (f.q_pitch > 0 ? f.q_pitch : f.t)) + w.tm * kBM;
+        const int32_t krow =
+            (int32_t)(f.k_row0 + (int64_t)(f.kdiv > 0 ? w.b / f.kdiv : w.b) * f.N);
+        // this CTA's feature rows of X^T: K~ [128 rank, +128) and V [128 rank, +128)
+        const int32_t xk = f.xbase_row + (w.b / f.bdiv) * 512 + 128 * (int32_t)rank;
+        const int32_t xv = xk + 256;
+        const int J = w.j1 - w.j0;
+        auto produce_px = [&](int i) {
+          const int j = w.j0 + i;
+          const int nch = flash_chunks<kPairKeys>(f, j);
+          for (int c = 0; c < nch && !bad; ++c) {
+            uint8_t* sa = acquire(3 * S::kXBox);
+            if (sa == nullptr) break;
+            const int32_t x = j * kPairKeys + c * kBK;
+            tma_load_2d(sa, &tmX, &full[stage], x, xk);
+            tma_load_2d(sa + S::kXBox, &tmX, &full[stage], x, xv);
+            tma_load_2d(sa + 2 * S::kXBox, &tmX, &full[stage], (int32_t)(f.Np + x), xk);
+            advance();
+          }
+        };
+        int px_next = 0;
+        for (int jj = 0; jj < J && !bad; ++jj) {
+          if (!pair_owner(jj, rank)) continue;
+          while (px_next <= jj - 2 && !bad) produce_px(px_next++);
+          const int32_t kr = krow + (w.j0 + jj) * kPairKeys;
+          for (int pass = 0; pass < 3 && !bad; ++pass) {
+            const int32_t qoff = pass == 2 ? f.D : 0;  // (q_hi,k_hi), (q_hi,k_lo), (q_lo,k_hi)
+            const int32_t koff = pass == 1 ? f.D : 0;
+            for (int c = 0; c < qchunks; ++c) {
+              uint8_t* sa = acquire(S::kQBytes + S::kKBytes);
+              if (sa == nullptr) break;
+              tma_load_2d(sa, &tmQ, &full[stage], qoff + c * kBK, qrow);
+              tma_load_2d(sa + S::kQBytes, &tmK, &full[stage], koff + c * kBK, kr);
+              advance();
+            }
+          }
+        }
+        while (px_next < J && !bad) produce_px(px_next++);
+      }
+      if (bad || *abort_flag) {
+        for (int s = 0; s < kStages; ++s)
+          if (armed & (1u << s)) (void)mbar_wait(&full[s], (armed_par >> s) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ MMA issuer
+      const uint32_t idesc_s = idesc_f16(kBM, kPairKeys, 1);   // bf16 q, k
+      const uint32_t idesc_hi = idesc_f16(kBM, kPairOCols, 0);  // fp16 P, X^T hi (K~ | V)
+      const uint32_t idesc_lo = idesc_f16(kBM, 128, 0);         // fp16 P, X^T lo (K~ half)
+      const uint32_t s_tmem = tmem_base;
+      const uint32_t o_tmem = tmem_base + 256;
+      const uint32_t p_smem = smem_u32(smem + S::kPOffset);
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t n_s = 0, n_px = 0, n_units = 0;
+      bool issued = false, bad = false;
+      auto fail = [&](int where) {
+        dev_set_error(f.err, DEV_WAIT_TIMEOUT, where);
+        *abort_flag = 1;
+        bad = true;
+      };
+      for (int u = cid; u < f.nunits && !bad && !*abort_flag; u += ncl) {
+        const FlashUnit w = flash_unit(f, u);
+        const int J = w.j1 - w.j0;
+        auto issue_px = [&](int i) {
+          const int nch = flash_chunks<kPairKeys>(f, w.j0 + i);
+          if (i == 0 && n_units > 0 && !mbar_wait(ofree, (n_units - 1) & 1)) {
+            fail(412);
+            return;
+          }
+          if (!mbar_wait(pfull, n_px & 1)) {
+            fail(413);
+            return;
+          }
+          tc_fence_after();
+          for (int c = 0; c < nch; ++c) {
+            if (!mbar_wait(&full[stage], phase)) {
+              fail(414);
+              return;
+            }
+            tc_fence_after();
+            const uint32_t sa = smem_u32(smem + stage * S::kStageBytes);
+            const uint64_t pd = sdesc_k_sw128(p_smem + c * S::kPChunkBytes);
+            const uint64_t hd = sdesc_k_sw128(sa);
+            const uint64_t ld = sdesc_k_sw128(sa + 2 * S::kXBox);
+#pragma unroll
+            for (int k = 0; k < kBK / 16; ++k)
+              tc_mma_f16(o_tmem, pd + 2 * k, hd + 2 * k, idesc_hi,
+                         (i > 0 || c > 0 || k > 0) ? 1u : 0u);
+#pragma unroll
+            for (int k = 0; k < kBK / 16; ++k)
+              tc_mma_f16(o_tmem, pd + 2 * k, ld + 2 * k, idesc_lo, 1u);
+            issued = true;
+            tc_commit(&empty[stage]);
+            if (++stage == kStages) {
+              stage = 0;
+              phase ^= 1;
+            }
+          }
+          tc_commit(pempty);
+          ++n_px;
+        };
+        int px_next = 0;
+        for (int jj = 0; jj < J && !bad; ++jj) {
+          if (!pair_owner(jj, rank)) continue;
+          while (px_next <= jj - 2 && !bad) issue_px(px_next++);
+          if (bad) break;
+          if (n_s > 0 && !mbar_wait(sfree, (n_s - 1) & 1)) {
+            fail(410);
+            break;
+          }
+          tc_fence_after();
+          const int nst = 3 * qchunks;
+          for (int st = 0; st < nst; ++st) {
+            if (!mbar_wait(&full[stage], phase)) {
+              fail(411);
+              break;
+            }
+            tc_fence_after();
+            const uint32_t sa = smem_u32(smem + stage * S::kStageBytes);
+            const uint64_t ad = sdesc_k_sw128(sa);
+            const uint64_t bd = sdesc_k_sw128(sa + S::kQBytes);
+#pragma unroll
+            for (int k = 0; k < kBK / 16; ++k)
+              tc_mma_f16(s_tmem, ad + 2 * k, bd + 2 * k, idesc_s, (st > 0 || k > 0) ? 1u : 0u);
+            issued = true;
+            tc_commit(&empty[stage]);
+            if (++stage == kStages) {
+              stage = 0;
+              phase ^= 1;
+            }
+          }
+          if (bad) break;
+          tc_commit(sfull);
+          ++n_s;
+        }
+        while (px_next < J && !bad) issue_px(px_next++);
+        ++n_units;
+      }
+      if ((bad || *abort_flag) && issued) {
+        tc_commit(drain);
+        (void)mbar_wait(drain, 0);
+      }
+    }
+  } else {
+    // -------------------------------------------------------------- softmax / output warps
+    const int sw = warp - 2;
+    const int quarter = warp & 3;  // TMEM lanes [32 quarter, 32 quarter + 32)
+    const int half = sw >> 2;      // S columns [128 half, +128), O columns [128 half, +128)
+    const int row = quarter * 32 + lane;
+    const uint32_t lane_base = tmem_base + ((uint32_t)(quarter * 32) << 16);
+    float* kw = reinterpret_cast<float*>(smem + S::kKinvOffset) + sw * 128;
+    float* xch = reinterpret_cast<float*>(smem + S::kXchOffset);    // [2][2][128]
+    float* msg = reinterpret_cast<float*>(smem + S::kMsgOffset);    // [2][128]
+    float* lslot = reinterpret_cast<float*>(smem + S::kLslotOffset);  // [128]
+    uint8_t* pbuf = smem + S::kPOffset;
+    // the peer's copies of this CTA's message slots, barriers and P buffer
+    const uint32_t r_msg = cluster_map(smem_u32(msg), peer);
+    const uint32_t r_lslot = cluster_map(smem_u32(lslot), peer);
+    const uint32_t r_mmsg = cluster_map(smem_u32(mmsg), peer);
+    const uint32_t r_rfree = cluster_map(smem_u32(rfree), peer);
+    const uint32_t r_lmsg = cluster_map(smem_u32(lmsg), peer);
+    const uint32_t r_pfull = cluster_map(smem_u32(pfull), peer);
+    const uint32_t r_pbuf = cluster_map(smem_u32(pbuf), peer);
+    constexpr float kLog2e = 1.4426950408889634f;
+    uint32_t n_sf = 0, n_pe = 0, n_pf = 0, n_x = 0;
+    uint32_t n_msent = 0, n_mrecv = 0, n_l = 0;
+    uint32_t g = 0;  // P tiles handled so far (both CTAs count the same sequence)
+    bool bad = false;
+    auto wait_all = [&](uint64_t* bar, uint32_t parity, int where, bool cluster) -> bool {
+      bool ok = cluster ? mbar_wait_cluster(bar, parity) : mbar_wait(bar, parity);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) {
+        if (lane == 0) {
+          dev_set_error(f.err, DEV_WAIT_TIMEOUT, where);
+          *abort_flag = 1;
+        }
+        bad = true;
+      }
+      return ok;
+    };
+    // Exchanges one value per row with the other warp of this lane quarter; returns its value.
+    auto exchange = [&](float mine, int where) -> float {
+      float* slot = xch + (n_x & 1) * 256;
+      slot[half * 128 + row] = mine;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&xb[quarter]);
+      const bool ok = wait_all(&xb[quarter], n_x & 1, where, false);
+      ++n_x;
+      return ok ? slot[(1 - half) * 128 + row] : mine;
+    };
+    // The previous P X of this CTA is complete (its P buffer and O may be touched); tell the
+    // peer, whose next P copy overwrites this buffer.
+    auto prev_px_done = [&](int where) -> bool {
+      if (n_pf > n_pe) {
+        if (!wait_all(pempty, n_pe & 1, where, false)) return false;
+        ++n_pe;
+        tc_fence_after();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(r_rfree);
+      }
+      return true;
+    };
+    auto rescale_o = [&](bool rescale, float fac) {
+      // tcgen05.ld / st are warp-collective: the warp rescales when any of its rows needs it
+      if (__any_sync(0xffffffffu, rescale)) {
+#pragma unroll
+        for (int gq = 0; gq < kOCols / 32; ++gq) {
+          const uint32_t ta = lane_base + 256u + (uint32_t)(kOCols * half + 32 * gq);
+          float o[32];
+          tmem_ld32(ta, o);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) o[e] *= fac;
+          tmem_st32(ta, o);
+        }
+      }
+    };
+
+    for (int u = cid; u < f.nunits && !bad && !warp_flag(abort_flag); u += ncl) {
+      const FlashUnit w = flash_unit(f, u);
+      const int J = w.j1 - w.j0;
+      float m_run = -INFINITY, l_part = 0.f;
+      for (int jj = 0; jj < J; ++jj, ++g) {
+        const int j = w.j0 + jj;
+        if (pair_owner(jj, rank)) {
+          // ---------------- own tile: softmax of S_j
+          const int key0 = j * kPairKeys + kCols * half;
+          float kv[kCols / 32];
+#pragma unroll
+          for (int e = 0; e < kCols / 32; ++e) {
+            const int key = key0 + lane + 32 * e;
+            kv[e] = key < f.N ? f.kinv[(int64_t)w.b * f.N + key] * kLog2e : 0.f;
+          }
+          if (!wait_all(sfull, n_sf & 1, 420, false)) break;
+          ++n_sf;
+          tc_fence_after();
+          float v[kCols];
+#pragma unroll
+          for (int gq = 0; gq < kCols / 32; ++gq) {
+            float tmp[32];
+            tmem_ld32(lane_base + (uint32_t)(kCols * half + 32 * gq), tmp);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) v[32 * gq + e] = tmp[e];
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(sfree);
+#pragma unroll
+          for (int e = 0; e < kCols / 32; ++e) kw[lane + 32 * e] = kv[e];
+          __syncwarp();
+          const int cvalid = f.N - key0;
+          float mx = -INFINITY;
+#pragma unroll
+          for (int c = 0; c < kCols; c += 4) {
+            const float4 k4 = *reinterpret_cast<const float4*>(kw + c);
+            v[c] = c < cvalid ? v[c] * k4.x : -INFINITY;
+            v[c + 1] = c + 1 < cvalid ? v[c + 1] * k4.y : -INFINITY;
+            v[c + 2] = c + 2 < cvalid ? v[c + 2] * k4.z : -INFINITY;
+            v[c + 3] = c + 3 < cvalid ? v[c + 3] * k4.w : -INFINITY;
+            mx = fmaxf(mx, fmaxf(fmaxf(v[c], v[c + 1]), fmaxf(v[c + 2], v[c + 3])));
+          }
+          __syncwarp();
+          mx = fmaxf(mx, exchange(mx, 421));
+          if (bad) break;
+          bool rescale = false;
+          float fac = 1.f;
+          if (m_run == -INFINITY) {
+            m_run = mx;
+          } else if (mx > m_run + kRescaleLog2) {
+            fac = exp2f(m_run - mx);
+            m_run = mx;
+            l_part *= fac;
+            rescale = true;
+          }
+          // the tile's running max to the peer, before anything else of this tile
+          if (half == 0) {
+            st_cluster_f32(r_msg + (uint32_t)(((n_msent & 1) * 128 + row) * 4), m_run);
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(r_mmsg);
+          }
+          ++n_msent;
+          uint32_t pk[kCols / 2];
+#pragma unroll
+          for (int c = 0; c < kCols; c += 2) {
+            const float p0 = exp2f(v[c] - m_run), p1 = exp2f(v[c + 1] - m_run);
+            const __half2 h = __floats2half2_rn(p0, p1);
+            const float2 r2 = __half22float2(h);
+            pk[c / 2] = *reinterpret_cast<const uint32_t*>(&h);
+            l_part += r2.x + r2.y;
+          }
+          // This CTA's previous P X done (buffer, O) and the peer's (its buffer).
+          if (!prev_px_done(422)) break;
+          if (g > 0 && !wait_all(rfree, (g - 1) & 1, 423, true)) break;
+          rescale_o(rescale, fac);
+#pragma unroll
+          for (int q = 0; q < kCols / 64; ++q) {
+            const int chunk = (kCols / 64) * half + q;
+            uint4* dst = reinterpret_cast<uint4*>(pbuf + chunk * S::kPChunkBytes + row * 128);
+#pragma unroll
+            for (int un = 0; un < 8; ++un) {
+              const int base = (64 * q + 8 * un) / 2;
+              dst[un ^ (row & 7)] = make_uint4(pk[base], pk[base + 1], pk[base + 2], pk[base + 3]);
+            }
+          }
+          fence_proxy_async_smem();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) {
+            // this warp's rows of its two chunks, 4 KB each, into the peer's P buffer
+#pragma unroll
+            for (int q = 0; q < kCols / 64; ++q) {
+              const uint32_t off =
+                  (uint32_t)(((kCols / 64) * half + q) * S::kPChunkBytes + quarter * 32 * 128);
+              bulk_copy_to_cluster(r_pbuf + off, pbuf + off, 32 * 128, r_pfull);
+            }
+            mbar_arrive(pfull);
+          }
+          ++n_pf;
+        } else {
+          // ---------------- peer tile: its running max, O rescale, P arrives by bulk copy
+          if (!wait_all(mmsg, n_mrecv & 1, 424, true)) break;
+          const float m_new = msg[(n_mrecv & 1) * 128 + row];
+          ++n_mrecv;
+          bool rescale = false;
+          float fac = 1.f;
+          if (m_run != -INFINITY && m_new != m_run) {
+            fac = exp2f(m_run - m_new);
+            l_part *= fac;
+            rescale = true;
+          }
+          m_run = m_new;
+          if (!prev_px_done(425)) break;
+          rescale_o(rescale, fac);
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) {
+            if (sw == 0)
+              mbar_arrive_expect_tx(pfull, kPairPBytes);
+            else
+              mbar_arrive(pfull);
+          }
+          ++n_pf;
+        }
+      }
+      if (bad) break;
+      // ---- unit output: wait for the last P X, drain O, hand TMEM back, store.
+      if (!prev_px_done(426)) break;
+      tc_fence_after();
+      float o[kOCols];
+#pragma unroll
+      for (int gq = 0; gq < kOCols / 32; ++gq) {
+        float tmp[32];
+        tmem_ld32(lane_base + 256u + (uint32_t)(kOCols * half + 32 * gq), tmp);
+#pragma unroll
+        for (int e = 0; e < 32; ++e) o[32 * gq + e] = tmp[e];
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(ofree);
+      const float l_cta = l_part + exchange(l_part, 427);
+      if (bad) break;
+      // row sums of both CTAs, added in rank order so that both hold the same bits
+      if (half == 0) {
+        st_cluster_f32(r_lslot + (uint32_t)(row * 4), l_cta);
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(r_lmsg);
+      }
+      if (!wait_all(lmsg, n_l & 1, 428, true)) break;
+      ++n_l;
+      const float l_peer = lslot[row];
+      const float l_tot = rank == 0 ? l_cta + l_peer : l_peer + l_cta;
+      const int r = w.tm * kBM + row;
+      if (r < f.t) {
+        const int64_t orow = ((int64_t)w.split * f.nb + w.b) * f.t + r;
+        // local columns [0, 128): K~ features 128 rank + c; [128, 256): V features
+        const int feat0 = (half == 0 ? 0 : 256) + 128 * (int)rank;
+        float4* dst = reinterpret_cast<float4*>(f.O + orow * 512 + feat0);
+#pragma unroll
+        for (int c = 0; c < kOCols; c += 4) dst[c / 4] = make_float4(o[c], o[c + 1], o[c + 2], o[c + 3]);
+        if (rank == 0 && half == 0) f.stats[orow] = make_float2(m_run, l_tot);
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, 512);
+  }
+  // Neither CTA leaves while the other may still copy into or arrive on its shared memory.
+  cluster_sync();
+}
+
+}  // namespace
+
+// The persistent grid holds no more clusters than can be resident at once (a cluster needs two
+// free SMs of one GPC): a cluster that waited for another to exit would start its whole share
+// of the units late.
+int ca_pair_clusters(int num_sms) {
+  static thread_local int resident = 0;
+  if (resident == 0) {
+    if (cudaFuncSetAttribute(ca_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             PairSmem::kBytes) != cudaSuccess) {
+      cudaGetLastError();
+      return std::max(1, num_sms / 2);
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * std::max(1, num_sms / 2), 1, 1);
+    cfg.blockDim = dim3(kFlashThreads, 1, 1);
+    cfg.dynamicSmemBytes = PairSmem::kBytes;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, ca_pair_kernel, &cfg) != cudaSuccess || n < 1) {
+      cudaGetLastError();
+      n = num_sms / 2;
+    }
+    resident = std::max(1, std::min(n, num_sms / 2));
+  }
+  return resident;
+}
+
+cudaError_t launch_ca_pair(const Operand2D& Q, const Operand2D& K, const Operand2D& XT,
+                           const FlashParams& f, int num_sms, cudaStream_t stream) {
+  using S = PairSmem;
+  if (f.D <= 0 || f.D % kBK != 0 || f.t <= 0 || f.N <= 0 || f.Np % kBK != 0 || f.Np < f.N ||
+      f.nunits <= 0)
+    return cudaErrorInvalidValue;
+  CUtensorMap tq, tk, tx;
+  if (!make_tmap(&tq, Q, kBM) || !make_tmap(&tk, K, kPairKeys) || !make_tmap(&tx, XT, 128))
+    return cudaErrorInvalidValue;
+  static thread_local bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(ca_pair_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, S::kBytes);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(kFlashThreads, 1, 1);
+  cfg.dynamicSmemBytes = S::kBytes;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const int clusters = std::max(1, std::min(f.nunits, ca_pair_clusters(num_sms)));
+  cfg.gridDim = dim3(2 * clusters, 1, 1);
+  return cudaLaunchKernelEx(&cfg, ca_pair_kernel, tq, tk, tx, f);
+}
+
+}  // namespace still

@@ -337,6 +337,14 @@ struct Plan {
 
 size_t a256(size_t x) { return (x + 255) & ~size_t(255); }
 
+// The self-attention value path (probabilities, values, head outputs) and the FFN run in bf16
+// hi | lo rather than plain bf16 in layers of more than one block (the next block's queries
+// amplify their rounding) and in compactors of width d_l >= 2048. There the self-attention
+// output, whose logits d_l cos(q, k) are the sharpest, dominates the latent state: emulating
+// plain-bf16 probabilities, values and FFN activations on the Gemma-shaped compactor moves C_k
+// from the output-rounding floor of 0.009 to 0.015 x RMS, against 0.009 in hi | lo.
+bool value_hilo(const still_layer_config& c) { return c.n_blocks > 1 || c.d_latent >= 2048; }
+
 bool make_plan(const still_layer_config& c, bool lazy_q, int Kp, int64_t N, int t, double pmin,
                double pmax, size_t limit, Plan& P) {
   P.H = c.n_kv_heads;
@@ -368,7 +376,7 @@ bool make_plan(const still_layer_config& c, bool lazy_q, int Kp, int64_t N, int 
   P.oZ1 = take(H * T * D * 4);
   P.oA1 = take(H * T * 2 * D * 2);
   // A block that feeds another keeps its value path in hi/lo (x2 buffers below).
-  const int64_t hl = c.n_blocks > 1 ? 2 : 1;
+  const int64_t hl = value_hilo(c) ? 2 : 1;
   P.oCat = take(H * T * n * D * 2 * hl);
   P.oZ2 = take(H * T * D * 4);
   P.oA2 = take(H * T * D * 2 * hl);
@@ -382,9 +390,9 @@ bool make_plan(const still_layer_config& c, bool lazy_q, int Kp, int64_t N, int 
   P.kb_b = Kp > 0 ? 0 : a256(N * 2 * D * 2);
   P.kss_b = a256(N * 4 * (kparts + 1));
   P.q_b = Kp > 0 ? 0 : a256(T * 2 * D * 2);
-  // The fused kernel serves every block when 2d <= 256 (a block that feeds another takes its
-  // split-precision variant); 2d = 512 takes the scores + P X kernels.
-  P.flash = d == 64 || d == 128;
+  // The fused kernel serves every block (a block that feeds another takes its split-precision
+  // variant); 2d = 512 runs it on clusters of two CTAs that split the O columns.
+  P.flash = d == 64 || d == 128 || d == 256;
   P.split_ca = !P.flash;
   P.S_b = 0;
   P.P_b = 0;
@@ -582,7 +590,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
   // hi | lo too, and the first block's value chains (P X, W_V W_O, RMSNorm(Z'), the
   // self-attention q, k, v, P and head outputs) are fp16 hi | lo rather than bf16 hi | lo.
   const bool exact = !last;
-  const bool vexact = exact || L.f16;
+  const bool vexact = exact || L.f16 || value_hilo(c);
   const bool f16v = exact && L.f16 && P.flash;
   const int vfmt = f16v ? 0 : 1;
   const int32_t vkind = f16v ? OUT_HILO16 : OUT_HILO;
@@ -742,7 +750,9 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       fp.tiles_m = (t + kBM - 1) / kBM;
       const int fkeys = exact ? FlashSmem<256, true>::kKeys : kFlashKeys;
       fp.tiles_k = (int)((N + fkeys - 1) / fkeys);
-      fp.nsplit = flash_split((int64_t)fp.tiles_m * nbl, fp.tiles_k, ctx->nsm, kMaxFlashSplit);
+      // 2d = 512: a unit occupies a cluster of two SMs
+      const int slots = d == 256 ? ca_pair_clusters(ctx->nsm) : ctx->nsm;
+      fp.nsplit = flash_split((int64_t)fp.tiles_m * nbl, fp.tiles_k, slots, kMaxFlashSplit);
       const int64_t nunits = (int64_t)fp.tiles_m * nbl * fp.nsplit;
       if (nunits > 0x7fffffff || (int64_t)nbl * N > 0x7fffffff) return STILL_ERR_UNSUPPORTED;
       fp.nunits = (int)nunits;
@@ -765,10 +775,12 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       const Operand2D xop = op(XT, (int64_t)H * 2 * d, 2 * Np);
       ctx->prof.begin(STILL_K_CA_FUSED, s);
       cudaError_t r =
-          exact ? (d == 64 ? launch_ca_flash<128, true>(qop, kop, xop, fp, ctx->nsm, s)
-                           : launch_ca_flash<256, true>(qop, kop, xop, fp, ctx->nsm, s))
-                : (d == 64 ? launch_ca_flash<128>(qop, kop, xop, fp, ctx->nsm, s)
-                           : launch_ca_flash<256>(qop, kop, xop, fp, ctx->nsm, s));
+          d == 256 ? (exact ? cudaErrorInvalidValue  // two-block layers at d = 256 are refused
+                            : launch_ca_pair(qop, kop, xop, fp, ctx->nsm, s))
+          : exact  ? (d == 64 ? launch_ca_flash<128, true>(qop, kop, xop, fp, ctx->nsm, s)
+                              : launch_ca_flash<256, true>(qop, kop, xop, fp, ctx->nsm, s))
+                   : (d == 64 ? launch_ca_flash<128>(qop, kop, xop, fp, ctx->nsm, s)
+                              : launch_ca_flash<256>(qop, kop, xop, fp, ctx->nsm, s));
       ctx->prof.end(STILL_K_CA_FUSED, s);
       if (r == cudaErrorInvalidValue) return STILL_ERR_INVALID_ARG;
       if (r != cudaSuccess) return STILL_ERR_CUDA;

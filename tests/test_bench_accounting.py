@@ -29,8 +29,8 @@ def test_one_block_flops(name, t):
     assert fl["scores"] == 2 * t * N * H * n * D
     assert fl["px"] == 2 * t * N * H * n * 2 * d
     assert fl["px_passes"] == 1.5
-    # the two-kernel path (2d = 512) times the scores GEMM; otherwise the fused kernel
-    assert fl["scores_gemm"] == (fl["scores"] if 2 * d > 256 else 0)
+    # every head size takes the fused kernel (2d = 512 on clusters of two CTAs)
+    assert fl["scores_gemm"] == 0
 
 
 def test_two_block_flops_count_both_blocks():

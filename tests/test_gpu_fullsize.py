@@ -7,9 +7,12 @@
   per call and a workspace limit small enough that the cross-attention runs in groups of part
   of a KV-head and the self-attention bank in head sub-groups.
 * The iterative workload (Qwen-8B shape, 8 ragged sequences, 32x): the initial compaction and
-  16 rounds of [compact | 8192 new tokens] re-compaction of one layer; the oracle runs the same
-  17 compactions for one sequence and one KV-head on its own state, which it stores between
-  rounds in the cache dtype (bf16) as the library's outputs are (Sec. 2.3).
+  16 rounds of [compact | 8192 new tokens] re-compaction of one layer (Sec. 2.3), every round
+  compared with the oracle. The oracle carries one sequence's compact cache of one KV-head
+  from round to round in the cache dtype (bf16), and the GPU recompacts that same cache: the
+  recursion amplifies any difference in its state (two runs that each meet the bar every
+  round drift apart over 16 rounds), so each round is checked on identical inputs. The other
+  sequences and KV-heads carry the GPU's own outputs.
 
 Bar: max |err| <= 2e-2 RMS(oracle), row cosine >= 0.999, C_k and C_v separately.
 """
@@ -55,14 +58,19 @@ def test_gemma_shape_8192_latents_per_call_queries_and_head_subgroups():
         still.still_load_layer_weights(ctx, 0, still.config_from_workload(wl, t), W)
         rk, rv, _, _ = oracle_layer(wl, W, K, V, t)
         total = still.still_workspace_size(ctx, wl["N"], t)
-        subgroups = 0
-        for frac in (1.0, 0.5, 0.3):
+        subgroups, runs = 0, 0
+        for frac in (1.0, 0.6, 0.45, 0.3):
             still.still_set_workspace_limit(ctx, int(total * frac))
             still.still_profile_enable(ctx, True)
             still.still_profile_enable_classes(ctx, [])  # launch counts only
             Ck = torch.empty((t, 1, wl["d"]), dtype=torch.bfloat16, device=DEV)
             Cv = torch.empty_like(Ck)
-            still.still_compact_layer(ctx, 0, K, V, t, Ck, Cv)
+            try:
+                still.still_compact_layer(ctx, 0, K, V, t, Ck, Cv)
+            except still.StillError as e:  # below the smallest grouping of this shape
+                assert e.name == "STILL_ERR_OOM", e.name
+                continue
+            runs += 1
             code, det = still.still_get_device_status(ctx)
             assert code == 0, det
             prof = still.still_profile_read(ctx)
@@ -72,7 +80,7 @@ def test_gemma_shape_8192_latents_per_call_queries_and_head_subgroups():
                 subgroups += 1
             assert_parity(rk, synth.bf16_to_f64(Ck), f"C_k limit {frac}")
             assert_parity(rv, synth.bf16_to_f64(Cv), f"C_v limit {frac}")
-        assert subgroups >= 1
+        assert runs >= 3 and subgroups >= 1, (runs, subgroups)
     finally:
         still.still_destroy(ctx)
 
@@ -88,6 +96,7 @@ def test_iterative_16_rounds_one_sequence_matches_oracle():
     r = Runner(dict(wl, N=0), t_max)
     cfg = O.cfg_from_workload(wl)
     Wf = O.as_f64(r.W[0])
+    bf = lambda x: torch.from_numpy(x).to(torch.bfloat16)
     try:
         ts = [O.budget(x, ratio) for x in lens]
         parts = [synth.gen_kv(wl, 0, N=x, device=DEV, stream=s) for s, x in enumerate(lens)]
@@ -97,16 +106,23 @@ def test_iterative_16_rounds_one_sequence_matches_oracle():
         still.still_compact_layer_ragged(r.ctx, 0, torch.cat([p[0] for p in parts]),
                                          torch.cat([p[1] for p in parts]), cu, ts, Ck, Cv)
         r.check_status()
-        # the oracle's round 0 on sequence b, KV-head h; its state is kept in bf16
         kb, vb = synth.bf16_to_f64(parts[b][0][:, h]), synth.bf16_to_f64(parts[b][1][:, h])
         del parts
         ok, ov, opos = O.compact_head(kb, vb, Wf["Z"][h, :ts[b]], Wf, cfg,
                                       np.arange(lens[b], dtype=np.float64))
-        bf = lambda x: torch.from_numpy(x).to(torch.bfloat16).to(torch.float64).numpy()
-        ok, ov = bf(ok), bf(ov)
         cu_prev = np.concatenate([[0], np.cumsum(ts)]).tolist()
         prev_len = list(lens)
-        for rnd in range(rounds):
+        for rnd in range(rounds + 1):
+            rows = slice(cu_prev[b], cu_prev[b + 1])
+            assert_parity(ok, synth.bf16_to_f64(Ck[rows, h]), f"C_k seq {b} head {h} round {rnd}")
+            assert_parity(ov, synth.bf16_to_f64(Cv[rows, h]), f"C_v seq {b} head {h} round {rnd}")
+            if rnd == rounds:
+                break
+            # the state both sides carry into the next round: the oracle's cache, in bf16
+            ok, ov = bf(ok), bf(ov)
+            Ck[rows, h] = ok.to(DEV)
+            Cv[rows, h] = ov.to(DEV)
+            ok, ov = ok.double().numpy(), ov.double().numpy()
             newkv = [synth.gen_kv(wl, 0, N=chunk, device=DEV, stream=1000 * (rnd + 1) + s,
                                   positions=torch.arange(prev_len[s], prev_len[s] + chunk,
                                                          dtype=torch.float64))
@@ -121,7 +137,7 @@ def test_iterative_16_rounds_one_sequence_matches_oracle():
             r.check_status()
             assert len_out == [x + chunk for x in prev_len]
             assert cu_out == np.concatenate([[0], np.cumsum(t_next)]).tolist()
-            # oracle: [its compact cache at its output positions | the new tokens]
+            # oracle: [the compact cache at its output positions | the new tokens]
             kn = synth.bf16_to_f64(newkv[b][0][:, h])
             vn = synth.bf16_to_f64(newkv[b][1][:, h])
             kpos = np.concatenate([opos, np.arange(prev_len[b], prev_len[b] + chunk,
@@ -129,11 +145,6 @@ def test_iterative_16_rounds_one_sequence_matches_oracle():
             ok, ov, opos = O.compact_head(np.concatenate([ok, kn]), np.concatenate([ov, vn]),
                                           Wf["Z"][h, :t_next[b]], Wf, cfg, kpos)
             np.testing.assert_allclose(opos, O.linspace_positions(0, len_out[b] - 1, t_next[b]))
-            if rnd + 1 < rounds:
-                ok, ov = bf(ok), bf(ov)
             Ck, Cv, cu_prev, prev_len = Ck2, Cv2, cu_out, len_out
-        rows = slice(cu_prev[b], cu_prev[b + 1])
-        assert_parity(ok, synth.bf16_to_f64(Ck[rows, h]), f"C_k seq {b} head {h} round {rounds}")
-        assert_parity(ov, synth.bf16_to_f64(Cv[rows, h]), f"C_v seq {b} head {h} round {rounds}")
     finally:
         r.close()
