@@ -43,6 +43,12 @@ def folded(wl):
     return Kp if ok else 0
 
 
+def one_pass_scores(wl):
+    """Whether the library computes this workload's cross-attention scores in one fp16 pass
+    with a repair of each row's heaviest logits (one block, head dim 256, 512 <= d_l <= 2048)."""
+    return wl.get("n_blocks", 1) == 1 and wl["d"] == 256 and 512 <= wl["D"] <= 2048
+
+
 def describe(name, wl, t):
     nb = wl.get("n_blocks", 1)
     blocks = "" if nb == 1 else (f", {nb} blocks" + (" (CA in every block)"
@@ -682,7 +688,10 @@ def main():
     fused = kname == "ca_fused"
     n_k, ms_k = prof_timed[kname]  # one step's launches (the captured event pairs)
     alg = fl["scores"] + fl["px"] if fused else fl["scores_gemm"]
-    issued = (3 * fl["scores"] + fl["px_passes"] * fl["px_blk"] if fused
+    # one fp16 pass for the scores where the library takes them (head dim 256, one block,
+    # 512 <= d_l <= 2048), else three split-bf16 passes
+    qk_passes = 1 if one_pass_scores(wl) else 3
+    issued = (qk_passes * fl["scores"] + fl["px_passes"] * fl["px_blk"] if fused
               else 3 * fl["scores_gemm"])
     per_launch_flops = alg * L / max(n_k, 1)
     achieved = per_launch_flops / (ms_k / max(n_k, 1) / 1e3) / 1e12 if ms_k > 0 else None
@@ -690,7 +699,9 @@ def main():
     traffic = None
     if tr["kernel_hash"] == _kernel_hash(tr["files"]) and tr["workload"] == (name, t):
         traffic = tr["bytes_per_launch"]
-    kdesc = ("ca_fused (3-pass split-bf16 scores + online softmax + P X, one tcgen05 kernel"
+    kdesc = ("ca_fused (" + ("1-pass fp16 scores with a top-k logit repair" if qk_passes == 1
+                             else "3-pass split-bf16 scores")
+             + " + online softmax + P X, one tcgen05 kernel"
              + ("; clusters of two CTAs that split the 512 O columns" if 2 * d == 512 else "")
              + ("; the first block's launches in split fp16 with P hi + lo)"
                 if wl.get("n_blocks", 1) > 1 and wl.get("cross_every_block", 1) else ")")

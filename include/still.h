@@ -443,9 +443,10 @@ typedef enum {
   STILL_K_HEADS,        /* C_k, C_v output heads + re-rotation              */
   STILL_K_NORMS,        /* QK-norm factors from sum-of-squares partials     */
   STILL_K_LOAD,         /* weight-load precompute GEMMs                     */
-  STILL_K_CA_FUSED,     /* fused scores + online softmax + P X (d <= 128)   */
+  STILL_K_CA_FUSED,     /* fused scores + online softmax + P X              */
   STILL_K_BETA,         /* beta head: Z_out w_beta, shaped                  */
   STILL_K_DECODE,       /* biased decode attention (chunks + merge)         */
+  STILL_K_REPAIR,       /* top-k repair of one-pass cross-attention scores  */
   STILL_K_COUNT
 } still_kernel_class;
 

@@ -42,7 +42,15 @@ struct FlashParams {
   float* O = nullptr;           // [nsplit][nb][t][2d] unnormalised
   float2* stats = nullptr;      // [nsplit][nb][t]: (running max m in log2 units, sum l)
   int* err = nullptr;
+  // One-pass scores with a top-k repair (ca_pair_kernel<true>): per (split, b, row), kTopK
+  // candidates per list and kTopLists lists, as (key, c = m + log2 p of the weight used);
+  // key -1 marks an empty slot.
+  int* cand_key = nullptr;      // [nsplit][nb][t][kTopLists][kTopK]
+  float* cand_c = nullptr;
 };
+
+constexpr int kTopK = 8;       // repair candidates per list
+constexpr int kTopLists = 4;   // lists per row: (CTA of the pair, half of the key tile)
 
 constexpr int kFlashKeys = 256;       // keys per S tile (EX: 128)
 constexpr int kFlashSoftWarps = 8;    // two per TMEM lane quarter
@@ -568,9 +576,35 @@ inline cudaError_t launch_ca_flash(const Operand2D& Q, const Operand2D& K, const
 // 2d = 512 (head dim 256): the same computation on a cluster of two CTAs that split the O
 // columns and take turns computing S (ca_pair.cu). Q, K as for launch_ca_flash; XT: [H*512][2*Np]
 // fp16 (hi | lo). num_sms: SMs of the device (two per cluster).
+// one_pass: q, k as fp16 hi | lo with S from the hi parts only (one MMA pass) and repair
+// candidates in f.cand_key / f.cand_c for ca_topk_repair; else 3-pass split-bf16 scores.
 cudaError_t launch_ca_pair(const Operand2D& Q, const Operand2D& K, const Operand2D& XT,
-                           const FlashParams& f, int num_sms, cudaStream_t stream);
+                           const FlashParams& f, int num_sms, cudaStream_t stream,
+                           bool one_pass = false);
 // Clusters of that kernel that can be resident at once (its persistent grid size).
 int ca_pair_clusters(int num_sms);
+
+// Top-k repair of one-pass scores: for each (b, row), over the splits whose running max is within
+// `cut` (log2 units) of the row's largest, each candidate's exact logit
+// e = kinv (q_hi + q_lo) . (k_hi + k_lo) log2 e replaces the one-pass value c that the fused
+// kernel used: delta = 2^(e - m) - 2^(c - m) is added to the split's l and delta X_key to its O.
+// A split whose weight outside its candidates exceeds `guard` of its l is recomputed exactly
+// over all its keys. Candidates below 2^-cut of the row's largest weight are left as they are.
+// Deterministic: splits and candidates in a fixed order, one warp per row.
+struct TopkRepairParams {
+  const __half* q = nullptr;          // [nb * t][2D] fp16 hi | lo (times the q scale)
+  const __half* k = nullptr;          // [nb * N][2D] fp16 hi | lo
+  const float* kinv = nullptr;        // [nb][N]: logit scale / (q scale |k~|)
+  const __nv_bfloat16* X = nullptr;   // KV-head h0's rows [N][3d]: hi [0, 2d), lo of K~ [2d, 3d)
+  float* O = nullptr;                 // [nsplit][nb][t][2d]
+  float2* stats = nullptr;            // [nsplit][nb][t]: (m log2 units, l)
+  const int* cand_key = nullptr;      // [nsplit][nb][t][nlists][kTopK]
+  const float* cand_c = nullptr;
+  int32_t D = 0, d = 0, t = 0, N = 0, nb = 0, nsplit = 1, bdiv = 1, nlists = 0;
+  int32_t tiles_k = 0, keys_per_tile = 256;  // the fused kernel's key tiles and splits
+  float cut = 24.f;
+  float guard = 1.f / 64.f;
+};
+cudaError_t launch_ca_topk_repair(const TopkRepairParams& f, int d2, cudaStream_t stream);
 
 }  // namespace still

@@ -70,10 +70,13 @@ __device__ __forceinline__ bool pair_owner(int jj, uint32_t rank) {
   return (uint32_t)(jj & 1) == rank;
 }
 
+// TK: one-pass fp16 scores (q_hi . k_hi) with repair candidates; else 3-pass split-bf16.
+template <bool TK>
 __global__ void __launch_bounds__(kFlashThreads, 1)
     ca_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmX, const FlashParams f) {
   using S = PairSmem;
+  constexpr int kPasses = TK ? 1 : 3;
   constexpr int kStages = S::kStages;
   constexpr int kCols = kPairKeys / 2;   // S columns per softmax warp (its half of the tile)
   constexpr int kOCols = kPairOCols / 2;  // O columns per softmax warp
@@ -186,7 +189,7 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
           if (!pair_owner(jj, rank)) continue;
           while (px_next <= jj - 2 && !bad) produce_px(px_next++);
           const int32_t kr = krow + (w.j0 + jj) * kPairKeys;
-          for (int pass = 0; pass < 3 && !bad; ++pass) {
+          for (int pass = 0; pass < kPasses && !bad; ++pass) {
             const int32_t qoff = pass == 2 ? f.D : 0;  // (q_hi,k_hi), (q_hi,k_lo), (q_lo,k_hi)
             const int32_t koff = pass == 1 ? f.D : 0;
             for (int c = 0; c < qchunks; ++c) {
@@ -208,7 +211,7 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
   } else if (warp == 1) {
     if (lane == 0) {
       // ------------------------------------------------------------ MMA issuer
-      const uint32_t idesc_s = idesc_f16(kBM, kPairKeys, 1);   // bf16 q, k
+      const uint32_t idesc_s = idesc_f16(kBM, kPairKeys, TK ? 0 : 1);  // fp16 / bf16 q, k
       const uint32_t idesc_hi = idesc_f16(kBM, kPairOCols, 0);  // fp16 P, X^T hi (K~ | V)
       const uint32_t idesc_lo = idesc_f16(kBM, 128, 0);         // fp16 P, X^T lo (K~ half)
       const uint32_t s_tmem = tmem_base;
@@ -274,7 +277,7 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
             break;
           }
           tc_fence_after();
-          const int nst = 3 * qchunks;
+          const int nst = kPasses * qchunks;
           for (int st = 0; st < nst; ++st) {
             if (!mbar_wait(&full[stage], phase)) {
               fail(411);
@@ -384,6 +387,16 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
       const FlashUnit w = flash_unit(f, u);
       const int J = w.j1 - w.j0;
       float m_run = -INFINITY, l_part = 0.f;
+      // TK: the kTopK keys of this row half (own tiles) with the largest weights used
+      int tk_key[TK ? kTopK : 1];
+      float tk_c[TK ? kTopK : 1];
+      float tk_tau = -INFINITY;  // smallest c in the list (-inf while a slot is free)
+      int tk_slot = 0;           // its slot
+#pragma unroll
+      for (int e = 0; e < (TK ? kTopK : 1); ++e) {
+        tk_key[e] = -1;
+        tk_c[e] = -INFINITY;
+      }
       for (int jj = 0; jj < J; ++jj, ++g) {
         const int j = w.j0 + jj;
         if (pair_owner(jj, rank)) {
@@ -424,6 +437,7 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
             mx = fmaxf(mx, fmaxf(fmaxf(v[c], v[c + 1]), fmaxf(v[c + 2], v[c + 3])));
           }
           __syncwarp();
+          const float mx_own = mx;
           mx = fmaxf(mx, exchange(mx, 421));
           if (bad) break;
           bool rescale = false;
@@ -480,6 +494,50 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
             mbar_arrive(pfull);
           }
           ++n_pf;
+          if constexpr (TK) {
+            // This row half's weights, read back from the P tile (the tensor core and the bulk
+            // copies only read it; the buffer is written again after this thread's next wait),
+            // when the tile holds a logit above the list's smallest: rare once the list holds
+            // the row's heavy keys.
+            if (mx_own > tk_tau) {
+#pragma unroll 1
+              for (int q = 0; q < kCols / 64; ++q) {
+                const int chunk = (kCols / 64) * half + q;
+                const uint4* src =
+                    reinterpret_cast<const uint4*>(pbuf + chunk * S::kPChunkBytes + row * 128);
+#pragma unroll 1
+                for (int un = 0; un < 8; ++un) {
+                  const uint4 w4 = src[un ^ (row & 7)];
+                  const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
+#pragma unroll
+                  for (int e = 0; e < 8; ++e) {
+                    const uint16_t hb = (uint16_t)(wv[e >> 1] >> (16 * (e & 1)));
+                    const float p = __half2float(__ushort_as_half(hb));
+                    if (p > 0.f) {
+                      const float c = m_run + log2f(p);
+                      if (c > tk_tau) {
+                        const int key = key0 + 64 * q + 8 * un + e;
+#pragma unroll
+                        for (int sl = 0; sl < kTopK; ++sl)
+                          if (sl == tk_slot) {
+                            tk_key[sl] = key;
+                            tk_c[sl] = c;
+                          }
+                        tk_tau = tk_c[0];
+                        tk_slot = 0;
+#pragma unroll
+                        for (int sl = 1; sl < kTopK; ++sl)
+                          if (tk_c[sl] < tk_tau) {
+                            tk_tau = tk_c[sl];
+                            tk_slot = sl;
+                          }
+                      }
+                    }
+                  }
+                }
+              }
+            }
+          }
         } else {
           // ---------------- peer tile: its running max, O rescale, P arrives by bulk copy
           if (!wait_all(mmsg, n_mrecv & 1, 424, true)) break;
@@ -542,6 +600,14 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
 #pragma unroll
         for (int c = 0; c < kOCols; c += 4) dst[c / 4] = make_float4(o[c], o[c + 1], o[c + 2], o[c + 3]);
         if (rank == 0 && half == 0) f.stats[orow] = make_float2(m_run, l_tot);
+        if constexpr (TK) {
+          const int64_t cb = (orow * kTopLists + 2 * (int)rank + half) * kTopK;
+#pragma unroll
+          for (int sl = 0; sl < kTopK; ++sl) {
+            f.cand_key[cb + sl] = tk_key[sl];
+            f.cand_c[cb + sl] = tk_c[sl];
+          }
+        }
       }
     }
   }
@@ -556,7 +622,154 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
   cluster_sync();
 }
 
+// One warp per (batch b, row r): the exact logits of the row's repair candidates replace the
+// one-pass ones in every split's (O, l). See launch_ca_topk_repair.
+template <int D2>
+__global__ void __launch_bounds__(256) ca_topk_repair_kernel(const TopkRepairParams f) {
+  constexpr float kLog2e = 1.4426950408889634f;
+  constexpr int kG = D2 / 128;  // 4-column groups of O per lane
+  constexpr int kQ = 8;         // 8-element q groups per lane (D <= 2048)
+  const int64_t rows = (int64_t)f.nb * f.t;
+  const int64_t rj = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (rj >= rows) return;
+  const int b = (int)(rj / f.t);
+  float M = -INFINITY;
+  for (int s = 0; s < f.nsplit; ++s) M = fmaxf(M, f.stats[s * rows + rj].x);
+  uint4 qh[kQ], ql[kQ];
+  const __half* qrow = f.q + rj * 2 * (int64_t)f.D;
+#pragma unroll
+  for (int it = 0; it < kQ; ++it) {
+    const int i = 8 * lane + 256 * it;
+    qh[it] = i < f.D ? *reinterpret_cast<const uint4*>(qrow + i) : make_uint4(0, 0, 0, 0);
+    ql[it] = i < f.D ? *reinterpret_cast<const uint4*>(qrow + f.D + i) : make_uint4(0, 0, 0, 0);
+  }
+  // exact logit of one key in log2 units (q_hi k_hi + q_hi k_lo + q_lo k_hi, fp32), the same
+  // value in every lane
+  auto logit = [&](int key) -> float {
+    const __half* krow = f.k + ((int64_t)b * f.N + key) * 2 * (int64_t)f.D;
+    float acc = 0.f;
+#pragma unroll
+    for (int it = 0; it < kQ; ++it) {
+      const int i = 8 * lane + 256 * it;
+      if (i < f.D) {
+        const uint4 kh = *reinterpret_cast<const uint4*>(krow + i);
+        const uint4 kl = *reinterpret_cast<const uint4*>(krow + f.D + i);
+        const __half2* a = reinterpret_cast<const __half2*>(&qh[it]);
+        const __half2* al = reinterpret_cast<const __half2*>(&ql[it]);
+        const __half2* c = reinterpret_cast<const __half2*>(&kh);
+        const __half2* cl = reinterpret_cast<const __half2*>(&kl);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 x = __half22float2(a[e]), xl = __half22float2(al[e]);
+          const float2 y = __half22float2(c[e]), yl = __half22float2(cl[e]);
+          acc = fmaf(x.x, y.x, fmaf(x.x, yl.x, fmaf(xl.x, y.x, acc)));
+          acc = fmaf(x.y, y.y, fmaf(x.y, yl.y, fmaf(xl.y, y.y, acc)));
+        }
+      }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+    return acc * (f.kinv[(int64_t)b * f.N + key] * kLog2e);
+  };
+  const __nv_bfloat16* xbase = f.X + (int64_t)(b / f.bdiv) * f.N * 3 * f.d;
+  float oacc[kG][4];
+  // oacc += w * X_key (hi, plus lo on the K~ half)
+  auto add_x = [&](int key, float w) {
+    const __nv_bfloat16* xr = xbase + (int64_t)key * 3 * f.d;
+#pragma unroll
+    for (int gq = 0; gq < kG; ++gq) {
+      const int col = 4 * lane + 128 * gq;
+      const uint2 hv = *reinterpret_cast<const uint2*>(xr + col);
+      const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&hv);
+      float2 x01 = __bfloat1622float2(h2[0]), x23 = __bfloat1622float2(h2[1]);
+      if (col < f.d) {
+        const uint2 lv = *reinterpret_cast<const uint2*>(xr + 2 * f.d + col);
+        const __nv_bfloat162* l2 = reinterpret_cast<const __nv_bfloat162*>(&lv);
+        const float2 l01 = __bfloat1622float2(l2[0]), l23 = __bfloat1622float2(l2[1]);
+        x01.x += l01.x;
+        x01.y += l01.y;
+        x23.x += l23.x;
+        x23.y += l23.y;
+      }
+      oacc[gq][0] = fmaf(w, x01.x, oacc[gq][0]);
+      oacc[gq][1] = fmaf(w, x01.y, oacc[gq][1]);
+      oacc[gq][2] = fmaf(w, x23.x, oacc[gq][2]);
+      oacc[gq][3] = fmaf(w, x23.y, oacc[gq][3]);
+    }
+  };
+  const int nc = f.nlists * kTopK;
+  for (int s = 0; s < f.nsplit; ++s) {
+    const int64_t sr = s * rows + rj;
+    const float2 st = f.stats[sr];
+    if (!(st.x >= M - f.cut)) continue;  // this split's weights are negligible in the row
+    const int* ck = f.cand_key + sr * nc;
+    const float* cc = f.cand_c + sr * nc;
+#pragma unroll
+    for (int gq = 0; gq < kG; ++gq) oacc[gq][0] = oacc[gq][1] = oacc[gq][2] = oacc[gq][3] = 0.f;
+    float4* orow = reinterpret_cast<float4*>(f.O + sr * D2);
+    float wc = 0.f;  // the candidates' one-pass weights
+    for (int sl = 0; sl < nc; ++sl)
+      if (ck[sl] >= 0) wc += exp2f(cc[sl] - st.x);
+    if (st.y - wc > f.guard * st.y) {
+      // weight spread beyond the candidates: every key of the split, exact, in key order
+      const int j0 = (int)(((int64_t)f.tiles_k * s) / f.nsplit);
+      const int j1 = (int)(((int64_t)f.tiles_k * (s + 1)) / f.nsplit);
+      const int k1 = min(j1 * f.keys_per_tile, f.N);
+      float lsum = 0.f;
+      for (int key = j0 * f.keys_per_tile; key < k1; ++key) {
+        const float w = exp2f(logit(key) - st.x);
+        lsum += w;
+        add_x(key, w);
+      }
+#pragma unroll
+      for (int gq = 0; gq < kG; ++gq)
+        orow[lane + 32 * gq] = make_float4(oacc[gq][0], oacc[gq][1], oacc[gq][2], oacc[gq][3]);
+      if (lane == 0) f.stats[sr].y = lsum;
+      continue;
+    }
+    float dl = 0.f;
+    for (int sl = 0; sl < nc; ++sl) {
+      const int key = ck[sl];  // warp-uniform
+      if (key < 0 || !(cc[sl] >= M - f.cut)) continue;
+      const float delta = exp2f(logit(key) - st.x) - exp2f(cc[sl] - st.x);
+      dl += delta;
+      add_x(key, delta);
+    }
+#pragma unroll
+    for (int gq = 0; gq < kG; ++gq) {
+      float4 o = orow[lane + 32 * gq];
+      o.x += oacc[gq][0];
+      o.y += oacc[gq][1];
+      o.z += oacc[gq][2];
+      o.w += oacc[gq][3];
+      orow[lane + 32 * gq] = o;
+    }
+    if (lane == 0) f.stats[sr].y = st.y + dl;
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_ca_topk_repair(const TopkRepairParams& f, int d2, cudaStream_t stream) {
+  if (f.D <= 0 || f.D % 8 != 0 || f.D > 2048 || f.d * 2 != d2 || f.t <= 0 || f.nb <= 0 ||
+      f.N <= 0 || f.nsplit < 1 || f.nlists < 1 || f.tiles_k < f.nsplit ||
+      (int64_t)f.tiles_k * f.keys_per_tile < f.N || f.q == nullptr || f.k == nullptr ||
+      f.X == nullptr || f.O == nullptr || f.stats == nullptr || f.cand_key == nullptr ||
+      f.cand_c == nullptr || f.bdiv < 1)
+    return cudaErrorInvalidValue;
+  const int64_t rows = (int64_t)f.nb * f.t;
+  const unsigned grid = (unsigned)((rows + 7) / 8);
+  if (d2 == 512)
+    ca_topk_repair_kernel<512><<<grid, 256, 0, stream>>>(f);
+  else if (d2 == 256)
+    ca_topk_repair_kernel<256><<<grid, 256, 0, stream>>>(f);
+  else if (d2 == 128)
+    ca_topk_repair_kernel<128><<<grid, 256, 0, stream>>>(f);
+  else
+    return cudaErrorInvalidValue;
+  return cudaGetLastError();
+}
 
 // The persistent grid holds no more clusters than can be resident at once (a cluster needs two
 // free SMs of one GPC): a cluster that waited for another to exit would start its whole share
@@ -564,7 +777,7 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
 int ca_pair_clusters(int num_sms) {
   static thread_local int resident = 0;
   if (resident == 0) {
-    if (cudaFuncSetAttribute(ca_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if (cudaFuncSetAttribute(ca_pair_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              PairSmem::kBytes) != cudaSuccess) {
       cudaGetLastError();
       return std::max(1, num_sms / 2);
@@ -581,7 +794,7 @@ int ca_pair_clusters(int num_sms) {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, ca_pair_kernel, &cfg) != cudaSuccess || n < 1) {
+    if (cudaOccupancyMaxActiveClusters(&n, ca_pair_kernel<false>, &cfg) != cudaSuccess || n < 1) {
       cudaGetLastError();
       n = num_sms / 2;
     }
@@ -591,20 +804,22 @@ int ca_pair_clusters(int num_sms) {
 }
 
 cudaError_t launch_ca_pair(const Operand2D& Q, const Operand2D& K, const Operand2D& XT,
-                           const FlashParams& f, int num_sms, cudaStream_t stream) {
+                           const FlashParams& f, int num_sms, cudaStream_t stream,
+                           bool one_pass) {
   using S = PairSmem;
   if (f.D <= 0 || f.D % kBK != 0 || f.t <= 0 || f.N <= 0 || f.Np % kBK != 0 || f.Np < f.N ||
-      f.nunits <= 0)
+      f.nunits <= 0 || (one_pass && (f.cand_key == nullptr || f.cand_c == nullptr)))
     return cudaErrorInvalidValue;
   CUtensorMap tq, tk, tx;
   if (!make_tmap(&tq, Q, kBM) || !make_tmap(&tk, K, kPairKeys) || !make_tmap(&tx, XT, 128))
     return cudaErrorInvalidValue;
-  static thread_local bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(ca_pair_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, S::kBytes);
+  auto kern = one_pass ? ca_pair_kernel<true> : ca_pair_kernel<false>;
+  static thread_local bool attr_set[2] = {false, false};
+  if (!attr_set[one_pass]) {
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::kBytes);
     if (e != cudaSuccess) return e;
-    attr_set = true;
+    attr_set[one_pass] = true;
   }
   cudaLaunchConfig_t cfg = {};
   cfg.blockDim = dim3(kFlashThreads, 1, 1);
@@ -619,7 +834,7 @@ cudaError_t launch_ca_pair(const Operand2D& Q, const Operand2D& K, const Operand
   cfg.numAttrs = 1;
   const int clusters = std::max(1, std::min(f.nunits, ca_pair_clusters(num_sms)));
   cfg.gridDim = dim3(2 * clusters, 1, 1);
-  return cudaLaunchKernelEx(&cfg, ca_pair_kernel, tq, tk, tx, f);
+  return cudaLaunchKernelEx(&cfg, kern, tq, tk, tx, f);
 }
 
 }  // namespace still

@@ -359,3 +359,12 @@ STILL_DEV void bulk_copy_to_cluster(uint32_t dst_cluster, const void* src, uint3
       "r"(smem_u32(src)), "r"(bytes), "r"(mbar_cluster)
       : "memory");
 }
+
+// Prefetch of one box of a tiled tensor into L2 (no shared memory, no completion to wait for).
+// x (innermost coordinate) * 2 bytes must be a multiple of 16: callers pass multiples of 64.
+STILL_DEV void tma_prefetch_l2_2d(const CUtensorMap* m, int32_t x, int32_t y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                   reinterpret_cast<uint64_t>(m)),
+               "r"(x), "r"(y)
+               : "memory");
+}

@@ -327,7 +327,7 @@ struct Plan {
   size_t oX, oXT, oCoarse, oOmega, oGD, oHrot, oPX, oZ1, oA1, oCat, oZ2, oA2, oG, oZ3;
   size_t oCA, oSA;
   size_t ca_unit_bytes, sa_unit_bytes;
-  size_t kb_b, kss_b, q_b, S_b, P_b, O_b, qt_b;  // per CA unit
+  size_t kb_b, kss_b, q_b, S_b, P_b, O_b, qt_b, cand_b;  // per CA unit
   bool lazy_q;
   size_t oZn;
   size_t qk_b, sss_b, vT_b, Ssa_b, Psa_b;        // per SA bank (KV-head)
@@ -338,12 +338,24 @@ struct Plan {
 size_t a256(size_t x) { return (x + 255) & ~size_t(255); }
 
 // The self-attention value path (probabilities, values, head outputs) and the FFN run in bf16
-// hi | lo rather than plain bf16 in layers of more than one block (the next block's queries
-// amplify their rounding) and in compactors of width d_l >= 2048. There the self-attention
-// output, whose logits d_l cos(q, k) are the sharpest, dominates the latent state: emulating
-// plain-bf16 probabilities, values and FFN activations on the Gemma-shaped compactor moves C_k
-// from the output-rounding floor of 0.009 to 0.015 x RMS, against 0.009 in hi | lo.
-bool value_hilo(const still_layer_config& c) { return c.n_blocks > 1 || c.d_latent >= 2048; }
+// hi | lo rather than plain bf16. The self-attention logits d_l cos(q, k) over t latents are
+// sharp enough that the rounding of its output moves the next sublayers by far more than its
+// own size, and more so as d_l and t grow: emulating plain-bf16 probabilities, values and FFN
+// activations on the Gemma-shaped compactor moves C_k from the output-rounding floor of 0.009
+// to 0.015 x RMS (0.009 in hi | lo), and on the iterative Qwen-8B-shaped workload the plain
+// path reaches 0.020 once t passes 4000. In a layer of two blocks the next block's queries
+// amplify it further.
+bool value_hilo(const still_layer_config&) { return true; }
+
+// The cross-attention scores of a one-block layer of head dim 256 take one fp16 MMA pass
+// (q_hi . k_hi) instead of three split-bf16 passes, and a repair kernel then recomputes the
+// logits of each row's heaviest keys from the fp16 hi | lo operands (about 22 bits). At
+// d_l >= 512 the rows put nearly all their weight on a few keys: CPU emulation at the Gemma
+// shape gives a cross-attention output error of 5.1e-4 with the 8 heaviest keys of a row
+// repaired and 1.5e-5 with 16, against 3.7e-3 for the three-pass split.
+bool one_pass_scores(const still_layer_config& c) {
+  return c.n_blocks == 1 && c.head_dim == 256 && c.d_latent >= 512 && c.d_latent <= 2048;
+}
 
 bool make_plan(const still_layer_config& c, bool lazy_q, int Kp, int64_t N, int t, double pmin,
                double pmax, size_t limit, Plan& P) {
@@ -397,9 +409,12 @@ bool make_plan(const still_layer_config& c, bool lazy_q, int Kp, int64_t N, int 
   P.S_b = 0;
   P.P_b = 0;
   P.O_b = 0;
+  P.cand_b = 0;
   if (P.flash) {
     P.P_b = a256(T * 8) * kMaxFlashSplit;          // per-split row statistics (m, l)
     P.O_b = a256(T * 2 * d * 4) * kMaxFlashSplit;  // per-split unnormalised O
+    // one-pass scores: repair candidates (key, c) per split, row and list
+    if (one_pass_scores(c)) P.cand_b = 2 * a256(T * kTopLists * kTopK * 4) * kMaxFlashSplit;
   }
   if (P.split_ca) {
     P.S_b = a256(T * P.ldS * 4);
@@ -408,7 +423,7 @@ bool make_plan(const still_layer_config& c, bool lazy_q, int Kp, int64_t N, int 
   }
   // lazy q^: fp32 q~ of the unit and its sum-of-squares partials + inverse norms
   P.qt_b = lazy_q ? a256(T * D * 4) + a256(T * 4 * (2 * (D / 256) + 1)) : 0;
-  P.ca_unit_bytes = P.kb_b + P.kss_b + P.q_b + P.S_b + P.P_b + P.O_b + P.qt_b;
+  P.ca_unit_bytes = P.kb_b + P.kss_b + P.q_b + P.S_b + P.P_b + P.O_b + P.qt_b + P.cand_b;
   P.qk_b = a256(2 * n * T * 2 * D * 2);
   P.sss_b = a256(2 * n * T * 4 * (2 * (D / 256) + 1));
   P.vT_b = a256(n * D * P.tp * 2 * hl);
@@ -591,6 +606,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
   // self-attention q, k, v, P and head outputs) are fp16 hi | lo rather than bf16 hi | lo.
   const bool exact = !last;
   const bool vexact = exact || L.f16 || value_hilo(c);
+  const bool tk = !exact && P.flash && !L.fold && one_pass_scores(c);  // one-pass scores
   const bool f16v = exact && L.f16 && P.flash;
   const int vfmt = f16v ? 0 : 1;
   const int32_t vkind = f16v ? OUT_HILO16 : OUT_HILO;
@@ -638,6 +654,9 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     g += P.P_b * nbl;
     float* O = reinterpret_cast<float*>(g);
     g += P.O_b * nbl;
+    int* cand_key = reinterpret_cast<int*>(g);  // one-pass scores: repair candidates
+    float* cand_c = reinterpret_cast<float*>(g + P.cand_b / 2 * nbl);
+    g += P.cand_b * nbl;
     // lazy q^: q~ [nbl][t][D] fp32 and its sum-of-squares partials / inverse norms
     float* qt = reinterpret_cast<float*>(g);
     float* qss = reinterpret_cast<float*>(g + a256((size_t)t * D * 4) * nbl);
@@ -709,7 +728,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
         e.D = D;
         e.nheads = ni;
         e.ncoarse = P.G;
-        e.fp16 = exact ? 1 : 0;  // k as fp16 hi / lo where the block feeds another
+        e.fp16 = exact || tk ? 1 : 0;  // k as fp16 hi / lo (block feeding another; one pass)
         e.Ntok = N;
       };
       const StoreView3D kv = store_view(kb, 2, 2 * D, N, nbl, 2 * D, N * 2 * D, 16, false);
@@ -729,13 +748,14 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     // A block that feeds another forms q and k as fp16 hi / lo (about 22 bits; bf16 hi / lo
     // keeps 16): its logits steer the next block's queries. q is unit-norm, so it is scaled by
     // a power of two near sqrt(D) into the fp16 normal range and the logit scale divided by it.
-    const float qscale = exact ? std::exp2(std::round(0.5 * std::log2((double)D))) : 1.f;
+    const float qscale =
+        exact || tk ? std::exp2(std::round(0.5 * std::log2((double)D))) : 1.f;
     KLAUNCH(STILL_K_NORMS, launch_inv_norms(kss, (int64_t)nbl * N, kparts, N, c.l2_eps,
                                             scale / qscale, kinv, s));
     if (!L.fold)
       KLAUNCH(STILL_K_QROPE, launch_q_rope(qsrc, q_tmax, q_b0, nbl, t, D, qstart, qstep,
-                                           L.omega_c, c.compactor_rope, qhl, exact ? 1 : 0,
-                                           qscale, s));
+                                           L.omega_c, c.compactor_rope, qhl,
+                                           exact || tk ? 1 : 0, qscale, s));
     if (P.flash) {
       // S, the online softmax and P X in one kernel; per-split partials merged in order.
       float2* fst = stp;  // [nsplit][nbl * t] (the statistics region of this path)
@@ -760,6 +780,10 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       fp.O = O;
       fp.stats = fst;
       fp.err = ctx->err;
+      if (tk) {
+        fp.cand_key = cand_key;
+        fp.cand_c = cand_c;
+      }
       Operand2D qop = op(qhl, (int64_t)nbl * t, 2 * D);
       Operand2D kop = op(kb, (int64_t)nbl * N, 2 * D);
       if (L.fold) {  // q := u (precomputed, t_max rows per (h, i)), k := x~ shared per KV-head
@@ -776,7 +800,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       ctx->prof.begin(STILL_K_CA_FUSED, s);
       cudaError_t r =
           d == 256 ? (exact ? cudaErrorInvalidValue  // two-block layers at d = 256 are refused
-                            : launch_ca_pair(qop, kop, xop, fp, ctx->nsm, s))
+                            : launch_ca_pair(qop, kop, xop, fp, ctx->nsm, s, tk))
           : exact  ? (d == 64 ? launch_ca_flash<128, true>(qop, kop, xop, fp, ctx->nsm, s)
                               : launch_ca_flash<256, true>(qop, kop, xop, fp, ctx->nsm, s))
                    : (d == 64 ? launch_ca_flash<128>(qop, kop, xop, fp, ctx->nsm, s)
@@ -784,6 +808,28 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       ctx->prof.end(STILL_K_CA_FUSED, s);
       if (r == cudaErrorInvalidValue) return STILL_ERR_INVALID_ARG;
       if (r != cudaSuccess) return STILL_ERR_CUDA;
+      if (tk) {  // exact logits of each row's heaviest keys, before the split merge
+        TopkRepairParams rp;
+        rp.q = reinterpret_cast<const __half*>(qhl);
+        rp.k = reinterpret_cast<const __half*>(kb);
+        rp.kinv = kinv;
+        rp.X = X + (size_t)h0 * N * 3 * d;
+        rp.O = O;
+        rp.stats = fst;
+        rp.cand_key = cand_key;
+        rp.cand_c = cand_c;
+        rp.D = D;
+        rp.d = d;
+        rp.t = t;
+        rp.N = (int)N;
+        rp.nb = nbl;
+        rp.nsplit = fp.nsplit;
+        rp.bdiv = ni;
+        rp.nlists = kTopLists;
+        rp.tiles_k = fp.tiles_k;
+        rp.keys_per_tile = kFlashKeys;
+        KLAUNCH(STILL_K_REPAIR, launch_ca_topk_repair(rp, 2 * d, s));
+      }
       KLAUNCH(STILL_K_PXSPLIT, launch_ca_merge(O, fst, fp.nsplit, b0, nbl, n, t, 2 * d,
                                                f16v ? 1 : 0, PX, s));
       b0 += nbl;
@@ -1993,7 +2039,7 @@ const char* still_kernel_class_name(int32_t cls) {
   static const char* names[STILL_K_COUNT] = {
       "strip", "rope_tables", "keyproj", "q_rope", "scores", "softmax", "px", "px_split",
       "vo", "rmsnorm", "sa_proj", "sa_v", "sa_scores", "sa_softmax", "sa_pv", "sa_out",
-      "ffn1", "ffn2", "heads", "norms", "load", "ca_fused", "beta", "decode"};
+      "ffn1", "ffn2", "heads", "norms", "load", "ca_fused", "beta", "decode", "repair"};
   return cls >= 0 && cls < STILL_K_COUNT ? names[cls] : "unknown";
 }
 

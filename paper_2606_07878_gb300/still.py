@@ -38,7 +38,7 @@ NOALLOC_SCRATCH_MIB = 64  # STILL_NOALLOC_SCRATCH_MIB in include/still.h
 KERNEL_CLASSES = ["strip", "rope_tables", "keyproj", "q_rope", "scores", "softmax", "px",
                   "px_split", "vo", "rmsnorm", "sa_proj", "sa_v", "sa_scores", "sa_softmax",
                   "sa_pv", "sa_out", "ffn1", "ffn2", "heads", "norms", "load", "ca_fused",
-                  "beta", "decode"]
+                  "beta", "decode", "repair"]
 
 
 class StillError(RuntimeError):

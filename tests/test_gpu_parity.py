@@ -86,6 +86,31 @@ def test_other_head_dims(over):
         r.close()
 
 
+@pytest.mark.parametrize("logit_scale", [0.0, 1.0 / np.sqrt(512.0)])
+def test_one_pass_scores_with_repair(logit_scale):
+    """Head dim 256 at d_l = 512: one fp16 pass for the cross-attention scores, then the exact
+    logits of each row's heaviest keys. With the d_l logit scale the rows are concentrated and
+    the candidates carry the repair; with 1/sqrt(d_l) they are nearly uniform, so every split
+    falls back to the exact recomputation over its keys."""
+    wl = _small(d=256, D=512, n=2, F=512, H=2, N=1500)
+    t = 100
+    over = dict(logit_scale=logit_scale) if logit_scale else {}
+    r = Runner(wl, t, cfg_over=over)
+    try:
+        K, V = synth.gen_kv(wl, 0, device=DEV)
+        still.still_profile_enable(r.ctx, True)
+        still.still_profile_enable_classes(r.ctx, [])
+        Ck, Cv, _ = r.layer(0, K, V, t)
+        assert still.still_profile_read(r.ctx)["repair"][0] > 0
+        still.still_profile_enable(r.ctx, False)
+        rk, rv, _, _ = oracle_layer(wl, r.W[0], K, V, t,
+                                    cfg_over=dict(logit_scale=logit_scale) if logit_scale else None)
+        assert_parity(rk, synth.bf16_to_f64(Ck), f"C_k scale {logit_scale}")
+        assert_parity(rv, synth.bf16_to_f64(Cv), f"C_v scale {logit_scale}")
+    finally:
+        r.close()
+
+
 def test_final_norm():
     wl = _small(N=300)
     t = 30
