@@ -426,9 +426,9 @@ typedef enum {
   STILL_K_TABLES,       /* compactor-RoPE angle table                       */
   STILL_K_KEYPROJ,      /* k = RoPE_c(X W_K + b_K) (2-pass tcgen05 GEMM)    */
   STILL_K_QROPE,        /* q = RoPE_c(q^) at the latent query positions     */
-  STILL_K_SCORES,       /* S = d_l q.k / |k| (3-pass tcgen05 GEMM)          */
-  STILL_K_SOFTMAX,      /* cross-attention row softmax                      */
-  STILL_K_PX,           /* O = P X (2-pass tcgen05 GEMM, split-K)           */
+  STILL_K_SCORES,       /* (unused: the scores are fused into STILL_K_CA_FUSED) */
+  STILL_K_SOFTMAX,      /* (unused: the softmax is fused)                   */
+  STILL_K_PX,           /* (unused: P X is fused)                           */
   STILL_K_PXSPLIT,      /* key-split merge of O, O -> hi/lo                 */
   STILL_K_VO,           /* Z' = Z + O (W_V W_O) (3-pass tcgen05 GEMM)       */
   STILL_K_NORM,         /* RMSNorm                                          */

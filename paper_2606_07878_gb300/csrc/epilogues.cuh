@@ -139,10 +139,6 @@ struct EpiAffine {
   // launcher (boxes of 32 x 32 fp32, 128-byte swizzled staging); rows / columns past the view
   // are clipped by the copy engine.
   int32_t tma_f32 = 0;
-  // Row-softmax partials of the (scaled) output: per (batch, row, column tile, part) the max m
-  // and sum of exp(v - m) over valid columns, at stat_out[(b * M + r) * stat_slots + 2 tn + part].
-  float2* stat_out = nullptr;
-  int32_t stat_slots = 0;
   int32_t tile_cols_ = 256;  // the tile width BN, set by the launcher
 
   // The residual rows of this warp's columns are pulled into L2 while the main loop runs.
@@ -166,7 +162,6 @@ struct EpiAffine {
     float rscale = alpha;
     if (row_scale != nullptr && rvalid) rscale *= row_scale[rsm.at(tc.b, r, 0)];
     float ss = 0.f;
-    float st_m = -INFINITY, st_l = 0.f;
     for (int cc = 32 * half; cc < tile_cols_; cc += 64) {
       float v[32];
       tmem_ld32(taddr + (uint32_t)cc, v);
@@ -224,19 +219,6 @@ struct EpiAffine {
         for (int e = 0; e < 32; ++e)
           if (e < nv) v[e] += bias[c0 + e];
       }
-      if (stat_out != nullptr) {
-        float mc = -INFINITY;
-#pragma unroll
-        for (int e = 0; e < 32; ++e)
-          if (e < nv) mc = fmaxf(mc, v[e]);
-        const float mn = fmaxf(st_m, mc);
-        float l = st_l * exp2f((st_m - mn) * 1.4426950408889634f);
-#pragma unroll
-        for (int e = 0; e < 32; ++e)
-          if (e < nv) l += exp2f((v[e] - mn) * 1.4426950408889634f);
-        st_m = mn;
-        st_l = l;
-      }
       if (sumsq != nullptr) {
 #pragma unroll
         for (int e = 0; e < 32; ++e)
@@ -268,8 +250,6 @@ struct EpiAffine {
       else
         store32(p, tc.b, r, c0, v, tc.split, rvalid, stage);
     }
-    if (stat_out != nullptr && rvalid)
-      stat_out[((int64_t)tc.b * p.M + r) * stat_slots + 2 * tc.tn + half] = make_float2(st_m, st_l);
     if (sumsq != nullptr && rvalid) {
       const int c_tile = tc.tn * tile_cols_;
       const int slot = ((c_tile % ss_seg) / tile_cols_) * 2 + half;

@@ -437,21 +437,6 @@ __global__ void __launch_bounds__(256) softmax_reg_kernel(const float* __restric
   }
 }
 
-// Row softmax statistics from per-tile partials (m_p, l_p = sum exp(v - m_p)):
-// out[row] = (M * log2 e, 1 / L), M = max_p m_p, L = sum_p l_p exp(m_p - M), fixed order.
-__global__ void row_stats_kernel(const float2* __restrict__ parts, int64_t rows, int slots,
-                                 float2* __restrict__ out) {
-  const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (r >= rows) return;
-  const float2* p = parts + r * slots;
-  float M = -INFINITY;
-  for (int k = 0; k < slots; ++k) M = fmaxf(M, p[k].x);
-  float L = 0.f;
-  for (int k = 0; k < slots; ++k)
-    if (p[k].x != -INFINITY) L += p[k].y * exp2f((p[k].x - M) * kLog2e);
-  out[r] = make_float2(M * kLog2e, 1.f / L);
-}
-
 // Failure-detection self-test: waits on an mbarrier that nothing arrives on, with a short
 // bound. The wait expires, the kernel records DEV_WAIT_TIMEOUT in the error record and returns.
 __global__ void wait_timeout_selftest_kernel(int* err, unsigned long long limit_ns) {
@@ -473,26 +458,6 @@ __global__ void wait_timeout_selftest_kernel(int* err, unsigned long long limit_
 __global__ void omega_kernel(double* out, int half, int width, double base) {
   const int m = blockIdx.x * blockDim.x + threadIdx.x;
   if (m < half) out[m] = pow(base, -2.0 * m / width);
-}
-
-__global__ void px_to_hilo_kernel(const float* __restrict__ O, int nsplit, int64_t split_stride,
-                                  int b0, int nb, int n, int t, int d2,
-                                  __nv_bfloat16* __restrict__ PX) {
-  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  const int64_t total = (int64_t)nb * t * d2;
-  if (idx >= total) return;
-  float o = O[idx];
-  for (int k = 1; k < nsplit; ++k) o += O[k * split_stride + idx];  // fixed order
-  const int f = (int)(idx % d2);
-  const int64_t rj = idx / d2;
-  const int j = (int)(rj % t), bb = (int)(rj / t);
-  const int b = b0 + bb, h = b / n, i = b % n;
-  const int64_t ld = 2 * (int64_t)n * d2;
-  __nv_bfloat16 hi, lo;
-  split_hilo(o, hi, lo);
-  __nv_bfloat16* row = PX + ((int64_t)h * t + j) * ld;
-  row[i * d2 + f] = hi;
-  row[(int64_t)n * d2 + i * d2 + f] = lo;
 }
 
 // Key-split merge of the fused cross-attention. Split s holds, per row, the unnormalised
@@ -1107,12 +1072,6 @@ static bool softmax_reg(const float* S, int64_t rows, int64_t ncols, int64_t ldS
   return true;
 }
 
-cudaError_t launch_row_stats(const float2* parts, int64_t rows, int slots, float2* out,
-                             cudaStream_t s) {
-  row_stats_kernel<<<blocks_for(rows, 256), 256, 0, s>>>(parts, rows, slots, out);
-  return cudaGetLastError();
-}
-
 cudaError_t launch_wait_timeout_selftest(int* err, unsigned long long limit_ns, cudaStream_t s) {
   wait_timeout_selftest_kernel<<<1, 32, 0, s>>>(err, limit_ns);
   return cudaGetLastError();
@@ -1141,14 +1100,6 @@ cudaError_t launch_softmax(const float* S, int64_t rows, int64_t ncols, int64_t 
   else
     softmax_kernel<__nv_bfloat16><<<(unsigned)rows, 256, 0, s>>>(
         S, ncols, ldS, static_cast<__nv_bfloat16*>(P), ldP);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_px_to_hilo(const float* O, int nsplit, int64_t split_stride, int b0, int nb,
-                              int n, int t, int d2, __nv_bfloat16* PX, cudaStream_t s) {
-  const int64_t total = (int64_t)nb * t * d2;
-  px_to_hilo_kernel<<<blocks_for(total, 256), 256, 0, s>>>(O, nsplit, split_stride, b0, nb, n,
-                                                           t, d2, PX);
   return cudaGetLastError();
 }
 

@@ -89,11 +89,6 @@ cudaError_t launch_q_rope(const float* qhat, int t_max, int b0, int nb, int t, i
                           double qstart, double qstep, const double* omega_c, int use_rope,
                           __nv_bfloat16* qhl, int fp16, float qscale, cudaStream_t s);
 
-// Row softmax statistics from the scores epilogue's per-tile partials (max, sum of exp):
-// out[row] = (M * log2 e, 1 / L) with M the row max and L the sum of exp(s - M).
-cudaError_t launch_row_stats(const float2* parts, int64_t rows, int slots, float2* out,
-                             cudaStream_t s);
-
 // One-block kernel whose bounded wait on an mbarrier can only expire (failure-detection test).
 cudaError_t launch_wait_timeout_selftest(int* err, unsigned long long limit_ns, cudaStream_t s);
 
@@ -106,15 +101,10 @@ cudaError_t launch_omega(double* out, int half, int width, double base, cudaStre
 cudaError_t launch_softmax(const float* S, int64_t rows, int64_t ncols, int64_t ldS, void* P,
                            int64_t ldP, int out_fp16, cudaStream_t s);
 
-// Cross-attention head outputs O [nsplit][nb][t][2d] fp32 split-K partials (batch b = b0 +
-// local), summed in split order -> hi/lo bf16 rows of PXcat [H*t][2 * n * 2d]: row h*t + j,
-// columns i*2d + f (hi) and n*2d + i*2d + f (lo).
-cudaError_t launch_px_to_hilo(const float* O, int nsplit, int64_t split_stride, int b0, int nb,
-                              int n, int t, int d2, __nv_bfloat16* PX, cudaStream_t s);
-
-// Key-split merge of the fused cross-attention: O [nsplit][nb][t][2d] unnormalised partials with
-// stats [nsplit][nb][t] = (max in log2 units, sum) -> normalised hi/lo bf16 rows of PXcat
-// (layout as launch_px_to_hilo; f16: fp16 hi | lo instead). Splits are combined in a fixed order.
+// Key-split merge of the fused cross-attention: O [nsplit][nb][t][2d] unnormalised partials (batch
+// b = b0 + local) with stats [nsplit][nb][t] = (max in log2 units, sum) -> normalised hi/lo bf16
+// rows of PXcat [H*t][2 * n * 2d]: row h*t + j, columns i*2d + f (hi) and n*2d + i*2d + f (lo)
+// (f16: fp16 hi | lo instead). Splits are combined in a fixed order.
 cudaError_t launch_ca_merge(const float* O, const float2* stats, int nsplit, int b0, int nb,
                             int n, int t, int d2, int f16, __nv_bfloat16* PX, cudaStream_t s);
 

@@ -7,9 +7,10 @@
 //   per group of (KV-head h, cross head i):
 //     keyproj  k~ = X W_K,i + b_K,i -> RoPE_c -> hi/lo, |k~|^2          (2-pass GEMM)
 //     qrope    q = RoPE_c(q^_i, p_j) -> hi/lo                         (q^ precomputed at load)
-//     scores   S = d_l * q.k / |k~|                                   (3-pass GEMM)
-//     softmax  P = softmax_rows(S) (fp16)
-//     PX       O_i = P X                                             (2-pass GEMM, split-K)
+//     ca_fused S = d_l * q.k / |k~|, online softmax, O_i += P X per key split, in one kernel
+//              (one CTA per unit for head dim <= 128, a cluster of two for 256)
+//     repair   (head dim 256) exact logits of each row's heaviest keys
+//     merge    the key splits of O_i and (m, l), in a fixed order -> hi/lo
 //   VO         Z' = Z + [O_1..O_n] (W_V,i W_O,i)_i                     (3-pass GEMM)
 //   SA         Z'' = Z' + Concat_i softmax(d_l q^ k^T) v . S_O          (per KV-head bank)
 //   FFN        Z''' = Z'' + GELU(RMSNorm(Z'') W_1) W_2
@@ -23,7 +24,6 @@
 #include "../../include/still.h"
 #include "gemm_host.cuh"
 #include "kernels.cuh"
-#include "px_fused.cuh"
 #include "ca_flash.cuh"
 
 using namespace still;
@@ -186,7 +186,6 @@ namespace {
 
 inline int64_t rup(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
 
-constexpr int kMaxSplit = 8;  // split-K factor cap (partials are reduced in a fixed order)
 constexpr int kMaxFlashSplit = 16;  // key-split cap of the fused cross-attention
 
 void free_layer(LayerW& L) {
@@ -299,13 +298,6 @@ StoreView3D store_view(void* ptr, int elem_bytes, int64_t nx, int64_t ny, int64_
     if (e_ != cudaSuccess) return STILL_ERR_CUDA; \
   } while (0)
 
-// Split-K factor that brings a GEMM with few output tiles up to about two waves.
-int auto_split(int64_t tiles, int iters, int nsm) {
-  if (tiles >= nsm) return 1;
-  int s = (int)((2 * nsm + tiles - 1) / tiles);
-  return std::max(1, std::min(s, iters / 4));
-}
-
 #define TRY(x)                          \
   do {                                  \
     still_status st_ = (x);             \
@@ -316,10 +308,9 @@ int auto_split(int64_t tiles, int iters, int nsm) {
 
 struct Plan {
   int H, d, D, n, F, t;
-  int64_t N, Np, ldS, tp, ldt;
+  int64_t N, Np, tp, ldt;
   int G;
   bool flash;     // fused cross-attention kernel (2d of 128 or 256) for the last block
-  bool split_ca;  // some block takes the scores + P X kernels
   int ca_units;   // (h, i) pairs per cross-attention group
   int sa_heads;   // KV-heads per self-attention group
   int sa_sub;     // self heads per scores / softmax / P.v pass (n unless one bank is too big)
@@ -327,7 +318,7 @@ struct Plan {
   size_t oX, oXT, oCoarse, oOmega, oGD, oHrot, oPX, oZ1, oA1, oCat, oZ2, oA2, oG, oZ3;
   size_t oCA, oSA;
   size_t ca_unit_bytes, sa_unit_bytes;
-  size_t kb_b, kss_b, q_b, S_b, P_b, O_b, qt_b, cand_b;  // per CA unit
+  size_t kb_b, kss_b, q_b, P_b, O_b, qt_b, cand_b;  // per CA unit
   bool lazy_q;
   size_t oZn;
   size_t qk_b, sss_b, vT_b, Ssa_b, Psa_b;        // per SA bank (KV-head)
@@ -347,12 +338,16 @@ size_t a256(size_t x) { return (x + 255) & ~size_t(255); }
 // amplify it further.
 bool value_hilo(const still_layer_config&) { return true; }
 
-// The cross-attention scores of a one-block layer of head dim 256 take one fp16 MMA pass
-// (q_hi . k_hi) instead of three split-bf16 passes, and a repair kernel then recomputes the
-// logits of each row's heaviest keys from the fp16 hi | lo operands (about 22 bits). At
-// d_l >= 512 the rows put nearly all their weight on a few keys: CPU emulation at the Gemma
-// shape gives a cross-attention output error of 5.1e-4 with the 8 heaviest keys of a row
-// repaired and 1.5e-5 with 16, against 3.7e-3 for the three-pass split.
+// The cross-attention scores of a one-block layer of head dim 256 (the kernel on clusters of
+// two CTAs) take one fp16 MMA pass (q_hi . k_hi) instead of three split-bf16 passes, and a
+// repair kernel then recomputes the logits of each row's heaviest keys from the fp16 hi | lo
+// operands (about 22 bits). At d_l >= 512 the rows put nearly all their weight on a few
+// keys: CPU emulation of the C_k error from the cross-attention logits alone, with the k
+// heaviest keys of every row repaired, gives 5.1e-4 (k = 8) and 1.5e-5 (k = 16) on the Gemma
+// shape at 16k tokens, against 3.7e-3 for the three-pass split. Head dims 64 and 128 keep the
+// split: there one CTA runs the softmax of every tile, a one-pass S tile takes no longer than
+// that softmax, and the kernel measured slower with one pass (the Qwen-7B-shaped stack went
+// from 76 to 109 ms, with 24 ms of repair).
 bool one_pass_scores(const still_layer_config& c) {
   return c.n_blocks == 1 && c.head_dim == 256 && c.d_latent >= 512 && c.d_latent <= 2048;
 }
@@ -367,7 +362,6 @@ bool make_plan(const still_layer_config& c, bool lazy_q, int Kp, int64_t N, int 
   P.t = t;
   P.N = N;
   P.Np = rup(N, 64);
-  P.ldS = rup(N, 4);
   P.tp = rup(t, 64);
   P.ldt = rup(t, 4);
   P.G = (int)std::floor((pmax - pmin) / kPosGrain) + 2;
@@ -405,25 +399,14 @@ bool make_plan(const still_layer_config& c, bool lazy_q, int Kp, int64_t N, int 
   // The fused kernel serves every block (a block that feeds another takes its split-precision
   // variant); 2d = 512 runs it on clusters of two CTAs that split the O columns.
   P.flash = d == 64 || d == 128 || d == 256;
-  P.split_ca = !P.flash;
-  P.S_b = 0;
-  P.P_b = 0;
-  P.O_b = 0;
-  P.cand_b = 0;
-  if (P.flash) {
-    P.P_b = a256(T * 8) * kMaxFlashSplit;          // per-split row statistics (m, l)
-    P.O_b = a256(T * 2 * d * 4) * kMaxFlashSplit;  // per-split unnormalised O
-    // one-pass scores: repair candidates (key, c) per split, row and list
-    if (one_pass_scores(c)) P.cand_b = 2 * a256(T * kTopLists * kTopK * 4) * kMaxFlashSplit;
-  }
-  if (P.split_ca) {
-    P.S_b = a256(T * P.ldS * 4);
-    P.P_b = std::max(P.P_b, a256(T * 8 * (2 * ((N + 255) / 256) + 1)));  // softmax partials
-    P.O_b = std::max(P.O_b, a256(T * 2 * d * 4) * kMaxSplit);  // split-K partials of P X
-  }
+  P.P_b = a256(T * 8) * kMaxFlashSplit;          // per-split row statistics (m, l)
+  P.O_b = a256(T * 2 * d * 4) * kMaxFlashSplit;  // per-split unnormalised O
+  // one-pass scores: repair candidates (key, c) per split, row and list
+  P.cand_b = one_pass_scores(c) && Kp == 0 ? 2 * a256(T * kTopLists * kTopK * 4) * kMaxFlashSplit
+                                           : 0;
   // lazy q^: fp32 q~ of the unit and its sum-of-squares partials + inverse norms
   P.qt_b = lazy_q ? a256(T * D * 4) + a256(T * 4 * (2 * (D / 256) + 1)) : 0;
-  P.ca_unit_bytes = P.kb_b + P.kss_b + P.q_b + P.S_b + P.P_b + P.O_b + P.qt_b + P.cand_b;
+  P.ca_unit_bytes = P.kb_b + P.kss_b + P.q_b + P.P_b + P.O_b + P.qt_b + P.cand_b;
   P.qk_b = a256(2 * n * T * 2 * D * 2);
   P.sss_b = a256(2 * n * T * 4 * (2 * (D / 256) + 1));
   P.vT_b = a256(n * D * P.tp * 2 * hl);
@@ -646,11 +629,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
     g += P.kss_b * nbl;
     bf16* qhl = reinterpret_cast<bf16*>(g);
     g += P.q_b * nbl;
-    float* S = reinterpret_cast<float*>(g);
-    g += P.S_b * nbl;
-    const int stat_slots = 2 * (int)((N + 255) / 256);
-    float2* stp = reinterpret_cast<float2*>(g);                      // [nbl * t][stat_slots]
-    float2* rstat = stp + (size_t)nbl * t * stat_slots;               // [nbl * t]
+    float2* fst = reinterpret_cast<float2*>(g);  // [nsplit][nbl * t]: per-split (m, l)
     g += P.P_b * nbl;
     float* O = reinterpret_cast<float*>(g);
     g += P.O_b * nbl;
@@ -756,9 +735,8 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       KLAUNCH(STILL_K_QROPE, launch_q_rope(qsrc, q_tmax, q_b0, nbl, t, D, qstart, qstep,
                                            L.omega_c, c.compactor_rope, qhl,
                                            exact || tk ? 1 : 0, qscale, s));
-    if (P.flash) {
+    {
       // S, the online softmax and P X in one kernel; per-split partials merged in order.
-      float2* fst = stp;  // [nsplit][nbl * t] (the statistics region of this path)
       FlashParams fp;
       fp.t = t;
       fp.N = (int)N;
@@ -833,80 +811,7 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       KLAUNCH(STILL_K_PXSPLIT, launch_ca_merge(O, fst, fp.nsplit, b0, nbl, n, t, 2 * d,
                                                f16v ? 1 : 0, PX, s));
       b0 += nbl;
-      continue;
     }
-    {  // S = scale * q.k / |k~|
-      GemmParams p = gp(t, (int)N, nbl, 1);
-      p.a_r1 = t;
-      p.b_r1 = N;
-      add_pass(p, 0, 0, 0, 0, D);
-      add_pass(p, 0, D, 0, 0, D);
-      add_pass(p, D, 0, 0, 0, D);
-      EpiAffine e;
-      e.kind = OUT_F32;
-      e.out = S;
-      e.om.b1 = (int64_t)t * P.ldS;
-      e.om.r0 = P.ldS;
-      e.om.c0 = 1;
-      e.col_scale = kinv;
-      e.csm.b1 = N;
-      e.csm.c0 = 1;
-      e.vec_ok = 1;
-      e.tma_f32 = 1;
-      e.stat_out = stp;
-      e.stat_slots = stat_slots;
-      const StoreView3D sv = store_view(S, 4, N, t, nbl, P.ldS, (int64_t)t * P.ldS, 32, true);
-      TRY(run_gemm256<STILL_K_SCORES>(ctx, op(qhl, (int64_t)nbl * t, 2 * D),
-                                      op(kb, (int64_t)nbl * N, 2 * D), p, e, exact ? 0 : 1, s, &sv));
-    }
-    KLAUNCH(STILL_K_SOFTMAX, launch_row_stats(stp, (int64_t)nbl * t, stat_slots, rstat, s));
-    int px_split = 1;
-    const int64_t px_stride = (int64_t)nbl * t * 2 * d;
-    {  // O = softmax(S) X: probabilities formed on the fly (fp16), X hi + key-half lo passes
-      GemmParams p = gp(t, 2 * d, nbl, ni);
-      add_pass(p, 0, 0, 0, 0, (int)Np);
-      const int bn = 2 * d <= 128 ? 128 : 256;
-      const int64_t tiles = (int64_t)((t + 127) / 128) * ((2 * d + bn - 1) / bn) * nbl;
-      p.ksplit = std::min(auto_split(tiles, (int)(Np / 64), ctx->nsm), kMaxSplit);
-      p.ksplit = std::min(p.ksplit, (int)(Np / 64));
-      px_split = p.ksplit;
-      p.err = ctx->err;
-      PxParams px;
-      px.S = S;
-      px.stats = rstat;
-      px.ldS = P.ldS;
-      px.t = t;
-      px.N = (int)N;
-      px.xbase_row = h0 * 2 * d;
-      px.d2 = 2 * d;
-      px.lo_rows = d;
-      px.Np = Np;
-      px.nb = nbl;
-      px.bdiv = ni;
-      EpiPxOut e;
-      e.out = O;
-      e.split_stride = px_stride;
-      e.om.bdiv = ni;
-      e.om.b1 = (int64_t)ni * t * 2 * d;
-      e.om.b0 = (int64_t)t * 2 * d;
-      e.om.r0 = 2 * d;
-      e.om.c0 = 1;
-      const Operand2D xt = op(XT, (int64_t)H * 2 * d, 2 * Np);
-      // Split probabilities (hi + lo) in a block whose output enters another block.
-      ctx->prof.begin(STILL_K_PX, s);
-      cudaError_t r =
-          d == 64    ? (exact ? launch_px_fused<128, 64, true>(xt, p, px, e, ctx->nsm, s)
-                              : launch_px_fused<128, 64>(xt, p, px, e, ctx->nsm, s))
-          : d == 128 ? (exact ? launch_px_fused<256, 128, true>(xt, p, px, e, ctx->nsm, s)
-                              : launch_px_fused<256, 128>(xt, p, px, e, ctx->nsm, s))
-                     : (exact ? launch_px_fused<256, 256, true>(xt, p, px, e, ctx->nsm, s)
-                              : launch_px_fused<256, 256>(xt, p, px, e, ctx->nsm, s));
-      ctx->prof.end(STILL_K_PX, s);
-      if (r == cudaErrorInvalidValue) return STILL_ERR_INVALID_ARG;
-      if (r != cudaSuccess) return STILL_ERR_CUDA;
-    }
-    KLAUNCH(STILL_K_PXSPLIT, launch_px_to_hilo(O, px_split, px_stride, b0, nbl, n, t, 2 * d, PX, s));
-    b0 += nbl;
   }
 
   // ---------------------------------------------------------------- Z' = Z + PX W_VO
