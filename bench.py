@@ -299,7 +299,8 @@ DECODE = dict(L=36, H=8, Hq=32, d=128, t=1311, S=4096, nq=1)
 
 def run_decode(args):
     """Biased decode attention (App. B, "Bias semantics in attention") over [C_k; K_fix] for
-    every layer, captured as one CUDA graph; one step = one decode token through all layers."""
+    every layer in one launch (captured as a CUDA graph); one step = one decode token through
+    all layers."""
     import numpy as np
     import torch
 
@@ -323,10 +324,8 @@ def run_decode(args):
     outs = [torch.empty((nq, Hq, d), dtype=torch.bfloat16, device=dev) for _ in range(L)]
     ctx = still.still_create(0)
 
-    def step():
-        for l in range(L):
-            still.still_attend_biased(ctx, qs[l], Cks[l], Cvs[l], betas[l], Kfs[l], Vfs[l],
-                                      outs[l], stream=stream)
+    def step():  # every layer in one launch pair (chunks + merge)
+        still.still_attend_biased_stack(ctx, qs, Cks, Cvs, betas, Kfs, Vfs, outs, stream=stream)
 
     still.still_profile_enable(ctx, True)
     for _ in range(max(args.warmup, 3)):
@@ -357,12 +356,11 @@ def run_decode(args):
     if code != 0:
         raise RuntimeError(f"device status {still.STATUS.get(code)} {det}")
     del graph
-    n_dec, ms_dec = prof["decode"]  # the last replay's launches (chunk + merge per layer)
+    n_dec, ms_dec = prof["decode"]  # the last replay's launches (chunk + merge)
     # Algorithmic bytes of one layer's attention: the compact slots and raw entries (K and V),
-    # the bias, the query and the output.
+    # the bias, the query and the output; one replay covers all L layers.
     layer_bytes = (t + S) * H * d * 2 * 2 + t * H * 4 + 2 * nq * Hq * d * 2
-    calls = n_dec // 2
-    achieved = layer_bytes * calls / (ms_dec / 1e3) / 1e9 if ms_dec > 0 else None
+    achieved = layer_bytes * L / (ms_dec / 1e3) / 1e9 if ms_dec > 0 else None
     hbm, _, _, src = _peaks()
     # end to end: the step's queries from pinned host memory in, outputs back to the host
     q_host = [x.cpu().pin_memory() for x in qs]
@@ -372,8 +370,8 @@ def run_decode(args):
     def e2e_step():
         for l in range(L):
             qs[l].copy_(q_host[l], non_blocking=True)
-            still.still_attend_biased(ctx, qs[l], Cks[l], Cvs[l], betas[l], Kfs[l], Vfs[l],
-                                      outs[l], stream=ds)
+        still.still_attend_biased_stack(ctx, qs, Cks, Cvs, betas, Kfs, Vfs, outs, stream=ds)
+        for l in range(L):
             o_host[l].copy_(outs[l], non_blocking=True)
         ds.synchronize()
 
@@ -408,12 +406,13 @@ def run_decode(args):
                    "l2": f"inputs larger than L2 ({L * layer_bytes / 1e6:.0f} MB per step)"},
         "e2e": {"value": steps / e2e_s, "unit": "tokens/s",
                 "h2d_bytes_per_step": L * nq * Hq * d * 2, "d2h_bytes_per_step": L * nq * Hq * d * 2},
-        "gpu_launches": n_dec,
-        "roofline": {"bound": "hbm", "kernel": "decode attention (chunks + merge)",
+        "gpu_launches": n_dec * steps,  # launches per replay x timed replays
+        "roofline": {"bound": "hbm", "kernel": f"decode attention over {L} layers in one "
+                                                 f"launch (chunks + merge)",
                      "achieved": achieved, "peak": hbm, "unit": "GB/s",
                      "frac": achieved / hbm if achieved else None, "traffic": None,
                      "peak_source": f"{src} HBM copy bandwidth",
-                     "bytes_per_launch": layer_bytes},
+                     "bytes_per_launch": layer_bytes * L},
         "cpu_baseline": cpu, "clocks": clk}))
 
 
@@ -489,6 +488,8 @@ def run_iterative(args):
     del Kn, Vn, Ck2, Cv2
     total_ms = 0.0
     launches = 0
+    clocks = ClockSampler(0)  # sampled over the rounds (their input generation included)
+    clocks.start()
     for r in range(rounds):
         Kn, Vn, Ck2, Cv2 = round_inputs(r)
         torch.cuda.synchronize()
@@ -505,6 +506,7 @@ def run_iterative(args):
         launches += sum(v[0] for k, v in prof.items() if k != "load")
         Cks, Cvs, cu_prev, prev_len = Ck2, Cv2, cu_out, len_out
         del Kn, Vn
+    clk = clocks.stop()
     code, det = still.still_get_device_status(ctx, stream)
     if code != 0:
         raise RuntimeError(f"device status {still.STATUS.get(code)} {det}")
@@ -519,7 +521,7 @@ def run_iterative(args):
                                f"H_kv={H}, d={d}, D={wl['D']}, {wl['n']} heads, "
                                f"{ratio}x, +{chunk} tokens per round",
                    "final_lengths": prev_len},
-        "gpu_launches": launches,
+        "gpu_launches": launches, "clocks": clk,
     }))
 
 

@@ -243,6 +243,20 @@ still_status still_attend_biased(still_ctx* ctx, const void* q, int32_t nq, int3
                                  const void* Kfix, const void* Vfix, int64_t S, int32_t H,
                                  int32_t d, float scale, void* out, void* stream);
 
+/* still_attend_biased for n_layers layers of one shape (the decode step of a model, App. B,
+ * "Bias semantics in attention"), in one launch: every argument as above, the tensors given as
+ * host arrays of n_layers device pointers (q[l], Ck[l], Cv[l], Kfix[l], Vfix[l], out[l]);
+ * beta is NULL (no bias in any layer) or an array whose entries may be NULL.
+ * 1 <= n_layers <= 64 (STILL_ERR_UNSUPPORTED otherwise). A single layer's cache is too small
+ * for one launch to keep HBM busy; layer l's result equals still_attend_biased on layer l
+ * bit for bit. */
+still_status still_attend_biased_stack(still_ctx* ctx, int32_t n_layers, const void* const* q,
+                                       int32_t nq, int32_t Hq, const void* const* Ck,
+                                       const void* const* Cv, const float* const* beta, int64_t t,
+                                       const void* const* Kfix, const void* const* Vfix,
+                                       int64_t S, int32_t H, int32_t d, float scale,
+                                       void* const* out, void* stream);
+
 /* Compacts layers 0..n_layers-1 (all loaded) over the same positions: the per-layer
  * compactors share nothing at forward time (App. M, "No inter-layer compactor channel"), so
  * this is one stream-ordered launch sequence over the layer stack. K[l], V[l], Ck[l], Cv[l] are device

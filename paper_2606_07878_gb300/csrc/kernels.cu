@@ -657,8 +657,8 @@ __global__ void beta_kernel(const __nv_bfloat16* __restrict__ Z, int64_t rows, i
 // ----------------------------------------------------------------- biased decode attention
 //
 // Attention of query rows over the entries [C (t compact slots, logit bias beta) ; F (S
-// uncompacted entries, bias 0)] (App. B, "Bias semantics in attention"). Grid (slot, KV-head),
-// one wave: the CTAs of a KV-head take its chunks of dec_chunk entries in turn (slot, slot +
+// uncompacted entries, bias 0)] (App. B, "Bias semantics in attention"). Grid (slot, KV-head,
+// layer): the CTAs of a KV-head take its chunks of dec_chunk entries in turn (slot, slot +
 // slots, ...). In a chunk each of the 16 warps holds 8 entries (4 at d = 256); a lane holds
 // DPL = d/32 dimensions of its warp's keys and values in registers (coalesced loads, all issued
 // up front), so the cache is read once and straight from global memory. Per query row of the
@@ -758,15 +758,24 @@ __device__ __forceinline__ float dec_across(float x) {
   return x;
 }
 
+// Grid (slot, KV-head, layer): layer z's arguments are st.layer[z]; its partials start
+// z * rows * slots rows into part_o / part_ml.
 template <int DPL>
 __global__ void __launch_bounds__(kDecThreads, 1)
-    decode_chunk_kernel(DecodeArgs a, float* __restrict__ part_o, float2* __restrict__ part_ml) {
+    decode_chunk_kernel(const __grid_constant__ DecodeStack st, float* __restrict__ part_o,
+                        float2* __restrict__ part_ml) {
   extern __shared__ float dsm[];
   constexpr int d = 32 * DPL;
   constexpr int kW = kDecThreads / 32;
   constexpr int kDecPerWarp = dec_per_warp(DPL);
   constexpr int kDecChunk = dec_chunk(DPL);
+  const DecodeArgs& a = st.layer[blockIdx.z];
   const int h = blockIdx.y, slot = blockIdx.x, nslots = gridDim.x;
+  {
+    const int64_t lrows = (int64_t)blockIdx.z * a.nq * a.Hq * nslots;
+    part_o += lrows * d;
+    part_ml += lrows;
+  }
   const int g = a.Hq / a.H;        // query heads per KV-head
   const int G = a.nq * g;          // query rows served by this CTA
   float* qs = dsm;                                  // [G][d]
@@ -911,12 +920,16 @@ __global__ void __launch_bounds__(kDecThreads, 1)
 
 // Output row (query n, query head qh): sum_s e^(m_s - M) O_s / sum_s e^(m_s - M) l_s over the
 // chunk partials, in chunk order. One CTA of d threads per row, one column per thread.
-__global__ void decode_merge_kernel(const float* __restrict__ part_o,
+__global__ void decode_merge_kernel(const __grid_constant__ DecodeStack st,
+                                    const float* __restrict__ part_o,
                                     const float2* __restrict__ part_ml, int64_t rows, int nch,
-                                    int d, __nv_bfloat16* __restrict__ out) {
+                                    int d) {
   extern __shared__ float2 mls[];  // the row's (m, l) per chunk, then (weight, -)
   const int64_t row = blockIdx.x;
   const int c = threadIdx.x;
+  __nv_bfloat16* __restrict__ out = st.layer[blockIdx.y].out;
+  part_o += (int64_t)blockIdx.y * rows * nch * d;  // layer blockIdx.y's partials
+  part_ml += (int64_t)blockIdx.y * rows * nch;
   for (int s = c; s < nch; s += blockDim.x) mls[s] = part_ml[row * nch + s];  // coalesced
   __syncthreads();
   float M = -INFINITY;
@@ -941,17 +954,21 @@ inline unsigned blocks_for(int64_t n, int per) { return (unsigned)((n + per - 1)
 
 }  // namespace
 
-size_t decode_workspace_bytes(int64_t rows, int64_t entries, int d) {
+size_t decode_workspace_bytes(int64_t rows, int64_t entries, int d, int layers) {
   const int chunk = dec_chunk(d / 32);
   const int64_t nch = (entries + chunk - 1) / chunk;
-  return (size_t)rows * nch * d * 4 + (size_t)rows * nch * 8 + 256;
+  const int64_t r = rows * layers;
+  return (size_t)r * nch * d * 4 + 256 + (size_t)r * nch * 8 + 256;
 }
 
-cudaError_t launch_decode_biased(const DecodeArgs& a, void* ws, int num_sms, cudaStream_t s) {
+cudaError_t launch_decode_biased(const DecodeStack& st, void* ws, int num_sms, cudaStream_t s) {
+  if (st.n < 1 || st.n > kDecodeMaxLayers) return cudaErrorInvalidValue;
+  const DecodeArgs& a = st.layer[0];  // every layer has the same shape
   const int64_t E = a.t + a.S;
   const int chunk = dec_chunk(a.d / 32);
   const int64_t nchunks = (E + chunk - 1) / chunk;
-  // One wave: the CTAs of a KV-head split its chunks (each CTA merges its own in order).
+  // One wave per layer: the CTAs of a KV-head split its chunks (each CTA merges its own in
+  // order).
   const int per_sm = 1;
   const int nch = (int)std::max<int64_t>(
       1, std::min<int64_t>(nchunks, (int64_t)num_sms * per_sm / std::max(1, a.H)));
@@ -960,7 +977,8 @@ cudaError_t launch_decode_biased(const DecodeArgs& a, void* ws, int num_sms, cud
   const int64_t rows = (int64_t)a.nq * a.Hq;
   float* part_o = static_cast<float*>(ws);
   float2* part_ml = reinterpret_cast<float2*>(
-      static_cast<uint8_t*>(ws) + (((size_t)rows * nch * a.d * 4 + 255) & ~size_t(255)));
+      static_cast<uint8_t*>(ws) +
+      (((size_t)rows * st.n * nch * a.d * 4 + 255) & ~size_t(255)));
   const size_t smem = ((size_t)G * a.d + (size_t)(kDecThreads / 32) * kDecRowGroup * (a.d + 2) +
                        (size_t)G * (a.d + 2) + 2 * kDecRowGroup) * 4;
   auto kern = a.d == 64 ? decode_chunk_kernel<2>
@@ -973,12 +991,13 @@ cudaError_t launch_decode_biased(const DecodeArgs& a, void* ws, int num_sms, cud
     if (e != cudaSuccess) return e;
     smem_set[ki] = smem;
   }
-  kern<<<dim3(nch, a.H), kDecThreads, smem, s>>>(a, part_o, part_ml);
+  kern<<<dim3(nch, a.H, st.n), kDecThreads, smem, s>>>(st, part_o, part_ml);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const size_t msm = (size_t)nch * sizeof(float2);
   if (msm > 48 * 1024) return cudaErrorInvalidValue;  // more than 6144 chunks
-  decode_merge_kernel<<<(unsigned)rows, a.d, msm, s>>>(part_o, part_ml, rows, nch, a.d, a.out);
+  decode_merge_kernel<<<dim3((unsigned)rows, st.n), a.d, msm, s>>>(st, part_o, part_ml, rows,
+                                                                   nch, a.d);
   return cudaGetLastError();
 }
 

@@ -63,8 +63,15 @@ struct DecodeArgs {
   int32_t nq = 0, Hq = 0, H = 0, d = 0;
   float scale = 0.f;
 };
-size_t decode_workspace_bytes(int64_t rows, int64_t entries, int d);
-cudaError_t launch_decode_biased(const DecodeArgs& a, void* ws, int num_sms, cudaStream_t s);
+// Several layers of one shape (t, S, nq, Hq, H, d equal) in one launch of the chunk kernel and
+// one of the merge: layer z's arguments are layer[z], z < n.
+constexpr int kDecodeMaxLayers = 64;
+struct DecodeStack {
+  DecodeArgs layer[kDecodeMaxLayers];
+  int32_t n = 0;
+};
+size_t decode_workspace_bytes(int64_t rows, int64_t entries, int d, int layers = 1);
+cudaError_t launch_decode_biased(const DecodeStack& st, void* ws, int num_sms, cudaStream_t s);
 
 // Converts n bf16 values to fp16 in place (exact within the fp16 range; values below it
 // become fp16 subnormals, absolute error <= 2^-25).

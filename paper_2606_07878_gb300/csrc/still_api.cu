@@ -1541,11 +1541,20 @@ still_status still_set_beta_head(still_ctx* ctx, int32_t layer, const void* w_be
   return STILL_OK;
 }
 
-still_status still_attend_biased(still_ctx* ctx, const void* q, int32_t nq, int32_t Hq,
-                                 const void* Ck, const void* Cv, const float* beta, int64_t t,
-                                 const void* Kfix, const void* Vfix, int64_t S, int32_t H,
-                                 int32_t d, float scale, void* out, void* stream) {
+}  // extern "C"
+
+namespace {
+
+// The decode-time attention of n_layers layers of one shape, in one launch of the chunk kernel
+// and one of the merge. Pointer arrays are host arrays of device pointers.
+still_status attend_biased_impl(still_ctx* ctx, int32_t n_layers, const void* const* q,
+                                int32_t nq, int32_t Hq, const void* const* Ck,
+                                const void* const* Cv, const float* const* beta, int64_t t,
+                                const void* const* Kfix, const void* const* Vfix, int64_t S,
+                                int32_t H, int32_t d, float scale, void* const* out,
+                                void* stream) {
   if (ctx == nullptr || q == nullptr || out == nullptr) return STILL_ERR_INVALID_ARG;
+  if (n_layers < 1 || n_layers > kDecodeMaxLayers) return STILL_ERR_UNSUPPORTED;
   if (nq < 1 || H < 1 || Hq < H || Hq % H != 0 || t < 0 || S < 0 || t + S < 1 ||
       (t > 0 && (Ck == nullptr || Cv == nullptr)) || (S > 0 && (Kfix == nullptr || Vfix == nullptr)))
     return STILL_ERR_INVALID_ARG;
@@ -1553,36 +1562,70 @@ still_status still_attend_biased(still_ctx* ctx, const void* q, int32_t nq, int3
       t + S > (int64_t(1) << 31) - 128)
     return STILL_ERR_UNSUPPORTED;
   if (!(scale >= 0.f) || !std::isfinite(scale)) return STILL_ERR_INVALID_ARG;
-  const uintptr_t al = reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(out) |
-                       reinterpret_cast<uintptr_t>(Ck) | reinterpret_cast<uintptr_t>(Cv) |
-                       reinterpret_cast<uintptr_t>(Kfix) | reinterpret_cast<uintptr_t>(Vfix);
-  if ((al & 15) || (reinterpret_cast<uintptr_t>(beta) & 3)) return STILL_ERR_ALIGNMENT;
+  DecodeStack st;
+  st.n = n_layers;
+  for (int l = 0; l < n_layers; ++l) {
+    const void* ck = t > 0 ? Ck[l] : nullptr;
+    const void* cv = t > 0 ? Cv[l] : nullptr;
+    const void* kf = S > 0 ? Kfix[l] : nullptr;
+    const void* vf = S > 0 ? Vfix[l] : nullptr;
+    const float* b = beta != nullptr ? beta[l] : nullptr;
+    if (q[l] == nullptr || out[l] == nullptr || (t > 0 && (ck == nullptr || cv == nullptr)) ||
+        (S > 0 && (kf == nullptr || vf == nullptr)))
+      return STILL_ERR_INVALID_ARG;
+    const uintptr_t al = reinterpret_cast<uintptr_t>(q[l]) | reinterpret_cast<uintptr_t>(out[l]) |
+                         reinterpret_cast<uintptr_t>(ck) | reinterpret_cast<uintptr_t>(cv) |
+                         reinterpret_cast<uintptr_t>(kf) | reinterpret_cast<uintptr_t>(vf);
+    if ((al & 15) || (reinterpret_cast<uintptr_t>(b) & 3)) return STILL_ERR_ALIGNMENT;
+    DecodeArgs& a = st.layer[l];
+    a.q = static_cast<const bf16*>(q[l]);
+    a.Ck = static_cast<const bf16*>(ck);
+    a.Cv = static_cast<const bf16*>(cv);
+    a.beta = b;
+    a.Kf = static_cast<const bf16*>(kf);
+    a.Vf = static_cast<const bf16*>(vf);
+    a.out = static_cast<bf16*>(out[l]);
+    a.t = t;
+    a.S = S;
+    a.cst = (int64_t)H * d;
+    a.fst = (int64_t)H * d;
+    a.nq = nq;
+    a.Hq = Hq;
+    a.H = H;
+    a.d = d;
+    a.scale = scale > 0.f ? scale : 1.f / std::sqrt((float)d);
+  }
   CK(cudaSetDevice(ctx->device));
-  DecodeArgs a;
-  a.q = static_cast<const bf16*>(q);
-  a.Ck = static_cast<const bf16*>(Ck);
-  a.Cv = static_cast<const bf16*>(Cv);
-  a.beta = beta;
-  a.Kf = static_cast<const bf16*>(Kfix);
-  a.Vf = static_cast<const bf16*>(Vfix);
-  a.out = static_cast<bf16*>(out);
-  a.t = t;
-  a.S = S;
-  a.cst = (int64_t)H * d;
-  a.fst = (int64_t)H * d;
-  a.nq = nq;
-  a.Hq = Hq;
-  a.H = H;
-  a.d = d;
-  a.scale = scale > 0.f ? scale : 1.f / std::sqrt((float)d);
-  TRY(ensure_ws(ctx, decode_workspace_bytes((int64_t)nq * Hq, t + S, d)));
+  TRY(ensure_ws(ctx, decode_workspace_bytes((int64_t)nq * Hq, t + S, d, n_layers)));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   ctx->prof.begin(STILL_K_DECODE, s);
-  cudaError_t r = launch_decode_biased(a, ctx->ws, ctx->nsm, s);
+  cudaError_t r = launch_decode_biased(st, ctx->ws, ctx->nsm, s);
   ctx->prof.end(STILL_K_DECODE, s);
   ctx->prof.launches[STILL_K_DECODE] += 1;  // the merge kernel (begin counted the first)
   if (r != cudaSuccess) return STILL_ERR_CUDA;
   return STILL_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+still_status still_attend_biased(still_ctx* ctx, const void* q, int32_t nq, int32_t Hq,
+                                 const void* Ck, const void* Cv, const float* beta, int64_t t,
+                                 const void* Kfix, const void* Vfix, int64_t S, int32_t H,
+                                 int32_t d, float scale, void* out, void* stream) {
+  return attend_biased_impl(ctx, 1, &q, nq, Hq, &Ck, &Cv, &beta, t, &Kfix, &Vfix, S, H, d, scale,
+                            &out, stream);
+}
+
+still_status still_attend_biased_stack(still_ctx* ctx, int32_t n_layers, const void* const* q,
+                                       int32_t nq, int32_t Hq, const void* const* Ck,
+                                       const void* const* Cv, const float* const* beta, int64_t t,
+                                       const void* const* Kfix, const void* const* Vfix,
+                                       int64_t S, int32_t H, int32_t d, float scale,
+                                       void* const* out, void* stream) {
+  return attend_biased_impl(ctx, n_layers, q, nq, Hq, Ck, Cv, beta, t, Kfix, Vfix, S, H, d,
+                            scale, out, stream);
 }
 
 still_status still_compact_layer_noalloc(still_ctx* ctx, int32_t layer, const void* K,

@@ -31,6 +31,7 @@ EXPORTS = [
     "still_selftest_wait_timeout", "still_compact_stack_masked", "still_lookahead_pass_info",
     "still_lookahead_totals", "still_lookahead_compact_layer", "still_lookahead_compact_stack",
     "still_set_beta_head", "still_compact_layer_beta", "still_attend_biased", "still_set_key_fold",
+    "still_attend_biased_stack",
 ]
 
 NOALLOC_SCRATCH_MIB = 64  # STILL_NOALLOC_SCRATCH_MIB in include/still.h
@@ -155,6 +156,11 @@ def lib():
                                           PD, PI64, P], ctypes.c_int),
             "still_attend_biased": ([P, P, I32, I32, P, P, P, I64, P, P, I64, I32, I32,
                                      ctypes.c_float, P, P], ctypes.c_int),
+            "still_attend_biased_stack": ([P, I32, ctypes.POINTER(P), I32, I32,
+                                           ctypes.POINTER(P), ctypes.POINTER(P),
+                                           ctypes.POINTER(P), I64, ctypes.POINTER(P),
+                                           ctypes.POINTER(P), I64, I32, I32, ctypes.c_float,
+                                           ctypes.POINTER(P), P], ctypes.c_int),
             "still_lookahead_pass_info": ([I64, I64, I32, ctypes.POINTER(LookaheadPass)],
                                           ctypes.c_int),
             "still_lookahead_totals": ([I64, I64, I32, PI64, PI64], ctypes.c_int),
@@ -354,6 +360,26 @@ def still_attend_biased(ctx, q, Ck, Cv, beta, Kfix, Vfix, out, scale=0.0, stream
                                      _ptr(Cv) if t else None, _ptr(beta), t,
                                      _ptr(Kfix) if S else None, _ptr(Vfix) if S else None, S, H,
                                      d, scale, _ptr(out), _stream(stream)), "still_attend_biased")
+
+
+def still_attend_biased_stack(ctx, q, Ck, Cv, beta, Kfix, Vfix, out, scale=0.0, stream=None):
+    """still_attend_biased over a list of layers of one shape, in one launch: q, Ck, Cv, Kfix,
+    Vfix, out are lists of per-layer tensors (shapes as in still_attend_biased); beta is None or
+    a list whose entries may be None."""
+    L = len(q)
+    nq, Hq, d = q[0].shape
+    t, H = Ck[0].shape[0], Ck[0].shape[1]
+    S = Kfix[0].shape[0]
+    P = ctypes.c_void_p
+
+    def arr(xs, use=True):
+        return (P * L)(*[(x.data_ptr() if use and x is not None else None) for x in xs])
+
+    betas = arr(beta) if beta is not None else None
+    _check(lib().still_attend_biased_stack(ctx, L, arr(q), nq, Hq, arr(Ck, t > 0),
+                                           arr(Cv, t > 0), betas, t, arr(Kfix, S > 0),
+                                           arr(Vfix, S > 0), S, H, d, scale, arr(out),
+                                           _stream(stream)), "still_attend_biased_stack")
 
 
 def still_lookahead_pass_info(k: int, c: int, t: int) -> dict:

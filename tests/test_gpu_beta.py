@@ -142,3 +142,44 @@ def test_biased_decode_rejects_bad_arguments():
         assert e.value.name == "STILL_ERR_UNSUPPORTED"
     finally:
         still.still_destroy(ctx)
+
+
+@pytest.mark.parametrize("d,t,S", [(128, 300, 77), (256, 129, 0), (64, 0, 200)])
+def test_decode_stack_equals_per_layer_calls_and_oracle(d, t, S):
+    """One launch over a stack of layers: every layer's result equals the single-layer call bit
+    for bit (same chunking, same merge order), and layer results match the oracle."""
+    L, nq, Hq, H = 5, 1, 16, 4
+    q = [_bf16((nq, Hq, d), 100 + l) for l in range(L)]
+    Ck = [_bf16((t, H, d), 200 + l) for l in range(L)]
+    Cv = [_bf16((t, H, d), 300 + l) for l in range(L)]
+    Kf = [_bf16((S, H, d), 400 + l) for l in range(L)]
+    Vf = [_bf16((S, H, d), 500 + l) for l in range(L)]
+    beta = [(2.0 * torch.randn((t, H), generator=torch.Generator().manual_seed(600 + l))).to(DEV)
+            for l in range(L)]
+    beta[2] = None  # a layer without the bias channel
+    out = [torch.empty((nq, Hq, d), dtype=torch.bfloat16, device=DEV) for _ in range(L)]
+    ctx = still.still_create(0)
+    try:
+        still.still_attend_biased_stack(ctx, q, Ck, Cv, beta, Kf, Vf, out)
+        code, det = still.still_get_device_status(ctx)
+        assert code == 0, det
+        f = lambda x: x.double().cpu().numpy()
+        for l in range(L):
+            one = torch.empty_like(out[l])
+            still.still_attend_biased(ctx, q[l], Ck[l], Cv[l], beta[l], Kf[l], Vf[l], one)
+            assert torch.equal(one, out[l]), l
+        for l in (0, 2, L - 1):
+            bn = f(beta[l]) if beta[l] is not None else np.zeros((t, H))
+            ref = np.empty((nq, Hq, d))
+            for qh in range(Hq):
+                h = qh // (Hq // H)
+                ref[:, qh] = O.biased_attention(f(q[l])[:, qh], f(Ck[l])[:, h], f(Cv[l])[:, h],
+                                                bn[:, h], f(Kf[l])[:, h], f(Vf[l])[:, h],
+                                                1 / math.sqrt(d))
+            assert_parity(ref.reshape(-1, d), f(out[l]).reshape(-1, d), f"layer {l}")
+        with pytest.raises(still.StillError) as e:  # more layers than one launch takes
+            still.still_attend_biased_stack(ctx, q * 13, Ck * 13, Cv * 13, None, Kf * 13,
+                                            Vf * 13, out * 13)
+        assert e.value.name == "STILL_ERR_UNSUPPORTED"
+    finally:
+        still.still_destroy(ctx)
