@@ -573,15 +573,17 @@ inline cudaError_t launch_ca_flash(const Operand2D& Q, const Operand2D& K, const
   return cudaGetLastError();
 }
 
-// 2d = 512 (head dim 256): the same computation on a cluster of two CTAs that split the O
-// columns and take turns computing S (ca_pair.cu). Q, K as for launch_ca_flash; XT: [H*512][2*Np]
-// fp16 (hi | lo). num_sms: SMs of the device (two per cluster).
+// 2d = 512 (head dim 256): the same computation on clusters of four CTAs, two query tiles x
+// two column halves; the CTAs of a query tile split the O columns and take turns computing S,
+// the CTAs of a half share their k and X^T loads (ca_pair.cu). Q, K as for launch_ca_flash;
+// XT: [H*512][2*Np] fp16 (hi | lo). f.nunits counts (query-tile pair, key split, batch) units.
+// num_sms: SMs of the device (four per cluster).
 // one_pass: q, k as fp16 hi | lo with S from the hi parts only (one MMA pass) and repair
 // candidates in f.cand_key / f.cand_c for ca_topk_repair; else 3-pass split-bf16 scores.
 cudaError_t launch_ca_pair(const Operand2D& Q, const Operand2D& K, const Operand2D& XT,
                            const FlashParams& f, int num_sms, cudaStream_t stream,
                            bool one_pass = false);
-// Clusters of that kernel that can be resident at once (its persistent grid size).
+// Four-CTA clusters of that kernel that can be resident at once (its persistent grid size).
 int ca_pair_clusters(int num_sms);
 
 // Top-k repair of one-pass scores: for each (b, row), over the splits whose running max is within

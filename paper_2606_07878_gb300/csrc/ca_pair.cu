@@ -6,13 +6,21 @@
 //   O(m, :)  = sum_k P(m, k) X(k, :)                unnormalised, with the row sum l per split
 //
 // The accumulator of a 128-row query tile over 2d = 512 columns fills a whole TMEM (512
-// fp32 columns), leaving no room for S. A cluster of two CTAs therefore shares each work unit
-// (batch b = (KV-head, cross head), 128-row query tile, key split): CTA r keeps the O columns
-// of features [128 r, 128 r + 128) of K~ and of V (256 columns, TMEM [256, 512)) and computes
-// S for every other 256-key tile (TMEM [0, 256)). The CTA that owns a tile forms its fp16
-// probabilities, sends the tile's running row maximum to its peer as soon as it is decided,
-// and copies the probability tile into the peer's shared memory with a bulk DSMEM copy; both
-// CTAs then accumulate P X for their column half. S and P never reach global memory.
+// fp32 columns), leaving no room for S. Two CTAs therefore share each query tile: CTA half r
+// keeps the O columns of features [128 r, 128 r + 128) of K~ and of V (256 columns, TMEM
+// [256, 512)) and computes S for every other 256-key tile (TMEM [0, 256)). The CTA that owns
+// a tile forms its fp16 probabilities, sends the tile's running row maximum to its peer as
+// soon as it is decided, and copies the probability tile into the peer's shared memory with a
+// bulk DSMEM copy; both CTAs then accumulate P X for their column half. S and P never reach
+// global memory.
+//
+// A work unit (batch b = (KV-head, cross head), two 128-row query tiles, key split) runs on
+// a cluster of four CTAs, rank = 2 x + r: query tile x of the pair, column half r. The two
+// CTAs of one half (its "twins", rank ^ 2) need the same k tiles and the same X^T columns in
+// the same order, so each loads one half of every k and X^T box and multicasts it to both:
+// the operand traffic per flop from L2 falls by a third for S and by half for P X, which is
+// what bounds the kernel (the loads of all SMs together). A ring slot is reloaded only when
+// both twins' MMAs have consumed it (their commits arrive on both CTAs' empty barriers).
 //
 // Both CTAs apply the same running-maximum sequence (the owner's decision travels with the
 // tile), so their O halves, and the row sums each accumulates from its own tiles, stay on one
@@ -45,6 +53,7 @@ namespace {
 constexpr int kPairKeys = 256;   // keys per S tile
 constexpr int kPairOCols = 256;  // O columns per CTA
 constexpr uint32_t kPairPBytes = kBM * kPairKeys * 2;  // one fp16 P tile, 64 KB
+constexpr int kPairCluster = 4;  // CTAs per cluster: two query tiles x two column halves
 
 struct PairSmem {
   static constexpr int kQBytes = kBM * kBK * 2;                // q chunk, 16 KB
@@ -64,10 +73,25 @@ struct PairSmem {
   static_assert(kBytes <= 232448, "shared memory budget");
 };
 
-// Owner of tile jj of a unit: CTA (jj & 1). Before its own tile jj a CTA issues every P X
-// tile up to jj - 2; the remaining ones after its last own tile.
-__device__ __forceinline__ bool pair_owner(int jj, uint32_t rank) {
-  return (uint32_t)(jj & 1) == rank;
+// Owner of tile jj of a unit: the CTAs of half (jj & 1). Before its own tile jj a CTA issues
+// every P X tile up to jj - 2; the remaining ones after its last own tile.
+__device__ __forceinline__ bool pair_owner(int jj, uint32_t half) {
+  return (uint32_t)(jj & 1) == half;
+}
+
+// Unit u of the four-CTA clusters: query tiles 2 m and 2 m + 1 (m fastest), then the key
+// split, then the batch; this CTA takes query tile 2 m + x. A tile past the last one (odd
+// tile count) is computed and not stored.
+__device__ __forceinline__ FlashUnit pair_unit(const FlashParams& f, int u, uint32_t x) {
+  const int mp = (f.tiles_m + 1) / 2;
+  FlashUnit r;
+  r.tm = 2 * (u % mp) + (int)x;
+  const int q = u / mp;
+  r.split = q % f.nsplit;
+  r.b = q / f.nsplit;
+  r.j0 = (int)(((int64_t)f.tiles_k * r.split) / f.nsplit);
+  r.j1 = (int)(((int64_t)f.tiles_k * (r.split + 1)) / f.nsplit);
+  return r;
 }
 
 // TK: one-pass fp16 scores (q_hi . k_hi) with repair candidates; else 3-pass split-bf16.
@@ -102,13 +126,17 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
   const int lane = threadIdx.x & 31;
   const int qchunks = f.D / kBK;
   const uint32_t rank = cluster_ctarank();
-  const uint32_t peer = rank ^ 1u;
+  const uint32_t chalf = rank & 1u;  // column half; S owner parity
+  const uint32_t qx = rank >> 1;     // query tile of the unit's pair
+  const uint32_t peer = rank ^ 1u;   // same query tile, other half: the P exchange
+  // same half, other query tile: shares the k and X^T loads
+  const uint16_t mc_mask = (uint16_t)((1u << rank) | (1u << (rank ^ 2u)));
   const int cid = (int)cluster_id_x(), ncl = (int)cluster_count_x();
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], 2);  // this CTA's and its twin's MMA commits
     }
     mbar_init(sfull, 1);
     mbar_init(sfree, kFlashSoftWarps);
@@ -162,14 +190,17 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
         }
       };
       for (int u = cid; u < f.nunits && !bad && !*abort_flag; u += ncl) {
-        const FlashUnit w = flash_unit(f, u);
+        const FlashUnit w = pair_unit(f, u, qx);
         const int32_t qrow =
             (int32_t)(f.q_row0 + (int64_t)w.b * (f.q_pitch > 0 ? f.q_pitch : f.t)) + w.tm * kBM;
         const int32_t krow =
             (int32_t)(f.k_row0 + (int64_t)(f.kdiv > 0 ? w.b / f.kdiv : w.b) * f.N);
-        // this CTA's feature rows of X^T: K~ [128 rank, +128) and V [128 rank, +128)
-        const int32_t xk = f.xbase_row + (w.b / f.bdiv) * 512 + 128 * (int32_t)rank;
+        // this half's feature rows of X^T: K~ [128 r, +128) and V [128 r, +128); this CTA
+        // loads rows [64 x, +64) of each box for both twins
+        const int32_t xk = f.xbase_row + (w.b / f.bdiv) * 512 + 128 * (int32_t)chalf;
         const int32_t xv = xk + 256;
+        const int32_t xo = 64 * (int32_t)qx;
+        const int xs = (S::kXBox / 2) * (int)qx;  // shared-memory offset of those rows
         const int J = w.j1 - w.j0;
         auto produce_px = [&](int i) {
           const int j = w.j0 + i;
@@ -178,15 +209,16 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
             uint8_t* sa = acquire(3 * S::kXBox);
             if (sa == nullptr) break;
             const int32_t x = j * kPairKeys + c * kBK;
-            tma_load_2d(sa, &tmX, &full[stage], x, xk);
-            tma_load_2d(sa + S::kXBox, &tmX, &full[stage], x, xv);
-            tma_load_2d(sa + 2 * S::kXBox, &tmX, &full[stage], (int32_t)(f.Np + x), xk);
+            tma_load_2d_mc(sa + xs, &tmX, &full[stage], x, xk + xo, mc_mask);
+            tma_load_2d_mc(sa + S::kXBox + xs, &tmX, &full[stage], x, xv + xo, mc_mask);
+            tma_load_2d_mc(sa + 2 * S::kXBox + xs, &tmX, &full[stage], (int32_t)(f.Np + x),
+                           xk + xo, mc_mask);
             advance();
           }
         };
         int px_next = 0;
         for (int jj = 0; jj < J && !bad; ++jj) {
-          if (!pair_owner(jj, rank)) continue;
+          if (!pair_owner(jj, chalf)) continue;
           while (px_next <= jj - 2 && !bad) produce_px(px_next++);
           const int32_t kr = krow + (w.j0 + jj) * kPairKeys;
           for (int pass = 0; pass < kPasses && !bad; ++pass) {
@@ -196,12 +228,25 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
               uint8_t* sa = acquire(S::kQBytes + S::kKBytes);
               if (sa == nullptr) break;
               tma_load_2d(sa, &tmQ, &full[stage], qoff + c * kBK, qrow);
-              tma_load_2d(sa + S::kQBytes, &tmK, &full[stage], koff + c * kBK, kr);
+              // keys [128 x, +128) of the tile, for both twins
+              tma_load_2d_mc(sa + S::kQBytes + (S::kKBytes / 2) * (int)qx, &tmK, &full[stage],
+                             koff + c * kBK, kr + 128 * (int32_t)qx, mc_mask);
               advance();
             }
           }
         }
         while (px_next < J && !bad) produce_px(px_next++);
+      }
+      // Every slot released by both twins' MMAs before the CTA may leave, so that no commit of
+      // the twin arrives on this CTA's barriers after it exited.
+      for (int i = 0; i < kStages && !bad && !*abort_flag; ++i) {
+        if (!mbar_wait(&empty[stage], phase ^ 1)) {
+          dev_set_error(f.err, DEV_WAIT_TIMEOUT, 401);
+          *abort_flag = 1;
+          bad = true;
+          break;
+        }
+        advance();
       }
       if (bad || *abort_flag) {
         for (int s = 0; s < kStages; ++s)
@@ -227,7 +272,7 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
         bad = true;
       };
       for (int u = cid; u < f.nunits && !bad && !*abort_flag; u += ncl) {
-        const FlashUnit w = flash_unit(f, u);
+        const FlashUnit w = pair_unit(f, u, qx);
         const int J = w.j1 - w.j0;
         auto issue_px = [&](int i) {
           const int nch = flash_chunks<kPairKeys>(f, w.j0 + i);
@@ -258,7 +303,7 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
             for (int k = 0; k < kBK / 16; ++k)
               tc_mma_f16(o_tmem, pd + 2 * k, ld + 2 * k, idesc_lo, 1u);
             issued = true;
-            tc_commit(&empty[stage]);
+            tc_commit_mc(&empty[stage], mc_mask);
             if (++stage == kStages) {
               stage = 0;
               phase ^= 1;
@@ -269,7 +314,7 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
         };
         int px_next = 0;
         for (int jj = 0; jj < J && !bad; ++jj) {
-          if (!pair_owner(jj, rank)) continue;
+          if (!pair_owner(jj, chalf)) continue;
           while (px_next <= jj - 2 && !bad) issue_px(px_next++);
           if (bad) break;
           if (n_s > 0 && !mbar_wait(sfree, (n_s - 1) & 1)) {
@@ -291,7 +336,7 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
             for (int k = 0; k < kBK / 16; ++k)
               tc_mma_f16(s_tmem, ad + 2 * k, bd + 2 * k, idesc_s, (st > 0 || k > 0) ? 1u : 0u);
             issued = true;
-            tc_commit(&empty[stage]);
+            tc_commit_mc(&empty[stage], mc_mask);
             if (++stage == kStages) {
               stage = 0;
               phase ^= 1;
@@ -384,7 +429,7 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
     };
 
     for (int u = cid; u < f.nunits && !bad && !warp_flag(abort_flag); u += ncl) {
-      const FlashUnit w = flash_unit(f, u);
+      const FlashUnit w = pair_unit(f, u, qx);
       const int J = w.j1 - w.j0;
       float m_run = -INFINITY, l_part = 0.f;
       // TK: the kTopK keys of this row half (own tiles) with the largest weights used
@@ -399,7 +444,7 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
       }
       for (int jj = 0; jj < J; ++jj, ++g) {
         const int j = w.j0 + jj;
-        if (pair_owner(jj, rank)) {
+        if (pair_owner(jj, chalf)) {
           // ---------------- own tile: softmax of S_j
           const int key0 = j * kPairKeys + kCols * half;
           float kv[kCols / 32];
@@ -590,18 +635,18 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
       if (!wait_all(lmsg, n_l & 1, 428, true)) break;
       ++n_l;
       const float l_peer = lslot[row];
-      const float l_tot = rank == 0 ? l_cta + l_peer : l_peer + l_cta;
+      const float l_tot = chalf == 0 ? l_cta + l_peer : l_peer + l_cta;
       const int r = w.tm * kBM + row;
       if (r < f.t) {
         const int64_t orow = ((int64_t)w.split * f.nb + w.b) * f.t + r;
-        // local columns [0, 128): K~ features 128 rank + c; [128, 256): V features
-        const int feat0 = (half == 0 ? 0 : 256) + 128 * (int)rank;
+        // local columns [0, 128): K~ features 128 r + c; [128, 256): V features
+        const int feat0 = (half == 0 ? 0 : 256) + 128 * (int)chalf;
         float4* dst = reinterpret_cast<float4*>(f.O + orow * 512 + feat0);
 #pragma unroll
         for (int c = 0; c < kOCols; c += 4) dst[c / 4] = make_float4(o[c], o[c + 1], o[c + 2], o[c + 3]);
-        if (rank == 0 && half == 0) f.stats[orow] = make_float2(m_run, l_tot);
+        if (chalf == 0 && half == 0) f.stats[orow] = make_float2(m_run, l_tot);
         if constexpr (TK) {
-          const int64_t cb = (orow * kTopLists + 2 * (int)rank + half) * kTopK;
+          const int64_t cb = (orow * kTopLists + 2 * (int)chalf + half) * kTopK;
 #pragma unroll
           for (int sl = 0; sl < kTopK; ++sl) {
             f.cand_key[cb + sl] = tk_key[sl];
@@ -776,19 +821,20 @@ cudaError_t launch_ca_topk_repair(const TopkRepairParams& f, int d2, cudaStream_
 // of the units late.
 int ca_pair_clusters(int num_sms) {
   static thread_local int resident = 0;
+  const int most = std::max(1, num_sms / kPairCluster);
   if (resident == 0) {
     if (cudaFuncSetAttribute(ca_pair_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              PairSmem::kBytes) != cudaSuccess) {
       cudaGetLastError();
-      return std::max(1, num_sms / 2);
+      return most;
     }
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(2 * std::max(1, num_sms / 2), 1, 1);
+    cfg.gridDim = dim3(kPairCluster * most, 1, 1);
     cfg.blockDim = dim3(kFlashThreads, 1, 1);
     cfg.dynamicSmemBytes = PairSmem::kBytes;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.x = kPairCluster;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
@@ -796,9 +842,9 @@ int ca_pair_clusters(int num_sms) {
     int n = 0;
     if (cudaOccupancyMaxActiveClusters(&n, ca_pair_kernel<false>, &cfg) != cudaSuccess || n < 1) {
       cudaGetLastError();
-      n = num_sms / 2;
+      n = most;
     }
-    resident = std::max(1, std::min(n, num_sms / 2));
+    resident = std::max(1, std::min(n, most));
   }
   return resident;
 }
@@ -810,8 +856,9 @@ cudaError_t launch_ca_pair(const Operand2D& Q, const Operand2D& K, const Operand
   if (f.D <= 0 || f.D % kBK != 0 || f.t <= 0 || f.N <= 0 || f.Np % kBK != 0 || f.Np < f.N ||
       f.nunits <= 0 || (one_pass && (f.cand_key == nullptr || f.cand_c == nullptr)))
     return cudaErrorInvalidValue;
+  // boxes: q 128 rows; k and X^T halves (128 and 64 rows), one per twin
   CUtensorMap tq, tk, tx;
-  if (!make_tmap(&tq, Q, kBM) || !make_tmap(&tk, K, kPairKeys) || !make_tmap(&tx, XT, 128))
+  if (!make_tmap(&tq, Q, kBM) || !make_tmap(&tk, K, kPairKeys / 2) || !make_tmap(&tx, XT, 64))
     return cudaErrorInvalidValue;
   auto kern = one_pass ? ca_pair_kernel<true> : ca_pair_kernel<false>;
   static thread_local bool attr_set[2] = {false, false};
@@ -827,13 +874,13 @@ cudaError_t launch_ca_pair(const Operand2D& Q, const Operand2D& K, const Operand
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.x = kPairCluster;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   const int clusters = std::max(1, std::min(f.nunits, ca_pair_clusters(num_sms)));
-  cfg.gridDim = dim3(2 * clusters, 1, 1);
+  cfg.gridDim = dim3(kPairCluster * clusters, 1, 1);
   return cudaLaunchKernelEx(&cfg, kern, tq, tk, tx, f);
 }
 
