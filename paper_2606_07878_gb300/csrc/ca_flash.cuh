@@ -575,7 +575,7 @@ inline cudaError_t launch_ca_flash(const Operand2D& Q, const Operand2D& K, const
 
 // 2d = 512 (head dim 256): the same computation on clusters of four CTAs, two query tiles x
 // two column halves; the CTAs of a query tile split the O columns and take turns computing S,
-// the CTAs of a half share their k and X^T loads (ca_pair.cu). Q, K as for launch_ca_flash;
+// the two CTAs of a half run their MMAs as one 2-SM MMA over both query tiles (ca_pair.cu). Q, K as for launch_ca_flash;
 // XT: [H*512][2*Np] fp16 (hi | lo). f.nunits counts (query-tile pair, key split, batch) units.
 // num_sms: SMs of the device (four per cluster).
 // one_pass: q, k as fp16 hi | lo with S from the hi parts only (one MMA pass) and repair

@@ -15,12 +15,14 @@
 // global memory.
 //
 // A work unit (batch b = (KV-head, cross head), two 128-row query tiles, key split) runs on
-// a cluster of four CTAs, rank = 2 x + r: query tile x of the pair, column half r. The two
-// CTAs of one half (its "twins", rank ^ 2) need the same k tiles and the same X^T columns in
-// the same order, so each loads one half of every k and X^T box and multicasts it to both:
-// the operand traffic per flop from L2 falls by a third for S and by half for P X, which is
-// what bounds the kernel (the loads of all SMs together). A ring slot is reloaded only when
-// both twins' MMAs have consumed it (their commits arrive on both CTAs' empty barriers).
+// a cluster of four CTAs, rank = 2 r + x: query tile x of the pair, column half r. The two
+// CTAs of one half (ranks 2 r and 2 r + 1, a CTA pair) need the same k tiles and X^T columns
+// in the same order, so their MMAs run as one 2-SM tcgen05.mma (cta_group::2, M = 256)
+// issued by the even CTA: each CTA holds its own query rows (or P rows) and one half of the
+// keys (or of the X^T rows) of every stage, and each SM's tensor core reads the other half
+// from its twin. Per SM this halves the shared-memory traffic of the B operand and its loads,
+// which is what bounds the S stream at M = 128 (128-byte/clock shared memory, read by the MMA
+// and written by TMA for every stage).
 //
 // Both CTAs apply the same running-maximum sequence (the owner's decision travels with the
 // tile), so their O halves, and the row sums each accumulates from its own tiles, stay on one
@@ -31,7 +33,12 @@
 // j - 2 (own or peer), so that a P buffer is never held behind a long S computation; the
 // softmax of tile j overlaps the peer's S computation of tile j + 1.
 //
-// Synchronisation between the two CTAs (all waits bounded):
+// Synchronisation inside a CTA pair: every stage's copies of both CTAs complete on the even
+// CTA's full barrier (cta_group::2 TMA); its MMA commits arrive on both CTAs' empty, sfull and
+// pempty barriers; both CTAs' softmax warps arrive on its sfree and ofree barriers, and the
+// odd CTA's warp 1 forwards each completion of its pfull barrier (its P and O rescale).
+//
+// Synchronisation between the two CTAs of a query tile (all waits bounded):
 //   mmsg   the owner's per-row running max of a tile (st.shared::cluster + remote arrive)
 //   pfull  P of the tile in this CTA's buffer and O rescaled: 8 local arrivals; for a peer
 //          tile one of them expects the 64 KB that the peer's bulk copies complete
@@ -41,7 +48,8 @@
 // Output per split: unnormalised O rows (natural feature order) and (m, l), m in log2 units;
 // ca_merge_kernel combines the splits in a fixed order.
 //
-// CTA = 10 warps: 0 TMA producer, 1 MMA issuer (TMEM owner), 2..9 softmax / output.
+// CTA = 10 warps: 0 TMA producer, 1 MMA issuer (even CTA) or P relay (odd CTA) and TMEM
+// allocation, 2..9 softmax / output.
 #include <algorithm>
 
 #include "ca_flash.cuh"
@@ -54,13 +62,18 @@ constexpr int kPairKeys = 256;   // keys per S tile
 constexpr int kPairOCols = 256;  // O columns per CTA
 constexpr uint32_t kPairPBytes = kBM * kPairKeys * 2;  // one fp16 P tile, 64 KB
 constexpr int kPairCluster = 4;  // CTAs per cluster: two query tiles x two column halves
+// S stages of an own tile issued after the own P X tile j - 2 (all of them: P X first)
+constexpr int kPxTail = 96;
 
 struct PairSmem {
+  // Per CTA: its 128 query rows and half of the keys (or of the X^T rows) of a stage; the
+  // 2-SM MMA reads the other half from the twin's shared memory at the same offset.
   static constexpr int kQBytes = kBM * kBK * 2;                // q chunk, 16 KB
-  static constexpr int kKBytes = kPairKeys * kBK * 2;          // k chunk, 32 KB
+  static constexpr int kKBytes = (kPairKeys / 2) * kBK * 2;    // half a k chunk, 16 KB
   static constexpr int kXBox = 128 * kBK * 2;                  // one 128-row X^T box, 16 KB
-  static constexpr int kStageBytes = kQBytes + kKBytes;        // = 3 X^T boxes
-  static constexpr int kStages = 3;
+  static constexpr int kXloBytes = 64 * kBK * 2;               // half the lo box, 8 KB
+  static constexpr int kStageBytes = kQBytes + kKBytes;        // 32 KB
+  static constexpr int kStages = 4;
   static constexpr int kPChunkBytes = kBM * kBK * 2;           // 128 rows x 64 keys fp16
   static constexpr int kPOffset = kStages * kStageBytes;
   static constexpr int kKinvOffset = kPOffset + (int)kPairPBytes;            // [8][128] f32
@@ -69,7 +82,7 @@ struct PairSmem {
   static constexpr int kLslotOffset = kMsgOffset + 2 * 128 * 4;              // [128] l
   static constexpr int kBarOffset = kLslotOffset + 128 * 4;
   static constexpr int kBytes = kBarOffset + 256 + 1024;
-  static_assert(3 * kXBox == kStageBytes, "an X^T chunk fills a stage");
+  static_assert(kXBox + kXloBytes <= kStageBytes, "an X^T chunk fits a stage");
   static_assert(kBytes <= 232448, "shared memory budget");
 };
 
@@ -107,13 +120,14 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::kBarOffset);
-  uint64_t* empty = full + kStages;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::kBarOffset);  // leader: stage loaded
+  uint64_t* empty = full + kStages;   // stage consumed (the leader's commit, in both CTAs)
   uint64_t* sfull = empty + kStages;  // own S tile complete in TMEM
-  uint64_t* sfree = sfull + 1;        // own S tile drained
+  uint64_t* sfree = sfull + 1;        // leader: own S tile drained in both CTAs
   uint64_t* pfull = sfree + 1;        // P of the tile in the local buffer, O rescaled
-  uint64_t* pempty = pfull + 1;       // local P X complete
-  uint64_t* ofree = pempty + 1;       // O drained at the end of a unit
+  uint64_t* ptwin = pfull + 1;        // leader: the same in the twin
+  uint64_t* pempty = ptwin + 1;       // P X complete
+  uint64_t* ofree = pempty + 1;       // leader: O drained in both CTAs at the end of a unit
   uint64_t* xb = ofree + 1;           // [4] row-value exchange per lane quarter
   uint64_t* mmsg = xb + 4;            // peer's running max of a tile (4 remote arrivals)
   uint64_t* rfree = mmsg + 1;         // peer's P X of the previous tile done (8 remote)
@@ -126,23 +140,25 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
   const int lane = threadIdx.x & 31;
   const int qchunks = f.D / kBK;
   const uint32_t rank = cluster_ctarank();
-  const uint32_t chalf = rank & 1u;  // column half; S owner parity
-  const uint32_t qx = rank >> 1;     // query tile of the unit's pair
-  const uint32_t peer = rank ^ 1u;   // same query tile, other half: the P exchange
-  // same half, other query tile: shares the k and X^T loads
-  const uint16_t mc_mask = (uint16_t)((1u << rank) | (1u << (rank ^ 2u)));
+  const uint32_t qx = rank & 1u;      // query tile of the unit's pair
+  const uint32_t chalf = rank >> 1;   // column half; S owner parity
+  const uint32_t peer = rank ^ 2u;    // same query tile, other half: the P exchange
+  const uint32_t twin = rank ^ 1u;    // same half, other query tile: the 2-SM MMA pair
+  const bool leader = qx == 0;        // issues the pair's MMAs
+  const uint16_t pair_mask = (uint16_t)((1u << rank) | (1u << twin));
   const int cid = (int)cluster_id_x(), ncl = (int)cluster_count_x();
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 2);  // this CTA's and its twin's MMA commits
+      mbar_init(&empty[s], 1);
     }
     mbar_init(sfull, 1);
-    mbar_init(sfree, kFlashSoftWarps);
+    mbar_init(sfree, 2 * kFlashSoftWarps);
     mbar_init(pfull, kFlashSoftWarps);
+    mbar_init(ptwin, 1);
     mbar_init(pempty, 1);
-    mbar_init(ofree, kFlashSoftWarps);
+    mbar_init(ofree, 2 * kFlashSoftWarps);
     for (int q = 0; q < 4; ++q) mbar_init(&xb[q], 2);
     mbar_init(mmsg, 4);
     mbar_init(rfree, kFlashSoftWarps);
@@ -154,19 +170,26 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
     tma_prefetch_desc(&tmK);
     tma_prefetch_desc(&tmX);
   }
-  if (warp == 1) {
-    tmem_alloc(tmem_slot, 512);
-    tmem_relinquish();
+  if (warp == 1) {  // one warp of each CTA of the pair allocates both TMEMs together
+    tmem_alloc_2sm(tmem_slot, 512);
+    tmem_relinquish_2sm();
   }
   tc_fence_before();
-  // Both CTAs' barriers are initialised before either arrives on the other's.
+  // Every CTA's barriers are initialised before any arrives on another's.
   cluster_sync();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  // the leader's barriers, as seen from this CTA
+  const uint32_t l_full = cluster_map(smem_u32(full), rank & ~1u);
+  const uint32_t l_sfree = cluster_map(smem_u32(sfree), rank & ~1u);
+  const uint32_t l_ofree = cluster_map(smem_u32(ofree), rank & ~1u);
+  const uint32_t l_ptwin = cluster_map(smem_u32(ptwin), rank & ~1u);
 
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------------------ TMA producer
+      // Both CTAs load their halves of every stage into their own shared memory; all the
+      // copies complete on the leader's full barrier, which the leader arms for both.
       int stage = 0;
       uint32_t phase = 0;
       uint32_t armed = 0, armed_par = 0;
@@ -178,9 +201,11 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
           bad = true;
           return nullptr;
         }
-        mbar_arrive_expect_tx(&full[stage], bytes);
-        armed |= 1u << stage;
-        armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
+        if (leader) {
+          mbar_arrive_expect_tx(&full[stage], 2 * bytes);
+          armed |= 1u << stage;
+          armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
+        }
         return smem + stage * S::kStageBytes;
       };
       auto advance = [&]() {
@@ -189,56 +214,59 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
           phase ^= 1;
         }
       };
+      const uint32_t fbar = l_full;  // + 8 stage
       for (int u = cid; u < f.nunits && !bad && !*abort_flag; u += ncl) {
         const FlashUnit w = pair_unit(f, u, qx);
         const int32_t qrow =
             (int32_t)(f.q_row0 + (int64_t)w.b * (f.q_pitch > 0 ? f.q_pitch : f.t)) + w.tm * kBM;
         const int32_t krow =
             (int32_t)(f.k_row0 + (int64_t)(f.kdiv > 0 ? w.b / f.kdiv : w.b) * f.N);
-        // this half's feature rows of X^T: K~ [128 r, +128) and V [128 r, +128); this CTA
-        // loads rows [64 x, +64) of each box for both twins
+        // this half's feature rows of X^T: K~ [128 r, +128) and V [128 r, +128). The leader
+        // holds the K~ box, the twin the V box (rows 0..127 and 128..255 of the P X operand
+        // B), and each half of the lo box of K~.
         const int32_t xk = f.xbase_row + (w.b / f.bdiv) * 512 + 128 * (int32_t)chalf;
-        const int32_t xv = xk + 256;
-        const int32_t xo = 64 * (int32_t)qx;
-        const int xs = (S::kXBox / 2) * (int)qx;  // shared-memory offset of those rows
+        const int32_t xhi = leader ? xk : xk + 256;
+        const int32_t xlo = xk + 64 * (int32_t)qx;
         const int J = w.j1 - w.j0;
         auto produce_px = [&](int i) {
           const int j = w.j0 + i;
           const int nch = flash_chunks<kPairKeys>(f, j);
           for (int c = 0; c < nch && !bad; ++c) {
-            uint8_t* sa = acquire(3 * S::kXBox);
+            uint8_t* sa = acquire(S::kXBox + S::kXloBytes);
             if (sa == nullptr) break;
             const int32_t x = j * kPairKeys + c * kBK;
-            tma_load_2d_mc(sa + xs, &tmX, &full[stage], x, xk + xo, mc_mask);
-            tma_load_2d_mc(sa + S::kXBox + xs, &tmX, &full[stage], x, xv + xo, mc_mask);
-            tma_load_2d_mc(sa + 2 * S::kXBox + xs, &tmX, &full[stage], (int32_t)(f.Np + x),
-                           xk + xo, mc_mask);
+            const uint32_t bar = fbar + 8u * (uint32_t)stage;
+            tma_load_2d_2sm(sa, &tmX, bar, x, xhi);  // 64-row boxes
+            tma_load_2d_2sm(sa + S::kXBox / 2, &tmX, bar, x, xhi + 64);
+            tma_load_2d_2sm(sa + S::kXBox, &tmX, bar, (int32_t)(f.Np + x), xlo);
             advance();
           }
         };
         int px_next = 0;
         for (int jj = 0; jj < J && !bad; ++jj) {
           if (!pair_owner(jj, chalf)) continue;
-          while (px_next <= jj - 2 && !bad) produce_px(px_next++);
+          while (px_next <= jj - 3 && !bad) produce_px(px_next++);
           const int32_t kr = krow + (w.j0 + jj) * kPairKeys;
-          for (int pass = 0; pass < kPasses && !bad; ++pass) {
+          const int nst = kPasses * qchunks, at = max(0, nst - kPxTail);
+          for (int st = 0; st < nst && !bad; ++st) {
+            if (st == at)
+              while (px_next <= jj - 2 && !bad) produce_px(px_next++);
+            const int pass = st / qchunks, c = st % qchunks;
             const int32_t qoff = pass == 2 ? f.D : 0;  // (q_hi,k_hi), (q_hi,k_lo), (q_lo,k_hi)
             const int32_t koff = pass == 1 ? f.D : 0;
-            for (int c = 0; c < qchunks; ++c) {
-              uint8_t* sa = acquire(S::kQBytes + S::kKBytes);
-              if (sa == nullptr) break;
-              tma_load_2d(sa, &tmQ, &full[stage], qoff + c * kBK, qrow);
-              // keys [128 x, +128) of the tile, for both twins
-              tma_load_2d_mc(sa + S::kQBytes + (S::kKBytes / 2) * (int)qx, &tmK, &full[stage],
-                             koff + c * kBK, kr + 128 * (int32_t)qx, mc_mask);
-              advance();
-            }
+            uint8_t* sa = acquire(S::kQBytes + S::kKBytes);
+            if (sa == nullptr) break;
+            const uint32_t bar = fbar + 8u * (uint32_t)stage;
+            tma_load_2d_2sm(sa, &tmQ, bar, qoff + c * kBK, qrow);
+            // keys [128 x, +128) of the tile: rows x of the S operand B
+            tma_load_2d_2sm(sa + S::kQBytes, &tmK, bar, koff + c * kBK, kr + 128 * (int32_t)qx);
+            advance();
           }
         }
         while (px_next < J && !bad) produce_px(px_next++);
       }
-      // Every slot released by both twins' MMAs before the CTA may leave, so that no commit of
-      // the twin arrives on this CTA's barriers after it exited.
+      // Every slot released by the leader's MMAs before the CTA may leave (its copies have
+      // landed and no commit arrives on its barriers after it exited).
       for (int i = 0; i < kStages && !bad && !*abort_flag; ++i) {
         if (!mbar_wait(&empty[stage], phase ^ 1)) {
           dev_set_error(f.err, DEV_WAIT_TIMEOUT, 401);
@@ -250,15 +278,35 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
       }
       if (bad || *abort_flag) {
         for (int s = 0; s < kStages; ++s)
-          if (armed & (1u << s)) (void)mbar_wait(&full[s], (armed_par >> s) & 1);
+          if (armed & (1u << s)) (void)mbar_wait_cluster(&full[s], (armed_par >> s) & 1);
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      // ------------------------------------------------------------ MMA issuer
-      const uint32_t idesc_s = idesc_f16(kBM, kPairKeys, TK ? 0 : 1);  // fp16 / bf16 q, k
-      const uint32_t idesc_hi = idesc_f16(kBM, kPairOCols, 0);  // fp16 P, X^T hi (K~ | V)
-      const uint32_t idesc_lo = idesc_f16(kBM, 128, 0);         // fp16 P, X^T lo (K~ half)
+    if (lane == 0 && !leader) {
+      // ------------------------------------------------------------ twin: P readiness relay
+      // The leader's P X of a tile needs P (and the O rescale) in both CTAs: forward each
+      // completion of this CTA's pfull to the leader.
+      uint32_t n = 0;
+      for (int u = cid; u < f.nunits && !*abort_flag; u += ncl) {
+        const FlashUnit w = pair_unit(f, u, qx);
+        bool bad = false;
+        for (int i = 0; i < w.j1 - w.j0; ++i, ++n) {
+          if (!mbar_wait(pfull, n & 1)) {
+            dev_set_error(f.err, DEV_WAIT_TIMEOUT, 415);
+            *abort_flag = 1;
+            bad = true;
+            break;
+          }
+          mbar_arrive_cluster(l_ptwin);
+        }
+        if (bad) break;
+      }
+    }
+    if (lane == 0 && leader) {
+      // ------------------------------------------------------------ MMA issuer (2-SM)
+      const uint32_t idesc_s = idesc_f16(2 * kBM, kPairKeys, TK ? 0 : 1);  // fp16 / bf16 q, k
+      const uint32_t idesc_hi = idesc_f16(2 * kBM, kPairOCols, 0);  // fp16 P, X^T hi (K~ | V)
+      const uint32_t idesc_lo = idesc_f16(2 * kBM, 128, 0);         // fp16 P, X^T lo (K~ half)
       const uint32_t s_tmem = tmem_base;
       const uint32_t o_tmem = tmem_base + 256;
       const uint32_t p_smem = smem_u32(smem + S::kPOffset);
@@ -276,17 +324,17 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
         const int J = w.j1 - w.j0;
         auto issue_px = [&](int i) {
           const int nch = flash_chunks<kPairKeys>(f, w.j0 + i);
-          if (i == 0 && n_units > 0 && !mbar_wait(ofree, (n_units - 1) & 1)) {
+          if (i == 0 && n_units > 0 && !mbar_wait_cluster(ofree, (n_units - 1) & 1)) {
             fail(412);
             return;
           }
-          if (!mbar_wait(pfull, n_px & 1)) {
+          if (!mbar_wait(pfull, n_px & 1) || !mbar_wait_cluster(ptwin, n_px & 1)) {
             fail(413);
             return;
           }
           tc_fence_after();
           for (int c = 0; c < nch; ++c) {
-            if (!mbar_wait(&full[stage], phase)) {
+            if (!mbar_wait_cluster(&full[stage], phase)) {
               fail(414);
               return;
             }
@@ -294,37 +342,41 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
             const uint32_t sa = smem_u32(smem + stage * S::kStageBytes);
             const uint64_t pd = sdesc_k_sw128(p_smem + c * S::kPChunkBytes);
             const uint64_t hd = sdesc_k_sw128(sa);
-            const uint64_t ld = sdesc_k_sw128(sa + 2 * S::kXBox);
+            const uint64_t ld = sdesc_k_sw128(sa + S::kXBox);
 #pragma unroll
             for (int k = 0; k < kBK / 16; ++k)
-              tc_mma_f16(o_tmem, pd + 2 * k, hd + 2 * k, idesc_hi,
-                         (i > 0 || c > 0 || k > 0) ? 1u : 0u);
+              tc_mma_f16_2sm(o_tmem, pd + 2 * k, hd + 2 * k, idesc_hi,
+                             (i > 0 || c > 0 || k > 0) ? 1u : 0u);
 #pragma unroll
             for (int k = 0; k < kBK / 16; ++k)
-              tc_mma_f16(o_tmem, pd + 2 * k, ld + 2 * k, idesc_lo, 1u);
+              tc_mma_f16_2sm(o_tmem, pd + 2 * k, ld + 2 * k, idesc_lo, 1u);
             issued = true;
-            tc_commit_mc(&empty[stage], mc_mask);
+            tc_commit_2sm_mc(&empty[stage], pair_mask);
             if (++stage == kStages) {
               stage = 0;
               phase ^= 1;
             }
           }
-          tc_commit(pempty);
+          tc_commit_2sm_mc(pempty, pair_mask);
           ++n_px;
         };
         int px_next = 0;
         for (int jj = 0; jj < J && !bad; ++jj) {
           if (!pair_owner(jj, chalf)) continue;
-          while (px_next <= jj - 2 && !bad) issue_px(px_next++);
+          while (px_next <= jj - 3 && !bad) issue_px(px_next++);
           if (bad) break;
-          if (n_s > 0 && !mbar_wait(sfree, (n_s - 1) & 1)) {
+          if (n_s > 0 && !mbar_wait_cluster(sfree, (n_s - 1) & 1)) {
             fail(410);
             break;
           }
           tc_fence_after();
-          const int nst = kPasses * qchunks;
+          const int nst = kPasses * qchunks, at = max(0, nst - kPxTail);
           for (int st = 0; st < nst; ++st) {
-            if (!mbar_wait(&full[stage], phase)) {
+            if (st == at) {
+              while (px_next <= jj - 2 && !bad) issue_px(px_next++);
+              if (bad) break;
+            }
+            if (!mbar_wait_cluster(&full[stage], phase)) {
               fail(411);
               break;
             }
@@ -334,23 +386,24 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
             const uint64_t bd = sdesc_k_sw128(sa + S::kQBytes);
 #pragma unroll
             for (int k = 0; k < kBK / 16; ++k)
-              tc_mma_f16(s_tmem, ad + 2 * k, bd + 2 * k, idesc_s, (st > 0 || k > 0) ? 1u : 0u);
+              tc_mma_f16_2sm(s_tmem, ad + 2 * k, bd + 2 * k, idesc_s,
+                             (st > 0 || k > 0) ? 1u : 0u);
             issued = true;
-            tc_commit_mc(&empty[stage], mc_mask);
+            tc_commit_2sm_mc(&empty[stage], pair_mask);
             if (++stage == kStages) {
               stage = 0;
               phase ^= 1;
             }
           }
           if (bad) break;
-          tc_commit(sfull);
+          tc_commit_2sm_mc(sfull, pair_mask);
           ++n_s;
         }
         while (px_next < J && !bad) issue_px(px_next++);
         ++n_units;
       }
       if ((bad || *abort_flag) && issued) {
-        tc_commit(drain);
+        tc_commit_2sm_mc(drain, (uint16_t)(1u << rank));
         (void)mbar_wait(drain, 0);
       }
     }
@@ -466,7 +519,7 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
           }
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive(sfree);
+          if (lane == 0) mbar_arrive_cluster(l_sfree);  // the leader's, for both CTAs
 #pragma unroll
           for (int e = 0; e < kCols / 32; ++e) kw[lane + 32 * e] = kv[e];
           __syncwarp();
@@ -623,7 +676,7 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(ofree);
+      if (lane == 0) mbar_arrive_cluster(l_ofree);
       const float l_cta = l_part + exchange(l_part, 427);
       if (bad) break;
       // row sums of both CTAs, added in rank order so that both hold the same bits
@@ -658,13 +711,13 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
   }
 
   tc_fence_before();
-  __syncthreads();
+  // Neither CTA frees its TMEM while the leader's MMAs may still write it, nor leaves while
+  // another CTA may still copy into or arrive on its shared memory.
+  cluster_sync();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, 512);
+    tmem_dealloc_2sm(tmem_base, 512);
   }
-  // Neither CTA leaves while the other may still copy into or arrive on its shared memory.
-  cluster_sync();
 }
 
 // One warp per (batch b, row r): the exact logits of the row's repair candidates replace the
@@ -856,7 +909,7 @@ cudaError_t launch_ca_pair(const Operand2D& Q, const Operand2D& K, const Operand
   if (f.D <= 0 || f.D % kBK != 0 || f.t <= 0 || f.N <= 0 || f.Np % kBK != 0 || f.Np < f.N ||
       f.nunits <= 0 || (one_pass && (f.cand_key == nullptr || f.cand_c == nullptr)))
     return cudaErrorInvalidValue;
-  // boxes: q 128 rows; k and X^T halves (128 and 64 rows), one per twin
+  // boxes: q 128 rows; k halves of 128 rows; X^T boxes of 64 rows (hi boxes in two copies)
   CUtensorMap tq, tk, tx;
   if (!make_tmap(&tq, Q, kBM) || !make_tmap(&tk, K, kPairKeys / 2) || !make_tmap(&tx, XT, 64))
     return cudaErrorInvalidValue;

@@ -108,6 +108,17 @@ STILL_DEV void tma_load_2d(void* smem_dst, const CUtensorMap* m, uint64_t* bar, 
       : "memory");
 }
 
+// A box into this CTA's shared memory whose completion counts on an mbarrier of either CTA of
+// its pair (cta_group::2; bar_cluster is a shared::cluster address).
+STILL_DEV void tma_load_2d_2sm(void* smem_dst, const CUtensorMap* m, uint32_t bar_cluster,
+                               int32_t x, int32_t y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(smem_dst)),
+      "l"(reinterpret_cast<uint64_t>(m)), "r"(bar_cluster), "r"(x), "r"(y)
+      : "memory");
+}
+
 // The same box written to the shared memory of every CTA in cta_mask (same offset in each),
 // each receiving CTA's mbarrier at the offset of bar counting the bytes it receives.
 STILL_DEV void tma_load_2d_mc(void* smem_dst, const CUtensorMap* m, uint64_t* bar, int32_t x,
@@ -153,6 +164,21 @@ STILL_DEV void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
   asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
                : "memory");
 }
+// The same for the TMEM of a CTA pair (cta_group::2): one warp of each of the two CTAs
+// executes it, and both get the same columns.
+STILL_DEV void tmem_alloc_2sm(uint32_t* slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_u32(slot)),
+               "r"(ncols)
+               : "memory");
+}
+STILL_DEV void tmem_relinquish_2sm() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+STILL_DEV void tmem_dealloc_2sm(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
 STILL_DEV void tc_fence_before() {
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
 }
@@ -168,6 +194,29 @@ STILL_DEV void tc_mma_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint3
       "setp.ne.b32 p, %4, 0;\n\t"
       "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
       "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// D[256 x N] (+)= A B^T on a CTA pair (cta_group::2), issued by the even CTA: A's rows
+// [0, 128) and B's rows [0, N/2) come from its shared memory, A's rows [128, 256) and B's rows
+// [N/2, N) from the same addresses in the odd CTA; each CTA's TMEM receives its 128 rows.
+STILL_DEV void tc_mma_f16_2sm(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                              uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive once on the mbarrier at the offset of bar in every CTA of cta_mask when all
+// previously issued cta_group::2 tcgen05.mma of this thread complete.
+STILL_DEV void tc_commit_2sm_mc(uint64_t* bar, uint16_t cta_mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(smem_u32(bar)),
+      "h"(cta_mask)
       : "memory");
 }
 
