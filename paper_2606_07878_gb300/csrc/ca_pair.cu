@@ -63,7 +63,7 @@ constexpr int kPairOCols = 256;  // O columns per CTA
 constexpr uint32_t kPairPBytes = kBM * kPairKeys * 2;  // one fp16 P tile, 64 KB
 constexpr int kPairCluster = 4;  // CTAs per cluster: two query tiles x two column halves
 // S stages of an own tile issued after the own P X tile j - 2 (all of them: P X first)
-constexpr int kPxTail = 96;
+constexpr int kPxTail = 12;
 
 struct PairSmem {
   // Per CTA: its 128 query rows and half of the keys (or of the X^T rows) of a stage; the

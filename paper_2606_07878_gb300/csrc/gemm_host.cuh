@@ -1,5 +1,6 @@
 // Host side of the tcgen05 GEMM: TMA descriptors, tile/split bookkeeping, launch.
 #pragma once
+#include <algorithm>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
 
@@ -121,6 +122,58 @@ inline cudaError_t launch_gemm(const Operand2D& A, const Operand2D& B, GemmParam
   const int grid = p.ntiles < num_sms ? p.ntiles : num_sms;
   kern<<<grid, gemm_threads<Epi>(), S::kBytes, stream>>>(ta, tb, tc, p, epi);
   return cudaGetLastError();
+}
+
+// The 2-SM form (tc_gemm2_kernel) on clusters of two CTAs: one 256 x BN tile per pair.
+template <int BN, int kRole, class Epi>
+inline cudaError_t launch_gemm_2sm(const Operand2D& A, const Operand2D& B, GemmParams p, Epi epi,
+                                   int ab_fmt, int num_sms, cudaStream_t stream,
+                                   const StoreView3D* out_view = nullptr) {
+  using S = Gemm2Smem<BN, Epi>;
+  if (!finalize_gemm<BN>(p, ab_fmt)) return cudaErrorInvalidValue;
+  CUtensorMap ta, tb, tc;
+  if (!make_tmap(&ta, A, kBM) || !make_tmap(&tb, B, BN / 2)) return cudaErrorInvalidValue;
+  std::memset(&tc, 0, sizeof(tc));
+  if (out_view != nullptr && !make_store_tmap(&tc, *out_view)) return cudaErrorInvalidValue;
+  epi.tile_cols_ = BN;
+  auto kern = tc_gemm2_kernel<BN, Epi, kRole>;
+  static thread_local int clusters = 0;  // per instantiation: resident clusters of two
+  if (clusters == 0) {
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::kBytes);
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t q = {};
+    q.gridDim = dim3(2 * std::max(1, num_sms / 2), 1, 1);
+    q.blockDim = dim3(gemm_threads<Epi>(), 1, 1);
+    q.dynamicSmemBytes = S::kBytes;
+    cudaLaunchAttribute qa[1];
+    qa[0].id = cudaLaunchAttributeClusterDimension;
+    qa[0].val.clusterDim.x = 2;
+    qa[0].val.clusterDim.y = 1;
+    qa[0].val.clusterDim.z = 1;
+    q.attrs = qa;
+    q.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &q) != cudaSuccess || n < 1) {
+      cudaGetLastError();
+      n = num_sms / 2;
+    }
+    clusters = std::max(1, std::min(n, num_sms / 2));
+  }
+  const int64_t npairs = (int64_t)((p.tiles_m + 1) / 2) * p.tiles_n * p.ksplit * p.batch;
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(gemm_threads<Epi>(), 1, 1);
+  cfg.dynamicSmemBytes = S::kBytes;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cfg.gridDim = dim3(2 * (unsigned)std::min<int64_t>(npairs, clusters), 1, 1);
+  return cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, p, epi);
 }
 
 }  // namespace still

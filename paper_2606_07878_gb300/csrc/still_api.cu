@@ -274,6 +274,20 @@ still_status run_gemm256(still_ctx* ctx, const Operand2D& A, const Operand2D& B,
   return run_gemm_bn<CLS, 256>(ctx, A, B, p, e, ab_fmt, s, view);
 }
 
+// The same on CTA pairs (2-SM MMAs, 256 x 256 tiles): for the key projection, whose 1-SM form
+// is bound by shared-memory traffic.
+template <int CLS, class Epi>
+still_status run_gemm256_2sm(still_ctx* ctx, const Operand2D& A, const Operand2D& B,
+                             GemmParams p, const Epi& e, int ab_fmt, cudaStream_t s,
+                             const StoreView3D* view = nullptr) {
+  p.err = ctx->err;
+  ctx->prof.begin(CLS, s);
+  cudaError_t r = launch_gemm_2sm<256, CLS>(A, B, p, e, ab_fmt, ctx->nsm, s, view);
+  ctx->prof.end(CLS, s);
+  if (r == cudaErrorInvalidValue) return STILL_ERR_INVALID_ARG;
+  return r == cudaSuccess ? STILL_OK : STILL_ERR_CUDA;
+}
+
 StoreView3D store_view(void* ptr, int elem_bytes, int64_t nx, int64_t ny, int64_t nz,
                        int64_t ystride, int64_t zstride, int bx, bool swz) {
   StoreView3D v;
@@ -716,11 +730,11 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       if (pos.frac) {
         EpiRopeCT<true> e;
         fill(e);
-        TRY(run_gemm256<STILL_K_KEYPROJ>(ctx, xop, wop, p, e, w_fmt, s, &kv));
+        TRY(run_gemm256_2sm<STILL_K_KEYPROJ>(ctx, xop, wop, p, e, w_fmt, s, &kv));
       } else {
         EpiRopeCT<false> e;
         fill(e);
-        TRY(run_gemm256<STILL_K_KEYPROJ>(ctx, xop, wop, p, e, w_fmt, s, &kv));
+        TRY(run_gemm256_2sm<STILL_K_KEYPROJ>(ctx, xop, wop, p, e, w_fmt, s, &kv));
       }
     }  // key projection
     // scale / |k~_n| per key (the d_l logit scale folded in)

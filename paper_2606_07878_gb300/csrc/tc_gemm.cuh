@@ -358,4 +358,252 @@ __global__ void __launch_bounds__(gemm_threads<Epi>(), 1)
   }
 }
 
+// ------------------------------------------------------------------ 2-SM form (CTA pairs)
+//
+// The same GEMM on clusters of two CTAs that compute a 256 x BN tile as one 2-SM
+// tcgen05.mma (cta_group::2, M = 256) issued by the even CTA: CTA x holds the A rows of
+// m-tile 2 m + x and rows [x BN / 2, +BN / 2) of the B tile, and each SM's tensor core reads
+// the other half of B from its twin. Per SM this halves the B operand's shared-memory traffic
+// and loads (the 1-SM kernel at 128 x 256 is bound by its shared memory: TMA writes and MMA
+// reads of every stage, with the epilogue's staging on top). Both CTAs run the epilogue on
+// their own 128 rows. Stage copies of both CTAs complete on the even CTA's full barrier; its
+// commits arrive on both CTAs' empty and tfull barriers; both CTAs' epilogue warps arrive on
+// its tempty barrier. An m-tile past the last one (odd count) is computed, and the epilogue
+// skips its rows (they lie outside M).
+template <int BN, class Epi>
+struct Gemm2Smem {
+  static constexpr int kStages = 4;
+  static constexpr int kABytes = kBM * kBK * 2;
+  static constexpr int kBBytes = (BN / 2) * kBK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kEpiOffset = kStages * kStageBytes;  // a multiple of 1024
+  static constexpr int kWarpStage = kWarpStageBytes * Epi::kStoreBufs;
+  static constexpr int kBarOffset = kEpiOffset + Epi::kWarps * kWarpStage;
+  static constexpr int kBytes = kBarOffset + 256 + 1024;
+  static_assert(kBytes <= 232448, "shared memory budget");
+};
+
+// Tile pair t: as decode_tile over ceil(tiles_m / 2) m-tile pairs; this CTA takes 2 m + x.
+__device__ __forceinline__ TileCoord decode_tile2(const GemmParams& p, int tile, int x) {
+  GemmParams q = p;
+  q.tiles_m = (p.tiles_m + 1) / 2;
+  TileCoord c = decode_tile(q, tile);
+  c.tm = 2 * c.tm + x;
+  return c;
+}
+
+template <int BN, class Epi, int kRole>
+__global__ void __launch_bounds__(gemm_threads<Epi>(), 1)
+    tc_gemm2_kernel(const __grid_constant__ CUtensorMap tmA,
+                    const __grid_constant__ CUtensorMap tmB,
+                    const __grid_constant__ CUtensorMap tmC, const GemmParams p, const Epi epi) {
+  using S = Gemm2Smem<BN, Epi>;
+  constexpr int kEpiWarps = Epi::kWarps;
+  constexpr int kStages = S::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::kBarOffset);  // even CTA's
+  uint64_t* empty = full + kStages;
+  uint64_t* tfull = empty + kStages;  // [2]
+  uint64_t* tempty = tfull + 2;       // [2], even CTA's
+  uint64_t* drain = tempty + 2;       // [1]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const int x = (int)(rank & 1u);
+  const bool leader = x == 0;
+  const uint16_t pair_mask = (uint16_t)((1u << rank) | (1u << (rank ^ 1u)));
+  const int cid = (int)cluster_id_x(), ncl = (int)cluster_count_x();
+  const int npairs = ((p.tiles_m + 1) / 2) * p.tiles_n * p.ksplit * p.batch;
+  // the 2-SM instruction descriptor: M = 256
+  const uint32_t idesc2 = (p.idesc & ~(0x1Fu << 24)) | ((uint32_t)(2 * kBM >> 4) << 24);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 2 * kEpiWarps);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) {
+    tmem_alloc_2sm(tmem_slot, 2 * BN);
+    tmem_relinquish_2sm();
+  }
+  tc_fence_before();
+  cluster_sync();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const uint32_t l_full = cluster_map(smem_u32(full), rank & ~1u);
+  const uint32_t l_tempty = cluster_map(smem_u32(tempty), rank & ~1u);
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ TMA producer
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t armed = 0, armed_par = 0;
+      bool bad = false;
+      for (int tile = cid; tile < npairs && !bad && !*abort_flag; tile += ncl) {
+        const TileCoord tc = decode_tile2(p, tile, x);
+        const int bo = tc.b / p.bdiv, bi = tc.b % p.bdiv;
+        const int64_t ar = bo * p.a_r1 + bi * p.a_r0 + (int64_t)tc.tm * kBM;
+        const int64_t ak = bo * p.a_k1 + bi * p.a_k0;
+        const int64_t br = bo * p.b_r1 + bi * p.b_r0 + (int64_t)tc.tn * BN + (BN / 2) * x;
+        const int64_t bk = bo * p.b_k1 + bi * p.b_k0;
+        int it0, it1;
+        split_range(p, tc.split, it0, it1);
+        int pass = 0, base = 0;
+        for (int it = it0; it < it1; ++it) {
+          while (pass < p.npass - 1 && it >= base + p.pass[pass].klen / kBK) {
+            base += p.pass[pass].klen / kBK;
+            ++pass;
+          }
+          const GemmPass& ps = p.pass[pass];
+          const int kk = (it - base) * kBK;
+          if (!mbar_wait(&empty[stage], phase ^ 1)) {
+            dev_set_error(p.err, DEV_WAIT_TIMEOUT, 104);
+            *abort_flag = 1;
+            bad = true;
+            break;
+          }
+          if (leader) {
+            mbar_arrive_expect_tx(&full[stage], 2 * S::kStageBytes);
+            armed |= 1u << stage;
+            armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
+          }
+          uint8_t* sa = smem + stage * S::kStageBytes;
+          const uint32_t bar = l_full + 8u * (uint32_t)stage;
+          tma_load_2d_2sm(sa, &tmA, bar, (int32_t)(ak + ps.a_koff + kk), (int32_t)(ar + ps.a_roff));
+          tma_load_2d_2sm(sa + S::kABytes, &tmB, bar, (int32_t)(bk + ps.b_koff + kk),
+                          (int32_t)(br + ps.b_roff));
+          if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      // every slot released by the even CTA's MMAs before the CTA may leave
+      for (int i = 0; i < kStages && !bad && !*abort_flag; ++i) {
+        if (!mbar_wait(&empty[stage], phase ^ 1)) {
+          dev_set_error(p.err, DEV_WAIT_TIMEOUT, 105);
+          *abort_flag = 1;
+          break;
+        }
+        if (++stage == kStages) {
+          stage = 0;
+          phase ^= 1;
+        }
+      }
+      if (*abort_flag) {
+        for (int s = 0; s < kStages; ++s)
+          if (armed & (1u << s)) (void)mbar_wait_cluster(&full[s], (armed_par >> s) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && leader) {
+      // ------------------------------------------------------------ MMA issuer (2-SM)
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool issued = false;
+      for (int tile = cid; tile < npairs && !*abort_flag; tile += ncl) {
+        const TileCoord tc = decode_tile2(p, tile, x);
+        int it0, it1;
+        split_range(p, tc.split, it0, it1);
+        if (!mbar_wait_cluster(&tempty[acc], acc_phase ^ 1)) {
+          dev_set_error(p.err, DEV_WAIT_TIMEOUT, 106);
+          *abort_flag = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+        for (int it = it0; it < it1; ++it) {
+          if (!mbar_wait_cluster(&full[stage], phase)) {
+            dev_set_error(p.err, DEV_WAIT_TIMEOUT, 107);
+            *abort_flag = 1;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + stage * S::kStageBytes);
+          const uint64_t ad = sdesc_k_sw128(sa);
+          const uint64_t bd = sdesc_k_sw128(sa + S::kABytes);
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k)
+            tc_mma_f16_2sm(d_tmem, ad + 2 * k, bd + 2 * k, idesc2, (it > it0 || k > 0) ? 1u : 0u);
+          issued = true;
+          tc_commit_2sm_mc(&empty[stage], pair_mask);
+          if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (*abort_flag) break;
+        tc_commit_2sm_mc(&tfull[acc], pair_mask);
+        if (++acc == 2) {
+          acc = 0;
+          acc_phase ^= 1;
+        }
+      }
+      if (*abort_flag && issued) {
+        tc_commit_2sm_mc(drain, (uint16_t)(1u << rank));
+        (void)mbar_wait(drain, 0);
+      }
+    }
+  } else {
+    // -------------------------------------------------------------- epilogue (warps 2..)
+    const int quarter = warp & 3;
+    const int half = (warp - 2) >> 2;
+    const int row = quarter * 32 + lane;
+    uint4* stage = reinterpret_cast<uint4*>(smem + S::kEpiOffset + (warp - 2) * S::kWarpStage);
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = cid; tile < npairs; tile += ncl) {
+      const TileCoord tc = decode_tile2(p, tile, x);
+      epi.prefetch(p, tc, row, half);
+      bool ok = mbar_wait(&tfull[acc], acc_phase);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok || warp_flag(abort_flag)) {
+        if (lane == 0 && !ok) {
+          dev_set_error(p.err, DEV_WAIT_TIMEOUT, 108);
+          *abort_flag = 1;
+        }
+        break;
+      }
+      tc_fence_after();
+      const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * BN);
+      epi(p, tc, row, taddr, half, stage, &tmC);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(l_tempty + 8u * (uint32_t)acc);
+      if (++acc == 2) {
+        acc = 0;
+        acc_phase ^= 1;
+      }
+    }
+    if (lane == 0) bulk_wait_all();
+  }
+
+  tc_fence_before();
+  // No CTA frees its TMEM while the even CTA's MMAs may still write it, nor leaves while the
+  // other may still copy into or arrive on its shared memory.
+  cluster_sync();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_2sm(tmem_base, 2 * BN);
+  }
+}
+
 }  // namespace still
