@@ -64,12 +64,21 @@ def describe(name, wl, t):
 # The fused cross-attention kernel (the scores GEMM entry is kept for the record: no workload
 # takes it any more).
 TRAFFIC = {
-    "scores": {"files": ["tc_gemm.cuh", "epilogues.cuh"], "kernel_hash": None,
-               "bytes_per_launch": None, "workload": None, "profile": None},
-    # 1.287 GB read + 0.132 GB written per launch (profiles/ca_fused_qwen7b_8k_t1024.md)
-    "ca_fused": {"files": ["ca_flash.cuh", "ptx.cuh"], "kernel_hash": "1024714c3c99a223",
-                 "bytes_per_launch": 1.4191e9, "workload": ("qwen7b_8k", 1024),
-                 "profile": "profiles/ca_fused_qwen7b_8k_t1024.md"},
+    "scores": [],
+    # one entry per captured workload
+    "ca_fused": [
+        # 1.287 GB read + 0.132 GB written per launch (profiles/ca_fused_qwen7b_8k_t1024.md)
+        {"files": ["ca_flash.cuh", "ptx.cuh"], "kernel_hash": "1024714c3c99a223",
+         "bytes_per_launch": 1.4191e9, "workload": ("qwen7b_8k", 1024),
+         "profile": "profiles/ca_fused_qwen7b_8k_t1024.md"},
+        # the head-dim-256 kernel captured on one KV-head of a 16k-token cache (1.231 GB read
+        # + 0.086 GB written, profiles/ca_pair_gemma_n16k_t655.md), scaled by the units of a
+        # full-size launch (2 KV-heads x 131072 tokens: x16); its traffic (k read once, X^T,
+        # partials) grows in proportion
+        {"files": ["ca_pair.cu", "ca_flash.cuh", "ptx.cuh"], "kernel_hash": "73816e4e32bc125d",
+         "bytes_per_launch": 16 * 1.3165e9, "workload": ("gemma_128k", 655),
+         "profile": "profiles/ca_pair_gemma_n16k_t655.md"},
+    ],
 }
 
 
@@ -191,7 +200,7 @@ def algorithmic_flops(wl, t, N):
           + 2 * t * H * n * 2 * d * D + 2 * t * H * n * D * D)
     sa = 6 * t * H * D * n * D + 4 * t * t * H * n * D + 2 * t * H * n * D * D
     # Every block's cross-attention is one fused kernel (a block that feeds another in its
-    # split-precision form, P X in 2.5 passes; 2d = 512 on clusters of two CTAs).
+    # split-precision form, P X in 2.5 passes; 2d = 512 on clusters of four CTAs).
     fused = True
     return {"total": n_ca * ca + nb * (sa + 4 * t * H * D * F) + 4 * t * H * D * d,
             "scores": n_ca * 2 * t * N * H * n * kw, "px": n_ca * 2 * t * N * H * n * 2 * d,
@@ -697,14 +706,15 @@ def main():
               else 3 * fl["scores_gemm"])
     per_launch_flops = alg * L / max(n_k, 1)
     achieved = per_launch_flops / (ms_k / max(n_k, 1) / 1e3) / 1e12 if ms_k > 0 else None
-    tr = TRAFFIC[kname]
     traffic = None
-    if tr["kernel_hash"] == _kernel_hash(tr["files"]) and tr["workload"] == (name, t):
-        traffic = tr["bytes_per_launch"]
+    for tr in TRAFFIC[kname]:
+        if tr["workload"] == (name, t) and tr["kernel_hash"] == _kernel_hash(tr["files"]):
+            traffic = tr["bytes_per_launch"]
     kdesc = ("ca_fused (" + ("1-pass fp16 scores with a top-k logit repair" if qk_passes == 1
                              else "3-pass split-bf16 scores")
              + " + online softmax + P X, one tcgen05 kernel"
-             + ("; clusters of two CTAs that split the 512 O columns" if 2 * d == 512 else "")
+             + ("; clusters of four CTAs: two query tiles x two O-column halves, 2-SM MMAs"
+                if 2 * d == 512 else "")
              + ("; the first block's launches in split fp16 with P hi + lo)"
                 if wl.get("n_blocks", 1) > 1 and wl.get("cross_every_block", 1) else ")")
              if fused else "scores (3-pass split-bf16 tcgen05 GEMM)")
