@@ -119,17 +119,6 @@ STILL_DEV void tma_load_2d_2sm(void* smem_dst, const CUtensorMap* m, uint32_t ba
       : "memory");
 }
 
-// The same box written to the shared memory of every CTA in cta_mask (same offset in each),
-// each receiving CTA's mbarrier at the offset of bar counting the bytes it receives.
-STILL_DEV void tma_load_2d_mc(void* smem_dst, const CUtensorMap* m, uint64_t* bar, int32_t x,
-                              int32_t y, uint16_t cta_mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
-      ".multicast::cluster [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(smem_dst)),
-      "l"(reinterpret_cast<uint64_t>(m)), "r"(smem_u32(bar)), "r"(x), "r"(y), "h"(cta_mask)
-      : "memory");
-}
-
 // 3-D tiled store of one box from shared memory (bulk async group of the calling thread).
 STILL_DEV void tma_store_3d(const CUtensorMap* m, const void* smem_src, int32_t x, int32_t y,
                             int32_t z) {
@@ -225,16 +214,6 @@ STILL_DEV void tc_commit(uint64_t* bar) {
   asm volatile(
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
           smem_u32(bar))
-      : "memory");
-}
-
-// The same completion arriving once on the mbarrier at the offset of bar in every CTA of
-// cta_mask.
-STILL_DEV void tc_commit_mc(uint64_t* bar, uint16_t cta_mask) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
-      " [%0], %1;" ::"r"(smem_u32(bar)),
-      "h"(cta_mask)
       : "memory");
 }
 
@@ -430,11 +409,3 @@ STILL_DEV void bulk_copy_to_cluster(uint32_t dst_cluster, const void* src, uint3
       : "memory");
 }
 
-// Prefetch of one box of a tiled tensor into L2 (no shared memory, no completion to wait for).
-// x (innermost coordinate) * 2 bytes must be a multiple of 16: callers pass multiples of 64.
-STILL_DEV void tma_prefetch_l2_2d(const CUtensorMap* m, int32_t x, int32_t y) {
-  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
-                   reinterpret_cast<uint64_t>(m)),
-               "r"(x), "r"(y)
-               : "memory");
-}
