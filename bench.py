@@ -75,7 +75,7 @@ TRAFFIC = {
         # + 0.086 GB written, profiles/ca_pair_gemma_n16k_t655.md), scaled by the units of a
         # full-size launch (2 KV-heads x 131072 tokens: x16); its traffic (k read once, X^T,
         # partials) grows in proportion
-        {"files": ["ca_pair.cu", "ca_flash.cuh", "ptx.cuh"], "kernel_hash": "73816e4e32bc125d",
+        {"files": ["ca_pair.cu", "ca_flash.cuh", "ptx.cuh"], "kernel_hash": "f9ea4b8c7c0d1bea",
          "bytes_per_launch": 16 * 1.3165e9, "workload": ("gemma_128k", 655),
          "profile": "profiles/ca_pair_gemma_n16k_t655.md"},
     ],
