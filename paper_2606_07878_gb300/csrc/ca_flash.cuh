@@ -63,14 +63,16 @@ constexpr float kRescaleLog2 = 8.f;
 template <int D2, bool EX = false>
 struct FlashSmem {
   static_assert(D2 == 128 || D2 == 256, "2d must be 128 or 256");
+  // Per CTA of a pair: its own q rows and half of the B operand of every stage (the 2-SM MMA
+  // reads the other half from the twin's shared memory at the same offset).
   static constexpr int kKeys = EX ? 128 : kFlashKeys;     // keys per S tile
   static constexpr int kQBytes = kBM * kBK * 2;            // q chunk, 16 KB
-  static constexpr int kKBytes = kKeys * kBK * 2;          // k chunk
-  static constexpr int kXhiBytes = D2 * kBK * 2;           // X^T hi chunk
-  static constexpr int kXloBytes = (D2 / 2) * kBK * 2;     // X^T lo chunk (key half)
+  static constexpr int kKBytes = (kKeys / 2) * kBK * 2;    // half a k chunk
+  static constexpr int kXhiBytes = (D2 / 2) * kBK * 2;     // half the X^T hi chunk
+  static constexpr int kXloBytes = (D2 / 4) * kBK * 2;     // half the X^T lo chunk (key half)
   static constexpr int kStageBytes = (kQBytes + kKBytes) > (kXhiBytes + kXloBytes)
                                          ? (kQBytes + kKBytes) : (kXhiBytes + kXloBytes);
-  static constexpr int kStages = 3;
+  static constexpr int kStages = 4;
   static constexpr int kPChunkBytes = kBM * kBK * 2;       // 128 rows x 64 keys fp16
   static constexpr int kPChunks = kKeys / kBK;             // chunks of one P tile (hi)
   static constexpr int kPOffset = kStages * kStageBytes;
@@ -79,6 +81,7 @@ struct FlashSmem {
   static constexpr int kBarOffset = kXchOffset + 2 * 2 * 128 * 4;
   static constexpr int kBytes = kBarOffset + 256 + 1024;
   static_assert(kXhiBytes + kXloBytes <= kStageBytes, "X chunk fits a stage");
+  static_assert(kStageBytes % 1024 == 0 && kXhiBytes % 1024 == 0, "swizzle-atom alignment");
   static_assert(kBytes <= 232448, "shared memory budget");
 };
 
@@ -86,10 +89,14 @@ struct FlashUnit {
   int b, tm, split, j0, j1;
 };
 
-__device__ __forceinline__ FlashUnit flash_unit(const FlashParams& f, int u) {
+// Unit u of the CTA pairs: query tiles 2 m and 2 m + 1 (m fastest), then the key split, then
+// the batch; the CTA x of the pair takes query tile 2 m + x (one past the last tile, for an odd
+// count, is computed and not stored).
+__device__ __forceinline__ FlashUnit flash_pair_unit(const FlashParams& f, int u, uint32_t x) {
+  const int mp = (f.tiles_m + 1) / 2;
   FlashUnit r;
-  r.tm = u % f.tiles_m;
-  int q = u / f.tiles_m;
+  r.tm = 2 * (u % mp) + (int)x;
+  const int q = u / mp;
   r.split = q % f.nsplit;
   r.b = q / f.nsplit;
   r.j0 = (int)(((int64_t)f.tiles_k * r.split) / f.nsplit);
@@ -117,13 +124,14 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::kBarOffset);
-  uint64_t* empty = full + kStages;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::kBarOffset);  // even CTA: stage loaded
+  uint64_t* empty = full + kStages;   // stage consumed (the even CTA's commit, in both CTAs)
   uint64_t* sfull = empty + kStages;  // S tile complete in TMEM
-  uint64_t* sfree = sfull + 1;        // S tile drained by the softmax warps
+  uint64_t* sfree = sfull + 1;        // even CTA: S tile drained in both CTAs
   uint64_t* pfull = sfree + 1;        // P tile written (and O rescaled if needed)
-  uint64_t* pempty = pfull + 1;       // PX MMA complete (P buffer free, O up to date)
-  uint64_t* ofree = pempty + 1;       // O drained at the end of a unit
+  uint64_t* ptwin = pfull + 1;        // even CTA: the same in the odd CTA
+  uint64_t* pempty = ptwin + 1;       // PX MMA complete (P buffer free, O up to date)
+  uint64_t* ofree = pempty + 1;       // even CTA: O drained in both CTAs at the end of a unit
   uint64_t* xb = ofree + 1;           // [4] row-value exchange per lane quarter
   uint64_t* drain = xb + 4;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
@@ -132,6 +140,11 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int qchunks = f.D / kBK;
+  const uint32_t rank = cluster_ctarank();
+  const uint32_t qx = rank & 1u;  // query tile of the unit's pair
+  const bool leader = qx == 0;    // issues the pair's MMAs
+  const uint16_t pair_mask = (uint16_t)(3u << (rank & ~1u));
+  const int cid = (int)cluster_id_x(), ncl = (int)cluster_count_x();
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -139,10 +152,11 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
       mbar_init(&empty[s], 1);
     }
     mbar_init(sfull, 1);
-    mbar_init(sfree, kFlashSoftWarps);
+    mbar_init(sfree, 2 * kFlashSoftWarps);
     mbar_init(pfull, kFlashSoftWarps);
+    mbar_init(ptwin, 1);
     mbar_init(pempty, 1);
-    mbar_init(ofree, kFlashSoftWarps);
+    mbar_init(ofree, 2 * kFlashSoftWarps);
     for (int q = 0; q < 4; ++q) mbar_init(&xb[q], 2);
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -152,18 +166,25 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
     tma_prefetch_desc(&tmXhi);
     tma_prefetch_desc(&tmXlo);
   }
-  if (warp == 1) {
-    tmem_alloc(tmem_slot, 512);
-    tmem_relinquish();
+  if (warp == 1) {  // one warp of each CTA of the pair allocates both TMEMs together
+    tmem_alloc_2sm(tmem_slot, 512);
+    tmem_relinquish_2sm();
   }
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  // the even CTA's barriers, as seen from this CTA
+  const uint32_t l_full = cluster_map(smem_u32(full), rank & ~1u);
+  const uint32_t l_sfree = cluster_map(smem_u32(sfree), rank & ~1u);
+  const uint32_t l_ofree = cluster_map(smem_u32(ofree), rank & ~1u);
+  const uint32_t l_ptwin = cluster_map(smem_u32(ptwin), rank & ~1u);
 
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------------------ TMA producer
+      // Both CTAs load their halves of every stage into their own shared memory; all the
+      // copies complete on the even CTA's full barrier, which it arms for both.
       int stage = 0;
       uint32_t phase = 0;
       uint32_t armed = 0, armed_par = 0;
@@ -175,9 +196,11 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
           bad = true;
           return nullptr;
         }
-        mbar_arrive_expect_tx(&full[stage], bytes);
-        armed |= 1u << stage;
-        armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
+        if (leader) {
+          mbar_arrive_expect_tx(&full[stage], 2 * bytes);
+          armed |= 1u << stage;
+          armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
+        }
         return smem + stage * S::kStageBytes;
       };
       auto advance = [&]() {
@@ -186,25 +209,31 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
           phase ^= 1;
         }
       };
-      for (int u = blockIdx.x; u < f.nunits && !bad && !*abort_flag; u += gridDim.x) {
-        const FlashUnit w = flash_unit(f, u);
+      for (int u = cid; u < f.nunits && !bad && !*abort_flag; u += ncl) {
+        const FlashUnit w = flash_pair_unit(f, u, qx);
         const int32_t qrow =
             (int32_t)(f.q_row0 + (int64_t)w.b * (f.q_pitch > 0 ? f.q_pitch : f.t)) + w.tm * kBM;
         const int32_t krow =
             (int32_t)(f.k_row0 + (int64_t)(f.kdiv > 0 ? w.b / f.kdiv : w.b) * f.N);
+        // X^T rows of this CTA: hi rows [D2/2 x, +D2/2) (K~ in the even CTA, V in the odd one),
+        // lo rows [D2/4 x, +D2/4) of K~
         const int32_t xrow = f.xbase_row + (w.b / f.bdiv) * D2;
+        const int32_t xhi = xrow + (D2 / 2) * (int32_t)qx;
+        const int32_t xlo = xrow + (D2 / 4) * (int32_t)qx;
         const int J = w.j1 - w.j0;
         for (int jj = 0; jj <= J && !bad; ++jj) {
           if (jj < J) {
-            const int32_t kr = krow + (w.j0 + jj) * kKeys;
+            // keys [kKeys/2 x, +kKeys/2) of the tile: rows x of the S operand B
+            const int32_t kr = krow + (w.j0 + jj) * kKeys + (kKeys / 2) * (int32_t)qx;
             for (int pass = 0; pass < 3 && !bad; ++pass) {
               const int32_t qoff = pass == 2 ? f.D : 0;  // (q_hi,k_hi), (q_hi,k_lo), (q_lo,k_hi)
               const int32_t koff = pass == 1 ? f.D : 0;
               for (int c = 0; c < qchunks; ++c) {
-                uint8_t* sa = acquire(S::kQBytes + S::kKBytes);  // the bytes these two copies bring
+                uint8_t* sa = acquire(S::kQBytes + S::kKBytes);  // this CTA's bytes
                 if (sa == nullptr) break;
-                tma_load_2d(sa, &tmQ, &full[stage], qoff + c * kBK, qrow);
-                tma_load_2d(sa + S::kQBytes, &tmK, &full[stage], koff + c * kBK, kr);
+                const uint32_t bar = l_full + 8u * (uint32_t)stage;
+                tma_load_2d_2sm(sa, &tmQ, bar, qoff + c * kBK, qrow);
+                tma_load_2d_2sm(sa + S::kQBytes, &tmK, bar, koff + c * kBK, kr);
                 advance();
               }
             }
@@ -216,24 +245,53 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
               uint8_t* sa = acquire(S::kXhiBytes + S::kXloBytes);
               if (sa == nullptr) break;
               const int32_t x = j * kKeys + c * kBK;
-              tma_load_2d(sa, &tmXhi, &full[stage], x, xrow);
-              tma_load_2d(sa + S::kXhiBytes, &tmXlo, &full[stage], (int32_t)(f.Np + x), xrow);
+              const uint32_t bar = l_full + 8u * (uint32_t)stage;
+              tma_load_2d_2sm(sa, &tmXhi, bar, x, xhi);
+              tma_load_2d_2sm(sa + S::kXhiBytes, &tmXlo, bar, (int32_t)(f.Np + x), xlo);
               advance();
             }
           }
         }
       }
+      // every slot released by the even CTA's MMAs before the CTA may leave
+      for (int i = 0; i < kStages && !bad && !*abort_flag; ++i) {
+        if (!mbar_wait(&empty[stage], phase ^ 1)) {
+          dev_set_error(f.err, DEV_WAIT_TIMEOUT, 301);
+          *abort_flag = 1;
+          bad = true;
+          break;
+        }
+        advance();
+      }
       if (bad || *abort_flag) {
         for (int s = 0; s < kStages; ++s)
-          if (armed & (1u << s)) (void)mbar_wait(&full[s], (armed_par >> s) & 1);
+          if (armed & (1u << s)) (void)mbar_wait_cluster(&full[s], (armed_par >> s) & 1);
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      // ------------------------------------------------------------ MMA issuer
-      const uint32_t idesc_s = idesc_f16(kBM, kKeys, EX ? 0 : 1);  // fp16 (EX) or bf16 q, k
-      const uint32_t idesc_hi = idesc_f16(kBM, D2, 0);         // fp16 P, X^T hi
-      const uint32_t idesc_lo = idesc_f16(kBM, D2 / 2, 0);     // fp16 P, X^T lo (key half)
+    if (lane == 0 && !leader) {
+      // ------------------------------------------------------------ odd CTA: P readiness relay
+      uint32_t n = 0;
+      for (int u = cid; u < f.nunits && !*abort_flag; u += ncl) {
+        const FlashUnit w = flash_pair_unit(f, u, qx);
+        bool bad = false;
+        for (int i = 0; i < w.j1 - w.j0; ++i, ++n) {
+          if (!mbar_wait(pfull, n & 1)) {
+            dev_set_error(f.err, DEV_WAIT_TIMEOUT, 315);
+            *abort_flag = 1;
+            bad = true;
+            break;
+          }
+          mbar_arrive_cluster(l_ptwin);
+        }
+        if (bad) break;
+      }
+    }
+    if (lane == 0 && leader) {
+      // ------------------------------------------------------------ MMA issuer (2-SM)
+      const uint32_t idesc_s = idesc_f16(2 * kBM, kKeys, EX ? 0 : 1);  // fp16 (EX) or bf16 q, k
+      const uint32_t idesc_hi = idesc_f16(2 * kBM, D2, 0);         // fp16 P, X^T hi
+      const uint32_t idesc_lo = idesc_f16(2 * kBM, D2 / 2, 0);     // fp16 P, X^T lo (key half)
       const uint32_t s_tmem = tmem_base;
       const uint32_t o_tmem = tmem_base + 256;
       const uint32_t p_smem = smem_u32(smem + S::kPOffset);
@@ -246,19 +304,19 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
         *abort_flag = 1;
         bad = true;
       };
-      for (int u = blockIdx.x; u < f.nunits && !bad && !*abort_flag; u += gridDim.x) {
-        const FlashUnit w = flash_unit(f, u);
+      for (int u = cid; u < f.nunits && !bad && !*abort_flag; u += ncl) {
+        const FlashUnit w = flash_pair_unit(f, u, qx);
         const int J = w.j1 - w.j0;
         for (int jj = 0; jj <= J && !bad; ++jj) {
           if (jj < J) {
-            if (n_s > 0 && !mbar_wait(sfree, (n_s - 1) & 1)) {
+            if (n_s > 0 && !mbar_wait_cluster(sfree, (n_s - 1) & 1)) {
               fail(310);
               break;
             }
             tc_fence_after();
             const int nst = 3 * qchunks;
             for (int st = 0; st < nst; ++st) {
-              if (!mbar_wait(&full[stage], phase)) {
+              if (!mbar_wait_cluster(&full[stage], phase)) {
                 fail(311);
                 break;
               }
@@ -268,32 +326,33 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
               const uint64_t bd = sdesc_k_sw128(sa + S::kQBytes);
 #pragma unroll
               for (int k = 0; k < kBK / 16; ++k)
-                tc_mma_f16(s_tmem, ad + 2 * k, bd + 2 * k, idesc_s, (st > 0 || k > 0) ? 1u : 0u);
+                tc_mma_f16_2sm(s_tmem, ad + 2 * k, bd + 2 * k, idesc_s,
+                               (st > 0 || k > 0) ? 1u : 0u);
               issued = true;
-              tc_commit(&empty[stage]);
+              tc_commit_2sm_mc(&empty[stage], pair_mask);
               if (++stage == kStages) {
                 stage = 0;
                 phase ^= 1;
               }
             }
             if (bad) break;
-            tc_commit(sfull);
+            tc_commit_2sm_mc(sfull, pair_mask);
             ++n_s;
           }
           if (jj >= 1) {
             const int j = w.j0 + jj - 1;
             const int nch = flash_chunks<kKeys>(f, j);
-            if (jj == 1 && n_units > 0 && !mbar_wait(ofree, (n_units - 1) & 1)) {
+            if (jj == 1 && n_units > 0 && !mbar_wait_cluster(ofree, (n_units - 1) & 1)) {
               fail(312);
               break;
             }
-            if (!mbar_wait(pfull, n_px & 1)) {
+            if (!mbar_wait(pfull, n_px & 1) || !mbar_wait_cluster(ptwin, n_px & 1)) {
               fail(313);
               break;
             }
             tc_fence_after();
             for (int c = 0; c < nch; ++c) {
-              if (!mbar_wait(&full[stage], phase)) {
+              if (!mbar_wait_cluster(&full[stage], phase)) {
                 fail(314);
                 break;
               }
@@ -304,32 +363,33 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
               const uint64_t ld = sdesc_k_sw128(sa + S::kXhiBytes);
 #pragma unroll
               for (int k = 0; k < kBK / 16; ++k)
-                tc_mma_f16(o_tmem, pd + 2 * k, hd + 2 * k, idesc_hi,
-                           (jj > 1 || c > 0 || k > 0) ? 1u : 0u);
+                tc_mma_f16_2sm(o_tmem, pd + 2 * k, hd + 2 * k, idesc_hi,
+                               (jj > 1 || c > 0 || k > 0) ? 1u : 0u);
 #pragma unroll
-              for (int k = 0; k < kBK / 16; ++k) tc_mma_f16(o_tmem, pd + 2 * k, ld + 2 * k, idesc_lo, 1u);
+              for (int k = 0; k < kBK / 16; ++k)
+                tc_mma_f16_2sm(o_tmem, pd + 2 * k, ld + 2 * k, idesc_lo, 1u);
               if constexpr (EX) {  // + P_lo X^T hi
                 const uint64_t pld =
                     sdesc_k_sw128(p_smem + (S::kPChunks + c) * S::kPChunkBytes);
 #pragma unroll
                 for (int k = 0; k < kBK / 16; ++k)
-                  tc_mma_f16(o_tmem, pld + 2 * k, hd + 2 * k, idesc_hi, 1u);
+                  tc_mma_f16_2sm(o_tmem, pld + 2 * k, hd + 2 * k, idesc_hi, 1u);
               }
-              tc_commit(&empty[stage]);
+              tc_commit_2sm_mc(&empty[stage], pair_mask);
               if (++stage == kStages) {
                 stage = 0;
                 phase ^= 1;
               }
             }
             if (bad) break;
-            tc_commit(pempty);
+            tc_commit_2sm_mc(pempty, pair_mask);
             ++n_px;
           }
         }
         ++n_units;
       }
       if ((bad || *abort_flag) && issued) {
-        tc_commit(drain);
+        tc_commit_2sm_mc(drain, (uint16_t)(1u << rank));
         (void)mbar_wait(drain, 0);
       }
     }
@@ -369,8 +429,8 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
       return ok ? slot[(1 - half) * 128 + row] : mine;
     };
 
-    for (int u = blockIdx.x; u < f.nunits && !bad && !warp_flag(abort_flag); u += gridDim.x) {
-      const FlashUnit w = flash_unit(f, u);
+    for (int u = cid; u < f.nunits && !bad && !warp_flag(abort_flag); u += ncl) {
+      const FlashUnit w = flash_pair_unit(f, u, qx);
       const int J = w.j1 - w.j0;
       float m_run = -INFINITY, l_part = 0.f;
       for (int jj = 0; jj < J; ++jj) {
@@ -395,7 +455,7 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(sfree);
+        if (lane == 0) mbar_arrive_cluster(l_sfree);  // the even CTA's, for both CTAs
         // scale per key (log2 units), mask keys past N, tile max
 #pragma unroll
         for (int e = 0; e < kCols / 32; ++e) kw[lane + 32 * e] = kv[e];
@@ -508,7 +568,7 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(ofree);
+      if (lane == 0) mbar_arrive_cluster(l_ofree);
       const float l_tot = l_part + exchange(l_part, 324);
       if (bad) break;
       const int r = w.tm * kBM + row;
@@ -523,10 +583,12 @@ __global__ void __launch_bounds__(kFlashThreads, 1)
   }
 
   tc_fence_before();
-  __syncthreads();
+  // Neither CTA frees its TMEM while the even CTA's MMAs may still write it, nor leaves while
+  // the other may still copy into or arrive on its shared memory.
+  cluster_sync();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, 512);
+    tmem_dealloc_2sm(tmem_base, 512);
   }
 }
 
@@ -549,6 +611,8 @@ inline int flash_split(int64_t base_units, int tiles_k, int num_sms, int max_spl
 
 // Q: [nb*t][2D] bf16 (hi | lo), K: [nb*N][2D] bf16 (hi | lo), XT: [H*2d][2*Np] fp16 (hi | lo);
 // EX: Q and K fp16 hi | lo, key tiles of S::kKeys = 128 (f.tiles_k counts those).
+// The kernel runs on CTA pairs (clusters of two): f.nunits counts (query-tile pair, key split,
+// batch) units.
 template <int D2, bool EX = false>
 inline cudaError_t launch_ca_flash(const Operand2D& Q, const Operand2D& K, const Operand2D& XT,
                                    const FlashParams& f, int num_sms, cudaStream_t stream) {
@@ -556,21 +620,48 @@ inline cudaError_t launch_ca_flash(const Operand2D& Q, const Operand2D& K, const
   if (f.D <= 0 || f.D % kBK != 0 || f.t <= 0 || f.N <= 0 || f.Np % kBK != 0 || f.Np < f.N ||
       f.nunits <= 0)
     return cudaErrorInvalidValue;
+  // boxes per CTA of a pair: its q rows, half of the k tile, half of the X^T hi and lo rows
   CUtensorMap tq, tk, thi, tlo;
-  if (!make_tmap(&tq, Q, kBM) || !make_tmap(&tk, K, S::kKeys) || !make_tmap(&thi, XT, D2) ||
-      !make_tmap(&tlo, XT, D2 / 2))
+  if (!make_tmap(&tq, Q, kBM) || !make_tmap(&tk, K, S::kKeys / 2) ||
+      !make_tmap(&thi, XT, D2 / 2) || !make_tmap(&tlo, XT, D2 / 4))
     return cudaErrorInvalidValue;
   auto kern = ca_flash_kernel<D2, EX>;
-  static thread_local bool attr_set = false;
-  if (!attr_set) {
+  static thread_local int clusters = 0;  // resident CTA pairs (per instantiation)
+  if (clusters == 0) {
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::kBytes);
     if (e != cudaSuccess) return e;
-    attr_set = true;
+    cudaLaunchConfig_t q = {};
+    q.gridDim = dim3(2 * std::max(1, num_sms / 2), 1, 1);
+    q.blockDim = dim3(kFlashThreads, 1, 1);
+    q.dynamicSmemBytes = S::kBytes;
+    cudaLaunchAttribute qa[1];
+    qa[0].id = cudaLaunchAttributeClusterDimension;
+    qa[0].val.clusterDim.x = 2;
+    qa[0].val.clusterDim.y = 1;
+    qa[0].val.clusterDim.z = 1;
+    q.attrs = qa;
+    q.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &q) != cudaSuccess || n < 1) {
+      cudaGetLastError();
+      n = num_sms / 2;
+    }
+    clusters = std::max(1, std::min(n, num_sms / 2));
   }
-  const int grid = f.nunits < num_sms ? f.nunits : num_sms;
-  kern<<<grid, kFlashThreads, S::kBytes, stream>>>(tq, tk, thi, tlo, f);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(kFlashThreads, 1, 1);
+  cfg.dynamicSmemBytes = S::kBytes;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cfg.gridDim = dim3(2 * (unsigned)std::min(f.nunits, clusters), 1, 1);
+  return cudaLaunchKernelEx(&cfg, kern, tq, tk, thi, tlo, f);
 }
 
 // 2d = 512 (head dim 256): the same computation on clusters of four CTAs, two query tiles x

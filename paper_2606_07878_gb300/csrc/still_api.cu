@@ -762,9 +762,9 @@ still_status compact_one(still_ctx* ctx, const LayerW& L, const KVSource& src,
       fp.tiles_m = (t + kBM - 1) / kBM;
       const int fkeys = exact ? FlashSmem<256, true>::kKeys : kFlashKeys;
       fp.tiles_k = (int)((N + fkeys - 1) / fkeys);
-      // 2d = 512: a unit (two query tiles) occupies a cluster of four SMs
-      const int slots = d == 256 ? ca_pair_clusters(ctx->nsm) : ctx->nsm;
-      const int mt = d == 256 ? (fp.tiles_m + 1) / 2 : fp.tiles_m;
+      // a unit holds two query tiles: a CTA pair (2d <= 256) or a cluster of four (2d = 512)
+      const int slots = d == 256 ? ca_pair_clusters(ctx->nsm) : ctx->nsm / 2;
+      const int mt = (fp.tiles_m + 1) / 2;
       fp.nsplit = flash_split((int64_t)mt * nbl, fp.tiles_k, slots, kMaxFlashSplit);
       const int64_t nunits = (int64_t)mt * nbl * fp.nsplit;
       if (nunits > 0x7fffffff || (int64_t)nbl * N > 0x7fffffff) return STILL_ERR_UNSUPPORTED;
