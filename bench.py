@@ -67,15 +67,16 @@ TRAFFIC = {
     "scores": [],
     # one entry per captured workload
     "ca_fused": [
-        # 1.287 GB read + 0.132 GB written per launch (profiles/ca_fused_qwen7b_8k_t1024.md)
-        {"files": ["ca_flash.cuh", "ptx.cuh"], "kernel_hash": "1024714c3c99a223",
-         "bytes_per_launch": 1.4191e9, "workload": ("qwen7b_8k", 1024),
+        # 1.313 GB read + 0.127 GB written per launch (profiles/ca_fused_qwen7b_8k_t1024.md,
+        # the CTA-pair kernel, whose source is ca_flash.cuh)
+        {"files": ["ca_flash.cuh"], "kernel_hash": "1e46c485c8c9bbab",
+         "bytes_per_launch": 1.4405e9, "workload": ("qwen7b_8k", 1024),
          "profile": "profiles/ca_fused_qwen7b_8k_t1024.md"},
-        # the head-dim-256 kernel captured on one KV-head of a 16k-token cache (1.231 GB read
-        # + 0.086 GB written, profiles/ca_pair_gemma_n16k_t655.md), scaled by the units of a
-        # full-size launch (2 KV-heads x 131072 tokens: x16); its traffic (k read once, X^T,
-        # partials) grows in proportion
-        {"files": ["ca_pair.cu", "ca_flash.cuh", "ptx.cuh"], "kernel_hash": "f9ea4b8c7c0d1bea",
+        # the head-dim-256 kernel (source ca_pair.cu) captured on one KV-head of a 16k-token
+        # cache (1.231 GB read + 0.086 GB written, profiles/ca_pair_gemma_n16k_t655.md), scaled
+        # by the units of a full-size launch (2 KV-heads x 131072 tokens: x16); its traffic (k
+        # read once, X^T, partials) grows in proportion
+        {"files": ["ca_pair.cu"], "kernel_hash": "89e4b7a50e367c33",
          "bytes_per_launch": 16 * 1.3165e9, "workload": ("gemma_128k", 655),
          "profile": "profiles/ca_pair_gemma_n16k_t655.md"},
     ],
