@@ -69,7 +69,7 @@ TRAFFIC = {
     "ca_fused": [
         # 1.313 GB read + 0.127 GB written per launch (profiles/ca_fused_qwen7b_8k_t1024.md,
         # the CTA-pair kernel, whose source is ca_flash.cuh)
-        {"files": ["ca_flash.cuh"], "kernel_hash": "1e46c485c8c9bbab",
+        {"files": ["ca_flash.cuh"], "kernel_hash": "362e2f1dfbf525ed",
          "bytes_per_launch": 1.4405e9, "workload": ("qwen7b_8k", 1024),
          "profile": "profiles/ca_fused_qwen7b_8k_t1024.md"},
         # the head-dim-256 kernel (source ca_pair.cu) captured on one KV-head of a 16k-token

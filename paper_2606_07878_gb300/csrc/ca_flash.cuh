@@ -5,11 +5,14 @@
 //   P(m, k)  = exp(S(m, k) - M(m))                   online row softmax over 256-key tiles
 //   O(m, :)  = sum_k P(m, k) X(k, :) / sum_k P(m, k)
 //
-// A work unit is (batch b = (KV-head, cross head), 128-row query tile, key split). Per key tile
-// the MMA warp computes S into TMEM columns [0, 256); eight softmax warps drain it to registers,
-// form fp16 probabilities in the 128-byte-swizzled shared-memory layout the tensor core reads,
-// and the MMA warp accumulates P X^T into TMEM columns [256, 256 + 2d). S and P never reach
-// global memory. The running max is kept in log2 units and only moved (with a rescale of the
+// A work unit is (batch b = (KV-head, cross head), two 128-row query tiles, key split) on a
+// CTA pair (cluster of two): CTA x computes query tile 2 m + x. Per key tile the even CTA issues
+// S for both tiles as one 2-SM MMA (tcgen05.mma.cta_group::2, M = 256) into each CTA's TMEM
+// columns [0, 256); each CTA's eight softmax warps drain their S to registers and form fp16
+// probabilities in the 128-byte-swizzled shared-memory layout the tensor core reads, and the
+// even CTA accumulates P X^T for both into TMEM columns [256, 256 + 2d). Each CTA holds its own
+// q and P rows and half of every k and X^T stage (the B operands), which halves the B traffic of
+// each SM's shared memory. S and P never reach global memory. The running max is kept in log2 units and only moved (with a rescale of the
 // TMEM accumulator) when a tile raises it by more than kRescaleLog2, so that P <= 2^8 fits fp16.
 //
 // Issue order of the tensor pipe: S_0, S_1, PX_0, S_2, PX_1, ... . PX_{j-1} runs while the
@@ -21,7 +24,13 @@
 // EX (a block whose output feeds another block): q, k in fp16 hi | lo, probabilities as fp16
 // hi + lo with one more P X pass, 128-key tiles (S in TMEM columns [0, 128)).
 //
-// CTA = 10 warps: 0 TMA producer, 1 MMA issuer (TMEM owner), 2..9 softmax / output.
+// Synchronisation inside the pair (all waits bounded): every stage's copies of both CTAs
+// complete on the even CTA's full barrier (cta_group::2 TMA); its commits arrive on both CTAs'
+// empty, sfull and pempty barriers; both CTAs' softmax warps arrive on its sfree and ofree
+// barriers, and the odd CTA's warp 1 forwards each completion of its pfull barrier.
+//
+// CTA = 10 warps: 0 TMA producer, 1 MMA issuer (even CTA) or P relay (odd CTA) and TMEM
+// allocation, 2..9 softmax / output.
 #pragma once
 #include "gemm_host.cuh"
 
@@ -50,7 +59,7 @@ struct FlashParams {
 };
 
 constexpr int kTopK = 8;       // repair candidates per list
-constexpr int kTopLists = 4;   // lists per row: (CTA of the pair, half of the key tile)
+constexpr int kTopLists = 4;   // lists per row: (column half of its CTAs, half of the key tile)
 
 constexpr int kFlashKeys = 256;       // keys per S tile (EX: 128)
 constexpr int kFlashSoftWarps = 8;    // two per TMEM lane quarter
