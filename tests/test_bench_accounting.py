@@ -71,3 +71,17 @@ def test_describe_names_the_shape():
     s = bench.describe("qwen3_4b_64k", wl, 1311)
     assert "2 blocks (CA in every block)" in s and "t=1311" in s and f"({round(65536 / 1311)}x)" in s
     assert math.isclose(65536 / 1311, 49.99, rel_tol=1e-3)
+
+
+def test_traffic_records_name_existing_profiles_and_current_kernels():
+    """Every DRAM-traffic record of the bench line points at a committed ncu summary and was
+    taken on the kernel source as it is now (otherwise the bench would silently report null)."""
+    import os
+    for kname, recs in bench.TRAFFIC.items():
+        for tr in recs:
+            assert os.path.exists(os.path.join(bench.ROOT, tr["profile"])), tr["profile"]
+            assert tr["kernel_hash"] == bench._kernel_hash(tr["files"]), (kname, tr["workload"])
+            assert tr["bytes_per_launch"] > 0
+    # the default workload has one
+    assert any(tr["workload"] == (bench.WORKLOAD, bench.DEFAULT_T[bench.WORKLOAD])
+               for tr in bench.TRAFFIC["ca_fused"])
