@@ -5,10 +5,11 @@
 //   strip      K, V -> X = [unRoPE(K) | V]  (hi/lo bf16 and hi/lo fp16 transposed)
 //   tables     compactor-RoPE coarse angle table for the key positions
 //   per group of (KV-head h, cross head i):
-//     keyproj  k~ = X W_K,i + b_K,i -> RoPE_c -> hi/lo, |k~|^2          (2-pass GEMM)
+//     keyproj  k~ = X W_K,i + b_K,i -> RoPE_c -> hi/lo, |k~|^2          (2-pass GEMM, 2-SM)
 //     qrope    q = RoPE_c(q^_i, p_j) -> hi/lo                         (q^ precomputed at load)
 //     ca_fused S = d_l * q.k / |k~|, online softmax, O_i += P X per key split, in one kernel
-//              (one CTA per unit for head dim <= 128, a cluster of two for 256)
+//              (units of two query tiles: a CTA pair with 2-SM MMAs for head dim <= 128, a
+//              cluster of four for 256)
 //     repair   (head dim 256) exact logits of each row's heaviest keys
 //     merge    the key splits of O_i and (m, l), in a fixed order -> hi/lo
 //   VO         Z' = Z + [O_1..O_n] (W_V,i W_O,i)_i                     (3-pass GEMM)
@@ -411,7 +412,8 @@ bool make_plan(const still_layer_config& c, bool lazy_q, int Kp, int64_t N, int 
   P.kss_b = a256(N * 4 * (kparts + 1));
   P.q_b = Kp > 0 ? 0 : a256(T * 2 * D * 2);
   // The fused kernel serves every block (a block that feeds another takes its split-precision
-  // variant); 2d = 512 runs it on clusters of two CTAs that split the O columns.
+  // variant); 2d = 512 runs it on clusters of four CTAs whose query-tile pairs split the O
+  // columns.
   P.flash = d == 64 || d == 128 || d == 256;
   P.P_b = a256(T * 8) * kMaxFlashSplit;          // per-split row statistics (m, l)
   P.O_b = a256(T * 2 * d * 4) * kMaxFlashSplit;  // per-split unnormalised O

@@ -29,7 +29,7 @@ def test_one_block_flops(name, t):
     assert fl["scores"] == 2 * t * N * H * n * D
     assert fl["px"] == 2 * t * N * H * n * 2 * d
     assert fl["px_passes"] == 1.5
-    # every head size takes the fused kernel (2d = 512 on clusters of two CTAs)
+    # every head size takes the fused kernel (2d = 512 on clusters of four CTAs)
     assert fl["scores_gemm"] == 0
 
 
